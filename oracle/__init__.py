@@ -1,0 +1,153 @@
+"""ctypes binding of the CPU oracle (kvx_oracle.c).
+
+TEST INFRASTRUCTURE ONLY: imported by tests/, __graft_entry__.smoke() and
+bench.py's cpu_baseline / reference legs.  The product library never imports
+this package; the two share no code.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+from typing import Optional, Sequence
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "kvx_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libkvx_oracle.so")
+_lib = None
+
+I32P = ctypes.POINTER(ctypes.c_int32)
+F64P = ctypes.POINTER(ctypes.c_double)
+F32P = ctypes.POINTER(ctypes.c_float)
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (-O2, no fast-math)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if force or not os.path.exists(_LIB_PATH) or os.path.getmtime(_LIB_PATH) < os.path.getmtime(_SRC):
+        tmp = _LIB_PATH + f".tmp{os.getpid()}"
+        subprocess.check_call(["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fno-fast-math",
+                               "-o", tmp, _SRC, "-lm"])
+        os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+class Problem(ctypes.Structure):
+    _fields_ = [
+        ("Ls", ctypes.c_int32), ("Hs", ctypes.c_int32), ("ds", ctypes.c_int32), ("base_s", ctypes.c_double),
+        ("Lt", ctypes.c_int32), ("Ht", ctypes.c_int32), ("dt", ctypes.c_int32), ("base_t", ctypes.c_double),
+        ("layer_map", I32P),
+        ("batch", ctypes.c_int32), ("s_max", ctypes.c_int32), ("t_max", ctypes.c_int32),
+        ("src_len", I32P), ("tgt_seq_off", I32P),
+        ("span_lo", I32P), ("span_hi", I32P),
+        ("src_pos", I32P), ("tgt_pos", I32P),
+        ("src_k", ctypes.POINTER(F32P)), ("src_v", ctypes.POINTER(F32P)),
+        ("w_k", F32P), ("w_v", F32P),
+    ]
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = ctypes.CDLL(build())
+        _lib.kvxo_layer_map_nearest.argtypes = [ctypes.c_int, ctypes.c_int, I32P]
+        _lib.kvxo_build_alignment.argtypes = [ctypes.c_int, I32P, I32P, I32P, I32P, I32P, I32P]
+        _lib.kvxo_rope.argtypes = [F64P, ctypes.c_int, ctypes.c_double, ctypes.c_double, ctypes.c_int]
+        _lib.kvxo_rope.restype = None
+        _lib.kvxo_rope_cache.argtypes = [F32P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                         ctypes.c_double, I32P, ctypes.c_int]
+        _lib.kvxo_rope_cache.restype = None
+        _lib.kvxo_translate_row.argtypes = [ctypes.POINTER(Problem), ctypes.c_int, ctypes.c_int,
+                                            ctypes.c_int, ctypes.c_int, F64P]
+        _lib.kvxo_translate.argtypes = [ctypes.POINTER(Problem), F64P, F64P]
+    return _lib
+
+
+def _p(a, typ):
+    return a.ctypes.data_as(typ) if a is not None else ctypes.cast(None, typ)
+
+
+def _i32(a):
+    return None if a is None else np.ascontiguousarray(a, np.int32)
+
+
+def layer_map_nearest(Ls: int, Lt: int) -> np.ndarray:
+    out = np.zeros(Lt, np.int32)
+    if lib().kvxo_layer_map_nearest(Ls, Lt, _p(out, I32P)):
+        raise ValueError("bad layer counts")
+    return out
+
+
+def build_alignment(src_seq_off, src_end, tgt_seq_off, tgt_end):
+    src_seq_off, src_end = _i32(src_seq_off), _i32(src_end)
+    tgt_seq_off, tgt_end = _i32(tgt_seq_off), _i32(tgt_end)
+    T = int(tgt_seq_off[-1])
+    lo = np.zeros(T, np.int32)
+    hi = np.zeros(T, np.int32)
+    n = lib().kvxo_build_alignment(len(tgt_seq_off) - 1, _p(src_seq_off, I32P), _p(src_end, I32P),
+                                   _p(tgt_seq_off, I32P), _p(tgt_end, I32P), _p(lo, I32P), _p(hi, I32P))
+    return lo, hi, n
+
+
+def rope(x: np.ndarray, base: float, pos: float, sign: int) -> np.ndarray:
+    v = np.array(x, np.float64).copy()
+    lib().kvxo_rope(_p(v, F64P), v.shape[-1], base, float(pos), sign)
+    return v
+
+
+def rope_cache(x: np.ndarray, base: float, pos: Optional[np.ndarray] = None, sign: int = +1) -> np.ndarray:
+    """x: [B, H, S, d] float32; returns a rotated copy (float32)."""
+    y = np.ascontiguousarray(x, np.float32).copy()
+    B, H, S, d = y.shape
+    pos = _i32(pos)
+    lib().kvxo_rope_cache(_p(y, F32P), B, H, S, d, base, _p(pos, I32P), sign)
+    return y
+
+
+class OracleProblem:
+    """Holds numpy arrays alive for the ctypes Problem struct."""
+
+    def __init__(self, src_geom, dst_geom, layer_map, src_len, tgt_seq_off, s_max, t_max,
+                 src_k: Sequence[np.ndarray], src_v: Sequence[np.ndarray], w_k, w_v,
+                 span_lo=None, span_hi=None, src_pos=None, tgt_pos=None):
+        self.keep = []
+
+        def keep(a):
+            self.keep.append(a)
+            return a
+
+        lm = keep(_i32(layer_map))
+        sl = keep(_i32(src_len))
+        so = keep(_i32(tgt_seq_off))
+        lo, hi = keep(_i32(span_lo)), keep(_i32(span_hi))
+        sp, tp = keep(_i32(src_pos)), keep(_i32(tgt_pos))
+        ks = [keep(np.ascontiguousarray(a, np.float32)) for a in src_k]
+        vs = [keep(np.ascontiguousarray(a, np.float32)) for a in src_v]
+        kp = keep((F32P * len(ks))(*[_p(a, F32P) for a in ks]))
+        vp = keep((F32P * len(vs))(*[_p(a, F32P) for a in vs]))
+        wk, wv = keep(np.ascontiguousarray(w_k, np.float32)), keep(np.ascontiguousarray(w_v, np.float32))
+        self.T = int(so[-1])
+        self.Lt, self.Ht, self.dt = dst_geom.num_layers, dst_geom.num_kv_heads, dst_geom.head_dim
+        self.p = Problem(src_geom.num_layers, src_geom.num_kv_heads, src_geom.head_dim, src_geom.rope_base,
+                         dst_geom.num_layers, dst_geom.num_kv_heads, dst_geom.head_dim, dst_geom.rope_base,
+                         _p(lm, I32P), len(sl), s_max, t_max, _p(sl, I32P), _p(so, I32P),
+                         _p(lo, I32P), _p(hi, I32P), _p(sp, I32P), _p(tp, I32P),
+                         ctypes.cast(kp, ctypes.POINTER(F32P)), ctypes.cast(vp, ctypes.POINTER(F32P)),
+                         _p(wk, F32P), _p(wv, F32P))
+
+    def translate(self):
+        """Returns (K, V), each [Lt, Ht, T_total, dt] float64."""
+        ok = np.zeros((self.Lt, self.Ht, self.T, self.dt), np.float64)
+        ov = np.zeros_like(ok)
+        if lib().kvxo_translate(ctypes.byref(self.p), _p(ok, F64P), _p(ov, F64P)):
+            raise ValueError("oracle: unsupported geometry")
+        return ok, ov
+
+    def row(self, j: int, h: int, kv: int, tp: int) -> np.ndarray:
+        out = np.zeros(self.dt, np.float64)
+        if lib().kvxo_translate_row(ctypes.byref(self.p), j, h, kv, tp, _p(out, F64P)):
+            raise ValueError("oracle: unsupported geometry")
+        return out

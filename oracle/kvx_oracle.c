@@ -1,0 +1,224 @@
+/*
+ * kvx_oracle.c -- CPU oracle for cross-model KV translation.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Only tests/, __graft_entry__.smoke() and the
+ * cpu_baseline leg of bench.py may load this code.  The product path (the CUDA
+ * library under paper_2608_30963_gb300/) never calls it and shares no code,
+ * header, table or constant with it.
+ *
+ * What it computes (paper Section 4, translation operator KV^_B = T_{A->B}(KV_A),
+ * and Section 5, parameterised translator T_theta, applied per layer and per KV
+ * head, one of the granularities Section 5 lists).  For every target layer j,
+ * target KV head h, K or V, and target token t of sequence b:
+ *
+ *   1. source layer     l = layer_map[j]                 (nearest relative depth)
+ *   2. source span      [lo_t, hi_t) of the source tokens of sequence b
+ *   3. for every s in the span and every grouped source head g (GQA regroup):
+ *        K: u_g = R_{d_s,base_s}(-p_s) K[l,b,g,s]   (undo the source RoPE)
+ *        V: u_g = V[l,b,g,s]
+ *      and u = concat_g u_g  (length in = r*d_s, or d_s when target heads
+ *      outnumber source heads)
+ *   4. xbar = (1/|span|) sum_s u                      (span mean)
+ *   5. y = xbar . W[j,h]      with W[j,h] of shape [in, out=d_t]
+ *   6. K: y <- R_{d_t,base_t}(+p_t) y                 (apply the target RoPE)
+ *
+ * R_{d,base}(p) is the half-split rotary map: channel pairs (i, i+d/2) for
+ * i < d/2 are rotated by the angle p * base^(-2i/d).  The angle is taken in
+ * exact (double) arithmetic.  A base <= 0 means "no RoPE".
+ *
+ * Everything runs in double precision, in the order above, with no blocking,
+ * fusion or reordering.  Inputs are float32 arrays (bf16 storage is widened
+ * exactly by the caller).
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define KVXO_API __attribute__((visibility("default")))
+
+/* ---------------------------------------------------------------------- */
+/* Layer alignment: target layer j draws from the source layer nearest to it
+ * in relative depth, depth(j) = j/(L_t-1), depth(s) = s/(L_s-1).  Ties round
+ * to the deeper layer.  Implemented as an explicit argmin over all source
+ * layers with exact integer cross-multiplication. */
+KVXO_API int kvxo_layer_map_nearest(int Ls, int Lt, int32_t* out)
+{
+    if (Ls < 1 || Lt < 1 || !out) return 1;
+    for (int j = 0; j < Lt; ++j) {
+        if (Lt == 1 || Ls == 1) { out[j] = 0; continue; }
+        /* |s/(Ls-1) - j/(Lt-1)| compared as |s*(Lt-1) - j*(Ls-1)| */
+        int best = 0;
+        int64_t best_d = INT64_MAX;
+        for (int s = 0; s < Ls; ++s) {
+            int64_t d = (int64_t)s * (Lt - 1) - (int64_t)j * (Ls - 1);
+            if (d < 0) d = -d;
+            if (d <= best_d) { best = s; best_d = d; }   /* '<=': ties go deeper */
+        }
+        out[j] = best;
+    }
+    return 0;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Token-span alignment between two tokenisations of the same byte string
+ * (the paper names tokenizer differences among the model differences the
+ * translator must bridge, Sections 1 and 4).
+ *
+ * Byte-end offsets per sequence are strictly increasing and relative to the
+ * sequence start.  Source token s covers bytes [src_end[s-1], src_end[s]);
+ * target token t covers [tgt_end[t-1], tgt_end[t]).  Source token s belongs to
+ * the target token whose byte range holds s's last byte.  A target token that
+ * receives no source token takes the single source token holding its own last
+ * byte.  Output spans are within-sequence source indices [lo, hi).
+ *
+ * Walks both sequences with one merge pointer.  Returns the number of target
+ * tokens whose span had to be clamped because the source text ended first. */
+KVXO_API int kvxo_build_alignment(int batch,
+                                  const int32_t* src_seq_off, const int32_t* src_end,
+                                  const int32_t* tgt_seq_off, const int32_t* tgt_end,
+                                  int32_t* span_lo, int32_t* span_hi)
+{
+    int clamped = 0;
+    for (int b = 0; b < batch; ++b) {
+        const int32_t* se = src_end + src_seq_off[b];
+        const int32_t* te = tgt_end + tgt_seq_off[b];
+        int S = src_seq_off[b + 1] - src_seq_off[b];
+        int T = tgt_seq_off[b + 1] - tgt_seq_off[b];
+        int s = 0;                       /* first source token not yet assigned */
+        for (int t = 0; t < T; ++t) {
+            int lo = s;
+            while (s < S && se[s] <= te[t]) ++s;   /* last byte se[s]-1 < te[t] */
+            int hi = s;
+            if (hi == lo) {              /* empty: source token holding byte te[t]-1 */
+                hi = lo + 1;
+                if (lo >= S) { lo = S - 1; hi = S; ++clamped; }
+            }
+            span_lo[tgt_seq_off[b] + t] = lo;
+            span_hi[tgt_seq_off[b] + t] = hi;
+        }
+    }
+    return clamped;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Half-split rotary map on one head vector of length d (d even):
+ * x'[i] = x[i] cos a - x[i+d/2] sin a,  x'[i+d/2] = x[i+d/2] cos a + x[i] sin a,
+ * a = sign * pos * base^(-2i/d).  sign = +1 applies the RoPE, -1 undoes it. */
+KVXO_API void kvxo_rope(double* x, int d, double base, double pos, int sign)
+{
+    if (base <= 0.0) return;
+    int h = d / 2;
+    for (int i = 0; i < h; ++i) {
+        double inv_freq = pow(base, -2.0 * (double)i / (double)d);
+        double a = (double)sign * pos * inv_freq;
+        double c = cos(a), sn = sin(a);
+        double x0 = x[i], x1 = x[i + h];
+        x[i]     = x0 * c - x1 * sn;
+        x[i + h] = x1 * c + x0 * sn;
+    }
+}
+
+/* ---------------------------------------------------------------------- */
+typedef struct {
+    int32_t Ls, Hs, ds; double base_s;        /* source geometry */
+    int32_t Lt, Ht, dt; double base_t;        /* target geometry */
+    const int32_t* layer_map;                 /* [Lt] */
+    int32_t batch, s_max, t_max;
+    const int32_t* src_len;                   /* [B] */
+    const int32_t* tgt_seq_off;               /* [B+1] packed target offsets */
+    const int32_t* span_lo;                   /* [T_total] or NULL (identity) */
+    const int32_t* span_hi;
+    const int32_t* src_pos;                   /* [B*s_max] or NULL (= index) */
+    const int32_t* tgt_pos;                   /* [T_total] or NULL (= index) */
+    const float* const* src_k;                /* [Ls] -> [B][Hs][s_max][ds] */
+    const float* const* src_v;
+    const float* w_k;                         /* [Lt][Ht][in][dt] */
+    const float* w_v;
+} kvxo_problem;
+
+static int group_in(const kvxo_problem* p)
+{
+    return p->Hs >= p->Ht ? (p->Hs / p->Ht) * p->ds : p->ds;
+}
+
+/* One output row: target layer j, target head h, kv (0 = K, 1 = V), packed
+ * target token index tp.  Writes d_t doubles.  Returns nonzero on a
+ * geometry it cannot place. */
+KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int tp, double* out)
+{
+    if (p->Hs % p->Ht != 0 && p->Ht % p->Hs != 0) return 1;
+    int b = 0;
+    while (b < p->batch - 1 && p->tgt_seq_off[b + 1] <= tp) ++b;
+    int t = tp - p->tgt_seq_off[b];
+    int l = p->layer_map[j];                                   /* step 1 */
+    int lo = p->span_lo ? p->span_lo[tp] : t;                  /* step 2 */
+    int hi = p->span_hi ? p->span_hi[tp] : t + 1;
+    int in = group_in(p);
+    int r = p->Hs >= p->Ht ? p->Hs / p->Ht : 1;
+    int g0 = p->Hs >= p->Ht ? h * r : h / (p->Ht / p->Hs);
+    const float* src = kv == 0 ? p->src_k[l] : p->src_v[l];
+
+    double* sum = (double*)calloc((size_t)in, sizeof(double));
+    double* u = (double*)malloc(sizeof(double) * (size_t)p->ds);
+    for (int s = lo; s < hi; ++s) {                            /* step 3 */
+        double ps = p->src_pos ? (double)p->src_pos[(size_t)b * p->s_max + s] : (double)s;
+        for (int q = 0; q < r; ++q) {
+            int g = g0 + q;
+            const float* row = src + (((size_t)b * p->Hs + g) * p->s_max + s) * p->ds;
+            for (int e = 0; e < p->ds; ++e) u[e] = (double)row[e];
+            if (kv == 0) kvxo_rope(u, p->ds, p->base_s, ps, -1);
+            for (int e = 0; e < p->ds; ++e) sum[q * p->ds + e] += u[e];
+        }
+    }
+    double n = (double)(hi - lo);                              /* step 4 */
+    for (int i = 0; i < in; ++i) sum[i] /= n;
+
+    const float* W = (kv == 0 ? p->w_k : p->w_v) + ((size_t)j * p->Ht + h) * (size_t)in * p->dt;
+    for (int o = 0; o < p->dt; ++o) {                          /* step 5 */
+        double acc = 0.0;
+        for (int i = 0; i < in; ++i) acc += sum[i] * (double)W[(size_t)i * p->dt + o];
+        out[o] = acc;
+    }
+    if (kv == 0) {                                             /* step 6 */
+        double pt = p->tgt_pos ? (double)p->tgt_pos[tp] : (double)t;
+        kvxo_rope(out, p->dt, p->base_t, pt, +1);
+    }
+    free(sum);
+    free(u);
+    return 0;
+}
+
+/* Whole translation.  out_k / out_v: [Lt][Ht][T_total][dt] doubles. */
+KVXO_API int kvxo_translate(const kvxo_problem* p, double* out_k, double* out_v)
+{
+    int T = p->tgt_seq_off[p->batch];
+    for (int j = 0; j < p->Lt; ++j)
+        for (int h = 0; h < p->Ht; ++h)
+            for (int tp = 0; tp < T; ++tp) {
+                size_t o = (((size_t)j * p->Ht + h) * T + tp) * p->dt;
+                if (kvxo_translate_row(p, j, h, 0, tp, out_k + o)) return 1;
+                if (kvxo_translate_row(p, j, h, 1, tp, out_v + o)) return 1;
+            }
+    return 0;
+}
+
+/* Apply (sign=+1) or undo (sign=-1) the RoPE on every row of a KV cache laid
+ * out [B][H][S][d] (float32 in place, arithmetic in double).  pos: [B*S]
+ * positions or NULL (= token index).  Used to synthesise post-RoPE source
+ * caches the way a source model's prefill would have stored them. */
+KVXO_API void kvxo_rope_cache(float* x, int B, int H, int S, int d, double base,
+                              const int32_t* pos, int sign)
+{
+    double* row = (double*)malloc(sizeof(double) * (size_t)d);
+    for (int b = 0; b < B; ++b)
+        for (int h = 0; h < H; ++h)
+            for (int s = 0; s < S; ++s) {
+                float* xr = x + (((size_t)b * H + h) * S + s) * d;
+                for (int e = 0; e < d; ++e) row[e] = (double)xr[e];
+                double p = pos ? (double)pos[(size_t)b * S + s] : (double)s;
+                kvxo_rope(row, d, base, p, sign);
+                for (int e = 0; e < d; ++e) xr[e] = (float)row[e];
+            }
+    free(row);
+}

@@ -1,0 +1,282 @@
+"""Pins for the CPU oracle, independent of its own code.
+
+Each test checks the oracle against something the mathematics fixes: brute
+force on tiny inputs, closed forms, invariants, or special cases that reduce to
+a library routine.  Between them a dropped term, a wrong sign, a wrong index or
+a transposed operand anywhere in the oracle fails at least one test.
+"""
+from fractions import Fraction
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2608_30963_gb300 import synth
+
+
+# ---------------------------------------------------------------- layer map
+@pytest.mark.parametrize("Ls,Lt", [(4, 2), (28, 28), (28, 26), (80, 28), (5, 3), (3, 5), (7, 1), (1, 4), (2, 2),
+                                   (10, 4)])
+def test_layer_map_matches_exact_nearest_depth(Ls, Lt):
+    got = oracle.layer_map_nearest(Ls, Lt)
+    for j in range(Lt):
+        dj = Fraction(j, Lt - 1) if Lt > 1 else Fraction(0)
+        cands = [abs(Fraction(s, Ls - 1) - dj) if Ls > 1 else Fraction(0) for s in range(Ls)]
+        m = min(cands)
+        best = max(s for s in range(Ls) if cands[s] == m)  # ties go to the deeper layer
+        assert got[j] == best
+
+
+def test_layer_map_endpoints_and_identity():
+    assert list(oracle.layer_map_nearest(28, 28)) == list(range(28))
+    for Ls, Lt in [(80, 28), (28, 26), (4, 2)]:
+        m = oracle.layer_map_nearest(Ls, Lt)
+        assert m[0] == 0 and m[-1] == Ls - 1
+        assert np.all(np.diff(m) > 0)
+
+
+# ---------------------------------------------------------- token alignment
+def test_alignment_recovers_generated_partition():
+    for b, T in enumerate([1, 7, 300, 2048]):
+        lo, hi, S, se, te = synth.draw_spans(T, b)
+        so = np.array([0, S], np.int32)
+        to = np.array([0, T], np.int32)
+        glo, ghi, n = oracle.build_alignment(so, se, to, te)
+        assert n == 0
+        np.testing.assert_array_equal(glo, lo)
+        np.testing.assert_array_equal(ghi, hi)
+
+
+def _bytewise_spans(src_end, tgt_end):
+    """Brute force over bytes: owner of each byte in both tokenisations."""
+    n = int(src_end[-1])
+    src_of = np.searchsorted(src_end, np.arange(n), side="right")
+    tgt_of = np.searchsorted(tgt_end, np.arange(n), side="right")
+    members = [[] for _ in range(len(tgt_end))]
+    for s in range(len(src_end)):
+        members[tgt_of[int(src_end[s]) - 1]].append(s)   # s's last byte
+    lo, hi = [], []
+    for t in range(len(tgt_end)):
+        if members[t]:
+            assert members[t] == list(range(members[t][0], members[t][-1] + 1))
+            lo.append(members[t][0]); hi.append(members[t][-1] + 1)
+        else:
+            s = int(src_of[int(tgt_end[t]) - 1])            # holds t's last byte
+            lo.append(s); hi.append(s + 1)
+    return np.array(lo, np.int32), np.array(hi, np.int32)
+
+
+@pytest.mark.parametrize("key,ms,mt", [(0, 4.0, 4.0), (1, 5.0, 2.0), (2, 2.0, 6.0), (3, 1.0, 3.0), (4, 3.0, 1.0)])
+def test_alignment_bytewise_bruteforce(key, ms, mt):
+    # batch of 3 sequences of different byte lengths, including empty spans
+    src_ends, tgt_ends = [], []
+    for i, nb in enumerate([1, 57, 911]):
+        se, te = synth.draw_tokenizations(nb, ms, mt, key * 10 + i)
+        src_ends.append(se); tgt_ends.append(te)
+    so = np.concatenate([[0], np.cumsum([len(x) for x in src_ends])]).astype(np.int32)
+    to = np.concatenate([[0], np.cumsum([len(x) for x in tgt_ends])]).astype(np.int32)
+    lo, hi, n = oracle.build_alignment(so, np.concatenate(src_ends), to, np.concatenate(tgt_ends))
+    assert n == 0
+    for b in range(3):
+        elo, ehi = _bytewise_spans(src_ends[b], tgt_ends[b])
+        np.testing.assert_array_equal(lo[to[b]:to[b + 1]], elo)
+        np.testing.assert_array_equal(hi[to[b]:to[b + 1]], ehi)
+
+
+# --------------------------------------------------------------------- RoPE
+def test_rope_two_dims_is_plain_rotation_by_position():
+    # d = 2: the only frequency is base^0 = 1, so the angle is the position.
+    for base in (10.0, 1e4, 1e6):
+        y = oracle.rope(np.array([1.0, 0.0]), base, np.pi / 2, +1)
+        np.testing.assert_allclose(y, [0.0, 1.0], atol=1e-15)
+        y = oracle.rope(np.array([0.0, 2.0]), base, np.pi, +1)
+        np.testing.assert_allclose(y, [0.0, -2.0], atol=1e-14)
+
+
+def test_rope_roformer_frequencies_d4():
+    # RoFormer: theta_i = base^(-2(i-1)/d), i = 1..d/2; d = 4, base 1e4 -> {1, 1e-2}.
+    x = np.array([0.0, 1.0, 0.0, 0.0])     # unit vector in the second (slow) pair
+    y = oracle.rope(x, 1e4, 100.0, +1)     # angle 100 * 1e-2 = 1 rad
+    np.testing.assert_allclose(y, [0.0, np.cos(1.0), 0.0, np.sin(1.0)], atol=1e-14)
+
+
+def test_rope_equals_complex_multiplication():
+    rng = np.random.default_rng(11)
+    for d in (2, 8, 64, 128, 256):
+        for base, pos in ((1e4, 3.0), (1e6, 4095.0), (5e5, 31999.0)):
+            x = rng.standard_normal(d)
+            h = d // 2
+            z = x[:h] + 1j * x[h:]
+            ang = pos * np.exp(-np.log(base) * np.arange(0, d, 2) / d)
+            w = z * np.exp(1j * ang)
+            y = oracle.rope(x, base, pos, +1)
+            np.testing.assert_allclose(y, np.concatenate([w.real, w.imag]), rtol=0, atol=1e-9)
+
+
+def test_rope_inverse_norm_and_relative_position():
+    rng = np.random.default_rng(12)
+    for d, base in ((64, 1e4), (128, 1e6), (256, 1e4)):
+        x = rng.standard_normal(d)
+        q = rng.standard_normal(d)
+        back = oracle.rope(oracle.rope(x, base, 777.0, +1), base, 777.0, -1)
+        np.testing.assert_allclose(back, x, atol=1e-12)
+        np.testing.assert_array_equal(oracle.rope(x, base, 0.0, +1), x)
+        y = oracle.rope(x, base, 1234.0, +1)
+        h = d // 2
+        np.testing.assert_allclose(x[:h] ** 2 + x[h:] ** 2, y[:h] ** 2 + y[h:] ** 2, rtol=1e-12)
+        # <R(p)q, R(p')k> depends only on p - p'
+        a = oracle.rope(q, base, 100.0, +1) @ oracle.rope(x, base, 40.0, +1)
+        b = oracle.rope(q, base, 1160.0, +1) @ oracle.rope(x, base, 1100.0, +1)
+        assert abs(a - b) < 1e-9
+
+
+# ------------------------------------------------------------ translation
+def _geom(L, H, d, base):
+    return synth.ModelGeom(L, H, d, base)
+
+
+def _problem(sg, dg, layer_map, lens_src, lens_tgt, src_k, src_v, wk, wv, lo=None, hi=None, sp=None, tp=None):
+    so = np.concatenate([[0], np.cumsum(lens_tgt)]).astype(np.int32)
+    return oracle.OracleProblem(sg, dg, layer_map, np.array(lens_src, np.int32), so,
+                                src_k[0].shape[2], max(lens_tgt), src_k, src_v, wk, wv, lo, hi, sp, tp)
+
+
+def _rand_src(rng, g, B, S):
+    return ([rng.standard_normal((B, g.num_kv_heads, S, g.head_dim)).astype(np.float32) for _ in range(g.num_layers)],
+            [rng.standard_normal((B, g.num_kv_heads, S, g.head_dim)).astype(np.float32) for _ in range(g.num_layers)])
+
+
+def test_identity_translator_round_trip():
+    """Same geometry, same tokenizer, W = I: output equals the stored cache."""
+    rng = np.random.default_rng(1)
+    g = _geom(3, 2, 64, 1e4)
+    B, S = 2, 37
+    ks, vs = _rand_src(rng, g, B, S)
+    ks = [oracle.rope_cache(k, g.rope_base) for k in ks]
+    eye = np.broadcast_to(np.eye(64, dtype=np.float32), (3, 2, 64, 64)).copy()
+    p = _problem(g, g, [0, 1, 2], [S, S], [S, S], ks, vs, eye, eye)
+    ok, ov = p.translate()
+    for j in range(3):
+        for b in range(B):
+            np.testing.assert_allclose(ok[j, :, b * S:(b + 1) * S], ks[j][b], atol=2e-6)
+            np.testing.assert_array_equal(ov[j, :, b * S:(b + 1) * S], vs[j][b])
+
+
+def test_selection_matrix_picks_first_grouped_head():
+    """H_s = 2 H_t and W = [I; 0]: target head j reproduces source head 2j."""
+    rng = np.random.default_rng(2)
+    sg, dg = _geom(2, 4, 64, 1e6), _geom(2, 2, 64, 1e6)
+    S = 19
+    ks, vs = _rand_src(rng, sg, 1, S)
+    ks = [oracle.rope_cache(k, sg.rope_base) for k in ks]
+    sel = np.zeros((2, 2, 128, 64), np.float32)
+    sel[:, :, :64, :] = np.eye(64)
+    p = _problem(sg, dg, [1, 0], [S], [S], ks, vs, sel, sel)
+    ok, ov = p.translate()
+    for j, l in ((0, 1), (1, 0)):
+        for h in range(2):
+            np.testing.assert_allclose(ok[j, h], ks[l][0, 2 * h], atol=2e-6)
+            np.testing.assert_array_equal(ov[j, h], vs[l][0, 2 * h])
+    sel2 = np.zeros_like(sel)
+    sel2[:, :, 64:, :] = np.eye(64)      # second half selects head 2j+1
+    ok, ov = _problem(sg, dg, [1, 0], [S], [S], ks, vs, sel2, sel2).translate()
+    np.testing.assert_array_equal(ov[0, 1], vs[1][0, 3])
+
+
+def test_expansion_identity_repeats_kv_heads():
+    rng = np.random.default_rng(3)
+    sg, dg = _geom(1, 2, 64, 1e4), _geom(1, 4, 64, 1e4)
+    ks, vs = _rand_src(rng, sg, 1, 11)
+    ks = [oracle.rope_cache(k, sg.rope_base) for k in ks]
+    eye = np.broadcast_to(np.eye(64, dtype=np.float32), (1, 4, 64, 64)).copy()
+    ok, ov = _problem(sg, dg, [0], [11], [11], ks, vs, eye, eye).translate()
+    for h in range(4):
+        np.testing.assert_allclose(ok[0, h], ks[0][0, h // 2], atol=2e-6)
+        np.testing.assert_array_equal(ov[0, h], vs[0][0, h // 2])
+
+
+def test_no_rope_projection_is_a_matmul_of_the_concatenated_heads():
+    """Bases <= 0 and identity alignment reduce the operator to concat(heads) @ W."""
+    rng = np.random.default_rng(4)
+    sg, dg = _geom(2, 4, 64, 0.0), _geom(2, 2, 128, 0.0)
+    S = 9
+    ks, vs = _rand_src(rng, sg, 1, S)
+    wk = rng.standard_normal((2, 2, 128, 128)).astype(np.float32)
+    wv = rng.standard_normal((2, 2, 128, 128)).astype(np.float32)
+    ok, ov = _problem(sg, dg, [0, 1], [S], [S], ks, vs, wk, wv).translate()
+    for j in range(2):
+        for h in range(2):
+            xk = np.concatenate([ks[j][0, 2 * h], ks[j][0, 2 * h + 1]], axis=1).astype(np.float64)
+            xv = np.concatenate([vs[j][0, 2 * h], vs[j][0, 2 * h + 1]], axis=1).astype(np.float64)
+            np.testing.assert_allclose(ok[j, h], xk @ wk[j, h].astype(np.float64), rtol=1e-12, atol=1e-12)
+            np.testing.assert_allclose(ov[j, h], xv @ wv[j, h].astype(np.float64), rtol=1e-12, atol=1e-12)
+
+
+def test_span_closed_form_unrotates_before_the_mean():
+    """If every source token of span t stores R(p_s) u_t, the output is R(p_t) W u_t.
+
+    Also V: rows c_s * v_t reduce to mean(c) * W v_t.  Differing source and
+    target bases and head dims, cross-tokenizer spans of length 1-3.
+    """
+    rng = np.random.default_rng(5)
+    sg, dg = _geom(1, 2, 64, 1e6), _geom(1, 1, 128, 1e4)
+    T = 40
+    lo, hi, S, _, _ = synth.draw_spans(T, 9)
+    u = rng.standard_normal((T, 2, 64))
+    v = rng.standard_normal((T, 2, 64))
+    c = rng.uniform(0.5, 2.0, S)
+    k_store = np.zeros((1, 2, S, 64), np.float32)
+    v_store = np.zeros((1, 2, S, 64), np.float32)
+    for t in range(T):
+        for s in range(lo[t], hi[t]):
+            for g in range(2):
+                k_store[0, g, s] = oracle.rope(u[t, g], sg.rope_base, s, +1)
+                v_store[0, g, s] = c[s] * v[t, g]
+    w = rng.standard_normal((1, 1, 128, 128)).astype(np.float32)
+    p = _problem(sg, dg, [0], [S], [T], [k_store], [v_store], w, w, lo, hi)
+    ok, ov = p.translate()
+    W = w[0, 0].astype(np.float64)
+    for t in range(T):
+        uk = np.concatenate([k_store[0, 0, lo[t]], k_store[0, 1, lo[t]]]).astype(np.float64)
+        uk = np.concatenate([oracle.rope(uk[:64], sg.rope_base, lo[t], -1), oracle.rope(uk[64:], sg.rope_base, lo[t], -1)])
+        want_k = oracle.rope(uk @ W, dg.rope_base, t, +1)
+        np.testing.assert_allclose(ok[0, 0, t], want_k, atol=1e-5)
+        vt = np.concatenate([v[t, 0], v[t, 1]]).astype(np.float32).astype(np.float64)
+        want_v = np.mean(c[lo[t]:hi[t]]) * (vt @ W)
+        np.testing.assert_allclose(ov[0, 0, t], want_v, rtol=1e-5, atol=1e-5)
+
+
+def test_linearity_and_batch_invariance():
+    rng = np.random.default_rng(6)
+    sg, dg = _geom(2, 2, 64, 1e4), _geom(1, 2, 64, 1e6)
+    lens = [13, 29]
+    S = 29
+    k1, v1 = [[synth.bf16_round(x) for x in y] for y in _rand_src(rng, sg, 2, S)]
+    k2, v2 = [[synth.bf16_round(x) for x in y] for y in _rand_src(rng, sg, 2, S)]
+    w = rng.standard_normal((1, 2, 64, 64)).astype(np.float32)
+    a, b = 0.5, -2.0
+    km = [a * x + b * y for x, y in zip(k1, k2)]
+    vm = [a * x + b * y for x, y in zip(v1, v2)]
+    o1 = _problem(sg, dg, [1], lens, lens, k1, v1, w, w).translate()
+    o2 = _problem(sg, dg, [1], lens, lens, k2, v2, w, w).translate()
+    om = _problem(sg, dg, [1], lens, lens, km, vm, w, w).translate()
+    # inputs are bf16-valued, so a*x + b*y is exact in float32 unless the
+    # exponents are far apart; the tolerance covers that last rounding
+    for i in range(2):
+        np.testing.assert_allclose(om[i], a * o1[i] + b * o2[i], rtol=1e-6, atol=2e-5)
+    # batch invariance: sequence 1 alone gives the same rows
+    solo = _problem(sg, dg, [1], [29], [29], [k[1:2] for k in k1], [v[1:2] for v in v1], w, w).translate()
+    for i in range(2):
+        np.testing.assert_array_equal(o1[i][:, :, 13:], solo[i])
+
+
+def test_layer_map_is_followed():
+    rng = np.random.default_rng(7)
+    sg, dg = _geom(3, 2, 64, 1e4), _geom(2, 2, 64, 1e4)
+    ks, vs = _rand_src(rng, sg, 1, 5)
+    w = rng.standard_normal((2, 2, 64, 64)).astype(np.float32)
+    base = _problem(sg, dg, [2, 0], [5], [5], ks, vs, w, w).translate()
+    perm = [ks[2], ks[0], ks[1]], [vs[2], vs[0], vs[1]]
+    moved = _problem(sg, dg, [0, 1], [5], [5], perm[0], perm[1], w, w).translate()
+    for i in range(2):
+        np.testing.assert_array_equal(base[i], moved[i])
