@@ -1,0 +1,452 @@
+"""Benchmark: translated KV tokens/s and ms per handoff for cross-model KV translation.
+
+One step = one kvx_translate call over the whole workload (all target layers,
+heads, K and V, every target token): layer alignment, span gather, undo the
+source RoPE, span mean, GQA-regrouped projection, target RoPE and target cache
+write.  Default workload: Qwen2.5-7B-shaped -> Qwen2.5-1.5B-shaped KV caches,
+4096 tokens, batch 1, bf16 (the within-family handoff of the paper's
+Section 6.2 at the 4K context the headline metric names).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl kvx|reference] [--workload NAME]
+
+Prints ONE JSON line on rank 0.  Under torchrun (N > 1) every rank translates
+its own replica of the workload (no collective on the data path: the handoffs
+are independent); the timed region is bracketed by barriers and the time is
+the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import multiprocessing as mp
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_30963_gb300 import synth  # noqa: E402  (numpy only)
+
+DEFAULT_WORKLOAD = "qwen7b_to_qwen1p5b_4k"
+METRIC = "translated KV tokens/s and ms/handoff at 4K (7B→1.5B shapes); % of roofline"
+
+
+# ----------------------------------------------------------------------------- workload arithmetic
+def algorithmic(spec: synth.WorkloadSpec, wl: synth.Workload, layer_map) -> dict:
+    """Bytes a translate must move at least once, and its FLOPs."""
+    elt = 2 if spec.dtype == "bf16" else 4
+    S_tot = int(wl.src_len.sum())
+    T = wl.total_tgt
+    src_layers = len(set(int(x) for x in layer_map))
+    rd = src_layers * spec.src.num_kv_heads * S_tot * spec.src.head_dim * 2 * elt
+    wr = spec.dst.num_layers * spec.dst.num_kv_heads * T * spec.dst.head_dim * 2 * elt
+    wt = 2 * spec.dst.num_layers * spec.dst.num_kv_heads * spec.group_in * spec.dst.head_dim * elt
+    flops = 2.0 * T * spec.group_in * spec.dst.head_dim * spec.dst.num_layers * spec.dst.num_kv_heads * 2
+    return {"read": rd, "write": wr, "weights": wt, "bytes": rd + wr + wt, "flops": flops}
+
+
+def nearest_map(Ls, Lt):
+    return [0] * Lt if Lt == 1 else [(2 * j * (Ls - 1) + (Lt - 1)) // (2 * (Lt - 1)) for j in range(Lt)]
+
+
+# ----------------------------------------------------------------------------- CPU oracle (baseline / reference arm)
+def _oracle_worker(args):
+    """Time the oracle on target rows [t0, t0+n) of layer 0, K and V, all heads.
+
+    Runs in a spawned process; imports the oracle there."""
+    name, t0, n, budget_s = args
+    import oracle
+    spec = synth.config_specs()[name]
+    wl = synth.make_workload(spec)
+    lm = wl.layer_map if wl.layer_map is not None else oracle.layer_map_nearest(spec.src.num_layers,
+                                                                                spec.dst.num_layers)
+    l0 = int(lm[0])
+    k = synth.source_kv(wl, l0, 0)
+    if spec.src.rope_base > 0:
+        k = oracle.rope_cache(k, spec.src.rope_base)
+        if spec.dtype == "bf16":
+            k = synth.bf16_round(k)
+    v = synth.source_kv(wl, l0, 1)
+    ks = [k] * spec.src.num_layers
+    vs = [v] * spec.src.num_layers
+    p = oracle.OracleProblem(spec.src, spec.dst, lm, wl.src_len, wl.tgt_seq_off, wl.s_max, wl.t_max, ks, vs,
+                             synth.weights(wl, 0), synth.weights(wl, 1), wl.span_lo, wl.span_hi)
+    rows = 0
+    start = time.perf_counter()
+    T = wl.total_tgt
+    i = 0
+    while True:
+        tp = (t0 + i) % T
+        for h in range(spec.dst.num_kv_heads):
+            for kv in (0, 1):
+                p.row(0, h, kv, tp)
+                rows += 1
+        i += 1
+        el = time.perf_counter() - start
+        if (n and i >= n) or (not n and el >= budget_s):
+            break
+    return rows, time.perf_counter() - start
+
+
+def cpu_baseline(pool, name: str, budget_s: float, cores: int) -> dict:
+    """Oracle throughput on the host cores, as target tokens/s (one target token
+    = L_t * H_t * 2 output rows)."""
+    spec = synth.config_specs()[name]
+    args = [(name, 97 * i, 0, budget_s) for i in range(cores)]
+    t0 = time.perf_counter()
+    res = pool.map(_oracle_worker, args)
+    wall = time.perf_counter() - t0
+    rows = sum(r for r, _ in res)
+    busy = max(t for _, t in res)
+    rows_per_tok = spec.dst.num_layers * spec.dst.num_kv_heads * 2
+    tok_s = rows / busy / rows_per_tok
+    return {"value": tok_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{rows} output rows (target layer 0, all heads, K and V) of workload {name}, "
+                      f"{budget_s:.0f} s per core on {cores} spawned processes; scaled to tokens by "
+                      f"{rows_per_tok} rows per target token",
+            "wall_s": wall}
+
+
+# ----------------------------------------------------------------------------- clocks
+CLOCK_Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+           "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+           "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    def __init__(self, gpu_index: int):
+        self.proc = None
+        self.path = None
+        try:
+            os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+            self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(gpu_index), f"--query-gpu={CLOCK_Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self) -> dict:
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(nm)
+        try:
+            os.remove(self.path)
+        except OSError:
+            pass
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- input synthesis
+def rotate_np(x: np.ndarray, base: float) -> np.ndarray:
+    """Apply half-split RoPE at positions 0..S-1 (input synthesis: the post-RoPE
+    keys a source model's prefill stores)."""
+    B, H, S, d = x.shape
+    h = d // 2
+    ang = np.arange(S, dtype=np.float64)[:, None] * np.power(base, -2.0 * np.arange(h) / d)[None, :]
+    c, s = np.cos(ang), np.sin(ang)
+    x0, x1 = x[..., :h].astype(np.float64), x[..., h:].astype(np.float64)
+    return np.concatenate([x0 * c - x1 * s, x1 * c + x0 * s], axis=-1).astype(np.float32)
+
+
+def to_torch(x: np.ndarray, dtype: str, torch, pin=False):
+    if dtype == "bf16":
+        t = torch.from_numpy(synth.f32_to_bf16_bits(x).view(np.int16)).view(torch.bfloat16)
+    else:
+        t = torch.from_numpy(np.ascontiguousarray(x, np.float32))
+    return t.pin_memory() if pin else t
+
+
+# ----------------------------------------------------------------------------- main
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="kvx", choices=["kvx", "reference"])
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work per core")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=10)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    spec = synth.config_specs()[args.workload]
+
+    if args.impl == "reference":
+        return reference_arm(args, spec, rank, world)
+
+    # spawn the oracle pool before any CUDA call
+    pool = None
+    cores = os.cpu_count() or 1
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        pool = mp.get_context("spawn").Pool(cores)
+
+    import torch
+    import paper_2608_30963_gb300 as kvx
+
+    torch.cuda.set_device(local_rank)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
+
+    wl = synth.make_workload(spec)
+    lm = list(wl.layer_map) if wl.layer_map is not None else nearest_map(spec.src.num_layers, spec.dst.num_layers)
+    alg = algorithmic(spec, wl, lm)
+    tdt = torch.bfloat16 if spec.dtype == "bf16" else torch.float32
+    kdt = kvx.KVX_BF16 if spec.dtype == "bf16" else kvx.KVX_FP32
+
+    # host inputs (pinned) and the translator
+    mapped = sorted(set(int(x) for x in lm))
+    host_k, host_v = {}, {}
+    for l in mapped:
+        k = synth.source_kv(wl, l, 0)
+        if spec.src.rope_base > 0:
+            k = rotate_np(k, spec.src.rope_base)
+        host_k[l] = to_torch(k, spec.dtype, torch, pin=True)
+        host_v[l] = to_torch(synth.source_kv(wl, l, 1), spec.dtype, torch, pin=True)
+    tr = kvx.Translator(spec.src, spec.dst, to_torch(synth.weights(wl, 0), spec.dtype, torch),
+                        to_torch(synth.weights(wl, 1), spec.dtype, torch), layer_map=lm, dtype=kdt)
+    info = tr.info()
+
+    dev = torch.device("cuda", local_rank)
+    i32 = lambda a: None if a is None else torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
+    src_len, seq_off = i32(wl.src_len), i32(wl.tgt_seq_off)
+    span_lo, span_hi = i32(wl.span_lo), i32(wl.span_hi)
+    page_table = i32(wl.page_table) if spec.paged else None
+    Lt, Ht, dt = spec.dst.num_layers, spec.dst.num_kv_heads, spec.dst.head_dim
+    out_shape = (wl.num_pages, spec.page_size, Ht, dt) if spec.paged else (wl.batch, Ht, wl.t_max, dt)
+
+    # rotating input/output sets so that consecutive steps share nothing in L2
+    l2_bytes = 129 * 2 ** 20
+    set_bytes = alg["read"] + alg["write"]
+    nsets = max(2, min(8, math.ceil(4 * l2_bytes / set_bytes)))
+    sets = []
+    for _ in range(nsets):
+        sk = {l: host_k[l].to(dev) for l in mapped}
+        sv = {l: host_v[l].to(dev) for l in mapped}
+        src_k = [sk.get(l, sk[mapped[0]]) for l in range(spec.src.num_layers)]
+        src_v = [sv.get(l, sv[mapped[0]]) for l in range(spec.src.num_layers)]
+        dk = [torch.empty(out_shape, dtype=tdt, device=dev) for _ in range(Lt)]
+        dv = [torch.empty(out_shape, dtype=tdt, device=dev) for _ in range(Lt)]
+        sets.append((src_k, src_v, dk, dv))
+    stream = torch.cuda.current_stream()
+
+    def step(i):
+        src_k, src_v, dk, dv = sets[i % nsets]
+        tr.translate(src_k, src_v, src_len, seq_off, wl.total_tgt, dk, dv, span_lo=span_lo, span_hi=span_hi,
+                     page_table=page_table, page_size=spec.page_size, num_pages=wl.num_pages, stream=stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if tr.device_status() != 0:
+        raise RuntimeError("device status nonzero after warm-up")
+
+    clocks = ClockSampler(local_rank)
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        ev[i][0].record(stream)
+        step(i)
+        ev[i][1].record(stream)
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    elapsed_ms = t_start.elapsed_time(t_end)
+    launch_ms = [a.elapsed_time(b) for a, b in ev]
+
+    # keep the GPU loaded long enough for the clock sampler to see it (>= 1 s)
+    extra = 0
+    t0 = time.perf_counter()
+    while time.perf_counter() - t0 < 1.0:
+        for i in range(50):
+            step(i)
+        torch.cuda.synchronize()
+        extra += 50
+    clk = clocks.stop()
+    if tr.device_status() != 0:
+        raise RuntimeError("device status nonzero after the timed region")
+
+    if dist:
+        t = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+
+    # end to end through the C ABI with host buffers: H2D source, translate, D2H target
+    e2e_steps = max(1, args.e2e_steps)
+    host_out = [torch.empty(out_shape, dtype=tdt).pin_memory() for _ in range(2 * Lt)]
+    src_k, src_v, dk, dv = sets[0]
+    h2d = sum(host_k[l].numel() * host_k[l].element_size() * 2 for l in mapped)
+    d2h = sum(t.numel() * t.element_size() for t in dk) * 2
+
+    def e2e_step():
+        for l in mapped:
+            src_k[l].copy_(host_k[l], non_blocking=True)
+            src_v[l].copy_(host_v[l], non_blocking=True)
+        tr.translate(src_k, src_v, src_len, seq_off, wl.total_tgt, dk, dv, span_lo=span_lo, span_hi=span_hi,
+                     page_table=page_table, page_size=spec.page_size, num_pages=wl.num_pages, stream=stream)
+        for j in range(Lt):
+            host_out[j].copy_(dk[j], non_blocking=True)
+            host_out[Lt + j].copy_(dv[j], non_blocking=True)
+
+    e2e_step()
+    torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = a.elapsed_time(b)
+    if dist:
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    if rank != 0:
+        if dist:
+            dist.destroy_process_group()
+        return
+
+    T = wl.total_tgt
+    value = T * args.steps * world / (elapsed_ms / 1e3)
+    ms_step = elapsed_ms / args.steps
+    avg_launch_ms = statistics.mean(launch_ms)
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        pass
+    hbm_peak = peaks.get("hbm_gbs")
+    peak_src = "measured" if hbm_peak else "fallback"
+    hbm_peak = hbm_peak or 6800.0
+    achieved = alg["bytes"] / (avg_launch_ms / 1e3) / 1e9
+    traffic = None
+    try:
+        tr_info = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))
+        if tr_info.get("workload") == args.workload and tr_info.get("kernel_rev") == kernel_rev():
+            traffic = tr_info.get("dram_bytes_per_launch")
+    except Exception:
+        pass
+    line = {
+        "metric": METRIC,
+        "value": value,
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_step,
+        "ms_per_handoff": ms_step,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": spec.dtype,
+        "data": "synthetic",
+        "config": {"workload": args.workload,
+                   "src": f"L{spec.src.num_layers} H{spec.src.num_kv_heads} d{spec.src.head_dim} base{spec.src.rope_base:g}",
+                   "dst": f"L{spec.dst.num_layers} H{spec.dst.num_kv_heads} d{spec.dst.head_dim} base{spec.dst.rope_base:g}",
+                   "target_tokens": T, "batch": wl.batch, "paged": spec.paged,
+                   "l2": f"inputs larger than L2: {nsets} rotating input/output sets of {set_bytes / 1e6:.1f} MB "
+                         f"(L2 129 MB)",
+                   "parallelism": f"replicas{world}" if world > 1 else "single"},
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "traffic": traffic,
+                     "peak_source": f"{peak_src} hbm_gbs (copy)",
+                     "algorithmic_bytes_per_launch": alg["bytes"], "avg_launch_ms": avg_launch_ms,
+                     "tensor_tflops": alg["flops"] / (avg_launch_ms / 1e3) / 1e12},
+        "clocks": clk,
+        "e2e": {"value": T * e2e_steps * world / (e2e_ms / 1e3), "unit": "tokens/s",
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / e2e_steps},
+        "gpu_launches": args.steps * tr.launches_per_translate(),
+        "kernel_path": {1: "simt", 2: "tcgen05"}.get(info.path, str(info.path)),
+    }
+    if pool is not None:
+        line["cpu_baseline"] = cpu_baseline(pool, args.workload, args.cpu_budget, cores)
+        pool.close()
+    print(json.dumps(line), flush=True)
+    tr.close()
+    if dist:
+        dist.destroy_process_group()
+
+
+def kernel_rev() -> str:
+    """Hash of the kernel sources, so a stored ncu traffic figure is only used for the kernel it measured."""
+    import hashlib
+    h = hashlib.sha1()
+    csrc = os.path.join(ROOT, "paper_2608_30963_gb300", "csrc")
+    for f in sorted(os.listdir(csrc)):
+        if f.endswith((".cu", ".cuh", ".h")):
+            h.update(open(os.path.join(csrc, f), "rb").read())
+    return h.hexdigest()[:12]
+
+
+def reference_arm(args, spec, rank, world):
+    """The oracle as the reference implementation, timed on the host cores."""
+    if rank != 0:
+        return
+    cores = os.cpu_count() or 1
+    pool = mp.get_context("spawn").Pool(cores)
+    budget = max(1.0, min(10.0, 120.0 / (args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        pool.map(_oracle_worker, [(args.workload, 13 * i, 2, 0) for i in range(cores)])
+    vals = []
+    for _ in range(args.steps):
+        cb = cpu_baseline(pool, args.workload, budget, cores)
+        vals.append(cb["value"])
+    pool.close()
+    value = statistics.mean(vals)
+    wl = synth.make_workload(spec)
+    line = {
+        "metric": METRIC, "value": value, "unit": "tokens/s", "impl": "reference", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": wl.total_tgt / value * 1e3,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": {"workload": args.workload, "target_tokens": wl.total_tgt},
+        "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                         "sample": cb["sample"]},
+        "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,215 @@
+/*
+ * kvx.h -- C ABI of the cross-model KV translation library (libkvx.so).
+ *
+ * Cross-model KV sharing (paper Section 4) turns the KV cache a source model A
+ * built for a context C into a cache a different target model B can decode
+ * from without its own prefill:  KV^_B(C) = T_{A->B}(KV_A(C)).  Section 5
+ * writes the translator as a parameterised map T_theta and lists the
+ * granularities it may act on (layers, groups of layers, KV heads, ...).  This
+ * library implements a per-target-layer, per-target-KV-head linear T_theta:
+ *
+ *   for target layer j, target KV head h, target token t (span [lo_t, hi_t)):
+ *     K^_j,h[t] = R_dst(p_t) . W_K[j,h]^T . mean_{s in span} concat_g R_src(-p_s) K_{map[j],g}[s]
+ *     V^_j,h[t] =              W_V[j,h]^T . mean_{s in span} concat_g            V_{map[j],g}[s]
+ *
+ * where map[] is the layer alignment, g runs over the source KV heads grouped
+ * into target head h (GQA regrouping), R(p) is the half-split rotary map at
+ * position p (angle p * base^(-2i/d) on channel pair (i, i+d/2)), and the
+ * result is written into the target model's contiguous or paged KV cache
+ * (the paper's "cache assembly", Section 6.1 and Table 4).
+ *
+ * Conventions for every entry point:
+ *   - All sizes are element counts unless a name says bytes.
+ *   - "device" pointers are CUDA device (or managed) memory of the current
+ *     device; "host" pointers are ordinary host memory.  The caller owns every
+ *     buffer it passes; the library never frees a caller buffer.
+ *   - stream is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *   - Calls return a kvx_status; on failure kvx_last_error() gives a message
+ *     for the calling thread.  Argument errors are detected on the host before
+ *     anything is launched.  Data errors that only the device can see (a span,
+ *     position or page index out of range) are clamped or skipped on the
+ *     device and recorded in the translator's device status word; read it with
+ *     kvx_get_device_status().  No kernel traps or waits without bound.
+ */
+#ifndef KVX_H
+#define KVX_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define KVX_API __attribute__((visibility("default")))
+
+typedef enum {
+    KVX_OK = 0,
+    KVX_ERR_INVALID_ARG = 1,    /* a pointer, size or stride is invalid */
+    KVX_ERR_UNSUPPORTED = 2,    /* a geometry this build has no kernel for */
+    KVX_ERR_CUDA = 3,           /* a CUDA runtime call failed */
+    KVX_ERR_OOM = 4,            /* device allocation failed (create only) */
+    KVX_ERR_DEVICE_STATUS = 5   /* kvx_get_device_status found a nonzero status */
+} kvx_status;
+
+typedef enum {
+    KVX_BF16 = 0,               /* bfloat16 caches and weights; fp32 arithmetic */
+    KVX_FP32 = 1                /* float32 caches and weights; fp32 arithmetic */
+} kvx_dtype;
+
+typedef enum {
+    KVX_PATH_AUTO = 0,          /* tcgen05 kernel for bf16 where supported, else SIMT */
+    KVX_PATH_SIMT = 1,          /* CUDA-core kernel (any supported geometry, both dtypes) */
+    KVX_PATH_TCGEN05 = 2        /* tensor-core kernel (bf16 only) */
+} kvx_path;
+
+/* Bits of the device status word. */
+#define KVX_DEV_SPAN_CLAMPED  0x01u  /* a span fell outside [0, seq_len) or was empty; clamped */
+#define KVX_DEV_POS_CLAMPED   0x02u  /* a RoPE position fell outside [0, max_position); clamped */
+#define KVX_DEV_PAGE_INVALID  0x04u  /* a page-table entry fell outside [0, num_pages); row not written */
+#define KVX_DEV_SEQ_CLAMPED   0x08u  /* a seq_len exceeded max_seq, or a target row fell outside the cache */
+#define KVX_DEV_WAIT_TIMEOUT  0x10u  /* an on-chip pipeline wait gave up after ~1 s; output incomplete */
+
+#define KVX_MAX_TARGET_LAYERS 128  /* target layers a translator may have */
+
+/* Geometry of one model's KV cache. */
+typedef struct {
+    int32_t num_layers;         /* N in KV_M(C) = {(K^(1),V^(1)) .. (K^(N),V^(N))} (Section 2.1) */
+    int32_t num_kv_heads;       /* KV heads per layer */
+    int32_t head_dim;           /* channels per head: 64, 128 or 256 */
+    double  rope_base;          /* RoPE base of K; <= 0 means K carries no rotary encoding */
+} kvx_model_geom;
+
+/* Translator description (the theta of T_theta, Section 5, plus the layer alignment). */
+typedef struct {
+    kvx_model_geom src;         /* source model A */
+    kvx_model_geom dst;         /* target model B */
+    const int32_t* layer_map;   /* host int32[dst.num_layers]: source layer feeding each target
+                                   layer, each in [0, src.num_layers); NULL = nearest relative
+                                   depth (kvx_layer_map_nearest) */
+    int32_t dtype;              /* kvx_dtype of caches and weights */
+    int32_t max_position;       /* RoPE positions must lie in [0, max_position); 0 = 1<<17.
+                                   At most 1<<22. Sizes the rotation tables. */
+    int32_t path;               /* kvx_path */
+} kvx_translator_desc;
+
+typedef struct kvx_translator kvx_translator;
+
+/* Build a translator.
+ *   w_k, w_v: translator matrices, row-major [dst.num_layers][dst.num_kv_heads][in][out] of
+ *     desc->dtype, with out = dst.head_dim and in = (src.num_kv_heads/dst.num_kv_heads) *
+ *     src.head_dim when src has at least as many KV heads as dst (the input row of target head
+ *     h concatenates source heads h*r .. h*r+r-1 in order), else in = src.head_dim (target
+ *     head h reads source head h / (dst.num_kv_heads/src.num_kv_heads)).
+ *   weights_on_device: 0 = host pointers, 1 = device pointers.
+ * The library copies the weights into its own device memory (re-laid out for its kernels) and
+ * builds its RoPE tables; the caller may free its copies on return.  Synchronous on the
+ * current device.  Returns KVX_ERR_UNSUPPORTED unless one head count divides the other,
+ * both head dims are in {64, 128, 256} and in <= 512 (in <= 256 for the tcgen05 path).
+ * On success *out owns device memory until kvx_destroy. */
+KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* desc, const void* w_k, const void* w_v,
+                                         int32_t weights_on_device, kvx_translator** out);
+
+/* Source KV cache KV_A(C) (Section 2.1), one K and one V tensor per source layer, each
+ * [batch][src.num_kv_heads][max_seq][src.head_dim] addressed by the strides below with the
+ * head_dim channels contiguous.  K holds the source model's post-RoPE keys. */
+typedef struct {
+    int32_t batch;
+    int32_t max_seq;            /* padded tokens per sequence in the source tensors */
+    const void* const* k;       /* host array [src.num_layers] of device pointers */
+    const void* const* v;       /* host array [src.num_layers] of device pointers */
+    int64_t stride_b, stride_h, stride_s;   /* elements; multiples of 8 for bf16, 4 for fp32 */
+    const int32_t* seq_len;     /* device int32[batch]: source tokens of each sequence (<= max_seq) */
+    const int32_t* pos;         /* device int32[batch*max_seq]: RoPE position of each source token,
+                                   or NULL for 0..seq_len-1 */
+} kvx_src_kv;
+
+/* Target tokens and their alignment to source tokens.  Target tokens of all sequences are
+ * packed: sequence b owns packed indices [seq_off[b], seq_off[b+1]). */
+typedef struct {
+    int32_t total_tokens;       /* T_total = seq_off[batch] (host copy, sizes the launch) */
+    const int32_t* seq_off;     /* device int32[batch+1], seq_off[0] = 0, non-decreasing */
+    const int32_t* span_lo;     /* device int32[T_total]: first source token (index within its
+                                   sequence) of each target token's span; NULL with span_hi
+                                   NULL = identity alignment (span of t is [t, t+1)) */
+    const int32_t* span_hi;     /* device int32[T_total]: one past the span's last source token */
+    const int32_t* pos;         /* device int32[T_total]: RoPE position of each target token, or
+                                   NULL for its index within its sequence */
+} kvx_tgt_tokens;
+
+/* Target KV cache written by kvx_translate: one K and one V tensor per target layer.
+ * Contiguous (paged = 0): element (b, h, t, c) at b*stride_b + h*stride_h + t*stride_t + c,
+ *   t < max_seq.
+ * Paged (paged = 1): pool [num_pages][page_size][dst.num_kv_heads][dst.head_dim]; token t of
+ *   sequence b lives in page page_table[b*max_pages_per_seq + t/page_size], slot t%page_size.
+ * Rows of padding tokens and of unlisted pages are not touched. */
+typedef struct {
+    void* const* k;             /* host array [dst.num_layers] of device pointers */
+    void* const* v;             /* host array [dst.num_layers] of device pointers */
+    int32_t paged;
+    int32_t max_seq;                        /* contiguous: token capacity per sequence */
+    int64_t stride_b, stride_h, stride_t;   /* contiguous: elements; multiples of 8 (bf16) / 4 (fp32) */
+    const int32_t* page_table;              /* paged: device int32[batch*max_pages_per_seq] */
+    int32_t max_pages_per_seq;
+    int32_t page_size;                      /* paged: tokens per page (16 in the evaluated setups) */
+    int32_t num_pages;                      /* paged: pages in the pool */
+} kvx_dst_kv;
+
+/* Translate KV_A(C) into the target cache: KV^_B(C) = T_theta(KV_A(C)) (Sections 4 and 5).
+ * Asynchronous on stream; allocates nothing; never synchronises.  The source, alignment and
+ * position buffers must stay valid and unchanged until the work on stream completes.  Output
+ * rows of distinct target tokens are written exactly once. */
+KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
+                                 const kvx_dst_kv* dst, void* stream);
+
+/* Token-span alignment from byte offsets (a target token is aligned to the source tokens whose
+ * last byte lies in its byte range; a target token that receives none takes the source token
+ * holding its own last byte).  Tokenizer differences are among the model differences the
+ * paper's translator must bridge (Sections 1 and 4).
+ *   src_end: device int32[total_src], tgt_end: device int32[total_tgt]: byte-end offsets of
+ *     each token, strictly increasing within a sequence and relative to the sequence start.
+ *   src_seq_off, tgt_seq_off: device int32[batch+1] packed offsets.
+ *   span_lo, span_hi: device int32[total_tgt] outputs (indices within each sequence).
+ *   dev_status: device uint32 or NULL; KVX_DEV_SPAN_CLAMPED is OR-ed in when a target text
+ *     runs past the end of its source text (span clamped to the last source token).
+ * Asynchronous on stream; allocates nothing. */
+KVX_API kvx_status kvx_build_alignment(int32_t batch, int32_t total_src, int32_t total_tgt,
+                                       const int32_t* src_seq_off, const int32_t* src_end,
+                                       const int32_t* tgt_seq_off, const int32_t* tgt_end,
+                                       int32_t* span_lo, int32_t* span_hi, uint32_t* dev_status,
+                                       void* stream);
+
+/* Layer alignment: out[j] = the source layer nearest target layer j in relative depth,
+ * round(j*(L_s-1)/(L_t-1)) with halves rounded up; out[0] = 0 when L_t = 1.  Host only. */
+KVX_API kvx_status kvx_layer_map_nearest(int32_t src_layers, int32_t dst_layers, int32_t* out);
+
+/* Synchronise stream, then read the translator's device status word into *bits (may be NULL)
+ * and, if clear != 0, reset it to zero.  Returns KVX_ERR_DEVICE_STATUS when it was nonzero. */
+KVX_API kvx_status kvx_get_device_status(kvx_translator* tr, void* stream, uint32_t* bits, int32_t clear);
+
+/* What kvx_translate will launch for this translator. */
+typedef struct {
+    int32_t path;               /* KVX_PATH_SIMT or KVX_PATH_TCGEN05 */
+    int32_t group_in;           /* in: input width of one translator matrix */
+    int32_t n_tile;             /* output columns per tensor-core tile (tcgen05) */
+    int32_t smem_bytes;         /* dynamic shared memory per CTA */
+    int32_t threads;            /* threads per CTA */
+    int32_t num_sms;            /* SMs of the device */
+    int64_t weight_bytes;       /* device bytes held for weights */
+    int64_t table_bytes;        /* device bytes held for RoPE tables */
+} kvx_translator_info;
+
+KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_translator_info* info);
+
+/* Kernel launches one kvx_translate call makes (for launch accounting). */
+KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
+
+/* Message of the last failed call on this thread ("" if none). */
+KVX_API const char* kvx_last_error(void);
+
+/* Free the translator's device memory.  Synchronises the device first.  NULL is accepted. */
+KVX_API kvx_status kvx_destroy(kvx_translator* tr);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* KVX_H */

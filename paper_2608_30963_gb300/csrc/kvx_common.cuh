@@ -1,0 +1,158 @@
+// kvx_common.cuh -- shared definitions of the kvx CUDA kernels (library-internal).
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/kvx.h"
+
+namespace kvx {
+
+// Rotation tables.  cos/sin of the exact angle p * f_i, f_i = base^(-2i/d), for
+// p = 64*a + c are rebuilt from two tables of fp32 (cos, sin) pairs computed in
+// double precision:  hi[a][i] = e^{j 64 a f_i},  lo[c][i] = e^{j c f_i},
+// e^{j p f_i} = hi[a][i] * lo[c][i] (complex product, fp32).  Error ~3 fp32 ulp.
+constexpr int kRopeLoBits = 6;
+constexpr int kRopeLo = 1 << kRopeLoBits;
+
+struct RopeTable {
+    const float2* hi;   // [max_position / 64 + 1][d/2]
+    const float2* lo;   // [64][d/2]
+    int half;           // d/2
+    int enabled;        // 0: no rotation
+};
+
+// Everything one kvx_translate launch needs, passed by value (graph-capturable;
+// no per-call device allocation or copy).
+struct TranslateParams {
+    // geometry
+    int Hs, ds, Ht, dt;
+    int in_dim;     // input width of one translator matrix
+    int r;          // source heads grouped into one target head (Hs >= Ht), else 1
+    int e;          // target heads sharing one source head (Ht > Hs), else 1
+    int Lt;
+    // source cache
+    int batch, src_max_seq;
+    long long sb, sh, ss;
+    const int* src_seq_len;
+    const int* src_pos;
+    // target tokens
+    int T_total;
+    const int* seq_off;
+    const int* span_lo;
+    const int* span_hi;
+    const int* tgt_pos;
+    // target cache
+    int paged, dst_max_seq;
+    long long db, dh, dts;
+    const int* page_table;
+    int max_pages, page_size, num_pages;
+    // rotation
+    RopeTable rs, rt;
+    int max_position;
+    unsigned* status;
+    // weights (layout depends on the kernel)
+    const void* w;
+    // per TARGET layer: the mapped source layer's K/V and the target layer's K/V
+    const void* src_k[KVX_MAX_TARGET_LAYERS];
+    const void* src_v[KVX_MAX_TARGET_LAYERS];
+    void* dst_k[KVX_MAX_TARGET_LAYERS];
+    void* dst_v[KVX_MAX_TARGET_LAYERS];
+};
+
+__device__ __forceinline__ void set_status(unsigned* status, unsigned bit)
+{
+    if (status) atomicOr(status, bit);
+}
+
+// (cos, sin) of angle p * f_i, with p clamped to [0, max_position).
+__device__ __forceinline__ float2 rope_cs(const RopeTable& t, int p, int i)
+{
+    float2 a = __ldg(&t.hi[(size_t)(p >> kRopeLoBits) * t.half + i]);
+    float2 b = __ldg(&t.lo[(size_t)(p & (kRopeLo - 1)) * t.half + i]);
+    return make_float2(a.x * b.x - a.y * b.y, a.y * b.x + a.x * b.y);
+}
+
+__device__ __forceinline__ int clamp_pos(int p, int max_position, unsigned* status)
+{
+    if (p < 0 || p >= max_position) {
+        set_status(status, KVX_DEV_POS_CLAMPED);
+        p = p < 0 ? 0 : max_position - 1;
+    }
+    return p;
+}
+
+// Sequence holding packed target token tp (seq_off non-decreasing; empty sequences skipped).
+__device__ __forceinline__ int find_seq(const int* seq_off, int batch, int tp)
+{
+    int lo = 0, hi = batch - 1;
+    while (lo < hi) {
+        int mid = (lo + hi + 1) >> 1;
+        if (__ldg(&seq_off[mid]) <= tp) lo = mid; else hi = mid - 1;
+    }
+    return lo;
+}
+
+template <typename T> __device__ __forceinline__ float to_f32(T x);
+template <> __device__ __forceinline__ float to_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ float to_f32<__nv_bfloat16>(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T> __device__ __forceinline__ T from_f32(float x);
+template <> __device__ __forceinline__ float from_f32<float>(float x) { return x; }
+template <> __device__ __forceinline__ __nv_bfloat16 from_f32<__nv_bfloat16>(float x) { return __float2bfloat16_rn(x); }
+
+// Per-target-token information resolved once per tile.
+struct TokenInfo {
+    int b;        // sequence
+    int t;        // index within the sequence
+    int lo, hi;   // clamped source span (within sequence), hi > lo unless the source is empty
+    int pt;       // target RoPE position (clamped)
+    long long dst_off;  // element offset of the output row for head 0 in the target cache, -1 = skip
+};
+
+__device__ __forceinline__ TokenInfo resolve_token(const TranslateParams& P, int tp)
+{
+    TokenInfo ti;
+    ti.b = find_seq(P.seq_off, P.batch, tp);
+    ti.t = tp - __ldg(&P.seq_off[ti.b]);
+    int S = __ldg(&P.src_seq_len[ti.b]);
+    if (S > P.src_max_seq || S < 0) { set_status(P.status, KVX_DEV_SEQ_CLAMPED); S = S < 0 ? 0 : P.src_max_seq; }
+    int lo, hi;
+    if (P.span_lo) { lo = __ldg(&P.span_lo[tp]); hi = __ldg(&P.span_hi[tp]); }
+    else { lo = ti.t; hi = ti.t + 1; }
+    if (lo < 0 || hi > S || hi <= lo) {
+        set_status(P.status, KVX_DEV_SPAN_CLAMPED);
+        lo = lo < 0 ? 0 : (lo > S - 1 ? S - 1 : lo);
+        hi = hi > S ? S : hi;
+        if (hi <= lo) hi = lo + 1;
+        if (S == 0) { lo = 0; hi = 0; }
+    }
+    ti.lo = lo; ti.hi = hi;
+    int p = P.tgt_pos ? __ldg(&P.tgt_pos[tp]) : ti.t;
+    ti.pt = P.rt.enabled ? clamp_pos(p, P.max_position, P.status) : 0;
+    if (!P.paged) {
+        if (ti.t >= P.dst_max_seq) { set_status(P.status, KVX_DEV_SEQ_CLAMPED); ti.dst_off = -1; }
+        else ti.dst_off = (long long)ti.b * P.db + (long long)ti.t * P.dts;
+    } else {
+        int pi = ti.t / P.page_size;
+        int page = pi < P.max_pages ? __ldg(&P.page_table[(size_t)ti.b * P.max_pages + pi]) : -1;
+        if (page < 0 || page >= P.num_pages) { set_status(P.status, KVX_DEV_PAGE_INVALID); ti.dst_off = -1; }
+        else ti.dst_off = ((long long)page * P.page_size + (ti.t % P.page_size)) * (long long)P.Ht * P.dt;
+    }
+    return ti;
+}
+
+// Element offset of head h within an output row block.
+__device__ __forceinline__ long long dst_head_off(const TranslateParams& P, int h)
+{
+    return P.paged ? (long long)h * P.dt : (long long)h * P.dh;
+}
+
+__device__ __forceinline__ int src_pos_of(const TranslateParams& P, int b, int s)
+{
+    int p = P.src_pos ? __ldg(&P.src_pos[(size_t)b * P.src_max_seq + s]) : s;
+    return clamp_pos(p, P.max_position, P.status);
+}
+
+}  // namespace kvx

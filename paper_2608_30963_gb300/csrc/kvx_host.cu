@@ -1,0 +1,336 @@
+// kvx_host.cu -- host side of the kvx C ABI: validation, translator state,
+// weight upload and re-layout, RoPE tables, launch selection, error status.
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include <string>
+
+#include "kvx_common.cuh"
+#include "kvx_kernels.h"
+
+using namespace kvx;
+
+struct kvx_translator {
+    kvx_translator_desc desc;
+    int layer_map[KVX_MAX_TARGET_LAYERS];
+    int device = 0;
+    int num_sms = 0;
+    int in_dim = 0, r = 1, e = 1;
+    int path = KVX_PATH_SIMT;
+    int max_position = 0;
+    void* w = nullptr;           // SIMT: [2][Lt][Ht][in][out] dtype; tcgen05: pre-swizzled images
+    size_t w_bytes = 0;
+    float2* rope = nullptr;      // src hi | src lo | dst hi | dst lo
+    size_t rope_bytes = 0;
+    RopeTable rs{}, rt{};
+    unsigned* status = nullptr;
+    TcConfig tc{};
+};
+
+static thread_local std::string g_last_error;
+
+static kvx_status fail(kvx_status s, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+static kvx_status fail(kvx_status s, const char* fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_last_error = buf;
+    return s;
+}
+
+#define CUDA_OR_FAIL(call)                                                                       \
+    do {                                                                                         \
+        cudaError_t e_ = (call);                                                                 \
+        if (e_ != cudaSuccess)                                                                   \
+            return fail(KVX_ERR_CUDA, "%s: %s (%s:%d)", #call, cudaGetErrorString(e_), __FILE__, \
+                        __LINE__);                                                               \
+    } while (0)
+
+static bool head_dim_ok(int d) { return d == 64 || d == 128 || d == 256; }
+
+extern "C" KVX_API const char* kvx_last_error(void) { return g_last_error.c_str(); }
+
+extern "C" KVX_API kvx_status kvx_layer_map_nearest(int32_t Ls, int32_t Lt, int32_t* out)
+{
+    if (Ls < 1 || Lt < 1 || !out) return fail(KVX_ERR_INVALID_ARG, "layer_map_nearest: bad arguments");
+    for (int j = 0; j < Lt; ++j) {
+        if (Lt == 1) { out[j] = 0; continue; }
+        // round(j (Ls-1) / (Lt-1)), halves up, in exact integers
+        const long long num = 2LL * j * (Ls - 1) + (Lt - 1);
+        out[j] = (int32_t)(num / (2LL * (Lt - 1)));
+    }
+    return KVX_OK;
+}
+
+static void free_translator(kvx_translator* t)
+{
+    if (!t) return;
+    if (t->w) cudaFree(t->w);
+    if (t->rope) cudaFree(t->rope);
+    if (t->status) cudaFree(t->status);
+    delete t;
+}
+
+extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* desc, const void* w_k,
+                                                    const void* w_v, int32_t weights_on_device,
+                                                    kvx_translator** out)
+{
+    if (!desc || !w_k || !w_v || !out) return fail(KVX_ERR_INVALID_ARG, "create: NULL argument");
+    *out = nullptr;
+    const kvx_model_geom& s = desc->src;
+    const kvx_model_geom& d = desc->dst;
+    if (s.num_layers < 1 || d.num_layers < 1 || s.num_kv_heads < 1 || d.num_kv_heads < 1)
+        return fail(KVX_ERR_INVALID_ARG, "create: layer and head counts must be >= 1");
+    if (d.num_layers > KVX_MAX_TARGET_LAYERS)
+        return fail(KVX_ERR_UNSUPPORTED, "create: at most %d target layers", KVX_MAX_TARGET_LAYERS);
+    if (!head_dim_ok(s.head_dim) || !head_dim_ok(d.head_dim))
+        return fail(KVX_ERR_UNSUPPORTED, "create: head dims must be 64, 128 or 256 (got %d, %d)", s.head_dim,
+                    d.head_dim);
+    if (s.num_kv_heads % d.num_kv_heads != 0 && d.num_kv_heads % s.num_kv_heads != 0)
+        return fail(KVX_ERR_UNSUPPORTED, "create: neither KV head count divides the other (%d, %d)",
+                    s.num_kv_heads, d.num_kv_heads);
+    if (desc->dtype != KVX_BF16 && desc->dtype != KVX_FP32)
+        return fail(KVX_ERR_INVALID_ARG, "create: unknown dtype %d", desc->dtype);
+    if (desc->path < KVX_PATH_AUTO || desc->path > KVX_PATH_TCGEN05)
+        return fail(KVX_ERR_INVALID_ARG, "create: unknown path %d", desc->path);
+    int max_pos = desc->max_position ? desc->max_position : (1 << 17);
+    if (max_pos < 1 || max_pos > (1 << 22))
+        return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<22]");
+
+    kvx_translator* t = new kvx_translator();
+    t->desc = *desc;
+    t->desc.layer_map = nullptr;
+    t->max_position = max_pos;
+    if (desc->layer_map) {
+        for (int j = 0; j < d.num_layers; ++j) {
+            if (desc->layer_map[j] < 0 || desc->layer_map[j] >= s.num_layers) {
+                delete t;
+                return fail(KVX_ERR_INVALID_ARG, "create: layer_map[%d] = %d outside [0, %d)", j,
+                            desc->layer_map[j], s.num_layers);
+            }
+            t->layer_map[j] = desc->layer_map[j];
+        }
+    } else {
+        kvx_layer_map_nearest(s.num_layers, d.num_layers, t->layer_map);
+    }
+    if (s.num_kv_heads >= d.num_kv_heads) {
+        t->r = s.num_kv_heads / d.num_kv_heads;
+        t->in_dim = t->r * s.head_dim;
+    } else {
+        t->e = d.num_kv_heads / s.num_kv_heads;
+        t->in_dim = s.head_dim;
+    }
+    if (t->in_dim > 512) {
+        delete t;
+        return fail(KVX_ERR_UNSUPPORTED, "create: translator input width %d > 512", t->in_dim);
+    }
+
+    if (cudaGetDevice(&t->device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&t->num_sms, cudaDevAttrMultiProcessorCount, t->device) != cudaSuccess) {
+        delete t;
+        return fail(KVX_ERR_CUDA, "create: no CUDA device");
+    }
+
+    // kernel choice
+    t->tc = tc_config(t->in_dim, d.head_dim, s.head_dim);
+    const bool tc_ok = desc->dtype == KVX_BF16 && t->tc.ok;
+    if (desc->path == KVX_PATH_TCGEN05 && !tc_ok) {
+        delete t;
+        return fail(KVX_ERR_UNSUPPORTED, "create: no tcgen05 kernel for this geometry/dtype (in=%d, d_t=%d)",
+                    t->in_dim, d.head_dim);
+    }
+    t->path = (desc->path == KVX_PATH_SIMT || !tc_ok) ? KVX_PATH_SIMT : KVX_PATH_TCGEN05;
+    if (t->path == KVX_PATH_SIMT && simt_smem_bytes(t->in_dim, d.head_dim) > 200 * 1024) {
+        delete t;
+        return fail(KVX_ERR_UNSUPPORTED, "create: SIMT kernel shared memory too large");
+    }
+
+    const size_t elt = desc->dtype == KVX_BF16 ? 2 : 4;
+    const size_t mat = (size_t)t->in_dim * d.head_dim;
+    const size_t one = (size_t)d.num_layers * d.num_kv_heads * mat * elt;   // bytes of w_k
+    kvx_status st = KVX_OK;
+    void* raw = nullptr;
+    cudaError_t ce;
+    const cudaMemcpyKind kind = weights_on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+
+    if (t->path == KVX_PATH_SIMT) {
+        t->w_bytes = 2 * one;
+        if (cudaMalloc(&t->w, t->w_bytes) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: weight allocation"); goto err; }
+        if ((ce = cudaMemcpy(t->w, w_k, one, kind)) != cudaSuccess ||
+            (ce = cudaMemcpy((char*)t->w + one, w_v, one, kind)) != cudaSuccess) {
+            st = fail(KVX_ERR_CUDA, "create: weight copy: %s", cudaGetErrorString(ce));
+            goto err;
+        }
+    } else {
+        t->w_bytes = tc_weight_image_bytes(t->in_dim, d.head_dim, d.num_layers, d.num_kv_heads);
+        if (cudaMalloc(&t->w, t->w_bytes) != cudaSuccess || cudaMalloc(&raw, 2 * one) != cudaSuccess) {
+            st = fail(KVX_ERR_OOM, "create: weight allocation");
+            goto err;
+        }
+        if ((ce = cudaMemcpy(raw, w_k, one, kind)) != cudaSuccess ||
+            (ce = cudaMemcpy((char*)raw + one, w_v, one, kind)) != cudaSuccess ||
+            (ce = launch_tc_weight_relayout(raw, (char*)raw + one, t->w, d.num_layers, d.num_kv_heads,
+                                            t->in_dim, d.head_dim, t->tc.n_tile, 0)) != cudaSuccess ||
+            (ce = cudaDeviceSynchronize()) != cudaSuccess) {
+            st = fail(KVX_ERR_CUDA, "create: weight re-layout: %s", cudaGetErrorString(ce));
+            goto err;
+        }
+        cudaFree(raw);
+        raw = nullptr;
+    }
+
+    {   // RoPE tables
+        const int n_hi = (max_pos + kRopeLo - 1) / kRopeLo + 1;
+        const size_t src_n = (size_t)(n_hi + kRopeLo) * (s.head_dim / 2);
+        const size_t dst_n = (size_t)(n_hi + kRopeLo) * (d.head_dim / 2);
+        t->rope_bytes = (src_n + dst_n) * sizeof(float2);
+        if (cudaMalloc(&t->rope, t->rope_bytes) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: table allocation"); goto err; }
+        float2* sh = t->rope;
+        float2* sl = sh + (size_t)n_hi * (s.head_dim / 2);
+        float2* dh = t->rope + src_n;
+        float2* dl = dh + (size_t)n_hi * (d.head_dim / 2);
+        t->rs = RopeTable{sh, sl, s.head_dim / 2, s.rope_base > 0.0};
+        t->rt = RopeTable{dh, dl, d.head_dim / 2, d.rope_base > 0.0};
+        if (t->rs.enabled && (ce = launch_rope_table(sh, sl, n_hi, s.head_dim, s.rope_base, 0)) != cudaSuccess) {
+            st = fail(KVX_ERR_CUDA, "create: rope table: %s", cudaGetErrorString(ce));
+            goto err;
+        }
+        if (t->rt.enabled && (ce = launch_rope_table(dh, dl, n_hi, d.head_dim, d.rope_base, 0)) != cudaSuccess) {
+            st = fail(KVX_ERR_CUDA, "create: rope table: %s", cudaGetErrorString(ce));
+            goto err;
+        }
+    }
+    if (cudaMalloc(&t->status, sizeof(unsigned)) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: status allocation"); goto err; }
+    if ((ce = cudaMemset(t->status, 0, sizeof(unsigned))) != cudaSuccess ||
+        (ce = cudaDeviceSynchronize()) != cudaSuccess) {
+        st = fail(KVX_ERR_CUDA, "create: %s", cudaGetErrorString(ce));
+        goto err;
+    }
+    *out = t;
+    return KVX_OK;
+err:
+    if (raw) cudaFree(raw);
+    free_translator(t);
+    return st;
+}
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
+                                            const kvx_dst_kv* dst, void* stream)
+{
+    if (!tr || !src || !tgt || !dst) return fail(KVX_ERR_INVALID_ARG, "translate: NULL argument");
+    const kvx_translator_desc& D = tr->desc;
+    const int Lt = D.dst.num_layers;
+    const int vec = D.dtype == KVX_BF16 ? 8 : 4;   // elements per 16 bytes
+    if (src->batch < 1) return fail(KVX_ERR_INVALID_ARG, "translate: batch must be >= 1");
+    if (src->max_seq < 0 || tgt->total_tokens < 0) return fail(KVX_ERR_INVALID_ARG, "translate: negative size");
+    if (!src->k || !src->v || !src->seq_len || !tgt->seq_off || !dst->k || !dst->v)
+        return fail(KVX_ERR_INVALID_ARG, "translate: NULL array");
+    if ((tgt->span_lo == nullptr) != (tgt->span_hi == nullptr))
+        return fail(KVX_ERR_INVALID_ARG, "translate: span_lo and span_hi must both be set or both NULL");
+    if (src->stride_s < D.src.head_dim || src->stride_h < 1 || src->stride_b < 1 || src->stride_s % vec ||
+        src->stride_h % vec || src->stride_b % vec)
+        return fail(KVX_ERR_INVALID_ARG, "translate: source strides must be positive multiples of %d "
+                                         "elements with stride_s >= head_dim", vec);
+    if (!dst->paged) {
+        if (dst->stride_t < D.dst.head_dim || dst->stride_h < 1 || dst->stride_b < 1 || dst->stride_t % vec ||
+            dst->stride_h % vec || dst->stride_b % vec || dst->max_seq < 0)
+            return fail(KVX_ERR_INVALID_ARG, "translate: target strides must be positive multiples of %d "
+                                             "elements with stride_t >= head_dim", vec);
+    } else if (!dst->page_table || dst->page_size < 1 || dst->max_pages_per_seq < 1 || dst->num_pages < 1) {
+        return fail(KVX_ERR_INVALID_ARG, "translate: paged target needs page_table, page_size, "
+                                         "max_pages_per_seq and num_pages >= 1");
+    }
+    if (tgt->total_tokens == 0) return KVX_OK;
+
+    TranslateParams P;
+    memset(&P, 0, sizeof P);
+    P.Hs = D.src.num_kv_heads; P.ds = D.src.head_dim;
+    P.Ht = D.dst.num_kv_heads; P.dt = D.dst.head_dim;
+    P.in_dim = tr->in_dim; P.r = tr->r; P.e = tr->e; P.Lt = Lt;
+    P.batch = src->batch; P.src_max_seq = src->max_seq;
+    P.sb = src->stride_b; P.sh = src->stride_h; P.ss = src->stride_s;
+    P.src_seq_len = src->seq_len; P.src_pos = src->pos;
+    P.T_total = tgt->total_tokens; P.seq_off = tgt->seq_off;
+    P.span_lo = tgt->span_lo; P.span_hi = tgt->span_hi; P.tgt_pos = tgt->pos;
+    P.paged = dst->paged; P.dst_max_seq = dst->max_seq;
+    P.db = dst->stride_b; P.dh = dst->stride_h; P.dts = dst->stride_t;
+    P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
+    P.page_size = dst->page_size; P.num_pages = dst->num_pages;
+    P.rs = tr->rs; P.rt = tr->rt; P.max_position = tr->max_position;
+    P.status = tr->status;
+    P.w = tr->w;
+    for (int j = 0; j < Lt; ++j) {
+        const int l = tr->layer_map[j];
+        P.src_k[j] = src->k[l]; P.src_v[j] = src->v[l];
+        P.dst_k[j] = dst->k[j]; P.dst_v[j] = dst->v[j];
+        if (!P.src_k[j] || !P.src_v[j] || !P.dst_k[j] || !P.dst_v[j])
+            return fail(KVX_ERR_INVALID_ARG, "translate: NULL cache pointer for target layer %d", j);
+        if (!aligned16(P.src_k[j]) || !aligned16(P.src_v[j]) || !aligned16(P.dst_k[j]) || !aligned16(P.dst_v[j]))
+            return fail(KVX_ERR_INVALID_ARG, "translate: cache pointers must be 16-byte aligned (layer %d)", j);
+    }
+    cudaError_t ce;
+    if (tr->path == KVX_PATH_TCGEN05) ce = launch_translate_tc(P, tr->tc, tr->num_sms, (cudaStream_t)stream);
+    else ce = launch_translate_simt(P, D.dtype, (cudaStream_t)stream);
+    if (ce != cudaSuccess) return fail(KVX_ERR_CUDA, "translate: launch failed: %s", cudaGetErrorString(ce));
+    return KVX_OK;
+}
+
+extern "C" KVX_API kvx_status kvx_build_alignment(int32_t batch, int32_t total_src, int32_t total_tgt,
+                                                  const int32_t* src_seq_off, const int32_t* src_end,
+                                                  const int32_t* tgt_seq_off, const int32_t* tgt_end,
+                                                  int32_t* span_lo, int32_t* span_hi, uint32_t* dev_status,
+                                                  void* stream)
+{
+    if (batch < 1 || total_src < 0 || total_tgt < 0)
+        return fail(KVX_ERR_INVALID_ARG, "build_alignment: bad sizes");
+    if (total_tgt == 0) return KVX_OK;
+    if (!src_seq_off || !tgt_seq_off || !tgt_end || !span_lo || !span_hi || (total_src > 0 && !src_end))
+        return fail(KVX_ERR_INVALID_ARG, "build_alignment: NULL array");
+    cudaError_t ce = launch_build_alignment(batch, total_tgt, src_seq_off, src_end, tgt_seq_off, tgt_end, span_lo,
+                                            span_hi, dev_status, (cudaStream_t)stream);
+    if (ce != cudaSuccess) return fail(KVX_ERR_CUDA, "build_alignment: %s", cudaGetErrorString(ce));
+    return KVX_OK;
+}
+
+extern "C" KVX_API kvx_status kvx_get_device_status(kvx_translator* tr, void* stream, uint32_t* bits, int32_t clear)
+{
+    if (!tr) return fail(KVX_ERR_INVALID_ARG, "get_device_status: NULL translator");
+    unsigned v = 0;
+    CUDA_OR_FAIL(cudaStreamSynchronize((cudaStream_t)stream));
+    CUDA_OR_FAIL(cudaMemcpy(&v, tr->status, sizeof v, cudaMemcpyDeviceToHost));
+    if (clear) CUDA_OR_FAIL(cudaMemset(tr->status, 0, sizeof v));
+    if (bits) *bits = v;
+    if (v) return fail(KVX_ERR_DEVICE_STATUS, "device status 0x%x", v);
+    return KVX_OK;
+}
+
+extern "C" KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_translator_info* info)
+{
+    if (!tr || !info) return fail(KVX_ERR_INVALID_ARG, "get_info: NULL argument");
+    info->path = tr->path;
+    info->group_in = tr->in_dim;
+    info->n_tile = tr->path == KVX_PATH_TCGEN05 ? tr->tc.n_tile : 0;
+    info->smem_bytes = tr->path == KVX_PATH_TCGEN05 ? tr->tc.smem_bytes
+                                                    : (int)simt_smem_bytes(tr->in_dim, tr->desc.dst.head_dim);
+    info->threads = tr->path == KVX_PATH_TCGEN05 ? tr->tc.threads : 256;
+    info->num_sms = tr->num_sms;
+    info->weight_bytes = (int64_t)tr->w_bytes;
+    info->table_bytes = (int64_t)tr->rope_bytes;
+    return KVX_OK;
+}
+
+extern "C" KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr) { return tr ? 1 : 0; }
+
+extern "C" KVX_API kvx_status kvx_destroy(kvx_translator* tr)
+{
+    if (!tr) return KVX_OK;
+    cudaDeviceSynchronize();
+    free_translator(tr);
+    return KVX_OK;
+}

@@ -1,0 +1,31 @@
+// kvx_kernels.h -- launchers of the kvx CUDA kernels (library-internal).
+#pragma once
+#include <cuda_runtime.h>
+#include <stddef.h>
+
+namespace kvx {
+struct TranslateParams;
+
+size_t simt_smem_bytes(int in_dim, int dt);
+cudaError_t launch_translate_simt(const TranslateParams& P, int dtype, cudaStream_t stream);
+
+cudaError_t launch_build_alignment(int batch, int total_tgt, const int* src_seq_off, const int* src_end,
+                                   const int* tgt_seq_off, const int* tgt_end, int* span_lo, int* span_hi,
+                                   unsigned* status, cudaStream_t stream);
+
+cudaError_t launch_rope_table(float2* hi, float2* lo, int n_hi, int d, double base, cudaStream_t stream);
+
+// tensor-core path
+struct TcConfig {
+    int n_tile;        // output columns per MMA tile
+    int n_split;       // d_t / n_tile
+    int smem_bytes;
+    int threads;
+    int ok;            // geometry supported
+};
+TcConfig tc_config(int in_dim, int dt, int ds);
+size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht);
+cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
+                                      int dt, int n_tile, cudaStream_t stream);
+cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, cudaStream_t stream);
+}  // namespace kvx

@@ -1,0 +1,215 @@
+"""CUDA path vs the CPU oracle, through the C ABI, on seeded synthetic inputs.
+
+Small cases are compared element by element over the whole output (several
+128-token tiles plus a ragged tail).  Full-size workloads, in the launch
+configuration bench.py times, are compared on sampled rows the oracle computes
+one by one.  Integer outputs (alignment spans) must be bit-exact.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle
+import paper_2608_30963_gb300 as kvx
+from paper_2608_30963_gb300 import synth
+
+from harness import compare, make_case, oracle_problem, sample_rows
+
+pytestmark = pytest.mark.gpu
+
+SPECS = synth.config_specs()
+PATHS = [kvx.KVX_PATH_SIMT, kvx.KVX_PATH_AUTO]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    kvx.build()
+    yield
+
+
+def _run(c, path, paged=None):
+    from gpu_harness import GpuRun
+    g = GpuRun(c, path=path, paged=paged)
+    g.run()
+    torch.cuda.synchronize()
+    return g
+
+
+def _full_compare(c, path, paged=None):
+    g = _run(c, path, paged)
+    ok, ov = oracle_problem(c).translate()
+    gk, gv = g.gather()
+    sk = compare(gk, ok, c.spec.dtype)
+    sv = compare(gv, ov, c.spec.dtype)
+    assert g.status() == 0
+    return g, sk, sv
+
+
+def _shrink(spec, Ls, Lt, **kw):
+    return dataclasses.replace(spec, src=dataclasses.replace(spec.src, num_layers=Ls),
+                               dst=dataclasses.replace(spec.dst, num_layers=Lt), **kw)
+
+
+# ------------------------------------------------------------------ small, whole output
+def test_tiny_fp32_full():
+    c = make_case(SPECS["tiny_fp32"])
+    _, sk, sv = _full_compare(c, kvx.KVX_PATH_AUTO)
+    assert sk["max_abs"] < 1e-4 and sv["max_abs"] < 1e-4
+
+
+SMALL = {
+    # name: (base spec, Ls, Lt, target lengths)
+    "qwen7b_qwen1p5b": ("qwen7b_to_qwen1p5b_4k", 3, 3, [300]),
+    "qwen1p5b_gemma2b": ("qwen1p5b_to_gemma2b_1k", 4, 3, [300]),
+    "llama70b_qwen7b": ("llama70b_to_qwen7b_8k", 9, 4, [300]),
+    "longctx_paged_varlen": ("longctx_8k_b4", 2, 2, [37, 300, 129, 1]),
+}
+
+
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+@pytest.mark.parametrize("name", list(SMALL))
+def test_small_full_output(name, path):
+    base, Ls, Lt, lens = SMALL[name]
+    spec = _shrink(SPECS[base], Ls, Lt)
+    c = make_case(spec, lens, pad_value=float("nan"))
+    _full_compare(c, path)
+
+
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+def test_explicit_positions_and_layer_map(path):
+    spec = _shrink(SPECS["llama70b_to_qwen7b_8k"], 5, 3, layer_map=[4, 0, 2])
+    wl = synth.make_workload(spec, [200, 77])
+    rng = np.random.default_rng(3)
+    src_pos = rng.integers(0, 120000, size=(wl.batch, wl.s_max)).astype(np.int32)
+    tgt_pos = (np.arange(wl.total_tgt) * 7 + 3000).astype(np.int32)
+    c = make_case(spec, [200, 77], src_pos=src_pos, tgt_pos=tgt_pos)
+    _full_compare(c, path)
+
+
+def test_tiny_token_counts_and_empty_sequences():
+    spec = _shrink(SPECS["qwen1p5b_to_gemma2b_1k"], 2, 2)
+    c = make_case(spec, [1, 0, 2, 0, 129])
+    for path in PATHS:
+        _full_compare(c, path)
+
+
+# ------------------------------------------------------------------ invariances (bit-exact)
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+def test_paged_equals_contiguous_and_batch_invariance(path):
+    spec = _shrink(SPECS["longctx_8k_b4"], 2, 2)
+    c = make_case(spec, [37, 300, 129])
+    gp = _run(c, path, paged=True)
+    gc = _run(c, path, paged=False)
+    pk, pv = gp.gather()
+    ck, cv = gc.gather()
+    np.testing.assert_array_equal(pk, ck)
+    np.testing.assert_array_equal(pv, cv)
+    solo = make_case(spec, [300])
+    # the second sequence alone: same source rows, same weights
+    for l in solo.src_k:
+        solo.src_k[l] = c.src_k[l][1:2, :, :300]
+        solo.src_v[l] = c.src_v[l][1:2, :, :300]
+    gs = _run(solo, path, paged=False)
+    sk, sv = gs.gather()
+    np.testing.assert_array_equal(sk, ck[:, :, 37:337])
+    np.testing.assert_array_equal(sv, cv[:, :, 37:337])
+
+
+# ------------------------------------------------------------------ full-size, sampled rows
+FULL = ["qwen7b_to_qwen1p5b_4k", "qwen1p5b_to_gemma2b_4k", "llama70b_to_qwen7b_8k", "longctx_8k_b4"]
+
+
+@pytest.mark.parametrize("name", FULL)
+def test_full_size_sampled(name):
+    c = make_case(SPECS[name])
+    g = _run(c, kvx.KVX_PATH_AUTO)
+    p = oracle_problem(c)
+    rows = sample_rows(c, 400)
+    gpu = np.stack([g.row(*r) for r in rows])
+    ref = np.stack([p.row(*r) for r in rows])
+    compare(gpu, ref, c.spec.dtype)
+    assert g.status() == 0
+
+
+# ------------------------------------------------------------------ alignment builder
+@pytest.mark.parametrize("key,ms,mt", [(0, 4.0, 4.0), (1, 5.0, 2.0), (2, 2.0, 6.0), (3, 1.0, 1.0)])
+def test_alignment_builder_bit_exact(key, ms, mt):
+    from gpu_harness import i32
+    src_ends, tgt_ends = [], []
+    for i, nb in enumerate([1, 57, 5000, 911]):
+        se, te = synth.draw_tokenizations(nb, ms, mt, key * 10 + i)
+        src_ends.append(se); tgt_ends.append(te)
+    so = np.concatenate([[0], np.cumsum([len(x) for x in src_ends])]).astype(np.int32)
+    to = np.concatenate([[0], np.cumsum([len(x) for x in tgt_ends])]).astype(np.int32)
+    se, te = np.concatenate(src_ends), np.concatenate(tgt_ends)
+    lo_ref, hi_ref, n = oracle.build_alignment(so, se, to, te)
+    T = int(to[-1])
+    lo = torch.full((T,), -7, dtype=torch.int32, device="cuda")
+    hi = torch.full((T,), -7, dtype=torch.int32, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    kvx.build_alignment(i32(so), i32(se), i32(to), i32(te), lo, hi, st)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(lo.cpu().numpy(), lo_ref)
+    np.testing.assert_array_equal(hi.cpu().numpy(), hi_ref)
+    assert int(st.item()) == 0 and n == 0
+
+
+def test_alignment_builder_recovers_generated_spans():
+    from gpu_harness import i32
+    spec = SPECS["qwen1p5b_to_gemma2b_4k"]
+    wl = synth.make_workload(spec, [4096, 1000, 3])
+    T = wl.total_tgt
+    lo = torch.empty(T, dtype=torch.int32, device="cuda")
+    hi = torch.empty(T, dtype=torch.int32, device="cuda")
+    kvx.build_alignment(i32(wl.src_seq_off), i32(wl.src_end), i32(wl.tgt_seq_off), i32(wl.tgt_end), lo, hi)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(lo.cpu().numpy(), wl.span_lo)
+    np.testing.assert_array_equal(hi.cpu().numpy(), wl.span_hi)
+
+
+# ------------------------------------------------------------------ device status (no faults)
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+def test_bad_spans_pages_positions_set_status_bits(path):
+    from gpu_harness import GpuRun, i32
+    spec = _shrink(SPECS["longctx_8k_b4"], 2, 2)
+    c = make_case(spec, [40, 20])
+    g = GpuRun(c, path=path, paged=True)
+    T = c.wl.total_tgt
+    lo = np.arange(T, dtype=np.int32) - np.repeat(c.wl.tgt_seq_off[:-1], c.wl.tgt_len)
+    hi = lo + 1
+    hi[5] = 10_000          # past the source length
+    g.span_lo, g.span_hi = i32(lo), i32(hi)
+    g.run()
+    assert g.status() & kvx.KVX_DEV_SPAN_CLAMPED
+    g.span_lo = g.span_hi = None
+    pt = c.wl.page_table.copy()
+    pt[1, 0] = 10_000       # page outside the pool
+    g.page_table = i32(pt)
+    g.run()
+    assert g.status() == kvx.KVX_DEV_PAGE_INVALID
+    g.page_table = i32(c.wl.page_table)
+    g.tgt_pos = i32(np.full(T, 1 << 30, np.int32))
+    g.run()
+    assert g.status() == kvx.KVX_DEV_POS_CLAMPED
+    g.tgt_pos = None
+    g.run()
+    assert g.status() == 0
+
+
+def test_invalid_arguments_rejected_before_launch():
+    from gpu_harness import GpuRun
+    spec = _shrink(SPECS["qwen7b_to_qwen1p5b_4k"], 2, 2)
+    c = make_case(spec, [64])
+    g = GpuRun(c)
+    g.span_hi = None          # span_lo without span_hi
+    g.span_lo = g.seq_off
+    with pytest.raises(kvx.KvxError) as e:
+        g.run()
+    assert e.value.status == kvx.KVX_ERR_INVALID_ARG
+    bad = synth.ModelGeom(2, 3, 128, 1e6)
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.Translator(bad, spec.dst, torch.zeros(1, device="cuda"), torch.zeros(1, device="cuda"))
+    assert e.value.status == kvx.KVX_ERR_UNSUPPORTED

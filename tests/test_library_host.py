@@ -1,0 +1,88 @@
+"""Host-side checks of libkvx.so (no GPU needed).
+
+The library builds for sm_103a, loads, exports every symbol include/kvx.h
+declares, and its host-only logic (layer map, argument validation) behaves.
+"""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle
+import paper_2608_30963_gb300 as kvx
+from paper_2608_30963_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    kvx.build()
+    return kvx.lib()
+
+
+def declared_symbols():
+    txt = open(os.path.join(ROOT, "include", "kvx.h")).read()
+    return sorted(set(re.findall(r"KVX_API\s+[\w\s\*]+?\b(kvx_\w+)\s*\(", txt)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    for must in ("kvx_translator_create", "kvx_translate", "kvx_destroy", "kvx_build_alignment",
+                 "kvx_layer_map_nearest", "kvx_get_device_status", "kvx_last_error"):
+        assert must in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_symbols():
+        assert hasattr(lib, name), name
+    assert sorted(declared_symbols()) == sorted(kvx.EXPORTS) or set(kvx.EXPORTS) <= set(declared_symbols())
+
+
+@pytest.mark.parametrize("Ls,Lt", [(4, 2), (28, 28), (28, 26), (80, 28), (1, 3), (5, 1), (3, 7)])
+def test_layer_map_matches_oracle(lib, Ls, Lt):
+    assert kvx.kvx_layer_map_nearest(Ls, Lt) == list(oracle.layer_map_nearest(Ls, Lt))
+
+
+def _desc(src, dst, dtype=kvx.KVX_BF16, path=kvx.KVX_PATH_AUTO, layer_map=None):
+    g = lambda m: kvx.kvx_model_geom(m.num_layers, m.num_kv_heads, m.head_dim, m.rope_base)
+    return kvx.kvx_translator_desc(g(src), g(dst), layer_map, dtype, 0, path)
+
+
+@pytest.mark.parametrize("src,dst,code", [
+    (synth.ModelGeom(2, 3, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),   # 3 vs 2 heads
+    (synth.ModelGeom(2, 2, 96, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),    # head_dim 96
+    (synth.ModelGeom(2, 16, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),  # in = 1024
+    (synth.ModelGeom(0, 2, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_INVALID_ARG),
+    (synth.ModelGeom(2, 2, 128, 1e6), synth.ModelGeom(200, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),
+])
+def test_create_rejects_bad_geometry_without_touching_cuda(lib, src, dst, code):
+    h = ctypes.c_void_p()
+    w = (ctypes.c_uint16 * 4)()
+    st = lib.kvx_translator_create(ctypes.byref(_desc(src, dst)), ctypes.cast(w, ctypes.c_void_p),
+                                   ctypes.cast(w, ctypes.c_void_p), 0, ctypes.byref(h))
+    assert st == code
+    assert h.value is None
+    assert kvx.kvx_last_error()
+
+
+def test_create_rejects_out_of_range_layer_map(lib):
+    lm = (ctypes.c_int32 * 2)(0, 5)
+    d = _desc(synth.ModelGeom(4, 2, 64, 1e4), synth.ModelGeom(2, 1, 64, 1e4),
+              layer_map=ctypes.cast(lm, kvx.I32P))
+    h = ctypes.c_void_p()
+    w = (ctypes.c_float * 4)()
+    st = lib.kvx_translator_create(ctypes.byref(d), ctypes.cast(w, ctypes.c_void_p),
+                                   ctypes.cast(w, ctypes.c_void_p), 0, ctypes.byref(h))
+    assert st == kvx.KVX_ERR_INVALID_ARG
+    assert "layer_map" in kvx.kvx_last_error()
+
+
+def test_null_arguments_rejected(lib):
+    assert lib.kvx_translate(None, None, None, None, None) == kvx.KVX_ERR_INVALID_ARG
+    assert lib.kvx_get_device_status(None, None, None, 0) == kvx.KVX_ERR_INVALID_ARG
+    assert lib.kvx_destroy(None) == kvx.KVX_OK
+    assert lib.kvx_build_alignment(0, 0, 0, None, None, None, None, None, None, None, None) == \
+        kvx.KVX_ERR_INVALID_ARG
