@@ -1,16 +1,842 @@
-// kvx_tc.cu -- tensor-core (tcgen05/TMEM) translation kernel.  Placeholder: not yet built.
+// kvx_tc.cu -- tensor-core translation kernel for sm_103a (tcgen05 / TMEM / bulk copies).
+//
+// The per-(target layer, target KV head, K|V) projection of T_theta (paper
+// Section 5) is a dense [T x in] . [in x d_t] contraction; everything around it
+// (span gather, RoPE undo, span mean, RoPE apply, cache write) is streaming work
+// fused into the GEMM's prologue and epilogue.
+//
+// Persistent kernel, one CTA per SM, work unit = (group, 128-token tile) with
+// group = (target layer j, target head h, K|V, output split nt).  A CTA walks a
+// contiguous range of units, so the group's weight tile (B operand) stays in
+// shared memory across its token tiles.  Warp roles:
+//   warp 0      producer: resolves the spans of each 32-token sub-tile and
+//               streams the needed source rows into a byte ring in shared memory
+//               with cp.async.bulk (mbarrier transaction counts); loads B images.
+//   warp 1      MMA: allocates TMEM, issues tcgen05.mma (M=128, N=n_tile, K=16
+//               steps over in) into a double-buffered fp32 accumulator.
+//   warps 2-5   epilogue: tcgen05.ld the accumulator (one thread per token row),
+//               apply the target RoPE, round to bf16, stage the row and write it
+//               to the target cache (contiguous or paged) with cp.async.bulk.
+//   warps 6-13  prologue: one warp per target token at a time, lanes across the
+//               in channels: undo the source RoPE of each span row, take the span
+//               mean, round to bf16 and store the A tile in the UMMA K-major
+//               128-byte-swizzled layout.
+// Every wait is a bounded mbarrier poll: after ~1 s it records
+// KVX_DEV_WAIT_TIMEOUT, raises a CTA-wide abort flag and the kernel drains and
+// returns (no trap, no hang).
 #include "kvx_common.cuh"
 #include "kvx_kernels.h"
 
 namespace kvx {
-TcConfig tc_config(int, int, int) { return TcConfig{0, 0, 0, 0, 0}; }
-size_t tc_weight_image_bytes(int, int, int, int) { return 0; }
-cudaError_t launch_tc_weight_relayout(const void*, const void*, void*, int, int, int, int, int, cudaStream_t)
+namespace {
+
+constexpr int kTileM = 128;
+constexpr int kSub = 32;
+constexpr int kSubPerTile = kTileM / kSub;
+constexpr int kNumSlots = 8;
+constexpr int kProducerWarp = 0;
+constexpr int kMmaWarp = 1;
+constexpr int kEpiWarp0 = 2;
+constexpr int kNumEpiWarps = 4;
+constexpr int kXfWarp0 = 6;
+constexpr int kNumXfWarps = 8;
+constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
+constexpr int kSmemMax = 232448;          // 227 KB opt-in per block
+constexpr unsigned long long kWaitNs = 1000000000ull;
+
+// barrier indices
+constexpr int kBarBFull = 0, kBarBEmpty = 1, kBarAFull = 2, kBarAEmpty = 3;
+constexpr int kBarDFull = 4;               // +buf (2)
+constexpr int kBarDEmpty = 6;              // +buf (2)
+constexpr int kBarSlotFull = 8;            // +slot
+constexpr int kBarSlotEmpty = 8 + kNumSlots;
+constexpr int kNumBars = 8 + 2 * kNumSlots;
+
+struct SubMeta {
+    int stage_row;   // stage row of the span start; < 0: rows are read from global memory
+    int lo, hi;      // source span within the sequence (hi <= lo: nothing to gather)
+    int b;           // sequence
+};
+
+struct SlotHdr {
+    unsigned rows;     // rows per head staged for the sub-tile
+    unsigned offset;   // byte offset of the sub-tile's region in the ring
+};
+
+struct TcLaunch {
+    int n_tile, n_split, in_dim, groups, m_tiles;
+    unsigned b_bytes, a_bytes, row_bytes, stage_row_bytes, ring_bytes;
+    unsigned off_b, off_a, off_stage, off_ring, off_meta, off_hdr, off_bar, off_misc;
+    unsigned idesc;
+    unsigned tmem_cols;
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
 {
-    return cudaErrorNotSupported;
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
 }
-cudaError_t launch_translate_tc(const TranslateParams&, const TcConfig&, int, cudaStream_t)
+__device__ __forceinline__ void mbar_arrive(uint32_t bar)
 {
-    return cudaErrorNotSupported;
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
+{
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+__device__ __forceinline__ unsigned long long globaltimer()
+{
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
+    return t;
+}
+__device__ __forceinline__ uint64_t policy_evict_first()
+{
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+__device__ __forceinline__ uint64_t policy_evict_last()
+{
+    uint64_t p;
+    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+    return p;
+}
+// global -> shared bulk copy completing on an mbarrier (16-byte aligned, size % 16 == 0)
+__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar, uint64_t pol)
+{
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(dst),
+        "l"(src), "r"(bytes), "r"(bar), "l"(pol)
+        : "memory");
+}
+// shared -> global bulk copy in the thread's bulk group
+__device__ __forceinline__ void bulk_s2g(void* dst, uint32_t src, uint32_t bytes)
+{
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
+
+__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols)
+{
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish()
+{
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
+{
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// D[tmem] (+)= A[smem] . B[smem]^T, bf16 inputs, fp32 accumulate
+__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                          uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+__device__ __forceinline__ void umma_commit(uint32_t bar)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row atoms 1024 B apart.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);      // start address
+    d |= (uint64_t)1 << 16;                         // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024u >> 4) << 32;              // stride byte offset between 8-row atoms
+    d |= (uint64_t)1 << 46;                         // descriptor version
+    d |= (uint64_t)2 << 61;                         // 128-byte swizzle
+    return d;
+}
+
+// Byte offset of element (row, k) in a K-major SW128 tile with `rows` rows
+// (K split into 64-element blocks of rows*128 bytes).
+__device__ __forceinline__ uint32_t sw128_off(int row, int k, int rows)
+{
+    const int kb = k >> 6, c = (k >> 3) & 7, e = k & 7;
+    return (uint32_t)(kb * rows * 128 + (row >> 3) * 1024 + (row & 7) * 128 + ((c ^ (row & 7)) << 4) + e * 2);
+}
+
+// ------------------------------------------------------------------ bounded waits
+struct Waiter {
+    volatile int* abort;
+    unsigned* status;
+    __device__ __forceinline__ bool wait(uint32_t bar, uint32_t parity) const
+    {
+        if (mbar_try_wait(bar, parity)) return true;
+        const unsigned long long t0 = globaltimer();
+        while (true) {
+            if (mbar_try_wait(bar, parity)) return true;
+            if (*abort) return false;
+            if (globaltimer() - t0 > kWaitNs) {
+                *abort = 1;
+                set_status(status, KVX_DEV_WAIT_TIMEOUT);
+                return false;
+            }
+        }
+    }
+};
+
+struct Unit {
+    int j, h, kv, nt, tile, g;
+};
+__device__ __forceinline__ Unit decode(long long u, const TcLaunch& L, int Ht)
+{
+    Unit x;
+    x.g = (int)(u / L.m_tiles);
+    x.tile = (int)(u - (long long)x.g * L.m_tiles);
+    int rest = x.g;
+    x.nt = rest % L.n_split;
+    rest /= L.n_split;
+    x.kv = rest & 1;
+    rest >>= 1;
+    x.h = rest % Ht;
+    x.j = rest / Ht;
+    return x;
+}
+
+// Source-side resolution of one target token (sequence, clamped span).
+__device__ __forceinline__ void resolve_src(const TranslateParams& P, int tp, int& b, int& lo, int& hi)
+{
+    b = find_seq(P.seq_off, P.batch, tp);
+    const int t = tp - __ldg(&P.seq_off[b]);
+    int S = __ldg(&P.src_seq_len[b]);
+    if (S > P.src_max_seq || S < 0) {
+        set_status(P.status, KVX_DEV_SEQ_CLAMPED);
+        S = S < 0 ? 0 : P.src_max_seq;
+    }
+    if (P.span_lo) { lo = __ldg(&P.span_lo[tp]); hi = __ldg(&P.span_hi[tp]); }
+    else { lo = t; hi = t + 1; }
+    if (lo < 0 || hi > S || hi <= lo) {
+        set_status(P.status, KVX_DEV_SPAN_CLAMPED);
+        lo = lo < 0 ? 0 : (lo > S - 1 ? S - 1 : lo);
+        hi = hi > S ? S : hi;
+        if (hi <= lo) hi = lo + 1;
+        if (S == 0) { lo = 0; hi = 0; }
+    }
+}
+
+__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ uint32_t pack_bf16(float a, float b)
+{
+    __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// Load PP consecutive bf16 values (PP in {1,2,4}) into floats.
+template <int PP>
+__device__ __forceinline__ void load_bf16(const __nv_bfloat16* p, float (&x)[PP])
+{
+    if constexpr (PP == 4) {
+        const uint2 w = *reinterpret_cast<const uint2*>(p);
+        x[0] = bf_lo(w.x); x[1] = bf_hi(w.x); x[2] = bf_lo(w.y); x[3] = bf_hi(w.y);
+    } else if constexpr (PP == 2) {
+        const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
+        x[0] = bf_lo(w); x[1] = bf_hi(w);
+    } else {
+        const unsigned short w = *reinterpret_cast<const unsigned short*>(p);
+        x[0] = __uint_as_float((uint32_t)w << 16);
+    }
+}
+template <int PP>
+__device__ __forceinline__ void store_bf16_smem(uint8_t* p, const float (&x)[PP])
+{
+    if constexpr (PP == 4) {
+        *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]));
+    } else if constexpr (PP == 2) {
+        *reinterpret_cast<uint32_t*>(p) = pack_bf16(x[0], x[1]);
+    } else {
+        __nv_bfloat16 v = __float2bfloat16_rn(x[0]);
+        *reinterpret_cast<__nv_bfloat16*>(p) = v;
+    }
+}
+
+// (cos, sin) for PP consecutive frequencies i0.. at position p.
+template <int PP>
+__device__ __forceinline__ void rope_cs_vec(const RopeTable& t, int p, int i0, float (&c)[PP], float (&s)[PP])
+{
+    const float2* hp = t.hi + (size_t)(p >> kRopeLoBits) * t.half + i0;
+    const float2* lp = t.lo + (size_t)(p & (kRopeLo - 1)) * t.half + i0;
+    float2 a[PP], b[PP];
+    if constexpr (PP >= 2) {
+#pragma unroll
+        for (int q = 0; q < PP; q += 2) {
+            const float4 va = __ldg(reinterpret_cast<const float4*>(hp + q));
+            const float4 vb = __ldg(reinterpret_cast<const float4*>(lp + q));
+            a[q] = make_float2(va.x, va.y); a[q + 1] = make_float2(va.z, va.w);
+            b[q] = make_float2(vb.x, vb.y); b[q + 1] = make_float2(vb.z, vb.w);
+        }
+    } else {
+        a[0] = __ldg(hp);
+        b[0] = __ldg(lp);
+    }
+#pragma unroll
+    for (int q = 0; q < PP; ++q) {
+        c[q] = a[q].x * b[q].x - a[q].y * b[q].y;
+        s[q] = a[q].y * b[q].x + a[q].x * b[q].y;
+    }
+}
+
+// ------------------------------------------------------------------ the kernel
+template <int PP>
+__global__ void __launch_bounds__(kThreads, 1)
+translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_constant__ TcLaunch L)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t* sB = smem + L.off_b;
+    uint8_t* sA = smem + L.off_a;
+    uint8_t* sStage = smem + L.off_stage;
+    uint8_t* sRing = smem + L.off_ring;
+    SubMeta* sMeta = reinterpret_cast<SubMeta*>(smem + L.off_meta);
+    SlotHdr* sHdr = reinterpret_cast<SlotHdr*>(smem + L.off_hdr);
+    uint64_t* sBar = reinterpret_cast<uint64_t*>(smem + L.off_bar);
+    volatile int* sAbort = reinterpret_cast<volatile int*>(smem + L.off_misc);
+    uint32_t* sTmemBase = reinterpret_cast<uint32_t*>(smem + L.off_misc + 4);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    auto bar = [&](int i) { return smem_u32(&sBar[i]); };
+
+    if (threadIdx.x == 0) {
+        *sAbort = 0;
+        mbar_init(bar(kBarBFull), 1);
+        mbar_init(bar(kBarBEmpty), 1);
+        mbar_init(bar(kBarAFull), kNumXfWarps);
+        mbar_init(bar(kBarAEmpty), 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(kBarDFull + i), 1);
+            mbar_init(bar(kBarDEmpty + i), kNumEpiWarps);
+        }
+        for (int i = 0; i < kNumSlots; ++i) {
+            mbar_init(bar(kBarSlotFull + i), 1);
+            mbar_init(bar(kBarSlotEmpty + i), kNumXfWarps);
+        }
+        fence_mbar_init();
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc(smem_u32(sTmemBase), L.tmem_cols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *sTmemBase;
+
+    const Waiter W{sAbort, P.status};
+    const long long U = (long long)L.groups * L.m_tiles;
+    const long long u_begin = (long long)blockIdx.x * U / gridDim.x;
+    const long long u_end = (long long)(blockIdx.x + 1) * U / gridDim.x;
+    const int hw = L.n_tile >> 1;                 // pair half-width of an output split
+    const int half_t = P.dt >> 1;
+
+    if (warp == kProducerWarp) {
+        // ------------------------------------------------------------ producer
+        const uint64_t pol_stream = policy_evict_first();
+        const uint64_t pol_keep = policy_evict_last();
+        const int r_heads = L.in_dim / P.ds;         // source heads per A row (1 when expanding)
+        const bool rows_contig = P.ss == P.ds;
+        int cur_g = -1;
+        uint32_t b_loads = 0, issued = 0, released = 0;
+        unsigned long long head = 0;                 // monotonic ring byte counter
+        unsigned long long slot_start[kNumSlots];
+        bool ok = true;
+        // wait until sub-tile k (0-based) has been released by the prologue warps
+        auto release_upto = [&](uint32_t k) -> bool {
+            while (released < k) {
+                if (!W.wait(bar(kBarSlotEmpty + released % kNumSlots), (released / kNumSlots) & 1)) return false;
+                ++released;
+            }
+            return true;
+        };
+        for (long long u = u_begin; u < u_end && ok; ++u) {
+            const Unit x = decode(u, L, P.Ht);
+            if (x.g != cur_g) {
+                if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
+                if (lane == 0) mbar_arrive_expect_tx(bar(kBarBFull), L.b_bytes);
+                __syncwarp();
+                const uint8_t* img = (const uint8_t*)P.w + (size_t)x.g * L.b_bytes;
+                const uint32_t piece = L.b_bytes / 4;
+                if (lane < 4)
+                    bulk_g2s(smem_u32(sB) + lane * piece, img + (size_t)lane * piece, piece, bar(kBarBFull), pol_keep);
+                ++b_loads;
+                cur_g = x.g;
+            }
+            const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
+            const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
+            for (int sq = 0; sq < kSubPerTile; ++sq) {
+                const int tp = x.tile * kTileM + sq * kSub + lane;
+                const bool valid = tp < P.T_total;
+                int b = -1, lo = 0, hi = 0;
+                if (valid) resolve_src(P, tp, b, lo, hi);
+                const int b_prev = __shfl_up_sync(0xffffffffu, b, 1);
+                const int lo_prev = __shfl_up_sync(0xffffffffu, lo, 1);
+                const int hi_prev = __shfl_up_sync(0xffffffffu, hi, 1);
+                const bool first = valid && (lane == 0 || b_prev != b);
+                const bool nonmono = valid && !first && (lo < lo_prev || hi < hi_prev);
+                const int cover = first ? lo : max(lo, hi_prev);
+                const int n_new = valid ? max(0, hi - cover) : 0;
+                int incl = n_new;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+                    if (lane >= o) incl += v;
+                }
+                const int start = incl - n_new;
+                const unsigned R = (unsigned)__shfl_sync(0xffffffffu, incl, 31);
+                const unsigned need_rows = R * (unsigned)r_heads;
+                const bool direct = __any_sync(0xffffffffu, nonmono) ||
+                                    (unsigned long long)need_rows * L.row_bytes > L.ring_bytes;
+                const unsigned need = direct ? 0u : need_rows * L.row_bytes;
+
+                // slot reuse and ring space
+                const uint32_t slot = issued % kNumSlots;
+                if (issued >= kNumSlots && !release_upto(issued - kNumSlots + 1)) { ok = false; break; }
+                unsigned long long off = head;
+                if (need) {
+                    if (off % L.ring_bytes + need > L.ring_bytes) off = (off / L.ring_bytes + 1) * L.ring_bytes;
+                    while (true) {
+                        const unsigned long long tail = released == issued ? off : slot_start[released % kNumSlots];
+                        if (off + need - tail <= L.ring_bytes) break;
+                        if (!release_upto(released + 1)) { ok = false; break; }
+                    }
+                    if (!ok) break;
+                }
+                head = off + need;
+                slot_start[slot] = off;
+                const unsigned roff = (unsigned)(off % L.ring_bytes);
+
+                SubMeta mt;
+                mt.stage_row = direct ? -1 : start - (cover - lo);
+                mt.lo = lo;
+                mt.hi = hi;
+                mt.b = b;
+                if (!valid) { mt.lo = 0; mt.hi = 0; mt.b = 0; }
+                sMeta[slot * kSub + lane] = mt;
+                if (lane == 0) sHdr[slot] = SlotHdr{R, roff};
+                __threadfence_block();
+                __syncwarp();
+                if (lane == 0) {
+                    if (need) mbar_arrive_expect_tx(bar(kBarSlotFull + slot), need);
+                    else mbar_arrive(bar(kBarSlotFull + slot));
+                }
+                __syncwarp();
+                if (need) {
+                    const uint32_t ring0 = smem_u32(sRing) + roff;
+                    if (rows_contig) {
+                        // one copy per (contiguous run of source rows, head)
+                        const bool run_start = n_new > 0 && (first || lo > hi_prev);
+                        const unsigned runs = __ballot_sync(0xffffffffu, run_start);
+                        const unsigned later = lane < 31 ? runs & (0xffffffffu << (lane + 1)) : 0u;
+                        const int nxt = later ? __ffs(later) - 1 : 32;
+                        const int nxt_start = __shfl_sync(0xffffffffu, start, nxt < 32 ? nxt : lane);
+                        if (run_start) {
+                            const unsigned rows = (nxt < 32 ? (unsigned)nxt_start : R) - (unsigned)start;
+                            for (int q = 0; q < r_heads; ++q) {
+                                const __nv_bfloat16* s0 =
+                                    src + (long long)b * P.sb + (long long)(g0 + q) * P.sh + (long long)cover * P.ss;
+                                bulk_g2s(ring0 + ((unsigned)q * R + (unsigned)start) * L.row_bytes, s0,
+                                         rows * L.row_bytes, bar(kBarSlotFull + slot), pol_stream);
+                            }
+                        }
+                    } else {
+                        for (int s = cover; s < cover + n_new; ++s)
+                            for (int q = 0; q < r_heads; ++q) {
+                                const __nv_bfloat16* s0 =
+                                    src + (long long)b * P.sb + (long long)(g0 + q) * P.sh + (long long)s * P.ss;
+                                bulk_g2s(ring0 + ((unsigned)q * R + (unsigned)(start + s - cover)) * L.row_bytes,
+                                         s0, L.row_bytes, bar(kBarSlotFull + slot), pol_stream);
+                            }
+                    }
+                }
+                ++issued;
+            }
+        }
+        // on abort, let copies already in flight land before the CTA leaves
+        if (*sAbort) {
+            const unsigned long long t0 = globaltimer();
+            for (uint32_t c = issued > kNumSlots ? issued - kNumSlots : 0; c < issued; ++c)
+                while (!mbar_try_wait(bar(kBarSlotFull + c % kNumSlots), (c / kNumSlots) & 1) &&
+                       globaltimer() - t0 < kWaitNs) {}
+            if (b_loads)
+                while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < kWaitNs) {}
+        }
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            int cur_g = -1;
+            uint32_t b_cnt = 0, tcount = 0;
+            for (long long u = u_begin; u < u_end; ++u) {
+                const Unit x = decode(u, L, P.Ht);
+                if (x.g != cur_g) {
+                    if (!W.wait(bar(kBarBFull), b_cnt & 1)) break;
+                    ++b_cnt;
+                    cur_g = x.g;
+                }
+                const uint32_t buf = tcount & 1;
+                if (!W.wait(bar(kBarDEmpty + buf), ((tcount >> 1) & 1) ^ 1)) break;
+                if (!W.wait(bar(kBarAFull), tcount & 1)) break;
+                tc_fence_after();
+                const uint32_t d = tmem_base + buf * (uint32_t)L.n_tile;
+                const uint32_t a0 = smem_u32(sA), b0 = smem_u32(sB);
+                for (int kk = 0; kk < L.in_dim / 16; ++kk) {
+                    const uint32_t kb = kk >> 2, ko = (kk & 3) * 32;
+                    const uint64_t ad = sw128_desc(a0 + kb * (kTileM * 128) + ko);
+                    const uint64_t bd = sw128_desc(b0 + kb * (L.n_tile * 128) + ko);
+                    umma_bf16(d, ad, bd, L.idesc, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(bar(kBarAEmpty));
+                umma_commit(bar(kBarDFull + buf));
+                const bool last_of_group = (u + 1 == u_end) || ((u + 1) / L.m_tiles != x.g);
+                if (last_of_group) umma_commit(bar(kBarBEmpty));
+                ++tcount;
+            }
+        }
+        __syncwarp();
+    } else if (warp < kEpiWarp0 + kNumEpiWarps) {
+        // ------------------------------------------------------------ epilogue
+        const int quad = warp & 3;
+        const int m = quad * 32 + lane;
+        uint8_t* srow = sStage + (size_t)m * L.stage_row_bytes;
+        const uint32_t srow_u32 = smem_u32(srow);
+        uint32_t tcount = 0;
+        for (long long u = u_begin; u < u_end; ++u) {
+            const Unit x = decode(u, L, P.Ht);
+            const uint32_t buf = tcount & 1;
+            if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
+            tc_fence_after();
+            const int tp = x.tile * kTileM + m;
+            const bool valid = tp < P.T_total;
+            long long dst_off = -1;
+            int pt = 0;
+            if (valid) {
+                const TokenInfo ti = resolve_token(P, tp);
+                dst_off = ti.dst_off;
+                pt = ti.pt;
+            }
+            const bool rot = x.kv == 0 && P.rt.enabled;
+            bulk_wait_read0();
+            const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)L.n_tile;
+            for (int pc = 0; pc < hw; pc += 16) {
+                uint32_t r0[16], r1[16];
+                tmem_ld16(taddr + pc, r0);
+                tmem_ld16(taddr + hw + pc, r1);
+                tmem_ld_wait();
+                float y0[16], y1[16];
+#pragma unroll
+                for (int e = 0; e < 16; ++e) { y0[e] = __uint_as_float(r0[e]); y1[e] = __uint_as_float(r1[e]); }
+                if (rot) {
+#pragma unroll
+                    for (int hb = 0; hb < 16; hb += 8) {
+                        float c[8], s[8];
+                        rope_cs_vec<8>(P.rt, pt, x.nt * hw + pc + hb, c, s);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) {
+                            const float a = y0[hb + e], bb = y1[hb + e];
+                            y0[hb + e] = fmaf(a, c[e], -bb * s[e]);
+                            y1[hb + e] = fmaf(bb, c[e], a * s[e]);
+                        }
+                    }
+                }
+                uint4* p0 = reinterpret_cast<uint4*>(srow + pc * 2);
+                uint4* p1 = reinterpret_cast<uint4*>(srow + (hw + pc) * 2);
+                p0[0] = make_uint4(pack_bf16(y0[0], y0[1]), pack_bf16(y0[2], y0[3]), pack_bf16(y0[4], y0[5]),
+                                   pack_bf16(y0[6], y0[7]));
+                p0[1] = make_uint4(pack_bf16(y0[8], y0[9]), pack_bf16(y0[10], y0[11]), pack_bf16(y0[12], y0[13]),
+                                   pack_bf16(y0[14], y0[15]));
+                p1[0] = make_uint4(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]), pack_bf16(y1[4], y1[5]),
+                                   pack_bf16(y1[6], y1[7]));
+                p1[1] = make_uint4(pack_bf16(y1[8], y1[9]), pack_bf16(y1[10], y1[11]), pack_bf16(y1[12], y1[13]),
+                                   pack_bf16(y1[14], y1[15]));
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarDEmpty + buf));
+            if (valid && dst_off >= 0) {
+                fence_proxy_async();
+                __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
+                                     dst_head_off(P, x.h);
+                if (L.n_split == 1) {
+                    bulk_s2g(dst, srow_u32, (uint32_t)P.dt * 2);
+                } else {
+                    bulk_s2g(dst + x.nt * hw, srow_u32, (uint32_t)hw * 2);
+                    bulk_s2g(dst + half_t + x.nt * hw, srow_u32 + hw * 2, (uint32_t)hw * 2);
+                }
+                bulk_commit();
+            }
+            ++tcount;
+        }
+        bulk_wait0();
+    } else {
+        // ------------------------------------------------------------ prologue (A tile)
+        const int tw = warp - kXfWarp0;
+        const int lanes_per_head = 32 * P.ds / L.in_dim;
+        const int q = lane / lanes_per_head;              // head within the A row
+        const int i0 = (lane % lanes_per_head) * PP;      // first rotary pair of this lane
+        const int hs = P.ds >> 1;
+        const int k0 = q * P.ds + i0, k1 = k0 + hs;       // A columns of the two halves
+        uint32_t sub = 0, tcount = 0;
+        bool ok = true;
+        for (long long u = u_begin; u < u_end && ok; ++u) {
+            const Unit x = decode(u, L, P.Ht);
+            const bool rot = x.kv == 0 && P.rs.enabled;
+            const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
+            const int g = (P.r > 1 ? x.h * P.r : x.h / P.e) + q;
+            if (!W.wait(bar(kBarAEmpty), (tcount & 1) ^ 1)) break;
+            for (int sq = 0; sq < kSubPerTile; ++sq) {
+                const uint32_t slot = sub % kNumSlots;
+                if (!W.wait(bar(kBarSlotFull + slot), (sub / kNumSlots) & 1)) { ok = false; break; }
+                const SlotHdr hdr = sHdr[slot];
+                const uint8_t* ring = sRing + hdr.offset;
+                for (int tt = tw; tt < kSub; tt += kNumXfWarps) {
+                    const SubMeta mt = sMeta[slot * kSub + tt];
+                    const int row = sq * kSub + tt;
+                    if (x.tile * kTileM + row >= P.T_total) continue;
+                    float a0[PP], a1[PP];
+#pragma unroll
+                    for (int e = 0; e < PP; ++e) { a0[e] = 0.f; a1[e] = 0.f; }
+                    const long long gbase = (long long)mt.b * P.sb + (long long)g * P.sh;
+                    for (int s = mt.lo; s < mt.hi; ++s) {
+                        float x0[PP], x1[PP];
+                        const __nv_bfloat16* rp;
+                        if (mt.stage_row >= 0)
+                            rp = reinterpret_cast<const __nv_bfloat16*>(
+                                ring + ((size_t)q * hdr.rows + (size_t)(mt.stage_row + s - mt.lo)) * L.row_bytes);
+                        else
+                            rp = src + gbase + (long long)s * P.ss;
+                        load_bf16<PP>(rp + i0, x0);
+                        load_bf16<PP>(rp + hs + i0, x1);
+                        if (rot) {
+                            float c[PP], sn[PP];
+                            rope_cs_vec<PP>(P.rs, src_pos_of(P, mt.b, s), i0, c, sn);
+#pragma unroll
+                            for (int e = 0; e < PP; ++e) {
+                                // undo the rotation: R(-theta)
+                                const float u0 = fmaf(x0[e], c[e], x1[e] * sn[e]);
+                                const float u1 = fmaf(x1[e], c[e], -x0[e] * sn[e]);
+                                x0[e] = u0;
+                                x1[e] = u1;
+                            }
+                        }
+#pragma unroll
+                        for (int e = 0; e < PP; ++e) { a0[e] += x0[e]; a1[e] += x1[e]; }
+                    }
+                    const int n = mt.hi - mt.lo;
+#pragma unroll
+                    for (int e = 0; e < PP; ++e) {
+                        a0[e] = n > 0 ? a0[e] / (float)n : 0.f;
+                        a1[e] = n > 0 ? a1[e] / (float)n : 0.f;
+                    }
+                    store_bf16_smem<PP>(sA + sw128_off(row, k0, kTileM), a0);
+                    store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1);
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(kBarSlotEmpty + slot));
+                ++sub;
+            }
+            if (!ok) break;
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarAFull));
+            ++tcount;
+        }
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, L.tmem_cols);
+    }
+}
+
+// Weight images: for group g = ((j*Ht + h)*2 + kv)*n_split + nt, the B operand
+// [n_tile rows = output columns][in] in K-major SW128 layout.  Output column of
+// image row n: n < n_tile/2 -> nt*hw + n, else d_t/2 + nt*hw + (n - hw), so an
+// image holds whole RoPE pairs.
+__global__ void tc_weight_relayout_kernel(const __nv_bfloat16* __restrict__ wk, const __nv_bfloat16* __restrict__ wv,
+                                          uint8_t* __restrict__ img, int Lt, int Ht, int in_dim, int dt, int n_tile)
+{
+    const int n_split = dt / n_tile, hw = n_tile / 2;
+    const long long chunks_per_img = (long long)n_tile * in_dim / 8;
+    const long long total = (long long)Lt * Ht * 2 * n_split * chunks_per_img;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int gimg = (int)(idx / chunks_per_img);
+    const int c = (int)(idx - (long long)gimg * chunks_per_img);   // chunk within image
+    int rest = gimg;
+    const int nt = rest % n_split; rest /= n_split;
+    const int kv = rest & 1; rest >>= 1;
+    const int h = rest % Ht;
+    const int j = rest / Ht;
+    // chunk c enumerates (n, k/8) with k fastest
+    const int n = c / (in_dim / 8);
+    const int k8 = c - n * (in_dim / 8);
+    const int col = n < hw ? nt * hw + n : dt / 2 + nt * hw + (n - hw);
+    const __nv_bfloat16* w = (kv ? wv : wk) + ((size_t)j * Ht + h) * (size_t)in_dim * dt;
+    uint32_t v[4];
+    for (int e = 0; e < 4; ++e) {
+        const int k = k8 * 8 + 2 * e;
+        const __nv_bfloat16 lo = w[(size_t)k * dt + col];
+        const __nv_bfloat16 hi = w[(size_t)(k + 1) * dt + col];
+        v[e] = (uint32_t)__bfloat16_as_ushort(lo) | ((uint32_t)__bfloat16_as_ushort(hi) << 16);
+    }
+    const int k = k8 * 8;
+    const size_t off = (size_t)gimg * ((size_t)n_tile * in_dim * 2) + (size_t)(k >> 6) * n_tile * 128 +
+                       (size_t)(n >> 3) * 1024 + (n & 7) * 128 + ((((k >> 3) & 7) ^ (n & 7)) << 4);
+    *reinterpret_cast<uint4*>(img + off) = make_uint4(v[0], v[1], v[2], v[3]);
+}
+
+uint32_t make_idesc(int M, int N)
+{
+    return (1u << 4)                  // D format: f32
+           | (1u << 7)                // A format: bf16
+           | (1u << 10)               // B format: bf16
+           | ((uint32_t)(N >> 3) << 17)
+           | ((uint32_t)(M >> 4) << 24);   // A and B K-major, no negate, dense
+}
+
+bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
+{
+    if (in_dim % 64 || in_dim > 256 || in_dim < 64) return false;
+    if (dt != 64 && dt != 128 && dt != 256) return false;
+    if (ds != 64 && ds != 128 && ds != 256) return false;
+    if (in_dim % ds) return false;
+    L.in_dim = in_dim;
+    L.n_tile = (in_dim * dt * 2 <= 65536) ? dt : dt / 2;
+    L.n_split = dt / L.n_tile;
+    L.b_bytes = (unsigned)(in_dim * L.n_tile * 2);
+    L.a_bytes = (unsigned)(kTileM * in_dim * 2);
+    L.row_bytes = (unsigned)(ds * 2);
+    L.stage_row_bytes = (unsigned)(L.n_tile * 2 + 16);
+    unsigned off = 0;
+    auto take = [&](unsigned bytes, unsigned align) {
+        off = (off + align - 1) / align * align;
+        const unsigned o = off;
+        off += bytes;
+        return o;
+    };
+    L.off_b = take(L.b_bytes, 1024);
+    L.off_a = take(L.a_bytes, 1024);
+    L.off_stage = take(kTileM * L.stage_row_bytes, 128);
+    L.off_meta = take(kNumSlots * kSub * sizeof(SubMeta), 16);
+    L.off_hdr = take(kNumSlots * sizeof(SlotHdr), 16);
+    L.off_bar = take(kNumBars * 8, 8);
+    L.off_misc = take(16, 16);
+    L.off_ring = (off + 127) / 128 * 128;
+    const int avail = kSmemMax - 1024 - (int)L.off_ring;   // 1024: alignment slack of the dynamic base
+    L.ring_bytes = avail > 0 ? (unsigned)(avail / 1024 * 1024) : 0;
+    if (L.ring_bytes < 3u * kSub * (unsigned)(in_dim / ds) * L.row_bytes) return false;   // one worst sub-tile
+    L.idesc = make_idesc(kTileM, L.n_tile);
+    unsigned cols = 32;
+    while (cols < 2u * (unsigned)L.n_tile) cols <<= 1;
+    L.tmem_cols = cols;
+    return cols <= 512;
+}
+
+}  // namespace
+
+TcConfig tc_config(int in_dim, int dt, int ds)
+{
+    TcLaunch L{};
+    TcConfig c{0, 0, 0, kThreads, 0};
+    if (!tc_layout(in_dim, dt, ds, L)) return c;
+    c.n_tile = L.n_tile;
+    c.n_split = L.n_split;
+    c.smem_bytes = kSmemMax;
+    c.ok = 1;
+    return c;
+}
+
+size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht)
+{
+    return (size_t)Lt * Ht * 2 * (size_t)in_dim * dt * 2;
+}
+
+cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
+                                      int dt, int n_tile, cudaStream_t stream)
+{
+    const long long total = (long long)Lt * Ht * 2 * dt * in_dim / 8;
+    const int threads = 256;
+    tc_weight_relayout_kernel<<<(unsigned)((total + threads - 1) / threads), threads, 0, stream>>>(
+        (const __nv_bfloat16*)w_k, (const __nv_bfloat16*)w_v, (uint8_t*)image, Lt, Ht, in_dim, dt, n_tile);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, cudaStream_t stream)
+{
+    TcLaunch L{};
+    if (!tc_layout(P.in_dim, P.dt, P.ds, L)) return cudaErrorNotSupported;
+    L.groups = P.Lt * P.Ht * 2 * L.n_split;
+    L.m_tiles = (P.T_total + kTileM - 1) / kTileM;
+    const long long U = (long long)L.groups * L.m_tiles;
+    const int grid = (int)(U < num_sms ? U : num_sms);
+    const int pp = L.in_dim / 64;
+    cudaError_t err;
+    switch (pp) {
+    case 4:
+        err = cudaFuncSetAttribute(translate_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+        if (err != cudaSuccess) return err;
+        translate_tc_kernel<4><<<grid, kThreads, kSmemMax, stream>>>(P, L);
+        break;
+    case 2:
+        err = cudaFuncSetAttribute(translate_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+        if (err != cudaSuccess) return err;
+        translate_tc_kernel<2><<<grid, kThreads, kSmemMax, stream>>>(P, L);
+        break;
+    case 1:
+        err = cudaFuncSetAttribute(translate_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+        if (err != cudaSuccess) return err;
+        translate_tc_kernel<1><<<grid, kThreads, kSmemMax, stream>>>(P, L);
+        break;
+    default:
+        return cudaErrorNotSupported;
+    }
+    (void)cfg;
+    return cudaGetLastError();
+}
+
 }  // namespace kvx
