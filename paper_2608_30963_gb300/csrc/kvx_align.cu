@@ -54,28 +54,24 @@ cudaError_t launch_build_alignment(int batch, int total_tgt, const int* src_seq_
     return cudaGetLastError();
 }
 
-// Rotation tables: hi[a][i] = e^{j (64 a) f_i}, lo[c][i] = e^{j c f_i}, f_i = base^(-2i/d),
-// angles and sin/cos in double, stored as fp32 (cos, sin).
-__global__ void rope_table_kernel(float2* hi, float2* lo, int n_hi, int d, double base)
+// Rotation table: cs[p][i] = (cos, sin)(p * f_i), f_i = base^(-2i/d); angle and
+// trigonometry in double, stored as fp32.
+__global__ void rope_table_kernel(float2* cs, int max_pos, int d, double base)
 {
     const int half = d >> 1;
-    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
-    const int rows = n_hi + kRopeLo;
-    if (idx >= rows * half) return;
-    const int row = idx / half, i = idx - row * half;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)max_pos * half) return;
+    const int p = (int)(idx / half), i = (int)(idx - (long long)p * half);
     const double f = pow(base, -2.0 * (double)i / (double)d);
-    const double p = row < n_hi ? (double)row * kRopeLo : (double)(row - n_hi);
     double s, c;
-    sincos(p * f, &s, &c);
-    const float2 v = make_float2((float)c, (float)s);
-    if (row < n_hi) hi[(size_t)row * half + i] = v;
-    else lo[(size_t)(row - n_hi) * half + i] = v;
+    sincos((double)p * f, &s, &c);
+    cs[idx] = make_float2((float)c, (float)s);
 }
 
-cudaError_t launch_rope_table(float2* hi, float2* lo, int n_hi, int d, double base, cudaStream_t stream)
+cudaError_t launch_rope_table(float2* cs, int max_pos, int d, double base, cudaStream_t stream)
 {
-    const int n = (n_hi + kRopeLo) * (d / 2);
-    rope_table_kernel<<<(n + 255) / 256, 256, 0, stream>>>(hi, lo, n_hi, d, base);
+    const long long n = (long long)max_pos * (d / 2);
+    rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(cs, max_pos, d, base);
     return cudaGetLastError();
 }
 

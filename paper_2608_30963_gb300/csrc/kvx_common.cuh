@@ -9,16 +9,11 @@
 
 namespace kvx {
 
-// Rotation tables.  cos/sin of the exact angle p * f_i, f_i = base^(-2i/d), for
-// p = 64*a + c are rebuilt from two tables of fp32 (cos, sin) pairs computed in
-// double precision:  hi[a][i] = e^{j 64 a f_i},  lo[c][i] = e^{j c f_i},
-// e^{j p f_i} = hi[a][i] * lo[c][i] (complex product, fp32).  Error ~3 fp32 ulp.
-constexpr int kRopeLoBits = 6;
-constexpr int kRopeLo = 1 << kRopeLoBits;
-
+// Rotation table: cos/sin of the exact angle p * f_i, f_i = base^(-2i/d), for
+// every position p < max_position and frequency i < d/2, computed in double
+// precision and stored as fp32 (cos, sin) pairs, row p contiguous.
 struct RopeTable {
-    const float2* hi;   // [max_position / 64 + 1][d/2]
-    const float2* lo;   // [64][d/2]
+    const float2* cs;   // [max_position][d/2]
     int half;           // d/2
     int enabled;        // 0: no rotation
 };
@@ -66,12 +61,10 @@ __device__ __forceinline__ void set_status(unsigned* status, unsigned bit)
     if (status) atomicOr(status, bit);
 }
 
-// (cos, sin) of angle p * f_i, with p clamped to [0, max_position).
+// (cos, sin) of angle p * f_i (p already clamped to [0, max_position)).
 __device__ __forceinline__ float2 rope_cs(const RopeTable& t, int p, int i)
 {
-    float2 a = __ldg(&t.hi[(size_t)(p >> kRopeLoBits) * t.half + i]);
-    float2 b = __ldg(&t.lo[(size_t)(p & (kRopeLo - 1)) * t.half + i]);
-    return make_float2(a.x * b.x - a.y * b.y, a.y * b.x + a.x * b.y);
+    return __ldg(&t.cs[(size_t)p * t.half + i]);
 }
 
 __device__ __forceinline__ int clamp_pos(int p, int max_position, unsigned* status)

@@ -97,9 +97,9 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         return fail(KVX_ERR_INVALID_ARG, "create: unknown dtype %d", desc->dtype);
     if (desc->path < KVX_PATH_AUTO || desc->path > KVX_PATH_TCGEN05)
         return fail(KVX_ERR_INVALID_ARG, "create: unknown path %d", desc->path);
-    int max_pos = desc->max_position ? desc->max_position : (1 << 17);
-    if (max_pos < 1 || max_pos > (1 << 22))
-        return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<22]");
+    int max_pos = desc->max_position ? desc->max_position : (1 << 16);
+    if (max_pos < 1 || max_pos > (1 << 20))
+        return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<20]");
 
     kvx_translator* t = new kvx_translator();
     t->desc = *desc;
@@ -183,23 +183,24 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         raw = nullptr;
     }
 
-    {   // RoPE tables
-        const int n_hi = (max_pos + kRopeLo - 1) / kRopeLo + 1;
-        const size_t src_n = (size_t)(n_hi + kRopeLo) * (s.head_dim / 2);
-        const size_t dst_n = (size_t)(n_hi + kRopeLo) * (d.head_dim / 2);
+    {   // RoPE tables (one shared table when both models rotate alike)
+        const size_t src_n = s.rope_base > 0.0 ? (size_t)max_pos * (s.head_dim / 2) : 0;
+        const bool same = s.rope_base > 0.0 && s.rope_base == d.rope_base && s.head_dim == d.head_dim;
+        const size_t dst_n = d.rope_base > 0.0 && !same ? (size_t)max_pos * (d.head_dim / 2) : 0;
         t->rope_bytes = (src_n + dst_n) * sizeof(float2);
-        if (cudaMalloc(&t->rope, t->rope_bytes) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: table allocation"); goto err; }
-        float2* sh = t->rope;
-        float2* sl = sh + (size_t)n_hi * (s.head_dim / 2);
-        float2* dh = t->rope + src_n;
-        float2* dl = dh + (size_t)n_hi * (d.head_dim / 2);
-        t->rs = RopeTable{sh, sl, s.head_dim / 2, s.rope_base > 0.0};
-        t->rt = RopeTable{dh, dl, d.head_dim / 2, d.rope_base > 0.0};
-        if (t->rs.enabled && (ce = launch_rope_table(sh, sl, n_hi, s.head_dim, s.rope_base, 0)) != cudaSuccess) {
+        if (t->rope_bytes && cudaMalloc(&t->rope, t->rope_bytes) != cudaSuccess) {
+            st = fail(KVX_ERR_OOM, "create: table allocation");
+            goto err;
+        }
+        float2* stab = src_n ? t->rope : nullptr;
+        float2* dtab = same ? stab : (dst_n ? t->rope + src_n : nullptr);
+        t->rs = RopeTable{stab, s.head_dim / 2, s.rope_base > 0.0};
+        t->rt = RopeTable{dtab, d.head_dim / 2, d.rope_base > 0.0};
+        if (src_n && (ce = launch_rope_table(stab, max_pos, s.head_dim, s.rope_base, 0)) != cudaSuccess) {
             st = fail(KVX_ERR_CUDA, "create: rope table: %s", cudaGetErrorString(ce));
             goto err;
         }
-        if (t->rt.enabled && (ce = launch_rope_table(dh, dl, n_hi, d.head_dim, d.rope_base, 0)) != cudaSuccess) {
+        if (dst_n && (ce = launch_rope_table(dtab, max_pos, d.head_dim, d.rope_base, 0)) != cudaSuccess) {
             st = fail(KVX_ERR_CUDA, "create: rope table: %s", cudaGetErrorString(ce));
             goto err;
         }

@@ -43,6 +43,7 @@ constexpr int kNumXfWarps = 8;
 constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
 constexpr int kSmemMax = 232448;          // 227 KB opt-in per block
 constexpr unsigned long long kWaitNs = 1000000000ull;
+constexpr int kMaxSeqCache = 512;         // sequences whose metadata is kept in shared memory
 
 // barrier indices
 constexpr int kBarBFull = 0, kBarBEmpty = 1, kBarAFull = 2, kBarAEmpty = 3;
@@ -66,7 +67,8 @@ struct SlotHdr {
 struct TcLaunch {
     int n_tile, n_split, in_dim, groups, m_tiles;
     unsigned b_bytes, a_bytes, row_bytes, stage_row_bytes, ring_bytes;
-    unsigned off_b, off_a, off_stage, off_ring, off_meta, off_hdr, off_bar, off_misc;
+    unsigned off_b, off_a, off_stage, off_ring, off_meta, off_hdr, off_bar, off_misc, off_seq;
+    int seq_cached;   // per-sequence offsets and source lengths copied to shared memory
     unsigned idesc;
     unsigned tmem_cols;
 };
@@ -168,14 +170,11 @@ __device__ __forceinline__ void umma_commit(uint32_t bar)
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                  : "memory");
 }
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16])
+__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&r)[8])
 {
-    asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
-        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
+                 : "r"(taddr));
 }
 __device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
 
@@ -237,12 +236,30 @@ __device__ __forceinline__ Unit decode(long long u, const TcLaunch& L, int Ht)
     return x;
 }
 
+// Sequence metadata view: shared-memory copies of seq_off / src_seq_len when the
+// batch is small enough, else the global arrays.
+struct SeqView {
+    const int* off;    // [batch+1]
+    const int* slen;   // [batch]
+    int batch;
+    __device__ __forceinline__ int find(int tp) const
+    {
+        int lo = 0, hi = batch - 1;
+        while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (off[mid] <= tp) lo = mid; else hi = mid - 1;
+        }
+        return lo;
+    }
+};
+
 // Source-side resolution of one target token (sequence, clamped span).
-__device__ __forceinline__ void resolve_src(const TranslateParams& P, int tp, int& b, int& lo, int& hi)
+__device__ __forceinline__ void resolve_src(const TranslateParams& P, const SeqView& sv, int tp, int& b, int& lo,
+                                            int& hi)
 {
-    b = find_seq(P.seq_off, P.batch, tp);
-    const int t = tp - __ldg(&P.seq_off[b]);
-    int S = __ldg(&P.src_seq_len[b]);
+    b = sv.find(tp);
+    const int t = tp - sv.off[b];
+    int S = sv.slen[b];
     if (S > P.src_max_seq || S < 0) {
         set_status(P.status, KVX_DEV_SEQ_CLAMPED);
         S = S < 0 ? 0 : P.src_max_seq;
@@ -258,6 +275,25 @@ __device__ __forceinline__ void resolve_src(const TranslateParams& P, int tp, in
     }
 }
 
+// Target-side resolution: output row offset (-1: not written) and RoPE position.
+__device__ __forceinline__ void resolve_dst(const TranslateParams& P, const SeqView& sv, int tp, long long& dst_off,
+                                            int& pt)
+{
+    const int b = sv.find(tp);
+    const int t = tp - sv.off[b];
+    const int p = P.tgt_pos ? __ldg(&P.tgt_pos[tp]) : t;
+    pt = P.rt.enabled ? clamp_pos(p, P.max_position, P.status) : 0;
+    if (!P.paged) {
+        if (t >= P.dst_max_seq) { set_status(P.status, KVX_DEV_SEQ_CLAMPED); dst_off = -1; }
+        else dst_off = (long long)b * P.db + (long long)t * P.dts;
+    } else {
+        const int pi = t / P.page_size;
+        const int page = pi < P.max_pages ? __ldg(&P.page_table[(size_t)b * P.max_pages + pi]) : -1;
+        if (page < 0 || page >= P.num_pages) { set_status(P.status, KVX_DEV_PAGE_INVALID); dst_off = -1; }
+        else dst_off = ((long long)page * P.page_size + (t % P.page_size)) * (long long)P.Ht * P.dt;
+    }
+}
+
 __device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
 __device__ __forceinline__ uint32_t pack_bf16(float a, float b)
@@ -266,21 +302,24 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b)
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
-// Load PP consecutive bf16 values (PP in {1,2,4}) into floats.
+// PP consecutive bf16 values (PP in {1,2,4}) as one raw load.
+template <int PP> struct Raw;
+template <> struct Raw<4> { using T = uint2; };
+template <> struct Raw<2> { using T = uint32_t; };
+template <> struct Raw<1> { using T = unsigned short; };
+
 template <int PP>
-__device__ __forceinline__ void load_bf16(const __nv_bfloat16* p, float (&x)[PP])
+__device__ __forceinline__ typename Raw<PP>::T load_raw(const __nv_bfloat16* p)
 {
-    if constexpr (PP == 4) {
-        const uint2 w = *reinterpret_cast<const uint2*>(p);
-        x[0] = bf_lo(w.x); x[1] = bf_hi(w.x); x[2] = bf_lo(w.y); x[3] = bf_hi(w.y);
-    } else if constexpr (PP == 2) {
-        const uint32_t w = *reinterpret_cast<const uint32_t*>(p);
-        x[0] = bf_lo(w); x[1] = bf_hi(w);
-    } else {
-        const unsigned short w = *reinterpret_cast<const unsigned short*>(p);
-        x[0] = __uint_as_float((uint32_t)w << 16);
-    }
+    return *reinterpret_cast<const typename Raw<PP>::T*>(p);
 }
+__device__ __forceinline__ void unpack(uint2 w, float (&x)[4])
+{
+    x[0] = bf_lo(w.x); x[1] = bf_hi(w.x); x[2] = bf_lo(w.y); x[3] = bf_hi(w.y);
+}
+__device__ __forceinline__ void unpack(uint32_t w, float (&x)[2]) { x[0] = bf_lo(w); x[1] = bf_hi(w); }
+__device__ __forceinline__ void unpack(unsigned short w, float (&x)[1]) { x[0] = __uint_as_float((uint32_t)w << 16); }
+
 template <int PP>
 __device__ __forceinline__ void store_bf16_smem(uint8_t* p, const float (&x)[PP])
 {
@@ -294,29 +333,20 @@ __device__ __forceinline__ void store_bf16_smem(uint8_t* p, const float (&x)[PP]
     }
 }
 
-// (cos, sin) for PP consecutive frequencies i0.. at position p.
+// (cos, sin) for PP consecutive frequencies i0.. at position p (PP even: 16-byte loads).
 template <int PP>
-__device__ __forceinline__ void rope_cs_vec(const RopeTable& t, int p, int i0, float (&c)[PP], float (&s)[PP])
+__device__ __forceinline__ void rope_cs_vec(const RopeTable& t, int p, int i0, float2 (&cs)[PP])
 {
-    const float2* hp = t.hi + (size_t)(p >> kRopeLoBits) * t.half + i0;
-    const float2* lp = t.lo + (size_t)(p & (kRopeLo - 1)) * t.half + i0;
-    float2 a[PP], b[PP];
+    const float2* hp = t.cs + (size_t)p * t.half + i0;
     if constexpr (PP >= 2) {
 #pragma unroll
         for (int q = 0; q < PP; q += 2) {
-            const float4 va = __ldg(reinterpret_cast<const float4*>(hp + q));
-            const float4 vb = __ldg(reinterpret_cast<const float4*>(lp + q));
-            a[q] = make_float2(va.x, va.y); a[q + 1] = make_float2(va.z, va.w);
-            b[q] = make_float2(vb.x, vb.y); b[q + 1] = make_float2(vb.z, vb.w);
+            const float4 v = __ldg(reinterpret_cast<const float4*>(hp + q));
+            cs[q] = make_float2(v.x, v.y);
+            cs[q + 1] = make_float2(v.z, v.w);
         }
     } else {
-        a[0] = __ldg(hp);
-        b[0] = __ldg(lp);
-    }
-#pragma unroll
-    for (int q = 0; q < PP; ++q) {
-        c[q] = a[q].x * b[q].x - a[q].y * b[q].y;
-        s[q] = a[q].y * b[q].x + a[q].x * b[q].y;
+        cs[0] = __ldg(hp);
     }
 }
 
@@ -361,12 +391,19 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         tmem_alloc(smem_u32(sTmemBase), L.tmem_cols);
         tmem_relinquish();
     }
+    int* sSeqOff = reinterpret_cast<int*>(smem + L.off_seq);
+    int* sSrcLen = sSeqOff + kMaxSeqCache + 1;
+    if (L.seq_cached) {
+        for (int i = threadIdx.x; i <= P.batch; i += blockDim.x) sSeqOff[i] = __ldg(&P.seq_off[i]);
+        for (int i = threadIdx.x; i < P.batch; i += blockDim.x) sSrcLen[i] = __ldg(&P.src_seq_len[i]);
+    }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *sTmemBase;
 
     const Waiter W{sAbort, P.status};
+    const SeqView sv{L.seq_cached ? sSeqOff : P.seq_off, L.seq_cached ? sSrcLen : P.src_seq_len, P.batch};
     const long long U = (long long)L.groups * L.m_tiles;
     const long long u_begin = (long long)blockIdx.x * U / gridDim.x;
     const long long u_end = (long long)(blockIdx.x + 1) * U / gridDim.x;
@@ -407,11 +444,22 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             }
             const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
             const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
+            // spans of the tile's 128 tokens, 4 per lane, loads issued together
+            int rb[kSubPerTile], rlo[kSubPerTile], rhi[kSubPerTile];
+#pragma unroll
+            for (int sq = 0; sq < kSubPerTile; ++sq) {
+                const int tp = x.tile * kTileM + sq * kSub + lane;
+                rb[sq] = -1; rlo[sq] = 0; rhi[sq] = 0;
+                if (tp < P.T_total) resolve_src(P, sv, tp, rb[sq], rlo[sq], rhi[sq]);
+            }
+#pragma unroll 1
             for (int sq = 0; sq < kSubPerTile; ++sq) {
                 const int tp = x.tile * kTileM + sq * kSub + lane;
                 const bool valid = tp < P.T_total;
-                int b = -1, lo = 0, hi = 0;
-                if (valid) resolve_src(P, tp, b, lo, hi);
+                int b = rb[0], lo = rlo[0], hi = rhi[0];
+#pragma unroll
+                for (int z = 1; z < kSubPerTile; ++z)
+                    if (sq == z) { b = rb[z]; lo = rlo[z]; hi = rhi[z]; }
                 const int b_prev = __shfl_up_sync(0xffffffffu, b, 1);
                 const int lo_prev = __shfl_up_sync(0xffffffffu, lo, 1);
                 const int hi_prev = __shfl_up_sync(0xffffffffu, hi, 1);
@@ -546,51 +594,45 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         for (long long u = u_begin; u < u_end; ++u) {
             const Unit x = decode(u, L, P.Ht);
             const uint32_t buf = tcount & 1;
-            if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
-            tc_fence_after();
+            // resolve the output row while the tile is still being computed
             const int tp = x.tile * kTileM + m;
             const bool valid = tp < P.T_total;
             long long dst_off = -1;
             int pt = 0;
-            if (valid) {
-                const TokenInfo ti = resolve_token(P, tp);
-                dst_off = ti.dst_off;
-                pt = ti.pt;
-            }
+            if (valid) resolve_dst(P, sv, tp, dst_off, pt);
             const bool rot = x.kv == 0 && P.rt.enabled;
+            float2 cs[8];
+            if (rot) rope_cs_vec<8>(P.rt, pt, x.nt * hw, cs);
+            if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
+            tc_fence_after();
             bulk_wait_read0();
             const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)L.n_tile;
-            for (int pc = 0; pc < hw; pc += 16) {
-                uint32_t r0[16], r1[16];
-                tmem_ld16(taddr + pc, r0);
-                tmem_ld16(taddr + hw + pc, r1);
+            for (int pc = 0; pc < hw; pc += 8) {
+                float2 csn[8];
+                if (rot && pc + 8 < hw) rope_cs_vec<8>(P.rt, pt, x.nt * hw + pc + 8, csn);
+                uint32_t r0[8], r1[8];
+                tmem_ld8(taddr + pc, r0);
+                tmem_ld8(taddr + hw + pc, r1);
                 tmem_ld_wait();
-                float y0[16], y1[16];
+                float y0[8], y1[8];
 #pragma unroll
-                for (int e = 0; e < 16; ++e) { y0[e] = __uint_as_float(r0[e]); y1[e] = __uint_as_float(r1[e]); }
+                for (int e = 0; e < 8; ++e) { y0[e] = __uint_as_float(r0[e]); y1[e] = __uint_as_float(r1[e]); }
                 if (rot) {
 #pragma unroll
-                    for (int hb = 0; hb < 16; hb += 8) {
-                        float c[8], s[8];
-                        rope_cs_vec<8>(P.rt, pt, x.nt * hw + pc + hb, c, s);
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) {
-                            const float a = y0[hb + e], bb = y1[hb + e];
-                            y0[hb + e] = fmaf(a, c[e], -bb * s[e]);
-                            y1[hb + e] = fmaf(bb, c[e], a * s[e]);
-                        }
+                    for (int e = 0; e < 8; ++e) {
+                        const float a = y0[e], bb = y1[e];
+                        y0[e] = fmaf(a, cs[e].x, -bb * cs[e].y);
+                        y1[e] = fmaf(bb, cs[e].x, a * cs[e].y);
                     }
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) cs[e] = csn[e];
                 }
-                uint4* p0 = reinterpret_cast<uint4*>(srow + pc * 2);
-                uint4* p1 = reinterpret_cast<uint4*>(srow + (hw + pc) * 2);
-                p0[0] = make_uint4(pack_bf16(y0[0], y0[1]), pack_bf16(y0[2], y0[3]), pack_bf16(y0[4], y0[5]),
-                                   pack_bf16(y0[6], y0[7]));
-                p0[1] = make_uint4(pack_bf16(y0[8], y0[9]), pack_bf16(y0[10], y0[11]), pack_bf16(y0[12], y0[13]),
-                                   pack_bf16(y0[14], y0[15]));
-                p1[0] = make_uint4(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]), pack_bf16(y1[4], y1[5]),
-                                   pack_bf16(y1[6], y1[7]));
-                p1[1] = make_uint4(pack_bf16(y1[8], y1[9]), pack_bf16(y1[10], y1[11]), pack_bf16(y1[12], y1[13]),
-                                   pack_bf16(y1[14], y1[15]));
+                *reinterpret_cast<uint4*>(srow + pc * 2) =
+                    make_uint4(pack_bf16(y0[0], y0[1]), pack_bf16(y0[2], y0[3]), pack_bf16(y0[4], y0[5]),
+                               pack_bf16(y0[6], y0[7]));
+                *reinterpret_cast<uint4*>(srow + (hw + pc) * 2) =
+                    make_uint4(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]), pack_bf16(y1[4], y1[5]),
+                               pack_bf16(y1[6], y1[7]));
             }
             tc_fence_before();
             __syncwarp();
@@ -631,47 +673,73 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 if (!W.wait(bar(kBarSlotFull + slot), (sub / kNumSlots) & 1)) { ok = false; break; }
                 const SlotHdr hdr = sHdr[slot];
                 const uint8_t* ring = sRing + hdr.offset;
-                for (int tt = tw; tt < kSub; tt += kNumXfWarps) {
-                    const SubMeta mt = sMeta[slot * kSub + tt];
-                    const int row = sq * kSub + tt;
-                    if (x.tile * kTileM + row >= P.T_total) continue;
-                    float a0[PP], a1[PP];
+                constexpr int kTok = kSub / kNumXfWarps;   // tokens of this warp in the sub-tile
+                SubMeta mt[kTok];
+                int n[kTok];
+                int maxn = 0;
 #pragma unroll
-                    for (int e = 0; e < PP; ++e) { a0[e] = 0.f; a1[e] = 0.f; }
-                    const long long gbase = (long long)mt.b * P.sb + (long long)g * P.sh;
-                    for (int s = mt.lo; s < mt.hi; ++s) {
-                        float x0[PP], x1[PP];
-                        const __nv_bfloat16* rp;
-                        if (mt.stage_row >= 0)
-                            rp = reinterpret_cast<const __nv_bfloat16*>(
-                                ring + ((size_t)q * hdr.rows + (size_t)(mt.stage_row + s - mt.lo)) * L.row_bytes);
-                        else
-                            rp = src + gbase + (long long)s * P.ss;
-                        load_bf16<PP>(rp + i0, x0);
-                        load_bf16<PP>(rp + hs + i0, x1);
-                        if (rot) {
-                            float c[PP], sn[PP];
-                            rope_cs_vec<PP>(P.rs, src_pos_of(P, mt.b, s), i0, c, sn);
+                for (int u4 = 0; u4 < kTok; ++u4) {
+                    const int tt = tw + u4 * kNumXfWarps;
+                    mt[u4] = sMeta[slot * kSub + tt];
+                    const bool valid = x.tile * kTileM + sq * kSub + tt < P.T_total;
+                    n[u4] = valid ? max(mt[u4].hi - mt[u4].lo, 0) : -1;
+                    maxn = max(maxn, n[u4]);
+                }
+                float a0[kTok][PP], a1[kTok][PP];
 #pragma unroll
-                            for (int e = 0; e < PP; ++e) {
-                                // undo the rotation: R(-theta)
-                                const float u0 = fmaf(x0[e], c[e], x1[e] * sn[e]);
-                                const float u1 = fmaf(x1[e], c[e], -x0[e] * sn[e]);
-                                x0[e] = u0;
-                                x1[e] = u1;
-                            }
+                for (int u4 = 0; u4 < kTok; ++u4)
+#pragma unroll
+                    for (int e = 0; e < PP; ++e) { a0[u4][e] = 0.f; a1[u4][e] = 0.f; }
+                for (int o = 0; o < maxn; ++o) {
+                    typename Raw<PP>::T w0[kTok], w1[kTok];
+                    float2 cs[kTok][PP];
+#pragma unroll
+                    for (int u4 = 0; u4 < kTok; ++u4) {
+                        if (o < n[u4]) {
+                            const int srow = mt[u4].lo + o;
+                            const __nv_bfloat16* rp;
+                            if (mt[u4].stage_row >= 0)
+                                rp = reinterpret_cast<const __nv_bfloat16*>(
+                                    ring + ((size_t)q * hdr.rows + (size_t)(mt[u4].stage_row + o)) * L.row_bytes);
+                            else
+                                rp = src + (long long)mt[u4].b * P.sb + (long long)g * P.sh + (long long)srow * P.ss;
+                            w0[u4] = load_raw<PP>(rp + i0);
+                            w1[u4] = load_raw<PP>(rp + hs + i0);
+                            if (rot) rope_cs_vec<PP>(P.rs, src_pos_of(P, mt[u4].b, srow), i0, cs[u4]);
                         }
-#pragma unroll
-                        for (int e = 0; e < PP; ++e) { a0[e] += x0[e]; a1[e] += x1[e]; }
                     }
-                    const int n = mt.hi - mt.lo;
+#pragma unroll
+                    for (int u4 = 0; u4 < kTok; ++u4) {
+                        if (o < n[u4]) {
+                            float x0[PP], x1[PP];
+                            unpack(w0[u4], x0);
+                            unpack(w1[u4], x1);
+                            if (rot) {
+#pragma unroll
+                                for (int e = 0; e < PP; ++e) {
+                                    // undo the rotation: R(-theta)
+                                    const float u0 = fmaf(x0[e], cs[u4][e].x, x1[e] * cs[u4][e].y);
+                                    const float u1 = fmaf(x1[e], cs[u4][e].x, -x0[e] * cs[u4][e].y);
+                                    x0[e] = u0;
+                                    x1[e] = u1;
+                                }
+                            }
+#pragma unroll
+                            for (int e = 0; e < PP; ++e) { a0[u4][e] += x0[e]; a1[u4][e] += x1[e]; }
+                        }
+                    }
+                }
+#pragma unroll
+                for (int u4 = 0; u4 < kTok; ++u4) {
+                    if (n[u4] < 0) continue;
+                    const int row = sq * kSub + tw + u4 * kNumXfWarps;
 #pragma unroll
                     for (int e = 0; e < PP; ++e) {
-                        a0[e] = n > 0 ? a0[e] / (float)n : 0.f;
-                        a1[e] = n > 0 ? a1[e] / (float)n : 0.f;
+                        a0[u4][e] = n[u4] > 0 ? a0[u4][e] / (float)n[u4] : 0.f;
+                        a1[u4][e] = n[u4] > 0 ? a1[u4][e] / (float)n[u4] : 0.f;
                     }
-                    store_bf16_smem<PP>(sA + sw128_off(row, k0, kTileM), a0);
-                    store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1);
+                    store_bf16_smem<PP>(sA + sw128_off(row, k0, kTileM), a0[u4]);
+                    store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1[u4]);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(kBarSlotEmpty + slot));
@@ -766,6 +834,7 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
     L.off_hdr = take(kNumSlots * sizeof(SlotHdr), 16);
     L.off_bar = take(kNumBars * 8, 8);
     L.off_misc = take(16, 16);
+    L.off_seq = take((2 * kMaxSeqCache + 1) * sizeof(int), 16);
     L.off_ring = (off + 127) / 128 * 128;
     const int avail = kSmemMax - 1024 - (int)L.off_ring;   // 1024: alignment slack of the dynamic base
     L.ring_bytes = avail > 0 ? (unsigned)(avail / 1024 * 1024) : 0;
@@ -811,6 +880,7 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
     TcLaunch L{};
     if (!tc_layout(P.in_dim, P.dt, P.ds, L)) return cudaErrorNotSupported;
     L.groups = P.Lt * P.Ht * 2 * L.n_split;
+    L.seq_cached = P.batch <= kMaxSeqCache;
     L.m_tiles = (P.T_total + kTileM - 1) / kTileM;
     const long long U = (long long)L.groups * L.m_tiles;
     const int grid = (int)(U < num_sms ? U : num_sms);

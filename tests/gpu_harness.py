@@ -32,7 +32,7 @@ def i32(x, device="cuda") -> Optional[torch.Tensor]:
 
 class GpuRun:
     def __init__(self, c: Case, path: int = kvx.KVX_PATH_AUTO, paged: Optional[bool] = None,
-                 explicit_layer_map: bool = True, fill=float("nan")):
+                 explicit_layer_map: bool = True, fill=float("nan"), max_position: int = 0):
         self.c = c
         s = c.spec
         self.dtype = s.dtype
@@ -40,7 +40,7 @@ class GpuRun:
         kdt = kvx.KVX_BF16 if s.dtype == "bf16" else kvx.KVX_FP32
         self.tr = kvx.Translator(s.src, s.dst, to_dev(c.w_k, s.dtype), to_dev(c.w_v, s.dtype),
                                  layer_map=list(c.layer_map) if explicit_layer_map else None,
-                                 dtype=kdt, path=path)
+                                 dtype=kdt, path=path, max_position=max_position)
         wl = c.wl
         any_l = next(iter(c.src_k))
         self.src_k_dev = {l: to_dev(c.src_k[l], s.dtype) for l in c.src_k}

@@ -30,16 +30,16 @@ def _lib():
     yield
 
 
-def _run(c, path, paged=None):
+def _run(c, path, paged=None, max_position=0):
     from gpu_harness import GpuRun
-    g = GpuRun(c, path=path, paged=paged)
+    g = GpuRun(c, path=path, paged=paged, max_position=max_position)
     g.run()
     torch.cuda.synchronize()
     return g
 
 
-def _full_compare(c, path, paged=None):
-    g = _run(c, path, paged)
+def _full_compare(c, path, paged=None, max_position=0):
+    g = _run(c, path, paged, max_position)
     ok, ov = oracle_problem(c).translate()
     gk, gv = g.gather()
     sk = compare(gk, ok, c.spec.dtype)
@@ -86,7 +86,7 @@ def test_explicit_positions_and_layer_map(path):
     src_pos = rng.integers(0, 120000, size=(wl.batch, wl.s_max)).astype(np.int32)
     tgt_pos = (np.arange(wl.total_tgt) * 7 + 3000).astype(np.int32)
     c = make_case(spec, [200, 77], src_pos=src_pos, tgt_pos=tgt_pos)
-    _full_compare(c, path)
+    _full_compare(c, path, max_position=1 << 17)
 
 
 def test_tiny_token_counts_and_empty_sequences():
