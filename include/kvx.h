@@ -87,9 +87,8 @@ typedef struct {
                                    layer, each in [0, src.num_layers); NULL = nearest relative
                                    depth (kvx_layer_map_nearest) */
     int32_t dtype;              /* kvx_dtype of caches and weights */
-    int32_t max_position;       /* RoPE positions must lie in [0, max_position); 0 = 1<<16.
-                                   At most 1<<20.  Sizes the rotation tables
-                                   (max_position * head_dim * 4 bytes per rotating model). */
+    int32_t max_position;       /* RoPE positions must lie in [0, max_position); 0 = 1<<24,
+                                   at most 1<<30.  Positions outside are clamped and flagged. */
     int32_t path;               /* kvx_path */
 } kvx_translator_desc;
 

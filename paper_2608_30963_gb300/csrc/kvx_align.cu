@@ -54,25 +54,4 @@ cudaError_t launch_build_alignment(int batch, int total_tgt, const int* src_seq_
     return cudaGetLastError();
 }
 
-// Rotation table: cs[p][i] = (cos, sin)(p * f_i), f_i = base^(-2i/d); angle and
-// trigonometry in double, stored as fp32.
-__global__ void rope_table_kernel(float2* cs, int max_pos, int d, double base)
-{
-    const int half = d >> 1;
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= (long long)max_pos * half) return;
-    const int p = (int)(idx / half), i = (int)(idx - (long long)p * half);
-    const double f = pow(base, -2.0 * (double)i / (double)d);
-    double s, c;
-    sincos((double)p * f, &s, &c);
-    cs[idx] = make_float2((float)c, (float)s);
-}
-
-cudaError_t launch_rope_table(float2* cs, int max_pos, int d, double base, cudaStream_t stream)
-{
-    const long long n = (long long)max_pos * (d / 2);
-    rope_table_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(cs, max_pos, d, base);
-    return cudaGetLastError();
-}
-
 }  // namespace kvx

@@ -9,13 +9,15 @@
 
 namespace kvx {
 
-// Rotation table: cos/sin of the exact angle p * f_i, f_i = base^(-2i/d), for
-// every position p < max_position and frequency i < d/2, computed in double
-// precision and stored as fp32 (cos, sin) pairs, row p contiguous.
+// Rotation frequencies as fixed-point turns: turns[i] = round(2^64 * f_i / (2 pi)),
+// f_i = base^(-2i/d) (computed in double on the host).  For an integer position
+// p, p * turns[i] mod 2^64 is the fractional part of the angle p * f_i in turns,
+// exact up to the rounding of turns[i] (|error| <= p * 2^-53 turn), so the
+// range reduction costs one 64-bit multiply and no table of angles.
 struct RopeTable {
-    const float2* cs;   // [max_position][d/2]
-    int half;           // d/2
-    int enabled;        // 0: no rotation
+    const unsigned long long* turns;   // device [d/2]
+    int half;                          // d/2
+    int enabled;                       // 0: no rotation
 };
 
 // Everything one kvx_translate launch needs, passed by value (graph-capturable;
@@ -61,10 +63,22 @@ __device__ __forceinline__ void set_status(unsigned* status, unsigned bit)
     if (status) atomicOr(status, bit);
 }
 
+// (cos, sin) of the angle whose turns are p * G (mod 1): the top 32 bits of the
+// 64-bit product are the signed fraction of a turn in [-1/2, 1/2), i.e. an
+// angle in [-pi, pi) where the hardware sine/cosine is accurate to ~4e-7.
+__device__ __forceinline__ float2 turn_cs(unsigned long long G, int p)
+{
+    const unsigned long long t = G * (unsigned long long)(unsigned)p;
+    const float a = (float)(int)(t >> 32) * 1.4629180792671596e-09f;   // 2 pi / 2^32
+    float sn, cs;
+    __sincosf(a, &sn, &cs);
+    return make_float2(cs, sn);
+}
+
 // (cos, sin) of angle p * f_i (p already clamped to [0, max_position)).
 __device__ __forceinline__ float2 rope_cs(const RopeTable& t, int p, int i)
 {
-    return __ldg(&t.cs[(size_t)p * t.half + i]);
+    return turn_cs(__ldg(&t.turns[i]), p);
 }
 
 __device__ __forceinline__ int clamp_pos(int p, int max_position, unsigned* status)

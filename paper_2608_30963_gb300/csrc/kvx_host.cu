@@ -1,5 +1,6 @@
 // kvx_host.cu -- host side of the kvx C ABI: validation, translator state,
 // weight upload and re-layout, RoPE tables, launch selection, error status.
+#include <math.h>
 #include <stdarg.h>
 #include <stdio.h>
 #include <string.h>
@@ -21,7 +22,7 @@ struct kvx_translator {
     int max_position = 0;
     void* w = nullptr;           // SIMT: [2][Lt][Ht][in][out] dtype; tcgen05: pre-swizzled images
     size_t w_bytes = 0;
-    float2* rope = nullptr;      // src hi | src lo | dst hi | dst lo
+    unsigned long long* rope = nullptr;   // fixed-point turns: source [d_s/2] | target [d_t/2]
     size_t rope_bytes = 0;
     RopeTable rs{}, rt{};
     unsigned* status = nullptr;
@@ -97,9 +98,9 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         return fail(KVX_ERR_INVALID_ARG, "create: unknown dtype %d", desc->dtype);
     if (desc->path < KVX_PATH_AUTO || desc->path > KVX_PATH_TCGEN05)
         return fail(KVX_ERR_INVALID_ARG, "create: unknown path %d", desc->path);
-    int max_pos = desc->max_position ? desc->max_position : (1 << 16);
-    if (max_pos < 1 || max_pos > (1 << 20))
-        return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<20]");
+    int max_pos = desc->max_position ? desc->max_position : (1 << 24);
+    if (max_pos < 1 || max_pos > (1 << 30))
+        return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<30]");
 
     kvx_translator* t = new kvx_translator();
     t->desc = *desc;
@@ -183,27 +184,29 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         raw = nullptr;
     }
 
-    {   // RoPE tables (one shared table when both models rotate alike)
-        const size_t src_n = s.rope_base > 0.0 ? (size_t)max_pos * (s.head_dim / 2) : 0;
-        const bool same = s.rope_base > 0.0 && s.rope_base == d.rope_base && s.head_dim == d.head_dim;
-        const size_t dst_n = d.rope_base > 0.0 && !same ? (size_t)max_pos * (d.head_dim / 2) : 0;
-        t->rope_bytes = (src_n + dst_n) * sizeof(float2);
-        if (t->rope_bytes && cudaMalloc(&t->rope, t->rope_bytes) != cudaSuccess) {
+    {   // rotation frequencies as fixed-point turns (kvx_common.cuh)
+        const int hs = s.head_dim / 2, hd = d.head_dim / 2;
+        unsigned long long h_turns[256];
+        auto fill = [&](const kvx_model_geom& g, unsigned long long* out) {
+            for (int i = 0; i < g.head_dim / 2; ++i) {
+                if (g.rope_base <= 0.0) { out[i] = 0; continue; }
+                const double f = pow(g.rope_base, -2.0 * (double)i / (double)g.head_dim);
+                out[i] = (unsigned long long)ldexp(f / (2.0 * M_PI), 64);
+            }
+        };
+        fill(s, h_turns);
+        fill(d, h_turns + hs);
+        t->rope_bytes = (size_t)(hs + hd) * sizeof(unsigned long long);
+        if (cudaMalloc(&t->rope, t->rope_bytes) != cudaSuccess) {
             st = fail(KVX_ERR_OOM, "create: table allocation");
             goto err;
         }
-        float2* stab = src_n ? t->rope : nullptr;
-        float2* dtab = same ? stab : (dst_n ? t->rope + src_n : nullptr);
-        t->rs = RopeTable{stab, s.head_dim / 2, s.rope_base > 0.0};
-        t->rt = RopeTable{dtab, d.head_dim / 2, d.rope_base > 0.0};
-        if (src_n && (ce = launch_rope_table(stab, max_pos, s.head_dim, s.rope_base, 0)) != cudaSuccess) {
-            st = fail(KVX_ERR_CUDA, "create: rope table: %s", cudaGetErrorString(ce));
+        if ((ce = cudaMemcpy(t->rope, h_turns, t->rope_bytes, cudaMemcpyHostToDevice)) != cudaSuccess) {
+            st = fail(KVX_ERR_CUDA, "create: table upload: %s", cudaGetErrorString(ce));
             goto err;
         }
-        if (dst_n && (ce = launch_rope_table(dtab, max_pos, d.head_dim, d.rope_base, 0)) != cudaSuccess) {
-            st = fail(KVX_ERR_CUDA, "create: rope table: %s", cudaGetErrorString(ce));
-            goto err;
-        }
+        t->rs = RopeTable{t->rope, hs, s.rope_base > 0.0};
+        t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0};
     }
     if (cudaMalloc(&t->status, sizeof(unsigned)) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: status allocation"); goto err; }
     if ((ce = cudaMemset(t->status, 0, sizeof(unsigned))) != cudaSuccess ||

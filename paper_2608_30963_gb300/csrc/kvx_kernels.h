@@ -13,7 +13,6 @@ cudaError_t launch_build_alignment(int batch, int total_tgt, const int* src_seq_
                                    const int* tgt_seq_off, const int* tgt_end, int* span_lo, int* span_hi,
                                    unsigned* status, cudaStream_t stream);
 
-cudaError_t launch_rope_table(float2* cs, int max_pos, int d, double base, cudaStream_t stream);
 
 // tensor-core path
 struct TcConfig {

@@ -67,7 +67,7 @@ struct SlotHdr {
 struct TcLaunch {
     int n_tile, n_split, in_dim, groups, m_tiles;
     unsigned b_bytes, a_bytes, row_bytes, stage_row_bytes, ring_bytes;
-    unsigned off_b, off_a, off_stage, off_ring, off_meta, off_hdr, off_bar, off_misc, off_seq;
+    unsigned off_b, off_a, off_stage, off_ring, off_meta, off_hdr, off_bar, off_misc, off_seq, off_turns, off_slot;
     int seq_cached;   // per-sequence offsets and source lengths copied to shared memory
     unsigned idesc;
     unsigned tmem_cols;
@@ -97,6 +97,20 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
         : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+// As above, but the thread may sleep in hardware (up to hint_ns) until the
+// phase completes, instead of spinning on the barrier word.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity), "r"(hint_ns)
         : "memory");
     return ok != 0;
 }
@@ -207,7 +221,7 @@ struct Waiter {
         if (mbar_try_wait(bar, parity)) return true;
         const unsigned long long t0 = globaltimer();
         while (true) {
-            if (mbar_try_wait(bar, parity)) return true;
+            if (mbar_try_wait_sleep(bar, parity, 100000u)) return true;
             if (*abort) return false;
             if (globaltimer() - t0 > kWaitNs) {
                 *abort = 1;
@@ -333,21 +347,13 @@ __device__ __forceinline__ void store_bf16_smem(uint8_t* p, const float (&x)[PP]
     }
 }
 
-// (cos, sin) for PP consecutive frequencies i0.. at position p (PP even: 16-byte loads).
+// (cos, sin) for PP consecutive frequencies i0.. at position p, from the
+// fixed-point turns held in shared memory.
 template <int PP>
-__device__ __forceinline__ void rope_cs_vec(const RopeTable& t, int p, int i0, float2 (&cs)[PP])
+__device__ __forceinline__ void rope_cs_vec(const unsigned long long* turns, int p, int i0, float2 (&cs)[PP])
 {
-    const float2* hp = t.cs + (size_t)p * t.half + i0;
-    if constexpr (PP >= 2) {
 #pragma unroll
-        for (int q = 0; q < PP; q += 2) {
-            const float4 v = __ldg(reinterpret_cast<const float4*>(hp + q));
-            cs[q] = make_float2(v.x, v.y);
-            cs[q + 1] = make_float2(v.z, v.w);
-        }
-    } else {
-        cs[0] = __ldg(hp);
-    }
+    for (int q = 0; q < PP; ++q) cs[q] = turn_cs(turns[i0 + q], p);
 }
 
 // ------------------------------------------------------------------ the kernel
@@ -391,6 +397,10 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         tmem_alloc(smem_u32(sTmemBase), L.tmem_cols);
         tmem_relinquish();
     }
+    unsigned long long* sTurnS = reinterpret_cast<unsigned long long*>(smem + L.off_turns);
+    unsigned long long* sTurnT = sTurnS + (P.ds >> 1);
+    for (int i = threadIdx.x; i < (P.ds >> 1); i += blockDim.x) sTurnS[i] = P.rs.enabled ? __ldg(&P.rs.turns[i]) : 0ull;
+    for (int i = threadIdx.x; i < (P.dt >> 1); i += blockDim.x) sTurnT[i] = P.rt.enabled ? __ldg(&P.rt.turns[i]) : 0ull;
     int* sSeqOff = reinterpret_cast<int*>(smem + L.off_seq);
     int* sSrcLen = sSeqOff + kMaxSeqCache + 1;
     if (L.seq_cached) {
@@ -419,7 +429,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         int cur_g = -1;
         uint32_t b_loads = 0, issued = 0, released = 0;
         unsigned long long head = 0;                 // monotonic ring byte counter
-        unsigned long long slot_start[kNumSlots];
+        unsigned long long* slot_start = reinterpret_cast<unsigned long long*>(smem + L.off_slot);   // lane 0's copy
         bool ok = true;
         // wait until sub-tile k (0-based) has been released by the prologue warps
         auto release_upto = [&](uint32_t k) -> bool {
@@ -602,14 +612,14 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             if (valid) resolve_dst(P, sv, tp, dst_off, pt);
             const bool rot = x.kv == 0 && P.rt.enabled;
             float2 cs[8];
-            if (rot) rope_cs_vec<8>(P.rt, pt, x.nt * hw, cs);
+            if (rot) rope_cs_vec<8>(sTurnT, pt, x.nt * hw, cs);
             if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
             tc_fence_after();
             bulk_wait_read0();
             const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)L.n_tile;
             for (int pc = 0; pc < hw; pc += 8) {
                 float2 csn[8];
-                if (rot && pc + 8 < hw) rope_cs_vec<8>(P.rt, pt, x.nt * hw + pc + 8, csn);
+                if (rot && pc + 8 < hw) rope_cs_vec<8>(sTurnT, pt, x.nt * hw + pc + 8, csn);
                 uint32_t r0[8], r1[8];
                 tmem_ld8(taddr + pc, r0);
                 tmem_ld8(taddr + hw + pc, r1);
@@ -692,7 +702,6 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     for (int e = 0; e < PP; ++e) { a0[u4][e] = 0.f; a1[u4][e] = 0.f; }
                 for (int o = 0; o < maxn; ++o) {
                     typename Raw<PP>::T w0[kTok], w1[kTok];
-                    float2 cs[kTok][PP];
 #pragma unroll
                     for (int u4 = 0; u4 < kTok; ++u4) {
                         if (o < n[u4]) {
@@ -705,7 +714,6 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                                 rp = src + (long long)mt[u4].b * P.sb + (long long)g * P.sh + (long long)srow * P.ss;
                             w0[u4] = load_raw<PP>(rp + i0);
                             w1[u4] = load_raw<PP>(rp + hs + i0);
-                            if (rot) rope_cs_vec<PP>(P.rs, src_pos_of(P, mt[u4].b, srow), i0, cs[u4]);
                         }
                     }
 #pragma unroll
@@ -715,11 +723,13 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                             unpack(w0[u4], x0);
                             unpack(w1[u4], x1);
                             if (rot) {
+                                float2 cs[PP];
+                                rope_cs_vec<PP>(sTurnS, src_pos_of(P, mt[u4].b, mt[u4].lo + o), i0, cs);
 #pragma unroll
                                 for (int e = 0; e < PP; ++e) {
                                     // undo the rotation: R(-theta)
-                                    const float u0 = fmaf(x0[e], cs[u4][e].x, x1[e] * cs[u4][e].y);
-                                    const float u1 = fmaf(x1[e], cs[u4][e].x, -x0[e] * cs[u4][e].y);
+                                    const float u0 = fmaf(x0[e], cs[e].x, x1[e] * cs[e].y);
+                                    const float u1 = fmaf(x1[e], cs[e].x, -x0[e] * cs[e].y);
                                     x0[e] = u0;
                                     x1[e] = u1;
                                 }
@@ -733,10 +743,12 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 for (int u4 = 0; u4 < kTok; ++u4) {
                     if (n[u4] < 0) continue;
                     const int row = sq * kSub + tw + u4 * kNumXfWarps;
+                    // span mean; 1/n is exact for n = 1, 2 (the common spans)
+                    const float inv_n = n[u4] > 0 ? __frcp_rn((float)n[u4]) : 0.f;
 #pragma unroll
                     for (int e = 0; e < PP; ++e) {
-                        a0[u4][e] = n[u4] > 0 ? a0[u4][e] / (float)n[u4] : 0.f;
-                        a1[u4][e] = n[u4] > 0 ? a1[u4][e] / (float)n[u4] : 0.f;
+                        a0[u4][e] *= inv_n;
+                        a1[u4][e] *= inv_n;
                     }
                     store_bf16_smem<PP>(sA + sw128_off(row, k0, kTileM), a0[u4]);
                     store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1[u4]);
@@ -835,6 +847,8 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
     L.off_bar = take(kNumBars * 8, 8);
     L.off_misc = take(16, 16);
     L.off_seq = take((2 * kMaxSeqCache + 1) * sizeof(int), 16);
+    L.off_turns = take((unsigned)(ds / 2 + dt / 2) * 8, 16);
+    L.off_slot = take(kNumSlots * 8, 16);
     L.off_ring = (off + 127) / 128 * 128;
     const int avail = kSmemMax - 1024 - (int)L.off_ring;   // 1024: alignment slack of the dynamic base
     L.ring_bytes = avail > 0 ? (unsigned)(avail / 1024 * 1024) : 0;
