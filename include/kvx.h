@@ -131,7 +131,10 @@ typedef struct {
     const int32_t* span_lo;     /* device int32[T_total]: first source token (index within its
                                    sequence) of each target token's span; NULL with span_hi
                                    NULL = identity alignment (span of t is [t, t+1)) */
-    const int32_t* span_hi;     /* device int32[T_total]: one past the span's last source token */
+    const int32_t* span_hi;     /* device int32[T_total]: one past the span's last source token.
+                                   With identity alignment a target token at or past its
+                                   sequence's source length is flagged (KVX_DEV_SPAN_CLAMPED)
+                                   and its output row is unspecified. */
     const int32_t* pos;         /* device int32[T_total]: RoPE position of each target token, or
                                    NULL for its index within its sequence */
 } kvx_tgt_tokens;

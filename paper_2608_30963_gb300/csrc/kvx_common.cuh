@@ -9,6 +9,9 @@
 
 namespace kvx {
 
+constexpr int KVX_MAX_ALIGNED_LAYERS = 96;   // target layers the identity-alignment kernel takes (param space)
+constexpr int KVX_MAX_ALIGNED_BATCH = 256;   // sequences whose metadata it keeps in shared memory
+
 // Rotation frequencies as fixed-point turns: turns[i] = round(2^64 * f_i / (2 pi)),
 // f_i = base^(-2i/d) (computed in double on the host).  For an integer position
 // p, p * turns[i] mod 2^64 is the fractional part of the angle p * f_i in turns,
@@ -154,6 +157,13 @@ __device__ __forceinline__ TokenInfo resolve_token(const TranslateParams& P, int
 __device__ __forceinline__ long long dst_head_off(const TranslateParams& P, int h)
 {
     return P.paged ? (long long)h * P.dt : (long long)h * P.dh;
+}
+
+__device__ __forceinline__ int src_pos_of_seq(const int* src_pos, int src_max_seq, int b, int s, int max_position,
+                                              unsigned* status)
+{
+    const int p = src_pos ? __ldg(&src_pos[(size_t)b * src_max_seq + s]) : s;
+    return clamp_pos(p, max_position, status);
 }
 
 __device__ __forceinline__ int src_pos_of(const TranslateParams& P, int b, int s)

@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <string>
+#include <vector>
 
 #include "kvx_common.cuh"
 #include "kvx_kernels.h"
@@ -27,7 +28,46 @@ struct kvx_translator {
     RopeTable rs{}, rt{};
     unsigned* status = nullptr;
     TcConfig tc{};
+    // encoded source tensor maps of the identity-alignment kernel, a few per (target layer, K|V)
+    struct MapEntry {
+        const void* ptr = nullptr;
+        int S = 0, B = 0;
+        long long ss = 0, sh = 0, sb = 0;
+        unsigned long long stamp = 0;
+        alignas(64) unsigned char map[128];
+    };
+    static constexpr int kMapWays = 4;
+    std::vector<MapEntry> maps;
+    unsigned long long map_stamp = 0;
 };
+
+// Encoded tensor map for the source K or V cache of target layer j (cached by
+// pointer, length, batch and strides).  Returns nullptr if encoding fails.
+static const void* source_map(kvx_translator* t, int j, int kv, const void* ptr, const kvx_src_kv* src)
+{
+    const int slot = (j * 2 + kv) * kvx_translator::kMapWays;
+    kvx_translator::MapEntry* lru = nullptr;
+    for (int w = 0; w < kvx_translator::kMapWays; ++w) {
+        kvx_translator::MapEntry& e = t->maps[slot + w];
+        if (e.ptr == ptr && e.S == src->max_seq && e.B == src->batch && e.ss == src->stride_s &&
+            e.sh == src->stride_h && e.sb == src->stride_b) {
+            e.stamp = ++t->map_stamp;
+            return e.map;
+        }
+        if (!lru || e.stamp < lru->stamp) lru = &e;
+    }
+    if (!encode_source_map(lru->map, ptr, t->desc.src.head_dim, src->max_seq, t->desc.src.num_kv_heads, src->batch,
+                           src->stride_s, src->stride_h, src->stride_b))
+        return nullptr;
+    lru->ptr = ptr;
+    lru->S = src->max_seq;
+    lru->B = src->batch;
+    lru->ss = src->stride_s;
+    lru->sh = src->stride_h;
+    lru->sb = src->stride_b;
+    lru->stamp = ++t->map_stamp;
+    return lru->map;
+}
 
 static thread_local std::string g_last_error;
 
@@ -279,8 +319,24 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
             return fail(KVX_ERR_INVALID_ARG, "translate: cache pointers must be 16-byte aligned (layer %d)", j);
     }
     cudaError_t ce;
-    if (tr->path == KVX_PATH_TCGEN05) ce = launch_translate_tc(P, tr->tc, tr->num_sms, (cudaStream_t)stream);
-    else ce = launch_translate_simt(P, D.dtype, (cudaStream_t)stream);
+    if (tr->path == KVX_PATH_TCGEN05 && !tgt->span_lo &&
+        aligned_supported(tr->in_dim, D.dst.head_dim, D.src.head_dim, Lt, src->batch)) {
+        // identity alignment: tensor-TMA fed kernel
+        if (tr->maps.empty()) tr->maps.resize((size_t)2 * KVX_MAX_ALIGNED_LAYERS * kvx_translator::kMapWays);
+        const void* maps[2 * KVX_MAX_ALIGNED_LAYERS];
+        for (int j = 0; j < Lt; ++j)
+            for (int kv = 0; kv < 2; ++kv) {
+                maps[2 * j + kv] = source_map(tr, j, kv, kv ? P.src_v[j] : P.src_k[j], src);
+                if (!maps[2 * j + kv])
+                    return fail(KVX_ERR_INVALID_ARG, "translate: cannot describe the source cache of layer %d to the "
+                                                     "tensor-copy unit (strides, sizes)", tr->layer_map[j]);
+            }
+        ce = launch_translate_tc_aligned(P, maps, tr->num_sms, (cudaStream_t)stream);
+    } else if (tr->path == KVX_PATH_TCGEN05) {
+        ce = launch_translate_tc(P, tr->tc, tr->num_sms, (cudaStream_t)stream);
+    } else {
+        ce = launch_translate_simt(P, D.dtype, (cudaStream_t)stream);
+    }
     if (ce != cudaSuccess) return fail(KVX_ERR_CUDA, "translate: launch failed: %s", cudaGetErrorString(ce));
     return KVX_OK;
 }

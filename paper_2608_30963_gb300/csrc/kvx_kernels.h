@@ -27,4 +27,12 @@ size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht);
 cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
                                       int dt, int n_tile, cudaStream_t stream);
 cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, cudaStream_t stream);
+
+// identity-alignment tensor-core path (tensor-TMA fed)
+bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch);
+size_t aligned_map_bytes();
+bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int Hs, int batch, long long ss,
+                       long long sh, long long sb);
+cudaError_t launch_translate_tc_aligned(const TranslateParams& P, const void* const* maps, int num_sms,
+                                        cudaStream_t stream);
 }  // namespace kvx

@@ -26,6 +26,7 @@
 // returns (no trap, no hang).
 #include "kvx_common.cuh"
 #include "kvx_kernels.h"
+#include "kvx_tc_common.cuh"
 
 namespace kvx {
 namespace {
@@ -41,8 +42,6 @@ constexpr int kNumEpiWarps = 4;
 constexpr int kXfWarp0 = 6;
 constexpr int kNumXfWarps = 8;
 constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
-constexpr int kSmemMax = 232448;          // 227 KB opt-in per block
-constexpr unsigned long long kWaitNs = 1000000000ull;
 constexpr int kMaxSeqCache = 512;         // sequences whose metadata is kept in shared memory
 
 // barrier indices
@@ -73,174 +72,15 @@ struct TcLaunch {
     unsigned tmem_cols;
 };
 
-// ------------------------------------------------------------------ PTX wrappers
-__device__ __forceinline__ uint32_t smem_u32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count)
-{
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive(uint32_t bar)
-{
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t bar, uint32_t bytes)
-{
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-// As above, but the thread may sleep in hardware (up to hint_ns) until the
-// phase completes, instead of spinning on the barrier word.
-__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t bar, uint32_t parity, uint32_t hint_ns)
-{
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity), "r"(hint_ns)
-        : "memory");
-    return ok != 0;
-}
-__device__ __forceinline__ unsigned long long globaltimer()
-{
-    unsigned long long t;
-    asm volatile("mov.u64 %0, %globaltimer;" : "=l"(t));
-    return t;
-}
-__device__ __forceinline__ uint64_t policy_evict_first()
-{
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-__device__ __forceinline__ uint64_t policy_evict_last()
-{
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-// global -> shared bulk copy completing on an mbarrier (16-byte aligned, size % 16 == 0)
-__device__ __forceinline__ void bulk_g2s(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar, uint64_t pol)
-{
-    asm volatile(
-        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint [%0], [%1], %2, [%3], %4;" ::"r"(dst),
-        "l"(src), "r"(bytes), "r"(bar), "l"(pol)
-        : "memory");
-}
-// shared -> global bulk copy in the thread's bulk group
-__device__ __forceinline__ void bulk_s2g(void* dst, uint32_t src, uint32_t bytes)
-{
-    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
-                 : "memory");
-}
-__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
-__device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-__device__ __forceinline__ void fence_mbar_init() { asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory"); }
-
-__device__ __forceinline__ void tmem_alloc(uint32_t dst_smem, uint32_t ncols)
-{
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
-                 : "memory");
-}
-__device__ __forceinline__ void tmem_relinquish()
-{
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-}
-__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols)
-{
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
-}
-__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
-__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
-
-// D[tmem] (+)= A[smem] . B[smem]^T, bf16 inputs, fp32 accumulate
-__device__ __forceinline__ void umma_bf16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
-                                          uint32_t accumulate)
-{
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "setp.ne.b32 p, %4, 0;\n\t"
-        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate)
-        : "memory");
-}
-__device__ __forceinline__ void umma_commit(uint32_t bar)
-{
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-                 : "memory");
-}
-__device__ __forceinline__ void tmem_ld8(uint32_t taddr, uint32_t (&r)[8])
-{
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x8.b32 {%0,%1,%2,%3,%4,%5,%6,%7}, [%8];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7])
-                 : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
-
-// Shared-memory matrix descriptor: K-major, 128-byte swizzle, 8-row atoms 1024 B apart.
-__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr)
-{
-    uint64_t d = 0;
-    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);      // start address
-    d |= (uint64_t)1 << 16;                         // leading byte offset (unused for swizzled K-major)
-    d |= (uint64_t)(1024u >> 4) << 32;              // stride byte offset between 8-row atoms
-    d |= (uint64_t)1 << 46;                         // descriptor version
-    d |= (uint64_t)2 << 61;                         // 128-byte swizzle
-    return d;
-}
-
-// Byte offset of element (row, k) in a K-major SW128 tile with `rows` rows
-// (K split into 64-element blocks of rows*128 bytes).
-__device__ __forceinline__ uint32_t sw128_off(int row, int k, int rows)
-{
-    const int kb = k >> 6, c = (k >> 3) & 7, e = k & 7;
-    return (uint32_t)(kb * rows * 128 + (row >> 3) * 1024 + (row & 7) * 128 + ((c ^ (row & 7)) << 4) + e * 2);
-}
-
-// ------------------------------------------------------------------ bounded waits
-struct Waiter {
-    volatile int* abort;
-    unsigned* status;
-    __device__ __forceinline__ bool wait(uint32_t bar, uint32_t parity) const
-    {
-        if (mbar_try_wait(bar, parity)) return true;
-        const unsigned long long t0 = globaltimer();
-        while (true) {
-            if (mbar_try_wait_sleep(bar, parity, 100000u)) return true;
-            if (*abort) return false;
-            if (globaltimer() - t0 > kWaitNs) {
-                *abort = 1;
-                set_status(status, KVX_DEV_WAIT_TIMEOUT);
-                return false;
-            }
-        }
-    }
-};
-
 struct Unit {
     int j, h, kv, nt, tile, g;
 };
-__device__ __forceinline__ Unit decode(long long u, const TcLaunch& L, int Ht)
+__device__ __forceinline__ Unit make_unit(int g, int tile, const TcLaunch& L, int Ht)
 {
     Unit x;
-    x.g = (int)(u / L.m_tiles);
-    x.tile = (int)(u - (long long)x.g * L.m_tiles);
-    int rest = x.g;
+    x.g = g;
+    x.tile = tile;
+    int rest = g;
     x.nt = rest % L.n_split;
     rest /= L.n_split;
     x.kv = rest & 1;
@@ -249,6 +89,19 @@ __device__ __forceinline__ Unit decode(long long u, const TcLaunch& L, int Ht)
     x.j = rest / Ht;
     return x;
 }
+// The CTA's contiguous range of units (group-major, tile-minor), walked without divisions.
+struct UnitRange {
+    int g0, t0, count;
+    __device__ __forceinline__ void init(const TcLaunch& L)
+    {
+        const long long U = (long long)L.groups * L.m_tiles;
+        const long long b = (long long)blockIdx.x * U / gridDim.x;
+        const long long e = (long long)(blockIdx.x + 1) * U / gridDim.x;
+        g0 = (int)(b / L.m_tiles);
+        t0 = (int)(b - (long long)g0 * L.m_tiles);
+        count = (int)(e - b);
+    }
+};
 
 // Sequence metadata view: shared-memory copies of seq_off / src_seq_len when the
 // batch is small enough, else the global arrays.
@@ -305,45 +158,6 @@ __device__ __forceinline__ void resolve_dst(const TranslateParams& P, const SeqV
         const int page = pi < P.max_pages ? __ldg(&P.page_table[(size_t)b * P.max_pages + pi]) : -1;
         if (page < 0 || page >= P.num_pages) { set_status(P.status, KVX_DEV_PAGE_INVALID); dst_off = -1; }
         else dst_off = ((long long)page * P.page_size + (t % P.page_size)) * (long long)P.Ht * P.dt;
-    }
-}
-
-__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b)
-{
-    __nv_bfloat162 v = __floats2bfloat162_rn(a, b);
-    return *reinterpret_cast<uint32_t*>(&v);
-}
-
-// PP consecutive bf16 values (PP in {1,2,4}) as one raw load.
-template <int PP> struct Raw;
-template <> struct Raw<4> { using T = uint2; };
-template <> struct Raw<2> { using T = uint32_t; };
-template <> struct Raw<1> { using T = unsigned short; };
-
-template <int PP>
-__device__ __forceinline__ typename Raw<PP>::T load_raw(const __nv_bfloat16* p)
-{
-    return *reinterpret_cast<const typename Raw<PP>::T*>(p);
-}
-__device__ __forceinline__ void unpack(uint2 w, float (&x)[4])
-{
-    x[0] = bf_lo(w.x); x[1] = bf_hi(w.x); x[2] = bf_lo(w.y); x[3] = bf_hi(w.y);
-}
-__device__ __forceinline__ void unpack(uint32_t w, float (&x)[2]) { x[0] = bf_lo(w); x[1] = bf_hi(w); }
-__device__ __forceinline__ void unpack(unsigned short w, float (&x)[1]) { x[0] = __uint_as_float((uint32_t)w << 16); }
-
-template <int PP>
-__device__ __forceinline__ void store_bf16_smem(uint8_t* p, const float (&x)[PP])
-{
-    if constexpr (PP == 4) {
-        *reinterpret_cast<uint2*>(p) = make_uint2(pack_bf16(x[0], x[1]), pack_bf16(x[2], x[3]));
-    } else if constexpr (PP == 2) {
-        *reinterpret_cast<uint32_t*>(p) = pack_bf16(x[0], x[1]);
-    } else {
-        __nv_bfloat16 v = __float2bfloat16_rn(x[0]);
-        *reinterpret_cast<__nv_bfloat16*>(p) = v;
     }
 }
 
@@ -414,9 +228,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
 
     const Waiter W{sAbort, P.status};
     const SeqView sv{L.seq_cached ? sSeqOff : P.seq_off, L.seq_cached ? sSrcLen : P.src_seq_len, P.batch};
-    const long long U = (long long)L.groups * L.m_tiles;
-    const long long u_begin = (long long)blockIdx.x * U / gridDim.x;
-    const long long u_end = (long long)(blockIdx.x + 1) * U / gridDim.x;
+    UnitRange ur;
+    ur.init(L);
     const int hw = L.n_tile >> 1;                 // pair half-width of an output split
     const int half_t = P.dt >> 1;
 
@@ -439,8 +252,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             }
             return true;
         };
-        for (long long u = u_begin; u < u_end && ok; ++u) {
-            const Unit x = decode(u, L, P.Ht);
+        for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count && ok; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
+            const Unit x = make_unit(ug, ut, L, P.Ht);
             if (x.g != cur_g) {
                 if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
                 if (lane == 0) mbar_arrive_expect_tx(bar(kBarBFull), L.b_bytes);
@@ -487,8 +300,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 const unsigned R = (unsigned)__shfl_sync(0xffffffffu, incl, 31);
                 const unsigned need_rows = R * (unsigned)r_heads;
                 const bool direct = __any_sync(0xffffffffu, nonmono) ||
-                                    (unsigned long long)need_rows * L.row_bytes > L.ring_bytes;
-                const unsigned need = direct ? 0u : need_rows * L.row_bytes;
+                                    (unsigned long long)need_rows * L.row_bytes + 128ull * r_heads > L.ring_bytes;
+                const unsigned hstride = R * L.row_bytes + 128;   // pad: the head halves of a warp hit different banks
+                const unsigned need = direct || R == 0 ? 0u : (unsigned)r_heads * hstride;
 
                 // slot reuse and ring space
                 const uint32_t slot = issued % kNumSlots;
@@ -518,7 +332,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 __threadfence_block();
                 __syncwarp();
                 if (lane == 0) {
-                    if (need) mbar_arrive_expect_tx(bar(kBarSlotFull + slot), need);
+                    if (need) mbar_arrive_expect_tx(bar(kBarSlotFull + slot), need_rows * L.row_bytes);   // bytes copied
                     else mbar_arrive(bar(kBarSlotFull + slot));
                 }
                 __syncwarp();
@@ -536,7 +350,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                             for (int q = 0; q < r_heads; ++q) {
                                 const __nv_bfloat16* s0 =
                                     src + (long long)b * P.sb + (long long)(g0 + q) * P.sh + (long long)cover * P.ss;
-                                bulk_g2s(ring0 + ((unsigned)q * R + (unsigned)start) * L.row_bytes, s0,
+                                bulk_g2s(ring0 + (unsigned)q * hstride + (unsigned)start * L.row_bytes, s0,
                                          rows * L.row_bytes, bar(kBarSlotFull + slot), pol_stream);
                             }
                         }
@@ -545,7 +359,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                             for (int q = 0; q < r_heads; ++q) {
                                 const __nv_bfloat16* s0 =
                                     src + (long long)b * P.sb + (long long)(g0 + q) * P.sh + (long long)s * P.ss;
-                                bulk_g2s(ring0 + ((unsigned)q * R + (unsigned)(start + s - cover)) * L.row_bytes,
+                                bulk_g2s(ring0 + (unsigned)q * hstride + (unsigned)(start + s - cover) * L.row_bytes,
                                          s0, L.row_bytes, bar(kBarSlotFull + slot), pol_stream);
                             }
                     }
@@ -567,8 +381,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         if (lane == 0) {
             int cur_g = -1;
             uint32_t b_cnt = 0, tcount = 0;
-            for (long long u = u_begin; u < u_end; ++u) {
-                const Unit x = decode(u, L, P.Ht);
+            for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
+                const Unit x = make_unit(ug, ut, L, P.Ht);
                 if (x.g != cur_g) {
                     if (!W.wait(bar(kBarBFull), b_cnt & 1)) break;
                     ++b_cnt;
@@ -588,7 +402,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 }
                 umma_commit(bar(kBarAEmpty));
                 umma_commit(bar(kBarDFull + buf));
-                const bool last_of_group = (u + 1 == u_end) || ((u + 1) / L.m_tiles != x.g);
+                const bool last_of_group = (it + 1 == ur.count) || (ut + 1 == L.m_tiles);
                 if (last_of_group) umma_commit(bar(kBarBEmpty));
                 ++tcount;
             }
@@ -601,8 +415,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         uint8_t* srow = sStage + (size_t)m * L.stage_row_bytes;
         const uint32_t srow_u32 = smem_u32(srow);
         uint32_t tcount = 0;
-        for (long long u = u_begin; u < u_end; ++u) {
-            const Unit x = decode(u, L, P.Ht);
+        for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
+            const Unit x = make_unit(ug, ut, L, P.Ht);
             const uint32_t buf = tcount & 1;
             // resolve the output row while the tile is still being computed
             const int tp = x.tile * kTileM + m;
@@ -670,10 +484,20 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         const int i0 = (lane % lanes_per_head) * PP;      // first rotary pair of this lane
         const int hs = P.ds >> 1;
         const int k0 = q * P.ds + i0, k1 = k0 + hs;       // A columns of the two halves
+        // Two heads per A row: the lanes of head 0 and head 1 rotate the same
+        // frequencies at the same positions, so each computes half and they swap.
+        const bool share = lanes_per_head == 16 && PP >= 2;
+        constexpr int kHalf = PP >= 2 ? PP / 2 : 1;
+        unsigned long long turn[PP];
+#pragma unroll
+        for (int e = 0; e < PP; ++e) {
+            const int f = share ? i0 + (q * kHalf + e) % PP : i0 + e;   // share: first kHalf entries are own
+            turn[e] = sTurnS[f];
+        }
         uint32_t sub = 0, tcount = 0;
         bool ok = true;
-        for (long long u = u_begin; u < u_end && ok; ++u) {
-            const Unit x = decode(u, L, P.Ht);
+        for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count && ok; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
+            const Unit x = make_unit(ug, ut, L, P.Ht);
             const bool rot = x.kv == 0 && P.rs.enabled;
             const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
             const int g = (P.r > 1 ? x.h * P.r : x.h / P.e) + q;
@@ -682,11 +506,13 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 const uint32_t slot = sub % kNumSlots;
                 if (!W.wait(bar(kBarSlotFull + slot), (sub / kNumSlots) & 1)) { ok = false; break; }
                 const SlotHdr hdr = sHdr[slot];
-                const uint8_t* ring = sRing + hdr.offset;
+                // heads of a staged sub-tile are 128 bytes off bank alignment (see producer)
+                const uint8_t* ring = sRing + hdr.offset + q * (hdr.rows * L.row_bytes + 128);
                 constexpr int kTok = kSub / kNumXfWarps;   // tokens of this warp in the sub-tile
                 SubMeta mt[kTok];
                 int n[kTok];
                 int maxn = 0;
+                bool copy_only = !rot;
 #pragma unroll
                 for (int u4 = 0; u4 < kTok; ++u4) {
                     const int tt = tw + u4 * kNumXfWarps;
@@ -694,37 +520,81 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     const bool valid = x.tile * kTileM + sq * kSub + tt < P.T_total;
                     n[u4] = valid ? max(mt[u4].hi - mt[u4].lo, 0) : -1;
                     maxn = max(maxn, n[u4]);
+                    copy_only = copy_only && n[u4] <= 1 && mt[u4].stage_row >= 0;
                 }
-                float a0[kTok][PP], a1[kTok][PP];
-#pragma unroll
-                for (int u4 = 0; u4 < kTok; ++u4)
-#pragma unroll
-                    for (int e = 0; e < PP; ++e) { a0[u4][e] = 0.f; a1[u4][e] = 0.f; }
-                for (int o = 0; o < maxn; ++o) {
-                    typename Raw<PP>::T w0[kTok], w1[kTok];
+                if (copy_only) {
+                    // V rows with single-token spans: the A row is the source row itself
 #pragma unroll
                     for (int u4 = 0; u4 < kTok; ++u4) {
-                        if (o < n[u4]) {
-                            const int srow = mt[u4].lo + o;
-                            const __nv_bfloat16* rp;
-                            if (mt[u4].stage_row >= 0)
-                                rp = reinterpret_cast<const __nv_bfloat16*>(
-                                    ring + ((size_t)q * hdr.rows + (size_t)(mt[u4].stage_row + o)) * L.row_bytes);
-                            else
-                                rp = src + (long long)mt[u4].b * P.sb + (long long)g * P.sh + (long long)srow * P.ss;
-                            w0[u4] = load_raw<PP>(rp + i0);
-                            w1[u4] = load_raw<PP>(rp + hs + i0);
+                        const int row = sq * kSub + tw + u4 * kNumXfWarps;
+                        if (n[u4] < 0) continue;
+                        typename Raw<PP>::T w0, w1;
+                        if (n[u4] == 1) {
+                            const __nv_bfloat16* rp =
+                                reinterpret_cast<const __nv_bfloat16*>(ring + (size_t)mt[u4].stage_row * L.row_bytes);
+                            w0 = load_raw<PP>(rp + i0);
+                            w1 = load_raw<PP>(rp + hs + i0);
+                        } else {
+                            w0 = typename Raw<PP>::T{};
+                            w1 = typename Raw<PP>::T{};
                         }
+                        *reinterpret_cast<typename Raw<PP>::T*>(sA + sw128_off(row, k0, kTileM)) = w0;
+                        *reinterpret_cast<typename Raw<PP>::T*>(sA + sw128_off(row, k1, kTileM)) = w1;
                     }
+                } else {
+                    float a0[kTok][PP], a1[kTok][PP];
 #pragma unroll
-                    for (int u4 = 0; u4 < kTok; ++u4) {
-                        if (o < n[u4]) {
+                    for (int u4 = 0; u4 < kTok; ++u4)
+#pragma unroll
+                        for (int e = 0; e < PP; ++e) { a0[u4][e] = 0.f; a1[u4][e] = 0.f; }
+                    for (int o = 0; o < maxn; ++o) {
+                        typename Raw<PP>::T w0[kTok], w1[kTok];
+#pragma unroll
+                        for (int u4 = 0; u4 < kTok; ++u4) {
+                            if (o < n[u4]) {
+                                const int srow = mt[u4].lo + o;
+                                const __nv_bfloat16* rp;
+                                if (mt[u4].stage_row >= 0)
+                                    rp = reinterpret_cast<const __nv_bfloat16*>(
+                                        ring + (size_t)(mt[u4].stage_row + o) * L.row_bytes);
+                                else
+                                    rp = src + (long long)mt[u4].b * P.sb + (long long)g * P.sh +
+                                         (long long)srow * P.ss;
+                                w0[u4] = load_raw<PP>(rp + i0);
+                                w1[u4] = load_raw<PP>(rp + hs + i0);
+                            }
+                        }
+#pragma unroll
+                        for (int u4 = 0; u4 < kTok; ++u4) {
+                            // rows beyond a token's span leave its sums untouched; the sine/cosine
+                            // exchange below is warp-wide, so every lane takes part
+                            const bool act = o < n[u4];
                             float x0[PP], x1[PP];
                             unpack(w0[u4], x0);
                             unpack(w1[u4], x1);
                             if (rot) {
+                                const int pos = act ? src_pos_of(P, mt[u4].b, mt[u4].lo + o) : 0;
                                 float2 cs[PP];
-                                rope_cs_vec<PP>(sTurnS, src_pos_of(P, mt[u4].b, mt[u4].lo + o), i0, cs);
+                                if (share) {
+#pragma unroll
+                                    for (int e = 0; e < kHalf; ++e) cs[e] = turn_cs(turn[e], pos);
+#pragma unroll
+                                    for (int e = 0; e < kHalf; ++e) {
+                                        cs[kHalf + e].x = __shfl_xor_sync(0xffffffffu, cs[e].x, 16);
+                                        cs[kHalf + e].y = __shfl_xor_sync(0xffffffffu, cs[e].y, 16);
+                                    }
+                                    if (q) {   // own entries are the second half of the lane's pairs
+#pragma unroll
+                                        for (int e = 0; e < kHalf; ++e) {
+                                            const float2 t = cs[e];
+                                            cs[e] = cs[kHalf + e];
+                                            cs[kHalf + e] = t;
+                                        }
+                                    }
+                                } else {
+#pragma unroll
+                                    for (int e = 0; e < PP; ++e) cs[e] = turn_cs(turn[e], pos);
+                                }
 #pragma unroll
                                 for (int e = 0; e < PP; ++e) {
                                     // undo the rotation: R(-theta)
@@ -734,24 +604,26 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                                     x1[e] = u1;
                                 }
                             }
+                            if (act) {
 #pragma unroll
-                            for (int e = 0; e < PP; ++e) { a0[u4][e] += x0[e]; a1[u4][e] += x1[e]; }
+                                for (int e = 0; e < PP; ++e) { a0[u4][e] += x0[e]; a1[u4][e] += x1[e]; }
+                            }
                         }
                     }
-                }
 #pragma unroll
-                for (int u4 = 0; u4 < kTok; ++u4) {
-                    if (n[u4] < 0) continue;
-                    const int row = sq * kSub + tw + u4 * kNumXfWarps;
-                    // span mean; 1/n is exact for n = 1, 2 (the common spans)
-                    const float inv_n = n[u4] > 0 ? __frcp_rn((float)n[u4]) : 0.f;
+                    for (int u4 = 0; u4 < kTok; ++u4) {
+                        if (n[u4] < 0) continue;
+                        const int row = sq * kSub + tw + u4 * kNumXfWarps;
+                        // span mean; 1/n is exact for n = 1, 2 (the common spans)
+                        const float inv_n = n[u4] > 0 ? __frcp_rn((float)n[u4]) : 0.f;
 #pragma unroll
-                    for (int e = 0; e < PP; ++e) {
-                        a0[u4][e] *= inv_n;
-                        a1[u4][e] *= inv_n;
+                        for (int e = 0; e < PP; ++e) {
+                            a0[u4][e] *= inv_n;
+                            a1[u4][e] *= inv_n;
+                        }
+                        store_bf16_smem<PP>(sA + sw128_off(row, k0, kTileM), a0[u4]);
+                        store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1[u4]);
                     }
-                    store_bf16_smem<PP>(sA + sw128_off(row, k0, kTileM), a0[u4]);
-                    store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1[u4]);
                 }
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(kBarSlotEmpty + slot));
@@ -852,7 +724,7 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
     L.off_ring = (off + 127) / 128 * 128;
     const int avail = kSmemMax - 1024 - (int)L.off_ring;   // 1024: alignment slack of the dynamic base
     L.ring_bytes = avail > 0 ? (unsigned)(avail / 1024 * 1024) : 0;
-    if (L.ring_bytes < 3u * kSub * (unsigned)(in_dim / ds) * L.row_bytes) return false;   // one worst sub-tile
+    if (L.ring_bytes < (3u * kSub * L.row_bytes + 128u) * (unsigned)(in_dim / ds)) return false;   // one worst sub-tile
     L.idesc = make_idesc(kTileM, L.n_tile);
     unsigned cols = 32;
     while (cols < 2u * (unsigned)L.n_tile) cols <<= 1;

@@ -1,0 +1,595 @@
+// kvx_tc_aligned.cu -- tensor-core translation kernel for identity token alignment.
+//
+// When the source and target tokenisations coincide (span of target token t is
+// source token t, the within-family handoff of paper Section 6.2), the A operand
+// of the projection is the source cache itself: row t of the tile is the
+// concatenation of the grouped source heads at token t, un-rotated for K.  The
+// kernel therefore loads A straight into the UMMA K-major 128-byte-swizzled
+// layout with tensor-TMA boxes (one box = [128 tokens x 64 channels] of one
+// head = one K-block of A), un-rotates K tiles in place, and feeds the tensor
+// core from those buffers.  V tiles need no prologue work at all.
+//
+// Persistent, one CTA per SM.  Work unit = (group, tile) with group = (target
+// layer j, target head h, K|V, output split nt) and tiles of 128 tokens laid
+// per sequence.  K-blocks stream through a ring of NS slots:
+//   warp 0 (lane 0)  producer: B image per group (bulk copy), A K-blocks (tensor TMA)
+//   warp 1           MMA: TMEM allocation, tcgen05.mma per K-block, commits
+//   warps 2-5        epilogue: TMEM -> target RoPE -> bf16 -> cache (bulk stores)
+//   warps 6-13       prologue: in-place source-RoPE undo of K tiles
+// Every wait is bounded (~1 s, then KVX_DEV_WAIT_TIMEOUT and a drained exit).
+#include <cuda.h>
+#include <stddef.h>
+#include <string.h>
+
+#include "kvx_common.cuh"
+#include "kvx_kernels.h"
+#include "kvx_tc_common.cuh"
+
+namespace kvx {
+namespace {
+
+constexpr int kTileM = 128;
+constexpr int kBlockK = 64;                       // channels per K-block (one 128-byte swizzle row)
+constexpr int kBlockBytes = kTileM * kBlockK * 2;  // 16 KB
+constexpr int kMaxSlots = 16;
+constexpr int kProducerWarp = 0;
+constexpr int kMmaWarp = 1;
+constexpr int kEpiWarp0 = 2;
+constexpr int kNumEpiWarps = 4;
+constexpr int kXfWarp0 = 6;
+constexpr int kNumXfWarps = 8;
+constexpr int kXfThreads = kNumXfWarps * 32;
+constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
+
+// barrier indices
+constexpr int kBarBFull = 0, kBarBEmpty = 1;
+constexpr int kBarDFull = 2;                        // +buf (2)
+constexpr int kBarDEmpty = 4;                       // +buf (2)
+constexpr int kBarFull = 6;                         // +slot: TMA landed
+constexpr int kBarEmpty = kBarFull + kMaxSlots;     // +slot: MMA done with it
+// +(K tile % nkready): every K-block of that K tile has been un-rotated.  At most
+// nslots/nblk + 1 K tiles sit between "rotated" and "consumed by the MMA" (the
+// slot ring bounds it), so a ring of nkready = nslots/nblk + 2 barriers never
+// completes one twice before the MMA has waited on it.
+constexpr int kBarKReady = kBarEmpty + kMaxSlots;
+constexpr int kMaxKReady = kMaxSlots + 2;
+constexpr int kNumBars = kBarKReady + kMaxKReady;
+
+struct AlignedParams {
+    // geometry
+    int Hs, ds, Ht, dt, in_dim, r, e, Lt;
+    int n_tile, n_split, groups, nblk, nslots, nkready, m_tiles_max;
+    // source
+    int batch, src_max_seq;
+    const int* src_seq_len;
+    const int* src_pos;
+    // target
+    int T_total;
+    const int* seq_off;
+    const int* tgt_pos;
+    int paged, dst_max_seq;
+    long long db, dh, dts;
+    const int* page_table;
+    int max_pages, page_size, num_pages;
+    RopeTable rs, rt;
+    int max_position;
+    unsigned* status;
+    const void* w;
+    unsigned idesc, tmem_cols, b_bytes, stage_row_bytes;
+    unsigned off_b, off_ring, off_stage, off_bar, off_misc, off_seq, off_turns;
+    void* dst_k[KVX_MAX_ALIGNED_LAYERS];
+    void* dst_v[KVX_MAX_ALIGNED_LAYERS];
+    CUtensorMap maps[2 * KVX_MAX_ALIGNED_LAYERS];   // [j*2 + kv]: source K/V of target layer j
+};
+
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
+                                            uint32_t bar, uint64_t pol)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.L2::cache_hint"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6], %7;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar), "l"(pol)
+        : "memory");
+}
+
+static_assert(sizeof(AlignedParams) <= 32764, "kernel parameter space");
+
+struct AUnit {
+    int j, h, kv, nt, g;
+    int b, t0, rows;   // sequence, first token, valid rows (0: no such tile)
+};
+
+// tile index k -> (sequence, first token); tiles are laid per sequence
+__device__ __forceinline__ AUnit make_aunit(int g, int k, const AlignedParams& P, const int* tile_off,
+                                            const int* seq_off, int batch)
+{
+    AUnit x;
+    x.g = g;
+    int rest = g;
+    x.nt = rest % P.n_split;
+    rest /= P.n_split;
+    x.kv = rest & 1;
+    rest >>= 1;
+    x.h = rest % P.Ht;
+    x.j = rest / P.Ht;
+    if (k >= tile_off[batch]) { x.b = 0; x.t0 = 0; x.rows = 0; return x; }
+    int lo = 0, hi = batch - 1;
+    while (lo < hi) {
+        const int mid = (lo + hi + 1) >> 1;
+        if (tile_off[mid] <= k) lo = mid; else hi = mid - 1;
+    }
+    x.b = lo;
+    x.t0 = (k - tile_off[lo]) * kTileM;
+    const int T = seq_off[lo + 1] - seq_off[lo];
+    x.rows = min(kTileM, T - x.t0);
+    return x;
+}
+
+template <int HS>   // half head_dim of the source (32, 64 or 128)
+__global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const __grid_constant__ AlignedParams P)
+{
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    uint8_t* sB = smem + P.off_b;
+    uint8_t* sRing = smem + P.off_ring;
+    uint8_t* sStage = smem + P.off_stage;
+    uint64_t* sBar = reinterpret_cast<uint64_t*>(smem + P.off_bar);
+    volatile int* sAbort = reinterpret_cast<volatile int*>(smem + P.off_misc);
+    uint32_t* sTmemBase = reinterpret_cast<uint32_t*>(smem + P.off_misc + 4);
+    int* sSeqOff = reinterpret_cast<int*>(smem + P.off_seq);            // [batch+1]
+    int* sSrcLen = sSeqOff + (P.batch + 1);                              // [batch]
+    int* sTileOff = sSrcLen + P.batch;                                   // [batch+1]
+    unsigned long long* sTurnS = reinterpret_cast<unsigned long long*>(smem + P.off_turns);
+    unsigned long long* sTurnT = sTurnS + HS;
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    auto bar = [&](int i) { return (uint32_t)__cvta_generic_to_shared(&sBar[i]); };
+
+    for (int i = threadIdx.x; i <= P.batch; i += blockDim.x) sSeqOff[i] = __ldg(&P.seq_off[i]);
+    for (int i = threadIdx.x; i < P.batch; i += blockDim.x) sSrcLen[i] = __ldg(&P.src_seq_len[i]);
+    for (int i = threadIdx.x; i < HS; i += blockDim.x) sTurnS[i] = P.rs.enabled ? __ldg(&P.rs.turns[i]) : 0ull;
+    for (int i = threadIdx.x; i < (P.dt >> 1); i += blockDim.x)
+        sTurnT[i] = P.rt.enabled ? __ldg(&P.rt.turns[i]) : 0ull;
+    if (threadIdx.x == 0) {
+        *sAbort = 0;
+        mbar_init(bar(kBarBFull), 1);
+        mbar_init(bar(kBarBEmpty), 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(kBarDFull + i), 1);
+            mbar_init(bar(kBarDEmpty + i), kNumEpiWarps);
+        }
+        for (int i = 0; i < P.nslots; ++i) {
+            mbar_init(bar(kBarFull + i), 1);
+            mbar_init(bar(kBarEmpty + i), 2);   // the MMA's commit and the prologue's release
+        }
+        for (int i = 0; i < P.nkready; ++i) mbar_init(bar(kBarKReady + i), kNumXfWarps);
+        fence_mbar_init();
+    }
+    if (warp == kMmaWarp) {
+        tmem_alloc((uint32_t)__cvta_generic_to_shared(sTmemBase), P.tmem_cols);
+        tmem_relinquish();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {   // per-sequence tile offsets
+        int acc = 0;
+        for (int b = 0; b < P.batch; ++b) {
+            sTileOff[b] = acc;
+            const int T = sSeqOff[b + 1] - sSeqOff[b];
+            acc += T > 0 ? (T + kTileM - 1) / kTileM : 0;
+        }
+        sTileOff[P.batch] = acc;
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_base = *sTmemBase;
+
+    const Waiter W{sAbort, P.status};
+    const long long U = (long long)P.groups * P.m_tiles_max;
+    const long long ub = (long long)blockIdx.x * U / gridDim.x;
+    const long long ue = (long long)(blockIdx.x + 1) * U / gridDim.x;
+    const int count = (int)(ue - ub);
+    const int g_begin = (int)(ub / P.m_tiles_max);
+    const int k_begin = (int)(ub - (long long)g_begin * P.m_tiles_max);
+    const int blk_per_head = (2 * HS) / kBlockK;       // K-blocks of one source head
+    const int hw = P.n_tile >> 1;
+
+#define KVX_FOR_UNITS                                                                                   \
+    for (int it = 0, ug = g_begin, uk = k_begin; it < count; ++it, (++uk == P.m_tiles_max ? (uk = 0, ++ug) : 0))
+
+    if (warp == kProducerWarp) {
+        // ------------------------------------------------------------ producer (one thread)
+        if (lane == 0) {
+            const uint64_t pol_stream = policy_evict_first();
+            const uint64_t pol_keep = policy_evict_last();
+            int cur_g = -1;
+            uint32_t b_loads = 0, slot_cnt = 0;
+            bool ok = true;
+            KVX_FOR_UNITS {
+                const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+                if (x.rows <= 0) continue;
+                if (x.g != cur_g) {
+                    if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
+                    mbar_arrive_expect_tx(bar(kBarBFull), P.b_bytes);
+                    const uint8_t* img = (const uint8_t*)P.w + (size_t)x.g * P.b_bytes;
+                    const uint32_t piece = P.b_bytes / 4;
+                    for (int q = 0; q < 4; ++q)
+                        bulk_g2s((uint32_t)__cvta_generic_to_shared(sB) + q * piece, img + (size_t)q * piece, piece,
+                                 bar(kBarBFull), pol_keep);
+                    ++b_loads;
+                    cur_g = x.g;
+                }
+                const CUtensorMap* map = &P.maps[x.j * 2 + x.kv];
+                const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
+                for (int kb = 0; kb < P.nblk; ++kb) {
+                    const uint32_t slot = slot_cnt % P.nslots;
+                    if (!W.wait(bar(kBarEmpty + slot), ((slot_cnt / P.nslots) & 1) ^ 1)) { ok = false; break; }
+                    mbar_arrive_expect_tx(bar(kBarFull + slot), kBlockBytes);
+                    tma_load_4d((uint32_t)__cvta_generic_to_shared(sRing) + slot * kBlockBytes, map,
+                                (kb % blk_per_head) * kBlockK, x.t0, g0 + kb / blk_per_head, x.b,
+                                bar(kBarFull + slot), pol_stream);
+                    ++slot_cnt;
+                }
+                if (!ok) break;
+            }
+            if (*sAbort) {   // let copies in flight land before leaving
+                const unsigned long long t0 = globaltimer();
+                for (uint32_t c = slot_cnt > (uint32_t)P.nslots ? slot_cnt - P.nslots : 0; c < slot_cnt; ++c)
+                    while (!mbar_try_wait(bar(kBarFull + c % P.nslots), (c / P.nslots) & 1) &&
+                           globaltimer() - t0 < kWaitNs) {}
+                if (b_loads)
+                    while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < kWaitNs) {}
+            }
+        }
+        __syncwarp();
+    } else if (warp == kMmaWarp) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            int cur_g = -1;
+            uint32_t b_cnt = 0, tcount = 0, slot_cnt = 0, kcount = 0;
+            bool ok = true;
+            KVX_FOR_UNITS {
+                const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+                if (x.rows <= 0) continue;
+                if (x.g != cur_g) {
+                    if (!W.wait(bar(kBarBFull), b_cnt & 1)) break;
+                    ++b_cnt;
+                    cur_g = x.g;
+                }
+                const bool rot = x.kv == 0 && P.rs.enabled;
+                const uint32_t buf = tcount & 1;
+                if (!W.wait(bar(kBarDEmpty + buf), ((tcount >> 1) & 1) ^ 1)) break;
+                const uint32_t d = tmem_base + buf * (uint32_t)P.n_tile;
+                const uint32_t b0 = (uint32_t)__cvta_generic_to_shared(sB);
+                if (rot) {   // K tile: wait until the prologue has un-rotated all its K-blocks
+                    if (!W.wait(bar(kBarKReady + kcount % P.nkready), (kcount / P.nkready) & 1)) break;
+                    ++kcount;
+                }
+                for (int kb = 0; kb < P.nblk; ++kb) {
+                    const uint32_t slot = slot_cnt % P.nslots;
+                    const uint32_t par = (slot_cnt / P.nslots) & 1;
+                    if (!rot && !W.wait(bar(kBarFull + slot), par)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a0 = (uint32_t)__cvta_generic_to_shared(sRing) + slot * kBlockBytes;
+#pragma unroll
+                    for (int kk = 0; kk < kBlockK / 16; ++kk) {
+                        const uint64_t ad = sw128_desc(a0 + kk * 32);
+                        const uint64_t bd = sw128_desc(b0 + kb * (P.n_tile * 128) + kk * 32);
+                        umma_bf16(d, ad, bd, P.idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    umma_commit(bar(kBarEmpty + slot));
+                    ++slot_cnt;
+                }
+                if (!ok) break;
+                umma_commit(bar(kBarDFull + buf));
+                // the last valid tile of this group in the CTA's range releases B
+                bool last = true;
+                {
+                    int g2 = ug, k2 = uk;
+                    for (int it2 = it + 1; it2 < count; ++it2) {
+                        if (++k2 == P.m_tiles_max) { k2 = 0; ++g2; }
+                        if (g2 != ug) break;
+                        if (k2 < sTileOff[P.batch]) { last = false; break; }
+                    }
+                }
+                if (last) umma_commit(bar(kBarBEmpty));
+                ++tcount;
+            }
+        }
+        __syncwarp();
+    } else if (warp < kEpiWarp0 + kNumEpiWarps) {
+        // ------------------------------------------------------------ epilogue
+        const int quad = warp & 3;
+        const int m = quad * 32 + lane;
+        uint8_t* srow = sStage + (size_t)m * P.stage_row_bytes;
+        const uint32_t srow_u32 = (uint32_t)__cvta_generic_to_shared(srow);
+        uint32_t tcount = 0;
+        KVX_FOR_UNITS {
+            const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+            if (x.rows <= 0) continue;
+            const uint32_t buf = tcount & 1;
+            // output row of this thread, resolved while the tile is computed
+            const int t = x.t0 + m;
+            bool valid = m < x.rows;
+            long long dst_off = -1;
+            int pt = 0;
+            if (valid) {
+                int S = sSrcLen[x.b];
+                if (S > P.src_max_seq) S = P.src_max_seq;
+                if (t >= S) { set_status(P.status, KVX_DEV_SPAN_CLAMPED); valid = false; }
+                const int p = P.tgt_pos ? __ldg(&P.tgt_pos[sSeqOff[x.b] + t]) : t;
+                pt = P.rt.enabled ? clamp_pos(p, P.max_position, P.status) : 0;
+                if (!P.paged) {
+                    if (t >= P.dst_max_seq) { set_status(P.status, KVX_DEV_SEQ_CLAMPED); valid = false; }
+                    else dst_off = (long long)x.b * P.db + (long long)t * P.dts;
+                } else {
+                    const int pi = t / P.page_size;
+                    const int page = pi < P.max_pages ? __ldg(&P.page_table[(size_t)x.b * P.max_pages + pi]) : -1;
+                    if (page < 0 || page >= P.num_pages) { set_status(P.status, KVX_DEV_PAGE_INVALID); valid = false; }
+                    else dst_off = ((long long)page * P.page_size + (t % P.page_size)) * (long long)P.Ht * P.dt;
+                }
+            }
+            const bool rot = x.kv == 0 && P.rt.enabled;
+            if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
+            tc_fence_after();
+            bulk_wait_read0();
+            const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)P.n_tile;
+            for (int pc = 0; pc < hw; pc += 8) {
+                uint32_t r0[8], r1[8];
+                tmem_ld8(taddr + pc, r0);
+                tmem_ld8(taddr + hw + pc, r1);
+                float2 cs[8];
+                if (rot) {
+#pragma unroll
+                    for (int e2 = 0; e2 < 8; ++e2) cs[e2] = turn_cs(sTurnT[x.nt * hw + pc + e2], pt);
+                }
+                tmem_ld_wait();
+                float y0[8], y1[8];
+#pragma unroll
+                for (int e2 = 0; e2 < 8; ++e2) { y0[e2] = __uint_as_float(r0[e2]); y1[e2] = __uint_as_float(r1[e2]); }
+                if (rot) {
+#pragma unroll
+                    for (int e2 = 0; e2 < 8; ++e2) {
+                        const float a = y0[e2], bb = y1[e2];
+                        y0[e2] = fmaf(a, cs[e2].x, -bb * cs[e2].y);
+                        y1[e2] = fmaf(bb, cs[e2].x, a * cs[e2].y);
+                    }
+                }
+                *reinterpret_cast<uint4*>(srow + pc * 2) =
+                    make_uint4(pack_bf16(y0[0], y0[1]), pack_bf16(y0[2], y0[3]), pack_bf16(y0[4], y0[5]),
+                               pack_bf16(y0[6], y0[7]));
+                *reinterpret_cast<uint4*>(srow + (hw + pc) * 2) =
+                    make_uint4(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]), pack_bf16(y1[4], y1[5]),
+                               pack_bf16(y1[6], y1[7]));
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarDEmpty + buf));
+            if (valid && dst_off >= 0) {
+                fence_proxy_async();
+                __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
+                                     (P.paged ? (long long)x.h * P.dt : (long long)x.h * P.dh);
+                if (P.n_split == 1) {
+                    bulk_s2g(dst, srow_u32, (uint32_t)P.dt * 2);
+                } else {
+                    bulk_s2g(dst + x.nt * hw, srow_u32, (uint32_t)hw * 2);
+                    bulk_s2g(dst + (P.dt >> 1) + x.nt * hw, srow_u32 + hw * 2, (uint32_t)hw * 2);
+                }
+                bulk_commit();
+            }
+            ++tcount;
+        }
+        bulk_wait0();
+    } else {
+        // ------------------------------------------------------------ prologue: undo source RoPE in place
+        // Thread layout over a K tile: 2 threads per token row; each owns HS/2
+        // rotary pairs (i, i+HS) of every grouped head and computes each (cos, sin)
+        // once for all heads.  Pairs are handled 8 at a time (one 16-byte chunk of
+        // each half).  A thread visits its chunks in an order staggered by row so
+        // that the 8 threads of a shared-memory phase hit distinct bank groups.
+        const int xt = threadIdx.x - kXfWarp0 * 32;
+        const int heads = P.in_dim / (2 * HS);            // heads in one A row
+        constexpr int kChunks = HS / 8;                    // 16-byte chunks per half head
+        constexpr int kMine = kChunks / 2;                 // chunks per thread
+        uint32_t slot_cnt = 0, kcount = 0;
+        bool ok = true;
+        KVX_FOR_UNITS {
+            const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+            if (x.rows <= 0) continue;
+            const bool rot = x.kv == 0 && P.rs.enabled;
+            // Walk every slot use in order (V tiles too), so that each wait is at most
+            // one phase away from its barrier; the slot is refilled only after both
+            // this release and the MMA's commit.
+            for (int kb = 0; kb < P.nblk; ++kb) {
+                const uint32_t c = slot_cnt + kb;
+                if (!W.wait(bar(kBarFull + c % P.nslots), (c / P.nslots) & 1)) { ok = false; break; }
+            }
+            if (!ok) break;
+            if (!rot) {
+                if (xt == 0)
+                    for (int kb = 0; kb < P.nblk; ++kb) mbar_arrive(bar(kBarEmpty + (slot_cnt + kb) % P.nslots));
+                slot_cnt += P.nblk;
+                continue;
+            }
+            for (int pass = 0; pass < (2 * kTileM) / kXfThreads; ++pass) {
+                const int row = (pass * kXfThreads + xt) >> 1;
+                const int part = xt & 1;
+                if (row >= x.rows) continue;
+                const int t = x.t0 + row;
+                const int p = src_pos_of_seq(P.src_pos, P.src_max_seq, x.b, t, P.max_position, P.status);
+#pragma unroll
+                for (int cc = 0; cc < kMine; ++cc) {
+                    const int c = part * kMine + ((cc + (row >> 2)) % kMine);   // staggered chunk
+                    const int i = c * 8;                                        // first pair index
+                    float2 cs[8];
+#pragma unroll
+                    for (int e2 = 0; e2 < 8; ++e2) cs[e2] = turn_cs(sTurnS[i + e2], p);
+                    for (int q = 0; q < heads; ++q) {
+                        // element i (and i+HS) of head q: K-block and column within it
+                        const int k_lo = q * 2 * HS + i, k_hi = k_lo + HS;
+                        const uint32_t s_lo = (slot_cnt + (k_lo >> 6)) % P.nslots;
+                        const uint32_t s_hi = (slot_cnt + (k_hi >> 6)) % P.nslots;
+                        uint8_t* p_lo = sRing + s_lo * kBlockBytes + sw128_off(row, k_lo & 63, kTileM);
+                        uint8_t* p_hi = sRing + s_hi * kBlockBytes + sw128_off(row, k_hi & 63, kTileM);
+                        const uint4 wl = *reinterpret_cast<const uint4*>(p_lo);
+                        const uint4 wh = *reinterpret_cast<const uint4*>(p_hi);
+                        const uint32_t al[4] = {wl.x, wl.y, wl.z, wl.w};
+                        const uint32_t ah[4] = {wh.x, wh.y, wh.z, wh.w};
+                        uint32_t ol[4], oh[4];
+#pragma unroll
+                        for (int w2 = 0; w2 < 4; ++w2) {
+                            float x0a = bf_lo(al[w2]), x0b = bf_hi(al[w2]);
+                            float x1a = bf_lo(ah[w2]), x1b = bf_hi(ah[w2]);
+                            const float2 ca = cs[2 * w2], cb = cs[2 * w2 + 1];
+                            // undo the rotation: R(-theta)
+                            const float u0a = fmaf(x0a, ca.x, x1a * ca.y), u1a = fmaf(x1a, ca.x, -x0a * ca.y);
+                            const float u0b = fmaf(x0b, cb.x, x1b * cb.y), u1b = fmaf(x1b, cb.x, -x0b * cb.y);
+                            ol[w2] = pack_bf16(u0a, u0b);
+                            oh[w2] = pack_bf16(u1a, u1b);
+                        }
+                        *reinterpret_cast<uint4*>(p_lo) = make_uint4(ol[0], ol[1], ol[2], ol[3]);
+                        *reinterpret_cast<uint4*>(p_hi) = make_uint4(oh[0], oh[1], oh[2], oh[3]);
+                    }
+                }
+            }
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarKReady + kcount % P.nkready));
+            // the MMA's commit (after every prologue warp's "ready") completes the release
+            if (xt == 0)
+                for (int kb = 0; kb < P.nblk; ++kb) mbar_arrive(bar(kBarEmpty + (slot_cnt + kb) % P.nslots));
+            ++kcount;
+            slot_cnt += P.nblk;
+        }
+    }
+#undef KVX_FOR_UNITS
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == kMmaWarp) {
+        tc_fence_after();
+        tmem_dealloc(tmem_base, P.tmem_cols);
+    }
+}
+
+using EncodeTiled = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                 const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encoder()
+{
+    static EncodeTiled fn = nullptr;
+    static bool tried = false;
+    if (!tried) {
+        tried = true;
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = (EncodeTiled)p;
+    }
+    return fn;
+}
+
+}  // namespace
+
+bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch)
+{
+    TcConfig c = tc_config(in_dim, dt, ds);
+    return c.ok && Lt <= KVX_MAX_ALIGNED_LAYERS && batch <= KVX_MAX_ALIGNED_BATCH && encoder() != nullptr;
+}
+
+bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int Hs, int batch, long long ss,
+                       long long sh, long long sb)
+{
+    EncodeTiled enc = encoder();
+    if (!enc) return false;
+    const cuuint64_t dims[4] = {(cuuint64_t)ds, (cuuint64_t)(S_max > 0 ? S_max : 1), (cuuint64_t)Hs,
+                                (cuuint64_t)batch};
+    const cuuint64_t strides[3] = {(cuuint64_t)ss * 2, (cuuint64_t)sh * 2, (cuuint64_t)sb * 2};
+    const cuuint32_t box[4] = {(cuuint32_t)kBlockK, (cuuint32_t)kTileM, 1, 1};
+    const cuuint32_t estr[4] = {1, 1, 1, 1};
+    return enc(reinterpret_cast<CUtensorMap*>(map_out), CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base),
+               dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+size_t aligned_map_bytes() { return sizeof(CUtensorMap); }
+
+cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps, int num_sms,
+                                        cudaStream_t stream)
+{
+    TcConfig cfg = tc_config(T.in_dim, T.dt, T.ds);
+    if (!cfg.ok || T.Lt > KVX_MAX_ALIGNED_LAYERS || T.batch > KVX_MAX_ALIGNED_BATCH) return cudaErrorNotSupported;
+    static thread_local AlignedParams P;   // large (~27 KB): filled on the host, passed by value
+    memset(&P, 0, offsetof(AlignedParams, maps));
+    P.Hs = T.Hs; P.ds = T.ds; P.Ht = T.Ht; P.dt = T.dt; P.in_dim = T.in_dim; P.r = T.r; P.e = T.e; P.Lt = T.Lt;
+    P.n_tile = cfg.n_tile;
+    P.n_split = cfg.n_split;
+    P.groups = T.Lt * T.Ht * 2 * cfg.n_split;
+    P.nblk = T.in_dim / kBlockK;
+    P.m_tiles_max = (T.T_total + kTileM - 1) / kTileM + T.batch - 1;
+    P.batch = T.batch; P.src_max_seq = T.src_max_seq; P.src_seq_len = T.src_seq_len; P.src_pos = T.src_pos;
+    P.T_total = T.T_total; P.seq_off = T.seq_off; P.tgt_pos = T.tgt_pos;
+    P.paged = T.paged; P.dst_max_seq = T.dst_max_seq; P.db = T.db; P.dh = T.dh; P.dts = T.dts;
+    P.page_table = T.page_table; P.max_pages = T.max_pages; P.page_size = T.page_size; P.num_pages = T.num_pages;
+    P.rs = T.rs; P.rt = T.rt; P.max_position = T.max_position; P.status = T.status; P.w = T.w;
+    P.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(P.n_tile >> 3) << 17) | ((uint32_t)(kTileM >> 4) << 24);
+    unsigned cols = 32;
+    while (cols < 2u * (unsigned)P.n_tile) cols <<= 1;
+    P.tmem_cols = cols;
+    P.b_bytes = (unsigned)(T.in_dim * P.n_tile * 2);
+    P.stage_row_bytes = (unsigned)(P.n_tile * 2 + 16);
+    unsigned off = 0;
+    auto take = [&](unsigned bytes, unsigned align) {
+        off = (off + align - 1) / align * align;
+        const unsigned o = off;
+        off += bytes;
+        return o;
+    };
+    P.off_b = take(P.b_bytes, 1024);
+    P.off_stage = take(kTileM * P.stage_row_bytes, 128);
+    P.off_bar = take(kNumBars * 8, 8);
+    P.off_misc = take(16, 16);
+    P.off_seq = take((unsigned)(3 * T.batch + 2) * 4, 16);
+    P.off_turns = take((unsigned)(T.ds / 2 + T.dt / 2) * 8, 16);
+    P.off_ring = take(0, 1024);
+    const int avail = kSmemMax - 1024 - (int)P.off_ring;
+    P.nslots = avail / kBlockBytes;
+    if (P.nslots > kMaxSlots) P.nslots = kMaxSlots;
+    if (P.nslots < P.nblk) return cudaErrorNotSupported;
+    P.nkready = P.nslots / P.nblk + 2;
+    for (int j = 0; j < T.Lt; ++j) {
+        P.dst_k[j] = T.dst_k[j];
+        P.dst_v[j] = T.dst_v[j];
+        memcpy(&P.maps[2 * j], maps[2 * j], sizeof(CUtensorMap));
+        memcpy(&P.maps[2 * j + 1], maps[2 * j + 1], sizeof(CUtensorMap));
+    }
+    const long long U = (long long)P.groups * P.m_tiles_max;
+    const int grid = (int)(U < num_sms ? U : num_sms);
+    cudaError_t err;
+    switch (T.ds) {
+    case 64:
+        err = cudaFuncSetAttribute(translate_tc_aligned_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+        if (err != cudaSuccess) return err;
+        translate_tc_aligned_kernel<32><<<grid, kThreads, kSmemMax, stream>>>(P);
+        break;
+    case 128:
+        err = cudaFuncSetAttribute(translate_tc_aligned_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+        if (err != cudaSuccess) return err;
+        translate_tc_aligned_kernel<64><<<grid, kThreads, kSmemMax, stream>>>(P);
+        break;
+    case 256:
+        err = cudaFuncSetAttribute(translate_tc_aligned_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+        if (err != cudaSuccess) return err;
+        translate_tc_aligned_kernel<128><<<grid, kThreads, kSmemMax, stream>>>(P);
+        break;
+    default:
+        return cudaErrorNotSupported;
+    }
+    return cudaGetLastError();
+}
+
+}  // namespace kvx

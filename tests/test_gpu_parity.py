@@ -213,3 +213,27 @@ def test_invalid_arguments_rejected_before_launch():
     with pytest.raises(kvx.KvxError) as e:
         kvx.Translator(bad, spec.dst, torch.zeros(1, device="cuda"), torch.zeros(1, device="cuda"))
     assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
+
+
+# ------------------------------------------------------------------ the two tensor-core kernels agree
+@pytest.mark.parametrize("base,Ls,Lt,lens", [("qwen7b_to_qwen1p5b_4k", 2, 2, [300, 5, 129]),
+                                             ("qwen1p5b_to_gemma2b_1k", 2, 2, [300]),
+                                             ("llama70b_to_qwen7b_8k", 3, 2, [257])])
+def test_identity_kernel_equals_span_kernel(base, Ls, Lt, lens):
+    """Identity alignment (no span arrays) runs the tensor-TMA kernel; the same
+    spans given explicitly run the span-gather kernel.  Same arithmetic: equal bits."""
+    from gpu_harness import i32
+    spec = _shrink(SPECS[base], Ls, Lt, cross_tokenizer=False)
+    c = make_case(spec, lens)
+    ga = _run(c, kvx.KVX_PATH_AUTO)
+    from gpu_harness import GpuRun
+    gs = GpuRun(c, path=kvx.KVX_PATH_AUTO)
+    lo = np.concatenate([np.arange(t, dtype=np.int32) for t in lens])
+    gs.span_lo, gs.span_hi = i32(lo), i32(lo + 1)
+    gs.run()
+    torch.cuda.synchronize()
+    ak, av = ga.gather()
+    sk, sv = gs.gather()
+    np.testing.assert_array_equal(ak, sk)
+    np.testing.assert_array_equal(av, sv)
+    assert ga.status() == 0 and gs.status() == 0
