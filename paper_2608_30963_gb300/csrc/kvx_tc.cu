@@ -771,21 +771,26 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
     const long long U = (long long)L.groups * L.m_tiles;
     const int grid = (int)(U < num_sms ? U : num_sms);
     const int pp = L.in_dim / 64;
-    cudaError_t err;
     switch (pp) {
     case 4:
-        err = cudaFuncSetAttribute(translate_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-        if (err != cudaSuccess) return err;
+        {
+            static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (once != cudaSuccess) return once;
+        }
         translate_tc_kernel<4><<<grid, kThreads, kSmemMax, stream>>>(P, L);
         break;
     case 2:
-        err = cudaFuncSetAttribute(translate_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-        if (err != cudaSuccess) return err;
+        {
+            static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (once != cudaSuccess) return once;
+        }
         translate_tc_kernel<2><<<grid, kThreads, kSmemMax, stream>>>(P, L);
         break;
     case 1:
-        err = cudaFuncSetAttribute(translate_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-        if (err != cudaSuccess) return err;
+        {
+            static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (once != cudaSuccess) return once;
+        }
         translate_tc_kernel<1><<<grid, kThreads, kSmemMax, stream>>>(P, L);
         break;
     default:

@@ -14,8 +14,9 @@
 // per sequence.  K-blocks stream through a ring of NS slots:
 //   warp 0 (lane 0)  producer: B image per group (bulk copy), A K-blocks (tensor TMA)
 //   warp 1           MMA: TMEM allocation, tcgen05.mma per K-block, commits
-//   warps 2-5        epilogue: TMEM -> target RoPE -> bf16 -> cache (bulk stores)
-//   warps 6-13       prologue: in-place source-RoPE undo of K tiles
+//   warps 2-9        epilogue: TMEM -> target RoPE -> bf16 -> cache (bulk stores);
+//                    two warps per TMEM lane quadrant, each taking half of the RoPE pairs
+//   warps 10-17      prologue: in-place source-RoPE undo of K tiles
 // Every wait is bounded (~1 s, then KVX_DEV_WAIT_TIMEOUT and a drained exit).
 #include <cuda.h>
 #include <stddef.h>
@@ -35,8 +36,8 @@ constexpr int kMaxSlots = 16;
 constexpr int kProducerWarp = 0;
 constexpr int kMmaWarp = 1;
 constexpr int kEpiWarp0 = 2;
-constexpr int kNumEpiWarps = 4;
-constexpr int kXfWarp0 = 6;
+constexpr int kNumEpiWarps = 8;                    // two per TMEM lane quadrant, splitting the columns
+constexpr int kXfWarp0 = kEpiWarp0 + kNumEpiWarps;
 constexpr int kNumXfWarps = 8;
 constexpr int kXfThreads = kNumXfWarps * 32;
 constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
@@ -53,7 +54,10 @@ constexpr int kBarEmpty = kBarFull + kMaxSlots;     // +slot: MMA done with it
 // completes one twice before the MMA has waited on it.
 constexpr int kBarKReady = kBarEmpty + kMaxSlots;
 constexpr int kMaxKReady = kMaxSlots + 2;
-constexpr int kNumBars = kBarKReady + kMaxKReady;
+// +quad*2 + {0,1}: the two epilogue warps of a TMEM lane quadrant meet here before
+// writing the shared staging rows (0) and before storing them (1)
+constexpr int kBarPair = kBarKReady + kMaxKReady;
+constexpr int kNumBars = kBarPair + 8;
 
 struct AlignedParams {
     // geometry
@@ -164,6 +168,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             mbar_init(bar(kBarEmpty + i), 2);   // the MMA's commit and the prologue's release
         }
         for (int i = 0; i < P.nkready; ++i) mbar_init(bar(kBarKReady + i), kNumXfWarps);
+        for (int i = 0; i < 8; ++i) mbar_init(bar(kBarPair + i), 2);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -186,17 +191,26 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     const uint32_t tmem_base = *sTmemBase;
 
     const Waiter W{sAbort, P.status};
-    const long long U = (long long)P.groups * P.m_tiles_max;
-    const long long ub = (long long)blockIdx.x * U / gridDim.x;
-    const long long ue = (long long)(blockIdx.x + 1) * U / gridDim.x;
-    const int count = (int)(ue - ub);
-    const int g_begin = (int)(ub / P.m_tiles_max);
-    const int k_begin = (int)(ub - (long long)g_begin * P.m_tiles_max);
+    // Work split: each CTA takes an equal share of the K units and of the V units
+    // (K units cost more: the source RoPE undo), K share first.  Within each share
+    // units run group-major, so a group's weight tile stays resident.
+    const int hgroups = P.groups / 2;                          // (j, h, nt) per K|V
+    const long long UH = (long long)hgroups * P.m_tiles_max;
+    const int u0 = (int)((long long)blockIdx.x * UH / gridDim.x);
+    const int u1 = (int)((long long)(blockIdx.x + 1) * UH / gridDim.x);
+    const int count = 2 * (u1 - u0);
+    // unit #it of this CTA -> (group, tile)
+    auto unit_at = [&](int it, int& g, int& k) {
+        const int kv = it >= (u1 - u0);
+        const int idx = u0 + (kv ? it - (u1 - u0) : it);
+        const int hg = idx / P.m_tiles_max;
+        k = idx - hg * P.m_tiles_max;
+        g = ((hg / P.n_split) * 2 + kv) * P.n_split + hg % P.n_split;
+    };
     const int blk_per_head = (2 * HS) / kBlockK;       // K-blocks of one source head
     const int hw = P.n_tile >> 1;
 
-#define KVX_FOR_UNITS                                                                                   \
-    for (int it = 0, ug = g_begin, uk = k_begin; it < count; ++it, (++uk == P.m_tiles_max ? (uk = 0, ++ug) : 0))
+#define KVX_FOR_UNITS for (int it = 0, ug = 0, uk = 0; it < count && (unit_at(it, ug, uk), true); ++it)
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------ producer (one thread)
@@ -286,9 +300,9 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 // the last valid tile of this group in the CTA's range releases B
                 bool last = true;
                 {
-                    int g2 = ug, k2 = uk;
                     for (int it2 = it + 1; it2 < count; ++it2) {
-                        if (++k2 == P.m_tiles_max) { k2 = 0; ++g2; }
+                        int g2, k2;
+                        unit_at(it2, g2, k2);
                         if (g2 != ug) break;
                         if (k2 < sTileOff[P.batch]) { last = false; break; }
                     }
@@ -301,7 +315,9 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     } else if (warp < kEpiWarp0 + kNumEpiWarps) {
         // ------------------------------------------------------------ epilogue
         const int quad = warp & 3;
+        const int half = (warp - kEpiWarp0) >> 2;          // which half of the RoPE pairs
         const int m = quad * 32 + lane;
+        const int pc_begin = half * (hw >> 1), pc_end = pc_begin + (hw >> 1);
         uint8_t* srow = sStage + (size_t)m * P.stage_row_bytes;
         const uint32_t srow_u32 = (uint32_t)__cvta_generic_to_shared(srow);
         uint32_t tcount = 0;
@@ -333,9 +349,14 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             const bool rot = x.kv == 0 && P.rt.enabled;
             if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
             tc_fence_after();
-            bulk_wait_read0();
+            // the staging row is shared by the two warps of this quadrant; the row's
+            // previous store (issued by the half-0 thread) must have read it
+            if (half == 0) bulk_wait_read0();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2));
+            if (!W.wait(bar(kBarPair + quad * 2), tcount & 1)) break;
             const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)P.n_tile;
-            for (int pc = 0; pc < hw; pc += 8) {
+            for (int pc = pc_begin; pc < pc_end; pc += 8) {
                 uint32_t r0[8], r1[8];
                 tmem_ld8(taddr + pc, r0);
                 tmem_ld8(taddr + hw + pc, r1);
@@ -366,8 +387,11 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarDEmpty + buf));
-            if (valid && dst_off >= 0) {
-                fence_proxy_async();
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2 + 1));
+            if (!W.wait(bar(kBarPair + quad * 2 + 1), tcount & 1)) break;
+            if (half == 0 && valid && dst_off >= 0) {
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      (P.paged ? (long long)x.h * P.dt : (long long)x.h * P.dh);
                 if (P.n_split == 1) {
@@ -567,23 +591,28 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
         memcpy(&P.maps[2 * j], maps[2 * j], sizeof(CUtensorMap));
         memcpy(&P.maps[2 * j + 1], maps[2 * j + 1], sizeof(CUtensorMap));
     }
-    const long long U = (long long)P.groups * P.m_tiles_max;
-    const int grid = (int)(U < num_sms ? U : num_sms);
-    cudaError_t err;
+    const long long UH = (long long)(P.groups / 2) * P.m_tiles_max;
+    const int grid = (int)(UH < num_sms ? UH : num_sms);
     switch (T.ds) {
     case 64:
-        err = cudaFuncSetAttribute(translate_tc_aligned_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-        if (err != cudaSuccess) return err;
+        {
+            static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (once != cudaSuccess) return once;
+        }
         translate_tc_aligned_kernel<32><<<grid, kThreads, kSmemMax, stream>>>(P);
         break;
     case 128:
-        err = cudaFuncSetAttribute(translate_tc_aligned_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-        if (err != cudaSuccess) return err;
+        {
+            static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (once != cudaSuccess) return once;
+        }
         translate_tc_aligned_kernel<64><<<grid, kThreads, kSmemMax, stream>>>(P);
         break;
     case 256:
-        err = cudaFuncSetAttribute(translate_tc_aligned_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-        if (err != cudaSuccess) return err;
+        {
+            static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+            if (once != cudaSuccess) return once;
+        }
         translate_tc_aligned_kernel<128><<<grid, kThreads, kSmemMax, stream>>>(P);
         break;
     default:
