@@ -103,31 +103,76 @@ struct AUnit {
     int b, t0, rows;   // sequence, first token, valid rows (0: no such tile)
 };
 
-// tile index k -> (sequence, first token); tiles are laid per sequence
-__device__ __forceinline__ AUnit make_aunit(int g, int k, const AlignedParams& P, const int* tile_off,
-                                            const int* seq_off, int batch)
-{
+// Iterates a CTA's units in order with counters only (no divisions per unit):
+// its share of K units, then its share of V units; each share group-major.
+struct Walker {
+    int count, nK, it;
+    int kv, j, h, nt, k, b;
+    int u0, m_tiles, n_split, Ht, batch;
+    const int* tile_off;
+    const int* seq_off;
     AUnit x;
-    x.g = g;
-    int rest = g;
-    x.nt = rest % P.n_split;
-    rest /= P.n_split;
-    x.kv = rest & 1;
-    rest >>= 1;
-    x.h = rest % P.Ht;
-    x.j = rest / P.Ht;
-    if (k >= tile_off[batch]) { x.b = 0; x.t0 = 0; x.rows = 0; return x; }
-    int lo = 0, hi = batch - 1;
-    while (lo < hi) {
-        const int mid = (lo + hi + 1) >> 1;
-        if (tile_off[mid] <= k) lo = mid; else hi = mid - 1;
+
+    __device__ __forceinline__ void fill()
+    {
+        x.j = j; x.h = h; x.kv = kv; x.nt = nt;
+        x.g = ((j * Ht + h) * 2 + kv) * n_split + nt;
+        if (k >= tile_off[batch]) { x.b = 0; x.t0 = 0; x.rows = 0; return; }
+        while (b + 1 < batch && tile_off[b + 1] <= k) ++b;
+        x.b = b;
+        x.t0 = (k - tile_off[b]) * kTileM;
+        x.rows = min(kTileM, seq_off[b + 1] - seq_off[b] - x.t0);
     }
-    x.b = lo;
-    x.t0 = (k - tile_off[lo]) * kTileM;
-    const int T = seq_off[lo + 1] - seq_off[lo];
-    x.rows = min(kTileM, T - x.t0);
-    return x;
-}
+    __device__ __forceinline__ void seek(int idx, int kv_)
+    {
+        kv = kv_;
+        const int hg = idx / m_tiles;
+        k = idx - hg * m_tiles;
+        nt = hg % n_split;
+        const int jh = hg / n_split;
+        h = jh % Ht;
+        j = jh / Ht;
+        b = 0;
+        fill();
+    }
+    __device__ __forceinline__ void start(int u0_, int u1_, const AlignedParams& P, const int* tile_off_,
+                                          const int* seq_off_)
+    {
+        u0 = u0_; nK = u1_ - u0_; count = 2 * nK; it = 0;
+        m_tiles = P.m_tiles_max; n_split = P.n_split; Ht = P.Ht; batch = P.batch;
+        tile_off = tile_off_; seq_off = seq_off_;
+        if (count > 0) seek(u0, 0);
+    }
+    __device__ __forceinline__ bool more() const { return it < count; }
+    __device__ __forceinline__ void next()
+    {
+        if (++it >= count) return;
+        if (it == nK) { seek(u0, 1); return; }
+        if (++k == m_tiles) {
+            k = 0;
+            b = 0;
+            if (++nt == n_split) {
+                nt = 0;
+                if (++h == Ht) { h = 0; ++j; }
+            }
+        }
+        fill();
+    }
+    // no later unit of this CTA uses the current group's weights
+    __device__ __forceinline__ bool last_of_group() const
+    {
+        return it + 1 == count || it + 1 == nK || k + 1 >= tile_off[batch];
+    }
+};
+
+// position in the K-block slot ring
+struct SlotPos {
+    uint32_t idx, phase;
+    __device__ __forceinline__ void adv(uint32_t n)
+    {
+        if (++idx == n) { idx = 0; phase ^= 1; }
+    }
+};
 
 template <int HS>   // half head_dim of the source (32, 64 or 128)
 __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const __grid_constant__ AlignedParams P)
@@ -198,19 +243,9 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     const long long UH = (long long)hgroups * P.m_tiles_max;
     const int u0 = (int)((long long)blockIdx.x * UH / gridDim.x);
     const int u1 = (int)((long long)(blockIdx.x + 1) * UH / gridDim.x);
-    const int count = 2 * (u1 - u0);
-    // unit #it of this CTA -> (group, tile)
-    auto unit_at = [&](int it, int& g, int& k) {
-        const int kv = it >= (u1 - u0);
-        const int idx = u0 + (kv ? it - (u1 - u0) : it);
-        const int hg = idx / P.m_tiles_max;
-        k = idx - hg * P.m_tiles_max;
-        g = ((hg / P.n_split) * 2 + kv) * P.n_split + hg % P.n_split;
-    };
     const int blk_per_head = (2 * HS) / kBlockK;       // K-blocks of one source head
     const int hw = P.n_tile >> 1;
-
-#define KVX_FOR_UNITS for (int it = 0, ug = 0, uk = 0; it < count && (unit_at(it, ug, uk), true); ++it)
+    const uint32_t NS = (uint32_t)P.nslots;
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------ producer (one thread)
@@ -219,9 +254,11 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             const uint64_t pol_keep = policy_evict_last();
             int cur_g = -1;
             uint32_t b_loads = 0, slot_cnt = 0;
+            SlotPos sp{0, 0};
             bool ok = true;
-            KVX_FOR_UNITS {
-                const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+            Walker wk;
+            for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+                const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
                 if (x.g != cur_g) {
                     if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
@@ -237,13 +274,14 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 const CUtensorMap* map = &P.maps[x.j * 2 + x.kv];
                 const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
                 for (int kb = 0; kb < P.nblk; ++kb) {
-                    const uint32_t slot = slot_cnt % P.nslots;
-                    if (!W.wait(bar(kBarEmpty + slot), ((slot_cnt / P.nslots) & 1) ^ 1)) { ok = false; break; }
+                    const uint32_t slot = sp.idx;
+                    if (!W.wait(bar(kBarEmpty + slot), sp.phase ^ 1)) { ok = false; break; }
                     mbar_arrive_expect_tx(bar(kBarFull + slot), kBlockBytes);
                     tma_load_4d((uint32_t)__cvta_generic_to_shared(sRing) + slot * kBlockBytes, map,
                                 (kb % blk_per_head) * kBlockK, x.t0, g0 + kb / blk_per_head, x.b,
                                 bar(kBarFull + slot), pol_stream);
                     ++slot_cnt;
+                    sp.adv(NS);
                 }
                 if (!ok) break;
             }
@@ -261,10 +299,13 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             int cur_g = -1;
-            uint32_t b_cnt = 0, tcount = 0, slot_cnt = 0, kcount = 0;
+            uint32_t b_cnt = 0, tcount = 0;
+            SlotPos sp{0, 0};
+            uint32_t kr_idx = 0, kr_phase = 0;
             bool ok = true;
-            KVX_FOR_UNITS {
-                const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+            Walker wk;
+            for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+                const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
                 if (x.g != cur_g) {
                     if (!W.wait(bar(kBarBFull), b_cnt & 1)) break;
@@ -277,12 +318,12 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 const uint32_t d = tmem_base + buf * (uint32_t)P.n_tile;
                 const uint32_t b0 = (uint32_t)__cvta_generic_to_shared(sB);
                 if (rot) {   // K tile: wait until the prologue has un-rotated all its K-blocks
-                    if (!W.wait(bar(kBarKReady + kcount % P.nkready), (kcount / P.nkready) & 1)) break;
-                    ++kcount;
+                    if (!W.wait(bar(kBarKReady + kr_idx), kr_phase)) break;
+                    if (++kr_idx == (uint32_t)P.nkready) { kr_idx = 0; kr_phase ^= 1; }
                 }
                 for (int kb = 0; kb < P.nblk; ++kb) {
-                    const uint32_t slot = slot_cnt % P.nslots;
-                    const uint32_t par = (slot_cnt / P.nslots) & 1;
+                    const uint32_t slot = sp.idx;
+                    const uint32_t par = sp.phase;
                     if (!rot && !W.wait(bar(kBarFull + slot), par)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t a0 = (uint32_t)__cvta_generic_to_shared(sRing) + slot * kBlockBytes;
@@ -293,20 +334,12 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                         umma_bf16(d, ad, bd, P.idesc, (kb > 0 || kk > 0) ? 1u : 0u);
                     }
                     umma_commit(bar(kBarEmpty + slot));
-                    ++slot_cnt;
+                    sp.adv(NS);
                 }
                 if (!ok) break;
                 umma_commit(bar(kBarDFull + buf));
                 // the last valid tile of this group in the CTA's range releases B
-                bool last = true;
-                {
-                    for (int it2 = it + 1; it2 < count; ++it2) {
-                        int g2, k2;
-                        unit_at(it2, g2, k2);
-                        if (g2 != ug) break;
-                        if (k2 < sTileOff[P.batch]) { last = false; break; }
-                    }
-                }
+                const bool last = wk.last_of_group();
                 if (last) umma_commit(bar(kBarBEmpty));
                 ++tcount;
             }
@@ -321,8 +354,9 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         uint8_t* srow = sStage + (size_t)m * P.stage_row_bytes;
         const uint32_t srow_u32 = (uint32_t)__cvta_generic_to_shared(srow);
         uint32_t tcount = 0;
-        KVX_FOR_UNITS {
-            const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+        Walker wk;
+        for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+            const AUnit& x = wk.x;
             if (x.rows <= 0) continue;
             const uint32_t buf = tcount & 1;
             // output row of this thread, resolved while the tile is computed
@@ -416,24 +450,30 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         const int heads = P.in_dim / (2 * HS);            // heads in one A row
         constexpr int kChunks = HS / 8;                    // 16-byte chunks per half head
         constexpr int kMine = kChunks / 2;                 // chunks per thread
-        uint32_t slot_cnt = 0, kcount = 0;
+        SlotPos sp{0, 0};
+        uint32_t kr_idx = 0;
         bool ok = true;
-        KVX_FOR_UNITS {
-            const AUnit x = make_aunit(ug, uk, P, sTileOff, sSeqOff, P.batch);
+        Walker wk;
+        for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+            const AUnit& x = wk.x;
             if (x.rows <= 0) continue;
             const bool rot = x.kv == 0 && P.rs.enabled;
             // Walk every slot use in order (V tiles too), so that each wait is at most
             // one phase away from its barrier; the slot is refilled only after both
             // this release and the MMA's commit.
             for (int kb = 0; kb < P.nblk; ++kb) {
-                const uint32_t c = slot_cnt + kb;
-                if (!W.wait(bar(kBarFull + c % P.nslots), (c / P.nslots) & 1)) { ok = false; break; }
+                uint32_t si = sp.idx + kb, ph = sp.phase;
+                if (si >= NS) { si -= NS; ph ^= 1; }
+                if (!W.wait(bar(kBarFull + si), ph)) { ok = false; break; }
             }
             if (!ok) break;
             if (!rot) {
                 if (xt == 0)
-                    for (int kb = 0; kb < P.nblk; ++kb) mbar_arrive(bar(kBarEmpty + (slot_cnt + kb) % P.nslots));
-                slot_cnt += P.nblk;
+                    for (int kb = 0; kb < P.nblk; ++kb) {
+                        const uint32_t si = sp.idx + kb;
+                        mbar_arrive(bar(kBarEmpty + (si >= NS ? si - NS : si)));
+                    }
+                for (int kb = 0; kb < P.nblk; ++kb) sp.adv(NS);
                 continue;
             }
             for (int pass = 0; pass < (2 * kTileM) / kXfThreads; ++pass) {
@@ -452,8 +492,9 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                     for (int q = 0; q < heads; ++q) {
                         // element i (and i+HS) of head q: K-block and column within it
                         const int k_lo = q * 2 * HS + i, k_hi = k_lo + HS;
-                        const uint32_t s_lo = (slot_cnt + (k_lo >> 6)) % P.nslots;
-                        const uint32_t s_hi = (slot_cnt + (k_hi >> 6)) % P.nslots;
+                        uint32_t s_lo = sp.idx + (k_lo >> 6), s_hi = sp.idx + (k_hi >> 6);
+                        s_lo -= s_lo >= NS ? NS : 0;
+                        s_hi -= s_hi >= NS ? NS : 0;
                         uint8_t* p_lo = sRing + s_lo * kBlockBytes + sw128_off(row, k_lo & 63, kTileM);
                         uint8_t* p_hi = sRing + s_hi * kBlockBytes + sw128_off(row, k_hi & 63, kTileM);
                         const uint4 wl = *reinterpret_cast<const uint4*>(p_lo);
@@ -479,15 +520,17 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             }
             fence_proxy_async();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kBarKReady + kcount % P.nkready));
+            if (lane == 0) mbar_arrive(bar(kBarKReady + kr_idx));
+            if (++kr_idx == (uint32_t)P.nkready) kr_idx = 0;
             // the MMA's commit (after every prologue warp's "ready") completes the release
             if (xt == 0)
-                for (int kb = 0; kb < P.nblk; ++kb) mbar_arrive(bar(kBarEmpty + (slot_cnt + kb) % P.nslots));
-            ++kcount;
-            slot_cnt += P.nblk;
+                for (int kb = 0; kb < P.nblk; ++kb) {
+                    const uint32_t si = sp.idx + kb;
+                    mbar_arrive(bar(kBarEmpty + (si >= NS ? si - NS : si)));
+                }
+            for (int kb = 0; kb < P.nblk; ++kb) sp.adv(NS);
         }
     }
-#undef KVX_FOR_UNITS
 
     tc_fence_before();
     __syncthreads();
