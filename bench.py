@@ -51,6 +51,17 @@ def algorithmic(spec: synth.WorkloadSpec, wl: synth.Workload, layer_map) -> dict
     return {"read": rd, "write": wr, "weights": wt, "bytes": rd + wr + wt, "flops": flops}
 
 
+def aggregate(elapsed_ms: float, tokens_per_step: int, steps: int, world: int, dist=None, device=None):
+    """Whole-job throughput: every rank translates its own replica; the job time
+    is the slowest rank's.  Returns (max elapsed ms, tokens/s over all ranks)."""
+    if dist is not None and world > 1:
+        import torch
+        t = torch.tensor([float(elapsed_ms)], dtype=torch.float64, device=device)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    return elapsed_ms, tokens_per_step * steps * world / (elapsed_ms / 1e3)
+
+
 def nearest_map(Ls, Lt):
     return [0] * Lt if Lt == 1 else [(2 * j * (Ls - 1) + (Lt - 1)) // (2 * (Lt - 1)) for j in range(Lt)]
 
@@ -316,10 +327,7 @@ def main():
     if tr.device_status() != 0:
         raise RuntimeError("device status nonzero after the timed region")
 
-    if dist:
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms, value = aggregate(elapsed_ms, wl.total_tgt, args.steps, world, dist, dev)
 
     # end to end through the C ABI with host buffers: H2D source, translate, D2H target
     e2e_steps = max(1, args.e2e_steps)
@@ -349,10 +357,7 @@ def main():
     b.record(stream)
     torch.cuda.synchronize()
     e2e_ms = a.elapsed_time(b)
-    if dist:
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms, e2e_value = aggregate(e2e_ms, wl.total_tgt, e2e_steps, world, dist, dev)
 
     if rank != 0:
         if dist:
@@ -360,7 +365,6 @@ def main():
         return
 
     T = wl.total_tgt
-    value = T * args.steps * world / (elapsed_ms / 1e3)
     ms_step = elapsed_ms / args.steps
     avg_launch_ms = statistics.mean(launch_ms)
     peaks = {}
@@ -407,7 +411,7 @@ def main():
                      "algorithmic_bytes_per_launch": alg["bytes"], "avg_launch_ms": avg_launch_ms,
                      "tensor_tflops": alg["flops"] / (avg_launch_ms / 1e3) / 1e12},
         "clocks": clk,
-        "e2e": {"value": T * e2e_steps * world / (e2e_ms / 1e3), "unit": "tokens/s",
+        "e2e": {"value": e2e_value, "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / e2e_steps},
         "gpu_launches": args.steps * tr.launches_per_translate(),
         "kernel_path": ({1: "simt", 2: "tcgen05"}.get(info.path, str(info.path)) +
