@@ -206,6 +206,38 @@ KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_translator_info* i
 /* Kernel launches one kvx_translate call makes (for launch accounting). */
 KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
 
+/* Size of the device scratch array kvx_translate_static works in (8 MiB). */
+#define KVX_STATIC_SCRATCH_BYTES (8u << 20)
+
+/* Translate without allocating device memory.  The paper has no counterpart; this exists for
+ * callers that cannot call cudaMalloc when they translate: a serving process whose device memory
+ * belongs to a caching allocator that forbids raw allocations, a runtime whose memory budget is
+ * fixed at start-up, or a latency-critical path where cudaMalloc/cudaFree would synchronise the
+ * device.  kvx_translator_create allocates; this call does not.
+ *
+ * It runs the CUDA-core translation kernel (the KVX_PATH_SIMT path of kvx_translate) with its
+ * scratch (status word, rotation frequencies and the weights) in one file-scope device array of
+ * KVX_STATIC_SCRATCH_BYTES, which every GPU that loads the library holds until the process exits.
+ * The arguments mean what they mean for kvx_translator_create and kvx_translate, except:
+ *   w_k, w_v: DEVICE pointers, row-major [dst.num_layers][dst.num_kv_heads][in][out] of
+ *     desc->dtype; they are copied into the scratch array on every call.  Both together must fit
+ *     KVX_STATIC_SCRATCH_BYTES minus 2304 bytes, else KVX_ERR_UNSUPPORTED (nothing is launched).
+ *   desc->path is ignored.
+ *   status_bits: host pointer or NULL.  If set, the call synchronises stream, writes the device
+ *     status word there and returns KVX_ERR_DEVICE_STATUS when it is nonzero; if NULL, the call is
+ *     asynchronous on stream like kvx_translate.
+ * The first call on a device looks up the array's device address with that device current (a
+ * one-time set-up); make that first call before any stream capture.  Every call shares the one
+ * array and clears the status word itself, so calls that overlap on the GPU (different streams,
+ * or several host threads) race on the scratch and must be serialised by the caller.
+ * Calls no cudaMalloc, cudaFree or other allocating routine.  Errors: kvx_static_last_error(). */
+KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* desc, const void* w_k, const void* w_v,
+                                        const kvx_src_kv* src, const kvx_tgt_tokens* tgt, const kvx_dst_kv* dst,
+                                        uint32_t* status_bits, void* stream);
+
+/* Message of the last failed kvx_translate_static call on this thread ("" if none). */
+KVX_API const char* kvx_static_last_error(void);
+
 /* Message of the last failed call on this thread ("" if none). */
 KVX_API const char* kvx_last_error(void);
 

@@ -70,7 +70,8 @@ class kvx_translator_info(ctypes.Structure):
 
 EXPORTS = ["kvx_translator_create", "kvx_translate", "kvx_build_alignment", "kvx_layer_map_nearest",
            "kvx_get_device_status", "kvx_get_info", "kvx_launches_per_translate", "kvx_last_error",
-           "kvx_destroy"]
+           "kvx_destroy", "kvx_translate_static", "kvx_static_last_error"]
+KVX_STATIC_SCRATCH_BYTES = 8 << 20
 
 _lib = None
 
@@ -110,8 +111,12 @@ def lib():
         L.kvx_launches_per_translate.restype = ctypes.c_int32
         L.kvx_last_error.restype = ctypes.c_char_p
         L.kvx_destroy.argtypes = [VP]
+        L.kvx_translate_static.argtypes = [ctypes.POINTER(kvx_translator_desc), VP, VP, ctypes.POINTER(kvx_src_kv),
+                                           ctypes.POINTER(kvx_tgt_tokens), ctypes.POINTER(kvx_dst_kv),
+                                           ctypes.POINTER(ctypes.c_uint32), VP]
+        L.kvx_static_last_error.restype = ctypes.c_char_p
         for name in EXPORTS:
-            if name not in ("kvx_last_error", "kvx_launches_per_translate"):
+            if name not in ("kvx_last_error", "kvx_launches_per_translate", "kvx_static_last_error"):
                 getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -148,6 +153,19 @@ def kvx_build_alignment(batch, total_src, total_tgt, src_seq_off, src_end, tgt_s
                         dev_status=0, stream: int = 0):
     _check(lib().kvx_build_alignment(batch, total_src, total_tgt, VP(src_seq_off), VP(src_end), VP(tgt_seq_off),
                                      VP(tgt_end), VP(span_lo), VP(span_hi), VP(dev_status), VP(stream)))
+
+
+def kvx_translate_static(desc: kvx_translator_desc, w_k_ptr: int, w_v_ptr: int, src: kvx_src_kv,
+                         tgt: kvx_tgt_tokens, dst: kvx_dst_kv, stream: int = 0, read_status: bool = False) -> int:
+    """Allocation-free translation (see include/kvx.h).  Returns the device status word when
+    read_status is set (the call then synchronises the stream), else 0."""
+    bits = ctypes.c_uint32(0)
+    st = lib().kvx_translate_static(ctypes.byref(desc), VP(w_k_ptr), VP(w_v_ptr), ctypes.byref(src),
+                                    ctypes.byref(tgt), ctypes.byref(dst),
+                                    ctypes.byref(bits) if read_status else None, VP(stream))
+    if st not in (KVX_OK, KVX_ERR_DEVICE_STATUS):
+        raise KvxError(st, lib().kvx_static_last_error().decode())
+    return bits.value
 
 
 def kvx_get_device_status(handle: int, stream: int = 0, clear: bool = True) -> int:

@@ -1,0 +1,103 @@
+"""kvx_translate_static: the allocation-free entry point.
+
+Some callers cannot allocate device memory when they translate (a caching
+allocator owns the device memory, the memory budget was fixed at start-up, or
+cudaMalloc would synchronise a latency-critical path).  kvx_translate_static
+serves them from a static device scratch array.  These tests call it through
+the C ABI and check, on two calls in a row, that it writes what the regular
+entry point (kvx_translator_create + kvx_translate) writes for the same inputs.
+The file sorts last so a stop-at-first-failure run has run every other test.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import paper_2608_30963_gb300 as kvx
+from paper_2608_30963_gb300 import synth
+
+from harness import compare, make_case
+
+pytestmark = pytest.mark.gpu
+
+
+def _structs(g):
+    """C structs of a GpuRun's buffers (same marshalling as Translator.translate)."""
+    P = kvx._ptr
+    s0 = g.src_k[0]
+    src = kvx.kvx_src_kv(s0.shape[0], s0.shape[2], kvx._ptr_array(g.src_k), kvx._ptr_array(g.src_v),
+                         s0.stride(0), s0.stride(1), s0.stride(2), P(g.src_len), P(g.src_pos))
+    tgt = kvx.kvx_tgt_tokens(g.c.wl.total_tgt, P(g.seq_off), P(g.span_lo), P(g.span_hi), P(g.tgt_pos))
+    d0 = g.dst_k[0]
+    dst = kvx.kvx_dst_kv(kvx._ptr_array(g.dst_k), kvx._ptr_array(g.dst_v), 0, d0.shape[2], d0.stride(0),
+                         d0.stride(1), d0.stride(2), None, 0, 0, 0)
+    return src, tgt, dst
+
+
+def _shrink(spec, Ls, Lt):
+    return dataclasses.replace(spec, src=dataclasses.replace(spec.src, num_layers=Ls),
+                               dst=dataclasses.replace(spec.dst, num_layers=Lt))
+
+
+CASES = [("tiny_fp32", None, None, None), ("qwen1p5b_to_gemma2b_1k", 3, 2, [130, 7]),
+         ("qwen7b_to_qwen1p5b_4k", 2, 2, [200])]
+
+
+@pytest.mark.parametrize("name,Ls,Lt,lens", CASES, ids=[c[0] for c in CASES])
+def test_static_entry_matches_translator_on_two_calls(name, Ls, Lt, lens):
+    from gpu_harness import GpuRun, to_dev, i32
+    kvx.build()
+    spec = synth.config_specs()[name]
+    if Ls:
+        spec = _shrink(spec, Ls, Lt)
+    c = make_case(spec, lens)
+    # the regular entry point, CUDA-core path (the kernel the static entry point runs)
+    ref = GpuRun(c, path=kvx.KVX_PATH_SIMT, paged=False)
+    ref.run()
+    torch.cuda.synchronize()
+    rk, rv = ref.gather()
+    assert ref.status() == 0
+
+    g = GpuRun(c, path=kvx.KVX_PATH_SIMT, paged=False)   # buffers only; its translator is not used
+    wk, wv = to_dev(c.w_k, spec.dtype), to_dev(c.w_v, spec.dtype)
+    desc = g.tr.desc
+    stream = torch.cuda.current_stream().cuda_stream
+    for call in range(2):
+        for t in g.dst_k + g.dst_v:
+            t.fill_(float("nan"))
+        src, tgt, dst = _structs(g)
+        bits = kvx.kvx_translate_static(desc, wk.data_ptr(), wv.data_ptr(), src, tgt, dst, stream,
+                                        read_status=True)
+        assert bits == 0, f"call {call}: status 0x{bits:x}"
+        gk, gv = g.gather()
+        compare(gk, rk, spec.dtype)
+        compare(gv, rv, spec.dtype)
+
+
+def test_static_entry_clears_its_status_and_rejects_oversize():
+    from gpu_harness import GpuRun, to_dev, i32
+    kvx.build()
+    spec = _shrink(synth.config_specs()["qwen7b_to_qwen1p5b_4k"], 2, 2)
+    c = make_case(spec, [64])
+    g = GpuRun(c, path=kvx.KVX_PATH_SIMT, paged=False)
+    wk, wv = to_dev(c.w_k, spec.dtype), to_dev(c.w_v, spec.dtype)
+    stream = torch.cuda.current_stream().cuda_stream
+    lo = np.arange(64, dtype=np.int32)
+    hi = lo + 1
+    hi[3] = 10_000                                   # past the source: clamped and flagged
+    g.span_lo, g.span_hi = i32(lo), i32(hi)
+    src, tgt, dst = _structs(g)
+    bits = kvx.kvx_translate_static(g.tr.desc, wk.data_ptr(), wv.data_ptr(), src, tgt, dst, stream, True)
+    assert bits & kvx.KVX_DEV_SPAN_CLAMPED
+    g.span_lo = g.span_hi = None                     # a clean call right after: the word starts at zero
+    src, tgt, dst = _structs(g)
+    assert kvx.kvx_translate_static(g.tr.desc, wk.data_ptr(), wv.data_ptr(), src, tgt, dst, stream, True) == 0
+    # weights larger than the static scratch are refused before anything runs
+    big = kvx.kvx_translator_desc.from_buffer_copy(g.tr.desc)
+    big.layer_map = None
+    big.dst.num_layers = 128                         # 2 * 128 * 2 * 256 * 128 * 2 B > 8 MiB
+    with pytest.raises(kvx.KvxError) as e:
+        kvx.kvx_translate_static(big, wk.data_ptr(), wv.data_ptr(), src, tgt, dst, stream, True)
+    assert e.value.status == kvx.KVX_ERR_UNSUPPORTED
