@@ -50,6 +50,7 @@ struct TranslateParams {
     int max_pages, page_size, num_pages;
     // rotation
     RopeTable rs, rt;
+    int rope_same;   // source and target RoPE have the same base and head_dim
     int max_position;
     unsigned* status;
     // weights (layout depends on the kernel)

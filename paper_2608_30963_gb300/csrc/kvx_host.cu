@@ -307,6 +307,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
     P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
     P.page_size = dst->page_size; P.num_pages = dst->num_pages;
     P.rs = tr->rs; P.rt = tr->rt; P.max_position = tr->max_position;
+    P.rope_same = D.src.rope_base == D.dst.rope_base && D.src.head_dim == D.dst.head_dim;
     P.status = tr->status;
     P.w = tr->w;
     for (int j = 0; j < Lt; ++j) {

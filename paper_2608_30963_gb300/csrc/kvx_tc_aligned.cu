@@ -57,7 +57,9 @@ constexpr int kMaxKReady = kMaxSlots + 2;
 // +quad*2 + {0,1}: the two epilogue warps of a TMEM lane quadrant meet here before
 // writing the shared staging rows (0) and before storing them (1)
 constexpr int kBarPair = kBarKReady + kMaxKReady;
-constexpr int kNumBars = kBarPair + 8;
+// +buf: the epilogue has read the (cos, sin) the prologue left in TMEM for a K tile
+constexpr int kBarCsFree = kBarPair + 8;
+constexpr int kNumBars = kBarCsFree + 2;
 
 struct AlignedParams {
     // geometry
@@ -80,6 +82,10 @@ struct AlignedParams {
     unsigned* status;
     const void* w;
     unsigned idesc, tmem_cols, b_bytes, stage_row_bytes;
+    // When source and target rotations coincide (same base, head_dim and positions), the prologue
+    // leaves each K tile's (cos, sin) in TMEM columns [cs_col + buf*d, +d) for the epilogue.
+    int share_cs;
+    unsigned cs_col;
     unsigned off_b, off_ring, off_stage, off_bar, off_misc, off_seq, off_turns;
     void* dst_k[KVX_MAX_ALIGNED_LAYERS];
     void* dst_v[KVX_MAX_ALIGNED_LAYERS];
@@ -214,6 +220,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         }
         for (int i = 0; i < P.nkready; ++i) mbar_init(bar(kBarKReady + i), kNumXfWarps);
         for (int i = 0; i < 8; ++i) mbar_init(bar(kBarPair + i), 2);
+        for (int i = 0; i < 2; ++i) mbar_init(bar(kBarCsFree + i), kNumEpiWarps);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -260,17 +267,8 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
                 const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
-                if (x.g != cur_g) {
-                    if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
-                    mbar_arrive_expect_tx(bar(kBarBFull), P.b_bytes);
-                    const uint8_t* img = (const uint8_t*)P.w + (size_t)x.g * P.b_bytes;
-                    const uint32_t piece = P.b_bytes / 4;
-                    for (int q = 0; q < 4; ++q)
-                        bulk_g2s((uint32_t)__cvta_generic_to_shared(sB) + q * piece, img + (size_t)q * piece, piece,
-                                 bar(kBarBFull), pol_keep);
-                    ++b_loads;
-                    cur_g = x.g;
-                }
+                // A K-blocks first: they do not depend on the weights, so at a group switch the
+                // ring refills while the previous group's last tiles drain
                 const CUtensorMap* map = &P.maps[x.j * 2 + x.kv];
                 const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
                 for (int kb = 0; kb < P.nblk; ++kb) {
@@ -282,6 +280,18 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                                 bar(kBarFull + slot), pol_stream);
                     ++slot_cnt;
                     sp.adv(NS);
+                }
+                if (!ok) break;
+                if (x.g != cur_g) {
+                    if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
+                    mbar_arrive_expect_tx(bar(kBarBFull), P.b_bytes);
+                    const uint8_t* img = (const uint8_t*)P.w + (size_t)x.g * P.b_bytes;
+                    const uint32_t piece = P.b_bytes / 4;
+                    for (int q = 0; q < 4; ++q)
+                        bulk_g2s((uint32_t)__cvta_generic_to_shared(sB) + q * piece, img + (size_t)q * piece, piece,
+                                 bar(kBarBFull), pol_keep);
+                    ++b_loads;
+                    cur_g = x.g;
                 }
                 if (!ok) break;
             }
@@ -353,7 +363,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         const int pc_begin = half * (hw >> 1), pc_end = pc_begin + (hw >> 1);
         uint8_t* srow = sStage + (size_t)m * P.stage_row_bytes;
         const uint32_t srow_u32 = (uint32_t)__cvta_generic_to_shared(srow);
-        uint32_t tcount = 0;
+        uint32_t tcount = 0, kc = 0;   // kc: K tiles seen (selects the shared (cos, sin) buffer)
         Walker wk;
         for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
             const AUnit& x = wk.x;
@@ -390,12 +400,20 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2));
             if (!W.wait(bar(kBarPair + quad * 2), tcount & 1)) break;
             const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)P.n_tile;
+            const bool shared_cs = rot && P.share_cs;          // (cos, sin) left in TMEM by the prologue
+            const uint32_t cs_addr = tmem_base + ((uint32_t)(quad * 32) << 16) + P.cs_col + (kc & 1) * (uint32_t)P.dt;
             for (int pc = pc_begin; pc < pc_end; pc += 8) {
                 uint32_t r0[8], r1[8];
                 tmem_ld8(taddr + pc, r0);
                 tmem_ld8(taddr + hw + pc, r1);
                 float2 cs[8];
-                if (rot) {
+                if (shared_cs) {
+                    uint32_t v[16];
+                    tmem_ld16(cs_addr + 2 * (x.nt * hw + pc), v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e2 = 0; e2 < 8; ++e2) cs[e2] = make_float2(__uint_as_float(v[2 * e2]), __uint_as_float(v[2 * e2 + 1]));
+                } else if (rot) {
 #pragma unroll
                     for (int e2 = 0; e2 < 8; ++e2) cs[e2] = turn_cs(sTurnT[x.nt * hw + pc + e2], pt);
                 }
@@ -420,7 +438,11 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             }
             tc_fence_before();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kBarDEmpty + buf));
+            if (lane == 0) {
+                mbar_arrive(bar(kBarDEmpty + buf));
+                if (shared_cs) mbar_arrive(bar(kBarCsFree + (kc & 1)));
+            }
+            if (x.kv == 0) ++kc;
             fence_proxy_async();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2 + 1));
@@ -441,17 +463,20 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         bulk_wait0();
     } else {
         // ------------------------------------------------------------ prologue: undo source RoPE in place
-        // Thread layout over a K tile: 2 threads per token row; each owns HS/2
-        // rotary pairs (i, i+HS) of every grouped head and computes each (cos, sin)
-        // once for all heads.  Pairs are handled 8 at a time (one 16-byte chunk of
-        // each half).  A thread visits its chunks in an order staggered by row so
-        // that the 8 threads of a shared-memory phase hit distinct bank groups.
+        // Thread layout over a K tile: thread = token row = TMEM lane of its warp's
+        // quadrant (row = 32*(warp%4) + lane), and the two warps of a quadrant split
+        // the rotary pairs (i, i+HS).  Each (cos, sin) is computed once for all
+        // grouped heads.  Pairs go 8 at a time (one 16-byte chunk of each half); under
+        // the 128-byte swizzle the 8 rows of a shared-memory phase hit distinct banks.
         const int xt = threadIdx.x - kXfWarp0 * 32;
+        const int row = (warp & 3) * 32 + lane;
+        const int part = (warp - kXfWarp0) >> 2;          // 0 or 1
         const int heads = P.in_dim / (2 * HS);            // heads in one A row
         constexpr int kChunks = HS / 8;                    // 16-byte chunks per half head
         constexpr int kMine = kChunks / 2;                 // chunks per thread
+        const uint32_t cs_lane = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + P.cs_col;
         SlotPos sp{0, 0};
-        uint32_t kr_idx = 0;
+        uint32_t kr_idx = 0, kc = 0;
         bool ok = true;
         Walker wk;
         for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
@@ -476,52 +501,65 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 for (int kb = 0; kb < P.nblk; ++kb) sp.adv(NS);
                 continue;
             }
-            for (int pass = 0; pass < (2 * kTileM) / kXfThreads; ++pass) {
-                const int row = (pass * kXfThreads + xt) >> 1;
-                const int part = xt & 1;
-                if (row >= x.rows) continue;
-                const int t = x.t0 + row;
-                const int p = src_pos_of_seq(P.src_pos, P.src_max_seq, x.b, t, P.max_position, P.status);
+            const uint32_t csbuf = kc & 1;
+            if (P.share_cs) {   // the epilogue must be done with this buffer's previous K tile
+                if (!W.wait(bar(kBarCsFree + csbuf), ((kc >> 1) & 1) ^ 1)) break;
+                tc_fence_after();
+            }
+            // rows past the sequence are rotated too (harmless: not stored) so that the
+            // warp-collective TMEM stores below see every lane
+            const int t = x.t0 + row;
+            const int p = row < x.rows ? src_pos_of_seq(P.src_pos, P.src_max_seq, x.b, t, P.max_position, P.status)
+                                       : 0;
 #pragma unroll
-                for (int cc = 0; cc < kMine; ++cc) {
-                    const int c = part * kMine + ((cc + (row >> 2)) % kMine);   // staggered chunk
-                    const int i = c * 8;                                        // first pair index
-                    float2 cs[8];
+            for (int cc = 0; cc < kMine; ++cc) {
+                const int i = (part * kMine + cc) * 8;             // first pair index of the chunk
+                float2 cs[8];
 #pragma unroll
-                    for (int e2 = 0; e2 < 8; ++e2) cs[e2] = turn_cs(sTurnS[i + e2], p);
-                    for (int q = 0; q < heads; ++q) {
-                        // element i (and i+HS) of head q: K-block and column within it
-                        const int k_lo = q * 2 * HS + i, k_hi = k_lo + HS;
-                        uint32_t s_lo = sp.idx + (k_lo >> 6), s_hi = sp.idx + (k_hi >> 6);
-                        s_lo -= s_lo >= NS ? NS : 0;
-                        s_hi -= s_hi >= NS ? NS : 0;
-                        uint8_t* p_lo = sRing + s_lo * kBlockBytes + sw128_off(row, k_lo & 63, kTileM);
-                        uint8_t* p_hi = sRing + s_hi * kBlockBytes + sw128_off(row, k_hi & 63, kTileM);
-                        const uint4 wl = *reinterpret_cast<const uint4*>(p_lo);
-                        const uint4 wh = *reinterpret_cast<const uint4*>(p_hi);
-                        const uint32_t al[4] = {wl.x, wl.y, wl.z, wl.w};
-                        const uint32_t ah[4] = {wh.x, wh.y, wh.z, wh.w};
-                        uint32_t ol[4], oh[4];
+                for (int e2 = 0; e2 < 8; ++e2) cs[e2] = turn_cs(sTurnS[i + e2], p);
+                if (P.share_cs) {
+                    uint32_t v[16];
 #pragma unroll
-                        for (int w2 = 0; w2 < 4; ++w2) {
-                            float x0a = bf_lo(al[w2]), x0b = bf_hi(al[w2]);
-                            float x1a = bf_lo(ah[w2]), x1b = bf_hi(ah[w2]);
-                            const float2 ca = cs[2 * w2], cb = cs[2 * w2 + 1];
-                            // undo the rotation: R(-theta)
-                            const float u0a = fmaf(x0a, ca.x, x1a * ca.y), u1a = fmaf(x1a, ca.x, -x0a * ca.y);
-                            const float u0b = fmaf(x0b, cb.x, x1b * cb.y), u1b = fmaf(x1b, cb.x, -x0b * cb.y);
-                            ol[w2] = pack_bf16(u0a, u0b);
-                            oh[w2] = pack_bf16(u1a, u1b);
-                        }
-                        *reinterpret_cast<uint4*>(p_lo) = make_uint4(ol[0], ol[1], ol[2], ol[3]);
-                        *reinterpret_cast<uint4*>(p_hi) = make_uint4(oh[0], oh[1], oh[2], oh[3]);
-                    }
+                    for (int e2 = 0; e2 < 8; ++e2) { v[2 * e2] = __float_as_uint(cs[e2].x); v[2 * e2 + 1] = __float_as_uint(cs[e2].y); }
+                    tmem_st16(cs_lane + csbuf * (uint32_t)(2 * HS) + 2 * i, v);
                 }
+                for (int q = 0; q < heads; ++q) {
+                    // element i (and i+HS) of head q: K-block and column within it
+                    const int k_lo = q * 2 * HS + i, k_hi = k_lo + HS;
+                    uint32_t s_lo = sp.idx + (k_lo >> 6), s_hi = sp.idx + (k_hi >> 6);
+                    s_lo -= s_lo >= NS ? NS : 0;
+                    s_hi -= s_hi >= NS ? NS : 0;
+                    uint8_t* p_lo = sRing + s_lo * kBlockBytes + sw128_off(row, k_lo & 63, kTileM);
+                    uint8_t* p_hi = sRing + s_hi * kBlockBytes + sw128_off(row, k_hi & 63, kTileM);
+                    const uint4 wl = *reinterpret_cast<const uint4*>(p_lo);
+                    const uint4 wh = *reinterpret_cast<const uint4*>(p_hi);
+                    const uint32_t al[4] = {wl.x, wl.y, wl.z, wl.w};
+                    const uint32_t ah[4] = {wh.x, wh.y, wh.z, wh.w};
+                    uint32_t ol[4], oh[4];
+#pragma unroll
+                    for (int w2 = 0; w2 < 4; ++w2) {
+                        float x0a = bf_lo(al[w2]), x0b = bf_hi(al[w2]);
+                        float x1a = bf_lo(ah[w2]), x1b = bf_hi(ah[w2]);
+                        const float2 ca = cs[2 * w2], cb = cs[2 * w2 + 1];
+                        // undo the rotation: R(-theta)
+                        const float u0a = fmaf(x0a, ca.x, x1a * ca.y), u1a = fmaf(x1a, ca.x, -x0a * ca.y);
+                        const float u0b = fmaf(x0b, cb.x, x1b * cb.y), u1b = fmaf(x1b, cb.x, -x0b * cb.y);
+                        ol[w2] = pack_bf16(u0a, u0b);
+                        oh[w2] = pack_bf16(u1a, u1b);
+                    }
+                    *reinterpret_cast<uint4*>(p_lo) = make_uint4(ol[0], ol[1], ol[2], ol[3]);
+                    *reinterpret_cast<uint4*>(p_hi) = make_uint4(oh[0], oh[1], oh[2], oh[3]);
+                }
+            }
+            if (P.share_cs) {
+                tmem_st_wait();
+                tc_fence_before();
             }
             fence_proxy_async();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarKReady + kr_idx));
             if (++kr_idx == (uint32_t)P.nkready) kr_idx = 0;
+            ++kc;
             // the MMA's commit (after every prologue warp's "ready") completes the release
             if (xt == 0)
                 for (int kb = 0; kb < P.nblk; ++kb) {
@@ -604,8 +642,11 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     P.page_table = T.page_table; P.max_pages = T.max_pages; P.page_size = T.page_size; P.num_pages = T.num_pages;
     P.rs = T.rs; P.rt = T.rt; P.max_position = T.max_position; P.status = T.status; P.w = T.w;
     P.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(P.n_tile >> 3) << 17) | ((uint32_t)(kTileM >> 4) << 24);
+    P.share_cs = T.rs.enabled && T.rt.enabled && T.ds == T.dt && !T.src_pos && !T.tgt_pos &&
+                 T.rope_same && 2 * P.n_tile + 2 * T.dt <= 512;
+    P.cs_col = (unsigned)(2 * P.n_tile);
     unsigned cols = 32;
-    while (cols < 2u * (unsigned)P.n_tile) cols <<= 1;
+    while (cols < 2u * (unsigned)P.n_tile + (P.share_cs ? 2u * (unsigned)T.dt : 0u)) cols <<= 1;
     P.tmem_cols = cols;
     P.b_bytes = (unsigned)(T.in_dim * P.n_tile * 2);
     P.stage_row_bytes = (unsigned)(P.n_tile * 2 + 16);
