@@ -24,6 +24,7 @@ struct kvx_translator {
     void* w = nullptr;           // SIMT: [2][Lt][Ht][in][out] dtype; tcgen05: pre-swizzled images
     size_t w_bytes = 0;
     unsigned long long* rope = nullptr;   // fixed-point turns: source [d_s/2] | target [d_t/2]
+    unsigned long long host_turns[256];   // host copy of the same
     size_t rope_bytes = 0;
     RopeTable rs{}, rt{};
     unsigned* status = nullptr;
@@ -241,6 +242,7 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
             st = fail(KVX_ERR_OOM, "create: table allocation");
             goto err;
         }
+        memcpy(t->host_turns, h_turns, t->rope_bytes);
         if ((ce = cudaMemcpy(t->rope, h_turns, t->rope_bytes, cudaMemcpyHostToDevice)) != cudaSuccess) {
             st = fail(KVX_ERR_CUDA, "create: table upload: %s", cudaGetErrorString(ce));
             goto err;
@@ -332,7 +334,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
                     return fail(KVX_ERR_INVALID_ARG, "translate: cannot describe the source cache of layer %d to the "
                                                      "tensor-copy unit (strides, sizes)", tr->layer_map[j]);
             }
-        ce = launch_translate_tc_aligned(P, maps, tr->num_sms, (cudaStream_t)stream);
+        ce = launch_translate_tc_aligned(P, maps, tr->host_turns, tr->num_sms, (cudaStream_t)stream);
     } else if (tr->path == KVX_PATH_TCGEN05) {
         ce = launch_translate_tc(P, tr->tc, tr->num_sms, (cudaStream_t)stream);
     } else {

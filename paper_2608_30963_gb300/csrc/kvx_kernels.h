@@ -33,6 +33,6 @@ bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch);
 size_t aligned_map_bytes();
 bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int Hs, int batch, long long ss,
                        long long sh, long long sb);
-cudaError_t launch_translate_tc_aligned(const TranslateParams& P, const void* const* maps, int num_sms,
-                                        cudaStream_t stream);
+cudaError_t launch_translate_tc_aligned(const TranslateParams& P, const void* const* maps,
+                                        const unsigned long long* host_turns, int num_sms, cudaStream_t stream);
 }  // namespace kvx

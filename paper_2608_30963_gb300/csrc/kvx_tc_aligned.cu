@@ -86,7 +86,10 @@ struct AlignedParams {
     // leaves each K tile's (cos, sin) in TMEM columns [cs_col + buf*d, +d) for the epilogue.
     int share_cs;
     unsigned cs_col;
-    unsigned off_b, off_ring, off_stage, off_bar, off_misc, off_seq, off_turns;
+    unsigned off_b, off_ring, off_stage, off_bar, off_misc, off_seq;
+    // rotation turns (kvx_common.cuh): source [0, ds/2), target [128, 128 + dt/2); read
+    // warp-uniformly, so from the constant bank rather than shared memory
+    unsigned long long turns[256];
     void* dst_k[KVX_MAX_ALIGNED_LAYERS];
     void* dst_v[KVX_MAX_ALIGNED_LAYERS];
     CUtensorMap maps[2 * KVX_MAX_ALIGNED_LAYERS];   // [j*2 + kv]: source K/V of target layer j
@@ -114,7 +117,7 @@ struct AUnit {
 struct Walker {
     int count, nK, it;
     int kv, j, h, nt, k, b;
-    int u0, m_tiles, n_split, Ht, batch;
+    int u0, v0, m_tiles, n_split, Ht, batch;
     const int* tile_off;
     const int* seq_off;
     AUnit x;
@@ -141,19 +144,21 @@ struct Walker {
         b = 0;
         fill();
     }
-    __device__ __forceinline__ void start(int u0_, int u1_, const AlignedParams& P, const int* tile_off_,
-                                          const int* seq_off_)
+    // K units [u0, u1) and V units [v0, v1) of the per-K|V unit index space
+    __device__ __forceinline__ void start(int u0_, int u1_, int v0_, int v1_, const AlignedParams& P,
+                                          const int* tile_off_, const int* seq_off_)
     {
-        u0 = u0_; nK = u1_ - u0_; count = 2 * nK; it = 0;
+        u0 = u0_; v0 = v0_; nK = u1_ - u0_; count = nK + (v1_ - v0_); it = 0;
         m_tiles = P.m_tiles_max; n_split = P.n_split; Ht = P.Ht; batch = P.batch;
         tile_off = tile_off_; seq_off = seq_off_;
-        if (count > 0) seek(u0, 0);
+        if (nK > 0) seek(u0, 0);
+        else if (count > 0) seek(v0, 1);
     }
     __device__ __forceinline__ bool more() const { return it < count; }
     __device__ __forceinline__ void next()
     {
         if (++it >= count) return;
-        if (it == nK) { seek(u0, 1); return; }
+        if (it == nK) { seek(v0, 1); return; }
         if (++k == m_tiles) {
             k = 0;
             b = 0;
@@ -183,7 +188,7 @@ struct SlotPos {
 template <int HS>   // half head_dim of the source (32, 64 or 128)
 __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const __grid_constant__ AlignedParams P)
 {
-    extern __shared__ uint8_t smem_raw[];
+    extern __shared__ __align__(1024) uint8_t smem_raw[];
     uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     uint8_t* sB = smem + P.off_b;
     uint8_t* sRing = smem + P.off_ring;
@@ -194,8 +199,14 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     int* sSeqOff = reinterpret_cast<int*>(smem + P.off_seq);            // [batch+1]
     int* sSrcLen = sSeqOff + (P.batch + 1);                              // [batch]
     int* sTileOff = sSrcLen + P.batch;                                   // [batch+1]
-    unsigned long long* sTurnS = reinterpret_cast<unsigned long long*>(smem + P.off_turns);
-    unsigned long long* sTurnT = sTurnS + HS;
+    const unsigned long long* sTurnS = P.turns;
+    const unsigned long long* sTurnT = P.turns + 128;
+    // K-block slots: as many as fit after the fixed regions, given the actual alignment of the
+    // dynamic shared memory base (the host sized P.nslots for a 1024-byte-aligned base)
+    const uint32_t pad = (uint32_t)((uintptr_t)smem - (uintptr_t)smem_raw);
+    const uint32_t fit = ((uint32_t)kSmemMax - pad - P.off_ring) / kBlockBytes;
+    const uint32_t NS = fit < (uint32_t)P.nslots ? fit : (uint32_t)P.nslots;
+    const uint32_t NKR = NS / P.nblk + 2;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -203,9 +214,6 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
 
     for (int i = threadIdx.x; i <= P.batch; i += blockDim.x) sSeqOff[i] = __ldg(&P.seq_off[i]);
     for (int i = threadIdx.x; i < P.batch; i += blockDim.x) sSrcLen[i] = __ldg(&P.src_seq_len[i]);
-    for (int i = threadIdx.x; i < HS; i += blockDim.x) sTurnS[i] = P.rs.enabled ? __ldg(&P.rs.turns[i]) : 0ull;
-    for (int i = threadIdx.x; i < (P.dt >> 1); i += blockDim.x)
-        sTurnT[i] = P.rt.enabled ? __ldg(&P.rt.turns[i]) : 0ull;
     if (threadIdx.x == 0) {
         *sAbort = 0;
         mbar_init(bar(kBarBFull), 1);
@@ -214,11 +222,11 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             mbar_init(bar(kBarDFull + i), 1);
             mbar_init(bar(kBarDEmpty + i), kNumEpiWarps);
         }
-        for (int i = 0; i < P.nslots; ++i) {
+        for (uint32_t i = 0; i < NS; ++i) {
             mbar_init(bar(kBarFull + i), 1);
             mbar_init(bar(kBarEmpty + i), 2);   // the MMA's commit and the prologue's release
         }
-        for (int i = 0; i < P.nkready; ++i) mbar_init(bar(kBarKReady + i), kNumXfWarps);
+        for (uint32_t i = 0; i < NKR; ++i) mbar_init(bar(kBarKReady + i), kNumXfWarps);
         for (int i = 0; i < 8; ++i) mbar_init(bar(kBarPair + i), 2);
         for (int i = 0; i < 2; ++i) mbar_init(bar(kBarCsFree + i), kNumEpiWarps);
         fence_mbar_init();
@@ -250,9 +258,12 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     const long long UH = (long long)hgroups * P.m_tiles_max;
     const int u0 = (int)((long long)blockIdx.x * UH / gridDim.x);
     const int u1 = (int)((long long)(blockIdx.x + 1) * UH / gridDim.x);
+    // the V share mirrors the CTA order, so a CTA with one K unit more gets one V unit fewer
+    const int vr = gridDim.x - 1 - blockIdx.x;
+    const int v0 = (int)((long long)vr * UH / gridDim.x);
+    const int v1 = (int)((long long)(vr + 1) * UH / gridDim.x);
     const int blk_per_head = (2 * HS) / kBlockK;       // K-blocks of one source head
     const int hw = P.n_tile >> 1;
-    const uint32_t NS = (uint32_t)P.nslots;
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------ producer (one thread)
@@ -264,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             SlotPos sp{0, 0};
             bool ok = true;
             Walker wk;
-            for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+            for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
                 const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
                 // A K-blocks first: they do not depend on the weights, so at a group switch the
@@ -297,8 +308,8 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             }
             if (*sAbort) {   // let copies in flight land before leaving
                 const unsigned long long t0 = globaltimer();
-                for (uint32_t c = slot_cnt > (uint32_t)P.nslots ? slot_cnt - P.nslots : 0; c < slot_cnt; ++c)
-                    while (!mbar_try_wait(bar(kBarFull + c % P.nslots), (c / P.nslots) & 1) &&
+                for (uint32_t c = slot_cnt > NS ? slot_cnt - NS : 0; c < slot_cnt; ++c)
+                    while (!mbar_try_wait(bar(kBarFull + c % NS), (c / NS) & 1) &&
                            globaltimer() - t0 < kWaitNs) {}
                 if (b_loads)
                     while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < kWaitNs) {}
@@ -314,7 +325,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             uint32_t kr_idx = 0, kr_phase = 0;
             bool ok = true;
             Walker wk;
-            for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+            for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
                 const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
                 if (x.g != cur_g) {
@@ -329,7 +340,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 const uint32_t b0 = (uint32_t)__cvta_generic_to_shared(sB);
                 if (rot) {   // K tile: wait until the prologue has un-rotated all its K-blocks
                     if (!W.wait(bar(kBarKReady + kr_idx), kr_phase)) break;
-                    if (++kr_idx == (uint32_t)P.nkready) { kr_idx = 0; kr_phase ^= 1; }
+                    if (++kr_idx == NKR) { kr_idx = 0; kr_phase ^= 1; }
                 }
                 for (int kb = 0; kb < P.nblk; ++kb) {
                     const uint32_t slot = sp.idx;
@@ -365,7 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         const uint32_t srow_u32 = (uint32_t)__cvta_generic_to_shared(srow);
         uint32_t tcount = 0, kc = 0;   // kc: K tiles seen (selects the shared (cos, sin) buffer)
         Walker wk;
-        for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+        for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
             const AUnit& x = wk.x;
             if (x.rows <= 0) continue;
             const uint32_t buf = tcount & 1;
@@ -479,7 +490,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         uint32_t kr_idx = 0, kc = 0;
         bool ok = true;
         Walker wk;
-        for (wk.start(u0, u1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+        for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
             const AUnit& x = wk.x;
             if (x.rows <= 0) continue;
             const bool rot = x.kv == 0 && P.rs.enabled;
@@ -558,7 +569,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             fence_proxy_async();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarKReady + kr_idx));
-            if (++kr_idx == (uint32_t)P.nkready) kr_idx = 0;
+            if (++kr_idx == NKR) kr_idx = 0;
             ++kc;
             // the MMA's commit (after every prologue warp's "ready") completes the release
             if (xt == 0)
@@ -623,8 +634,8 @@ bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int H
 
 size_t aligned_map_bytes() { return sizeof(CUtensorMap); }
 
-cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps, int num_sms,
-                                        cudaStream_t stream)
+cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps,
+                                        const unsigned long long* host_turns, int num_sms, cudaStream_t stream)
 {
     TcConfig cfg = tc_config(T.in_dim, T.dt, T.ds);
     if (!cfg.ok || T.Lt > KVX_MAX_ALIGNED_LAYERS || T.batch > KVX_MAX_ALIGNED_BATCH) return cudaErrorNotSupported;
@@ -662,13 +673,16 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     P.off_bar = take(kNumBars * 8, 8);
     P.off_misc = take(16, 16);
     P.off_seq = take((unsigned)(3 * T.batch + 2) * 4, 16);
-    P.off_turns = take((unsigned)(T.ds / 2 + T.dt / 2) * 8, 16);
     P.off_ring = take(0, 1024);
-    const int avail = kSmemMax - 1024 - (int)P.off_ring;
+    // slots for a 1024-byte-aligned dynamic shared memory base (the kernel recounts for the actual
+    // base); the kernel needs a full tile's K-blocks even in the worst alignment
+    const int avail = kSmemMax - (int)P.off_ring;
     P.nslots = avail / kBlockBytes;
     if (P.nslots > kMaxSlots) P.nslots = kMaxSlots;
-    if (P.nslots < P.nblk) return cudaErrorNotSupported;
+    if ((kSmemMax - 1024 - (int)P.off_ring) / kBlockBytes < P.nblk) return cudaErrorNotSupported;
     P.nkready = P.nslots / P.nblk + 2;
+    for (int i = 0; i < T.ds / 2; ++i) P.turns[i] = T.rs.enabled ? host_turns[i] : 0ull;
+    for (int i = 0; i < T.dt / 2; ++i) P.turns[128 + i] = T.rt.enabled ? host_turns[T.ds / 2 + i] : 0ull;
     for (int j = 0; j < T.Lt; ++j) {
         P.dst_k[j] = T.dst_k[j];
         P.dst_v[j] = T.dst_v[j];
