@@ -212,8 +212,8 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     const int lane = threadIdx.x & 31;
     auto bar = [&](int i) { return (uint32_t)__cvta_generic_to_shared(&sBar[i]); };
 
-    for (int i = threadIdx.x; i <= P.batch; i += blockDim.x) sSeqOff[i] = __ldg(&P.seq_off[i]);
-    for (int i = threadIdx.x; i < P.batch; i += blockDim.x) sSrcLen[i] = __ldg(&P.src_seq_len[i]);
+    // On-chip set-up first (barriers, TMEM): with programmatic dependent launch it
+    // overlaps the tail of the previous kernel in the stream.
     if (threadIdx.x == 0) {
         *sAbort = 0;
         mbar_init(bar(kBarBFull), 1);
@@ -235,6 +235,12 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         tmem_alloc((uint32_t)__cvta_generic_to_shared(sTmemBase), P.tmem_cols);
         tmem_relinquish();
     }
+    // Nothing above touched global memory.  Every access below may read what an
+    // earlier kernel in the stream wrote (or overwrite what it reads), so wait for it.
+    grid_dependency_wait();
+    grid_launch_dependents();
+    for (int i = threadIdx.x; i <= P.batch; i += blockDim.x) sSeqOff[i] = __ldg(&P.seq_off[i]);
+    for (int i = threadIdx.x; i < P.batch; i += blockDim.x) sSrcLen[i] = __ldg(&P.src_seq_len[i]);
     __syncthreads();
     if (threadIdx.x == 0) {   // per-sequence tile offsets
         int acc = 0;
@@ -634,6 +640,26 @@ bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int H
 
 size_t aligned_map_bytes() { return sizeof(CUtensorMap); }
 
+// Launch with programmatic stream serialization: the kernel may start while the
+// previous kernel in the stream finishes; it waits (griddepcontrol.wait) before
+// touching global memory, so stream order is preserved for every memory access.
+template <typename K>
+cudaError_t launch_pdl(K kernel, int grid, cudaStream_t stream, const AlignedParams& P)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemMax;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, P);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps,
                                         const unsigned long long* host_turns, int num_sms, cudaStream_t stream)
 {
@@ -697,21 +723,21 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
             static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
             if (once != cudaSuccess) return once;
         }
-        translate_tc_aligned_kernel<32><<<grid, kThreads, kSmemMax, stream>>>(P);
+        return launch_pdl(translate_tc_aligned_kernel<32>, grid, stream, P);
         break;
     case 128:
         {
             static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
             if (once != cudaSuccess) return once;
         }
-        translate_tc_aligned_kernel<64><<<grid, kThreads, kSmemMax, stream>>>(P);
+        return launch_pdl(translate_tc_aligned_kernel<64>, grid, stream, P);
         break;
     case 256:
         {
             static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
             if (once != cudaSuccess) return once;
         }
-        translate_tc_aligned_kernel<128><<<grid, kThreads, kSmemMax, stream>>>(P);
+        return launch_pdl(translate_tc_aligned_kernel<128>, grid, stream, P);
         break;
     default:
         return cudaErrorNotSupported;
