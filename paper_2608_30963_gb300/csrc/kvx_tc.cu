@@ -38,8 +38,8 @@ constexpr int kNumSlots = 8;
 constexpr int kProducerWarp = 0;
 constexpr int kMmaWarp = 1;
 constexpr int kEpiWarp0 = 2;
-constexpr int kNumEpiWarps = 4;
-constexpr int kXfWarp0 = 6;
+constexpr int kNumEpiWarps = 8;               // two per TMEM lane quadrant, splitting the rotary pairs
+constexpr int kXfWarp0 = kEpiWarp0 + kNumEpiWarps;
 constexpr int kNumXfWarps = 8;
 constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
 constexpr int kMaxSeqCache = 512;         // sequences whose metadata is kept in shared memory
@@ -50,7 +50,8 @@ constexpr int kBarDFull = 4;               // +buf (2)
 constexpr int kBarDEmpty = 6;              // +buf (2)
 constexpr int kBarSlotFull = 8;            // +slot
 constexpr int kBarSlotEmpty = 8 + kNumSlots;
-constexpr int kNumBars = 8 + 2 * kNumSlots;
+constexpr int kBarPair = 8 + 2 * kNumSlots;   // +quad*2+{0,1}: the two epilogue warps of a quadrant meet
+constexpr int kNumBars = kBarPair + 8;
 
 struct SubMeta {
     int stage_row;   // stage row of the span start; < 0: rows are read from global memory
@@ -89,17 +90,61 @@ __device__ __forceinline__ Unit make_unit(int g, int tile, const TcLaunch& L, in
     x.j = rest / Ht;
     return x;
 }
-// The CTA's contiguous range of units (group-major, tile-minor), walked without divisions.
-struct UnitRange {
-    int g0, t0, count;
-    __device__ __forceinline__ void init(const TcLaunch& L)
+// The CTA's units: an equal share of the K units, then of the V units (each share
+// group-major, so a group's weights stay resident), walked with counters only.
+struct Walker {
+    int count, nK, it;
+    int kv, j, h, nt, tile;
+    int u0, v0, m_tiles, n_split, Ht;
+    Unit x;
+    __device__ __forceinline__ void fill()
     {
-        const long long U = (long long)L.groups * L.m_tiles;
-        const long long b = (long long)blockIdx.x * U / gridDim.x;
-        const long long e = (long long)(blockIdx.x + 1) * U / gridDim.x;
-        g0 = (int)(b / L.m_tiles);
-        t0 = (int)(b - (long long)g0 * L.m_tiles);
-        count = (int)(e - b);
+        x.j = j; x.h = h; x.kv = kv; x.nt = nt; x.tile = tile;
+        x.g = ((j * Ht + h) * 2 + kv) * n_split + nt;
+    }
+    __device__ __forceinline__ void seek(int idx, int kv_)
+    {
+        kv = kv_;
+        const int hg = idx / m_tiles;
+        tile = idx - hg * m_tiles;
+        nt = hg % n_split;
+        const int jh = hg / n_split;
+        h = jh % Ht;
+        j = jh / Ht;
+        fill();
+    }
+    __device__ __forceinline__ void start(const TcLaunch& L, int Ht_)
+    {
+        m_tiles = L.m_tiles; n_split = L.n_split; Ht = Ht_;
+        const long long UH = (long long)(L.groups / 2) * L.m_tiles;
+        const int G = gridDim.x, c = blockIdx.x, vr = G - 1 - c;
+        u0 = (int)((long long)c * UH / G);
+        const int u1 = (int)((long long)(c + 1) * UH / G);
+        v0 = (int)((long long)vr * UH / G);
+        const int v1 = (int)((long long)(vr + 1) * UH / G);
+        nK = u1 - u0;
+        count = nK + (v1 - v0);
+        it = 0;
+        if (nK > 0) seek(u0, 0);
+        else if (count > 0) seek(v0, 1);
+    }
+    __device__ __forceinline__ bool more() const { return it < count; }
+    __device__ __forceinline__ void next()
+    {
+        if (++it >= count) return;
+        if (it == nK) { seek(v0, 1); return; }
+        if (++tile == m_tiles) {
+            tile = 0;
+            if (++nt == n_split) {
+                nt = 0;
+                if (++h == Ht) { h = 0; ++j; }
+            }
+        }
+        fill();
+    }
+    __device__ __forceinline__ bool last_of_group() const
+    {
+        return it + 1 == count || it + 1 == nK || tile + 1 == m_tiles;
     }
 };
 
@@ -205,12 +250,17 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             mbar_init(bar(kBarSlotFull + i), 1);
             mbar_init(bar(kBarSlotEmpty + i), kNumXfWarps);
         }
+        for (int i = 0; i < 8; ++i) mbar_init(bar(kBarPair + i), 2);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
         tmem_alloc(smem_u32(sTmemBase), L.tmem_cols);
         tmem_relinquish();
     }
+    // Nothing above touched global memory: with programmatic dependent launch that set-up
+    // overlaps the previous kernel in the stream; everything below waits for it.
+    grid_dependency_wait();
+    grid_launch_dependents();
     unsigned long long* sTurnS = reinterpret_cast<unsigned long long*>(smem + L.off_turns);
     unsigned long long* sTurnT = sTurnS + (P.ds >> 1);
     for (int i = threadIdx.x; i < (P.ds >> 1); i += blockDim.x) sTurnS[i] = P.rs.enabled ? __ldg(&P.rs.turns[i]) : 0ull;
@@ -228,8 +278,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
 
     const Waiter W{sAbort, P.status};
     const SeqView sv{L.seq_cached ? sSeqOff : P.seq_off, L.seq_cached ? sSrcLen : P.src_seq_len, P.batch};
-    UnitRange ur;
-    ur.init(L);
+
     const int hw = L.n_tile >> 1;                 // pair half-width of an output split
     const int half_t = P.dt >> 1;
 
@@ -252,8 +301,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             }
             return true;
         };
-        for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count && ok; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
-            const Unit x = make_unit(ug, ut, L, P.Ht);
+        Walker wk;
+        for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
+            const Unit& x = wk.x;
             if (x.g != cur_g) {
                 if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
                 if (lane == 0) mbar_arrive_expect_tx(bar(kBarBFull), L.b_bytes);
@@ -381,8 +431,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         if (lane == 0) {
             int cur_g = -1;
             uint32_t b_cnt = 0, tcount = 0;
-            for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
-                const Unit x = make_unit(ug, ut, L, P.Ht);
+            Walker wk;
+            for (wk.start(L, P.Ht); wk.more(); wk.next()) {
+                const Unit& x = wk.x;
                 if (x.g != cur_g) {
                     if (!W.wait(bar(kBarBFull), b_cnt & 1)) break;
                     ++b_cnt;
@@ -402,7 +453,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 }
                 umma_commit(bar(kBarAEmpty));
                 umma_commit(bar(kBarDFull + buf));
-                const bool last_of_group = (it + 1 == ur.count) || (ut + 1 == L.m_tiles);
+                const bool last_of_group = wk.last_of_group();
                 if (last_of_group) umma_commit(bar(kBarBEmpty));
                 ++tcount;
             }
@@ -411,12 +462,15 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
     } else if (warp < kEpiWarp0 + kNumEpiWarps) {
         // ------------------------------------------------------------ epilogue
         const int quad = warp & 3;
+        const int half = (warp - kEpiWarp0) >> 2;          // which half of the rotary pairs
         const int m = quad * 32 + lane;
+        const int pc_begin = half * (hw >> 1), pc_end = pc_begin + (hw >> 1);
         uint8_t* srow = sStage + (size_t)m * L.stage_row_bytes;
         const uint32_t srow_u32 = smem_u32(srow);
         uint32_t tcount = 0;
-        for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
-            const Unit x = make_unit(ug, ut, L, P.Ht);
+        Walker wk;
+        for (wk.start(L, P.Ht); wk.more(); wk.next()) {
+            const Unit& x = wk.x;
             const uint32_t buf = tcount & 1;
             // resolve the output row while the tile is still being computed
             const int tp = x.tile * kTileM + m;
@@ -426,14 +480,19 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             if (valid) resolve_dst(P, sv, tp, dst_off, pt);
             const bool rot = x.kv == 0 && P.rt.enabled;
             float2 cs[8];
-            if (rot) rope_cs_vec<8>(sTurnT, pt, x.nt * hw, cs);
+            if (rot) rope_cs_vec<8>(sTurnT, pt, x.nt * hw + pc_begin, cs);
             if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
             tc_fence_after();
-            bulk_wait_read0();
+            // the staging row is shared by the two warps of this quadrant; the row's
+            // previous store (issued by the half-0 thread) must have read it
+            if (half == 0) bulk_wait_read0();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2));
+            if (!W.wait(bar(kBarPair + quad * 2), tcount & 1)) break;
             const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)L.n_tile;
-            for (int pc = 0; pc < hw; pc += 8) {
+            for (int pc = pc_begin; pc < pc_end; pc += 8) {
                 float2 csn[8];
-                if (rot && pc + 8 < hw) rope_cs_vec<8>(sTurnT, pt, x.nt * hw + pc + 8, csn);
+                if (rot && pc + 8 < pc_end) rope_cs_vec<8>(sTurnT, pt, x.nt * hw + pc + 8, csn);
                 uint32_t r0[8], r1[8];
                 tmem_ld8(taddr + pc, r0);
                 tmem_ld8(taddr + hw + pc, r1);
@@ -461,8 +520,11 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarDEmpty + buf));
-            if (valid && dst_off >= 0) {
-                fence_proxy_async();
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2 + 1));
+            if (!W.wait(bar(kBarPair + quad * 2 + 1), tcount & 1)) break;
+            if (half == 0 && valid && dst_off >= 0) {
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      dst_head_off(P, x.h);
                 if (L.n_split == 1) {
@@ -496,8 +558,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         }
         uint32_t sub = 0, tcount = 0;
         bool ok = true;
-        for (int it = 0, ug = ur.g0, ut = ur.t0; it < ur.count && ok; ++it, (++ut == L.m_tiles ? (ut = 0, ++ug) : 0)) {
-            const Unit x = make_unit(ug, ut, L, P.Ht);
+        Walker wk;
+        for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
+            const Unit& x = wk.x;
             const bool rot = x.kv == 0 && P.rs.enabled;
             const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
             const int g = (P.r > 1 ? x.h * P.r : x.h / P.e) + q;
@@ -508,14 +571,17 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 const SlotHdr hdr = sHdr[slot];
                 // heads of a staged sub-tile are 128 bytes off bank alignment (see producer)
                 const uint8_t* ring = sRing + hdr.offset + q * (hdr.rows * L.row_bytes + 128);
-                constexpr int kTok = kSub / kNumXfWarps;   // tokens of this warp in the sub-tile
+                // the warp's tokens of the sub-tile, kTok at a time (fewer when rows are wide,
+                // to stay within the register budget)
+                constexpr int kTok = PP == 4 ? 2 : kSub / kNumXfWarps;
+                for (int tg = 0; tg < kSub / kNumXfWarps; tg += kTok) {
                 SubMeta mt[kTok];
                 int n[kTok];
                 int maxn = 0;
                 bool copy_only = !rot;
 #pragma unroll
                 for (int u4 = 0; u4 < kTok; ++u4) {
-                    const int tt = tw + u4 * kNumXfWarps;
+                    const int tt = tw + (tg + u4) * kNumXfWarps;
                     mt[u4] = sMeta[slot * kSub + tt];
                     const bool valid = x.tile * kTileM + sq * kSub + tt < P.T_total;
                     n[u4] = valid ? max(mt[u4].hi - mt[u4].lo, 0) : -1;
@@ -526,7 +592,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     // V rows with single-token spans: the A row is the source row itself
 #pragma unroll
                     for (int u4 = 0; u4 < kTok; ++u4) {
-                        const int row = sq * kSub + tw + u4 * kNumXfWarps;
+                        const int row = sq * kSub + tw + (tg + u4) * kNumXfWarps;
                         if (n[u4] < 0) continue;
                         typename Raw<PP>::T w0, w1;
                         if (n[u4] == 1) {
@@ -613,7 +679,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
 #pragma unroll
                     for (int u4 = 0; u4 < kTok; ++u4) {
                         if (n[u4] < 0) continue;
-                        const int row = sq * kSub + tw + u4 * kNumXfWarps;
+                        const int row = sq * kSub + tw + (tg + u4) * kNumXfWarps;
                         // span mean; 1/n is exact for n = 1, 2 (the common spans)
                         const float inv_n = n[u4] > 0 ? __frcp_rn((float)n[u4]) : 0.f;
 #pragma unroll
@@ -625,6 +691,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                         store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1[u4]);
                     }
                 }
+                }   // token groups
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(kBarSlotEmpty + slot));
                 ++sub;
@@ -761,6 +828,24 @@ cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* im
     return cudaGetLastError();
 }
 
+// programmatic stream serialization: see the kernel's griddepcontrol.wait
+template <typename K>
+static cudaError_t launch_pdl_span(K kernel, int grid, cudaStream_t stream, const TranslateParams& P, const TcLaunch& L)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemMax;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, P, L);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, cudaStream_t stream)
 {
     TcLaunch L{};
@@ -768,8 +853,8 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
     L.groups = P.Lt * P.Ht * 2 * L.n_split;
     L.seq_cached = P.batch <= kMaxSeqCache;
     L.m_tiles = (P.T_total + kTileM - 1) / kTileM;
-    const long long U = (long long)L.groups * L.m_tiles;
-    const int grid = (int)(U < num_sms ? U : num_sms);
+    const long long UH = (long long)(L.groups / 2) * L.m_tiles;
+    const int grid = (int)(UH < num_sms ? UH : num_sms);
     const int pp = L.in_dim / 64;
     switch (pp) {
     case 4:
@@ -777,22 +862,19 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
             static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
             if (once != cudaSuccess) return once;
         }
-        translate_tc_kernel<4><<<grid, kThreads, kSmemMax, stream>>>(P, L);
-        break;
+        return launch_pdl_span(translate_tc_kernel<4>, grid, stream, P, L);
     case 2:
         {
             static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
             if (once != cudaSuccess) return once;
         }
-        translate_tc_kernel<2><<<grid, kThreads, kSmemMax, stream>>>(P, L);
-        break;
+        return launch_pdl_span(translate_tc_kernel<2>, grid, stream, P, L);
     case 1:
         {
             static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
             if (once != cudaSuccess) return once;
         }
-        translate_tc_kernel<1><<<grid, kThreads, kSmemMax, stream>>>(P, L);
-        break;
+        return launch_pdl_span(translate_tc_kernel<1>, grid, stream, P, L);
     default:
         return cudaErrorNotSupported;
     }
