@@ -30,7 +30,7 @@ def i32(x, device="cuda") -> Optional[torch.Tensor]:
     return None if x is None else torch.from_numpy(np.ascontiguousarray(x, np.int32)).to(device)
 
 
-class GpuRun:
+class DeviceCase:
     def __init__(self, c: Case, path: int = kvx.KVX_PATH_AUTO, paged: Optional[bool] = None,
                  explicit_layer_map: bool = True, fill=float("nan"), max_position: int = 0):
         self.c = c

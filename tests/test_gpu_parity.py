@@ -31,8 +31,8 @@ def _lib():
 
 
 def _run(c, path, paged=None, max_position=0):
-    from gpu_harness import GpuRun
-    g = GpuRun(c, path=path, paged=paged, max_position=max_position)
+    from gpu_harness import DeviceCase
+    g = DeviceCase(c, path=path, paged=paged, max_position=max_position)
     g.run()
     torch.cuda.synchronize()
     return g
@@ -119,7 +119,8 @@ def test_paged_equals_contiguous_and_batch_invariance(path):
 
 
 # ------------------------------------------------------------------ full-size, sampled rows
-FULL = ["qwen7b_to_qwen1p5b_4k", "qwen1p5b_to_gemma2b_4k", "llama70b_to_qwen7b_8k", "longctx_8k_b4"]
+FULL = ["qwen7b_to_qwen1p5b_4k", "qwen1p5b_to_gemma2b_1k", "qwen1p5b_to_gemma2b_2k", "qwen1p5b_to_gemma2b_4k",
+        "llama70b_to_qwen7b_8k", "longctx_8k_b4", "tiny_fp32"]
 
 
 @pytest.mark.parametrize("name", FULL)
@@ -173,10 +174,10 @@ def test_alignment_builder_recovers_generated_spans():
 # ------------------------------------------------------------------ device status (no faults)
 @pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
 def test_bad_spans_pages_positions_set_status_bits(path):
-    from gpu_harness import GpuRun, i32
+    from gpu_harness import DeviceCase, i32
     spec = _shrink(SPECS["longctx_8k_b4"], 2, 2)
     c = make_case(spec, [40, 20])
-    g = GpuRun(c, path=path, paged=True)
+    g = DeviceCase(c, path=path, paged=True)
     T = c.wl.total_tgt
     lo = np.arange(T, dtype=np.int32) - np.repeat(c.wl.tgt_seq_off[:-1], c.wl.tgt_len)
     hi = lo + 1
@@ -200,10 +201,10 @@ def test_bad_spans_pages_positions_set_status_bits(path):
 
 
 def test_invalid_arguments_rejected_before_launch():
-    from gpu_harness import GpuRun
+    from gpu_harness import DeviceCase
     spec = _shrink(SPECS["qwen7b_to_qwen1p5b_4k"], 2, 2)
     c = make_case(spec, [64])
-    g = GpuRun(c)
+    g = DeviceCase(c)
     g.span_hi = None          # span_lo without span_hi
     g.span_lo = g.seq_off
     with pytest.raises(kvx.KvxError) as e:
@@ -226,8 +227,8 @@ def test_identity_kernel_equals_span_kernel(base, Ls, Lt, lens):
     spec = _shrink(SPECS[base], Ls, Lt, cross_tokenizer=False)
     c = make_case(spec, lens)
     ga = _run(c, kvx.KVX_PATH_AUTO)
-    from gpu_harness import GpuRun
-    gs = GpuRun(c, path=kvx.KVX_PATH_AUTO)
+    from gpu_harness import DeviceCase
+    gs = DeviceCase(c, path=kvx.KVX_PATH_AUTO)
     lo = np.concatenate([np.arange(t, dtype=np.int32) for t in lens])
     gs.span_lo, gs.span_hi = i32(lo), i32(lo + 1)
     gs.run()
@@ -237,3 +238,78 @@ def test_identity_kernel_equals_span_kernel(base, Ls, Lt, lens):
     np.testing.assert_array_equal(ak, sk)
     np.testing.assert_array_equal(av, sv)
     assert ga.status() == 0 and gs.status() == 0
+
+
+# ------------------------------------------------------------------ largest workload: properties + sampled rows
+def test_longctx_32k_b8_device_generated():
+    """The 32K x 8 paged workload (~196K target tokens).  Inputs are drawn on the device
+    from a fixed seed (host fp32 copies would need ~30 GB).  Checks, bit-exact: paged ==
+    contiguous and identity kernel == span kernel (explicit identity spans); and sampled
+    rows against the oracle, which reads the sampled layers copied back to the host."""
+    from gpu_harness import i32, to_host
+    spec = SPECS["longctx_32k_b8"]
+    wl = synth.make_workload(spec)
+    s, d = spec.src, spec.dst
+    gen = torch.Generator(device="cuda").manual_seed(20260)
+    shape = (wl.batch, s.num_kv_heads, wl.s_max, s.head_dim)
+    ks = [torch.randn(shape, generator=gen, device="cuda").to(torch.bfloat16) for _ in range(s.num_layers)]
+    vs = [torch.randn(shape, generator=gen, device="cuda").to(torch.bfloat16) for _ in range(s.num_layers)]
+    w_k = torch.randn((d.num_layers, d.num_kv_heads, spec.group_in, d.head_dim), generator=gen, device="cuda")
+    w_v = torch.randn((d.num_layers, d.num_kv_heads, spec.group_in, d.head_dim), generator=gen, device="cuda")
+    w_k = (w_k / spec.group_in ** 0.5).to(torch.bfloat16)
+    w_v = (w_v / spec.group_in ** 0.5).to(torch.bfloat16)
+    lm = list(range(d.num_layers))
+    tr = kvx.Translator(s, d, w_k, w_v, layer_map=lm)
+    src_len, seq_off = i32(wl.src_len), i32(wl.tgt_seq_off)
+    T = wl.total_tgt
+    pt = i32(wl.page_table)
+    pool = (wl.num_pages, spec.page_size, d.num_kv_heads, d.head_dim)
+    cont = (wl.batch, d.num_kv_heads, wl.t_max, d.head_dim)
+    pk = [torch.full(pool, float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(d.num_layers)]
+    pv = [torch.full(pool, float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(d.num_layers)]
+    tr.translate(ks, vs, src_len, seq_off, T, pk, pv, page_table=pt, page_size=spec.page_size,
+                 num_pages=wl.num_pages)
+    assert tr.device_status() == 0
+    ck = [torch.full(cont, float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(d.num_layers)]
+    cv = [torch.full(cont, float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(d.num_layers)]
+    tr.translate(ks, vs, src_len, seq_off, T, ck, cv)
+    assert tr.device_status() == 0
+    lo = np.concatenate([np.arange(t, dtype=np.int32) for t in wl.tgt_len])
+    sk_ = [torch.full(cont, float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(3)]
+    sv_ = [torch.full(cont, float("nan"), dtype=torch.bfloat16, device="cuda") for _ in range(3)]
+    # span kernel on three layers (a 3-layer translator over the same source layers 0, 13, 27)
+    sub = [0, 13, 27]
+    tr3 = kvx.Translator(s, dataclasses.replace(d, num_layers=3), w_k[sub].contiguous(), w_v[sub].contiguous(),
+                         layer_map=sub)
+    tr3.translate(ks, vs, src_len, seq_off, T, sk_, sv_, span_lo=i32(lo), span_hi=i32(lo + 1))
+    assert tr3.device_status() == 0
+    torch.cuda.synchronize()
+    for b in range(wl.batch):
+        n = int(wl.tgt_len[b])
+        pages = torch.from_numpy(wl.page_table[b]).cuda().long()
+        for j in range(d.num_layers):
+            for P_, C_ in ((pk[j], ck[j]), (pv[j], cv[j])):
+                idx = torch.arange(n, device="cuda")
+                rows = P_[pages[idx // spec.page_size], idx % spec.page_size]       # [n, Ht, dt]
+                assert torch.equal(rows.transpose(0, 1).view(torch.int16), C_[b, :, :n].view(torch.int16))
+        for i, j in enumerate(sub):
+            assert torch.equal(sk_[i][b, :, :n].view(torch.int16), ck[j][b, :, :n].view(torch.int16))
+            assert torch.equal(sv_[i][b, :, :n].view(torch.int16), cv[j][b, :, :n].view(torch.int16))
+    # sampled rows against the oracle on the three layers
+    src_k = {l: to_host(ks[l]) for l in sub}
+    src_v = {l: to_host(vs[l]) for l in sub}
+    dummy = src_k[0]
+    p = oracle.OracleProblem(s, dataclasses.replace(d, num_layers=3), [0, 13, 27], wl.src_len, wl.tgt_seq_off,
+                             wl.s_max, wl.t_max, [src_k.get(l, dummy) for l in range(s.num_layers)],
+                             [src_v.get(l, dummy) for l in range(s.num_layers)],
+                             to_host(w_k[sub]), to_host(w_v[sub]))
+    r = np.random.default_rng(5)
+    gpu, ref = [], []
+    for _ in range(300):
+        i, h, kv = int(r.integers(3)), int(r.integers(d.num_kv_heads)), int(r.integers(2))
+        tp = int(r.integers(T))
+        b = int(np.searchsorted(wl.tgt_seq_off, tp, side="right") - 1)
+        t = tp - int(wl.tgt_seq_off[b])
+        gpu.append(to_host((ck if kv == 0 else cv)[sub[i]][b, h, t]))
+        ref.append(p.row(i, h, kv, tp))
+    compare(np.stack(gpu), np.stack(ref), "bf16")

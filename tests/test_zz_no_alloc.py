@@ -24,7 +24,7 @@ pytestmark = pytest.mark.gpu
 
 
 def _structs(g):
-    """C structs of a GpuRun's buffers (same marshalling as Translator.translate)."""
+    """C structs of a DeviceCase's buffers (same marshalling as Translator.translate)."""
     P = kvx._ptr
     s0 = g.src_k[0]
     src = kvx.kvx_src_kv(s0.shape[0], s0.shape[2], kvx._ptr_array(g.src_k), kvx._ptr_array(g.src_v),
@@ -47,20 +47,20 @@ CASES = [("tiny_fp32", None, None, None), ("qwen1p5b_to_gemma2b_1k", 3, 2, [130,
 
 @pytest.mark.parametrize("name,Ls,Lt,lens", CASES, ids=[c[0] for c in CASES])
 def test_static_entry_matches_translator_on_two_calls(name, Ls, Lt, lens):
-    from gpu_harness import GpuRun, to_dev, i32
+    from gpu_harness import DeviceCase, to_dev, i32
     kvx.build()
     spec = synth.config_specs()[name]
     if Ls:
         spec = _shrink(spec, Ls, Lt)
     c = make_case(spec, lens)
     # the regular entry point, CUDA-core path (the kernel the static entry point runs)
-    ref = GpuRun(c, path=kvx.KVX_PATH_SIMT, paged=False)
+    ref = DeviceCase(c, path=kvx.KVX_PATH_SIMT, paged=False)
     ref.run()
     torch.cuda.synchronize()
     rk, rv = ref.gather()
     assert ref.status() == 0
 
-    g = GpuRun(c, path=kvx.KVX_PATH_SIMT, paged=False)   # buffers only; its translator is not used
+    g = DeviceCase(c, path=kvx.KVX_PATH_SIMT, paged=False)   # buffers only; its translator is not used
     wk, wv = to_dev(c.w_k, spec.dtype), to_dev(c.w_v, spec.dtype)
     desc = g.tr.desc
     stream = torch.cuda.current_stream().cuda_stream
@@ -77,11 +77,11 @@ def test_static_entry_matches_translator_on_two_calls(name, Ls, Lt, lens):
 
 
 def test_static_entry_clears_its_status_and_rejects_oversize():
-    from gpu_harness import GpuRun, to_dev, i32
+    from gpu_harness import DeviceCase, to_dev, i32
     kvx.build()
     spec = _shrink(synth.config_specs()["qwen7b_to_qwen1p5b_4k"], 2, 2)
     c = make_case(spec, [64])
-    g = GpuRun(c, path=kvx.KVX_PATH_SIMT, paged=False)
+    g = DeviceCase(c, path=kvx.KVX_PATH_SIMT, paged=False)
     wk, wv = to_dev(c.w_k, spec.dtype), to_dev(c.w_v, spec.dtype)
     stream = torch.cuda.current_stream().cuda_stream
     lo = np.arange(64, dtype=np.int32)
