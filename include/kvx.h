@@ -203,7 +203,10 @@ typedef struct {
 
 KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_translator_info* info);
 
-/* Kernel launches one kvx_translate call makes (for launch accounting). */
+/* Kernel launches the most recent kvx_translate call on this translator made (for
+ * launch accounting): 1 for the identity-alignment and CUDA-core kernels; 2 per
+ * chunk of up to 65536 target tokens for the span kernel (a span-plan launch and the
+ * translation launch).  0 before the first call and after a call with no tokens. */
 KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
 
 /* Size of the device scratch array kvx_translate_static works in (8 MiB). */

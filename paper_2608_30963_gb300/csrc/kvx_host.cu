@@ -29,6 +29,11 @@ struct kvx_translator {
     RopeTable rs{}, rt{};
     unsigned* status = nullptr;
     TcConfig tc{};
+    // span plan of the tensor-core span kernel: sub-tile windows and per-token entries
+    // for up to kPlanTokens target tokens per launch (longer calls run in chunks)
+    static constexpr int kPlanTokens = 1 << 16;
+    void* plan = nullptr;
+    int last_launches = 0;       // kernel launches of the most recent kvx_translate
     // encoded source tensor maps of the identity-alignment kernel, a few per (target layer, K|V)
     struct MapEntry {
         const void* ptr = nullptr;
@@ -114,6 +119,7 @@ static void free_translator(kvx_translator* t)
     if (t->w) cudaFree(t->w);
     if (t->rope) cudaFree(t->rope);
     if (t->status) cudaFree(t->status);
+    if (t->plan) cudaFree(t->plan);
     delete t;
 }
 
@@ -251,6 +257,10 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0};
     }
     if (cudaMalloc(&t->status, sizeof(unsigned)) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: status allocation"); goto err; }
+    if (t->path == KVX_PATH_TCGEN05 && cudaMalloc(&t->plan, tc_plan_bytes(kvx_translator::kPlanTokens)) != cudaSuccess) {
+        st = fail(KVX_ERR_OOM, "create: span plan allocation");
+        goto err;
+    }
     if ((ce = cudaMemset(t->status, 0, sizeof(unsigned))) != cudaSuccess ||
         (ce = cudaDeviceSynchronize()) != cudaSuccess) {
         st = fail(KVX_ERR_CUDA, "create: %s", cudaGetErrorString(ce));
@@ -292,6 +302,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
         return fail(KVX_ERR_INVALID_ARG, "translate: paged target needs page_table, page_size, "
                                          "max_pages_per_seq and num_pages >= 1");
     }
+    tr->last_launches = 0;
     if (tgt->total_tokens == 0) return KVX_OK;
 
     TranslateParams P;
@@ -335,10 +346,13 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
                                                      "tensor-copy unit (strides, sizes)", tr->layer_map[j]);
             }
         ce = launch_translate_tc_aligned(P, maps, tr->host_turns, tr->num_sms, (cudaStream_t)stream);
+        tr->last_launches = 1;
     } else if (tr->path == KVX_PATH_TCGEN05) {
-        ce = launch_translate_tc(P, tr->tc, tr->num_sms, (cudaStream_t)stream);
+        ce = launch_translate_tc(P, tr->tc, tr->num_sms, tr->plan, kvx_translator::kPlanTokens, (cudaStream_t)stream,
+                                 &tr->last_launches);
     } else {
         ce = launch_translate_simt(P, D.dtype, (cudaStream_t)stream);
+        tr->last_launches = 1;
     }
     if (ce != cudaSuccess) return fail(KVX_ERR_CUDA, "translate: launch failed: %s", cudaGetErrorString(ce));
     return KVX_OK;
@@ -388,7 +402,7 @@ extern "C" KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_transla
     return KVX_OK;
 }
 
-extern "C" KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr) { return tr ? 1 : 0; }
+extern "C" KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr) { return tr ? tr->last_launches : 0; }
 
 extern "C" KVX_API kvx_status kvx_destroy(kvx_translator* tr)
 {

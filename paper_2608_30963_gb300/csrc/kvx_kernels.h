@@ -26,7 +26,11 @@ TcConfig tc_config(int in_dim, int dt, int ds);
 size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht);
 cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
                                       int dt, int n_tile, cudaStream_t stream);
-cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, cudaStream_t stream);
+size_t tc_plan_bytes(int tokens);
+// One span-plan launch and one translation launch per chunk of at most plan_tokens
+// target tokens; *launches receives the number of launches made.
+cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, void* plan,
+                                int plan_tokens, cudaStream_t stream, int* launches);
 
 // identity-alignment tensor-core path (tensor-TMA fed)
 bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch);

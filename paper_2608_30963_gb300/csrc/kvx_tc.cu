@@ -6,24 +6,30 @@
 // fused into the GEMM's prologue and epilogue.
 //
 // Persistent kernel, one CTA per SM, work unit = (group, 128-token tile) with
-// group = (target layer j, target head h, K|V, output split nt).  A CTA walks a
-// contiguous range of units, so the group's weight tile (B operand) stays in
-// shared memory across its token tiles.  Warp roles:
-//   warp 0      producer: resolves the spans of each 32-token sub-tile and
-//               streams the needed source rows into a byte ring in shared memory
-//               with cp.async.bulk (mbarrier transaction counts); loads B images.
+// group = (target layer j, target head h, K|V, output split nt).  A CTA walks an
+// equal share of the K units and of the V units, group-major, so the group's
+// weight tile (B operand) stays in shared memory across its token tiles.  Warp
+// roles:
+//   warp 0      producer: resolves the spans of each 32-token sub-tile and, per
+//               source head, copies the sub-tile's window of consecutive source
+//               rows into a byte ring in shared memory with one cp.async.bulk
+//               (mbarrier transaction counts); loads B images.
 //   warp 1      MMA: allocates TMEM, issues tcgen05.mma (M=128, N=n_tile, K=16
-//               steps over in) into a double-buffered fp32 accumulator.
-//   warps 2-5   epilogue: tcgen05.ld the accumulator (one thread per token row),
-//               apply the target RoPE, round to bf16, stage the row and write it
-//               to the target cache (contiguous or paged) with cp.async.bulk.
-//   warps 6-13  prologue: one warp per target token at a time, lanes across the
-//               in channels: undo the source RoPE of each span row, take the span
-//               mean, round to bf16 and store the A tile in the UMMA K-major
-//               128-byte-swizzled layout.
+//               steps over in, one source head's block of A at a time) into a
+//               double-buffered fp32 accumulator.
+//   warps 2-9   epilogue: tcgen05.ld the accumulator (one thread per token row,
+//               two warps per TMEM lane quadrant), apply the target RoPE, round to
+//               bf16, stage the row and write it to the target cache (contiguous
+//               or paged) with cp.async.bulk.
+//   warps 10-17 prologue: groups of d_s/16 lanes per target token, 16-byte
+//               chunks per lane: undo the source RoPE of each span row, take the
+//               span mean, round to bf16 and store A, one source head's block at
+//               a time, in the UMMA K-major 128-byte-swizzled layout.
 // Every wait is a bounded mbarrier poll: after ~1 s it records
 // KVX_DEV_WAIT_TIMEOUT, raises a CTA-wide abort flag and the kernel drains and
 // returns (no trap, no hang).
+#include <climits>
+
 #include "kvx_common.cuh"
 #include "kvx_kernels.h"
 #include "kvx_tc_common.cuh"
@@ -43,30 +49,48 @@ constexpr int kXfWarp0 = kEpiWarp0 + kNumEpiWarps;
 constexpr int kNumXfWarps = 8;
 constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
 constexpr int kMaxSeqCache = 512;         // sequences whose metadata is kept in shared memory
+constexpr int kMaxA = 2;                  // A head-block slots
 
 // barrier indices
-constexpr int kBarBFull = 0, kBarBEmpty = 1, kBarAFull = 2, kBarAEmpty = 3;
-constexpr int kBarDFull = 4;               // +buf (2)
-constexpr int kBarDEmpty = 6;              // +buf (2)
-constexpr int kBarSlotFull = 8;            // +slot
-constexpr int kBarSlotEmpty = 8 + kNumSlots;
-constexpr int kBarPair = 8 + 2 * kNumSlots;   // +quad*2+{0,1}: the two epilogue warps of a quadrant meet
+constexpr int kBarBFull = 0, kBarBEmpty = 1;
+constexpr int kBarAFull = 2;               // +A slot
+constexpr int kBarAEmpty = kBarAFull + kMaxA;
+constexpr int kBarDFull = kBarAEmpty + kMaxA;   // +buf (2)
+constexpr int kBarDEmpty = kBarDFull + 2;       // +buf (2)
+constexpr int kBarSlotFull = kBarDEmpty + 2;    // +slot
+constexpr int kBarSlotEmpty = kBarSlotFull + kNumSlots;
+constexpr int kBarPair = kBarSlotEmpty + kNumSlots;   // +quad*2+{0,1}: the two epilogue warps of a quadrant meet
 constexpr int kNumBars = kBarPair + 8;
 
-struct SubMeta {
-    int stage_row;   // stage row of the span start; < 0: rows are read from global memory
+// Span plan of one 32-token sub-tile, written by span_plan_kernel once per
+// translation and read by every (layer, head, K|V) group of the tile:
+//   header  {b0, c0, rows, 0}: the window of source rows [c0, c0 + rows) of sequence b0
+//   entries {w0, lo, hi, b} x 32, longest span first: w0 = window row of the span
+//           start (low 16 bits, signed; -1: read from global memory) | A row within
+//           the sub-tile << 16 (0xFFFF: token past the end); [lo, hi) the clamped
+//           source span of sequence b.
+
+struct SpanEnt {
+    int stage_row;   // window row of the span start; < 0: rows are read from global memory
     int lo, hi;      // source span within the sequence (hi <= lo: nothing to gather)
     int b;           // sequence
 };
 
 struct SlotHdr {
-    unsigned rows;     // rows per head staged for the sub-tile
-    unsigned offset;   // byte offset of the sub-tile's region in the ring
+    unsigned rows;     // source rows staged in the window
+    unsigned offset;   // byte offset of the window in the ring
 };
 
 struct TcLaunch {
     int n_tile, n_split, in_dim, groups, m_tiles;
-    unsigned b_bytes, a_bytes, row_bytes, stage_row_bytes, ring_bytes;
+    int t_begin, t_end;          // target tokens of this launch
+    const int4* plan_hdr;        // [sub-tiles of the launch]
+    const int4* plan_ent;        // [sub-tiles][32]
+    int r_heads;       // source heads per A row (in_dim / d_s)
+    int n_a;           // A head-block slots (1 or 2)
+    unsigned hb_bytes; // one A head-block: 128 rows x d_s bf16
+    unsigned cap_rows; // most source rows one window may stage
+    unsigned b_bytes, row_bytes, stage_row_bytes, ring_bytes;
     unsigned off_b, off_a, off_stage, off_ring, off_meta, off_hdr, off_bar, off_misc, off_seq, off_turns, off_slot;
     int seq_cached;   // per-sequence offsets and source lengths copied to shared memory
     unsigned idesc;
@@ -76,20 +100,6 @@ struct TcLaunch {
 struct Unit {
     int j, h, kv, nt, tile, g;
 };
-__device__ __forceinline__ Unit make_unit(int g, int tile, const TcLaunch& L, int Ht)
-{
-    Unit x;
-    x.g = g;
-    x.tile = tile;
-    int rest = g;
-    x.nt = rest % L.n_split;
-    rest /= L.n_split;
-    x.kv = rest & 1;
-    rest >>= 1;
-    x.h = rest % Ht;
-    x.j = rest / Ht;
-    return x;
-}
 // The CTA's units: an equal share of the K units, then of the V units (each share
 // group-major, so a group's weights stay resident), walked with counters only.
 struct Walker {
@@ -165,9 +175,17 @@ struct SeqView {
     }
 };
 
-// Source-side resolution of one target token (sequence, clamped span).
-__device__ __forceinline__ void resolve_src(const TranslateParams& P, const SeqView& sv, int tp, int& b, int& lo,
-                                            int& hi)
+// Span bounds of target token tp as given (loaded ahead of use; identity: unused).
+__device__ __forceinline__ int2 load_span(const TranslateParams& P, int tp)
+{
+    if (P.span_lo && tp < P.T_total) return make_int2(__ldg(&P.span_lo[tp]), __ldg(&P.span_hi[tp]));
+    return make_int2(0, 0);
+}
+
+// Source-side resolution of one target token (sequence, clamped span) from its
+// loaded span bounds.
+__device__ __forceinline__ void resolve_src(const TranslateParams& P, const SeqView& sv, int tp, int2 span, int& b,
+                                            int& lo, int& hi)
 {
     b = sv.find(tp);
     const int t = tp - sv.off[b];
@@ -176,7 +194,7 @@ __device__ __forceinline__ void resolve_src(const TranslateParams& P, const SeqV
         set_status(P.status, KVX_DEV_SEQ_CLAMPED);
         S = S < 0 ? 0 : P.src_max_seq;
     }
-    if (P.span_lo) { lo = __ldg(&P.span_lo[tp]); hi = __ldg(&P.span_hi[tp]); }
+    if (P.span_lo) { lo = span.x; hi = span.y; }
     else { lo = t; hi = t + 1; }
     if (lo < 0 || hi > S || hi <= lo) {
         set_status(P.status, KVX_DEV_SPAN_CLAMPED);
@@ -215,8 +233,17 @@ __device__ __forceinline__ void rope_cs_vec(const unsigned long long* turns, int
     for (int q = 0; q < PP; ++q) cs[q] = turn_cs(turns[i0 + q], p);
 }
 
+__device__ __forceinline__ void unpack8(uint4 w, float (&x)[8])
+{
+    x[0] = bf_lo(w.x); x[1] = bf_hi(w.x); x[2] = bf_lo(w.y); x[3] = bf_hi(w.y);
+    x[4] = bf_lo(w.z); x[5] = bf_hi(w.z); x[6] = bf_lo(w.w); x[7] = bf_hi(w.w);
+}
+
 // ------------------------------------------------------------------ the kernel
-template <int PP>
+// DS: source head dim.  A is built one head-block (128 tokens x DS channels of one
+// source head) at a time into a ring of n_a head-block slots, so the MMA of one
+// head-block overlaps the build of the next.
+template <int DS>
 __global__ void __launch_bounds__(kThreads, 1)
 translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_constant__ TcLaunch L)
 {
@@ -226,7 +253,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
     uint8_t* sA = smem + L.off_a;
     uint8_t* sStage = smem + L.off_stage;
     uint8_t* sRing = smem + L.off_ring;
-    SubMeta* sMeta = reinterpret_cast<SubMeta*>(smem + L.off_meta);
+    int4* sMeta = reinterpret_cast<int4*>(smem + L.off_meta);
     SlotHdr* sHdr = reinterpret_cast<SlotHdr*>(smem + L.off_hdr);
     uint64_t* sBar = reinterpret_cast<uint64_t*>(smem + L.off_bar);
     volatile int* sAbort = reinterpret_cast<volatile int*>(smem + L.off_misc);
@@ -240,8 +267,10 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         *sAbort = 0;
         mbar_init(bar(kBarBFull), 1);
         mbar_init(bar(kBarBEmpty), 1);
-        mbar_init(bar(kBarAFull), kNumXfWarps);
-        mbar_init(bar(kBarAEmpty), 1);
+        for (int i = 0; i < kMaxA; ++i) {
+            mbar_init(bar(kBarAFull + i), kNumXfWarps);
+            mbar_init(bar(kBarAEmpty + i), 1);
+        }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(kBarDFull + i), 1);
             mbar_init(bar(kBarDEmpty + i), kNumEpiWarps);
@@ -284,16 +313,21 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
 
     if (warp == kProducerWarp) {
         // ------------------------------------------------------------ producer
-        const uint64_t pol_stream = policy_evict_first();
+        // Per 32-token sub-tile and source head: one window of consecutive source
+        // rows [first span start, last span end) of the sub-tile's first sequence,
+        // copied into the byte ring with one bulk copy.  Tokens whose span falls
+        // outside the window (another sequence, a non-monotone span, a window cut at
+        // the cap) are read by the prologue from global memory.
+        const uint64_t pol_src = P.e > 1 ? policy_evict_last() : policy_evict_first();
         const uint64_t pol_keep = policy_evict_last();
-        const int r_heads = L.in_dim / P.ds;         // source heads per A row (1 when expanding)
         const bool rows_contig = P.ss == P.ds;
         int cur_g = -1;
         uint32_t b_loads = 0, issued = 0, released = 0;
         unsigned long long head = 0;                 // monotonic ring byte counter
+        unsigned head_pos = 0;                       // head modulo the ring size (kept without division)
         unsigned long long* slot_start = reinterpret_cast<unsigned long long*>(smem + L.off_slot);   // lane 0's copy
         bool ok = true;
-        // wait until sub-tile k (0-based) has been released by the prologue warps
+        // wait until sub-tile window k (0-based) has been released by the prologue warps
         auto release_upto = [&](uint32_t k) -> bool {
             while (released < k) {
                 if (!W.wait(bar(kBarSlotEmpty + released % kNumSlots), (released / kNumSlots) & 1)) return false;
@@ -302,7 +336,11 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             return true;
         };
         Walker wk;
-        for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
+        wk.start(L, P.Ht);
+        // window headers of the current unit's sub-tiles (lane sq), loaded one unit ahead
+        int4 hd = make_int4(0, 0, 0, 0);
+        if (wk.more() && lane < kSubPerTile) hd = __ldg(L.plan_hdr + wk.x.tile * kSubPerTile + lane);
+        for (; wk.more() && ok; wk.next()) {
             const Unit& x = wk.x;
             if (x.g != cur_g) {
                 if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
@@ -315,106 +353,56 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 ++b_loads;
                 cur_g = x.g;
             }
+            const int4 cur = hd;
+            {
+                Walker nx = wk;
+                nx.next();
+                if (nx.more() && lane < kSubPerTile) hd = __ldg(L.plan_hdr + nx.x.tile * kSubPerTile + lane);
+            }
             const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
             const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
-            // spans of the tile's 128 tokens, 4 per lane, loads issued together
-            int rb[kSubPerTile], rlo[kSubPerTile], rhi[kSubPerTile];
+            for (int q = 0; q < L.r_heads && ok; ++q) {
 #pragma unroll
-            for (int sq = 0; sq < kSubPerTile; ++sq) {
-                const int tp = x.tile * kTileM + sq * kSub + lane;
-                rb[sq] = -1; rlo[sq] = 0; rhi[sq] = 0;
-                if (tp < P.T_total) resolve_src(P, sv, tp, rb[sq], rlo[sq], rhi[sq]);
-            }
-#pragma unroll 1
-            for (int sq = 0; sq < kSubPerTile; ++sq) {
-                const int tp = x.tile * kTileM + sq * kSub + lane;
-                const bool valid = tp < P.T_total;
-                int b = rb[0], lo = rlo[0], hi = rhi[0];
-#pragma unroll
-                for (int z = 1; z < kSubPerTile; ++z)
-                    if (sq == z) { b = rb[z]; lo = rlo[z]; hi = rhi[z]; }
-                const int b_prev = __shfl_up_sync(0xffffffffu, b, 1);
-                const int lo_prev = __shfl_up_sync(0xffffffffu, lo, 1);
-                const int hi_prev = __shfl_up_sync(0xffffffffu, hi, 1);
-                const bool first = valid && (lane == 0 || b_prev != b);
-                const bool nonmono = valid && !first && (lo < lo_prev || hi < hi_prev);
-                const int cover = first ? lo : max(lo, hi_prev);
-                const int n_new = valid ? max(0, hi - cover) : 0;
-                int incl = n_new;
-#pragma unroll
-                for (int o = 1; o < 32; o <<= 1) {
-                    const int v = __shfl_up_sync(0xffffffffu, incl, o);
-                    if (lane >= o) incl += v;
-                }
-                const int start = incl - n_new;
-                const unsigned R = (unsigned)__shfl_sync(0xffffffffu, incl, 31);
-                const unsigned need_rows = R * (unsigned)r_heads;
-                const bool direct = __any_sync(0xffffffffu, nonmono) ||
-                                    (unsigned long long)need_rows * L.row_bytes + 128ull * r_heads > L.ring_bytes;
-                const unsigned hstride = R * L.row_bytes + 128;   // pad: the head halves of a warp hit different banks
-                const unsigned need = direct || R == 0 ? 0u : (unsigned)r_heads * hstride;
-
-                // slot reuse and ring space
-                const uint32_t slot = issued % kNumSlots;
-                if (issued >= kNumSlots && !release_upto(issued - kNumSlots + 1)) { ok = false; break; }
-                unsigned long long off = head;
-                if (need) {
-                    if (off % L.ring_bytes + need > L.ring_bytes) off = (off / L.ring_bytes + 1) * L.ring_bytes;
-                    while (true) {
-                        const unsigned long long tail = released == issued ? off : slot_start[released % kNumSlots];
-                        if (off + need - tail <= L.ring_bytes) break;
-                        if (!release_upto(released + 1)) { ok = false; break; }
-                    }
+                for (int sq = 0; sq < kSubPerTile; ++sq) {
                     if (!ok) break;
-                }
-                head = off + need;
-                slot_start[slot] = off;
-                const unsigned roff = (unsigned)(off % L.ring_bytes);
-
-                SubMeta mt;
-                mt.stage_row = direct ? -1 : start - (cover - lo);
-                mt.lo = lo;
-                mt.hi = hi;
-                mt.b = b;
-                if (!valid) { mt.lo = 0; mt.hi = 0; mt.b = 0; }
-                sMeta[slot * kSub + lane] = mt;
-                if (lane == 0) sHdr[slot] = SlotHdr{R, roff};
-                __threadfence_block();
-                __syncwarp();
-                if (lane == 0) {
-                    if (need) mbar_arrive_expect_tx(bar(kBarSlotFull + slot), need_rows * L.row_bytes);   // bytes copied
-                    else mbar_arrive(bar(kBarSlotFull + slot));
-                }
-                __syncwarp();
-                if (need) {
-                    const uint32_t ring0 = smem_u32(sRing) + roff;
-                    if (rows_contig) {
-                        // one copy per (contiguous run of source rows, head)
-                        const bool run_start = n_new > 0 && (first || lo > hi_prev);
-                        const unsigned runs = __ballot_sync(0xffffffffu, run_start);
-                        const unsigned later = lane < 31 ? runs & (0xffffffffu << (lane + 1)) : 0u;
-                        const int nxt = later ? __ffs(later) - 1 : 32;
-                        const int nxt_start = __shfl_sync(0xffffffffu, start, nxt < 32 ? nxt : lane);
-                        if (run_start) {
-                            const unsigned rows = (nxt < 32 ? (unsigned)nxt_start : R) - (unsigned)start;
-                            for (int q = 0; q < r_heads; ++q) {
-                                const __nv_bfloat16* s0 =
-                                    src + (long long)b * P.sb + (long long)(g0 + q) * P.sh + (long long)cover * P.ss;
-                                bulk_g2s(ring0 + (unsigned)q * hstride + (unsigned)start * L.row_bytes, s0,
-                                         rows * L.row_bytes, bar(kBarSlotFull + slot), pol_stream);
-                            }
+                    const int wb = __shfl_sync(0xffffffffu, cur.x, sq);
+                    const int wlo = __shfl_sync(0xffffffffu, cur.y, sq);
+                    const int wrows = __shfl_sync(0xffffffffu, cur.z, sq);
+                    const uint32_t slot = issued % kNumSlots;
+                    if (issued >= kNumSlots && !release_upto(issued - kNumSlots + 1)) { ok = false; break; }
+                    const unsigned need = (unsigned)wrows * L.row_bytes;
+                    unsigned long long off = head;
+                    unsigned pos = head_pos;
+                    if (need) {
+                        if (pos + need > L.ring_bytes) { off += L.ring_bytes - pos; pos = 0; }   // wrap to the ring start
+                        while (true) {
+                            const unsigned long long tail = released == issued ? off : slot_start[released % kNumSlots];
+                            if (off + need - tail <= L.ring_bytes) break;
+                            if (!release_upto(released + 1)) { ok = false; break; }
                         }
-                    } else {
-                        for (int s = cover; s < cover + n_new; ++s)
-                            for (int q = 0; q < r_heads; ++q) {
-                                const __nv_bfloat16* s0 =
-                                    src + (long long)b * P.sb + (long long)(g0 + q) * P.sh + (long long)s * P.ss;
-                                bulk_g2s(ring0 + (unsigned)q * hstride + (unsigned)(start + s - cover) * L.row_bytes,
-                                         s0, L.row_bytes, bar(kBarSlotFull + slot), pol_stream);
-                            }
+                        if (!ok) break;
                     }
+                    head = off + need;
+                    head_pos = pos + need == L.ring_bytes ? 0u : pos + need;
+                    slot_start[slot] = off;
+                    const uint32_t ring0 = smem_u32(sRing) + pos;
+                    const __nv_bfloat16* s0 =
+                        src + (long long)wb * P.sb + (long long)(g0 + q) * P.sh + (long long)wlo * P.ss;
+                    if (lane == 0) {
+                        // the header store is ordered before the consumers' wait by this arrive
+                        sHdr[slot] = SlotHdr{(unsigned)wrows, pos};
+                        mbar_arrive_expect_tx(bar(kBarSlotFull + slot), need + (unsigned)(kSub * sizeof(int4)));
+                        bulk_g2s(smem_u32(sMeta + slot * kSub), L.plan_ent + (size_t)(x.tile * kSubPerTile + sq) * kSub,
+                                 (uint32_t)(kSub * sizeof(int4)), bar(kBarSlotFull + slot), pol_keep);
+                        if (need && rows_contig) bulk_g2s(ring0, s0, need, bar(kBarSlotFull + slot), pol_src);
+                    }
+                    __syncwarp();
+                    if (need && !rows_contig)
+                        for (int r = lane; r < wrows; r += 32)
+                            bulk_g2s(ring0 + (unsigned)r * L.row_bytes, s0 + (long long)r * P.ss, L.row_bytes,
+                                     bar(kBarSlotFull + slot), pol_src);
+                    ++issued;
                 }
-                ++issued;
             }
         }
         // on abort, let copies already in flight land before the CTA leaves
@@ -430,9 +418,10 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             int cur_g = -1;
-            uint32_t b_cnt = 0, tcount = 0;
+            uint32_t b_cnt = 0, tcount = 0, a_cnt = 0;
+            bool ok = true;
             Walker wk;
-            for (wk.start(L, P.Ht); wk.more(); wk.next()) {
+            for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
                 const Unit& x = wk.x;
                 if (x.g != cur_g) {
                     if (!W.wait(bar(kBarBFull), b_cnt & 1)) break;
@@ -441,20 +430,27 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 }
                 const uint32_t buf = tcount & 1;
                 if (!W.wait(bar(kBarDEmpty + buf), ((tcount >> 1) & 1) ^ 1)) break;
-                if (!W.wait(bar(kBarAFull), tcount & 1)) break;
-                tc_fence_after();
                 const uint32_t d = tmem_base + buf * (uint32_t)L.n_tile;
-                const uint32_t a0 = smem_u32(sA), b0 = smem_u32(sB);
-                for (int kk = 0; kk < L.in_dim / 16; ++kk) {
-                    const uint32_t kb = kk >> 2, ko = (kk & 3) * 32;
-                    const uint64_t ad = sw128_desc(a0 + kb * (kTileM * 128) + ko);
-                    const uint64_t bd = sw128_desc(b0 + kb * (L.n_tile * 128) + ko);
-                    umma_bf16(d, ad, bd, L.idesc, kk > 0 ? 1u : 0u);
+                const uint32_t b0 = smem_u32(sB);
+                for (int q = 0; q < L.r_heads; ++q) {
+                    const uint32_t sa = a_cnt % (uint32_t)L.n_a;
+                    if (!W.wait(bar(kBarAFull + sa), (a_cnt / (uint32_t)L.n_a) & 1)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t a0 = smem_u32(sA) + sa * L.hb_bytes;
+#pragma unroll
+                    for (int kk = 0; kk < DS / 16; ++kk) {
+                        const uint32_t kb = kk >> 2, ko = (kk & 3) * 32;
+                        const uint32_t kbg = (uint32_t)q * (DS / 64) + kb;
+                        const uint64_t ad = sw128_desc(a0 + kb * (kTileM * 128) + ko);
+                        const uint64_t bd = sw128_desc(b0 + kbg * (L.n_tile * 128) + ko);
+                        umma_bf16(d, ad, bd, L.idesc, (q > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    umma_commit(bar(kBarAEmpty + sa));
+                    ++a_cnt;
                 }
-                umma_commit(bar(kBarAEmpty));
+                if (!ok) break;
                 umma_commit(bar(kBarDFull + buf));
-                const bool last_of_group = wk.last_of_group();
-                if (last_of_group) umma_commit(bar(kBarBEmpty));
+                if (wk.last_of_group()) umma_commit(bar(kBarBEmpty));
                 ++tcount;
             }
         }
@@ -473,8 +469,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             const Unit& x = wk.x;
             const uint32_t buf = tcount & 1;
             // resolve the output row while the tile is still being computed
-            const int tp = x.tile * kTileM + m;
-            const bool valid = tp < P.T_total;
+            const int tp = L.t_begin + x.tile * kTileM + m;
+            const bool valid = tp < L.t_end;
             long long dst_off = -1;
             int pt = 0;
             if (valid) resolve_dst(P, sv, tp, dst_off, pt);
@@ -539,168 +535,101 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         }
         bulk_wait0();
     } else {
-        // ------------------------------------------------------------ prologue (A tile)
+        // ------------------------------------------------------------ prologue (A head-blocks)
+        // Lanes split into groups of LPT, one target token per group; a lane owns one
+        // chunk pair: channels [8cp, 8cp+8) and their rotary partners [DS/2+8cp, ...),
+        // so each source row is read as two 16-byte loads per lane (a group reads whole
+        // 128-byte row segments: no bank conflicts on the linear window rows).
+        constexpr int LPT = DS / 16;
+        constexpr int TPW = 32 / LPT;
+        constexpr int HALF = DS / 2;
         const int tw = warp - kXfWarp0;
-        const int lanes_per_head = 32 * P.ds / L.in_dim;
-        const int q = lane / lanes_per_head;              // head within the A row
-        const int i0 = (lane % lanes_per_head) * PP;      // first rotary pair of this lane
-        const int hs = P.ds >> 1;
-        const int k0 = q * P.ds + i0, k1 = k0 + hs;       // A columns of the two halves
-        // Two heads per A row: the lanes of head 0 and head 1 rotate the same
-        // frequencies at the same positions, so each computes half and they swap.
-        const bool share = lanes_per_head == 16 && PP >= 2;
-        constexpr int kHalf = PP >= 2 ? PP / 2 : 1;
-        unsigned long long turn[PP];
+        const int cp = lane % LPT;
+        const int u = lane / LPT;
+        const uint32_t c_lo = (uint32_t)cp * 16, c_hi = (uint32_t)(HALF / 8 + cp) * 16;
+        const uint32_t a_lo = (uint32_t)((8 * cp) >> 6) * (kTileM * 128), a_hi = (uint32_t)((HALF + 8 * cp) >> 6) * (kTileM * 128);
+        const int ch_lo = cp & 7, ch_hi = ((HALF + 8 * cp) >> 3) & 7;
+        unsigned long long turn[8];
 #pragma unroll
-        for (int e = 0; e < PP; ++e) {
-            const int f = share ? i0 + (q * kHalf + e) % PP : i0 + e;   // share: first kHalf entries are own
-            turn[e] = sTurnS[f];
-        }
-        uint32_t sub = 0, tcount = 0;
+        for (int e = 0; e < 8; ++e) turn[e] = sTurnS[cp * 8 + e];
+        uint32_t sub = 0, a_cnt = 0;
         bool ok = true;
         Walker wk;
         for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
             const Unit& x = wk.x;
             const bool rot = x.kv == 0 && P.rs.enabled;
             const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
-            const int g = (P.r > 1 ? x.h * P.r : x.h / P.e) + q;
-            if (!W.wait(bar(kBarAEmpty), (tcount & 1) ^ 1)) break;
-            for (int sq = 0; sq < kSubPerTile; ++sq) {
-                const uint32_t slot = sub % kNumSlots;
-                if (!W.wait(bar(kBarSlotFull + slot), (sub / kNumSlots) & 1)) { ok = false; break; }
-                const SlotHdr hdr = sHdr[slot];
-                // heads of a staged sub-tile are 128 bytes off bank alignment (see producer)
-                const uint8_t* ring = sRing + hdr.offset + q * (hdr.rows * L.row_bytes + 128);
-                // the warp's tokens of the sub-tile, kTok at a time (fewer when rows are wide,
-                // to stay within the register budget)
-                constexpr int kTok = PP == 4 ? 2 : kSub / kNumXfWarps;
-                for (int tg = 0; tg < kSub / kNumXfWarps; tg += kTok) {
-                SubMeta mt[kTok];
-                int n[kTok];
-                int maxn = 0;
-                bool copy_only = !rot;
+            const int gbase = P.r > 1 ? x.h * P.r : x.h / P.e;
+            for (int q = 0; q < L.r_heads && ok; ++q) {
+                const uint32_t sa = a_cnt % (uint32_t)L.n_a;
+                if (!W.wait(bar(kBarAEmpty + sa), ((a_cnt / (uint32_t)L.n_a) & 1) ^ 1)) { ok = false; break; }
+                uint8_t* sAq = sA + sa * L.hb_bytes;
+                for (int sq = 0; sq < kSubPerTile; ++sq) {
+                    const uint32_t slot = sub % kNumSlots;
+                    if (!W.wait(bar(kBarSlotFull + slot), (sub / kNumSlots) & 1)) { ok = false; break; }
+                    const uint8_t* ring = sRing + sHdr[slot].offset;
+                    // entries are sorted by span length; the warp's chunk of them rotates with
+                    // the sub-tile so that long spans spread over the warps
+                    for (int tt = ((tw + 2 * sq) & (kNumXfWarps - 1)) * TPW + u; tt < kSub; tt += kNumXfWarps * TPW) {
+                        const int4 ent = sMeta[slot * kSub + tt];
+                        const int row_in = (int)((unsigned)ent.x >> 16);
+                        if (row_in >= kSub) continue;   // token past the end
+                        const int row = sq * kSub + row_in;
+                        const SpanEnt m{(int)(short)(ent.x & 0xFFFF), ent.y, ent.z, ent.w};
+                        const int n = max(m.hi - m.lo, 0);
+                        float a0[8], a1[8];
 #pragma unroll
-                for (int u4 = 0; u4 < kTok; ++u4) {
-                    const int tt = tw + (tg + u4) * kNumXfWarps;
-                    mt[u4] = sMeta[slot * kSub + tt];
-                    const bool valid = x.tile * kTileM + sq * kSub + tt < P.T_total;
-                    n[u4] = valid ? max(mt[u4].hi - mt[u4].lo, 0) : -1;
-                    maxn = max(maxn, n[u4]);
-                    copy_only = copy_only && n[u4] <= 1 && mt[u4].stage_row >= 0;
-                }
-                if (copy_only) {
-                    // V rows with single-token spans: the A row is the source row itself
-#pragma unroll
-                    for (int u4 = 0; u4 < kTok; ++u4) {
-                        const int row = sq * kSub + tw + (tg + u4) * kNumXfWarps;
-                        if (n[u4] < 0) continue;
-                        typename Raw<PP>::T w0, w1;
-                        if (n[u4] == 1) {
-                            const __nv_bfloat16* rp =
-                                reinterpret_cast<const __nv_bfloat16*>(ring + (size_t)mt[u4].stage_row * L.row_bytes);
-                            w0 = load_raw<PP>(rp + i0);
-                            w1 = load_raw<PP>(rp + hs + i0);
-                        } else {
-                            w0 = typename Raw<PP>::T{};
-                            w1 = typename Raw<PP>::T{};
-                        }
-                        *reinterpret_cast<typename Raw<PP>::T*>(sA + sw128_off(row, k0, kTileM)) = w0;
-                        *reinterpret_cast<typename Raw<PP>::T*>(sA + sw128_off(row, k1, kTileM)) = w1;
-                    }
-                } else {
-                    float a0[kTok][PP], a1[kTok][PP];
-#pragma unroll
-                    for (int u4 = 0; u4 < kTok; ++u4)
-#pragma unroll
-                        for (int e = 0; e < PP; ++e) { a0[u4][e] = 0.f; a1[u4][e] = 0.f; }
-                    for (int o = 0; o < maxn; ++o) {
-                        typename Raw<PP>::T w0[kTok], w1[kTok];
-#pragma unroll
-                        for (int u4 = 0; u4 < kTok; ++u4) {
-                            if (o < n[u4]) {
-                                const int srow = mt[u4].lo + o;
-                                const __nv_bfloat16* rp;
-                                if (mt[u4].stage_row >= 0)
-                                    rp = reinterpret_cast<const __nv_bfloat16*>(
-                                        ring + (size_t)(mt[u4].stage_row + o) * L.row_bytes);
-                                else
-                                    rp = src + (long long)mt[u4].b * P.sb + (long long)g * P.sh +
-                                         (long long)srow * P.ss;
-                                w0[u4] = load_raw<PP>(rp + i0);
-                                w1[u4] = load_raw<PP>(rp + hs + i0);
+                        for (int e = 0; e < 8; ++e) { a0[e] = 0.f; a1[e] = 0.f; }
+                        for (int o = 0; o < n; ++o) {
+                            uint4 w0, w1;
+                            if (m.stage_row >= 0) {
+                                const uint8_t* rp = ring + (size_t)(m.stage_row + o) * (DS * 2);
+                                w0 = *reinterpret_cast<const uint4*>(rp + c_lo);
+                                w1 = *reinterpret_cast<const uint4*>(rp + c_hi);
+                            } else {
+                                const uint8_t* rp = reinterpret_cast<const uint8_t*>(
+                                    src + (long long)m.b * P.sb + (long long)(gbase + q) * P.sh +
+                                    (long long)(m.lo + o) * P.ss);
+                                w0 = __ldg(reinterpret_cast<const uint4*>(rp + c_lo));
+                                w1 = __ldg(reinterpret_cast<const uint4*>(rp + c_hi));
                             }
-                        }
-#pragma unroll
-                        for (int u4 = 0; u4 < kTok; ++u4) {
-                            // rows beyond a token's span leave its sums untouched; the sine/cosine
-                            // exchange below is warp-wide, so every lane takes part
-                            const bool act = o < n[u4];
-                            float x0[PP], x1[PP];
-                            unpack(w0[u4], x0);
-                            unpack(w1[u4], x1);
+                            float x0[8], x1[8];
+                            unpack8(w0, x0);
+                            unpack8(w1, x1);
                             if (rot) {
-                                const int pos = act ? src_pos_of(P, mt[u4].b, mt[u4].lo + o) : 0;
-                                float2 cs[PP];
-                                if (share) {
+                                const int pos = src_pos_of(P, m.b, m.lo + o);
 #pragma unroll
-                                    for (int e = 0; e < kHalf; ++e) cs[e] = turn_cs(turn[e], pos);
-#pragma unroll
-                                    for (int e = 0; e < kHalf; ++e) {
-                                        cs[kHalf + e].x = __shfl_xor_sync(0xffffffffu, cs[e].x, 16);
-                                        cs[kHalf + e].y = __shfl_xor_sync(0xffffffffu, cs[e].y, 16);
-                                    }
-                                    if (q) {   // own entries are the second half of the lane's pairs
-#pragma unroll
-                                        for (int e = 0; e < kHalf; ++e) {
-                                            const float2 t = cs[e];
-                                            cs[e] = cs[kHalf + e];
-                                            cs[kHalf + e] = t;
-                                        }
-                                    }
-                                } else {
-#pragma unroll
-                                    for (int e = 0; e < PP; ++e) cs[e] = turn_cs(turn[e], pos);
-                                }
-#pragma unroll
-                                for (int e = 0; e < PP; ++e) {
+                                for (int e = 0; e < 8; ++e) {
                                     // undo the rotation: R(-theta)
-                                    const float u0 = fmaf(x0[e], cs[e].x, x1[e] * cs[e].y);
-                                    const float u1 = fmaf(x1[e], cs[e].x, -x0[e] * cs[e].y);
-                                    x0[e] = u0;
-                                    x1[e] = u1;
+                                    const float2 cs = turn_cs(turn[e], pos);
+                                    a0[e] += fmaf(x0[e], cs.x, x1[e] * cs.y);
+                                    a1[e] += fmaf(x1[e], cs.x, -x0[e] * cs.y);
                                 }
-                            }
-                            if (act) {
+                            } else {
 #pragma unroll
-                                for (int e = 0; e < PP; ++e) { a0[u4][e] += x0[e]; a1[u4][e] += x1[e]; }
+                                for (int e = 0; e < 8; ++e) { a0[e] += x0[e]; a1[e] += x1[e]; }
                             }
                         }
-                    }
-#pragma unroll
-                    for (int u4 = 0; u4 < kTok; ++u4) {
-                        if (n[u4] < 0) continue;
-                        const int row = sq * kSub + tw + (tg + u4) * kNumXfWarps;
                         // span mean; 1/n is exact for n = 1, 2 (the common spans)
-                        const float inv_n = n[u4] > 0 ? __frcp_rn((float)n[u4]) : 0.f;
-#pragma unroll
-                        for (int e = 0; e < PP; ++e) {
-                            a0[u4][e] *= inv_n;
-                            a1[u4][e] *= inv_n;
-                        }
-                        store_bf16_smem<PP>(sA + sw128_off(row, k0, kTileM), a0[u4]);
-                        store_bf16_smem<PP>(sA + sw128_off(row, k1, kTileM), a1[u4]);
+                        const float inv_n = n > 0 ? __frcp_rn((float)n) : 0.f;
+                        const uint32_t r7 = (uint32_t)(row & 7);
+                        *reinterpret_cast<uint4*>(sAq + a_lo + row * 128 + (((uint32_t)ch_lo ^ r7) << 4)) =
+                            make_uint4(pack_bf16(a0[0] * inv_n, a0[1] * inv_n), pack_bf16(a0[2] * inv_n, a0[3] * inv_n),
+                                       pack_bf16(a0[4] * inv_n, a0[5] * inv_n), pack_bf16(a0[6] * inv_n, a0[7] * inv_n));
+                        *reinterpret_cast<uint4*>(sAq + a_hi + row * 128 + (((uint32_t)ch_hi ^ r7) << 4)) =
+                            make_uint4(pack_bf16(a1[0] * inv_n, a1[1] * inv_n), pack_bf16(a1[2] * inv_n, a1[3] * inv_n),
+                                       pack_bf16(a1[4] * inv_n, a1[5] * inv_n), pack_bf16(a1[6] * inv_n, a1[7] * inv_n));
                     }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(bar(kBarSlotEmpty + slot));
+                    ++sub;
                 }
-                }   // token groups
+                if (!ok) break;
+                fence_proxy_async();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(bar(kBarSlotEmpty + slot));
-                ++sub;
+                if (lane == 0) mbar_arrive(bar(kBarAFull + sa));
+                ++a_cnt;
             }
-            if (!ok) break;
-            fence_proxy_async();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kBarAFull));
-            ++tcount;
         }
     }
 
@@ -710,6 +639,50 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         tc_fence_after();
         tmem_dealloc(tmem_base, L.tmem_cols);
     }
+}
+
+// Span plan of the sub-tiles of target tokens [t_begin, t_end): one warp per
+// 32-token sub-tile, one lane per token (layout: see the comment at the top).  Every
+// sub-tile of the launch's 128-token tiles gets a header and 32 entries; those past
+// the end get an empty window and entries marked past the end.
+__global__ void __launch_bounds__(128) span_plan_kernel(const __grid_constant__ TranslateParams P, int t_begin,
+                                                        int t_end, int cap_rows, int4* __restrict__ hdr,
+                                                        int4* __restrict__ ent)
+{
+    // the previous launch in the stream may still read the plan buffer
+    grid_dependency_wait();
+    grid_launch_dependents();
+    const int sub = (int)((blockIdx.x * blockDim.x + threadIdx.x) >> 5);
+    const int lane = threadIdx.x & 31;
+    const int nsub = (t_end - t_begin + kTileM - 1) / kTileM * kSubPerTile;
+    if (sub >= nsub) return;
+    const SeqView sv{P.seq_off, P.src_seq_len, P.batch};
+    const int tp = t_begin + sub * kSub + lane;
+    const bool valid = tp < t_end;
+    int b = -1, lo = 0, hi = 0;
+    if (valid) resolve_src(P, sv, tp, load_span(P, tp), b, lo, hi);
+    // valid tokens are a prefix of the sub-tile, so lane 0 opens the window
+    const int b0 = __shfl_sync(0xffffffffu, b, 0);
+    const int c0 = __shfl_sync(0xffffffffu, lo, 0);
+    const bool same = valid && b == b0;
+    const int hmax = __reduce_max_sync(0xffffffffu, same ? hi : INT_MIN);
+    int R = hmax == INT_MIN ? 0 : max(hmax - c0, 0);
+    R = min(R, cap_rows);
+    const bool inwin = same && lo >= c0 && hi <= c0 + R;
+    const int stage_row = inwin ? lo - c0 : -1;
+    // rank: longest span first (lengths above 3 share a bucket), then lane order;
+    // tokens past the end last
+    const int key = valid ? min(max(hi - lo, 0), 3) : -1;
+    int rank = 0;
+#pragma unroll
+    for (int k = 3; k >= -1; --k) {
+        const unsigned bal = __ballot_sync(0xffffffffu, key == k);
+        if (k > key) rank += __popc(bal);
+        else if (k == key) rank += __popc(bal & ((1u << lane) - 1u));
+    }
+    const int w0 = (int)(((unsigned)stage_row & 0xFFFFu) | ((valid ? (unsigned)lane : 0xFFFFu) << 16));
+    ent[(size_t)sub * kSub + rank] = make_int4(w0, lo, hi, b < 0 ? 0 : b);
+    if (lane == 0) hdr[sub] = make_int4(b0 < 0 ? 0 : b0, c0, R, 0);
 }
 
 // Weight images: for group g = ((j*Ht + h)*2 + kv)*n_split + nt, the B operand
@@ -765,33 +738,43 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
     if (ds != 64 && ds != 128 && ds != 256) return false;
     if (in_dim % ds) return false;
     L.in_dim = in_dim;
+    L.r_heads = in_dim / ds;
     L.n_tile = (in_dim * dt * 2 <= 65536) ? dt : dt / 2;
     L.n_split = dt / L.n_tile;
     L.b_bytes = (unsigned)(in_dim * L.n_tile * 2);
-    L.a_bytes = (unsigned)(kTileM * in_dim * 2);
+    L.hb_bytes = (unsigned)(kTileM * ds * 2);
     L.row_bytes = (unsigned)(ds * 2);
     L.stage_row_bytes = (unsigned)(L.n_tile * 2 + 16);
-    unsigned off = 0;
-    auto take = [&](unsigned bytes, unsigned align) {
-        off = (off + align - 1) / align * align;
-        const unsigned o = off;
-        off += bytes;
-        return o;
-    };
-    L.off_b = take(L.b_bytes, 1024);
-    L.off_a = take(L.a_bytes, 1024);
-    L.off_stage = take(kTileM * L.stage_row_bytes, 128);
-    L.off_meta = take(kNumSlots * kSub * sizeof(SubMeta), 16);
-    L.off_hdr = take(kNumSlots * sizeof(SlotHdr), 16);
-    L.off_bar = take(kNumBars * 8, 8);
-    L.off_misc = take(16, 16);
-    L.off_seq = take((2 * kMaxSeqCache + 1) * sizeof(int), 16);
-    L.off_turns = take((unsigned)(ds / 2 + dt / 2) * 8, 16);
-    L.off_slot = take(kNumSlots * 8, 16);
-    L.off_ring = (off + 127) / 128 * 128;
-    const int avail = kSmemMax - 1024 - (int)L.off_ring;   // 1024: alignment slack of the dynamic base
-    L.ring_bytes = avail > 0 ? (unsigned)(avail / 1024 * 1024) : 0;
-    if (L.ring_bytes < (3u * kSub * L.row_bytes + 128u) * (unsigned)(in_dim / ds)) return false;   // one worst sub-tile
+    // Two A slots when the window ring still holds three windows of 64 rows, else one.
+    for (int n_a = kMaxA; n_a >= 1; --n_a) {
+        unsigned off = 0;
+        auto take = [&](unsigned bytes, unsigned align) {
+            off = (off + align - 1) / align * align;
+            const unsigned o = off;
+            off += bytes;
+            return o;
+        };
+        L.n_a = n_a;
+        L.off_b = take(L.b_bytes, 1024);
+        L.off_a = take((unsigned)n_a * L.hb_bytes, 1024);
+        L.off_stage = take(kTileM * L.stage_row_bytes, 128);
+        L.off_meta = take(kNumSlots * kSub * sizeof(int4), 16);
+        L.off_hdr = take(kNumSlots * sizeof(SlotHdr), 16);
+        L.off_bar = take(kNumBars * 8, 8);
+        L.off_misc = take(16, 16);
+        L.off_seq = take((2 * kMaxSeqCache + 1) * sizeof(int), 16);
+        L.off_turns = take((unsigned)(ds / 2 + dt / 2) * 8, 16);
+        L.off_slot = take(kNumSlots * 8, 16);
+        L.off_ring = (off + 127) / 128 * 128;
+        const int avail = kSmemMax - 1024 - (int)L.off_ring;   // 1024: alignment slack of the dynamic base
+        L.ring_bytes = avail > 0 ? (unsigned)(avail / 1024 * 1024) : 0;
+        const unsigned rows = L.ring_bytes / L.row_bytes;
+        if (rows >= (n_a > 1 ? 3u * 64u : 2u * kSub)) {
+            L.cap_rows = rows / 2 < 3u * kSub ? rows / 2 : 3u * kSub;
+            break;
+        }
+        if (n_a == 1) return false;
+    }
     L.idesc = make_idesc(kTileM, L.n_tile);
     unsigned cols = 32;
     while (cols < 2u * (unsigned)L.n_tile) cols <<= 1;
@@ -828,58 +811,76 @@ cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* im
     return cudaGetLastError();
 }
 
-// programmatic stream serialization: see the kernel's griddepcontrol.wait
-template <typename K>
-static cudaError_t launch_pdl_span(K kernel, int grid, cudaStream_t stream, const TranslateParams& P, const TcLaunch& L)
+// programmatic stream serialization: see the kernels' griddepcontrol.wait
+template <typename K, typename... Args>
+static cudaError_t launch_pdl(K kernel, int grid, int threads, size_t smem, cudaStream_t stream, Args... args)
 {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemMax;
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, P, L);
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kernel, args...);
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, cudaStream_t stream)
+template <int DS>
+static cudaError_t launch_span_ds(int grid, cudaStream_t stream, const TranslateParams& P, const TcLaunch& L)
 {
+    static cudaError_t once =
+        cudaFuncSetAttribute(translate_tc_kernel<DS>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
+    if (once != cudaSuccess) return once;
+    return launch_pdl(translate_tc_kernel<DS>, grid, kThreads, kSmemMax, stream, P, L);
+}
+
+size_t tc_plan_bytes(int tokens)
+{
+    const size_t nsub = (size_t)(tokens + kSub - 1) / kSub;
+    return nsub * sizeof(int4) * (1 + kSub);
+}
+
+cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, void* plan,
+                                int plan_tokens, cudaStream_t stream, int* launches)
+{
+    *launches = 0;
     TcLaunch L{};
     if (!tc_layout(P.in_dim, P.dt, P.ds, L)) return cudaErrorNotSupported;
+    if (P.ds != 64 && P.ds != 128 && P.ds != 256) return cudaErrorNotSupported;
     L.groups = P.Lt * P.Ht * 2 * L.n_split;
     L.seq_cached = P.batch <= kMaxSeqCache;
-    L.m_tiles = (P.T_total + kTileM - 1) / kTileM;
-    const long long UH = (long long)(L.groups / 2) * L.m_tiles;
-    const int grid = (int)(UH < num_sms ? UH : num_sms);
-    const int pp = L.in_dim / 64;
-    switch (pp) {
-    case 4:
-        {
-            static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-            if (once != cudaSuccess) return once;
+    const int chunk = plan_tokens / kTileM * kTileM;
+    if (chunk <= 0 || !plan) return cudaErrorInvalidValue;
+    int4* hdr = reinterpret_cast<int4*>(plan);
+    int4* ent = hdr + (chunk + kSub - 1) / kSub;
+    // one plan + one translation launch per chunk of at most plan_tokens target tokens
+    for (int t0 = 0; t0 < P.T_total; t0 += chunk) {
+        const int t1 = P.T_total - t0 < chunk ? P.T_total : t0 + chunk;
+        L.t_begin = t0;
+        L.t_end = t1;
+        L.m_tiles = (t1 - t0 + kTileM - 1) / kTileM;
+        L.plan_hdr = hdr;
+        L.plan_ent = ent;
+        const int nsub = L.m_tiles * kSubPerTile;
+        cudaError_t e = launch_pdl(span_plan_kernel, (nsub + 3) / 4, 128, 0, stream, P, t0, t1, (int)L.cap_rows, hdr, ent);
+        if (e != cudaSuccess) return e;
+        ++*launches;
+        const long long UH = (long long)(L.groups / 2) * L.m_tiles;
+        const int grid = (int)(UH < num_sms ? UH : num_sms);
+        switch (P.ds) {
+        case 256: e = launch_span_ds<256>(grid, stream, P, L); break;
+        case 128: e = launch_span_ds<128>(grid, stream, P, L); break;
+        default: e = launch_span_ds<64>(grid, stream, P, L); break;
         }
-        return launch_pdl_span(translate_tc_kernel<4>, grid, stream, P, L);
-    case 2:
-        {
-            static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-            if (once != cudaSuccess) return once;
-        }
-        return launch_pdl_span(translate_tc_kernel<2>, grid, stream, P, L);
-    case 1:
-        {
-            static cudaError_t once = cudaFuncSetAttribute(translate_tc_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-            if (once != cudaSuccess) return once;
-        }
-        return launch_pdl_span(translate_tc_kernel<1>, grid, stream, P, L);
-    default:
-        return cudaErrorNotSupported;
+        if (e != cudaSuccess) return e;
+        ++*launches;
     }
     (void)cfg;
-    return cudaGetLastError();
+    return cudaSuccess;
 }
 
 }  // namespace kvx
