@@ -79,7 +79,6 @@ __device__ __forceinline__ float2 turn_cs(unsigned long long G, int p)
     return make_float2(cs, sn);
 }
 
-// (cos, sin) of angle p * f_i (p already clamped to [0, max_position)).
 __device__ __forceinline__ float2 rope_cs(const RopeTable& t, int p, int i)
 {
     return turn_cs(__ldg(&t.turns[i]), p);

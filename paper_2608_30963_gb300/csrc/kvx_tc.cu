@@ -76,11 +76,6 @@ struct SpanEnt {
     int b;           // sequence
 };
 
-struct SlotHdr {
-    unsigned rows;     // source rows staged in the window
-    unsigned offset;   // byte offset of the window in the ring
-};
-
 struct TcLaunch {
     int n_tile, n_split, in_dim, groups, m_tiles;
     int t_begin, t_end;          // target tokens of this launch
@@ -90,8 +85,9 @@ struct TcLaunch {
     int n_a;           // A head-block slots (1 or 2)
     unsigned hb_bytes; // one A head-block: 128 rows x d_s bf16
     unsigned cap_rows; // most source rows one window may stage
-    unsigned b_bytes, row_bytes, stage_row_bytes, ring_bytes;
-    unsigned off_b, off_a, off_stage, off_ring, off_meta, off_hdr, off_bar, off_misc, off_seq, off_turns, off_slot;
+    int n_slots;       // window slots of slot_bytes each
+    unsigned b_bytes, row_bytes, stage_row_bytes, slot_bytes;
+    unsigned off_b, off_a, off_stage, off_ring, off_meta, off_bar, off_misc, off_seq, off_turns;
     int seq_cached;   // per-sequence offsets and source lengths copied to shared memory
     unsigned idesc;
     unsigned tmem_cols;
@@ -233,12 +229,6 @@ __device__ __forceinline__ void rope_cs_vec(const unsigned long long* turns, int
     for (int q = 0; q < PP; ++q) cs[q] = turn_cs(turns[i0 + q], p);
 }
 
-__device__ __forceinline__ void unpack8(uint4 w, float (&x)[8])
-{
-    x[0] = bf_lo(w.x); x[1] = bf_hi(w.x); x[2] = bf_lo(w.y); x[3] = bf_hi(w.y);
-    x[4] = bf_lo(w.z); x[5] = bf_hi(w.z); x[6] = bf_lo(w.w); x[7] = bf_hi(w.w);
-}
-
 // ------------------------------------------------------------------ the kernel
 // DS: source head dim.  A is built one head-block (128 tokens x DS channels of one
 // source head) at a time into a ring of n_a head-block slots, so the MMA of one
@@ -254,7 +244,6 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
     uint8_t* sStage = smem + L.off_stage;
     uint8_t* sRing = smem + L.off_ring;
     int4* sMeta = reinterpret_cast<int4*>(smem + L.off_meta);
-    SlotHdr* sHdr = reinterpret_cast<SlotHdr*>(smem + L.off_hdr);
     uint64_t* sBar = reinterpret_cast<uint64_t*>(smem + L.off_bar);
     volatile int* sAbort = reinterpret_cast<volatile int*>(smem + L.off_misc);
     uint32_t* sTmemBase = reinterpret_cast<uint32_t*>(smem + L.off_misc + 4);
@@ -322,19 +311,10 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         const uint64_t pol_keep = policy_evict_last();
         const bool rows_contig = P.ss == P.ds;
         int cur_g = -1;
-        uint32_t b_loads = 0, issued = 0, released = 0;
-        unsigned long long head = 0;                 // monotonic ring byte counter
-        unsigned head_pos = 0;                       // head modulo the ring size (kept without division)
-        unsigned long long* slot_start = reinterpret_cast<unsigned long long*>(smem + L.off_slot);   // lane 0's copy
+        uint32_t b_loads = 0, issued = 0;
+        int wslot = 0;             // window slot of the next window
+        uint32_t wphase = 0;       // how often the slots have been cycled, mod 2
         bool ok = true;
-        // wait until sub-tile window k (0-based) has been released by the prologue warps
-        auto release_upto = [&](uint32_t k) -> bool {
-            while (released < k) {
-                if (!W.wait(bar(kBarSlotEmpty + released % kNumSlots), (released / kNumSlots) & 1)) return false;
-                ++released;
-            }
-            return true;
-        };
         Walker wk;
         wk.start(L, P.Ht);
         // window headers of the current unit's sub-tiles (lane sq), loaded one unit ahead
@@ -368,29 +348,19 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     const int wb = __shfl_sync(0xffffffffu, cur.x, sq);
                     const int wlo = __shfl_sync(0xffffffffu, cur.y, sq);
                     const int wrows = __shfl_sync(0xffffffffu, cur.z, sq);
-                    const uint32_t slot = issued % kNumSlots;
-                    if (issued >= kNumSlots && !release_upto(issued - kNumSlots + 1)) { ok = false; break; }
-                    const unsigned need = (unsigned)wrows * L.row_bytes;
-                    unsigned long long off = head;
-                    unsigned pos = head_pos;
-                    if (need) {
-                        if (pos + need > L.ring_bytes) { off += L.ring_bytes - pos; pos = 0; }   // wrap to the ring start
-                        while (true) {
-                            const unsigned long long tail = released == issued ? off : slot_start[released % kNumSlots];
-                            if (off + need - tail <= L.ring_bytes) break;
-                            if (!release_upto(released + 1)) { ok = false; break; }
-                        }
-                        if (!ok) break;
+                    const int slot = wslot;
+                    // the slot's previous window must have been released by the prologue warps
+                    if (issued >= (uint32_t)L.n_slots && !W.wait(bar(kBarSlotEmpty + slot), wphase ^ 1)) {
+                        ok = false;
+                        break;
                     }
-                    head = off + need;
-                    head_pos = pos + need == L.ring_bytes ? 0u : pos + need;
-                    slot_start[slot] = off;
+                    if (++wslot == L.n_slots) { wslot = 0; wphase ^= 1; }
+                    const unsigned need = (unsigned)wrows * L.row_bytes;
+                    const unsigned pos = (unsigned)slot * L.slot_bytes;
                     const uint32_t ring0 = smem_u32(sRing) + pos;
                     const __nv_bfloat16* s0 =
                         src + (long long)wb * P.sb + (long long)(g0 + q) * P.sh + (long long)wlo * P.ss;
                     if (lane == 0) {
-                        // the header store is ordered before the consumers' wait by this arrive
-                        sHdr[slot] = SlotHdr{(unsigned)wrows, pos};
                         mbar_arrive_expect_tx(bar(kBarSlotFull + slot), need + (unsigned)(kSub * sizeof(int4)));
                         bulk_g2s(smem_u32(sMeta + slot * kSub), L.plan_ent + (size_t)(x.tile * kSubPerTile + sq) * kSub,
                                  (uint32_t)(kSub * sizeof(int4)), bar(kBarSlotFull + slot), pol_keep);
@@ -408,9 +378,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         // on abort, let copies already in flight land before the CTA leaves
         if (*sAbort) {
             const unsigned long long t0 = globaltimer();
-            for (uint32_t c = issued > kNumSlots ? issued - kNumSlots : 0; c < issued; ++c)
-                while (!mbar_try_wait(bar(kBarSlotFull + c % kNumSlots), (c / kNumSlots) & 1) &&
-                       globaltimer() - t0 < kWaitNs) {}
+            const uint32_t ns = (uint32_t)L.n_slots;
+            for (uint32_t c = issued > ns ? issued - ns : 0; c < issued; ++c)
+                while (!mbar_try_wait(bar(kBarSlotFull + c % ns), (c / ns) & 1) && globaltimer() - t0 < kWaitNs) {}
             if (b_loads)
                 while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < kWaitNs) {}
         }
@@ -493,25 +463,14 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 tmem_ld8(taddr + pc, r0);
                 tmem_ld8(taddr + hw + pc, r1);
                 tmem_ld_wait();
-                float y0[8], y1[8];
-#pragma unroll
-                for (int e = 0; e < 8; ++e) { y0[e] = __uint_as_float(r0[e]); y1[e] = __uint_as_float(r1[e]); }
+                uint4 out0, out1;
+                rotate8_to_bf16(r0, r1, cs, rot, out0, out1);
                 if (rot) {
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) {
-                        const float a = y0[e], bb = y1[e];
-                        y0[e] = fmaf(a, cs[e].x, -bb * cs[e].y);
-                        y1[e] = fmaf(bb, cs[e].x, a * cs[e].y);
-                    }
 #pragma unroll
                     for (int e = 0; e < 8; ++e) cs[e] = csn[e];
                 }
-                *reinterpret_cast<uint4*>(srow + pc * 2) =
-                    make_uint4(pack_bf16(y0[0], y0[1]), pack_bf16(y0[2], y0[3]), pack_bf16(y0[4], y0[5]),
-                               pack_bf16(y0[6], y0[7]));
-                *reinterpret_cast<uint4*>(srow + (hw + pc) * 2) =
-                    make_uint4(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]), pack_bf16(y1[4], y1[5]),
-                               pack_bf16(y1[6], y1[7]));
+                *reinterpret_cast<uint4*>(srow + pc * 2) = out0;
+                *reinterpret_cast<uint4*>(srow + (hw + pc) * 2) = out1;
             }
             tc_fence_before();
             __syncwarp();
@@ -552,7 +511,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         unsigned long long turn[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) turn[e] = sTurnS[cp * 8 + e];
-        uint32_t sub = 0, a_cnt = 0;
+        uint32_t a_cnt = 0;
+        int wslot = 0;
+        uint32_t wphase = 0;
         bool ok = true;
         Walker wk;
         for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
@@ -565,9 +526,10 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 if (!W.wait(bar(kBarAEmpty + sa), ((a_cnt / (uint32_t)L.n_a) & 1) ^ 1)) { ok = false; break; }
                 uint8_t* sAq = sA + sa * L.hb_bytes;
                 for (int sq = 0; sq < kSubPerTile; ++sq) {
-                    const uint32_t slot = sub % kNumSlots;
-                    if (!W.wait(bar(kBarSlotFull + slot), (sub / kNumSlots) & 1)) { ok = false; break; }
-                    const uint8_t* ring = sRing + sHdr[slot].offset;
+                    const int slot = wslot;
+                    if (!W.wait(bar(kBarSlotFull + slot), wphase)) { ok = false; break; }
+                    if (++wslot == L.n_slots) { wslot = 0; wphase ^= 1; }
+                    const uint8_t* ring = sRing + (size_t)slot * L.slot_bytes;
                     // entries are sorted by span length; the warp's chunk of them rotates with
                     // the sub-tile so that long spans spread over the warps
                     for (int tt = ((tw + 2 * sq) & (kNumXfWarps - 1)) * TPW + u; tt < kSub; tt += kNumXfWarps * TPW) {
@@ -593,36 +555,46 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                                 w0 = __ldg(reinterpret_cast<const uint4*>(rp + c_lo));
                                 w1 = __ldg(reinterpret_cast<const uint4*>(rp + c_hi));
                             }
-                            float x0[8], x1[8];
-                            unpack8(w0, x0);
-                            unpack8(w1, x1);
+                            const uint32_t v0[4] = {w0.x, w0.y, w0.z, w0.w}, v1[4] = {w1.x, w1.y, w1.z, w1.w};
                             if (rot) {
                                 const int pos = src_pos_of(P, m.b, m.lo + o);
 #pragma unroll
-                                for (int e = 0; e < 8; ++e) {
-                                    // undo the rotation: R(-theta)
-                                    const float2 cs = turn_cs(turn[e], pos);
-                                    a0[e] += fmaf(x0[e], cs.x, x1[e] * cs.y);
-                                    a1[e] += fmaf(x1[e], cs.x, -x0[e] * cs.y);
+                                for (int k = 0; k < 4; ++k) {   // undo the rotation: R(-theta)
+                                    const float2 ca = turn_cs(turn[2 * k], pos), cb = turn_cs(turn[2 * k + 1], pos);
+                                    if (o == 0) {
+                                        unrotate1(bf_lo(v0[k]), bf_lo(v1[k]), ca, a0[2 * k], a1[2 * k]);
+                                        unrotate1(bf_hi(v0[k]), bf_hi(v1[k]), cb, a0[2 * k + 1], a1[2 * k + 1]);
+                                    } else {
+                                        unrotate_acc(bf_lo(v0[k]), bf_lo(v1[k]), ca, a0[2 * k], a1[2 * k]);
+                                        unrotate_acc(bf_hi(v0[k]), bf_hi(v1[k]), cb, a0[2 * k + 1], a1[2 * k + 1]);
+                                    }
                                 }
                             } else {
 #pragma unroll
-                                for (int e = 0; e < 8; ++e) { a0[e] += x0[e]; a1[e] += x1[e]; }
+                                for (int k = 0; k < 4; ++k) {
+                                    a0[2 * k] += bf_lo(v0[k]);
+                                    a0[2 * k + 1] += bf_hi(v0[k]);
+                                    a1[2 * k] += bf_lo(v1[k]);
+                                    a1[2 * k + 1] += bf_hi(v1[k]);
+                                }
                             }
                         }
                         // span mean; 1/n is exact for n = 1, 2 (the common spans)
                         const float inv_n = n > 0 ? __frcp_rn((float)n) : 0.f;
+                        uint32_t o0[4], o1[4];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            o0[k] = pack_bf16(a0[2 * k] * inv_n, a0[2 * k + 1] * inv_n);
+                            o1[k] = pack_bf16(a1[2 * k] * inv_n, a1[2 * k + 1] * inv_n);
+                        }
                         const uint32_t r7 = (uint32_t)(row & 7);
                         *reinterpret_cast<uint4*>(sAq + a_lo + row * 128 + (((uint32_t)ch_lo ^ r7) << 4)) =
-                            make_uint4(pack_bf16(a0[0] * inv_n, a0[1] * inv_n), pack_bf16(a0[2] * inv_n, a0[3] * inv_n),
-                                       pack_bf16(a0[4] * inv_n, a0[5] * inv_n), pack_bf16(a0[6] * inv_n, a0[7] * inv_n));
+                            make_uint4(o0[0], o0[1], o0[2], o0[3]);
                         *reinterpret_cast<uint4*>(sAq + a_hi + row * 128 + (((uint32_t)ch_hi ^ r7) << 4)) =
-                            make_uint4(pack_bf16(a1[0] * inv_n, a1[1] * inv_n), pack_bf16(a1[2] * inv_n, a1[3] * inv_n),
-                                       pack_bf16(a1[4] * inv_n, a1[5] * inv_n), pack_bf16(a1[6] * inv_n, a1[7] * inv_n));
+                            make_uint4(o1[0], o1[1], o1[2], o1[3]);
                     }
                     __syncwarp();
                     if (lane == 0) mbar_arrive(bar(kBarSlotEmpty + slot));
-                    ++sub;
                 }
                 if (!ok) break;
                 fence_proxy_async();
@@ -745,7 +717,11 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
     L.hb_bytes = (unsigned)(kTileM * ds * 2);
     L.row_bytes = (unsigned)(ds * 2);
     L.stage_row_bytes = (unsigned)(L.n_tile * 2 + 16);
-    // Two A slots when the window ring still holds three windows of 64 rows, else one.
+    // Window slots of 48 source rows: a 32-token sub-tile of spans averaging 1.3
+    // tokens needs ~42; tokens whose rows fall past the cap are read from global
+    // memory.  Two A slots when four window slots still fit, else one.
+    L.cap_rows = 48;
+    L.slot_bytes = L.cap_rows * L.row_bytes;
     for (int n_a = kMaxA; n_a >= 1; --n_a) {
         unsigned off = 0;
         auto take = [&](unsigned bytes, unsigned align) {
@@ -759,20 +735,15 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
         L.off_a = take((unsigned)n_a * L.hb_bytes, 1024);
         L.off_stage = take(kTileM * L.stage_row_bytes, 128);
         L.off_meta = take(kNumSlots * kSub * sizeof(int4), 16);
-        L.off_hdr = take(kNumSlots * sizeof(SlotHdr), 16);
         L.off_bar = take(kNumBars * 8, 8);
         L.off_misc = take(16, 16);
         L.off_seq = take((2 * kMaxSeqCache + 1) * sizeof(int), 16);
         L.off_turns = take((unsigned)(ds / 2 + dt / 2) * 8, 16);
-        L.off_slot = take(kNumSlots * 8, 16);
         L.off_ring = (off + 127) / 128 * 128;
         const int avail = kSmemMax - 1024 - (int)L.off_ring;   // 1024: alignment slack of the dynamic base
-        L.ring_bytes = avail > 0 ? (unsigned)(avail / 1024 * 1024) : 0;
-        const unsigned rows = L.ring_bytes / L.row_bytes;
-        if (rows >= (n_a > 1 ? 3u * 64u : 2u * kSub)) {
-            L.cap_rows = rows / 2 < 3u * kSub ? rows / 2 : 3u * kSub;
-            break;
-        }
+        const int slots = avail > 0 ? (int)((unsigned)avail / L.slot_bytes) : 0;
+        L.n_slots = slots < kNumSlots ? slots : kNumSlots;
+        if (L.n_slots >= (n_a > 1 ? 4 : 2)) break;
         if (n_a == 1) return false;
     }
     L.idesc = make_idesc(kTileM, L.n_tile);

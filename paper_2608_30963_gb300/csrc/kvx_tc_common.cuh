@@ -214,6 +214,51 @@ __device__ __forceinline__ uint32_t pack_bf16(float a, float b)
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Undo a rotation on one rotary pair (x0 from the first half, x1 from the second):
+//   u0 = x0 cos + x1 sin,  u1 = x1 cos - x0 sin,
+// evaluated as fma(x0, cos, x1 sin) and fma(x1, cos, -(x0 sin)), the order the
+// identity-alignment kernel uses, so the two kernels agree bit for bit on
+// single-token spans.
+__device__ __forceinline__ void unrotate1(float x0, float x1, float2 cs, float& u0, float& u1)
+{
+    u0 = fmaf(x0, cs.x, x1 * cs.y);
+    u1 = fmaf(x1, cs.x, -x0 * cs.y);
+}
+// The same, accumulated onto (a0, a1) for the later rows of a span:
+// a0 = fma(x1, sin, fma(x0, cos, a0)), a1 = fma(x0, -sin, fma(x1, cos, a1)).
+__device__ __forceinline__ void unrotate_acc(float x0, float x1, float2 cs, float& a0, float& a1)
+{
+    a0 = fmaf(x1, cs.y, fmaf(x0, cs.x, a0));
+    a1 = fmaf(x0, -cs.y, fmaf(x1, cs.x, a1));
+}
+
+// Apply a rotation to one rotary pair:  y0 = x0 cos - x1 sin,  y1 = x1 cos + x0 sin,
+// evaluated as fma(x0, cos, -(x1 sin)) and fma(x1, cos, x0 sin), as in the
+// identity-alignment kernel's epilogue.
+__device__ __forceinline__ void rotate1(float x0, float x1, float2 cs, float& y0, float& y1)
+{
+    const float a = x0, b = x1;
+    y0 = fmaf(a, cs.x, -b * cs.y);
+    y1 = fmaf(b, cs.x, a * cs.y);
+}
+
+// The fp32 of two 8-column TMEM loads (columns c..c+7 of the first and second
+// rotary halves) rotated by cs[0..7] (rot) and rounded to bf16: out0 = first half,
+// out1 = second half.
+__device__ __forceinline__ void rotate8_to_bf16(const uint32_t (&r0)[8], const uint32_t (&r1)[8], const float2 (&cs)[8],
+                                                bool rot, uint4& out0, uint4& out1)
+{
+    float y0[8], y1[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        y0[e] = __uint_as_float(r0[e]);
+        y1[e] = __uint_as_float(r1[e]);
+        if (rot) rotate1(y0[e], y1[e], cs[e], y0[e], y1[e]);
+    }
+    out0 = make_uint4(pack_bf16(y0[0], y0[1]), pack_bf16(y0[2], y0[3]), pack_bf16(y0[4], y0[5]), pack_bf16(y0[6], y0[7]));
+    out1 = make_uint4(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]), pack_bf16(y1[4], y1[5]), pack_bf16(y1[6], y1[7]));
+}
+
 // PP consecutive bf16 values (PP in {1,2,4}) as one raw load.
 template <int PP> struct Raw;
 template <> struct Raw<4> { using T = uint2; };
