@@ -238,7 +238,9 @@ __global__ void __launch_bounds__(kThreads, 1)
 translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_constant__ TcLaunch L)
 {
     extern __shared__ uint8_t smem_raw[];
-    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    // 1024-byte aligned base, derived from smem_raw by pointer arithmetic so that the
+    // compiler keeps every access below in the shared address space
+    uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     uint8_t* sB = smem + L.off_b;
     uint8_t* sA = smem + L.off_a;
     uint8_t* sStage = smem + L.off_stage;

@@ -189,7 +189,10 @@ template <int HS>   // half head_dim of the source (32, 64 or 128)
 __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const __grid_constant__ AlignedParams P)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
-    uint8_t* smem = (uint8_t*)(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    // 1024-byte aligned base, derived from smem_raw by pointer arithmetic so that the
+    // compiler keeps every access below in the shared address space
+    const uint32_t pad = (1024u - (smem_u32(smem_raw) & 1023u)) & 1023u;
+    uint8_t* smem = smem_raw + pad;
     uint8_t* sB = smem + P.off_b;
     uint8_t* sRing = smem + P.off_ring;
     uint8_t* sStage = smem + P.off_stage;
@@ -203,7 +206,6 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     const unsigned long long* sTurnT = P.turns + 128;
     // K-block slots: as many as fit after the fixed regions, given the actual alignment of the
     // dynamic shared memory base (the host sized P.nslots for a 1024-byte-aligned base)
-    const uint32_t pad = (uint32_t)((uintptr_t)smem - (uintptr_t)smem_raw);
     const uint32_t fit = ((uint32_t)kSmemMax - pad - P.off_ring) / kBlockBytes;
     const uint32_t NS = fit < (uint32_t)P.nslots ? fit : (uint32_t)P.nslots;
     const uint32_t NKR = NS / P.nblk + 2;
