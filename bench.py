@@ -81,7 +81,7 @@ def _oracle_worker(args):
     l0 = int(lm[0])
     k = synth.source_kv(wl, l0, 0)
     if spec.src.rope_base > 0:
-        k = oracle.rope_cache(k, spec.src.rope_base)
+        k = oracle.rope_cache(k, spec.src)
         if spec.dtype == "bf16":
             k = synth.bf16_round(k)
     v = synth.source_kv(wl, l0, 1)
@@ -177,8 +177,8 @@ class ClockSampler:
 
 # ----------------------------------------------------------------------------- input synthesis
 def rotate_np(x: np.ndarray, base: float) -> np.ndarray:
-    """Apply half-split RoPE at positions 0..S-1 (input synthesis: the post-RoPE
-    keys a source model's prefill stores)."""
+    """Apply half-split RoPE (plain frequency schedule) at positions 0..S-1 (input
+    synthesis: the post-RoPE keys a source model's prefill stores)."""
     B, H, S, d = x.shape
     h = d // 2
     ang = np.arange(S, dtype=np.float64)[:, None] * np.power(base, -2.0 * np.arange(h) / d)[None, :]
@@ -244,6 +244,8 @@ def main():
     for l in mapped:
         k = synth.source_kv(wl, l, 0)
         if spec.src.rope_base > 0:
+            if spec.src.rope_type != synth.ROPE_DEFAULT:
+                raise SystemExit("bench input synthesis rotates with the plain RoPE schedule only")
             k = rotate_np(k, spec.src.rope_base)
         host_k[l] = to_torch(k, spec.dtype, torch, pin=True)
         host_v[l] = to_torch(synth.source_kv(wl, l, 1), spec.dtype, torch, pin=True)

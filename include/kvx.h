@@ -71,12 +71,35 @@ typedef enum {
 
 #define KVX_MAX_TARGET_LAYERS 128  /* target layers a translator may have */
 
-/* Geometry of one model's KV cache. */
+/* Frequency schedule of a model's rotary encoding.  The plain schedule rotates channel pair
+ * (i, i+d/2) by p * f_i with f_i = base^(-2i/d).  The paper names the model pairs it evaluates
+ * (Section 6.1) but not their position encodings; these schedules are the ones the named
+ * families publish (Llama-3.1 ships the LLAMA3 schedule). */
+typedef enum {
+    KVX_ROPE_DEFAULT = 0,       /* f_i = base^(-2i/d) */
+    KVX_ROPE_LINEAR = 1,        /* position interpolation: angle (p / factor) * f_i */
+    KVX_ROPE_LLAMA3 = 2         /* frequency-dependent: with wavelength w_i = 2 pi / f_i,
+                                   lo_w = original_max_position / low_freq_factor and
+                                   hi_w = original_max_position / high_freq_factor,
+                                   f_i is kept where w_i < hi_w, divided by factor where
+                                   w_i > lo_w, and in between blended as
+                                   (1 - m) f_i / factor + m f_i with
+                                   m = (original_max_position / w_i - low_freq_factor) /
+                                       (high_freq_factor - low_freq_factor) */
+} kvx_rope_type;
+
+/* Geometry of one model's KV cache.  A zero-initialised tail (rope_type 0) is the plain
+ * schedule. */
 typedef struct {
     int32_t num_layers;         /* N in KV_M(C) = {(K^(1),V^(1)) .. (K^(N),V^(N))} (Section 2.1) */
     int32_t num_kv_heads;       /* KV heads per layer */
     int32_t head_dim;           /* channels per head: 64, 128 or 256 */
     double  rope_base;          /* RoPE base of K; <= 0 means K carries no rotary encoding */
+    int32_t rope_type;          /* kvx_rope_type */
+    double  rope_factor;        /* LINEAR, LLAMA3: scale factor, > 0 */
+    double  rope_low_freq_factor;       /* LLAMA3: > 0 */
+    double  rope_high_freq_factor;      /* LLAMA3: > rope_low_freq_factor */
+    int32_t rope_original_max_position; /* LLAMA3: context length of the unscaled model, > 0 */
 } kvx_model_geom;
 
 /* Translator description (the theta of T_theta, Section 5, plus the layer alignment). */
@@ -104,7 +127,8 @@ typedef struct kvx_translator kvx_translator;
  * The library copies the weights into its own device memory (re-laid out for its kernels) and
  * builds its RoPE tables; the caller may free its copies on return.  Synchronous on the
  * current device.  Returns KVX_ERR_UNSUPPORTED unless one head count divides the other,
- * both head dims are in {64, 128, 256} and in <= 512 (in <= 256 for the tcgen05 path).
+ * both head dims are in {64, 128, 256} and in <= 512 (in <= 256 for the tcgen05 path), and
+ * KVX_ERR_INVALID_ARG for an unknown rope_type or out-of-range schedule parameters.
  * On success *out owns device memory until kvx_destroy. */
 KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* desc, const void* w_k, const void* w_v,
                                          int32_t weights_on_device, kvx_translator** out);

@@ -35,10 +35,26 @@ def build(force: bool = False) -> str:
     return _LIB_PATH
 
 
+class RopeSched(ctypes.Structure):
+    _fields_ = [("base", ctypes.c_double), ("type", ctypes.c_int32), ("factor", ctypes.c_double),
+                ("low", ctypes.c_double), ("high", ctypes.c_double), ("orig_ctx", ctypes.c_int32)]
+
+
+def rope_sched(g=None, base: Optional[float] = None) -> RopeSched:
+    """The rotary schedule of a geometry object (attributes rope_base, rope_type, rope_factor,
+    rope_low_freq_factor, rope_high_freq_factor, rope_original_max_position; missing ones mean
+    the plain schedule), or the plain schedule of `base`."""
+    if g is None:
+        return RopeSched(float(base), 0, 1.0, 1.0, 1.0, 1)
+    return RopeSched(float(g.rope_base), int(getattr(g, "rope_type", 0)), float(getattr(g, "rope_factor", 1.0)),
+                     float(getattr(g, "rope_low_freq_factor", 1.0)), float(getattr(g, "rope_high_freq_factor", 4.0)),
+                     int(getattr(g, "rope_original_max_position", 8192)))
+
+
 class Problem(ctypes.Structure):
     _fields_ = [
-        ("Ls", ctypes.c_int32), ("Hs", ctypes.c_int32), ("ds", ctypes.c_int32), ("base_s", ctypes.c_double),
-        ("Lt", ctypes.c_int32), ("Ht", ctypes.c_int32), ("dt", ctypes.c_int32), ("base_t", ctypes.c_double),
+        ("Ls", ctypes.c_int32), ("Hs", ctypes.c_int32), ("ds", ctypes.c_int32), ("rope_s", RopeSched),
+        ("Lt", ctypes.c_int32), ("Ht", ctypes.c_int32), ("dt", ctypes.c_int32), ("rope_t", RopeSched),
         ("layer_map", I32P),
         ("batch", ctypes.c_int32), ("s_max", ctypes.c_int32), ("t_max", ctypes.c_int32),
         ("src_len", I32P), ("tgt_seq_off", I32P),
@@ -57,8 +73,11 @@ def lib():
         _lib.kvxo_build_alignment.argtypes = [ctypes.c_int, I32P, I32P, I32P, I32P, I32P, I32P]
         _lib.kvxo_rope.argtypes = [F64P, ctypes.c_int, ctypes.c_double, ctypes.c_double, ctypes.c_int]
         _lib.kvxo_rope.restype = None
+        _lib.kvxo_rope_sched_apply.argtypes = [F64P, ctypes.c_int, ctypes.POINTER(RopeSched), ctypes.c_double,
+                                               ctypes.c_int]
+        _lib.kvxo_rope_sched_apply.restype = None
         _lib.kvxo_rope_cache.argtypes = [F32P, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
-                                         ctypes.c_double, I32P, ctypes.c_int]
+                                         ctypes.POINTER(RopeSched), I32P, ctypes.c_int]
         _lib.kvxo_rope_cache.restype = None
         _lib.kvxo_translate_row.argtypes = [ctypes.POINTER(Problem), ctypes.c_int, ctypes.c_int,
                                             ctypes.c_int, ctypes.c_int, F64P]
@@ -93,17 +112,28 @@ def build_alignment(src_seq_off, src_end, tgt_seq_off, tgt_end):
 
 
 def rope(x: np.ndarray, base: float, pos: float, sign: int) -> np.ndarray:
+    """Plain-schedule rotary map of one head vector (double)."""
     v = np.array(x, np.float64).copy()
     lib().kvxo_rope(_p(v, F64P), v.shape[-1], base, float(pos), sign)
     return v
 
 
-def rope_cache(x: np.ndarray, base: float, pos: Optional[np.ndarray] = None, sign: int = +1) -> np.ndarray:
-    """x: [B, H, S, d] float32; returns a rotated copy (float32)."""
+def rope_g(x: np.ndarray, geom, pos: float, sign: int) -> np.ndarray:
+    """Rotary map of one head vector under geometry `geom`'s frequency schedule (double)."""
+    v = np.array(x, np.float64).copy()
+    r = rope_sched(geom)
+    lib().kvxo_rope_sched_apply(_p(v, F64P), v.shape[-1], ctypes.byref(r), float(pos), sign)
+    return v
+
+
+def rope_cache(x: np.ndarray, base, pos: Optional[np.ndarray] = None, sign: int = +1) -> np.ndarray:
+    """x: [B, H, S, d] float32; returns a rotated copy (float32).  `base` is a number (plain
+    schedule) or a geometry object carrying its schedule."""
     y = np.ascontiguousarray(x, np.float32).copy()
     B, H, S, d = y.shape
     pos = _i32(pos)
-    lib().kvxo_rope_cache(_p(y, F32P), B, H, S, d, base, _p(pos, I32P), sign)
+    r = rope_sched(base=base) if isinstance(base, (int, float)) else rope_sched(base)
+    lib().kvxo_rope_cache(_p(y, F32P), B, H, S, d, ctypes.byref(r), _p(pos, I32P), sign)
     return y
 
 
@@ -131,8 +161,8 @@ class OracleProblem:
         wk, wv = keep(np.ascontiguousarray(w_k, np.float32)), keep(np.ascontiguousarray(w_v, np.float32))
         self.T = int(so[-1])
         self.Lt, self.Ht, self.dt = dst_geom.num_layers, dst_geom.num_kv_heads, dst_geom.head_dim
-        self.p = Problem(src_geom.num_layers, src_geom.num_kv_heads, src_geom.head_dim, src_geom.rope_base,
-                         dst_geom.num_layers, dst_geom.num_kv_heads, dst_geom.head_dim, dst_geom.rope_base,
+        self.p = Problem(src_geom.num_layers, src_geom.num_kv_heads, src_geom.head_dim, rope_sched(src_geom),
+                         dst_geom.num_layers, dst_geom.num_kv_heads, dst_geom.head_dim, rope_sched(dst_geom),
                          _p(lm, I32P), len(sl), s_max, t_max, _p(sl, I32P), _p(so, I32P),
                          _p(lo, I32P), _p(hi, I32P), _p(sp, I32P), _p(tp, I32P),
                          ctypes.cast(kp, ctypes.POINTER(F32P)), ctypes.cast(vp, ctypes.POINTER(F32P)),

@@ -23,13 +23,15 @@
  *   6. K: y <- R_{d_t,base_t}(+p_t) y                 (apply the target RoPE)
  *
  * R_{d,base}(p) is the half-split rotary map: channel pairs (i, i+d/2) for
- * i < d/2 are rotated by the angle p * base^(-2i/d).  The angle is taken in
- * exact (double) arithmetic.  A base <= 0 means "no RoPE".
+ * i < d/2 are rotated by the angle p * theta_i, theta_i = base^(-2i/d) or its
+ * rescaled form under the model's frequency schedule (kvxo_theta).  The angle
+ * is taken in exact (double) arithmetic.  A base <= 0 means "no RoPE".
  *
  * Everything runs in double precision, in the order above, with no blocking,
  * fusion or reordering.  Inputs are float32 arrays (bf16 storage is widened
  * exactly by the caller).
  */
+#define _DEFAULT_SOURCE
 #include <math.h>
 #include <stdint.h>
 #include <stdlib.h>
@@ -102,16 +104,45 @@ KVXO_API int kvxo_build_alignment(int batch,
 }
 
 /* ---------------------------------------------------------------------- */
+/* Rotary frequency schedule of one model.  type 0: the plain RoFormer
+ * frequencies theta_i = base^(-2i/d).  type 1: linear position interpolation,
+ * the angle of position p is that of p / factor.  type 2: the Llama-3.1
+ * frequency-dependent rescaling: a pair whose wavelength 2 pi / theta_i is
+ * shorter than orig_ctx / high keeps theta_i, one longer than orig_ctx / low
+ * gets theta_i / factor, and in between the two are mixed with weight
+ * m = (orig_ctx / wavelength - low) / (high - low) on the unscaled frequency. */
+typedef struct {
+    double base;          /* <= 0: no rotary encoding */
+    int32_t type;
+    double factor, low, high;
+    int32_t orig_ctx;
+} kvxo_rope_sched;
+
+static double kvxo_theta(const kvxo_rope_sched* r, int i, int d)
+{
+    double theta = pow(r->base, -2.0 * (double)i / (double)d);
+    if (r->type == 1) return theta / r->factor;
+    if (r->type == 2) {
+        double wavelength = 2.0 * M_PI / theta;
+        double short_edge = (double)r->orig_ctx / r->high;   /* below: high-frequency band */
+        double long_edge = (double)r->orig_ctx / r->low;     /* above: low-frequency band */
+        if (wavelength < short_edge) return theta;
+        if (wavelength > long_edge) return theta / r->factor;
+        double m = ((double)r->orig_ctx / wavelength - r->low) / (r->high - r->low);
+        return m * theta + (1.0 - m) * theta / r->factor;
+    }
+    return theta;
+}
+
 /* Half-split rotary map on one head vector of length d (d even):
  * x'[i] = x[i] cos a - x[i+d/2] sin a,  x'[i+d/2] = x[i+d/2] cos a + x[i] sin a,
- * a = sign * pos * base^(-2i/d).  sign = +1 applies the RoPE, -1 undoes it. */
-KVXO_API void kvxo_rope(double* x, int d, double base, double pos, int sign)
+ * a = sign * pos * theta_i.  sign = +1 applies the RoPE, -1 undoes it. */
+KVXO_API void kvxo_rope_sched_apply(double* x, int d, const kvxo_rope_sched* r, double pos, int sign)
 {
-    if (base <= 0.0) return;
+    if (r->base <= 0.0) return;
     int h = d / 2;
     for (int i = 0; i < h; ++i) {
-        double inv_freq = pow(base, -2.0 * (double)i / (double)d);
-        double a = (double)sign * pos * inv_freq;
+        double a = (double)sign * pos * kvxo_theta(r, i, d);
         double c = cos(a), sn = sin(a);
         double x0 = x[i], x1 = x[i + h];
         x[i]     = x0 * c - x1 * sn;
@@ -119,10 +150,17 @@ KVXO_API void kvxo_rope(double* x, int d, double base, double pos, int sign)
     }
 }
 
+/* The plain schedule (type 0) with the given base. */
+KVXO_API void kvxo_rope(double* x, int d, double base, double pos, int sign)
+{
+    kvxo_rope_sched r = {base, 0, 1.0, 1.0, 1.0, 1};
+    kvxo_rope_sched_apply(x, d, &r, pos, sign);
+}
+
 /* ---------------------------------------------------------------------- */
 typedef struct {
-    int32_t Ls, Hs, ds; double base_s;        /* source geometry */
-    int32_t Lt, Ht, dt; double base_t;        /* target geometry */
+    int32_t Ls, Hs, ds; kvxo_rope_sched rope_s;   /* source geometry */
+    int32_t Lt, Ht, dt; kvxo_rope_sched rope_t;   /* target geometry */
     const int32_t* layer_map;                 /* [Lt] */
     int32_t batch, s_max, t_max;
     const int32_t* src_len;                   /* [B] */
@@ -167,7 +205,7 @@ KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int
             int g = g0 + q;
             const float* row = src + (((size_t)b * p->Hs + g) * p->s_max + s) * p->ds;
             for (int e = 0; e < p->ds; ++e) u[e] = (double)row[e];
-            if (kv == 0) kvxo_rope(u, p->ds, p->base_s, ps, -1);
+            if (kv == 0) kvxo_rope_sched_apply(u, p->ds, &p->rope_s, ps, -1);
             for (int e = 0; e < p->ds; ++e) sum[q * p->ds + e] += u[e];
         }
     }
@@ -182,7 +220,7 @@ KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int
     }
     if (kv == 0) {                                             /* step 6 */
         double pt = p->tgt_pos ? (double)p->tgt_pos[tp] : (double)t;
-        kvxo_rope(out, p->dt, p->base_t, pt, +1);
+        kvxo_rope_sched_apply(out, p->dt, &p->rope_t, pt, +1);
     }
     free(sum);
     free(u);
@@ -207,7 +245,7 @@ KVXO_API int kvxo_translate(const kvxo_problem* p, double* out_k, double* out_v)
  * out [B][H][S][d] (float32 in place, arithmetic in double).  pos: [B*S]
  * positions or NULL (= token index).  Used to synthesise post-RoPE source
  * caches the way a source model's prefill would have stored them. */
-KVXO_API void kvxo_rope_cache(float* x, int B, int H, int S, int d, double base,
+KVXO_API void kvxo_rope_cache(float* x, int B, int H, int S, int d, const kvxo_rope_sched* r,
                               const int32_t* pos, int sign)
 {
     double* row = (double*)malloc(sizeof(double) * (size_t)d);
@@ -217,7 +255,7 @@ KVXO_API void kvxo_rope_cache(float* x, int B, int H, int S, int d, double base,
                 float* xr = x + (((size_t)b * H + h) * S + s) * d;
                 for (int e = 0; e < d; ++e) row[e] = (double)xr[e];
                 double p = pos ? (double)pos[(size_t)b * S + s] : (double)s;
-                kvxo_rope(row, d, base, p, sign);
+                kvxo_rope_sched_apply(row, d, r, p, sign);
                 for (int e = 0; e < d; ++e) xr[e] = (float)row[e];
             }
     free(row);

@@ -32,9 +32,25 @@ I32P = ctypes.POINTER(ctypes.c_int32)
 VP = ctypes.c_void_p
 
 
+KVX_ROPE_DEFAULT, KVX_ROPE_LINEAR, KVX_ROPE_LLAMA3 = 0, 1, 2
+
+
 class kvx_model_geom(ctypes.Structure):
     _fields_ = [("num_layers", ctypes.c_int32), ("num_kv_heads", ctypes.c_int32),
-                ("head_dim", ctypes.c_int32), ("rope_base", ctypes.c_double)]
+                ("head_dim", ctypes.c_int32), ("rope_base", ctypes.c_double),
+                ("rope_type", ctypes.c_int32), ("rope_factor", ctypes.c_double),
+                ("rope_low_freq_factor", ctypes.c_double), ("rope_high_freq_factor", ctypes.c_double),
+                ("rope_original_max_position", ctypes.c_int32)]
+
+
+def model_geom(g) -> kvx_model_geom:
+    """kvx_model_geom from any object with the same attribute names (the RoPE schedule
+    attributes are optional and default to the plain schedule)."""
+    return kvx_model_geom(g.num_layers, g.num_kv_heads, g.head_dim, g.rope_base,
+                          int(getattr(g, "rope_type", 0)), float(getattr(g, "rope_factor", 1.0)),
+                          float(getattr(g, "rope_low_freq_factor", 1.0)),
+                          float(getattr(g, "rope_high_freq_factor", 4.0)),
+                          int(getattr(g, "rope_original_max_position", 8192)))
 
 
 class kvx_translator_desc(ctypes.Structure):
@@ -216,10 +232,7 @@ class Translator:
         if layer_map is not None:
             self._lm = (ctypes.c_int32 * len(layer_map))(*[int(x) for x in layer_map])
             lm = ctypes.cast(self._lm, I32P)
-        self.desc = kvx_translator_desc(
-            kvx_model_geom(src_geom.num_layers, src_geom.num_kv_heads, src_geom.head_dim, src_geom.rope_base),
-            kvx_model_geom(dst_geom.num_layers, dst_geom.num_kv_heads, dst_geom.head_dim, dst_geom.rope_base),
-            lm, dtype, max_position, path)
+        self.desc = kvx_translator_desc(model_geom(src_geom), model_geom(dst_geom), lm, dtype, max_position, path)
         w_k = w_k.contiguous()
         w_v = w_v.contiguous()
         self.handle = kvx_translator_create(self.desc, _ptr(w_k), _ptr(w_v), w_k.is_cuda)

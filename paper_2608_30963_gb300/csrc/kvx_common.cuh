@@ -23,6 +23,36 @@ struct RopeTable {
     int enabled;                       // 0: no rotation
 };
 
+// Rotation frequency f_i of channel pair (i, i + d/2) under the model's schedule
+// (kvx_rope_type in kvx.h), in double.  Host code turns it into fixed-point turns
+// once per translator; the allocation-free entry point does the same on the device.
+__host__ __device__ inline double rope_inv_freq(const kvx_model_geom& g, int i)
+{
+    const double f = pow(g.rope_base, -2.0 * (double)i / (double)g.head_dim);
+    if (g.rope_type == KVX_ROPE_LINEAR) return f / g.rope_factor;
+    if (g.rope_type != KVX_ROPE_LLAMA3) return f;
+    const double wavelen = 6.283185307179586 / f;
+    const double orig = (double)g.rope_original_max_position;
+    if (wavelen < orig / g.rope_high_freq_factor) return f;            // high-frequency band: kept
+    if (wavelen > orig / g.rope_low_freq_factor) return f / g.rope_factor;   // low band: interpolated
+    const double m = (orig / wavelen - g.rope_low_freq_factor) / (g.rope_high_freq_factor - g.rope_low_freq_factor);
+    return (1.0 - m) * (f / g.rope_factor) + m * f;
+}
+
+// Schedule parameters valid for the model's rope_type (host-side validation).
+inline bool rope_schedule_ok(const kvx_model_geom& g)
+{
+    if (g.rope_base <= 0.0) return g.rope_type >= KVX_ROPE_DEFAULT && g.rope_type <= KVX_ROPE_LLAMA3;
+    switch (g.rope_type) {
+    case KVX_ROPE_DEFAULT: return true;
+    case KVX_ROPE_LINEAR: return g.rope_factor > 0.0;
+    case KVX_ROPE_LLAMA3:
+        return g.rope_factor > 0.0 && g.rope_low_freq_factor > 0.0 &&
+               g.rope_high_freq_factor > g.rope_low_freq_factor && g.rope_original_max_position > 0;
+    default: return false;
+    }
+}
+
 // Everything one kvx_translate launch needs, passed by value (graph-capturable;
 // no per-call device allocation or copy).
 struct TranslateParams {
@@ -50,7 +80,7 @@ struct TranslateParams {
     int max_pages, page_size, num_pages;
     // rotation
     RopeTable rs, rt;
-    int rope_same;   // source and target RoPE have the same base and head_dim
+    int rope_same;   // source and target rotations coincide (same head_dim, same frequencies)
     int max_position;
     unsigned* status;
     // weights (layout depends on the kernel)

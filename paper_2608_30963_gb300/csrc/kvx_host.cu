@@ -27,6 +27,7 @@ struct kvx_translator {
     unsigned long long host_turns[256];   // host copy of the same
     size_t rope_bytes = 0;
     RopeTable rs{}, rt{};
+    int rope_same = 0;           // source and target turns identical (same d, same frequencies)
     unsigned* status = nullptr;
     TcConfig tc{};
     // span plan of the tensor-core span kernel: sub-tile windows and per-token entries
@@ -145,6 +146,9 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         return fail(KVX_ERR_INVALID_ARG, "create: unknown dtype %d", desc->dtype);
     if (desc->path < KVX_PATH_AUTO || desc->path > KVX_PATH_TCGEN05)
         return fail(KVX_ERR_INVALID_ARG, "create: unknown path %d", desc->path);
+    if (!rope_schedule_ok(s) || !rope_schedule_ok(d))
+        return fail(KVX_ERR_INVALID_ARG, "create: unknown rope_type or schedule parameters out of range "
+                                         "(source type %d, target type %d)", s.rope_type, d.rope_type);
     int max_pos = desc->max_position ? desc->max_position : (1 << 24);
     if (max_pos < 1 || max_pos > (1 << 30))
         return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<30]");
@@ -237,8 +241,7 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         auto fill = [&](const kvx_model_geom& g, unsigned long long* out) {
             for (int i = 0; i < g.head_dim / 2; ++i) {
                 if (g.rope_base <= 0.0) { out[i] = 0; continue; }
-                const double f = pow(g.rope_base, -2.0 * (double)i / (double)g.head_dim);
-                out[i] = (unsigned long long)ldexp(f / (2.0 * M_PI), 64);
+                out[i] = (unsigned long long)ldexp(rope_inv_freq(g, i) / (2.0 * M_PI), 64);
             }
         };
         fill(s, h_turns);
@@ -255,6 +258,9 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         }
         t->rs = RopeTable{t->rope, hs, s.rope_base > 0.0};
         t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0};
+        // the two rotations coincide when head dims, enablement and every frequency agree
+        t->rope_same = hs == hd && t->rs.enabled == t->rt.enabled &&
+                       memcmp(h_turns, h_turns + hs, (size_t)hs * sizeof(unsigned long long)) == 0;
     }
     if (cudaMalloc(&t->status, sizeof(unsigned)) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: status allocation"); goto err; }
     if (t->path == KVX_PATH_TCGEN05 && cudaMalloc(&t->plan, tc_plan_bytes(kvx_translator::kPlanTokens)) != cudaSuccess) {
@@ -320,7 +326,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
     P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
     P.page_size = dst->page_size; P.num_pages = dst->num_pages;
     P.rs = tr->rs; P.rt = tr->rt; P.max_position = tr->max_position;
-    P.rope_same = D.src.rope_base == D.dst.rope_base && D.src.head_dim == D.dst.head_dim;
+    P.rope_same = tr->rope_same;
     P.status = tr->status;
     P.w = tr->w;
     for (int j = 0; j < Lt; ++j) {

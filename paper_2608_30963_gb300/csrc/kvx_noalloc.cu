@@ -43,14 +43,14 @@ kvx_status fail(kvx_status s, const char* fmt, ...)
     return s;
 }
 
-// Fixed-point rotation turns round(2^64 f_i / 2 pi), f_i = base^(-2i/d), written on the device.
-__global__ void static_turns_kernel(unsigned long long* out, int half, int d, double base)
+// Fixed-point rotation turns round(2^64 f_i / 2 pi), f_i the model's scheduled frequency
+// of pair i, written on the device.
+__global__ void static_turns_kernel(unsigned long long* out, const kvx_model_geom g)
 {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= half) return;
-    if (base <= 0.0) { out[i] = 0ull; return; }
-    const double f = pow(base, -2.0 * (double)i / (double)d);
-    out[i] = (unsigned long long)ldexp(f / (2.0 * 3.14159265358979323846), 64);
+    if (i >= g.head_dim / 2) return;
+    if (g.rope_base <= 0.0) { out[i] = 0ull; return; }
+    out[i] = (unsigned long long)ldexp(rope_inv_freq(g, i) / (2.0 * 3.14159265358979323846), 64);
 }
 
 }  // namespace
@@ -79,6 +79,8 @@ extern "C" KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* de
         return fail(KVX_ERR_UNSUPPORTED, "translate_static: neither KV head count divides the other");
     if (desc->dtype != KVX_BF16 && desc->dtype != KVX_FP32)
         return fail(KVX_ERR_INVALID_ARG, "translate_static: unknown dtype %d", desc->dtype);
+    if (!rope_schedule_ok(s) || !rope_schedule_ok(d))
+        return fail(KVX_ERR_INVALID_ARG, "translate_static: unknown rope_type or schedule parameters out of range");
     const int max_pos = desc->max_position ? desc->max_position : (1 << 24);
     if (max_pos < 1 || max_pos > (1 << 30))
         return fail(KVX_ERR_INVALID_ARG, "translate_static: max_position must be in [1, 1<<30]");
@@ -149,8 +151,8 @@ extern "C" KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* de
         (ce = cudaMemcpyAsync(wts, w_k, one, cudaMemcpyDeviceToDevice, st)) != cudaSuccess ||
         (ce = cudaMemcpyAsync(wts + one, w_v, one, cudaMemcpyDeviceToDevice, st)) != cudaSuccess)
         return fail(KVX_ERR_CUDA, "translate_static: %s", cudaGetErrorString(ce));
-    static_turns_kernel<<<1, 128, 0, st>>>(turns, s.head_dim / 2, s.head_dim, s.rope_base);
-    static_turns_kernel<<<1, 128, 0, st>>>(turns + 128, d.head_dim / 2, d.head_dim, d.rope_base);
+    static_turns_kernel<<<1, 128, 0, st>>>(turns, s);
+    static_turns_kernel<<<1, 128, 0, st>>>(turns + 128, d);
     if ((ce = cudaGetLastError()) != cudaSuccess)
         return fail(KVX_ERR_CUDA, "translate_static: %s", cudaGetErrorString(ce));
 

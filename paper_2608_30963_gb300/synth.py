@@ -51,12 +51,21 @@ def bf16_round(x: np.ndarray) -> np.ndarray:
 # ----------------------------------------------------------------------------
 # geometry and workload description
 # ----------------------------------------------------------------------------
+ROPE_DEFAULT, ROPE_LINEAR, ROPE_LLAMA3 = 0, 1, 2
+
+
 @dataclasses.dataclass(frozen=True)
 class ModelGeom:
     num_layers: int
     num_kv_heads: int
     head_dim: int
     rope_base: float  # <= 0: the model applies no RoPE to K
+    # RoPE frequency schedule: 0 plain, 1 linear position interpolation, 2 Llama-3.1
+    rope_type: int = ROPE_DEFAULT
+    rope_factor: float = 1.0
+    rope_low_freq_factor: float = 1.0
+    rope_high_freq_factor: float = 4.0
+    rope_original_max_position: int = 8192
 
 
 @dataclasses.dataclass
@@ -115,6 +124,12 @@ QWEN7B = _g(28, 4, 128, 1e6)
 QWEN1P5B = _g(28, 2, 128, 1e6)
 GEMMA2B = _g(26, 4, 256, 1e4)
 LLAMA70B = _g(80, 8, 128, 5e5)
+# Llama-3.1's published RoPE schedule parameters (factor 8, low/high frequency factors 1 and 4,
+# original context 8192); the 70B -> 7B workload keeps the plain schedule its description gives,
+# this variant exercises the scaled one
+LLAMA70B_SCALED = dataclasses.replace(LLAMA70B, rope_type=ROPE_LLAMA3, rope_factor=8.0,
+                                      rope_low_freq_factor=1.0, rope_high_freq_factor=4.0,
+                                      rope_original_max_position=8192)
 
 
 def config_specs() -> Dict[str, WorkloadSpec]:

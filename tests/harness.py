@@ -49,7 +49,7 @@ def make_case(spec: synth.WorkloadSpec, tgt_lens=None, layers: Optional[Sequence
         k = synth.source_kv(wl, l, 0, pad_value)
         if spec.src.rope_base > 0:
             pos = None if src_pos is None else np.asarray(src_pos, np.int32)
-            k = oracle.rope_cache(k, spec.src.rope_base, pos, +1)
+            k = oracle.rope_cache(k, spec.src, pos, +1)
         if spec.dtype == "bf16":
             k = synth.bf16_round(k)
         if pad_value != 0.0:

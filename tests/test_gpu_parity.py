@@ -89,6 +89,33 @@ def test_explicit_positions_and_layer_map(path):
     _full_compare(c, path, max_position=1 << 17)
 
 
+LINEAR4 = dict(rope_type=synth.ROPE_LINEAR, rope_factor=4.0)
+SCHEDULES = {
+    # Llama-3.1 scaled source RoPE, cross-tokenizer (span kernel)
+    "llama3_src_spans": ("llama70b_to_qwen7b_8k", 5, 3, [300, 41], dict(src=synth.LLAMA70B_SCALED), {}),
+    # linear target schedule, identity alignment: source and target rotations differ
+    "linear_dst_identity": ("qwen7b_to_qwen1p5b_4k", 2, 2, [300, 5], {}, LINEAR4),
+    # the same scaled schedule on both sides: source and target rotations coincide
+    "llama3_both_identity": ("qwen7b_to_qwen1p5b_4k", 2, 2, [300],
+                             dict(rope_type=synth.ROPE_LLAMA3, rope_factor=8.0, rope_low_freq_factor=1.0,
+                                  rope_high_freq_factor=4.0, rope_original_max_position=256),
+                             dict(rope_type=synth.ROPE_LLAMA3, rope_factor=8.0, rope_low_freq_factor=1.0,
+                                  rope_high_freq_factor=4.0, rope_original_max_position=256)),
+}
+
+
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+@pytest.mark.parametrize("name", list(SCHEDULES))
+def test_rope_schedules(name, path):
+    base, Ls, Lt, lens, src_kw, dst_kw = SCHEDULES[name]
+    spec = _shrink(SPECS[base], Ls, Lt)
+    src = src_kw.get("src", dataclasses.replace(spec.src, **{k: v for k, v in src_kw.items() if k != "src"}))
+    src = dataclasses.replace(src, num_layers=Ls)
+    spec = dataclasses.replace(spec, src=src, dst=dataclasses.replace(spec.dst, **dst_kw))
+    c = make_case(spec, lens, pad_value=float("nan"))
+    _full_compare(c, path)
+
+
 def test_tiny_token_counts_and_empty_sequences():
     spec = _shrink(SPECS["qwen1p5b_to_gemma2b_1k"], 2, 2)
     c = make_case(spec, [1, 0, 2, 0, 129])

@@ -47,8 +47,7 @@ def test_layer_map_matches_oracle(lib, Ls, Lt):
 
 
 def _desc(src, dst, dtype=kvx.KVX_BF16, path=kvx.KVX_PATH_AUTO, layer_map=None):
-    g = lambda m: kvx.kvx_model_geom(m.num_layers, m.num_kv_heads, m.head_dim, m.rope_base)
-    return kvx.kvx_translator_desc(g(src), g(dst), layer_map, dtype, 0, path)
+    return kvx.kvx_translator_desc(kvx.model_geom(src), kvx.model_geom(dst), layer_map, dtype, 0, path)
 
 
 @pytest.mark.parametrize("src,dst,code", [
@@ -57,6 +56,12 @@ def _desc(src, dst, dtype=kvx.KVX_BF16, path=kvx.KVX_PATH_AUTO, layer_map=None):
     (synth.ModelGeom(2, 16, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),  # in = 1024
     (synth.ModelGeom(0, 2, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_INVALID_ARG),
     (synth.ModelGeom(2, 2, 128, 1e6), synth.ModelGeom(200, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),
+    (synth.ModelGeom(2, 2, 128, 1e6, rope_type=3), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_INVALID_ARG),
+    (synth.ModelGeom(2, 2, 128, 1e6, rope_type=1, rope_factor=0.0), synth.ModelGeom(2, 2, 128, 1e6),
+     kvx.KVX_ERR_INVALID_ARG),
+    (synth.ModelGeom(2, 2, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6, rope_type=2, rope_factor=8.0,
+                                                       rope_low_freq_factor=4.0, rope_high_freq_factor=1.0),
+     kvx.KVX_ERR_INVALID_ARG),
 ])
 def test_create_rejects_bad_geometry_without_touching_cuda(lib, src, dst, code):
     h = ctypes.c_void_p()

@@ -130,6 +130,111 @@ def test_rope_inverse_norm_and_relative_position():
         assert abs(a - b) < 1e-9
 
 
+# ------------------------------------------------- RoPE frequency schedules
+def _sched(base, d=4, **kw):
+    return synth.ModelGeom(1, 1, d, base, **kw)
+
+
+def _slow_pair_angle(g, pos=1.0):
+    """Angle by which the second pair of a d=4 head turns at `pos` (theta_1 = base^(-1/2))."""
+    y = oracle.rope_g(np.array([0.0, 1.0, 0.0, 0.0]), g, pos, +1)
+    return np.arctan2(y[3], y[1])
+
+
+def test_linear_schedule_is_position_interpolation():
+    # angle of position p under factor F equals the plain angle of position p / F
+    rng = np.random.default_rng(21)
+    for d, base, F in ((64, 1e4, 2.0), (128, 1e6, 4.0), (256, 1e4, 8.0)):
+        x = rng.standard_normal(d)
+        g = synth.ModelGeom(1, 1, d, base, rope_type=synth.ROPE_LINEAR, rope_factor=F)
+        for p in (1.0, 37.0, 4095.0):
+            np.testing.assert_allclose(oracle.rope_g(x, g, p, +1), oracle.rope(x, base, p / F, +1), atol=1e-9)
+
+
+def test_llama3_schedule_factor_one_is_plain():
+    rng = np.random.default_rng(22)
+    x = rng.standard_normal(128)
+    g = synth.ModelGeom(1, 1, 128, 5e5, rope_type=synth.ROPE_LLAMA3, rope_factor=1.0,
+                        rope_low_freq_factor=1.0, rope_high_freq_factor=4.0, rope_original_max_position=8192)
+    np.testing.assert_allclose(oracle.rope_g(x, g, 3000.0, +1), oracle.rope(x, 5e5, 3000.0, +1), atol=1e-12)
+
+
+def test_llama3_schedule_bands_and_continuity():
+    # d = 4: the slow pair's wavelength is 2 pi sqrt(base), so base places it anywhere.
+    F, lo, hi, orig = 8.0, 1.0, 4.0, 8192
+    kw = dict(rope_type=synth.ROPE_LLAMA3, rope_factor=F, rope_low_freq_factor=lo,
+              rope_high_freq_factor=hi, rope_original_max_position=orig)
+    base_of = lambda w: (w / (2 * np.pi)) ** 2
+    theta = lambda w: 2 * np.pi / w
+    short_edge, long_edge = orig / hi, orig / lo           # 2048 and 8192 tokens
+    # short wavelengths keep their frequency, long ones are divided by the factor
+    for w in (100.0, 2000.0):
+        assert _slow_pair_angle(_sched(base_of(w), **kw)) == pytest.approx(theta(w), rel=1e-12)
+    for w in (8300.0, 1e6):
+        assert _slow_pair_angle(_sched(base_of(w), **kw)) == pytest.approx(theta(w) / F, rel=1e-12)
+    # continuous at both band edges
+    for edge, inside in ((short_edge, theta(short_edge)), (long_edge, theta(long_edge) / F)):
+        a = _slow_pair_angle(_sched(base_of(edge * (1 - 1e-9)), **kw))
+        b = _slow_pair_angle(_sched(base_of(edge * (1 + 1e-9)), **kw))
+        assert a == pytest.approx(inside, rel=1e-6) and b == pytest.approx(inside, rel=1e-6)
+    # inside the band the frequency lies strictly between theta/F and theta and falls with w
+    ws = np.linspace(short_edge * 1.01, long_edge * 0.99, 9)
+    ang = np.array([_slow_pair_angle(_sched(base_of(w), **kw)) for w in ws])
+    assert np.all(ang < theta(ws)) and np.all(ang > theta(ws) / F) and np.all(np.diff(ang) < 0)
+    # where orig / w sits halfway between low and high the two frequencies weigh equally
+    w_mid = orig / ((lo + hi) / 2)
+    assert _slow_pair_angle(_sched(base_of(w_mid), **kw)) == pytest.approx(theta(w_mid) * (1 + 1 / F) / 2,
+                                                                            rel=1e-12)
+    # the fast pair (theta_0 = 1, wavelength 2 pi) is never rescaled
+    y = oracle.rope_g(np.array([1.0, 0.0, 0.0, 0.0]), _sched(1e9, **kw), 0.5, +1)
+    assert np.arctan2(y[2], y[0]) == pytest.approx(0.5, rel=1e-14)
+
+
+def test_llama31_parameters_split_128_dim_heads_29_6_29():
+    # base 5e5, d 128: wavelength 2 pi 5e5^(i/64) is below 2048 for i <= 28 and above 8192
+    # for i >= 35 (ln(2048/2pi)/ln(5e5)*64 = 28.2, ln(8192/2pi)/ln(5e5)*64 = 35.0)
+    g = synth.LLAMA70B_SCALED
+    kept = scaled = mixed = 0
+    for i in range(64):
+        x = np.zeros(128)
+        x[i] = 1.0
+        p = 0.25                                   # keeps every angle below pi
+        y = oracle.rope_g(x, g, p, +1)
+        got = np.arctan2(y[i + 64], y[i]) / p
+        plain = 5e5 ** (-i / 64)
+        if got == pytest.approx(plain, rel=1e-12):
+            kept += 1
+        elif got == pytest.approx(plain / 8, rel=1e-12):
+            scaled += 1
+        else:
+            assert plain / 8 < got < plain
+            mixed += 1
+    assert (kept, mixed, scaled) == (29, 6, 29)
+
+
+def test_scheduled_translation_undoes_and_reapplies_the_schedule():
+    # K stored with a scheduled source RoPE, W = I, identity alignment and the same scheduled
+    # target RoPE: the translation returns the stored keys (un-rotate then re-rotate).
+    g = synth.ModelGeom(1, 1, 64, 5e5, rope_type=synth.ROPE_LLAMA3, rope_factor=8.0,
+                        rope_low_freq_factor=1.0, rope_high_freq_factor=4.0, rope_original_max_position=64)
+    rng = np.random.default_rng(23)
+    S = 40
+    k = oracle.rope_cache(rng.standard_normal((1, 1, S, 64)).astype(np.float32), g)
+    v = rng.standard_normal((1, 1, S, 64)).astype(np.float32)
+    W = np.eye(64, dtype=np.float32)[None, None]
+    p = oracle.OracleProblem(g, g, [0], [S], [0, S], S, S, [k], [v], W, W)
+    ok, ov = p.translate()
+    np.testing.assert_allclose(ok[0, 0], k[0, 0], atol=1e-6)
+    np.testing.assert_allclose(ov[0, 0], v[0, 0], atol=1e-6)
+    # and a plain target RoPE gives plain-rotated keys of the un-rotated source
+    gp = synth.ModelGeom(1, 1, 64, 5e5)
+    p2 = oracle.OracleProblem(g, gp, [0], [S], [0, S], S, S, [k], [v], W, W)
+    ok2, _ = p2.translate()
+    for t in (0, 7, 39):
+        raw = oracle.rope_g(k[0, 0, t], g, t, -1)
+        np.testing.assert_allclose(ok2[0, 0, t], oracle.rope(raw, 5e5, t, +1), atol=1e-6)
+
+
 # ------------------------------------------------------------ translation
 def _geom(L, H, d, base):
     return synth.ModelGeom(L, H, d, base)

@@ -42,7 +42,7 @@ def _shrink(spec, Ls, Lt):
 
 
 CASES = [("tiny_fp32", None, None, None), ("qwen1p5b_to_gemma2b_1k", 3, 2, [130, 7]),
-         ("qwen7b_to_qwen1p5b_4k", 2, 2, [200])]
+         ("qwen7b_to_qwen1p5b_4k", 2, 2, [200]), ("llama70b_to_qwen7b_8k", 3, 2, [150])]
 
 
 @pytest.mark.parametrize("name,Ls,Lt,lens", CASES, ids=[c[0] for c in CASES])
@@ -52,6 +52,9 @@ def test_static_entry_matches_translator_on_two_calls(name, Ls, Lt, lens):
     spec = synth.config_specs()[name]
     if Ls:
         spec = _shrink(spec, Ls, Lt)
+    if name.startswith("llama70b"):
+        # the Llama-3.1 RoPE schedule on the source side (frequencies computed on the device here)
+        spec = dataclasses.replace(spec, src=dataclasses.replace(synth.LLAMA70B_SCALED, num_layers=Ls))
     c = make_case(spec, lens)
     # the regular entry point, CUDA-core path (the kernel the static entry point runs)
     ref = DeviceCase(c, path=kvx.KVX_PATH_SIMT, paged=False)
