@@ -44,10 +44,12 @@ def algorithmic(spec: synth.WorkloadSpec, wl: synth.Workload, layer_map) -> dict
     elt = 2 if spec.dtype == "bf16" else 4
     S_tot = int(wl.src_len.sum())
     T = wl.total_tgt
-    src_layers = len(set(int(x) for x in layer_map))
+    src_layers = len(set(int(x) for x in np.asarray(layer_map).reshape(-1)))
     rd = src_layers * spec.src.num_kv_heads * S_tot * spec.src.head_dim * 2 * elt
     wr = spec.dst.num_layers * spec.dst.num_kv_heads * T * spec.dst.head_dim * 2 * elt
-    wt = 2 * spec.dst.num_layers * spec.dst.num_kv_heads * spec.group_in * spec.dst.head_dim * elt
+    # translator parameters: the full matrices, or a latent adapter's two factors
+    per = spec.group_in * spec.dst.head_dim if spec.rank == 0 else spec.rank * (spec.group_in + spec.dst.head_dim)
+    wt = 2 * spec.dst.num_layers * spec.dst.num_kv_heads * per * elt
     flops = 2.0 * T * spec.group_in * spec.dst.head_dim * spec.dst.num_layers * spec.dst.num_kv_heads * 2
     return {"read": rd, "write": wr, "weights": wt, "bytes": rd + wr + wt, "flops": flops}
 
@@ -78,7 +80,7 @@ def _oracle_worker(args):
     wl = synth.make_workload(spec)
     lm = wl.layer_map if wl.layer_map is not None else oracle.layer_map_nearest(spec.src.num_layers,
                                                                                 spec.dst.num_layers)
-    l0 = int(lm[0])
+    l0 = int(np.asarray(lm).reshape(-1)[0])
     k = synth.source_kv(wl, l0, 0)
     if spec.src.rope_base > 0:
         k = oracle.rope_cache(k, spec.src)
@@ -87,8 +89,13 @@ def _oracle_worker(args):
     v = synth.source_kv(wl, l0, 1)
     ks = [k] * spec.src.num_layers
     vs = [v] * spec.src.num_layers
+    if spec.rank > 0:
+        low_rank, wk, wv = (*synth.latent_factors(wl, 0), *synth.latent_factors(wl, 1)), None, None
+    else:
+        low_rank, wk, wv = None, synth.weights(wl, 0), synth.weights(wl, 1)
     p = oracle.OracleProblem(spec.src, spec.dst, lm, wl.src_len, wl.tgt_seq_off, wl.s_max, wl.t_max, ks, vs,
-                             synth.weights(wl, 0), synth.weights(wl, 1), wl.span_lo, wl.span_hi)
+                             wk, wv, wl.span_lo, wl.span_hi, form=spec.form, k_layers=spec.layers_per_target,
+                             low_rank=low_rank)
     rows = 0
     start = time.perf_counter()
     T = wl.total_tgt
@@ -233,13 +240,13 @@ def main():
         dist.init_process_group("nccl", device_id=torch.device("cuda", local_rank))
 
     wl = synth.make_workload(spec)
-    lm = list(wl.layer_map) if wl.layer_map is not None else nearest_map(spec.src.num_layers, spec.dst.num_layers)
+    lm = wl.layer_map.tolist() if wl.layer_map is not None else nearest_map(spec.src.num_layers, spec.dst.num_layers)
     alg = algorithmic(spec, wl, lm)
     tdt = torch.bfloat16 if spec.dtype == "bf16" else torch.float32
     kdt = kvx.KVX_BF16 if spec.dtype == "bf16" else kvx.KVX_FP32
 
     # host inputs (pinned) and the translator
-    mapped = sorted(set(int(x) for x in lm))
+    mapped = sorted(set(int(x) for x in np.asarray(lm).reshape(-1)))
     host_k, host_v = {}, {}
     for l in mapped:
         k = synth.source_kv(wl, l, 0)
@@ -249,8 +256,15 @@ def main():
             k = rotate_np(k, spec.src.rope_base)
         host_k[l] = to_torch(k, spec.dtype, torch, pin=True)
         host_v[l] = to_torch(synth.source_kv(wl, l, 1), spec.dtype, torch, pin=True)
-    tr = kvx.Translator(spec.src, spec.dst, to_torch(synth.weights(wl, 0), spec.dtype, torch),
-                        to_torch(synth.weights(wl, 1), spec.dtype, torch), layer_map=lm, dtype=kdt)
+    if spec.rank > 0:
+        (a_k, b_k), (a_v, b_v) = synth.latent_factors(wl, 0), synth.latent_factors(wl, 1)
+        tr = kvx.Translator(spec.src, spec.dst, None, None, layer_map=lm, dtype=kdt, form=spec.form,
+                            layers_per_target=spec.layers_per_target,
+                            low_rank=tuple(to_torch(x, spec.dtype, torch) for x in (a_k, b_k, a_v, b_v)))
+    else:
+        tr = kvx.Translator(spec.src, spec.dst, to_torch(synth.weights(wl, 0), spec.dtype, torch),
+                            to_torch(synth.weights(wl, 1), spec.dtype, torch), layer_map=lm, dtype=kdt,
+                            form=spec.form, layers_per_target=spec.layers_per_target)
     info = tr.info()
 
     dev = torch.device("cuda", local_rank)

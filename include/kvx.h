@@ -102,36 +102,69 @@ typedef struct {
     int32_t rope_original_max_position; /* LLAMA3: context length of the unscaled model, > 0 */
 } kvx_model_geom;
 
-/* Translator description (the theta of T_theta, Section 5, plus the layer alignment). */
+/* Which source KV heads feed one target KV head.  Section 5 lists the granularities a
+ * translator may act on: individual KV heads, individual layers, groups of layers, and
+ * low-dimensional latent adapters (kvx_translator_create_low_rank). */
+typedef enum {
+    KVX_FORM_GROUPED = 0,       /* per KV head: target head h reads its GQA group of source heads
+                                   (h*r .. h*r+r-1 with r = src heads / dst heads), or source head
+                                   h/e when the target has e times more heads */
+    KVX_FORM_DENSE = 1          /* per layer: every target head reads all src.num_kv_heads heads */
+} kvx_form;
+
+/* Translator description (the theta of T_theta, Section 5, plus the layer alignment).  A
+ * zero-initialised tail (form 0, layers_per_target 0) is the per-KV-head form over one source
+ * layer per target layer. */
 typedef struct {
     kvx_model_geom src;         /* source model A */
     kvx_model_geom dst;         /* target model B */
-    const int32_t* layer_map;   /* host int32[dst.num_layers]: source layer feeding each target
-                                   layer, each in [0, src.num_layers); NULL = nearest relative
-                                   depth (kvx_layer_map_nearest) */
+    const int32_t* layer_map;   /* host int32[dst.num_layers][k] (k = layers_per_target): the source
+                                   layers feeding each target layer, each in [0, src.num_layers);
+                                   NULL = nearest relative depth (kvx_layer_map_nearest), k = 1 only */
     int32_t dtype;              /* kvx_dtype of caches and weights */
     int32_t max_position;       /* RoPE positions must lie in [0, max_position); 0 = 1<<24,
                                    at most 1<<30.  Positions outside are clamped and flagged. */
     int32_t path;               /* kvx_path */
+    int32_t form;               /* kvx_form */
+    int32_t layers_per_target;  /* k: source layers whose heads are concatenated into one target
+                                   layer's input (a group of layers); 0 or 1 = one; at most 4,
+                                   and dst.num_layers * k <= 256 */
 } kvx_translator_desc;
 
 typedef struct kvx_translator kvx_translator;
 
 /* Build a translator.
  *   w_k, w_v: translator matrices, row-major [dst.num_layers][dst.num_kv_heads][in][out] of
- *     desc->dtype, with out = dst.head_dim and in = (src.num_kv_heads/dst.num_kv_heads) *
- *     src.head_dim when src has at least as many KV heads as dst (the input row of target head
- *     h concatenates source heads h*r .. h*r+r-1 in order), else in = src.head_dim (target
- *     head h reads source head h / (dst.num_kv_heads/src.num_kv_heads)).
+ *     desc->dtype, with out = dst.head_dim and in = k * n * src.head_dim: the input row of
+ *     target head h concatenates, for each of its k source layers in layer_map order, the n
+ *     source heads that feed it in ascending order.  n is r = src.num_kv_heads/dst.num_kv_heads
+ *     (heads h*r .. h*r+r-1) in the grouped form when src has at least as many KV heads as dst,
+ *     1 (head h / (dst.num_kv_heads/src.num_kv_heads)) in the grouped form otherwise, and
+ *     src.num_kv_heads in the dense form.
  *   weights_on_device: 0 = host pointers, 1 = device pointers.
  * The library copies the weights into its own device memory (re-laid out for its kernels) and
  * builds its RoPE tables; the caller may free its copies on return.  Synchronous on the
  * current device.  Returns KVX_ERR_UNSUPPORTED unless one head count divides the other,
- * both head dims are in {64, 128, 256} and in <= 512 (in <= 256 for the tcgen05 path), and
- * KVX_ERR_INVALID_ARG for an unknown rope_type or out-of-range schedule parameters.
- * On success *out owns device memory until kvx_destroy. */
+ * both head dims are in {64, 128, 256} and in <= 1024, and KVX_ERR_INVALID_ARG for an unknown
+ * form or rope_type, out-of-range schedule parameters, or layers_per_target > 1 without a
+ * layer_map.  On success *out owns device memory until kvx_destroy. */
 KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* desc, const void* w_k, const void* w_v,
                                          int32_t weights_on_device, kvx_translator** out);
+
+/* Build a translator whose matrices are low-dimensional latent adapters (Section 5):
+ * W[j,h] = A[j,h] . B[j,h] with A [in][rank] and B [rank][out], applied to the span mean as the
+ * two maps x -> x.A -> (x.A).B.
+ *   a_k, b_k, a_v, b_v: row-major [dst.num_layers][dst.num_kv_heads][in][rank] (a_*) and
+ *     [dst.num_layers][dst.num_kv_heads][rank][out] (b_*) of desc->dtype; host or device per
+ *     weights_on_device.  1 <= rank <= 1024.
+ * The library multiplies the factors once, on the device (fp32 accumulation over rank, then
+ * rounded to desc->dtype), and from then on holds only W: the translation reads the source and
+ * writes the target cache at the same HBM cost whatever the rank, so the product costs the
+ * kernels nothing, while two chained contractions would add a round trip through on-chip
+ * memory.  Everything else is as for kvx_translator_create. */
+KVX_API kvx_status kvx_translator_create_low_rank(const kvx_translator_desc* desc, int32_t rank, const void* a_k,
+                                                  const void* b_k, const void* a_v, const void* b_v,
+                                                  int32_t weights_on_device, kvx_translator** out);
 
 /* Source KV cache KV_A(C) (Section 2.1), one K and one V tensor per source layer, each
  * [batch][src.num_kv_heads][max_seq][src.head_dim] addressed by the strides below with the
@@ -249,7 +282,8 @@ KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
  *   w_k, w_v: DEVICE pointers, row-major [dst.num_layers][dst.num_kv_heads][in][out] of
  *     desc->dtype; they are copied into the scratch array on every call.  Both together must fit
  *     KVX_STATIC_SCRATCH_BYTES minus 2304 bytes, else KVX_ERR_UNSUPPORTED (nothing is launched).
- *   desc->path is ignored.
+ *   desc->path is ignored; desc->form must be KVX_FORM_GROUPED and desc->layers_per_target at
+ *     most 1 (else KVX_ERR_UNSUPPORTED).
  *   status_bits: host pointer or NULL.  If set, the call synchronises stream, writes the device
  *     status word there and returns KVX_ERR_DEVICE_STATUS when it is nonzero; if NULL, the call is
  *     asynchronous on stream like kvx_translate.

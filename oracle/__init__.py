@@ -62,6 +62,8 @@ class Problem(ctypes.Structure):
         ("src_pos", I32P), ("tgt_pos", I32P),
         ("src_k", ctypes.POINTER(F32P)), ("src_v", ctypes.POINTER(F32P)),
         ("w_k", F32P), ("w_v", F32P),
+        ("form", ctypes.c_int32), ("k_layers", ctypes.c_int32), ("rank", ctypes.c_int32),
+        ("a_k", F32P), ("b_k", F32P), ("a_v", F32P), ("b_v", F32P),
     ]
 
 
@@ -142,14 +144,18 @@ class OracleProblem:
 
     def __init__(self, src_geom, dst_geom, layer_map, src_len, tgt_seq_off, s_max, t_max,
                  src_k: Sequence[np.ndarray], src_v: Sequence[np.ndarray], w_k, w_v,
-                 span_lo=None, span_hi=None, src_pos=None, tgt_pos=None):
+                 span_lo=None, span_hi=None, src_pos=None, tgt_pos=None, form: int = 0, k_layers: int = 1,
+                 low_rank=None):
+        """layer_map: [Lt] or [Lt, k_layers] source layers.  form 0: GQA group, 1: dense (all
+        source heads).  low_rank: (A_K, B_K, A_V, B_V) latent adapter factors; w_k/w_v are then
+        ignored (pass None)."""
         self.keep = []
 
         def keep(a):
             self.keep.append(a)
             return a
 
-        lm = keep(_i32(layer_map))
+        lm = keep(_i32(np.asarray(layer_map).reshape(-1)))
         sl = keep(_i32(src_len))
         so = keep(_i32(tgt_seq_off))
         lo, hi = keep(_i32(span_lo)), keep(_i32(span_hi))
@@ -158,7 +164,10 @@ class OracleProblem:
         vs = [keep(np.ascontiguousarray(a, np.float32)) for a in src_v]
         kp = keep((F32P * len(ks))(*[_p(a, F32P) for a in ks]))
         vp = keep((F32P * len(vs))(*[_p(a, F32P) for a in vs]))
-        wk, wv = keep(np.ascontiguousarray(w_k, np.float32)), keep(np.ascontiguousarray(w_v, np.float32))
+        f32 = lambda a: None if a is None else keep(np.ascontiguousarray(a, np.float32))
+        wk, wv = f32(w_k), f32(w_v)
+        ak, bk, av, bv = (None,) * 4 if low_rank is None else tuple(f32(a) for a in low_rank)
+        rank = 0 if low_rank is None else int(np.asarray(low_rank[0]).shape[-1])
         self.T = int(so[-1])
         self.Lt, self.Ht, self.dt = dst_geom.num_layers, dst_geom.num_kv_heads, dst_geom.head_dim
         self.p = Problem(src_geom.num_layers, src_geom.num_kv_heads, src_geom.head_dim, rope_sched(src_geom),
@@ -166,7 +175,8 @@ class OracleProblem:
                          _p(lm, I32P), len(sl), s_max, t_max, _p(sl, I32P), _p(so, I32P),
                          _p(lo, I32P), _p(hi, I32P), _p(sp, I32P), _p(tp, I32P),
                          ctypes.cast(kp, ctypes.POINTER(F32P)), ctypes.cast(vp, ctypes.POINTER(F32P)),
-                         _p(wk, F32P), _p(wv, F32P))
+                         _p(wk, F32P), _p(wv, F32P), int(form), int(k_layers), rank,
+                         _p(ak, F32P), _p(bk, F32P), _p(av, F32P), _p(bv, F32P))
 
     def translate(self):
         """Returns (K, V), each [Lt, Ht, T_total, dt] float64."""

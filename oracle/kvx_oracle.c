@@ -7,19 +7,24 @@
  * header, table or constant with it.
  *
  * What it computes (paper Section 4, translation operator KV^_B = T_{A->B}(KV_A),
- * and Section 5, parameterised translator T_theta, applied per layer and per KV
- * head, one of the granularities Section 5 lists).  For every target layer j,
- * target KV head h, K or V, and target token t of sequence b:
+ * and Section 5, parameterised translator T_theta, at the granularities
+ * Section 5 lists: individual KV heads, individual layers, groups of layers,
+ * low-dimensional latent adapters).  For every target layer j, target KV head
+ * h, K or V, and target token t of sequence b:
  *
- *   1. source layer     l = layer_map[j]                 (nearest relative depth)
+ *   1. source layers    l_k = layer_map[j][k], k < k_layers (one: nearest
+ *                       relative depth; several: a group of source layers)
  *   2. source span      [lo_t, hi_t) of the source tokens of sequence b
- *   3. for every s in the span and every grouped source head g (GQA regroup):
- *        K: u_g = R_{d_s,base_s}(-p_s) K[l,b,g,s]   (undo the source RoPE)
- *        V: u_g = V[l,b,g,s]
- *      and u = concat_g u_g  (length in = r*d_s, or d_s when target heads
- *      outnumber source heads)
+ *   3. for every s in the span, every source layer l_k and every source head
+ *      g feeding target head h (its GQA group, or all heads in the dense
+ *      per-layer form):
+ *        K: u = R_{d_s,base_s}(-p_s) K[l_k,b,g,s]   (undo the source RoPE)
+ *        V: u = V[l_k,b,g,s]
+ *      concatenated layer by layer, heads ascending within a layer (length in)
  *   4. xbar = (1/|span|) sum_s u                      (span mean)
- *   5. y = xbar . W[j,h]      with W[j,h] of shape [in, out=d_t]
+ *   5. y = xbar . W[j,h]      with W[j,h] of shape [in, out=d_t]; for a
+ *      low-rank latent adapter, z = xbar . A[j,h] ([in, rank]) and then
+ *      y = z . B[j,h] ([rank, out])
  *   6. K: y <- R_{d_t,base_t}(+p_t) y                 (apply the target RoPE)
  *
  * R_{d,base}(p) is the half-split rotary map: channel pairs (i, i+d/2) for
@@ -171,13 +176,27 @@ typedef struct {
     const int32_t* tgt_pos;                   /* [T_total] or NULL (= index) */
     const float* const* src_k;                /* [Ls] -> [B][Hs][s_max][ds] */
     const float* const* src_v;
-    const float* w_k;                         /* [Lt][Ht][in][dt] */
+    const float* w_k;                         /* [Lt][Ht][in][dt] (full-rank form) */
     const float* w_v;
+    int32_t form;                             /* 0: GQA group of source heads, 1: all source heads */
+    int32_t k_layers;                         /* source layers per target layer (layer_map [Lt][k]) */
+    int32_t rank;                             /* > 0: latent adapter A [Lt][Ht][in][rank], B [Lt][Ht][rank][dt] */
+    const float* a_k; const float* b_k;
+    const float* a_v; const float* b_v;
 } kvxo_problem;
+
+/* Source heads per source layer that feed one target head. */
+static int heads_per_layer(const kvxo_problem* p)
+{
+    if (p->form == 1) return p->Hs;
+    return p->Hs >= p->Ht ? p->Hs / p->Ht : 1;
+}
+
+static int layers_per_target(const kvxo_problem* p) { return p->k_layers > 0 ? p->k_layers : 1; }
 
 static int group_in(const kvxo_problem* p)
 {
-    return p->Hs >= p->Ht ? (p->Hs / p->Ht) * p->ds : p->ds;
+    return layers_per_target(p) * heads_per_layer(p) * p->ds;
 }
 
 /* One output row: target layer j, target head h, kv (0 = K, 1 = V), packed
@@ -186,37 +205,59 @@ static int group_in(const kvxo_problem* p)
 KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int tp, double* out)
 {
     if (p->Hs % p->Ht != 0 && p->Ht % p->Hs != 0) return 1;
+    if (p->form != 0 && p->form != 1) return 1;
     int b = 0;
     while (b < p->batch - 1 && p->tgt_seq_off[b + 1] <= tp) ++b;
     int t = tp - p->tgt_seq_off[b];
-    int l = p->layer_map[j];                                   /* step 1 */
+    int K = layers_per_target(p);
     int lo = p->span_lo ? p->span_lo[tp] : t;                  /* step 2 */
     int hi = p->span_hi ? p->span_hi[tp] : t + 1;
     int in = group_in(p);
-    int r = p->Hs >= p->Ht ? p->Hs / p->Ht : 1;
-    int g0 = p->Hs >= p->Ht ? h * r : h / (p->Ht / p->Hs);
-    const float* src = kv == 0 ? p->src_k[l] : p->src_v[l];
+    int nh = heads_per_layer(p);
+    int g0 = p->form == 1 ? 0 : (p->Hs >= p->Ht ? h * nh : h / (p->Ht / p->Hs));
 
     double* sum = (double*)calloc((size_t)in, sizeof(double));
     double* u = (double*)malloc(sizeof(double) * (size_t)p->ds);
     for (int s = lo; s < hi; ++s) {                            /* step 3 */
         double ps = p->src_pos ? (double)p->src_pos[(size_t)b * p->s_max + s] : (double)s;
-        for (int q = 0; q < r; ++q) {
-            int g = g0 + q;
-            const float* row = src + (((size_t)b * p->Hs + g) * p->s_max + s) * p->ds;
-            for (int e = 0; e < p->ds; ++e) u[e] = (double)row[e];
-            if (kv == 0) kvxo_rope_sched_apply(u, p->ds, &p->rope_s, ps, -1);
-            for (int e = 0; e < p->ds; ++e) sum[q * p->ds + e] += u[e];
+        for (int k = 0; k < K; ++k) {
+            int l = p->layer_map[j * K + k];                   /* step 1 */
+            const float* src = kv == 0 ? p->src_k[l] : p->src_v[l];
+            for (int q = 0; q < nh; ++q) {
+                int g = g0 + q;
+                const float* row = src + (((size_t)b * p->Hs + g) * p->s_max + s) * p->ds;
+                for (int e = 0; e < p->ds; ++e) u[e] = (double)row[e];
+                if (kv == 0) kvxo_rope_sched_apply(u, p->ds, &p->rope_s, ps, -1);
+                for (int e = 0; e < p->ds; ++e) sum[(k * nh + q) * p->ds + e] += u[e];
+            }
         }
     }
     double n = (double)(hi - lo);                              /* step 4 */
     for (int i = 0; i < in; ++i) sum[i] /= n;
 
-    const float* W = (kv == 0 ? p->w_k : p->w_v) + ((size_t)j * p->Ht + h) * (size_t)in * p->dt;
-    for (int o = 0; o < p->dt; ++o) {                          /* step 5 */
-        double acc = 0.0;
-        for (int i = 0; i < in; ++i) acc += sum[i] * (double)W[(size_t)i * p->dt + o];
-        out[o] = acc;
+    if (p->rank > 0) {                                         /* step 5, latent adapter */
+        size_t jh = (size_t)j * p->Ht + h;
+        const float* A = (kv == 0 ? p->a_k : p->a_v) + jh * (size_t)in * p->rank;
+        const float* B = (kv == 0 ? p->b_k : p->b_v) + jh * (size_t)p->rank * p->dt;
+        double* z = (double*)malloc(sizeof(double) * (size_t)p->rank);
+        for (int c = 0; c < p->rank; ++c) {
+            double acc = 0.0;
+            for (int i = 0; i < in; ++i) acc += sum[i] * (double)A[(size_t)i * p->rank + c];
+            z[c] = acc;
+        }
+        for (int o = 0; o < p->dt; ++o) {
+            double acc = 0.0;
+            for (int c = 0; c < p->rank; ++c) acc += z[c] * (double)B[(size_t)c * p->dt + o];
+            out[o] = acc;
+        }
+        free(z);
+    } else {                                                   /* step 5 */
+        const float* W = (kv == 0 ? p->w_k : p->w_v) + ((size_t)j * p->Ht + h) * (size_t)in * p->dt;
+        for (int o = 0; o < p->dt; ++o) {
+            double acc = 0.0;
+            for (int i = 0; i < in; ++i) acc += sum[i] * (double)W[(size_t)i * p->dt + o];
+            out[o] = acc;
+        }
     }
     if (kv == 0) {                                             /* step 6 */
         double pt = p->tgt_pos ? (double)p->tgt_pos[tp] : (double)t;

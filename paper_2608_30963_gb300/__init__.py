@@ -53,9 +53,13 @@ def model_geom(g) -> kvx_model_geom:
                           int(getattr(g, "rope_original_max_position", 8192)))
 
 
+KVX_FORM_GROUPED, KVX_FORM_DENSE = 0, 1
+
+
 class kvx_translator_desc(ctypes.Structure):
     _fields_ = [("src", kvx_model_geom), ("dst", kvx_model_geom), ("layer_map", I32P),
-                ("dtype", ctypes.c_int32), ("max_position", ctypes.c_int32), ("path", ctypes.c_int32)]
+                ("dtype", ctypes.c_int32), ("max_position", ctypes.c_int32), ("path", ctypes.c_int32),
+                ("form", ctypes.c_int32), ("layers_per_target", ctypes.c_int32)]
 
 
 class kvx_src_kv(ctypes.Structure):
@@ -84,7 +88,7 @@ class kvx_translator_info(ctypes.Structure):
                 ("weight_bytes", ctypes.c_int64), ("table_bytes", ctypes.c_int64)]
 
 
-EXPORTS = ["kvx_translator_create", "kvx_translate", "kvx_build_alignment", "kvx_layer_map_nearest",
+EXPORTS = ["kvx_translator_create", "kvx_translator_create_low_rank", "kvx_translate", "kvx_build_alignment", "kvx_layer_map_nearest",
            "kvx_get_device_status", "kvx_get_info", "kvx_launches_per_translate", "kvx_last_error",
            "kvx_destroy", "kvx_translate_static", "kvx_static_last_error"]
 KVX_STATIC_SCRATCH_BYTES = 8 << 20
@@ -116,6 +120,8 @@ def lib():
         L = ctypes.CDLL(path)
         L.kvx_translator_create.argtypes = [ctypes.POINTER(kvx_translator_desc), VP, VP, ctypes.c_int32,
                                             ctypes.POINTER(VP)]
+        L.kvx_translator_create_low_rank.argtypes = [ctypes.POINTER(kvx_translator_desc), ctypes.c_int32, VP, VP,
+                                                     VP, VP, ctypes.c_int32, ctypes.POINTER(VP)]
         L.kvx_translate.argtypes = [VP, ctypes.POINTER(kvx_src_kv), ctypes.POINTER(kvx_tgt_tokens),
                                     ctypes.POINTER(kvx_dst_kv), VP]
         L.kvx_build_alignment.argtypes = [ctypes.c_int32, ctypes.c_int32, ctypes.c_int32, VP, VP, VP, VP, VP, VP,
@@ -158,6 +164,14 @@ def kvx_translator_create(desc: kvx_translator_desc, w_k_ptr: int, w_v_ptr: int,
     h = VP()
     _check(lib().kvx_translator_create(ctypes.byref(desc), VP(w_k_ptr), VP(w_v_ptr), int(weights_on_device),
                                        ctypes.byref(h)))
+    return h.value
+
+
+def kvx_translator_create_low_rank(desc: kvx_translator_desc, rank: int, a_k_ptr: int, b_k_ptr: int, a_v_ptr: int,
+                                   b_v_ptr: int, weights_on_device: bool) -> int:
+    h = VP()
+    _check(lib().kvx_translator_create_low_rank(ctypes.byref(desc), int(rank), VP(a_k_ptr), VP(b_k_ptr),
+                                                VP(a_v_ptr), VP(b_v_ptr), int(weights_on_device), ctypes.byref(h)))
     return h.value
 
 
@@ -224,18 +238,29 @@ def _stream(stream) -> int:
 
 class Translator:
     """Owns one kvx_translator.  Weights are torch tensors (host or device)
-    [L_t, H_t, in, out] of the translator dtype; they are copied at creation."""
+    [L_t, H_t, in, out] of the translator dtype; they are copied at creation.
+    With low_rank=(A_K, B_K, A_V, B_V) ([L_t, H_t, in, rank] and [L_t, H_t, rank, out]),
+    w_k and w_v are ignored and the translator is a latent adapter.  layer_map is
+    [L_t] or, with layers_per_target = k > 1, [L_t, k] (nested or flat)."""
 
-    def __init__(self, src_geom, dst_geom, w_k, w_v, layer_map: Optional[Sequence[int]] = None,
-                 dtype: int = KVX_BF16, max_position: int = 0, path: int = KVX_PATH_AUTO):
+    def __init__(self, src_geom, dst_geom, w_k, w_v, layer_map: Optional[Sequence] = None,
+                 dtype: int = KVX_BF16, max_position: int = 0, path: int = KVX_PATH_AUTO,
+                 form: int = KVX_FORM_GROUPED, layers_per_target: int = 1, low_rank=None):
         lm = None
         if layer_map is not None:
-            self._lm = (ctypes.c_int32 * len(layer_map))(*[int(x) for x in layer_map])
+            flat = [int(x) for row in layer_map for x in (row if hasattr(row, "__len__") else [row])]
+            self._lm = (ctypes.c_int32 * len(flat))(*flat)
             lm = ctypes.cast(self._lm, I32P)
-        self.desc = kvx_translator_desc(model_geom(src_geom), model_geom(dst_geom), lm, dtype, max_position, path)
-        w_k = w_k.contiguous()
-        w_v = w_v.contiguous()
-        self.handle = kvx_translator_create(self.desc, _ptr(w_k), _ptr(w_v), w_k.is_cuda)
+        self.desc = kvx_translator_desc(model_geom(src_geom), model_geom(dst_geom), lm, dtype, max_position, path,
+                                        form, layers_per_target)
+        if low_rank is not None:
+            a_k, b_k, a_v, b_v = (t.contiguous() for t in low_rank)
+            self.handle = kvx_translator_create_low_rank(self.desc, a_k.shape[-1], _ptr(a_k), _ptr(b_k), _ptr(a_v),
+                                                         _ptr(b_v), a_k.is_cuda)
+        else:
+            w_k = w_k.contiguous()
+            w_v = w_v.contiguous()
+            self.handle = kvx_translator_create(self.desc, _ptr(w_k), _ptr(w_v), w_k.is_cuda)
         self.src_geom, self.dst_geom = src_geom, dst_geom
 
     def info(self) -> kvx_translator_info:

@@ -10,6 +10,7 @@
 namespace kvx {
 
 constexpr int KVX_MAX_ALIGNED_LAYERS = 96;   // target layers the identity-alignment kernel takes (param space)
+constexpr int KVX_MAX_SRC_SLOTS = 256;       // (target layer, source-layer slot) pairs one launch addresses
 constexpr int KVX_MAX_ALIGNED_BATCH = 256;   // sequences whose metadata it keeps in shared memory
 
 // Rotation frequencies as fixed-point turns: turns[i] = round(2^64 * f_i / (2 pi)),
@@ -61,6 +62,9 @@ struct TranslateParams {
     int in_dim;     // input width of one translator matrix
     int r;          // source heads grouped into one target head (Hs >= Ht), else 1
     int e;          // target heads sharing one source head (Ht > Hs), else 1
+    int dense;      // 1: every source KV head feeds each target head (per-layer form)
+    int kl;         // source layers concatenated into one target layer's input (group of layers)
+    int hpl;        // source heads per source layer in one input row: in_dim = kl * hpl * ds
     int Lt;
     // source cache
     int batch, src_max_seq;
@@ -85,12 +89,28 @@ struct TranslateParams {
     unsigned* status;
     // weights (layout depends on the kernel)
     const void* w;
-    // per TARGET layer: the mapped source layer's K/V and the target layer's K/V
-    const void* src_k[KVX_MAX_TARGET_LAYERS];
-    const void* src_v[KVX_MAX_TARGET_LAYERS];
+    // source K/V per (target layer j, layer slot k) at [j * kl + k], and the target layer's K/V
+    const void* src_k[KVX_MAX_SRC_SLOTS];
+    const void* src_v[KVX_MAX_SRC_SLOTS];
     void* dst_k[KVX_MAX_TARGET_LAYERS];
     void* dst_v[KVX_MAX_TARGET_LAYERS];
 };
+
+// First source head feeding target head h: its GQA group (h*r), the source head it
+// repeats (h/e), or head 0 in the dense per-layer form.
+__device__ __forceinline__ int src_head0(const TranslateParams& P, int h)
+{
+    return P.dense ? 0 : (P.r > 1 ? h * P.r : h / P.e);
+}
+
+// Head-block q of target head h's input row (d_s channels of one source head):
+// the source cache slot (index into src_k / src_v) and the source head.
+__device__ __forceinline__ void head_block(const TranslateParams& P, int j, int h, int q, int& slot, int& g)
+{
+    const int k = q / P.hpl;
+    slot = j * P.kl + k;
+    g = src_head0(P, h) + (q - k * P.hpl);
+}
 
 __device__ __forceinline__ void set_status(unsigned* status, unsigned bit)
 {

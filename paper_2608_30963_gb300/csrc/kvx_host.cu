@@ -15,10 +15,11 @@ using namespace kvx;
 
 struct kvx_translator {
     kvx_translator_desc desc;
-    int layer_map[KVX_MAX_TARGET_LAYERS];
+    int layer_map[KVX_MAX_SRC_SLOTS];   // [j * kl + k]: source layers of target layer j
     int device = 0;
     int num_sms = 0;
     int in_dim = 0, r = 1, e = 1;
+    int dense = 0, kl = 1, hpl = 1;     // form, source layers per target layer, heads per layer block
     int path = KVX_PATH_SIMT;
     int max_position = 0;
     void* w = nullptr;           // SIMT: [2][Lt][Ht][in][out] dtype; tcgen05: pre-swizzled images
@@ -152,33 +153,41 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
     int max_pos = desc->max_position ? desc->max_position : (1 << 24);
     if (max_pos < 1 || max_pos > (1 << 30))
         return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<30]");
+    if (desc->form != KVX_FORM_GROUPED && desc->form != KVX_FORM_DENSE)
+        return fail(KVX_ERR_INVALID_ARG, "create: unknown form %d", desc->form);
+    const int kl = desc->layers_per_target > 1 ? desc->layers_per_target : 1;
+    if (desc->layers_per_target < 0 || kl > 4 || d.num_layers * kl > KVX_MAX_SRC_SLOTS)
+        return fail(KVX_ERR_INVALID_ARG, "create: layers_per_target %d outside [0, 4] or more than %d "
+                                         "(target layer, source layer) pairs", desc->layers_per_target,
+                    KVX_MAX_SRC_SLOTS);
+    if (kl > 1 && !desc->layer_map)
+        return fail(KVX_ERR_INVALID_ARG, "create: layers_per_target > 1 needs an explicit layer_map");
 
     kvx_translator* t = new kvx_translator();
     t->desc = *desc;
     t->desc.layer_map = nullptr;
     t->max_position = max_pos;
+    t->kl = kl;
+    t->dense = desc->form == KVX_FORM_DENSE;
     if (desc->layer_map) {
-        for (int j = 0; j < d.num_layers; ++j) {
-            if (desc->layer_map[j] < 0 || desc->layer_map[j] >= s.num_layers) {
+        for (int i = 0; i < d.num_layers * kl; ++i) {
+            if (desc->layer_map[i] < 0 || desc->layer_map[i] >= s.num_layers) {
                 delete t;
-                return fail(KVX_ERR_INVALID_ARG, "create: layer_map[%d] = %d outside [0, %d)", j,
-                            desc->layer_map[j], s.num_layers);
+                return fail(KVX_ERR_INVALID_ARG, "create: layer_map[%d] = %d outside [0, %d)", i,
+                            desc->layer_map[i], s.num_layers);
             }
-            t->layer_map[j] = desc->layer_map[j];
+            t->layer_map[i] = desc->layer_map[i];
         }
     } else {
         kvx_layer_map_nearest(s.num_layers, d.num_layers, t->layer_map);
     }
-    if (s.num_kv_heads >= d.num_kv_heads) {
-        t->r = s.num_kv_heads / d.num_kv_heads;
-        t->in_dim = t->r * s.head_dim;
-    } else {
-        t->e = d.num_kv_heads / s.num_kv_heads;
-        t->in_dim = s.head_dim;
-    }
-    if (t->in_dim > 512) {
+    if (s.num_kv_heads >= d.num_kv_heads) t->r = s.num_kv_heads / d.num_kv_heads;
+    else t->e = d.num_kv_heads / s.num_kv_heads;
+    t->hpl = t->dense ? s.num_kv_heads : t->r;
+    t->in_dim = kl * t->hpl * s.head_dim;
+    if (t->in_dim > 1024) {
         delete t;
-        return fail(KVX_ERR_UNSUPPORTED, "create: translator input width %d > 512", t->in_dim);
+        return fail(KVX_ERR_UNSUPPORTED, "create: translator input width %d > 1024", t->in_dim);
     }
 
     if (cudaGetDevice(&t->device) != cudaSuccess ||
@@ -280,6 +289,52 @@ err:
     return st;
 }
 
+extern "C" KVX_API kvx_status kvx_translator_create_low_rank(const kvx_translator_desc* desc, int32_t rank,
+                                                             const void* a_k, const void* b_k, const void* a_v,
+                                                             const void* b_v, int32_t weights_on_device,
+                                                             kvx_translator** out)
+{
+    if (!desc || !a_k || !b_k || !a_v || !b_v || !out) return fail(KVX_ERR_INVALID_ARG, "create_low_rank: NULL argument");
+    *out = nullptr;
+    if (rank < 1 || rank > 1024) return fail(KVX_ERR_INVALID_ARG, "create_low_rank: rank %d outside [1, 1024]", rank);
+    const kvx_model_geom& s = desc->src;
+    const kvx_model_geom& d = desc->dst;
+    if (s.num_layers < 1 || d.num_layers < 1 || s.num_kv_heads < 1 || d.num_kv_heads < 1 ||
+        d.num_layers > KVX_MAX_TARGET_LAYERS || !head_dim_ok(s.head_dim) || !head_dim_ok(d.head_dim))
+        return fail(KVX_ERR_INVALID_ARG, "create_low_rank: bad layer, head or head_dim counts");
+    if (s.num_kv_heads % d.num_kv_heads != 0 && d.num_kv_heads % s.num_kv_heads != 0)
+        return fail(KVX_ERR_UNSUPPORTED, "create_low_rank: neither KV head count divides the other");
+    if (desc->dtype != KVX_BF16 && desc->dtype != KVX_FP32)
+        return fail(KVX_ERR_INVALID_ARG, "create_low_rank: unknown dtype %d", desc->dtype);
+    // the input width, as kvx_translator_create derives it (it validates the rest)
+    const int kl = desc->layers_per_target > 1 ? desc->layers_per_target : 1;
+    const int hpl = desc->form == KVX_FORM_DENSE ? s.num_kv_heads
+                                                 : (s.num_kv_heads >= d.num_kv_heads ? s.num_kv_heads / d.num_kv_heads : 1);
+    const long long in_dim = (long long)kl * hpl * s.head_dim;
+    if (in_dim > 1024) return fail(KVX_ERR_UNSUPPORTED, "create_low_rank: translator input width %lld > 1024", in_dim);
+    const size_t elt = desc->dtype == KVX_BF16 ? 2 : 4;
+    const int n = d.num_layers * d.num_kv_heads;
+    const size_t a_bytes = (size_t)n * in_dim * rank * elt, b_bytes = (size_t)n * rank * d.head_dim * elt;
+    const size_t w_bytes = (size_t)n * in_dim * d.head_dim * elt;
+    char* buf = nullptr;
+    if (cudaMalloc(&buf, 2 * (a_bytes + b_bytes + w_bytes)) != cudaSuccess)
+        return fail(KVX_ERR_OOM, "create_low_rank: factor allocation");
+    char *ak = buf, *av = ak + a_bytes, *bk = av + a_bytes, *bv = bk + b_bytes, *wk = bv + b_bytes, *wv = wk + w_bytes;
+    const cudaMemcpyKind kind = weights_on_device ? cudaMemcpyDeviceToDevice : cudaMemcpyHostToDevice;
+    cudaError_t ce;
+    if ((ce = cudaMemcpy(ak, a_k, a_bytes, kind)) != cudaSuccess || (ce = cudaMemcpy(av, a_v, a_bytes, kind)) != cudaSuccess ||
+        (ce = cudaMemcpy(bk, b_k, b_bytes, kind)) != cudaSuccess || (ce = cudaMemcpy(bv, b_v, b_bytes, kind)) != cudaSuccess ||
+        (ce = launch_fold_low_rank(ak, bk, wk, n, (int)in_dim, rank, d.head_dim, desc->dtype, 0)) != cudaSuccess ||
+        (ce = launch_fold_low_rank(av, bv, wv, n, (int)in_dim, rank, d.head_dim, desc->dtype, 0)) != cudaSuccess ||
+        (ce = cudaDeviceSynchronize()) != cudaSuccess) {
+        cudaFree(buf);
+        return fail(KVX_ERR_CUDA, "create_low_rank: factor product: %s", cudaGetErrorString(ce));
+    }
+    const kvx_status st = kvx_translator_create(desc, wk, wv, 1, out);
+    cudaFree(buf);
+    return st;
+}
+
 static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
@@ -316,6 +371,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
     P.Hs = D.src.num_kv_heads; P.ds = D.src.head_dim;
     P.Ht = D.dst.num_kv_heads; P.dt = D.dst.head_dim;
     P.in_dim = tr->in_dim; P.r = tr->r; P.e = tr->e; P.Lt = Lt;
+    P.dense = tr->dense; P.kl = tr->kl; P.hpl = tr->hpl;
     P.batch = src->batch; P.src_max_seq = src->max_seq;
     P.sb = src->stride_b; P.sh = src->stride_h; P.ss = src->stride_s;
     P.src_seq_len = src->seq_len; P.src_pos = src->pos;
@@ -329,18 +385,24 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
     P.rope_same = tr->rope_same;
     P.status = tr->status;
     P.w = tr->w;
+    for (int i = 0; i < Lt * tr->kl; ++i) {
+        const int l = tr->layer_map[i];
+        P.src_k[i] = src->k[l]; P.src_v[i] = src->v[l];
+        if (!P.src_k[i] || !P.src_v[i])
+            return fail(KVX_ERR_INVALID_ARG, "translate: NULL cache pointer for source layer %d", l);
+        if (!aligned16(P.src_k[i]) || !aligned16(P.src_v[i]))
+            return fail(KVX_ERR_INVALID_ARG, "translate: cache pointers must be 16-byte aligned (source layer %d)", l);
+    }
     for (int j = 0; j < Lt; ++j) {
-        const int l = tr->layer_map[j];
-        P.src_k[j] = src->k[l]; P.src_v[j] = src->v[l];
         P.dst_k[j] = dst->k[j]; P.dst_v[j] = dst->v[j];
-        if (!P.src_k[j] || !P.src_v[j] || !P.dst_k[j] || !P.dst_v[j])
+        if (!P.dst_k[j] || !P.dst_v[j])
             return fail(KVX_ERR_INVALID_ARG, "translate: NULL cache pointer for target layer %d", j);
-        if (!aligned16(P.src_k[j]) || !aligned16(P.src_v[j]) || !aligned16(P.dst_k[j]) || !aligned16(P.dst_v[j]))
-            return fail(KVX_ERR_INVALID_ARG, "translate: cache pointers must be 16-byte aligned (layer %d)", j);
+        if (!aligned16(P.dst_k[j]) || !aligned16(P.dst_v[j]))
+            return fail(KVX_ERR_INVALID_ARG, "translate: cache pointers must be 16-byte aligned (target layer %d)", j);
     }
     cudaError_t ce;
     if (tr->path == KVX_PATH_TCGEN05 && !tgt->span_lo &&
-        aligned_supported(tr->in_dim, D.dst.head_dim, D.src.head_dim, Lt, src->batch)) {
+        aligned_supported(tr->in_dim, D.dst.head_dim, D.src.head_dim, Lt, src->batch, tr->kl)) {
         // identity alignment: tensor-TMA fed kernel
         if (tr->maps.empty()) tr->maps.resize((size_t)2 * KVX_MAX_ALIGNED_LAYERS * kvx_translator::kMapWays);
         const void* maps[2 * KVX_MAX_ALIGNED_LAYERS];

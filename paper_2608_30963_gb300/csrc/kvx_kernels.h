@@ -8,6 +8,9 @@ struct TranslateParams;
 
 size_t simt_smem_bytes(int in_dim, int dt);
 cudaError_t launch_translate_simt(const TranslateParams& P, int dtype, cudaStream_t stream);
+// W = A . B for n (layer, head, K|V) matrices (latent adapters, at translator creation)
+cudaError_t launch_fold_low_rank(const void* a, const void* b, void* w, int n, int in_dim, int rank, int out,
+                                 int dtype, cudaStream_t stream);
 
 cudaError_t launch_build_alignment(int batch, int total_tgt, const int* src_seq_off, const int* src_end,
                                    const int* tgt_seq_off, const int* tgt_end, int* span_lo, int* span_hi,
@@ -33,7 +36,7 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
                                 int plan_tokens, cudaStream_t stream, int* launches);
 
 // identity-alignment tensor-core path (tensor-TMA fed)
-bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch);
+bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch, int kl);
 size_t aligned_map_bytes();
 bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int Hs, int batch, long long ss,
                        long long sh, long long sb);

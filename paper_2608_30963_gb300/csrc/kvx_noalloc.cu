@@ -79,6 +79,9 @@ extern "C" KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* de
         return fail(KVX_ERR_UNSUPPORTED, "translate_static: neither KV head count divides the other");
     if (desc->dtype != KVX_BF16 && desc->dtype != KVX_FP32)
         return fail(KVX_ERR_INVALID_ARG, "translate_static: unknown dtype %d", desc->dtype);
+    if (desc->form != KVX_FORM_GROUPED || desc->layers_per_target > 1)
+        return fail(KVX_ERR_UNSUPPORTED, "translate_static: only the per-KV-head form over one source layer per "
+                                         "target layer");
     if (!rope_schedule_ok(s) || !rope_schedule_ok(d))
         return fail(KVX_ERR_INVALID_ARG, "translate_static: unknown rope_type or schedule parameters out of range");
     const int max_pos = desc->max_position ? desc->max_position : (1 << 24);
@@ -161,6 +164,7 @@ extern "C" KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* de
         memset(&P, 0, sizeof P);
         P.Hs = s.num_kv_heads; P.ds = s.head_dim; P.Ht = d.num_kv_heads; P.dt = d.head_dim;
         P.in_dim = in_dim; P.r = r; P.e = e; P.Lt = d.num_layers;
+        P.dense = 0; P.kl = 1; P.hpl = r;
         P.batch = src->batch; P.src_max_seq = src->max_seq;
         P.sb = src->stride_b; P.sh = src->stride_h; P.ss = src->stride_s;
         P.src_seq_len = src->seq_len; P.src_pos = src->pos;

@@ -1,8 +1,10 @@
 // kvx_simt.cu -- CUDA-core translation kernel.
 //
 // One CTA per (32-token tile, target head, target layer, K|V).  Three phases:
-//   1. gather the span rows of the grouped source heads, undo the source RoPE
-//      (K), take the span mean -> A[32][in] (fp32, shared memory);
+//   1. gather the span rows of the source heads feeding the target head (its
+//      GQA group, or every head in the dense form, of one or several source
+//      layers), undo the source RoPE (K), take the span mean -> A[32][in]
+//      (fp32, shared memory);
 //   2. projection Y[32][d_t] = A . W[j,h] (fp32 FMA, W streamed from L2);
 //   3. apply the target RoPE (K) and store the rows into the target cache.
 // It serves the float32 caches and any geometry the tensor-core kernel does
@@ -31,7 +33,6 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
     if ((int)threadIdx.x < ntok) tinfo[threadIdx.x] = resolve_token(P, t0 + threadIdx.x);
     __syncthreads();
 
-    const T* src = (const T*)(kv ? P.src_v[j] : P.src_k[j]);
     const bool rot_s = kv == 0 && P.rs.enabled;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int hs = P.ds >> 1;
@@ -45,7 +46,9 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
         const TokenInfo ti = tinfo[tt];
         for (int k = lane; k < P.in_dim; k += 32) {
             const int q = k / P.ds, c = k - q * P.ds;
-            const int g = P.r > 1 ? h * P.r + q : h / P.e;
+            int slot, g;
+            head_block(P, j, h, q, slot, g);
+            const T* src = (const T*)(kv ? P.src_v[slot] : P.src_k[slot]);
             const T* base = src + (long long)ti.b * P.sb + (long long)g * P.sh;
             float acc = 0.f;
             for (int s = ti.lo; s < ti.hi; ++s) {
@@ -106,6 +109,40 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
         }
         dst[ti.dst_off + hoff + c] = from_f32<T>(y);
     }
+}
+
+// Latent adapter product W = A . B per (target layer, head, K|V), once at translator creation:
+// A [n][in][rank], B [n][rank][out] -> W [n][in][out], fp32 accumulation over rank in ascending
+// order, rounded to T.  One thread per output element.
+template <typename T>
+__global__ void fold_low_rank_kernel(const T* __restrict__ a, const T* __restrict__ b, T* __restrict__ w, int n,
+                                     int in_dim, int rank, int out)
+{
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const long long per = (long long)in_dim * out;
+    if (idx >= per * n) return;
+    const int m = (int)(idx / per);
+    const int rem = (int)(idx - (long long)m * per);
+    const int i = rem / out, o = rem - i * out;
+    const T* am = a + ((size_t)m * in_dim + i) * rank;
+    const T* bm = b + (size_t)m * rank * out + o;
+    float acc = 0.f;
+    for (int c = 0; c < rank; ++c) acc = fmaf(to_f32<T>(am[c]), to_f32<T>(bm[(size_t)c * out]), acc);
+    w[idx] = from_f32<T>(acc);
+}
+
+cudaError_t launch_fold_low_rank(const void* a, const void* b, void* w, int n, int in_dim, int rank, int out,
+                                 int dtype, cudaStream_t stream)
+{
+    const long long total = (long long)n * in_dim * out;
+    const unsigned blocks = (unsigned)((total + 255) / 256);
+    if (dtype == KVX_BF16)
+        fold_low_rank_kernel<__nv_bfloat16><<<blocks, 256, 0, stream>>>(
+            (const __nv_bfloat16*)a, (const __nv_bfloat16*)b, (__nv_bfloat16*)w, n, in_dim, rank, out);
+    else
+        fold_low_rank_kernel<float><<<blocks, 256, 0, stream>>>((const float*)a, (const float*)b, (float*)w, n,
+                                                                 in_dim, rank, out);
+    return cudaGetLastError();
 }
 
 size_t simt_smem_bytes(int in_dim, int dt)

@@ -13,7 +13,10 @@
 //   warp 0      producer: resolves the spans of each 32-token sub-tile and, per
 //               source head, copies the sub-tile's window of consecutive source
 //               rows into a byte ring in shared memory with one cp.async.bulk
-//               (mbarrier transaction counts); loads B images.
+//               (mbarrier transaction counts); loads B: a group's whole image,
+//               kept across its token tiles, when it fits 64 KB, else (wide
+//               inputs: the dense per-layer form, groups of source layers) one
+//               source head's piece of it per head-block through two slots.
 //   warp 1      MMA: allocates TMEM, issues tcgen05.mma (M=128, N=n_tile, K=16
 //               steps over in, one source head's block of A at a time) into a
 //               double-buffered fp32 accumulator.
@@ -49,11 +52,16 @@ constexpr int kXfWarp0 = kEpiWarp0 + kNumEpiWarps;
 constexpr int kNumXfWarps = 8;
 constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
 constexpr int kMaxSeqCache = 512;         // sequences whose metadata is kept in shared memory
+constexpr int kMaxTcIn = 1024;            // widest translator input row (in) this kernel takes
 constexpr int kMaxA = 2;                  // A head-block slots
+constexpr int kMaxB = 2;                  // B slots (1: the group's whole image; 2: head-block pieces)
+constexpr unsigned kBResidentMax = 65536; // largest B image kept resident per group
+constexpr unsigned kBPieceMax = 32768;    // largest streamed B piece (one source head's rows)
 
 // barrier indices
-constexpr int kBarBFull = 0, kBarBEmpty = 1;
-constexpr int kBarAFull = 2;               // +A slot
+constexpr int kBarBFull = 0;               // +B slot
+constexpr int kBarBEmpty = kBarBFull + kMaxB;
+constexpr int kBarAFull = kBarBEmpty + kMaxB;   // +A slot
 constexpr int kBarAEmpty = kBarAFull + kMaxA;
 constexpr int kBarDFull = kBarAEmpty + kMaxA;   // +buf (2)
 constexpr int kBarDEmpty = kBarDFull + 2;       // +buf (2)
@@ -86,7 +94,11 @@ struct TcLaunch {
     unsigned hb_bytes; // one A head-block: 128 rows x d_s bf16
     unsigned cap_rows; // most source rows one window may stage
     int n_slots;       // window slots of slot_bytes each
-    unsigned b_bytes, row_bytes, stage_row_bytes, slot_bytes;
+    int n_b;           // B slots: 1 = the group's image stays resident across its tiles;
+                       // 2 = streamed, one piece (one source head's rows of W) per head-block
+    unsigned b_bytes;  // one group's whole B image (in x n_tile bf16)
+    unsigned b_slot_bytes;   // one B slot: b_bytes (resident) or ds x n_tile bf16 (streamed)
+    unsigned row_bytes, stage_row_bytes, slot_bytes;
     unsigned off_b, off_a, off_stage, off_ring, off_meta, off_bar, off_misc, off_seq, off_turns;
     int seq_cached;   // per-sequence offsets and source lengths copied to shared memory
     unsigned idesc;
@@ -256,8 +268,10 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
 
     if (threadIdx.x == 0) {
         *sAbort = 0;
-        mbar_init(bar(kBarBFull), 1);
-        mbar_init(bar(kBarBEmpty), 1);
+        for (int i = 0; i < kMaxB; ++i) {
+            mbar_init(bar(kBarBFull + i), 1);
+            mbar_init(bar(kBarBEmpty + i), 1);
+        }
         for (int i = 0; i < kMaxA; ++i) {
             mbar_init(bar(kBarAFull + i), kNumXfWarps);
             mbar_init(bar(kBarAEmpty + i), 1);
@@ -309,11 +323,26 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         // copied into the byte ring with one bulk copy.  Tokens whose span falls
         // outside the window (another sequence, a non-monotone span, a window cut at
         // the cap) are read by the prologue from global memory.
-        const uint64_t pol_src = P.e > 1 ? policy_evict_last() : policy_evict_first();
+        // source rows read by more than one target head (repeated KV heads, dense form) stay in L2
+        const uint64_t pol_src = (P.e > 1 || P.dense) ? policy_evict_last() : policy_evict_first();
         const uint64_t pol_keep = policy_evict_last();
         const bool rows_contig = P.ss == P.ds;
+        const bool b_stream = L.n_b > 1;
         int cur_g = -1;
-        uint32_t b_loads = 0, issued = 0;
+        uint32_t b_loads = 0, issued = 0;   // B loads: slot b_loads % n_b, phase (b_loads / n_b) & 1
+        // one B load (the group's image or one head-block piece of it) into the next B slot
+        auto load_b = [&](const uint8_t* from, uint32_t bytes) -> bool {
+            const uint32_t bs = b_loads % (uint32_t)L.n_b;
+            if (!W.wait(bar(kBarBEmpty + bs), ((b_loads / (uint32_t)L.n_b) & 1) ^ 1)) return false;
+            if (lane == 0) mbar_arrive_expect_tx(bar(kBarBFull + bs), bytes);
+            __syncwarp();
+            const uint32_t piece = bytes / 4;
+            if (lane < 4)
+                bulk_g2s(smem_u32(sB) + bs * L.b_slot_bytes + lane * piece, from + (size_t)lane * piece, piece,
+                         bar(kBarBFull + bs), pol_keep);
+            ++b_loads;
+            return true;
+        };
         int wslot = 0;             // window slot of the next window
         uint32_t wphase = 0;       // how often the slots have been cycled, mod 2
         bool ok = true;
@@ -324,15 +353,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         if (wk.more() && lane < kSubPerTile) hd = __ldg(L.plan_hdr + wk.x.tile * kSubPerTile + lane);
         for (; wk.more() && ok; wk.next()) {
             const Unit& x = wk.x;
-            if (x.g != cur_g) {
-                if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) { ok = false; break; }
-                if (lane == 0) mbar_arrive_expect_tx(bar(kBarBFull), L.b_bytes);
-                __syncwarp();
-                const uint8_t* img = (const uint8_t*)P.w + (size_t)x.g * L.b_bytes;
-                const uint32_t piece = L.b_bytes / 4;
-                if (lane < 4)
-                    bulk_g2s(smem_u32(sB) + lane * piece, img + (size_t)lane * piece, piece, bar(kBarBFull), pol_keep);
-                ++b_loads;
+            const uint8_t* img = (const uint8_t*)P.w + (size_t)x.g * L.b_bytes;
+            if (!b_stream && x.g != cur_g) {
+                if (!load_b(img, L.b_bytes)) { ok = false; break; }
                 cur_g = x.g;
             }
             const int4 cur = hd;
@@ -341,9 +364,11 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 nx.next();
                 if (nx.more() && lane < kSubPerTile) hd = __ldg(L.plan_hdr + nx.x.tile * kSubPerTile + lane);
             }
-            const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
-            const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
             for (int q = 0; q < L.r_heads && ok; ++q) {
+                int src_slot, gq;
+                head_block(P, x.j, x.h, q, src_slot, gq);
+                const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[src_slot] : P.src_k[src_slot]);
+                if (b_stream && !load_b(img + (size_t)q * L.b_slot_bytes, L.b_slot_bytes)) { ok = false; break; }
 #pragma unroll
                 for (int sq = 0; sq < kSubPerTile; ++sq) {
                     if (!ok) break;
@@ -361,7 +386,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     const unsigned pos = (unsigned)slot * L.slot_bytes;
                     const uint32_t ring0 = smem_u32(sRing) + pos;
                     const __nv_bfloat16* s0 =
-                        src + (long long)wb * P.sb + (long long)(g0 + q) * P.sh + (long long)wlo * P.ss;
+                        src + (long long)wb * P.sb + (long long)gq * P.sh + (long long)wlo * P.ss;
                     if (lane == 0) {
                         mbar_arrive_expect_tx(bar(kBarSlotFull + slot), need + (unsigned)(kSub * sizeof(int4)));
                         bulk_g2s(smem_u32(sMeta + slot * kSub), L.plan_ent + (size_t)(x.tile * kSubPerTile + sq) * kSub,
@@ -383,19 +408,22 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             const uint32_t ns = (uint32_t)L.n_slots;
             for (uint32_t c = issued > ns ? issued - ns : 0; c < issued; ++c)
                 while (!mbar_try_wait(bar(kBarSlotFull + c % ns), (c / ns) & 1) && globaltimer() - t0 < kWaitNs) {}
-            if (b_loads)
-                while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < kWaitNs) {}
+            const uint32_t nb = (uint32_t)L.n_b;
+            for (uint32_t c = b_loads > nb ? b_loads - nb : 0; c < b_loads; ++c)
+                while (!mbar_try_wait(bar(kBarBFull + c % nb), (c / nb) & 1) && globaltimer() - t0 < kWaitNs) {}
         }
     } else if (warp == kMmaWarp) {
         // ------------------------------------------------------------ MMA issuer
         if (lane == 0) {
             int cur_g = -1;
-            uint32_t b_cnt = 0, tcount = 0, a_cnt = 0;
+            uint32_t b_cnt = 0, tcount = 0, a_cnt = 0;   // B slot b_cnt % n_b, phase (b_cnt / n_b) & 1
+            const bool b_stream = L.n_b > 1;
+            const uint32_t nb = (uint32_t)L.n_b;
             bool ok = true;
             Walker wk;
             for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
                 const Unit& x = wk.x;
-                if (x.g != cur_g) {
+                if (!b_stream && x.g != cur_g) {
                     if (!W.wait(bar(kBarBFull), b_cnt & 1)) break;
                     ++b_cnt;
                     cur_g = x.g;
@@ -403,26 +431,36 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 const uint32_t buf = tcount & 1;
                 if (!W.wait(bar(kBarDEmpty + buf), ((tcount >> 1) & 1) ^ 1)) break;
                 const uint32_t d = tmem_base + buf * (uint32_t)L.n_tile;
-                const uint32_t b0 = smem_u32(sB);
                 for (int q = 0; q < L.r_heads; ++q) {
                     const uint32_t sa = a_cnt % (uint32_t)L.n_a;
                     if (!W.wait(bar(kBarAFull + sa), (a_cnt / (uint32_t)L.n_a) & 1)) { ok = false; break; }
+                    // resident: the image's K-blocks of head-block q; streamed: the piece in its slot
+                    uint32_t b0 = smem_u32(sB), kb0 = (uint32_t)q * (DS / 64);
+                    const uint32_t bs = b_cnt % nb;
+                    if (b_stream) {
+                        if (!W.wait(bar(kBarBFull + bs), (b_cnt / nb) & 1)) { ok = false; break; }
+                        b0 += bs * L.b_slot_bytes;
+                        kb0 = 0;
+                    }
                     tc_fence_after();
                     const uint32_t a0 = smem_u32(sA) + sa * L.hb_bytes;
 #pragma unroll
                     for (int kk = 0; kk < DS / 16; ++kk) {
                         const uint32_t kb = kk >> 2, ko = (kk & 3) * 32;
-                        const uint32_t kbg = (uint32_t)q * (DS / 64) + kb;
                         const uint64_t ad = sw128_desc(a0 + kb * (kTileM * 128) + ko);
-                        const uint64_t bd = sw128_desc(b0 + kbg * (L.n_tile * 128) + ko);
+                        const uint64_t bd = sw128_desc(b0 + (kb0 + kb) * (L.n_tile * 128) + ko);
                         umma_bf16(d, ad, bd, L.idesc, (q > 0 || kk > 0) ? 1u : 0u);
                     }
                     umma_commit(bar(kBarAEmpty + sa));
                     ++a_cnt;
+                    if (b_stream) {
+                        umma_commit(bar(kBarBEmpty + bs));
+                        ++b_cnt;
+                    }
                 }
                 if (!ok) break;
                 umma_commit(bar(kBarDFull + buf));
-                if (wk.last_of_group()) umma_commit(bar(kBarBEmpty));
+                if (!b_stream && wk.last_of_group()) umma_commit(bar(kBarBEmpty));
                 ++tcount;
             }
         }
@@ -521,9 +559,10 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
             const Unit& x = wk.x;
             const bool rot = x.kv == 0 && P.rs.enabled;
-            const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[x.j] : P.src_k[x.j]);
-            const int gbase = P.r > 1 ? x.h * P.r : x.h / P.e;
             for (int q = 0; q < L.r_heads && ok; ++q) {
+                int src_slot, gq;
+                head_block(P, x.j, x.h, q, src_slot, gq);
+                const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[src_slot] : P.src_k[src_slot]);
                 const uint32_t sa = a_cnt % (uint32_t)L.n_a;
                 if (!W.wait(bar(kBarAEmpty + sa), ((a_cnt / (uint32_t)L.n_a) & 1) ^ 1)) { ok = false; break; }
                 uint8_t* sAq = sA + sa * L.hb_bytes;
@@ -552,7 +591,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                                 w1 = *reinterpret_cast<const uint4*>(rp + c_hi);
                             } else {
                                 const uint8_t* rp = reinterpret_cast<const uint8_t*>(
-                                    src + (long long)m.b * P.sb + (long long)(gbase + q) * P.sh +
+                                    src + (long long)m.b * P.sb + (long long)gq * P.sh +
                                     (long long)(m.lo + o) * P.ss);
                                 w0 = __ldg(reinterpret_cast<const uint4*>(rp + c_lo));
                                 w1 = __ldg(reinterpret_cast<const uint4*>(rp + c_hi));
@@ -707,15 +746,24 @@ uint32_t make_idesc(int M, int N)
 
 bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
 {
-    if (in_dim % 64 || in_dim > 256 || in_dim < 64) return false;
+    if (in_dim % 64 || in_dim > kMaxTcIn || in_dim < 64) return false;
     if (dt != 64 && dt != 128 && dt != 256) return false;
     if (ds != 64 && ds != 128 && ds != 256) return false;
     if (in_dim % ds) return false;
     L.in_dim = in_dim;
     L.r_heads = in_dim / ds;
-    L.n_tile = (in_dim * dt * 2 <= 65536) ? dt : dt / 2;
+    // B resident per group while one output split's image fits kBResidentMax; beyond that,
+    // streamed one head-block piece (ds x n_tile) at a time through two slots
+    L.n_tile = dt;
+    while ((unsigned)(in_dim * L.n_tile * 2) > kBResidentMax && L.n_tile > 64 && in_dim <= 256) L.n_tile >>= 1;
+    L.n_b = (unsigned)(in_dim * L.n_tile * 2) <= kBResidentMax ? 1 : kMaxB;
+    if (L.n_b > 1) {
+        L.n_tile = dt;
+        while ((unsigned)(ds * L.n_tile * 2) > kBPieceMax && L.n_tile > 64) L.n_tile >>= 1;
+    }
     L.n_split = dt / L.n_tile;
     L.b_bytes = (unsigned)(in_dim * L.n_tile * 2);
+    L.b_slot_bytes = L.n_b > 1 ? (unsigned)(ds * L.n_tile * 2) : L.b_bytes;
     L.hb_bytes = (unsigned)(kTileM * ds * 2);
     L.row_bytes = (unsigned)(ds * 2);
     L.stage_row_bytes = (unsigned)(L.n_tile * 2 + 16);
@@ -733,7 +781,7 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
             return o;
         };
         L.n_a = n_a;
-        L.off_b = take(L.b_bytes, 1024);
+        L.off_b = take((unsigned)L.n_b * L.b_slot_bytes, 1024);
         L.off_a = take((unsigned)n_a * L.hb_bytes, 1024);
         L.off_stage = take(kTileM * L.stage_row_bytes, 128);
         L.off_meta = take(kNumSlots * kSub * sizeof(int4), 16);

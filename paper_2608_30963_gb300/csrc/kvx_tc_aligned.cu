@@ -63,7 +63,7 @@ constexpr int kNumBars = kBarCsFree + 2;
 
 struct AlignedParams {
     // geometry
-    int Hs, ds, Ht, dt, in_dim, r, e, Lt;
+    int Hs, ds, Ht, dt, in_dim, r, e, dense, Lt;
     int n_tile, n_split, groups, nblk, nslots, nkready, m_tiles_max;
     // source
     int batch, src_max_seq;
@@ -289,7 +289,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 // A K-blocks first: they do not depend on the weights, so at a group switch the
                 // ring refills while the previous group's last tiles drain
                 const CUtensorMap* map = &P.maps[x.j * 2 + x.kv];
-                const int g0 = P.r > 1 ? x.h * P.r : x.h / P.e;
+                const int g0 = P.dense ? 0 : (P.r > 1 ? x.h * P.r : x.h / P.e);
                 for (int kb = 0; kb < P.nblk; ++kb) {
                     const uint32_t slot = sp.idx;
                     if (!W.wait(bar(kBarEmpty + slot), sp.phase ^ 1)) { ok = false; break; }
@@ -619,10 +619,12 @@ EncodeTiled encoder()
 
 }  // namespace
 
-bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch)
+bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch, int kl)
 {
+    // one source layer per target layer (one tensor map each) and a resident B image
     TcConfig c = tc_config(in_dim, dt, ds);
-    return c.ok && Lt <= KVX_MAX_ALIGNED_LAYERS && batch <= KVX_MAX_ALIGNED_BATCH && encoder() != nullptr;
+    return c.ok && in_dim <= 256 && kl == 1 && Lt <= KVX_MAX_ALIGNED_LAYERS && batch <= KVX_MAX_ALIGNED_BATCH &&
+           encoder() != nullptr;
 }
 
 bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int Hs, int batch, long long ss,
@@ -670,6 +672,7 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     static thread_local AlignedParams P;   // large (~27 KB): filled on the host, passed by value
     memset(&P, 0, offsetof(AlignedParams, maps));
     P.Hs = T.Hs; P.ds = T.ds; P.Ht = T.Ht; P.dt = T.dt; P.in_dim = T.in_dim; P.r = T.r; P.e = T.e; P.Lt = T.Lt;
+    P.dense = T.dense;
     P.n_tile = cfg.n_tile;
     P.n_split = cfg.n_split;
     P.groups = T.Lt * T.Ht * 2 * cfg.n_split;

@@ -12,7 +12,7 @@ and a long-context batch sweep with a paged target cache.  The paper's datasets
 shapes stand in for the source caches they would produce.
 
 Seeds: 0 source K/V, 1 W_K, 2 W_V, 3 outlier channels, 4 token alignment,
-5 varlen lengths, 6 page permutation.  Every stream is derived from
+5 varlen lengths, 6 page permutation, 7 and 8 latent adapter factors.  Every stream is derived from
 ``numpy.random.SeedSequence([seed, *indices])`` so one layer can be
 regenerated without drawing the others.
 """
@@ -23,7 +23,8 @@ from typing import Dict, List, Optional, Sequence
 
 import numpy as np
 
-SEED_KV, SEED_WK, SEED_WV, SEED_OUTLIER, SEED_ALIGN, SEED_VARLEN, SEED_PAGES = range(7)
+SEED_KV, SEED_WK, SEED_WV, SEED_OUTLIER, SEED_ALIGN, SEED_VARLEN, SEED_PAGES, SEED_LATENT_A, SEED_LATENT_B = range(9)
+FORM_GROUPED, FORM_DENSE = 0, 1
 
 
 # ----------------------------------------------------------------------------
@@ -80,12 +81,22 @@ class WorkloadSpec:
     outliers: bool                  # 4 channels per (layer, K/V, head) scaled x8 before source RoPE
     paged: bool = False
     page_size: int = 16
+    form: int = FORM_GROUPED        # which source heads feed a target head (grouped / dense)
+    layers_per_target: int = 1      # source layers per target layer (layer_map is then [L_t, k])
+    rank: int = 0                   # > 0: latent adapter factors instead of full matrices
+
+    @property
+    def heads_per_layer(self) -> int:
+        """Source heads of one source layer in a target head's input row."""
+        hs, ht = self.src.num_kv_heads, self.dst.num_kv_heads
+        if self.form == FORM_DENSE:
+            return hs
+        return hs // ht if hs >= ht else 1
 
     @property
     def group_in(self) -> int:
-        """Input width of one translator matrix (GQA regroup)."""
-        hs, ht = self.src.num_kv_heads, self.dst.num_kv_heads
-        return (hs // ht) * self.src.head_dim if hs >= ht else self.src.head_dim
+        """Input width of one translator matrix: k source layers x heads x d_s."""
+        return self.layers_per_target * self.heads_per_layer * self.src.head_dim
 
 
 @dataclasses.dataclass
@@ -141,6 +152,17 @@ def config_specs() -> Dict[str, WorkloadSpec]:
         "llama70b_to_qwen7b_8k": WorkloadSpec("llama70b_to_qwen7b_8k", LLAMA70B, QWEN7B, "bf16",
                                               [8192], True, None, True),
     }
+    # richer translator forms (the granularities the paper's Section 5 lists) on the
+    # 70B -> 7B pair: one map per target layer over all source heads (in = 8 x 128), a group of
+    # two source layers per target layer (in = 2 x 2 x 128), and a rank-64 latent adapter on
+    # the 7B -> 1.5B pair
+    specs["llama70b_to_qwen7b_8k_dense"] = WorkloadSpec(
+        "llama70b_to_qwen7b_8k_dense", LLAMA70B, QWEN7B, "bf16", [8192], True, None, True, form=FORM_DENSE)
+    specs["llama70b_to_qwen7b_8k_layers2"] = WorkloadSpec(
+        "llama70b_to_qwen7b_8k_layers2", LLAMA70B, QWEN7B, "bf16", [8192], True, layer_groups(80, 28, 2), True,
+        layers_per_target=2)
+    specs["qwen7b_to_qwen1p5b_4k_latent64"] = WorkloadSpec(
+        "qwen7b_to_qwen1p5b_4k_latent64", QWEN7B, QWEN1P5B, "bf16", [4096], False, None, True, rank=64)
     for t in (1024, 2048, 4096):
         n = f"qwen1p5b_to_gemma2b_{t // 1024}k"
         specs[n] = WorkloadSpec(n, QWEN1P5B, GEMMA2B, "bf16", [t], True, None, False)
@@ -150,6 +172,14 @@ def config_specs() -> Dict[str, WorkloadSpec]:
             lens = _varlen(L, B)
             specs[n] = WorkloadSpec(n, QWEN7B, QWEN1P5B, "bf16", lens, False, None, True, paged=True)
     return specs
+
+
+def layer_groups(Ls: int, Lt: int, k: int) -> List[List[int]]:
+    """A group of k consecutive source layers per target layer: target layer j takes the
+    first k layers of the j-th of Lt equal contiguous slices of the Ls source layers
+    (floor(j * Ls / Lt) onwards, clipped to the last layer).  A workload choice handed to
+    both sides as an explicit layer map."""
+    return [[min(Ls - 1, (j * Ls) // Lt + i) for i in range(k)] for j in range(Lt)]
 
 
 def _varlen(L: int, B: int) -> List[int]:
@@ -265,6 +295,22 @@ def source_kv(wl: Workload, layer: int, kv: int, pad_value: float = 0.0) -> np.n
     for b in range(wl.batch):
         x[b, :, int(wl.src_len[b]):, :] = pad_value
     return bf16_round(x) if wl.spec.dtype == "bf16" else x
+
+
+def latent_factors(wl: Workload, kv: int):
+    """Latent adapter factors of W_K (kv=0) / W_V (kv=1): A [L_t, H_t, in, rank] ~ N(0, 1/in)
+    and B [L_t, H_t, rank, out] ~ N(0, 1/rank)."""
+    s = wl.spec
+    din, r, dout = s.group_in, s.rank, s.dst.head_dim
+    ra = _rng(SEED_LATENT_A, kv, din, r)
+    rb = _rng(SEED_LATENT_B, kv, r, dout)
+    a = ra.standard_normal((s.dst.num_layers, s.dst.num_kv_heads, din, r), dtype=np.float32)
+    b = rb.standard_normal((s.dst.num_layers, s.dst.num_kv_heads, r, dout), dtype=np.float32)
+    a *= np.float32(1.0 / np.sqrt(din))
+    b *= np.float32(1.0 / np.sqrt(r))
+    if s.dtype == "bf16":
+        a, b = bf16_round(a), bf16_round(b)
+    return a, b
 
 
 def weights(wl: Workload, kv: int) -> np.ndarray:

@@ -38,9 +38,12 @@ class DeviceCase:
         self.dtype = s.dtype
         tdt = torch.bfloat16 if s.dtype == "bf16" else torch.float32
         kdt = kvx.KVX_BF16 if s.dtype == "bf16" else kvx.KVX_FP32
-        self.tr = kvx.Translator(s.src, s.dst, to_dev(c.w_k, s.dtype), to_dev(c.w_v, s.dtype),
-                                 layer_map=list(c.layer_map) if explicit_layer_map else None,
-                                 dtype=kdt, path=path, max_position=max_position)
+        lr = None if c.low_rank is None else tuple(to_dev(a, s.dtype) for a in c.low_rank)
+        self.tr = kvx.Translator(s.src, s.dst, None if lr else to_dev(c.w_k, s.dtype),
+                                 None if lr else to_dev(c.w_v, s.dtype),
+                                 layer_map=c.layer_map.tolist() if explicit_layer_map else None,
+                                 dtype=kdt, path=path, max_position=max_position, form=s.form,
+                                 layers_per_target=s.layers_per_target, low_rank=lr)
         wl = c.wl
         any_l = next(iter(c.src_k))
         self.src_k_dev = {l: to_dev(c.src_k[l], s.dtype) for l in c.src_k}

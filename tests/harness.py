@@ -32,6 +32,7 @@ class Case:
     layer_map: np.ndarray
     src_pos: Optional[np.ndarray] = None   # [B, S_max]
     tgt_pos: Optional[np.ndarray] = None   # [T_total]
+    low_rank: Optional[tuple] = None       # (A_K, B_K, A_V, B_V) latent adapter factors
 
     @property
     def spec(self):
@@ -43,7 +44,7 @@ def make_case(spec: synth.WorkloadSpec, tgt_lens=None, layers: Optional[Sequence
     wl = synth.make_workload(spec, tgt_lens)
     lm = wl.layer_map if wl.layer_map is not None else oracle.layer_map_nearest(spec.src.num_layers,
                                                                                 spec.dst.num_layers)
-    need = sorted(set(int(x) for x in lm)) if layers is None else sorted(set(layers))
+    need = sorted(set(int(x) for x in np.asarray(lm).reshape(-1))) if layers is None else sorted(set(layers))
     ks, vs = {}, {}
     for l in need:
         k = synth.source_kv(wl, l, 0, pad_value)
@@ -57,9 +58,17 @@ def make_case(spec: synth.WorkloadSpec, tgt_lens=None, layers: Optional[Sequence
                 k[b, :, int(wl.src_len[b]):, :] = pad_value
         ks[l] = k
         vs[l] = synth.source_kv(wl, l, 1, pad_value)
-    return Case(wl, ks, vs, synth.weights(wl, 0), synth.weights(wl, 1), np.asarray(lm, np.int32),
+    low_rank = None
+    if spec.rank > 0:
+        a_k, b_k = synth.latent_factors(wl, 0)
+        a_v, b_v = synth.latent_factors(wl, 1)
+        low_rank = (a_k, b_k, a_v, b_v)
+        w_k = w_v = None
+    else:
+        w_k, w_v = synth.weights(wl, 0), synth.weights(wl, 1)
+    return Case(wl, ks, vs, w_k, w_v, np.asarray(lm, np.int32),
                 None if src_pos is None else np.asarray(src_pos, np.int32),
-                None if tgt_pos is None else np.asarray(tgt_pos, np.int32))
+                None if tgt_pos is None else np.asarray(tgt_pos, np.int32), low_rank)
 
 
 def oracle_problem(c: Case) -> oracle.OracleProblem:
@@ -69,7 +78,8 @@ def oracle_problem(c: Case) -> oracle.OracleProblem:
     vs = [c.src_v.get(l, c.src_v[any_l]) for l in range(s.src.num_layers)]
     return oracle.OracleProblem(s.src, s.dst, c.layer_map, c.wl.src_len, c.wl.tgt_seq_off, c.wl.s_max,
                                 c.wl.t_max, ks, vs, c.w_k, c.w_v, c.wl.span_lo, c.wl.span_hi,
-                                None if c.src_pos is None else c.src_pos.reshape(-1), c.tgt_pos)
+                                None if c.src_pos is None else c.src_pos.reshape(-1), c.tgt_pos,
+                                form=s.form, k_layers=s.layers_per_target, low_rank=c.low_rank)
 
 
 def compare(gpu: np.ndarray, ref: np.ndarray, dtype: str) -> dict:

@@ -116,6 +116,38 @@ def test_rope_schedules(name, path):
     _full_compare(c, path)
 
 
+FORMS = {
+    # one map per target layer over all 8 source heads: in = 1024, streamed weight pieces
+    "dense_in1024_spans": ("llama70b_to_qwen7b_8k_dense", 5, 3, [300, 41], {}),
+    # dense over 2 source heads (in = 256, resident weights), expansion-shaped geometry, spans
+    "dense_in256_spans": ("qwen1p5b_to_gemma2b_1k", 3, 2, [300], dict(form=synth.FORM_DENSE)),
+    # dense in = 256 with identity alignment (tensor-TMA kernel)
+    "dense_in256_identity": ("qwen7b_to_qwen1p5b_4k", 2, 2, [300, 5],
+                             dict(form=synth.FORM_DENSE, src=synth.QWEN1P5B)),
+    # groups of two source layers: in = 512, streamed weight pieces
+    "layers2_in512_spans": ("llama70b_to_qwen7b_8k_layers2", 5, 3, [300, 41],
+                            dict(layer_map=[[0, 1], [2, 3], [4, 4]])),
+    # latent adapters, identity alignment and spans
+    "latent64_identity": ("qwen7b_to_qwen1p5b_4k_latent64", 2, 2, [300, 5], {}),
+    "latent16_spans": ("llama70b_to_qwen7b_8k", 5, 3, [300], dict(rank=16)),
+}
+
+
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+@pytest.mark.parametrize("name", list(FORMS))
+def test_translator_forms(name, path):
+    base, Ls, Lt, lens, kw = FORMS[name]
+    spec = _shrink(SPECS[base], Ls, Lt)
+    kw = dict(kw)
+    if "src" in kw:
+        kw["src"] = dataclasses.replace(kw["src"], num_layers=Ls)
+    spec = dataclasses.replace(spec, **kw)
+    c = make_case(spec, lens, pad_value=float("nan"))
+    g, _, _ = _full_compare(c, path)
+    if path == kvx.KVX_PATH_AUTO:
+        assert g.tr.info().path == kvx.KVX_PATH_TCGEN05
+
+
 def test_tiny_token_counts_and_empty_sequences():
     spec = _shrink(SPECS["qwen1p5b_to_gemma2b_1k"], 2, 2)
     c = make_case(spec, [1, 0, 2, 0, 129])
@@ -147,7 +179,22 @@ def test_paged_equals_contiguous_and_batch_invariance(path):
 
 # ------------------------------------------------------------------ full-size, sampled rows
 FULL = ["qwen7b_to_qwen1p5b_4k", "qwen1p5b_to_gemma2b_1k", "qwen1p5b_to_gemma2b_2k", "qwen1p5b_to_gemma2b_4k",
-        "llama70b_to_qwen7b_8k", "longctx_8k_b4", "tiny_fp32"]
+        "llama70b_to_qwen7b_8k", "longctx_8k_b4", "tiny_fp32", "llama70b_to_qwen7b_8k_dense",
+        "qwen7b_to_qwen1p5b_4k_latent64"]
+
+
+def test_layer_groups_8k_sampled():
+    """Groups of two source layers at the full 8K context, on 6 target layers (the full
+    28-layer map would hold 56 source layers in host memory)."""
+    spec = dataclasses.replace(SPECS["llama70b_to_qwen7b_8k_layers2"],
+                               dst=dataclasses.replace(SPECS["llama70b_to_qwen7b_8k_layers2"].dst, num_layers=6),
+                               layer_map=synth.layer_groups(80, 6, 2))
+    c = make_case(spec)
+    g = _run(c, kvx.KVX_PATH_AUTO)
+    p = oracle_problem(c)
+    rows = sample_rows(c, 300)
+    compare(np.stack([g.row(*r) for r in rows]), np.stack([p.row(*r) for r in rows]), "bf16")
+    assert g.status() == 0
 
 
 @pytest.mark.parametrize("name", FULL)

@@ -53,7 +53,7 @@ def _desc(src, dst, dtype=kvx.KVX_BF16, path=kvx.KVX_PATH_AUTO, layer_map=None):
 @pytest.mark.parametrize("src,dst,code", [
     (synth.ModelGeom(2, 3, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),   # 3 vs 2 heads
     (synth.ModelGeom(2, 2, 96, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),    # head_dim 96
-    (synth.ModelGeom(2, 16, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),  # in = 1024
+    (synth.ModelGeom(2, 32, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),  # in = 2048
     (synth.ModelGeom(0, 2, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_INVALID_ARG),
     (synth.ModelGeom(2, 2, 128, 1e6), synth.ModelGeom(200, 2, 128, 1e6), kvx.KVX_ERR_UNSUPPORTED),
     (synth.ModelGeom(2, 2, 128, 1e6, rope_type=3), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_INVALID_ARG),
@@ -71,6 +71,36 @@ def test_create_rejects_bad_geometry_without_touching_cuda(lib, src, dst, code):
     assert st == code
     assert h.value is None
     assert kvx.kvx_last_error()
+
+
+@pytest.mark.parametrize("form,k,with_map,code", [
+    (2, 1, False, kvx.KVX_ERR_INVALID_ARG),       # unknown form
+    (0, 5, True, kvx.KVX_ERR_INVALID_ARG),        # more than 4 source layers per target layer
+    (0, 2, False, kvx.KVX_ERR_INVALID_ARG),       # a group of layers needs an explicit map
+    (1, 1, False, kvx.KVX_ERR_UNSUPPORTED),       # dense over 16 heads of 128: in = 2048
+])
+def test_create_rejects_bad_translator_forms(lib, form, k, with_map, code):
+    src, dst = synth.ModelGeom(8, 16, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6)
+    lm = (ctypes.c_int32 * 10)(*range(10))
+    d = _desc(src, dst, layer_map=ctypes.cast(lm, kvx.I32P) if with_map else None)
+    d.form, d.layers_per_target = form, k
+    h = ctypes.c_void_p()
+    w = (ctypes.c_uint16 * 4)()
+    st = lib.kvx_translator_create(ctypes.byref(d), ctypes.cast(w, ctypes.c_void_p),
+                                   ctypes.cast(w, ctypes.c_void_p), 0, ctypes.byref(h))
+    assert st == code, kvx.kvx_last_error()
+    assert h.value is None
+
+
+def test_low_rank_create_rejects_bad_rank(lib):
+    d = _desc(synth.ModelGeom(2, 4, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6))
+    h = ctypes.c_void_p()
+    w = (ctypes.c_uint16 * 4)()
+    p = ctypes.cast(w, ctypes.c_void_p)
+    for rank in (0, 1025):
+        assert lib.kvx_translator_create_low_rank(ctypes.byref(d), rank, p, p, p, p, 0, ctypes.byref(h)) == \
+            kvx.KVX_ERR_INVALID_ARG
+    assert "rank" in kvx.kvx_last_error()
 
 
 def test_create_rejects_out_of_range_layer_map(lib):

@@ -385,3 +385,111 @@ def test_layer_map_is_followed():
     moved = _problem(sg, dg, [0, 1], [5], [5], perm[0], perm[1], w, w).translate()
     for i in range(2):
         np.testing.assert_array_equal(base[i], moved[i])
+
+
+# ----------------------------------------------- richer translator forms (Section 5)
+def _problem_f(sg, dg, layer_map, lens, src_k, src_v, wk, wv, lo=None, hi=None, **kw):
+    so = np.concatenate([[0], np.cumsum(lens)]).astype(np.int32)
+    S = src_k[0].shape[2]
+    lens_src = [S] * len(lens) if lo is not None else lens
+    return oracle.OracleProblem(sg, dg, layer_map, np.array(lens_src, np.int32), so, S, max(lens), src_k, src_v,
+                                wk, wv, lo, hi, **kw)
+
+
+def test_dense_form_without_rope_is_a_matmul_of_all_source_heads():
+    """Per-layer form: every target head reads concat(all source heads) @ W[j, h]."""
+    rng = np.random.default_rng(31)
+    sg, dg = _geom(2, 4, 64, 0.0), _geom(2, 2, 128, 0.0)
+    S = 7
+    ks, vs = _rand_src(rng, sg, 1, S)
+    wk = rng.standard_normal((2, 2, 256, 128)).astype(np.float32)
+    wv = rng.standard_normal((2, 2, 256, 128)).astype(np.float32)
+    ok, ov = _problem_f(sg, dg, [1, 0], [S], ks, vs, wk, wv, form=1).translate()
+    for j, l in ((0, 1), (1, 0)):
+        xk = np.concatenate([ks[l][0, g] for g in range(4)], axis=1).astype(np.float64)
+        xv = np.concatenate([vs[l][0, g] for g in range(4)], axis=1).astype(np.float64)
+        for h in range(2):
+            np.testing.assert_allclose(ok[j, h], xk @ wk[j, h].astype(np.float64), rtol=1e-12, atol=1e-12)
+            np.testing.assert_allclose(ov[j, h], xv @ wv[j, h].astype(np.float64), rtol=1e-12, atol=1e-12)
+
+
+def test_dense_form_restricted_to_the_group_equals_the_grouped_form():
+    """A dense W that is zero outside target head h's GQA rows gives the grouped result
+    (with RoPE on both sides and cross-tokenizer spans)."""
+    rng = np.random.default_rng(32)
+    sg, dg = _geom(1, 4, 64, 1e6), _geom(1, 2, 64, 1e4)
+    T = 25
+    lo, hi, S, _, _ = synth.draw_spans(T, 3)
+    ks, vs = _rand_src(rng, sg, 1, S)
+    ks = [oracle.rope_cache(k, sg.rope_base) for k in ks]
+    wg = rng.standard_normal((1, 2, 128, 64)).astype(np.float32)
+    wd = np.zeros((1, 2, 256, 64), np.float32)
+    for h in range(2):
+        wd[0, h, 128 * h:128 * h + 128] = wg[0, h]
+    grouped = _problem_f(sg, dg, [0], [T], ks, vs, wg, wg, lo, hi).translate()
+    dense = _problem_f(sg, dg, [0], [T], ks, vs, wd, wd, lo, hi, form=1).translate()
+    for i in range(2):
+        np.testing.assert_allclose(dense[i], grouped[i], rtol=1e-12, atol=1e-12)
+
+
+def test_layer_groups_concatenate_source_layers():
+    """k = 2 source layers per target layer: without RoPE the input is the concatenation of
+    both layers' grouped heads; with RoPE and spans, W = [W1; 0] and [0; W2] select one layer
+    each and their sum is linear."""
+    rng = np.random.default_rng(33)
+    sg, dg = _geom(3, 2, 64, 0.0), _geom(1, 1, 64, 0.0)
+    S = 6
+    ks, vs = _rand_src(rng, sg, 1, S)
+    w = rng.standard_normal((1, 1, 256, 64)).astype(np.float32)
+    ok, ov = _problem_f(sg, dg, [[2, 0]], [S], ks, vs, w, w, k_layers=2).translate()
+    x = np.concatenate([ks[2][0, 0], ks[2][0, 1], ks[0][0, 0], ks[0][0, 1]], axis=1).astype(np.float64)
+    np.testing.assert_allclose(ok[0, 0], x @ w[0, 0].astype(np.float64), rtol=1e-12, atol=1e-12)
+    # with RoPE and spans
+    sg, dg = _geom(3, 2, 64, 1e4), _geom(1, 1, 64, 1e6)
+    T = 21
+    lo, hi, S, _, _ = synth.draw_spans(T, 4)
+    ks, vs = _rand_src(rng, sg, 1, S)
+    ks = [oracle.rope_cache(k, sg.rope_base) for k in ks]
+    w1 = rng.standard_normal((1, 1, 128, 64)).astype(np.float32)
+    w2 = rng.standard_normal((1, 1, 128, 64)).astype(np.float32)
+    z = np.zeros_like(w1)
+    both = _problem_f(sg, dg, [[2, 1]], [T], ks, vs, np.concatenate([w1, w2], 2), np.concatenate([w1, w2], 2),
+                      lo, hi, k_layers=2).translate()
+    first = _problem_f(sg, dg, [[2, 1]], [T], ks, vs, np.concatenate([w1, z], 2), np.concatenate([w1, z], 2),
+                       lo, hi, k_layers=2).translate()
+    only2 = _problem_f(sg, dg, [2], [T], ks, vs, w1, w1, lo, hi).translate()
+    only1 = _problem_f(sg, dg, [1], [T], ks, vs, w2, w2, lo, hi).translate()
+    for i in range(2):
+        np.testing.assert_allclose(first[i], only2[i], rtol=1e-12, atol=1e-12)
+        np.testing.assert_allclose(both[i], only2[i] + only1[i], rtol=1e-9, atol=1e-9)
+
+
+def test_latent_adapter_equals_the_product_matrix():
+    """(x A) B = x (A B): the chained maps match a full-rank translator with W = A B, and a
+    rank-one adapter gives (x . a) b."""
+    rng = np.random.default_rng(34)
+    sg, dg = _geom(2, 4, 64, 1e6), _geom(2, 2, 128, 1e4)
+    T = 17
+    lo, hi, S, _, _ = synth.draw_spans(T, 5)
+    ks, vs = _rand_src(rng, sg, 1, S)
+    ks = [oracle.rope_cache(k, sg.rope_base) for k in ks]
+    for r in (1, 16):
+        A = [rng.standard_normal((2, 2, 128, r)).astype(np.float32) for _ in range(2)]
+        B = [rng.standard_normal((2, 2, r, 128)).astype(np.float32) for _ in range(2)]
+        lr = _problem_f(sg, dg, [1, 0], [T], ks, vs, None, None, lo, hi,
+                        low_rank=(A[0], B[0], A[1], B[1])).translate()
+        # the product in float64 is not float32-exact: compare with a float64-weight reference
+        Wk = np.einsum("jhir,jhro->jhio", A[0].astype(np.float64), B[0].astype(np.float64))
+        Wv = np.einsum("jhir,jhro->jhio", A[1].astype(np.float64), B[1].astype(np.float64))
+        full = _problem_f(sg, dg, [1, 0], [T], ks, vs, Wk.astype(np.float32), Wv.astype(np.float32),
+                          lo, hi).translate()
+        for i in range(2):
+            scale = np.abs(full[i]).max()
+            np.testing.assert_allclose(lr[i], full[i], rtol=0, atol=1e-6 * scale)
+    # rank one, V path without RoPE: y = (xbar . a) b
+    a, b = A[1][..., :1], B[1][:, :, :1, :]
+    _, ov = _problem_f(sg, dg, [1, 0], [T], ks, vs, None, None, lo, hi, low_rank=(a, b, a, b)).translate()
+    t = 3
+    xbar = np.concatenate([vs[1][0, g, lo[t]:hi[t]].astype(np.float64).mean(0) for g in (0, 1)])
+    np.testing.assert_allclose(ov[0, 0, t], (xbar @ a[0, 0, :, 0].astype(np.float64)) * b[0, 0, 0].astype(np.float64),
+                               rtol=1e-12, atol=1e-12)
