@@ -213,6 +213,8 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=12.0, help="seconds of oracle work per core")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=10)
+    ap.add_argument("--mode", default="translate", choices=["translate", "fit"],
+                    help="translate: the hot path (default); fit: the closed-form translator fit's accumulation")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
 
@@ -223,6 +225,8 @@ def main():
 
     if args.impl == "reference":
         return reference_arm(args, spec, rank, world)
+    if args.mode == "fit":
+        return fit_bench(args, spec)
 
     # spawn the oracle pool before any CUDA call
     pool = None
@@ -441,6 +445,78 @@ def main():
     tr.close()
     if dist:
         dist.destroy_process_group()
+
+
+def fit_bench(args, spec):
+    """Closed-form fit: calibration tokens/s of kvx_fit_accumulate (input rows, target rows, Gram
+    sums) over the workload, plus one solve.  Inputs resident on the device."""
+    import torch
+    import paper_2608_30963_gb300 as kvx
+    torch.cuda.set_device(0)
+    wl = synth.make_workload(spec)
+    lm = wl.layer_map.tolist() if wl.layer_map is not None else nearest_map(spec.src.num_layers, spec.dst.num_layers)
+    dev = torch.device("cuda", 0)
+    g = torch.Generator(device=dev).manual_seed(0)
+    s, d = spec.src, spec.dst
+    mapped = sorted(set(int(x) for x in np.asarray(lm).reshape(-1)))
+    shape = (wl.batch, s.num_kv_heads, wl.s_max, s.head_dim)
+    ks = {l: torch.randn(shape, generator=g, device=dev).to(torch.bfloat16) for l in mapped}
+    vs = {l: torch.randn(shape, generator=g, device=dev).to(torch.bfloat16) for l in mapped}
+    src_k = [ks.get(l, ks[mapped[0]]) for l in range(s.num_layers)]
+    src_v = [vs.get(l, vs[mapped[0]]) for l in range(s.num_layers)]
+    tshape = (wl.batch, d.num_kv_heads, wl.t_max, d.head_dim)
+    tk = [torch.randn(tshape, generator=g, device=dev).to(torch.bfloat16) for _ in range(d.num_layers)]
+    tv = [torch.randn(tshape, generator=g, device=dev).to(torch.bfloat16) for _ in range(d.num_layers)]
+    i32 = lambda a: None if a is None else torch.from_numpy(np.ascontiguousarray(a, np.int32)).to(dev)
+    src_len, seq_off = i32(wl.src_len), i32(wl.tgt_seq_off)
+    span_lo, span_hi = i32(wl.span_lo), i32(wl.span_hi)
+    f = kvx.Fitter(s, d, 1e-3, layer_map=lm, form=spec.form, layers_per_target=spec.layers_per_target)
+    T = wl.total_tgt
+
+    def step():
+        f.accumulate(src_k, src_v, src_len, seq_off, T, tk, tv, span_lo=span_lo, span_hi=span_hi)
+
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for _ in range(args.steps):
+        step()
+    b.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / args.steps
+    wk = torch.empty((d.num_layers, d.num_kv_heads, spec.group_in, d.head_dim), dtype=torch.bfloat16, device=dev)
+    wv = torch.empty_like(wk)
+    t0 = time.perf_counter()
+    bits = f.solve(wk, wv)
+    solve_ms = (time.perf_counter() - t0) * 1e3
+    elt = 2
+    groups = d.num_layers * d.num_kv_heads * 2
+    src_bytes = len(mapped) * s.num_kv_heads * int(wl.src_len.sum()) * s.head_dim * 2 * elt
+    tgt_bytes = d.num_layers * d.num_kv_heads * T * d.head_dim * 2 * elt
+    sums = groups * spec.group_in * (spec.group_in + d.head_dim) * 4 * 2
+    flops = groups * T * 2.0 * spec.group_in * (spec.group_in + d.head_dim)
+    peaks = {}
+    try:
+        peaks = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+    except Exception:
+        pass
+    hbm, tc = peaks.get("hbm_gbs", 6800.0), peaks.get("bf16_tflops", 1900.0)
+    byts = src_bytes + tgt_bytes + sums
+    t_roof = max(byts / (hbm * 1e9), flops / (tc * 1e12))
+    line = {"metric": "fit calibration tokens/s (kvx_fit_accumulate)", "value": T / (ms / 1e3), "unit": "tokens/s",
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "dtype": spec.dtype, "data": "synthetic", "mode": "fit",
+            "config": {"workload": args.workload, "target_tokens": T, "groups": groups, "in": spec.group_in,
+                       "lambda": 1e-3},
+            "roofline": {"bound": "hbm" if byts / (hbm * 1e9) >= flops / (tc * 1e12) else "tensor",
+                         "algorithmic_bytes": byts, "flops": flops, "roofline_ms": t_roof * 1e3,
+                         "frac": t_roof * 1e3 / ms, "achieved_tflops": flops / (ms / 1e3) / 1e12,
+                         "peaks": {"hbm_gbs": hbm, "bf16_tflops": tc}},
+            "solve_ms": solve_ms, "solve_status": bits}
+    print(json.dumps(line), flush=True)
+    f.close()
 
 
 def kernel_rev() -> str:

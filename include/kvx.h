@@ -266,6 +266,59 @@ KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_translator_info* i
  * translation launch).  0 before the first call and after a call with no tokens. */
 KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
 
+/* ------------------------------------------------------------------------------------------
+ * Closed-form fit of a linear translator (Section 5).  The paper gives the learning objective
+ * L_KV = D(T_theta(KV_A(C)), KV_B(C)): the distance between the translated cache and the cache
+ * the target's own prefill builds for the same context.  With D the squared Euclidean distance
+ * summed over target tokens plus a ridge term lambda |W|^2, and the linear T_theta of
+ * kvx_translate, every (target layer j, target head h, K|V) is an independent least-squares
+ * problem with the closed-form solution
+ *     W[j,h] = (X^T X + lambda I)^{-1} X^T Y,
+ * where row t of X is the translator's input row for target token t (the span mean of the
+ * un-rotated source rows, exactly as kvx_translate forms it, rounded to the cache dtype) and
+ * row t of Y is the target model's own cache row of token t with the target RoPE undone (K;
+ * the rotation is orthogonal, so the distance is unchanged) or as stored (V).
+ * The fitter accumulates X^T X and X^T Y over any number of calibration calls (fp32, on the
+ * tensor cores through cuBLAS batched GEMMs over the groups), then solves all systems at once
+ * (Cholesky factorisation in double on the device).  Forms as for kvx_translator_create;
+ * latent adapters are not fitted (fit W, then factor it if wanted). */
+typedef struct kvx_fitter kvx_fitter;
+
+/* desc: the translator to fit (its dtype is the cache dtype; desc->path is ignored).
+ * lambda: ridge weight, >= 0 (0 needs at least `in` well-spread tokens per system).
+ * chunk_tokens: target tokens one accumulation pass handles (calls longer than this run in
+ *   several passes); 0 = 4096.  The fitter holds (L_t * H_t * 2) * chunk_tokens * (in + out)
+ *   cache-dtype elements of row workspace plus the fp32 sums.
+ * Requires in <= 512.  Synchronous; on success *out owns device memory until kvx_fit_destroy. */
+KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, double lambda, int32_t chunk_tokens,
+                                  kvx_fitter** out);
+
+/* Add one calibration batch: source caches, the token alignment, and the target model's own
+ * caches for the same context (read-only here; same layouts as for kvx_translate, contiguous
+ * or paged).  Target rows that fall outside the target cache (a bad page, t >= max_seq) are
+ * left out of the sums and flagged in the fitter's status word.  Asynchronous on stream;
+ * allocates nothing. */
+KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
+                                      const kvx_dst_kv* target_cache, void* stream);
+
+/* Solve every system from the sums so far and write W_K and W_V as DEVICE arrays
+ * [dst.num_layers][dst.num_kv_heads][in][out] of the desc dtype (the layout
+ * kvx_translator_create takes).  Synchronises stream.  status_bits (host, may be NULL) receives
+ * the fitter's status word: KVX_DEV_* bits from the accumulation passes (rows left out) and
+ * 0x20 when a system was not positive definite (lambda = 0 with too few tokens; its W is zero),
+ * in which case the call returns KVX_ERR_DEVICE_STATUS.  Calls on one fitter must be ordered
+ * (one stream, or synchronised by the caller). */
+KVX_API kvx_status kvx_fit_solve(kvx_fitter* f, void* w_k, void* w_v, uint32_t* status_bits, void* stream);
+
+/* Clear the accumulated sums (start a new fit with the same fitter). */
+KVX_API kvx_status kvx_fit_reset(kvx_fitter* f, void* stream);
+
+/* Tokens accumulated so far (sum of total_tokens over kvx_fit_accumulate calls). */
+KVX_API int64_t kvx_fit_tokens(const kvx_fitter* f);
+
+/* Free the fitter.  Synchronises the device first.  NULL is accepted. */
+KVX_API kvx_status kvx_fit_destroy(kvx_fitter* f);
+
 /* Size of the device scratch array kvx_translate_static works in (8 MiB). */
 #define KVX_STATIC_SCRATCH_BYTES (8u << 20)
 

@@ -84,6 +84,11 @@ def lib():
         _lib.kvxo_translate_row.argtypes = [ctypes.POINTER(Problem), ctypes.c_int, ctypes.c_int,
                                             ctypes.c_int, ctypes.c_int, F64P]
         _lib.kvxo_translate.argtypes = [ctypes.POINTER(Problem), F64P, F64P]
+        _lib.kvxo_input_row.argtypes = [ctypes.POINTER(Problem), ctypes.c_int, ctypes.c_int, ctypes.c_int,
+                                        ctypes.c_int, F64P]
+        _lib.kvxo_group_in.argtypes = [ctypes.POINTER(Problem)]
+        _lib.kvxo_fit.argtypes = [ctypes.POINTER(Problem), ctypes.POINTER(F32P), ctypes.POINTER(F32P),
+                                  ctypes.c_double, F64P, F64P]
     return _lib
 
 
@@ -185,6 +190,29 @@ class OracleProblem:
         if lib().kvxo_translate(ctypes.byref(self.p), _p(ok, F64P), _p(ov, F64P)):
             raise ValueError("oracle: unsupported geometry")
         return ok, ov
+
+    def input_row(self, j: int, h: int, kv: int, tp: int) -> np.ndarray:
+        """The translator's input row (span mean of un-rotated source rows) of one target token."""
+        out = np.zeros(lib().kvxo_group_in(ctypes.byref(self.p)), np.float64)
+        if lib().kvxo_input_row(ctypes.byref(self.p), j, h, kv, tp, _p(out, F64P)):
+            raise ValueError("oracle: unsupported geometry")
+        return out
+
+    def fit(self, tgt_k: Sequence[np.ndarray], tgt_v: Sequence[np.ndarray], lam: float):
+        """Closed-form ridge fit of W_K, W_V against the target model's own caches
+        (per target layer [B, Ht, t_max, dt] float32).  Returns two [Lt, Ht, in, dt] float64."""
+        tk = [np.ascontiguousarray(a, np.float32) for a in tgt_k]
+        tv = [np.ascontiguousarray(a, np.float32) for a in tgt_v]
+        kp = (F32P * len(tk))(*[_p(a, F32P) for a in tk])
+        vp = (F32P * len(tv))(*[_p(a, F32P) for a in tv])
+        din = lib().kvxo_group_in(ctypes.byref(self.p))
+        wk = np.zeros((self.Lt, self.Ht, din, self.dt), np.float64)
+        wv = np.zeros_like(wk)
+        rc = lib().kvxo_fit(ctypes.byref(self.p), ctypes.cast(kp, ctypes.POINTER(F32P)),
+                            ctypes.cast(vp, ctypes.POINTER(F32P)), float(lam), _p(wk, F64P), _p(wv, F64P))
+        if rc:
+            raise ValueError(f"oracle fit failed ({rc})")
+        return wk, wv
 
     def row(self, j: int, h: int, kv: int, tp: int) -> np.ndarray:
         out = np.zeros(self.dt, np.float64)

@@ -199,10 +199,12 @@ static int group_in(const kvxo_problem* p)
     return layers_per_target(p) * heads_per_layer(p) * p->ds;
 }
 
-/* One output row: target layer j, target head h, kv (0 = K, 1 = V), packed
- * target token index tp.  Writes d_t doubles.  Returns nonzero on a
- * geometry it cannot place. */
-KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int tp, double* out)
+KVXO_API int kvxo_group_in(const kvxo_problem* p) { return group_in(p); }
+
+/* Steps 1-4 for one target token: the translator's input row xbar (length
+ * group_in) of target layer j, head h, kv (0 = K, 1 = V), packed target token
+ * tp.  Returns nonzero on a geometry it cannot place. */
+KVXO_API int kvxo_input_row(const kvxo_problem* p, int j, int h, int kv, int tp, double* sum)
 {
     if (p->Hs % p->Ht != 0 && p->Ht % p->Hs != 0) return 1;
     if (p->form != 0 && p->form != 1) return 1;
@@ -216,7 +218,7 @@ KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int
     int nh = heads_per_layer(p);
     int g0 = p->form == 1 ? 0 : (p->Hs >= p->Ht ? h * nh : h / (p->Ht / p->Hs));
 
-    double* sum = (double*)calloc((size_t)in, sizeof(double));
+    for (int i = 0; i < in; ++i) sum[i] = 0.0;
     double* u = (double*)malloc(sizeof(double) * (size_t)p->ds);
     for (int s = lo; s < hi; ++s) {                            /* step 3 */
         double ps = p->src_pos ? (double)p->src_pos[(size_t)b * p->s_max + s] : (double)s;
@@ -234,6 +236,21 @@ KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int
     }
     double n = (double)(hi - lo);                              /* step 4 */
     for (int i = 0; i < in; ++i) sum[i] /= n;
+    free(u);
+    return 0;
+}
+
+/* One output row: target layer j, target head h, kv (0 = K, 1 = V), packed
+ * target token index tp.  Writes d_t doubles.  Returns nonzero on a
+ * geometry it cannot place. */
+KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int tp, double* out)
+{
+    int in = group_in(p);
+    double* sum = (double*)malloc(sizeof(double) * (size_t)in);
+    if (kvxo_input_row(p, j, h, kv, tp, sum)) { free(sum); return 1; }
+    int b = 0;
+    while (b < p->batch - 1 && p->tgt_seq_off[b + 1] <= tp) ++b;
+    int t = tp - p->tgt_seq_off[b];
 
     if (p->rank > 0) {                                         /* step 5, latent adapter */
         size_t jh = (size_t)j * p->Ht + h;
@@ -264,7 +281,6 @@ KVXO_API int kvxo_translate_row(const kvxo_problem* p, int j, int h, int kv, int
         kvxo_rope_sched_apply(out, p->dt, &p->rope_t, pt, +1);
     }
     free(sum);
-    free(u);
     return 0;
 }
 
@@ -300,4 +316,90 @@ KVXO_API void kvxo_rope_cache(float* x, int B, int H, int S, int d, const kvxo_r
                 for (int e = 0; e < d; ++e) xr[e] = (float)row[e];
             }
     free(row);
+}
+
+/* ---------------------------------------------------------------------- */
+/* Closed-form fit of the linear translator.  Section 5 gives the objective
+ * L_KV = D(T_theta(KV_A(C)), KV_B(C)), the distance between the translated
+ * cache and the cache the target's own prefill builds.  With D the squared
+ * Euclidean distance summed over target tokens, plus a ridge term
+ * lambda |W|^2, and T_theta linear in W, each (target layer j, head h, K|V)
+ * is an independent least-squares problem:
+ *
+ *   W = argmin_W  sum_t |x_t W - y_t|^2 + lambda |W|^2,
+ *   i.e. the normal equations (X^T X + lambda I) W = X^T Y,
+ *
+ * where x_t is the input row of target token t (steps 1-4 above) and y_t the
+ * target model's own cache row with the target RoPE undone (K; the rotation
+ * is orthogonal, so the distance is the same before and after it) or as
+ * stored (V).  Solved with a Cholesky factorisation X^T X + lambda I = L L^T
+ * and two triangular solves per output column, all in double.
+ *
+ * tgt_k, tgt_v: [Lt] arrays of the target caches, each [B][Ht][t_max][dt].
+ * w_k_out, w_v_out: [Lt][Ht][in][dt].  Returns nonzero if a system is not
+ * positive definite or the geometry cannot be placed. */
+KVXO_API int kvxo_fit(const kvxo_problem* p, const float* const* tgt_k, const float* const* tgt_v, double lambda,
+                      double* w_k_out, double* w_v_out)
+{
+    int in = group_in(p), dt = p->dt, T = p->tgt_seq_off[p->batch];
+    double* G = (double*)malloc(sizeof(double) * (size_t)in * in);
+    double* Cm = (double*)malloc(sizeof(double) * (size_t)in * dt);
+    double* x = (double*)malloc(sizeof(double) * (size_t)in);
+    double* y = (double*)malloc(sizeof(double) * (size_t)dt);
+    int rc = 0;
+    for (int j = 0; j < p->Lt && !rc; ++j)
+        for (int h = 0; h < p->Ht && !rc; ++h)
+            for (int kv = 0; kv < 2 && !rc; ++kv) {
+                memset(G, 0, sizeof(double) * (size_t)in * in);
+                memset(Cm, 0, sizeof(double) * (size_t)in * dt);
+                for (int tp = 0; tp < T; ++tp) {
+                    if (kvxo_input_row(p, j, h, kv, tp, x)) { rc = 1; break; }
+                    int b = 0;
+                    while (b < p->batch - 1 && p->tgt_seq_off[b + 1] <= tp) ++b;
+                    int t = tp - p->tgt_seq_off[b];
+                    const float* row = (kv == 0 ? tgt_k[j] : tgt_v[j]) +
+                                       (((size_t)b * p->Ht + h) * p->t_max + t) * dt;
+                    for (int o = 0; o < dt; ++o) y[o] = (double)row[o];
+                    if (kv == 0) {
+                        double pt = p->tgt_pos ? (double)p->tgt_pos[tp] : (double)t;
+                        kvxo_rope_sched_apply(y, dt, &p->rope_t, pt, -1);
+                    }
+                    for (int a = 0; a < in; ++a) {
+                        for (int c = 0; c < in; ++c) G[(size_t)a * in + c] += x[a] * x[c];
+                        for (int o = 0; o < dt; ++o) Cm[(size_t)a * dt + o] += x[a] * y[o];
+                    }
+                }
+                if (rc) break;
+                for (int a = 0; a < in; ++a) G[(size_t)a * in + a] += lambda;
+                /* Cholesky: G = L L^T, L stored in the lower triangle of G */
+                for (int c = 0; c < in && !rc; ++c) {
+                    double d = G[(size_t)c * in + c];
+                    for (int k = 0; k < c; ++k) d -= G[(size_t)c * in + k] * G[(size_t)c * in + k];
+                    if (!(d > 0.0)) { rc = 2; break; }
+                    d = sqrt(d);
+                    G[(size_t)c * in + c] = d;
+                    for (int r = c + 1; r < in; ++r) {
+                        double v = G[(size_t)r * in + c];
+                        for (int k = 0; k < c; ++k) v -= G[(size_t)r * in + k] * G[(size_t)c * in + k];
+                        G[(size_t)r * in + c] = v / d;
+                    }
+                }
+                if (rc) break;
+                double* W = (kv == 0 ? w_k_out : w_v_out) + ((size_t)j * p->Ht + h) * (size_t)in * dt;
+                for (int o = 0; o < dt; ++o) {
+                    /* L z = c (forward), then L^T w = z (backward) */
+                    for (int r = 0; r < in; ++r) {
+                        double v = Cm[(size_t)r * dt + o];
+                        for (int k = 0; k < r; ++k) v -= G[(size_t)r * in + k] * x[k];
+                        x[r] = v / G[(size_t)r * in + r];
+                    }
+                    for (int r = in - 1; r >= 0; --r) {
+                        double v = x[r];
+                        for (int k = r + 1; k < in; ++k) v -= G[(size_t)k * in + r] * W[(size_t)k * dt + o];
+                        W[(size_t)r * dt + o] = v / G[(size_t)r * in + r];
+                    }
+                }
+            }
+    free(G); free(Cm); free(x); free(y);
+    return rc;
 }

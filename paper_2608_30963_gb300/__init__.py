@@ -88,7 +88,8 @@ class kvx_translator_info(ctypes.Structure):
                 ("weight_bytes", ctypes.c_int64), ("table_bytes", ctypes.c_int64)]
 
 
-EXPORTS = ["kvx_translator_create", "kvx_translator_create_low_rank", "kvx_translate", "kvx_build_alignment", "kvx_layer_map_nearest",
+EXPORTS = ["kvx_translator_create", "kvx_translator_create_low_rank", "kvx_translate", "kvx_fit_create",
+           "kvx_fit_accumulate", "kvx_fit_solve", "kvx_fit_reset", "kvx_fit_tokens", "kvx_fit_destroy", "kvx_build_alignment", "kvx_layer_map_nearest",
            "kvx_get_device_status", "kvx_get_info", "kvx_launches_per_translate", "kvx_last_error",
            "kvx_destroy", "kvx_translate_static", "kvx_static_last_error"]
 KVX_STATIC_SCRATCH_BYTES = 8 << 20
@@ -137,8 +138,18 @@ def lib():
                                            ctypes.POINTER(kvx_tgt_tokens), ctypes.POINTER(kvx_dst_kv),
                                            ctypes.POINTER(ctypes.c_uint32), VP]
         L.kvx_static_last_error.restype = ctypes.c_char_p
+        L.kvx_fit_create.argtypes = [ctypes.POINTER(kvx_translator_desc), ctypes.c_double, ctypes.c_int32,
+                                     ctypes.POINTER(VP)]
+        L.kvx_fit_accumulate.argtypes = [VP, ctypes.POINTER(kvx_src_kv), ctypes.POINTER(kvx_tgt_tokens),
+                                         ctypes.POINTER(kvx_dst_kv), VP]
+        L.kvx_fit_solve.argtypes = [VP, VP, VP, ctypes.POINTER(ctypes.c_uint32), VP]
+        L.kvx_fit_reset.argtypes = [VP, VP]
+        L.kvx_fit_tokens.argtypes = [VP]
+        L.kvx_fit_tokens.restype = ctypes.c_int64
+        L.kvx_fit_destroy.argtypes = [VP]
         for name in EXPORTS:
-            if name not in ("kvx_last_error", "kvx_launches_per_translate", "kvx_static_last_error"):
+            if name not in ("kvx_last_error", "kvx_launches_per_translate", "kvx_static_last_error",
+                            "kvx_fit_tokens"):
                 getattr(L, name).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -236,6 +247,84 @@ def _stream(stream) -> int:
     return int(getattr(stream, "cuda_stream", stream))
 
 
+def _call_structs(src_k, src_v, src_seq_len, tgt_seq_off, total_tokens, dst_k, dst_v, span_lo, span_hi, src_pos,
+                  tgt_pos, page_table, page_size, num_pages):
+    """The three call structs of kvx_translate / kvx_fit_accumulate for torch tensors."""
+    s0 = src_k[0]
+    src = kvx_src_kv(s0.shape[0], s0.shape[2], _ptr_array(src_k), _ptr_array(src_v),
+                     s0.stride(0), s0.stride(1), s0.stride(2), _ptr(src_seq_len), _ptr(src_pos))
+    tgt = kvx_tgt_tokens(int(total_tokens), _ptr(tgt_seq_off), _ptr(span_lo), _ptr(span_hi), _ptr(tgt_pos))
+    d0 = dst_k[0]
+    if page_table is None:
+        dst = kvx_dst_kv(_ptr_array(dst_k), _ptr_array(dst_v), 0, d0.shape[2], d0.stride(0), d0.stride(1),
+                         d0.stride(2), None, 0, 0, 0)
+    else:
+        dst = kvx_dst_kv(_ptr_array(dst_k), _ptr_array(dst_v), 1, 0, 0, 0, 0, _ptr(page_table),
+                         page_table.shape[1], page_size, num_pages or d0.shape[0])
+    return src, tgt, dst
+
+
+def _desc(src_geom, dst_geom, layer_map, dtype, max_position, path, form, layers_per_target, keep: list):
+    lm = None
+    if layer_map is not None:
+        flat = [int(x) for row in layer_map for x in (row if hasattr(row, "__len__") else [row])]
+        arr = (ctypes.c_int32 * len(flat))(*flat)
+        keep.append(arr)
+        lm = ctypes.cast(arr, I32P)
+    return kvx_translator_desc(model_geom(src_geom), model_geom(dst_geom), lm, dtype, max_position, path, form,
+                               layers_per_target)
+
+
+class Fitter:
+    """Owns one kvx_fitter: closed-form ridge fit of a linear translator's W_K, W_V from
+    calibration batches (source caches and the target model's own caches of the same contexts)."""
+
+    def __init__(self, src_geom, dst_geom, lam: float, layer_map: Optional[Sequence] = None, dtype: int = KVX_BF16,
+                 form: int = KVX_FORM_GROUPED, layers_per_target: int = 1, chunk_tokens: int = 0,
+                 max_position: int = 0):
+        self._keep = []
+        self.desc = _desc(src_geom, dst_geom, layer_map, dtype, max_position, KVX_PATH_AUTO, form, layers_per_target,
+                          self._keep)
+        h = VP()
+        _check(lib().kvx_fit_create(ctypes.byref(self.desc), float(lam), int(chunk_tokens), ctypes.byref(h)))
+        self.handle = h.value
+
+    def accumulate(self, src_k: Sequence, src_v: Sequence, src_seq_len, tgt_seq_off, total_tokens: int,
+                   tgt_k: Sequence, tgt_v: Sequence, *, span_lo=None, span_hi=None, src_pos=None, tgt_pos=None,
+                   page_table=None, page_size: int = 16, num_pages: int = 0, stream=None):
+        """Arguments as Translator.translate; tgt_k/tgt_v are the target model's own caches (read)."""
+        src, tgt, dst = _call_structs(src_k, src_v, src_seq_len, tgt_seq_off, total_tokens, tgt_k, tgt_v, span_lo,
+                                      span_hi, src_pos, tgt_pos, page_table, page_size, num_pages)
+        _check(lib().kvx_fit_accumulate(VP(self.handle), ctypes.byref(src), ctypes.byref(tgt), ctypes.byref(dst),
+                                        VP(_stream(stream))))
+
+    def solve(self, w_k, w_v, stream=None) -> int:
+        """Writes W_K, W_V (device tensors [L_t, H_t, in, out] of the cache dtype); returns the status word."""
+        bits = ctypes.c_uint32(0)
+        st = lib().kvx_fit_solve(VP(self.handle), VP(_ptr(w_k)), VP(_ptr(w_v)), ctypes.byref(bits),
+                                 VP(_stream(stream)))
+        if st not in (KVX_OK, KVX_ERR_DEVICE_STATUS):
+            _check(st)
+        return bits.value
+
+    def reset(self, stream=None):
+        _check(lib().kvx_fit_reset(VP(self.handle), VP(_stream(stream))))
+
+    def tokens(self) -> int:
+        return lib().kvx_fit_tokens(VP(self.handle))
+
+    def close(self):
+        if getattr(self, "handle", None):
+            _check(lib().kvx_fit_destroy(VP(self.handle)))
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
 class Translator:
     """Owns one kvx_translator.  Weights are torch tensors (host or device)
     [L_t, H_t, in, out] of the translator dtype; they are copied at creation.
@@ -275,17 +364,8 @@ class Translator:
         """src_k/src_v: per source layer [B, H_s, S_max, d_s] tensors (strided, d contiguous).
         dst_k/dst_v: per target layer, contiguous [B, H_t, T_max, d_t] (page_table None) or paged pools
         [num_pages, page_size, H_t, d_t]."""
-        s0 = src_k[0]
-        src = kvx_src_kv(s0.shape[0], s0.shape[2], _ptr_array(src_k), _ptr_array(src_v),
-                         s0.stride(0), s0.stride(1), s0.stride(2), _ptr(src_seq_len), _ptr(src_pos))
-        tgt = kvx_tgt_tokens(int(total_tokens), _ptr(tgt_seq_off), _ptr(span_lo), _ptr(span_hi), _ptr(tgt_pos))
-        d0 = dst_k[0]
-        if page_table is None:
-            dst = kvx_dst_kv(_ptr_array(dst_k), _ptr_array(dst_v), 0, d0.shape[2], d0.stride(0), d0.stride(1),
-                             d0.stride(2), None, 0, 0, 0)
-        else:
-            dst = kvx_dst_kv(_ptr_array(dst_k), _ptr_array(dst_v), 1, 0, 0, 0, 0, _ptr(page_table),
-                             page_table.shape[1], page_size, num_pages or d0.shape[0])
+        src, tgt, dst = _call_structs(src_k, src_v, src_seq_len, tgt_seq_off, total_tokens, dst_k, dst_v, span_lo,
+                                      span_hi, src_pos, tgt_pos, page_table, page_size, num_pages)
         kvx_translate(self.handle, src, tgt, dst, _stream(stream))
 
     def device_status(self, stream=None, clear: bool = True) -> int:

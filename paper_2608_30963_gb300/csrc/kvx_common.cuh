@@ -96,6 +96,25 @@ struct TranslateParams {
     void* dst_v[KVX_MAX_TARGET_LAYERS];
 };
 
+// Validated translator geometry (host side), shared by kvx_translator_create and the fitter.
+struct Geometry {
+    kvx_translator_desc desc;            // the caller's description, layer_map pointer cleared
+    int layer_map[KVX_MAX_SRC_SLOTS];    // [j * kl + k]: source layers of target layer j
+    int in_dim, r, e, dense, kl, hpl;
+    int max_position;
+    unsigned long long turns[256];       // fixed-point turns: source [ds/2] | target [dt/2]
+    int rope_same;                       // source and target turns identical
+};
+// Checks a description and derives the geometry; no CUDA call.  On failure returns the status
+// and writes a message (prefixed with who) to err[512].
+kvx_status make_geometry(const kvx_translator_desc* desc, const char* who, Geometry& g, char* err);
+// Launch parameters of one call over the caller's caches (argument checks included).
+kvx_status make_params(const Geometry& g, const unsigned long long* dev_turns, unsigned* status, const void* w,
+                       const kvx_src_kv* src, const kvx_tgt_tokens* tgt, const kvx_dst_kv* dst, TranslateParams& P,
+                       const char* who, char* err);
+// Thread-local message returned by kvx_last_error().
+void set_last_error(const char* msg);
+
 // First source head feeding target head h: its GQA group (h*r), the source head it
 // repeats (h/e), or head 0 in the dense per-layer form.
 __device__ __forceinline__ int src_head0(const TranslateParams& P, int h)

@@ -1,0 +1,380 @@
+// kvx_fit.cu -- closed-form fit of the linear translator (paper Section 5).
+//
+// Section 5 gives the learning objective L_KV = D(T_theta(KV_A(C)), KV_B(C)).  With D the
+// squared Euclidean distance over target tokens plus a ridge term lambda |W|^2, every
+// (target layer j, target head h, K|V) group is a least-squares problem solved by the normal
+// equations (X^T X + lambda I) W = X^T Y:
+//   X rows: the translator's input rows (span mean of the un-rotated source rows, as the
+//           translation forms them), rounded to the cache dtype;
+//   Y rows: the target model's own cache rows, target RoPE undone for K.
+// Three steps:
+//   1. fit_rows_kernel builds X and Y for one pass of up to chunk tokens, every group at once
+//      (HBM-bound gather, CUDA cores);
+//   2. two strided-batched cuBLAS GEMMs over the groups add X^T X and X^T Y into fp32 sums
+//      (a plain dense contraction over tokens: tensor cores through the library);
+//   3. at solve time, fit_solve_kernel (one CTA per group) factors X^T X + lambda I = L L^T in
+//      double and runs the two triangular solves per output column.
+#include <cublas_v2.h>
+#include <math.h>
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "kvx_common.cuh"
+#include "kvx_kernels.h"
+
+namespace kvx {
+namespace {
+
+constexpr int kFitTile = 32;
+constexpr int kFitThreads = 256;
+constexpr int kSolveThreads = 256;
+constexpr unsigned kFitNotPosDef = 0x20u;   // status bit: a system was not positive definite
+
+struct FitRows {
+    void* x;      // [groups][chunk][in]
+    void* y;      // [groups][chunk][dt]
+    int chunk;    // token capacity of one group's block
+    int t0;       // first packed target token of this pass
+    int n;        // tokens in this pass
+};
+
+// One CTA per (32-token tile of the pass, target head, target layer * 2 + K|V).
+template <typename T>
+__global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_constant__ TranslateParams P, const FitRows R)
+{
+    __shared__ TokenInfo tinfo[kFitTile];
+    const int h = blockIdx.y;
+    const int j = blockIdx.z >> 1;
+    const int kv = blockIdx.z & 1;
+    const int g = (j * P.Ht + h) * 2 + kv;
+    const int tt0 = blockIdx.x * kFitTile;
+    const int ntok = min(kFitTile, R.n - tt0);
+    if ((int)threadIdx.x < ntok) tinfo[threadIdx.x] = resolve_token(P, R.t0 + tt0 + (int)threadIdx.x);
+    __syncthreads();
+
+    T* X = (T*)R.x + ((size_t)g * R.chunk + tt0) * P.in_dim;
+    T* Y = (T*)R.y + ((size_t)g * R.chunk + tt0) * P.dt;
+    const T* tgt = (const T*)(kv ? P.dst_v[j] : P.dst_k[j]);
+    const long long hoff = dst_head_off(P, h);
+    const bool rot_s = kv == 0 && P.rs.enabled;
+    const bool rot_t = kv == 0 && P.rt.enabled;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int hs = P.ds >> 1, ht = P.dt >> 1;
+    for (int tt = warp; tt < ntok; tt += kFitThreads / 32) {
+        const TokenInfo ti = tinfo[tt];
+        const bool use = ti.dst_off >= 0 && ti.hi > ti.lo;   // rows without a target row stay zero
+        for (int k = lane; k < P.in_dim; k += 32) {
+            float acc = 0.f;
+            if (use) {
+                const int q = k / P.ds, c = k - q * P.ds;
+                int slot, gs;
+                head_block(P, j, h, q, slot, gs);
+                const T* src = (const T*)(kv ? P.src_v[slot] : P.src_k[slot]);
+                const T* base = src + (long long)ti.b * P.sb + (long long)gs * P.sh;
+                for (int s = ti.lo; s < ti.hi; ++s) {
+                    const T* row = base + (long long)s * P.ss;
+                    float x = to_f32<T>(row[c]);
+                    if (rot_s) {
+                        const int i = c < hs ? c : c - hs;
+                        const float xp = to_f32<T>(row[c < hs ? c + hs : c - hs]);
+                        const float2 cs = rope_cs(P.rs, src_pos_of(P, ti.b, s), i);
+                        x = c < hs ? fmaf(x, cs.x, xp * cs.y) : fmaf(x, cs.x, -xp * cs.y);   // R(-theta)
+                    }
+                    acc += x;
+                }
+                acc /= (float)(ti.hi - ti.lo);
+            }
+            X[(size_t)tt * P.in_dim + k] = from_f32<T>(acc);
+        }
+        for (int c = lane; c < P.dt; c += 32) {
+            float y = 0.f;
+            if (use) {
+                const T* row = tgt + ti.dst_off + hoff;
+                y = to_f32<T>(row[c]);
+                if (rot_t) {
+                    const int i = c < ht ? c : c - ht;
+                    const float yp = to_f32<T>(row[c < ht ? c + ht : c - ht]);
+                    const float2 cs = rope_cs(P.rt, ti.pt, i);
+                    y = c < ht ? fmaf(y, cs.x, yp * cs.y) : fmaf(y, cs.x, -yp * cs.y);       // R(-theta)
+                }
+            }
+            Y[(size_t)tt * P.dt + c] = from_f32<T>(y);
+        }
+    }
+}
+
+// One CTA per group g = (j*Ht + h)*2 + kv.  G: fp32 X^T X [in][in]; C: fp32 X^T Y, column-major
+// [dt][in] (element (a, o) at o*in + a); A, Z: double scratch [in][in] and [in][dt].
+// W out: the group's [in][dt] block of W_K or W_V in the cache dtype.
+template <typename T>
+__global__ void __launch_bounds__(kSolveThreads) fit_solve_kernel(const float* __restrict__ G,
+                                                                  const float* __restrict__ C, double* A, double* Z,
+                                                                  T* wk, T* wv, int in, int dt, double lambda,
+                                                                  unsigned* status)
+{
+    __shared__ int bad;
+    const int g = blockIdx.x;
+    double* a = A + (size_t)g * in * in;
+    double* z = Z + (size_t)g * in * dt;
+    const float* gg = G + (size_t)g * in * in;
+    const float* cc = C + (size_t)g * in * dt;
+    if (threadIdx.x == 0) bad = 0;
+    for (int i = threadIdx.x; i < in * in; i += blockDim.x) {
+        const int r = i / in, c = i - r * in;
+        a[i] = c <= r ? (double)gg[i] + (r == c ? lambda : 0.0) : 0.0;
+    }
+    __syncthreads();
+    // right-looking Cholesky on the lower triangle: a = L L^T
+    for (int k = 0; k < in; ++k) {
+        if (threadIdx.x == 0) {
+            double d = a[(size_t)k * in + k];
+            if (!(d > 0.0)) { bad = 1; d = 1.0; }
+            a[(size_t)k * in + k] = sqrt(d);
+        }
+        __syncthreads();
+        const double dk = a[(size_t)k * in + k];
+        for (int r = k + 1 + threadIdx.x; r < in; r += blockDim.x) a[(size_t)r * in + k] /= dk;
+        __syncthreads();
+        const int m = in - k - 1;
+        for (int idx = threadIdx.x; idx < m * m; idx += blockDim.x) {
+            const int rr = k + 1 + idx / m, c2 = k + 1 + idx % m;
+            if (c2 <= rr) a[(size_t)rr * in + c2] -= a[(size_t)rr * in + k] * a[(size_t)c2 * in + k];
+        }
+        __syncthreads();
+    }
+    // per output column o: L u = c (forward), L^T w = u (backward); z holds u then w, [in][dt]
+    for (int o = threadIdx.x; o < dt; o += blockDim.x) {
+        for (int r = 0; r < in; ++r) {
+            double v = (double)cc[(size_t)o * in + r];
+            for (int k = 0; k < r; ++k) v -= a[(size_t)r * in + k] * z[(size_t)k * dt + o];
+            z[(size_t)r * dt + o] = v / a[(size_t)r * in + r];
+        }
+        for (int r = in - 1; r >= 0; --r) {
+            double v = z[(size_t)r * dt + o];
+            for (int k = r + 1; k < in; ++k) v -= a[(size_t)k * in + r] * z[(size_t)k * dt + o];
+            z[(size_t)r * dt + o] = v / a[(size_t)r * in + r];
+        }
+    }
+    __syncthreads();
+    T* w = (g & 1) ? wv : wk;
+    const size_t off = (size_t)(g >> 1) * in * dt;   // (j*Ht + h) block of [Lt][Ht][in][dt]
+    for (int i = threadIdx.x; i < in * dt; i += blockDim.x) w[off + i] = from_f32<T>(bad ? 0.f : (float)z[i]);
+    if (bad && threadIdx.x == 0) set_status(status, kFitNotPosDef);
+}
+
+}  // namespace
+}  // namespace kvx
+
+using namespace kvx;
+
+struct kvx_fitter {
+    Geometry geo;
+    int device = 0;
+    int groups = 0, chunk = 0;
+    double lambda = 0.0;
+    long long tokens = 0;
+    unsigned long long* rope = nullptr;   // device turns
+    unsigned* status = nullptr;
+    void* rows = nullptr;                 // X [groups][chunk][in] | Y [groups][chunk][dt]
+    float* sums = nullptr;                // G [groups][in][in] | C [groups][dt][in]
+    void* blas_ws = nullptr;
+    cublasHandle_t blas = nullptr;
+};
+
+static const size_t kBlasWorkspace = 32u << 20;
+
+static kvx_status fit_fail(kvx_status s, const char* fmt, ...) __attribute__((format(printf, 2, 3)));
+static kvx_status fit_fail(kvx_status s, const char* fmt, ...)
+{
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    set_last_error(buf);
+    return s;
+}
+
+static void free_fitter(kvx_fitter* f)
+{
+    if (!f) return;
+    if (f->blas) cublasDestroy(f->blas);
+    if (f->blas_ws) cudaFree(f->blas_ws);
+    if (f->rows) cudaFree(f->rows);
+    if (f->sums) cudaFree(f->sums);
+    if (f->rope) cudaFree(f->rope);
+    if (f->status) cudaFree(f->status);
+    delete f;
+}
+
+static size_t fit_elt(const kvx_fitter* f) { return f->geo.desc.dtype == KVX_BF16 ? 2 : 4; }
+static size_t sums_floats(const kvx_fitter* f)
+{
+    const size_t in = f->geo.in_dim, dt = f->geo.desc.dst.head_dim;
+    return (size_t)f->groups * in * (in + dt);
+}
+
+extern "C" KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, double lambda, int32_t chunk_tokens,
+                                             kvx_fitter** out)
+{
+    if (!desc || !out) return fit_fail(KVX_ERR_INVALID_ARG, "fit_create: NULL argument");
+    *out = nullptr;
+    if (!(lambda >= 0.0)) return fit_fail(KVX_ERR_INVALID_ARG, "fit_create: lambda must be >= 0");
+    if (chunk_tokens < 0 || chunk_tokens > (1 << 20))
+        return fit_fail(KVX_ERR_INVALID_ARG, "fit_create: chunk_tokens outside [0, 1<<20]");
+    char err[512];
+    kvx_fitter* f = new kvx_fitter();
+    kvx_status st = make_geometry(desc, "fit_create", f->geo, err);
+    if (st != KVX_OK) {
+        delete f;
+        set_last_error(err);
+        return st;
+    }
+    if (f->geo.in_dim > 512) {
+        delete f;
+        return fit_fail(KVX_ERR_UNSUPPORTED, "fit_create: translator input width %d > 512", f->geo.in_dim);
+    }
+    const kvx_translator_desc& D = f->geo.desc;
+    f->lambda = lambda;
+    f->chunk = chunk_tokens ? chunk_tokens : 4096;
+    f->groups = D.dst.num_layers * D.dst.num_kv_heads * 2;
+    const size_t in = f->geo.in_dim, dt = D.dst.head_dim;
+    const size_t row_bytes = (size_t)f->groups * f->chunk * (in + dt) * fit_elt(f);
+    const size_t rope_bytes = (size_t)(D.src.head_dim / 2 + D.dst.head_dim / 2) * sizeof(unsigned long long);
+    cudaError_t ce;
+    if (cudaGetDevice(&f->device) != cudaSuccess) { free_fitter(f); return fit_fail(KVX_ERR_CUDA, "fit_create: no CUDA device"); }
+    if (cudaMalloc(&f->rows, row_bytes) != cudaSuccess || cudaMalloc(&f->sums, sums_floats(f) * sizeof(float)) != cudaSuccess ||
+        cudaMalloc(&f->rope, rope_bytes) != cudaSuccess || cudaMalloc(&f->status, sizeof(unsigned)) != cudaSuccess ||
+        cudaMalloc(&f->blas_ws, kBlasWorkspace) != cudaSuccess) {
+        free_fitter(f);
+        return fit_fail(KVX_ERR_OOM, "fit_create: device allocation (%zu bytes of rows)", row_bytes);
+    }
+    if ((ce = cudaMemcpy(f->rope, f->geo.turns, rope_bytes, cudaMemcpyHostToDevice)) != cudaSuccess ||
+        (ce = cudaMemset(f->sums, 0, sums_floats(f) * sizeof(float))) != cudaSuccess ||
+        (ce = cudaMemset(f->status, 0, sizeof(unsigned))) != cudaSuccess || (ce = cudaDeviceSynchronize()) != cudaSuccess) {
+        free_fitter(f);
+        return fit_fail(KVX_ERR_CUDA, "fit_create: %s", cudaGetErrorString(ce));
+    }
+    if (cublasCreate(&f->blas) != CUBLAS_STATUS_SUCCESS ||
+        cublasSetWorkspace(f->blas, f->blas_ws, kBlasWorkspace) != CUBLAS_STATUS_SUCCESS) {
+        free_fitter(f);
+        return fit_fail(KVX_ERR_CUDA, "fit_create: cuBLAS initialisation");
+    }
+    *out = f;
+    return KVX_OK;
+}
+
+extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
+                                                 const kvx_dst_kv* target_cache, void* stream)
+{
+    if (!f || !src || !tgt || !target_cache) return fit_fail(KVX_ERR_INVALID_ARG, "fit_accumulate: NULL argument");
+    TranslateParams P;
+    char err[512];
+    kvx_status st = make_params(f->geo, f->rope, f->status, nullptr, src, tgt, target_cache, P, "fit_accumulate", err);
+    if (st != KVX_OK) {
+        set_last_error(err);
+        return st;
+    }
+    if (tgt->total_tokens == 0) return KVX_OK;
+    const kvx_translator_desc& D = f->geo.desc;
+    const int in = f->geo.in_dim, dt = D.dst.head_dim;
+    const bool bf = D.dtype == KVX_BF16;
+    const size_t elt = fit_elt(f);
+    cudaStream_t s = (cudaStream_t)stream;
+    if (cublasSetStream(f->blas, s) != CUBLAS_STATUS_SUCCESS)
+        return fit_fail(KVX_ERR_CUDA, "fit_accumulate: cublasSetStream");
+    char* xbase = (char*)f->rows;
+    char* ybase = xbase + (size_t)f->groups * f->chunk * in * elt;
+    float* G = f->sums;
+    float* C = f->sums + (size_t)f->groups * in * in;
+    const float one = 1.f;
+    const cudaDataType_t ty = bf ? CUDA_R_16BF : CUDA_R_32F;
+    for (int t0 = 0; t0 < tgt->total_tokens; t0 += f->chunk) {
+        const int n = tgt->total_tokens - t0 < f->chunk ? tgt->total_tokens - t0 : f->chunk;
+        FitRows R{xbase, ybase, f->chunk, t0, n};
+        dim3 grid((n + kFitTile - 1) / kFitTile, D.dst.num_kv_heads, D.dst.num_layers * 2);
+        if (bf) fit_rows_kernel<__nv_bfloat16><<<grid, kFitThreads, 0, s>>>(P, R);
+        else fit_rows_kernel<float><<<grid, kFitThreads, 0, s>>>(P, R);
+        cudaError_t ce = cudaGetLastError();
+        if (ce != cudaSuccess) return fit_fail(KVX_ERR_CUDA, "fit_accumulate: %s", cudaGetErrorString(ce));
+        // G[g] += X^T X: column-major X is in x n (ld in); C[g] += X^T Y with Y column-major dt x n (ld dt)
+        cublasStatus_t bs = cublasGemmStridedBatchedEx(
+            f->blas, CUBLAS_OP_N, CUBLAS_OP_T, in, in, n, &one, xbase, ty, in, (long long)f->chunk * in, xbase, ty, in,
+            (long long)f->chunk * in, &one, G, CUDA_R_32F, in, (long long)in * in, f->groups, CUBLAS_COMPUTE_32F,
+            CUBLAS_GEMM_DEFAULT);
+        if (bs == CUBLAS_STATUS_SUCCESS)
+            bs = cublasGemmStridedBatchedEx(f->blas, CUBLAS_OP_N, CUBLAS_OP_T, in, dt, n, &one, xbase, ty, in,
+                                            (long long)f->chunk * in, ybase, ty, dt, (long long)f->chunk * dt, &one, C,
+                                            CUDA_R_32F, in, (long long)in * dt, f->groups, CUBLAS_COMPUTE_32F,
+                                            CUBLAS_GEMM_DEFAULT);
+        if (bs != CUBLAS_STATUS_SUCCESS) return fit_fail(KVX_ERR_CUDA, "fit_accumulate: cuBLAS GEMM failed (%d)", (int)bs);
+    }
+    f->tokens += tgt->total_tokens;
+    return KVX_OK;
+}
+
+extern "C" KVX_API kvx_status kvx_fit_solve(kvx_fitter* f, void* w_k, void* w_v, uint32_t* status_bits, void* stream)
+{
+    if (!f || !w_k || !w_v) return fit_fail(KVX_ERR_INVALID_ARG, "fit_solve: NULL argument");
+    const kvx_translator_desc& D = f->geo.desc;
+    const int in = f->geo.in_dim, dt = D.dst.head_dim;
+    cudaStream_t s = (cudaStream_t)stream;
+    // double scratch for the factorisation and the solutions: the row workspace is reused when it is
+    // large enough, otherwise a temporary allocation (solve is not on the translation path)
+    const size_t need = (size_t)f->groups * in * (in + dt) * sizeof(double);
+    const size_t have = (size_t)f->groups * f->chunk * (in + dt) * fit_elt(f);
+    double* scratch = nullptr;
+    bool own = false;
+    cudaError_t ce;
+    if (need <= have) {
+        scratch = (double*)f->rows;
+    } else {
+        if (cudaMalloc(&scratch, need) != cudaSuccess) return fit_fail(KVX_ERR_OOM, "fit_solve: scratch allocation");
+        own = true;
+    }
+    double* A = scratch;
+    double* Z = scratch + (size_t)f->groups * in * in;
+    const float* G = f->sums;
+    const float* C = f->sums + (size_t)f->groups * in * in;
+    if (D.dtype == KVX_BF16)
+        fit_solve_kernel<__nv_bfloat16><<<f->groups, kSolveThreads, 0, s>>>(G, C, A, Z, (__nv_bfloat16*)w_k,
+                                                                            (__nv_bfloat16*)w_v, in, dt, f->lambda,
+                                                                            f->status);
+    else
+        fit_solve_kernel<float><<<f->groups, kSolveThreads, 0, s>>>(G, C, A, Z, (float*)w_k, (float*)w_v, in, dt,
+                                                                    f->lambda, f->status);
+    unsigned bits = 0;
+    if ((ce = cudaGetLastError()) != cudaSuccess || (ce = cudaStreamSynchronize(s)) != cudaSuccess ||
+        (ce = cudaMemcpy(&bits, f->status, sizeof bits, cudaMemcpyDeviceToHost)) != cudaSuccess) {
+        if (own) cudaFree(scratch);
+        return fit_fail(KVX_ERR_CUDA, "fit_solve: %s", cudaGetErrorString(ce));
+    }
+    if (own) cudaFree(scratch);
+    if (status_bits) *status_bits = bits;
+    if (bits & kFitNotPosDef)
+        return fit_fail(KVX_ERR_DEVICE_STATUS, "fit_solve: a system was not positive definite (status 0x%x)", bits);
+    return KVX_OK;
+}
+
+extern "C" KVX_API kvx_status kvx_fit_reset(kvx_fitter* f, void* stream)
+{
+    if (!f) return fit_fail(KVX_ERR_INVALID_ARG, "fit_reset: NULL fitter");
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t ce;
+    if ((ce = cudaMemsetAsync(f->sums, 0, sums_floats(f) * sizeof(float), s)) != cudaSuccess ||
+        (ce = cudaMemsetAsync(f->status, 0, sizeof(unsigned), s)) != cudaSuccess)
+        return fit_fail(KVX_ERR_CUDA, "fit_reset: %s", cudaGetErrorString(ce));
+    f->tokens = 0;
+    return KVX_OK;
+}
+
+extern "C" KVX_API int64_t kvx_fit_tokens(const kvx_fitter* f) { return f ? f->tokens : 0; }
+
+extern "C" KVX_API kvx_status kvx_fit_destroy(kvx_fitter* f)
+{
+    if (!f) return KVX_OK;
+    cudaDeviceSynchronize();
+    free_fitter(f);
+    return KVX_OK;
+}

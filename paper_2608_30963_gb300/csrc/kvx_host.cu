@@ -14,6 +14,7 @@
 using namespace kvx;
 
 struct kvx_translator {
+    Geometry geo;                       // validated description (shared with the fitter)
     kvx_translator_desc desc;
     int layer_map[KVX_MAX_SRC_SLOTS];   // [j * kl + k]: source layers of target layer j
     int device = 0;
@@ -125,6 +126,152 @@ static void free_translator(kvx_translator* t)
     delete t;
 }
 
+namespace kvx {
+
+void set_last_error(const char* msg) { g_last_error = msg; }
+
+kvx_status make_geometry(const kvx_translator_desc* desc, const char* who, Geometry& g, char* err)
+{
+    auto bad = [&](kvx_status st, const char* fmt, auto... args) {
+        int n = snprintf(err, 512, "%s: ", who);
+        snprintf(err + n, 512 - n, fmt, args...);
+        return st;
+    };
+    const kvx_model_geom& s = desc->src;
+    const kvx_model_geom& d = desc->dst;
+    if (s.num_layers < 1 || d.num_layers < 1 || s.num_kv_heads < 1 || d.num_kv_heads < 1)
+        return bad(KVX_ERR_INVALID_ARG, "layer and head counts must be >= 1");
+    if (d.num_layers > KVX_MAX_TARGET_LAYERS)
+        return bad(KVX_ERR_UNSUPPORTED, "at most %d target layers", KVX_MAX_TARGET_LAYERS);
+    if (!head_dim_ok(s.head_dim) || !head_dim_ok(d.head_dim))
+        return bad(KVX_ERR_UNSUPPORTED, "head dims must be 64, 128 or 256 (got %d, %d)", s.head_dim, d.head_dim);
+    if (s.num_kv_heads % d.num_kv_heads != 0 && d.num_kv_heads % s.num_kv_heads != 0)
+        return bad(KVX_ERR_UNSUPPORTED, "neither KV head count divides the other (%d, %d)", s.num_kv_heads,
+                   d.num_kv_heads);
+    if (desc->dtype != KVX_BF16 && desc->dtype != KVX_FP32)
+        return bad(KVX_ERR_INVALID_ARG, "unknown dtype %d", desc->dtype);
+    if (desc->path < KVX_PATH_AUTO || desc->path > KVX_PATH_TCGEN05)
+        return bad(KVX_ERR_INVALID_ARG, "unknown path %d", desc->path);
+    if (!rope_schedule_ok(s) || !rope_schedule_ok(d))
+        return bad(KVX_ERR_INVALID_ARG, "unknown rope_type or schedule parameters out of range "
+                                        "(source type %d, target type %d)", s.rope_type, d.rope_type);
+    const int max_pos = desc->max_position ? desc->max_position : (1 << 24);
+    if (max_pos < 1 || max_pos > (1 << 30)) return bad(KVX_ERR_INVALID_ARG, "max_position must be in [1, 1<<30]");
+    if (desc->form != KVX_FORM_GROUPED && desc->form != KVX_FORM_DENSE)
+        return bad(KVX_ERR_INVALID_ARG, "unknown form %d", desc->form);
+    const int kl = desc->layers_per_target > 1 ? desc->layers_per_target : 1;
+    if (desc->layers_per_target < 0 || kl > 4 || d.num_layers * kl > KVX_MAX_SRC_SLOTS)
+        return bad(KVX_ERR_INVALID_ARG, "layers_per_target %d outside [0, 4] or more than %d "
+                                        "(target layer, source layer) pairs", desc->layers_per_target, KVX_MAX_SRC_SLOTS);
+    if (kl > 1 && !desc->layer_map) return bad(KVX_ERR_INVALID_ARG, "layers_per_target > 1 needs an explicit layer_map");
+    g.desc = *desc;
+    g.desc.layer_map = nullptr;
+    g.max_position = max_pos;
+    g.kl = kl;
+    g.dense = desc->form == KVX_FORM_DENSE;
+    if (desc->layer_map) {
+        for (int i = 0; i < d.num_layers * kl; ++i) {
+            if (desc->layer_map[i] < 0 || desc->layer_map[i] >= s.num_layers)
+                return bad(KVX_ERR_INVALID_ARG, "layer_map[%d] = %d outside [0, %d)", i, desc->layer_map[i],
+                           s.num_layers);
+            g.layer_map[i] = desc->layer_map[i];
+        }
+    } else {
+        kvx_layer_map_nearest(s.num_layers, d.num_layers, g.layer_map);
+    }
+    g.r = g.e = 1;
+    if (s.num_kv_heads >= d.num_kv_heads) g.r = s.num_kv_heads / d.num_kv_heads;
+    else g.e = d.num_kv_heads / s.num_kv_heads;
+    g.hpl = g.dense ? s.num_kv_heads : g.r;
+    g.in_dim = kl * g.hpl * s.head_dim;
+    if (g.in_dim > 1024) return bad(KVX_ERR_UNSUPPORTED, "translator input width %d > 1024", g.in_dim);
+    // rotation frequencies as fixed-point turns (kvx_common.cuh)
+    const int hs = s.head_dim / 2, hd = d.head_dim / 2;
+    auto fill = [&](const kvx_model_geom& m, unsigned long long* o) {
+        for (int i = 0; i < m.head_dim / 2; ++i)
+            o[i] = m.rope_base <= 0.0 ? 0ull : (unsigned long long)ldexp(rope_inv_freq(m, i) / (2.0 * M_PI), 64);
+    };
+    memset(g.turns, 0, sizeof g.turns);
+    fill(s, g.turns);
+    fill(d, g.turns + hs);
+    // the two rotations coincide when head dims, enablement and every frequency agree
+    g.rope_same = hs == hd && (s.rope_base > 0.0) == (d.rope_base > 0.0) &&
+                  memcmp(g.turns, g.turns + hs, (size_t)hs * sizeof(unsigned long long)) == 0;
+    return KVX_OK;
+}
+
+static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+kvx_status make_params(const Geometry& g, const unsigned long long* dev_turns, unsigned* status, const void* w,
+                       const kvx_src_kv* src, const kvx_tgt_tokens* tgt, const kvx_dst_kv* dst, TranslateParams& P,
+                       const char* who, char* err)
+{
+    auto bad = [&](kvx_status st, const char* fmt, auto... args) {
+        int n = snprintf(err, 512, "%s: ", who);
+        snprintf(err + n, 512 - n, fmt, args...);
+        return st;
+    };
+    const kvx_translator_desc& D = g.desc;
+    const int Lt = D.dst.num_layers;
+    const int vec = D.dtype == KVX_BF16 ? 8 : 4;   // elements per 16 bytes
+    if (src->batch < 1) return bad(KVX_ERR_INVALID_ARG, "batch must be >= 1");
+    if (src->max_seq < 0 || tgt->total_tokens < 0) return bad(KVX_ERR_INVALID_ARG, "negative size");
+    if (!src->k || !src->v || !src->seq_len || !tgt->seq_off || !dst->k || !dst->v)
+        return bad(KVX_ERR_INVALID_ARG, "NULL array");
+    if ((tgt->span_lo == nullptr) != (tgt->span_hi == nullptr))
+        return bad(KVX_ERR_INVALID_ARG, "span_lo and span_hi must both be set or both NULL");
+    if (src->stride_s < D.src.head_dim || src->stride_h < 1 || src->stride_b < 1 || src->stride_s % vec ||
+        src->stride_h % vec || src->stride_b % vec)
+        return bad(KVX_ERR_INVALID_ARG, "source strides must be positive multiples of %d elements with "
+                                        "stride_s >= head_dim", vec);
+    if (!dst->paged) {
+        if (dst->stride_t < D.dst.head_dim || dst->stride_h < 1 || dst->stride_b < 1 || dst->stride_t % vec ||
+            dst->stride_h % vec || dst->stride_b % vec || dst->max_seq < 0)
+            return bad(KVX_ERR_INVALID_ARG, "target strides must be positive multiples of %d elements with "
+                                            "stride_t >= head_dim", vec);
+    } else if (!dst->page_table || dst->page_size < 1 || dst->max_pages_per_seq < 1 || dst->num_pages < 1) {
+        return bad(KVX_ERR_INVALID_ARG, "paged target needs page_table, page_size, max_pages_per_seq and "
+                                        "num_pages >= 1");
+    }
+    memset(&P, 0, sizeof P);
+    P.Hs = D.src.num_kv_heads; P.ds = D.src.head_dim;
+    P.Ht = D.dst.num_kv_heads; P.dt = D.dst.head_dim;
+    P.in_dim = g.in_dim; P.r = g.r; P.e = g.e; P.Lt = Lt;
+    P.dense = g.dense; P.kl = g.kl; P.hpl = g.hpl;
+    P.batch = src->batch; P.src_max_seq = src->max_seq;
+    P.sb = src->stride_b; P.sh = src->stride_h; P.ss = src->stride_s;
+    P.src_seq_len = src->seq_len; P.src_pos = src->pos;
+    P.T_total = tgt->total_tokens; P.seq_off = tgt->seq_off;
+    P.span_lo = tgt->span_lo; P.span_hi = tgt->span_hi; P.tgt_pos = tgt->pos;
+    P.paged = dst->paged; P.dst_max_seq = dst->max_seq;
+    P.db = dst->stride_b; P.dh = dst->stride_h; P.dts = dst->stride_t;
+    P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
+    P.page_size = dst->page_size; P.num_pages = dst->num_pages;
+    const int hs = D.src.head_dim / 2;
+    P.rs = RopeTable{dev_turns, hs, D.src.rope_base > 0.0};
+    P.rt = RopeTable{dev_turns + hs, D.dst.head_dim / 2, D.dst.rope_base > 0.0};
+    P.max_position = g.max_position;
+    P.rope_same = g.rope_same;
+    P.status = status;
+    P.w = w;
+    for (int i = 0; i < Lt * g.kl; ++i) {
+        const int l = g.layer_map[i];
+        P.src_k[i] = src->k[l]; P.src_v[i] = src->v[l];
+        if (!P.src_k[i] || !P.src_v[i]) return bad(KVX_ERR_INVALID_ARG, "NULL cache pointer for source layer %d", l);
+        if (!aligned16(P.src_k[i]) || !aligned16(P.src_v[i]))
+            return bad(KVX_ERR_INVALID_ARG, "cache pointers must be 16-byte aligned (source layer %d)", l);
+    }
+    for (int j = 0; j < Lt; ++j) {
+        P.dst_k[j] = dst->k[j]; P.dst_v[j] = dst->v[j];
+        if (!P.dst_k[j] || !P.dst_v[j]) return bad(KVX_ERR_INVALID_ARG, "NULL cache pointer for target layer %d", j);
+        if (!aligned16(P.dst_k[j]) || !aligned16(P.dst_v[j]))
+            return bad(KVX_ERR_INVALID_ARG, "cache pointers must be 16-byte aligned (target layer %d)", j);
+    }
+    return KVX_OK;
+}
+
+}  // namespace kvx
+
 extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* desc, const void* w_k,
                                                     const void* w_v, int32_t weights_on_device,
                                                     kvx_translator** out)
@@ -133,61 +280,21 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
     *out = nullptr;
     const kvx_model_geom& s = desc->src;
     const kvx_model_geom& d = desc->dst;
-    if (s.num_layers < 1 || d.num_layers < 1 || s.num_kv_heads < 1 || d.num_kv_heads < 1)
-        return fail(KVX_ERR_INVALID_ARG, "create: layer and head counts must be >= 1");
-    if (d.num_layers > KVX_MAX_TARGET_LAYERS)
-        return fail(KVX_ERR_UNSUPPORTED, "create: at most %d target layers", KVX_MAX_TARGET_LAYERS);
-    if (!head_dim_ok(s.head_dim) || !head_dim_ok(d.head_dim))
-        return fail(KVX_ERR_UNSUPPORTED, "create: head dims must be 64, 128 or 256 (got %d, %d)", s.head_dim,
-                    d.head_dim);
-    if (s.num_kv_heads % d.num_kv_heads != 0 && d.num_kv_heads % s.num_kv_heads != 0)
-        return fail(KVX_ERR_UNSUPPORTED, "create: neither KV head count divides the other (%d, %d)",
-                    s.num_kv_heads, d.num_kv_heads);
-    if (desc->dtype != KVX_BF16 && desc->dtype != KVX_FP32)
-        return fail(KVX_ERR_INVALID_ARG, "create: unknown dtype %d", desc->dtype);
-    if (desc->path < KVX_PATH_AUTO || desc->path > KVX_PATH_TCGEN05)
-        return fail(KVX_ERR_INVALID_ARG, "create: unknown path %d", desc->path);
-    if (!rope_schedule_ok(s) || !rope_schedule_ok(d))
-        return fail(KVX_ERR_INVALID_ARG, "create: unknown rope_type or schedule parameters out of range "
-                                         "(source type %d, target type %d)", s.rope_type, d.rope_type);
-    int max_pos = desc->max_position ? desc->max_position : (1 << 24);
-    if (max_pos < 1 || max_pos > (1 << 30))
-        return fail(KVX_ERR_INVALID_ARG, "create: max_position must be in [1, 1<<30]");
-    if (desc->form != KVX_FORM_GROUPED && desc->form != KVX_FORM_DENSE)
-        return fail(KVX_ERR_INVALID_ARG, "create: unknown form %d", desc->form);
-    const int kl = desc->layers_per_target > 1 ? desc->layers_per_target : 1;
-    if (desc->layers_per_target < 0 || kl > 4 || d.num_layers * kl > KVX_MAX_SRC_SLOTS)
-        return fail(KVX_ERR_INVALID_ARG, "create: layers_per_target %d outside [0, 4] or more than %d "
-                                         "(target layer, source layer) pairs", desc->layers_per_target,
-                    KVX_MAX_SRC_SLOTS);
-    if (kl > 1 && !desc->layer_map)
-        return fail(KVX_ERR_INVALID_ARG, "create: layers_per_target > 1 needs an explicit layer_map");
-
+    char err[512];
     kvx_translator* t = new kvx_translator();
-    t->desc = *desc;
-    t->desc.layer_map = nullptr;
-    t->max_position = max_pos;
-    t->kl = kl;
-    t->dense = desc->form == KVX_FORM_DENSE;
-    if (desc->layer_map) {
-        for (int i = 0; i < d.num_layers * kl; ++i) {
-            if (desc->layer_map[i] < 0 || desc->layer_map[i] >= s.num_layers) {
-                delete t;
-                return fail(KVX_ERR_INVALID_ARG, "create: layer_map[%d] = %d outside [0, %d)", i,
-                            desc->layer_map[i], s.num_layers);
-            }
-            t->layer_map[i] = desc->layer_map[i];
-        }
-    } else {
-        kvx_layer_map_nearest(s.num_layers, d.num_layers, t->layer_map);
-    }
-    if (s.num_kv_heads >= d.num_kv_heads) t->r = s.num_kv_heads / d.num_kv_heads;
-    else t->e = d.num_kv_heads / s.num_kv_heads;
-    t->hpl = t->dense ? s.num_kv_heads : t->r;
-    t->in_dim = kl * t->hpl * s.head_dim;
-    if (t->in_dim > 1024) {
+    kvx_status gst = make_geometry(desc, "create", t->geo, err);
+    if (gst != KVX_OK) {
         delete t;
-        return fail(KVX_ERR_UNSUPPORTED, "create: translator input width %d > 1024", t->in_dim);
+        g_last_error = err;
+        return gst;
+    }
+    {
+        const Geometry& g = t->geo;
+        t->desc = g.desc;
+        memcpy(t->layer_map, g.layer_map, sizeof t->layer_map);
+        t->max_position = g.max_position;
+        t->kl = g.kl; t->dense = g.dense; t->r = g.r; t->e = g.e; t->hpl = g.hpl; t->in_dim = g.in_dim;
+        t->rope_same = g.rope_same;
     }
 
     if (cudaGetDevice(&t->device) != cudaSuccess ||
@@ -244,32 +351,20 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         raw = nullptr;
     }
 
-    {   // rotation frequencies as fixed-point turns (kvx_common.cuh)
+    {   // rotation frequencies as fixed-point turns (kvx_common.cuh), from the geometry
         const int hs = s.head_dim / 2, hd = d.head_dim / 2;
-        unsigned long long h_turns[256];
-        auto fill = [&](const kvx_model_geom& g, unsigned long long* out) {
-            for (int i = 0; i < g.head_dim / 2; ++i) {
-                if (g.rope_base <= 0.0) { out[i] = 0; continue; }
-                out[i] = (unsigned long long)ldexp(rope_inv_freq(g, i) / (2.0 * M_PI), 64);
-            }
-        };
-        fill(s, h_turns);
-        fill(d, h_turns + hs);
         t->rope_bytes = (size_t)(hs + hd) * sizeof(unsigned long long);
         if (cudaMalloc(&t->rope, t->rope_bytes) != cudaSuccess) {
             st = fail(KVX_ERR_OOM, "create: table allocation");
             goto err;
         }
-        memcpy(t->host_turns, h_turns, t->rope_bytes);
-        if ((ce = cudaMemcpy(t->rope, h_turns, t->rope_bytes, cudaMemcpyHostToDevice)) != cudaSuccess) {
+        memcpy(t->host_turns, t->geo.turns, sizeof t->host_turns);
+        if ((ce = cudaMemcpy(t->rope, t->geo.turns, t->rope_bytes, cudaMemcpyHostToDevice)) != cudaSuccess) {
             st = fail(KVX_ERR_CUDA, "create: table upload: %s", cudaGetErrorString(ce));
             goto err;
         }
         t->rs = RopeTable{t->rope, hs, s.rope_base > 0.0};
         t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0};
-        // the two rotations coincide when head dims, enablement and every frequency agree
-        t->rope_same = hs == hd && t->rs.enabled == t->rt.enabled &&
-                       memcmp(h_turns, h_turns + hs, (size_t)hs * sizeof(unsigned long long)) == 0;
     }
     if (cudaMalloc(&t->status, sizeof(unsigned)) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: status allocation"); goto err; }
     if (t->path == KVX_PATH_TCGEN05 && cudaMalloc(&t->plan, tc_plan_bytes(kvx_translator::kPlanTokens)) != cudaSuccess) {
@@ -335,71 +430,21 @@ extern "C" KVX_API kvx_status kvx_translator_create_low_rank(const kvx_translato
     return st;
 }
 
-static bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
-
 extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
                                             const kvx_dst_kv* dst, void* stream)
 {
     if (!tr || !src || !tgt || !dst) return fail(KVX_ERR_INVALID_ARG, "translate: NULL argument");
     const kvx_translator_desc& D = tr->desc;
     const int Lt = D.dst.num_layers;
-    const int vec = D.dtype == KVX_BF16 ? 8 : 4;   // elements per 16 bytes
-    if (src->batch < 1) return fail(KVX_ERR_INVALID_ARG, "translate: batch must be >= 1");
-    if (src->max_seq < 0 || tgt->total_tokens < 0) return fail(KVX_ERR_INVALID_ARG, "translate: negative size");
-    if (!src->k || !src->v || !src->seq_len || !tgt->seq_off || !dst->k || !dst->v)
-        return fail(KVX_ERR_INVALID_ARG, "translate: NULL array");
-    if ((tgt->span_lo == nullptr) != (tgt->span_hi == nullptr))
-        return fail(KVX_ERR_INVALID_ARG, "translate: span_lo and span_hi must both be set or both NULL");
-    if (src->stride_s < D.src.head_dim || src->stride_h < 1 || src->stride_b < 1 || src->stride_s % vec ||
-        src->stride_h % vec || src->stride_b % vec)
-        return fail(KVX_ERR_INVALID_ARG, "translate: source strides must be positive multiples of %d "
-                                         "elements with stride_s >= head_dim", vec);
-    if (!dst->paged) {
-        if (dst->stride_t < D.dst.head_dim || dst->stride_h < 1 || dst->stride_b < 1 || dst->stride_t % vec ||
-            dst->stride_h % vec || dst->stride_b % vec || dst->max_seq < 0)
-            return fail(KVX_ERR_INVALID_ARG, "translate: target strides must be positive multiples of %d "
-                                             "elements with stride_t >= head_dim", vec);
-    } else if (!dst->page_table || dst->page_size < 1 || dst->max_pages_per_seq < 1 || dst->num_pages < 1) {
-        return fail(KVX_ERR_INVALID_ARG, "translate: paged target needs page_table, page_size, "
-                                         "max_pages_per_seq and num_pages >= 1");
-    }
     tr->last_launches = 0;
-    if (tgt->total_tokens == 0) return KVX_OK;
-
     TranslateParams P;
-    memset(&P, 0, sizeof P);
-    P.Hs = D.src.num_kv_heads; P.ds = D.src.head_dim;
-    P.Ht = D.dst.num_kv_heads; P.dt = D.dst.head_dim;
-    P.in_dim = tr->in_dim; P.r = tr->r; P.e = tr->e; P.Lt = Lt;
-    P.dense = tr->dense; P.kl = tr->kl; P.hpl = tr->hpl;
-    P.batch = src->batch; P.src_max_seq = src->max_seq;
-    P.sb = src->stride_b; P.sh = src->stride_h; P.ss = src->stride_s;
-    P.src_seq_len = src->seq_len; P.src_pos = src->pos;
-    P.T_total = tgt->total_tokens; P.seq_off = tgt->seq_off;
-    P.span_lo = tgt->span_lo; P.span_hi = tgt->span_hi; P.tgt_pos = tgt->pos;
-    P.paged = dst->paged; P.dst_max_seq = dst->max_seq;
-    P.db = dst->stride_b; P.dh = dst->stride_h; P.dts = dst->stride_t;
-    P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
-    P.page_size = dst->page_size; P.num_pages = dst->num_pages;
-    P.rs = tr->rs; P.rt = tr->rt; P.max_position = tr->max_position;
-    P.rope_same = tr->rope_same;
-    P.status = tr->status;
-    P.w = tr->w;
-    for (int i = 0; i < Lt * tr->kl; ++i) {
-        const int l = tr->layer_map[i];
-        P.src_k[i] = src->k[l]; P.src_v[i] = src->v[l];
-        if (!P.src_k[i] || !P.src_v[i])
-            return fail(KVX_ERR_INVALID_ARG, "translate: NULL cache pointer for source layer %d", l);
-        if (!aligned16(P.src_k[i]) || !aligned16(P.src_v[i]))
-            return fail(KVX_ERR_INVALID_ARG, "translate: cache pointers must be 16-byte aligned (source layer %d)", l);
+    char err[512];
+    const kvx_status pst = make_params(tr->geo, tr->rope, tr->status, tr->w, src, tgt, dst, P, "translate", err);
+    if (pst != KVX_OK) {
+        g_last_error = err;
+        return pst;
     }
-    for (int j = 0; j < Lt; ++j) {
-        P.dst_k[j] = dst->k[j]; P.dst_v[j] = dst->v[j];
-        if (!P.dst_k[j] || !P.dst_v[j])
-            return fail(KVX_ERR_INVALID_ARG, "translate: NULL cache pointer for target layer %d", j);
-        if (!aligned16(P.dst_k[j]) || !aligned16(P.dst_v[j]))
-            return fail(KVX_ERR_INVALID_ARG, "translate: cache pointers must be 16-byte aligned (target layer %d)", j);
-    }
+    if (tgt->total_tokens == 0) return KVX_OK;
     cudaError_t ce;
     if (tr->path == KVX_PATH_TCGEN05 && !tgt->span_lo &&
         aligned_supported(tr->in_dim, D.dst.head_dim, D.src.head_dim, Lt, src->batch, tr->kl)) {

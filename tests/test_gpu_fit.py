@@ -1,0 +1,201 @@
+"""The closed-form translator fit (kvx_fit_*) against the oracle's fit, through the C ABI.
+
+The oracle solves the normal equations in double from exact span means; the library rounds
+the input rows X and the target rows Y to the cache dtype and sums X^T X, X^T Y in fp32.
+Tolerance for bf16: the rounding of X and Y is about 2^-9 / sqrt(3) ~ 1.1e-3 relative (RMS),
+and least squares amplifies it by cond(X) ~ (1 + sqrt(in/T)) / (1 - sqrt(in/T)), 2.4 at
+in = 256, T = 1500: ~3e-3 relative on W, so rel-L2 <= 1e-2.  fp32 caches: 1e-4.
+"""
+import dataclasses
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+import oracle
+import paper_2608_30963_gb300 as kvx
+from paper_2608_30963_gb300 import synth
+
+from harness import make_case, oracle_problem
+
+pytestmark = pytest.mark.gpu
+SPECS = synth.config_specs()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    kvx.build()
+    yield
+
+
+def _shrink(spec, Ls, Lt, **kw):
+    return dataclasses.replace(spec, src=dataclasses.replace(spec.src, num_layers=Ls),
+                               dst=dataclasses.replace(spec.dst, num_layers=Lt), **kw)
+
+
+def _rel(a, b):
+    return float(np.linalg.norm(np.asarray(a, np.float64) - b) / np.linalg.norm(b))
+
+
+def _targets_from(c, wk, wv):
+    """The target model's 'own' caches: the oracle's translation with planted weights,
+    stored in the cache dtype, per target layer [B, Ht, t_max, dt]."""
+    p = oracle_problem(dataclasses.replace(c, w_k=wk, w_v=wv))
+    ok, ov = p.translate()                                   # [Lt, Ht, T, dt]
+    wl, s = c.wl, c.spec
+    Lt, Ht, dt = s.dst.num_layers, s.dst.num_kv_heads, s.dst.head_dim
+    tk = np.zeros((Lt, wl.batch, Ht, max(wl.t_max, 1), dt), np.float32)
+    tv = np.zeros_like(tk)
+    for b in range(wl.batch):
+        a, e = int(wl.tgt_seq_off[b]), int(wl.tgt_seq_off[b + 1])
+        tk[:, b, :, :e - a] = ok[:, :, a:e]
+        tv[:, b, :, :e - a] = ov[:, :, a:e]
+    if s.dtype == "bf16":
+        tk, tv = synth.bf16_round(tk), synth.bf16_round(tv)
+    return tk, tv
+
+
+def _fit_gpu(c, tk, tv, lam, chunk=0, split=None, paged=False):
+    from gpu_harness import DeviceCase, to_dev, i32
+    s = c.spec
+    g = DeviceCase(c, path=kvx.KVX_PATH_SIMT, paged=False)     # device source buffers and metadata
+    dtk = [to_dev(tk[j], s.dtype) for j in range(s.dst.num_layers)]
+    dtv = [to_dev(tv[j], s.dtype) for j in range(s.dst.num_layers)]
+    f = kvx.Fitter(s.src, s.dst, lam, layer_map=c.layer_map.tolist(), dtype=g.tr.desc.dtype, form=s.form,
+                   layers_per_target=s.layers_per_target, chunk_tokens=chunk)
+    wl = c.wl
+    kw = dict(span_lo=g.span_lo, span_hi=g.span_hi)
+    if paged:
+        P = s.page_size
+        pages = [(int(t) + P - 1) // P for t in wl.tgt_len]
+        npg, mp = sum(pages), max(pages)
+        perm = np.random.default_rng(9).permutation(npg).astype(np.int32)
+        pt = np.full((wl.batch, mp), -1, np.int32)
+        k = 0
+        for b, n in enumerate(pages):
+            pt[b, :n] = perm[k:k + n]; k += n
+        pool_k = [torch.zeros((npg, P, s.dst.num_kv_heads, s.dst.head_dim), dtype=dtk[0].dtype, device="cuda")
+                  for _ in dtk]
+        pool_v = [torch.zeros_like(x) for x in pool_k]
+        for j in range(s.dst.num_layers):
+            for b in range(wl.batch):
+                for t in range(int(wl.tgt_len[b])):
+                    pool_k[j][pt[b, t // P], t % P] = dtk[j][b, :, t]
+                    pool_v[j][pt[b, t // P], t % P] = dtv[j][b, :, t]
+        dtk, dtv = pool_k, pool_v
+        kw.update(page_table=i32(pt), page_size=P, num_pages=npg)
+    if split is None:
+        f.accumulate(g.src_k, g.src_v, g.src_len, g.seq_off, wl.total_tgt, dtk, dtv, **kw)
+    else:
+        # two calibration calls over sequences [0, split) and [split, B)
+        for lo, hi in ((0, split), (split, wl.batch)):
+            a, e = int(wl.tgt_seq_off[lo]), int(wl.tgt_seq_off[hi])
+            sk = [x[lo:hi] for x in g.src_k]
+            sv = [x[lo:hi] for x in g.src_v]
+            off = i32(wl.tgt_seq_off[lo:hi + 1] - a)
+            kws = dict(span_lo=None if g.span_lo is None else g.span_lo[a:e],
+                       span_hi=None if g.span_hi is None else g.span_hi[a:e])
+            f.accumulate(sk, sv, g.src_len[lo:hi], off, e - a, [x[lo:hi] for x in dtk], [x[lo:hi] for x in dtv],
+                         **kws)
+    in_dim = s.group_in
+    tdt = torch.bfloat16 if s.dtype == "bf16" else torch.float32
+    wk = torch.empty((s.dst.num_layers, s.dst.num_kv_heads, in_dim, s.dst.head_dim), dtype=tdt, device="cuda")
+    wv = torch.empty_like(wk)
+    bits = f.solve(wk, wv)
+    assert f.tokens() == wl.total_tgt
+    from gpu_harness import to_host
+    return to_host(wk), to_host(wv), bits, f
+
+
+CASES = {
+    # name: (base spec, Ls, Lt, target lengths, extra spec fields)
+    "qwen7b_qwen1p5b_identity": ("qwen7b_to_qwen1p5b_4k", 3, 2, [900, 600], {}),
+    "gemma_expansion_spans": ("qwen1p5b_to_gemma2b_1k", 3, 2, [700, 500], {}),
+    # dense per-layer form over 2 source heads of 128 (in = 256), cross-tokenizer spans
+    "dense_spans": ("llama70b_to_qwen7b_8k", 4, 2, [1100, 700], dict(form=synth.FORM_DENSE,
+                                                                   src=synth.ModelGeom(4, 2, 128, 5e5),
+                                                                   dst=synth.ModelGeom(2, 2, 64, 1e6))),
+}
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_fit_recovers_planted_translator_and_matches_oracle(name):
+    base, Ls, Lt, lens, kw = CASES[name]
+    spec = _shrink(SPECS[base], Ls, Lt)
+    if "dst" in kw:
+        kw = dict(kw, dst=dataclasses.replace(kw["dst"], num_layers=Lt))
+    if "src" in kw:
+        kw = dict(kw, src=dataclasses.replace(kw["src"], num_layers=Ls))
+    spec = dataclasses.replace(spec, **kw)
+    c = make_case(spec, lens)
+    rng = np.random.default_rng(17)
+    din, dt = spec.group_in, spec.dst.head_dim
+    w_true = [synth.bf16_round(rng.standard_normal((Lt, spec.dst.num_kv_heads, din, dt)).astype(np.float32)
+                               / np.float32(np.sqrt(din))) for _ in range(2)]
+    tk, tv = _targets_from(c, *w_true)
+    lam = 1e-3
+    gk, gv, bits, _ = _fit_gpu(c, tk, tv, lam)
+    assert bits == 0
+    ok, ov = oracle_problem(c).fit(list(tk), list(tv), lam)
+    for gpu, ref, true in ((gk, ok, w_true[0]), (gv, ov, w_true[1])):
+        assert np.all(np.isfinite(gpu))
+        assert _rel(gpu, ref) <= 1e-2, _rel(gpu, ref)
+        assert _rel(gpu, true) <= 1e-2, _rel(gpu, true)
+        assert _rel(ref, true) <= 5e-3, _rel(ref, true)
+
+
+def test_fit_fp32_tiny_matches_oracle_tightly():
+    spec = SPECS["tiny_fp32"]
+    c = make_case(spec, [256, 200])
+    rng = np.random.default_rng(18)
+    tk = rng.standard_normal((2, 2, 1, 256, 64)).astype(np.float32)   # unrelated targets: a genuine fit
+    tv = rng.standard_normal((2, 2, 1, 256, 64)).astype(np.float32)
+    lam = 0.5
+    gk, gv, bits, _ = _fit_gpu(c, tk, tv, lam)
+    ok, ov = oracle_problem(c).fit(list(tk), list(tv), lam)
+    assert bits == 0
+    assert _rel(gk, ok) <= 1e-4 and _rel(gv, ov) <= 1e-4
+
+
+def test_fit_two_calls_chunked_and_paged_agree_with_one_call():
+    """Sums over calibration calls and accumulation passes add up: one call, two calls, a
+    small chunk (several passes) and a paged target cache give the same W (fp32 summation
+    order only)."""
+    spec = _shrink(SPECS["qwen1p5b_to_gemma2b_1k"], 2, 2)
+    c = make_case(spec, [500, 300, 400])
+    rng = np.random.default_rng(19)
+    w_true = [synth.bf16_round(rng.standard_normal((2, 4, 128, 256)).astype(np.float32) / np.float32(np.sqrt(128)))
+              for _ in range(2)]
+    tk, tv = _targets_from(c, *w_true)
+    one_k, one_v, _, f = _fit_gpu(c, tk, tv, 1e-2)
+    for kw in (dict(split=1), dict(chunk=160), dict(paged=True)):
+        k2, v2, bits, _ = _fit_gpu(c, tk, tv, 1e-2, **kw)
+        assert bits == 0
+        assert _rel(k2, one_k) <= 2e-3 and _rel(v2, one_v) <= 2e-3, kw
+    # reset: a second fit from the same fitter after reset equals the first
+    f.reset()
+    assert f.tokens() == 0
+
+
+def test_fitted_translator_reproduces_the_targets():
+    """End to end: fit on a calibration context, build a translator from the fitted W and
+    translate the same context: the output is the target cache up to bf16 rounding."""
+    from gpu_harness import DeviceCase, to_dev
+    from harness import compare
+    spec = _shrink(SPECS["qwen7b_to_qwen1p5b_4k"], 2, 2)
+    c = make_case(spec, [1200])
+    rng = np.random.default_rng(20)
+    w_true = [synth.bf16_round(rng.standard_normal((2, 2, 256, 128)).astype(np.float32) / np.float32(16.0))
+              for _ in range(2)]
+    tk, tv = _targets_from(c, *w_true)
+    gk, gv, bits, _ = _fit_gpu(c, tk, tv, 1e-3)
+    fitted = dataclasses.replace(c, w_k=synth.bf16_round(gk), w_v=synth.bf16_round(gv))
+    g = DeviceCase(fitted)
+    g.run()
+    torch.cuda.synchronize()
+    outk, outv = g.gather()
+    ref_k = np.stack([tk[j][0] for j in range(2)])    # [Lt, Ht, T, dt]
+    ref_v = np.stack([tv[j][0] for j in range(2)])
+    compare(outk, ref_k, "bf16")
+    compare(outv, ref_v, "bf16")

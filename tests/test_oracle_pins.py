@@ -493,3 +493,79 @@ def test_latent_adapter_equals_the_product_matrix():
     xbar = np.concatenate([vs[1][0, g, lo[t]:hi[t]].astype(np.float64).mean(0) for g in (0, 1)])
     np.testing.assert_allclose(ov[0, 0, t], (xbar @ a[0, 0, :, 0].astype(np.float64)) * b[0, 0, 0].astype(np.float64),
                                rtol=1e-12, atol=1e-12)
+
+
+# ------------------------------------------------ closed-form translator fit (Section 5, L_KV)
+def _fit_case(rng, sg, dg, layer_map, T, spans_key=None):
+    if spans_key is None:
+        lo = hi = None
+        S = T
+    else:
+        lo, hi, S, _, _ = synth.draw_spans(T, spans_key)
+    ks, vs = _rand_src(rng, sg, 1, S)
+    if sg.rope_base > 0:
+        ks = [oracle.rope_cache(k, sg.rope_base) for k in ks]
+    return ks, vs, lo, hi, S
+
+
+def test_fit_matches_numpy_least_squares_without_rope():
+    """No RoPE, identity alignment: x_t is concat(grouped heads) of row t, y_t the target row;
+    the oracle's W equals numpy's least-squares / ridge solutions on X built here from the raw
+    arrays."""
+    rng = np.random.default_rng(41)
+    sg, dg = _geom(2, 4, 64, 0.0), _geom(1, 2, 64, 0.0)
+    T = 300
+    ks, vs, _, _, S = _fit_case(rng, sg, dg, [1], T)
+    tk = [rng.standard_normal((1, 2, T, 64)).astype(np.float32)]
+    tv = [rng.standard_normal((1, 2, T, 64)).astype(np.float32)]
+    p = _problem_f(sg, dg, [1], [T], ks, vs, np.zeros((1, 2, 128, 64), np.float32),
+                   np.zeros((1, 2, 128, 64), np.float32))
+    for lam in (0.0, 3.5):
+        wk, wv = p.fit(tk, tv, lam)
+        for h in range(2):
+            for src, tgt, w in ((ks, tk, wk), (vs, tv, wv)):
+                X = np.concatenate([src[1][0, 2 * h], src[1][0, 2 * h + 1]], axis=1).astype(np.float64)
+                Y = tgt[0][0, h].astype(np.float64)
+                if lam == 0.0:
+                    ref = np.linalg.lstsq(X, Y, rcond=None)[0]
+                else:
+                    ref = np.linalg.solve(X.T @ X + lam * np.eye(128), X.T @ Y)
+                np.testing.assert_allclose(w[0, h], ref, rtol=1e-9, atol=1e-10)
+                # stationarity of the ridge objective
+                grad = X.T @ (X @ w[0, h] - Y) + lam * w[0, h]
+                assert np.abs(grad).max() < 1e-8 * max(1.0, np.abs(X.T @ Y).max())
+
+
+def test_fit_recovers_a_planted_translator():
+    """Target caches produced by translating with W_true (RoPE on both sides, spans, GQA):
+    the un-regularised fit recovers W_true."""
+    rng = np.random.default_rng(42)
+    sg, dg = _geom(3, 4, 64, 1e6), _geom(2, 2, 64, 1e4)
+    T = 400
+    ks, vs, lo, hi, S = _fit_case(rng, sg, dg, [2, 0], T, spans_key=7)
+    w_true_k = rng.standard_normal((2, 2, 128, 64)).astype(np.float32)
+    w_true_v = rng.standard_normal((2, 2, 128, 64)).astype(np.float32)
+    p = _problem_f(sg, dg, [2, 0], [T], ks, vs, w_true_k, w_true_v, lo, hi)
+    ok, ov = p.translate()                                    # [Lt, Ht, T, dt]
+    tk = [ok[j][None].astype(np.float32) for j in range(2)]   # [1, Ht, T, dt]
+    tv = [ov[j][None].astype(np.float32) for j in range(2)]
+    wk, wv = p.fit(tk, tv, 0.0)
+    # the targets were rounded to float32, so recovery is to ~1e-5 relative
+    np.testing.assert_allclose(wk, w_true_k, atol=2e-4)
+    np.testing.assert_allclose(wv, w_true_v, atol=2e-4)
+
+
+def test_fit_ridge_shrinks_toward_xty_over_lambda():
+    """As lambda grows, lambda W tends to X^T Y."""
+    rng = np.random.default_rng(43)
+    sg, dg = _geom(1, 1, 64, 1e4), _geom(1, 1, 64, 1e4)
+    T = 50
+    ks, vs, _, _, S = _fit_case(rng, sg, dg, [0], T)
+    tk = [rng.standard_normal((1, 1, T, 64)).astype(np.float32)]
+    tv = [rng.standard_normal((1, 1, T, 64)).astype(np.float32)]
+    z = np.zeros((1, 1, 64, 64), np.float32)
+    p = _problem_f(sg, dg, [0], [T], ks, vs, z, z)
+    lam = 1e9
+    _, wv = p.fit(tk, tv, lam)
+    X = vs[0][0, 0].astype(np.float64)
+    np.testing.assert_allclose(lam * wv[0, 0], X.T @ tv[0][0, 0].astype(np.float64), rtol=1e-6, atol=1e-6)
