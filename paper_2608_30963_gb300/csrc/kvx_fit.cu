@@ -39,10 +39,47 @@ struct FitRows {
     int n;        // tokens in this pass
 };
 
-// One CTA per (32-token tile of the pass, target head, target layer * 2 + K|V).
+// 16-byte chunks of T: VEC elements, as raw words and back.
+template <typename T> struct Chunk;
+template <> struct Chunk<__nv_bfloat16> {
+    static constexpr int VEC = 8;
+    __device__ static void unpack(const uint4& w, float (&x)[8])
+    {
+        const uint32_t v[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) { x[2 * i] = __uint_as_float(v[i] << 16); x[2 * i + 1] = __uint_as_float(v[i] & 0xFFFF0000u); }
+    }
+    __device__ static uint4 pack(const float (&x)[8])
+    {
+        uint32_t v[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            __nv_bfloat162 b = __floats2bfloat162_rn(x[2 * i], x[2 * i + 1]);
+            v[i] = *reinterpret_cast<uint32_t*>(&b);
+        }
+        return make_uint4(v[0], v[1], v[2], v[3]);
+    }
+};
+template <> struct Chunk<float> {
+    static constexpr int VEC = 4;
+    __device__ static void unpack(const uint4& w, float (&x)[4])
+    {
+        x[0] = __uint_as_float(w.x); x[1] = __uint_as_float(w.y); x[2] = __uint_as_float(w.z); x[3] = __uint_as_float(w.w);
+    }
+    __device__ static uint4 pack(const float (&x)[4])
+    {
+        return make_uint4(__float_as_uint(x[0]), __float_as_uint(x[1]), __float_as_uint(x[2]), __float_as_uint(x[3]));
+    }
+};
+
+// One CTA per (32-token tile of the pass, target head, target layer * 2 + K|V).  A work item is
+// one chunk pair: VEC channels [c, c+VEC) of the first rotary half of one head row and their
+// partners [c+d/2, ...), read and written as 16-byte words, with one (cos, sin) per pair.
+// X items: (token, head-block q, chunk pair); Y items: (token, chunk pair).
 template <typename T>
 __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_constant__ TranslateParams P, const FitRows R)
 {
+    constexpr int VEC = Chunk<T>::VEC;
     __shared__ TokenInfo tinfo[kFitTile];
     const int h = blockIdx.y;
     const int j = blockIdx.z >> 1;
@@ -59,48 +96,74 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
     const long long hoff = dst_head_off(P, h);
     const bool rot_s = kv == 0 && P.rs.enabled;
     const bool rot_t = kv == 0 && P.rt.enabled;
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int hs = P.ds >> 1, ht = P.dt >> 1;
-    for (int tt = warp; tt < ntok; tt += kFitThreads / 32) {
+    const int ncp_s = hs / VEC, ncp_t = ht / VEC;       // chunk pairs per head row
+    const int heads = P.in_dim / P.ds;                  // head-blocks in an input row
+    const int x_items = ntok * heads * ncp_s;
+    for (int it = threadIdx.x; it < x_items; it += blockDim.x) {
+        const int tt = it / (heads * ncp_s);
+        const int rem = it - tt * (heads * ncp_s);
+        const int q = rem / ncp_s, cp = rem - q * ncp_s;
         const TokenInfo ti = tinfo[tt];
-        const bool use = ti.dst_off >= 0 && ti.hi > ti.lo;   // rows without a target row stay zero
-        for (int k = lane; k < P.in_dim; k += 32) {
-            float acc = 0.f;
-            if (use) {
-                const int q = k / P.ds, c = k - q * P.ds;
-                int slot, gs;
-                head_block(P, j, h, q, slot, gs);
-                const T* src = (const T*)(kv ? P.src_v[slot] : P.src_k[slot]);
-                const T* base = src + (long long)ti.b * P.sb + (long long)gs * P.sh;
-                for (int s = ti.lo; s < ti.hi; ++s) {
-                    const T* row = base + (long long)s * P.ss;
-                    float x = to_f32<T>(row[c]);
-                    if (rot_s) {
-                        const int i = c < hs ? c : c - hs;
-                        const float xp = to_f32<T>(row[c < hs ? c + hs : c - hs]);
-                        const float2 cs = rope_cs(P.rs, src_pos_of(P, ti.b, s), i);
-                        x = c < hs ? fmaf(x, cs.x, xp * cs.y) : fmaf(x, cs.x, -xp * cs.y);   // R(-theta)
+        float a0[VEC], a1[VEC];
+#pragma unroll
+        for (int e = 0; e < VEC; ++e) { a0[e] = 0.f; a1[e] = 0.f; }
+        if (ti.dst_off >= 0 && ti.hi > ti.lo) {
+            int slot, gs;
+            head_block(P, j, h, q, slot, gs);
+            const T* base = (const T*)(kv ? P.src_v[slot] : P.src_k[slot]) + (long long)ti.b * P.sb +
+                            (long long)gs * P.sh + cp * VEC;
+            for (int s = ti.lo; s < ti.hi; ++s) {
+                const T* row = base + (long long)s * P.ss;
+                float x0[VEC], x1[VEC];
+                Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row)), x0);
+                Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + hs)), x1);
+                if (rot_s) {
+                    const int pos = src_pos_of(P, ti.b, s);
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e) {   // R(-theta)
+                        const float2 cs = rope_cs(P.rs, pos, cp * VEC + e);
+                        a0[e] += fmaf(x0[e], cs.x, x1[e] * cs.y);
+                        a1[e] += fmaf(x1[e], cs.x, -x0[e] * cs.y);
                     }
-                    acc += x;
-                }
-                acc /= (float)(ti.hi - ti.lo);
-            }
-            X[(size_t)tt * P.in_dim + k] = from_f32<T>(acc);
-        }
-        for (int c = lane; c < P.dt; c += 32) {
-            float y = 0.f;
-            if (use) {
-                const T* row = tgt + ti.dst_off + hoff;
-                y = to_f32<T>(row[c]);
-                if (rot_t) {
-                    const int i = c < ht ? c : c - ht;
-                    const float yp = to_f32<T>(row[c < ht ? c + ht : c - ht]);
-                    const float2 cs = rope_cs(P.rt, ti.pt, i);
-                    y = c < ht ? fmaf(y, cs.x, yp * cs.y) : fmaf(y, cs.x, -yp * cs.y);       // R(-theta)
+                } else {
+#pragma unroll
+                    for (int e = 0; e < VEC; ++e) { a0[e] += x0[e]; a1[e] += x1[e]; }
                 }
             }
-            Y[(size_t)tt * P.dt + c] = from_f32<T>(y);
+            const float inv = 1.f / (float)(ti.hi - ti.lo);
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) { a0[e] *= inv; a1[e] *= inv; }
         }
+        T* xr = X + (size_t)tt * P.in_dim + q * P.ds + cp * VEC;
+        *reinterpret_cast<uint4*>(xr) = Chunk<T>::pack(a0);
+        *reinterpret_cast<uint4*>(xr + hs) = Chunk<T>::pack(a1);
+    }
+    const int y_items = ntok * ncp_t;
+    for (int it = threadIdx.x; it < y_items; it += blockDim.x) {
+        const int tt = it / ncp_t, cp = it - tt * ncp_t;
+        const TokenInfo ti = tinfo[tt];
+        float y0[VEC], y1[VEC];
+        if (ti.dst_off >= 0 && ti.hi > ti.lo) {
+            const T* row = tgt + ti.dst_off + hoff + cp * VEC;
+            Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row)), y0);
+            Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + ht)), y1);
+            if (rot_t) {
+#pragma unroll
+                for (int e = 0; e < VEC; ++e) {   // R(-theta)
+                    const float2 cs = rope_cs(P.rt, ti.pt, cp * VEC + e);
+                    const float u0 = fmaf(y0[e], cs.x, y1[e] * cs.y), u1 = fmaf(y1[e], cs.x, -y0[e] * cs.y);
+                    y0[e] = u0;
+                    y1[e] = u1;
+                }
+            }
+        } else {
+#pragma unroll
+            for (int e = 0; e < VEC; ++e) { y0[e] = 0.f; y1[e] = 0.f; }
+        }
+        T* yr = Y + (size_t)tt * P.dt + cp * VEC;
+        *reinterpret_cast<uint4*>(yr) = Chunk<T>::pack(y0);
+        *reinterpret_cast<uint4*>(yr + ht) = Chunk<T>::pack(y1);
     }
 }
 
