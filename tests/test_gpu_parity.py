@@ -148,6 +148,27 @@ def test_translator_forms(name, path):
         assert g.tr.info().path == kvx.KVX_PATH_TCGEN05
 
 
+HEAD_DIMS = {
+    # source / target head dims other than 128: every instantiation of the tensor-core kernels
+    "ds64_dt64": (synth.ModelGeom(2, 4, 64, 1e4), synth.ModelGeom(2, 2, 64, 1e4)),
+    "ds256_dt128": (synth.ModelGeom(2, 2, 256, 1e4), synth.ModelGeom(2, 2, 128, 1e6)),
+    "ds256_dt256_expand": (synth.ModelGeom(2, 1, 256, 1e6), synth.ModelGeom(2, 2, 256, 1e4)),
+    "ds64_dt256": (synth.ModelGeom(3, 4, 64, 1e6), synth.ModelGeom(2, 1, 256, 1e4)),
+}
+
+
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+@pytest.mark.parametrize("spans", [False, True], ids=["identity", "spans"])
+@pytest.mark.parametrize("name", list(HEAD_DIMS))
+def test_head_dims(name, spans, path):
+    src, dst = HEAD_DIMS[name]
+    spec = synth.WorkloadSpec(name, src, dst, "bf16", [300], spans, None, True)
+    c = make_case(spec, [300, 77], pad_value=float("nan"))
+    g, _, _ = _full_compare(c, path)
+    if path == kvx.KVX_PATH_AUTO:
+        assert g.tr.info().path == kvx.KVX_PATH_TCGEN05
+
+
 def test_tiny_token_counts_and_empty_sequences():
     spec = _shrink(SPECS["qwen1p5b_to_gemma2b_1k"], 2, 2)
     c = make_case(spec, [1, 0, 2, 0, 129])
