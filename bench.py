@@ -447,9 +447,48 @@ def main():
         dist.destroy_process_group()
 
 
+def _oracle_fit_worker(args):
+    """Time the oracle's fit on a sub-problem: target layer 0, head 0 (K and V), the workload's
+    first n_tok target tokens.  Runs in a spawned process."""
+    name, n_tok = args
+    import dataclasses as dc
+    import oracle
+    spec = synth.config_specs()[name]
+    wl = synth.make_workload(spec, [n_tok])
+    lm = wl.layer_map if wl.layer_map is not None else oracle.layer_map_nearest(spec.src.num_layers,
+                                                                                spec.dst.num_layers)
+    lm = np.asarray(lm).reshape(spec.dst.num_layers, -1)[:1]
+    k = synth.source_kv(wl, int(lm.reshape(-1)[0]), 0)
+    v = synth.source_kv(wl, int(lm.reshape(-1)[0]), 1)
+    dst = dc.replace(spec.dst, num_layers=1, num_kv_heads=1)
+    src = spec.src if spec.src.num_kv_heads >= spec.dst.num_kv_heads else dc.replace(spec.src, num_kv_heads=1)
+    src = dc.replace(src, num_kv_heads=min(src.num_kv_heads, spec.heads_per_layer if spec.form else
+                                           max(1, spec.src.num_kv_heads // spec.dst.num_kv_heads)))
+    k, v = k[:, :src.num_kv_heads], v[:, :src.num_kv_heads]
+    ks, vs = [k] * spec.src.num_layers, [v] * spec.src.num_layers
+    rng = np.random.default_rng(0)
+    tk = [rng.standard_normal((1, 1, wl.t_max, dst.head_dim)).astype(np.float32)]
+    tv = [rng.standard_normal((1, 1, wl.t_max, dst.head_dim)).astype(np.float32)]
+    z = np.zeros((1, 1, spec.group_in, dst.head_dim), np.float32)
+    p = oracle.OracleProblem(src, dst, lm, wl.src_len, wl.tgt_seq_off, wl.s_max, wl.t_max, ks, vs, z, z,
+                             wl.span_lo, wl.span_hi, form=spec.form, k_layers=spec.layers_per_target)
+    t0 = time.perf_counter()
+    p.fit(tk, tv, 1e-3)
+    return time.perf_counter() - t0
+
+
 def fit_bench(args, spec):
     """Closed-form fit: calibration tokens/s of kvx_fit_accumulate (input rows, target rows, Gram
     sums) over the workload, plus one solve.  Inputs resident on the device."""
+    # the oracle's fit timed on the host cores (spawned before any CUDA call): one (layer, head)
+    # pair of systems per process over up to 4096 tokens, scaled to all groups
+    cores = os.cpu_count() or 1
+    n_tok = min(4096, int(sum(spec.tgt_lens)))
+    with mp.get_context("spawn").Pool(cores) as pool:
+        secs = pool.map(_oracle_fit_worker, [(args.workload, n_tok)] * cores)
+    groups_per_proc = 1   # one target layer, one head: a K and a V system
+    total_groups = spec.dst.num_layers * spec.dst.num_kv_heads
+    cpu_tok_s = n_tok * cores * groups_per_proc / max(secs) / total_groups
     import torch
     import paper_2608_30963_gb300 as kvx
     torch.cuda.set_device(0)
@@ -514,7 +553,11 @@ def fit_bench(args, spec):
                          "algorithmic_bytes": byts, "flops": flops, "roofline_ms": t_roof * 1e3,
                          "frac": t_roof * 1e3 / ms, "achieved_tflops": flops / (ms / 1e3) / 1e12,
                          "peaks": {"hbm_gbs": hbm, "bf16_tflops": tc}},
-            "solve_ms": solve_ms, "solve_status": bits}
+            "solve_ms": solve_ms, "solve_status": bits,
+            "cpu_baseline": {"value": cpu_tok_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                             "sample": f"oracle fit (fp64 Gram sums and Cholesky) of target layer 0, head 0, K and V "
+                                       f"over {n_tok} tokens in each of {cores} spawned processes, scaled by "
+                                       f"{total_groups} (layer, head) pairs"}}
     print(json.dumps(line), flush=True)
     f.close()
 
