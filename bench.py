@@ -348,35 +348,60 @@ def main():
 
     elapsed_ms, value = aggregate(elapsed_ms, wl.total_tgt, args.steps, world, dist, dev)
 
-    # end to end through the C ABI with host buffers: H2D source, translate, D2H target
+    # end to end through the C ABI with host buffers: every step copies its source caches in from
+    # pinned host memory, translates, and copies the target caches out.  Consecutive steps overlap
+    # on three streams (copy in, translate, copy out) over two device buffer sets and two host
+    # output sets, as a serving loop streaming handoffs would.
     e2e_steps = max(1, args.e2e_steps)
-    host_out = [torch.empty(out_shape, dtype=tdt).pin_memory() for _ in range(2 * Lt)]
-    src_k, src_v, dk, dv = sets[0]
+    host_out = [[torch.empty(out_shape, dtype=tdt).pin_memory() for _ in range(2 * Lt)] for _ in range(2)]
     h2d = sum(host_k[l].numel() * host_k[l].element_size() * 2 for l in mapped)
-    d2h = sum(t.numel() * t.element_size() for t in dk) * 2
+    d2h = sum(t.numel() * t.element_size() for t in sets[0][2]) * 2
+    s_in, s_tr, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
+    ev = lambda: torch.cuda.Event()
+    in_done, tr_done, out_done = [ev(), ev()], [ev(), ev()], [ev(), ev()]
+    used = [False, False]
 
-    def e2e_step():
-        for l in mapped:
-            src_k[l].copy_(host_k[l], non_blocking=True)
-            src_v[l].copy_(host_v[l], non_blocking=True)
+    def e2e_step(i):
+        k = i % 2
+        src_k, src_v, dk, dv = sets[k]
+        if used[k]:
+            s_in.wait_event(tr_done[k])       # the translate of step i-2 has read this source set
+            s_tr.wait_event(out_done[k])      # the copy-out of step i-2 has read this target set
+        with torch.cuda.stream(s_in):
+            for l in mapped:
+                src_k[l].copy_(host_k[l], non_blocking=True)
+                src_v[l].copy_(host_v[l], non_blocking=True)
+            in_done[k].record(s_in)
+        s_tr.wait_event(in_done[k])
         tr.translate(src_k, src_v, src_len, seq_off, wl.total_tgt, dk, dv, span_lo=span_lo, span_hi=span_hi,
-                     page_table=page_table, page_size=spec.page_size, num_pages=wl.num_pages, stream=stream)
-        for j in range(Lt):
-            host_out[j].copy_(dk[j], non_blocking=True)
-            host_out[Lt + j].copy_(dv[j], non_blocking=True)
+                     page_table=page_table, page_size=spec.page_size, num_pages=wl.num_pages, stream=s_tr)
+        tr_done[k].record(s_tr)
+        s_out.wait_event(tr_done[k])
+        with torch.cuda.stream(s_out):
+            for j in range(Lt):
+                host_out[k][j].copy_(dk[j], non_blocking=True)
+                host_out[k][Lt + j].copy_(dv[j], non_blocking=True)
+            out_done[k].record(s_out)
+        used[k] = True
 
-    e2e_step()
+    for s_ in (s_in, s_tr, s_out):
+        s_.wait_stream(stream)
+    e2e_step(0)
+    e2e_step(1)
     torch.cuda.synchronize()
     if dist:
         dist.barrier()
     a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    for _ in range(e2e_steps):
-        e2e_step()
-    b.record(stream)
+    a.record(s_in)
+    for i in range(e2e_steps):
+        e2e_step(i)
+    s_in.wait_stream(s_out)
+    b.record(s_in)
     torch.cuda.synchronize()
     e2e_ms = a.elapsed_time(b)
     e2e_ms, e2e_value = aggregate(e2e_ms, wl.total_tgt, e2e_steps, world, dist, dev)
+    if tr.device_status() != 0:
+        raise RuntimeError("device status nonzero after the end-to-end steps")
 
     if rank != 0:
         if dist:
@@ -432,7 +457,9 @@ def main():
                      "tensor_tflops": alg["flops"] / (avg_launch_ms / 1e3) / 1e12},
         "clocks": clk,
         "e2e": {"value": e2e_value, "unit": "tokens/s",
-                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / e2e_steps},
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / e2e_steps,
+                "how": "per step: H2D of the source caches from pinned memory, kvx_translate, D2H of the target "
+                       "caches; consecutive steps overlap on three streams over two buffer sets"},
         "gpu_launches": args.steps * tr.launches_per_translate(),
         "kernel_path": ({1: "simt", 2: "tcgen05"}.get(info.path, str(info.path)) +
                         ("+tma_identity" if info.path == 2 and span_lo is None else "")),

@@ -853,9 +853,8 @@ static cudaError_t launch_pdl(K kernel, int grid, int threads, size_t smem, cuda
 template <int DS>
 static cudaError_t launch_span_ds(int grid, cudaStream_t stream, const TranslateParams& P, const TcLaunch& L)
 {
-    static cudaError_t once =
-        cudaFuncSetAttribute(translate_tc_kernel<DS>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-    if (once != cudaSuccess) return once;
+    const cudaError_t e = smem_opt_in<translate_tc_kernel<DS>>(kSmemMax);
+    if (e != cudaSuccess) return e;
     return launch_pdl(translate_tc_kernel<DS>, grid, kThreads, kSmemMax, stream, P, L);
 }
 

@@ -725,22 +725,22 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     switch (T.ds) {
     case 64:
         {
-            static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<32>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-            if (once != cudaSuccess) return once;
+            const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<32>>(kSmemMax);
+            if (e != cudaSuccess) return e;
         }
         return launch_pdl(translate_tc_aligned_kernel<32>, grid, stream, P);
         break;
     case 128:
         {
-            static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-            if (once != cudaSuccess) return once;
+            const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<64>>(kSmemMax);
+            if (e != cudaSuccess) return e;
         }
         return launch_pdl(translate_tc_aligned_kernel<64>, grid, stream, P);
         break;
     case 256:
         {
-            static cudaError_t once = cudaFuncSetAttribute(translate_tc_aligned_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemMax);
-            if (once != cudaSuccess) return once;
+            const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<128>>(kSmemMax);
+            if (e != cudaSuccess) return e;
         }
         return launch_pdl(translate_tc_aligned_kernel<128>, grid, stream, P);
         break;

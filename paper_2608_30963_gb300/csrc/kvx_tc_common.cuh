@@ -3,12 +3,30 @@
 // UMMA shared-memory descriptor, bounded waits and bf16 packing.
 #pragma once
 
+#include <atomic>
+
 #include "kvx_common.cuh"
 
 namespace kvx {
 namespace {
 
 constexpr int kSmemMax = 232448;                      // 227 KB opt-in shared memory per block
+
+// Dynamic shared memory above 48 KB is a per-device opt-in of each kernel: set it the first time
+// the kernel is launched on each device (devices 0..63; others set it on every launch).
+template <auto Kernel>
+cudaError_t smem_opt_in(int bytes)
+{
+    static std::atomic<unsigned long long> done{0};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const unsigned long long bit = dev >= 0 && dev < 64 ? 1ull << dev : 0ull;
+    if (bit && (done.load(std::memory_order_acquire) & bit)) return cudaSuccess;
+    e = cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && bit) done.fetch_or(bit, std::memory_order_release);
+    return e;
+}
 constexpr unsigned long long kWaitNs = 1000000000ull;   // bound of every on-chip wait (~1 s)
 
 // ------------------------------------------------------------------ PTX wrappers
