@@ -280,7 +280,7 @@ KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
  * the rotation is orthogonal, so the distance is unchanged) or as stored (V).
  * The fitter accumulates X^T X and X^T Y over any number of calibration calls (fp32, on the
  * tensor cores through cuBLAS batched GEMMs over the groups), then solves all systems at once
- * (Cholesky factorisation in double on the device).  Forms as for kvx_translator_create;
+ * (Cholesky factorisation on the device: in fp32 shared memory for in <= 256, in double above).  Forms as for kvx_translator_create;
  * latent adapters are not fitted (fit W, then factor it if wanted). */
 typedef struct kvx_fitter kvx_fitter;
 

@@ -12,8 +12,9 @@
 //      (HBM-bound gather, CUDA cores);
 //   2. two strided-batched cuBLAS GEMMs over the groups add X^T X and X^T Y into fp32 sums
 //      (a plain dense contraction over tokens: tensor cores through the library);
-//   3. at solve time, fit_solve_kernel (one CTA per group) factors X^T X + lambda I = L L^T in
-//      double and runs the two triangular solves per output column.
+//   3. at solve time, one CTA per group factors X^T X + lambda I = L L^T and runs the two
+//      triangular solves per output column: fit_solve_small_kernel in fp32 shared memory for
+//      in <= 256, fit_solve_kernel in double global memory above.
 #include <cublas_v2.h>
 #include <math.h>
 #include <stdarg.h>
@@ -226,6 +227,105 @@ __global__ void __launch_bounds__(kSolveThreads) fit_solve_kernel(const float* _
     if (bad && threadIdx.x == 0) set_status(status, kFitNotPosDef);
 }
 
+// in <= kSmallSolve: the factor lives in shared memory as fp32, packed lower triangle (row r at
+// r(r+1)/2), followed by `cols` columns of solutions [in][cols].  The sums X^T X are fp32 already,
+// so a float factorisation loses nothing against them; it removes the L2 round trips of the
+// double, global-memory kernel above.  One CTA per group.
+constexpr int kSmallSolve = 256;
+constexpr int kSmallSolveThreads = 512;
+constexpr int kSmallSolveSmem = 227 * 1024 - 2048;   // dynamic shared memory budget
+
+template <typename T>
+__global__ void __launch_bounds__(kSmallSolveThreads) fit_solve_small_kernel(const float* __restrict__ G,
+                                                                             const float* __restrict__ C, T* wk,
+                                                                             T* wv, int in, int dt, int cols,
+                                                                             float lambda, unsigned* status)
+{
+    extern __shared__ float Lp[];          // packed lower triangle, then the solution block
+    __shared__ float colk[kSmallSolve];    // column k of L below the diagonal
+    __shared__ int bad;
+    const int g = blockIdx.x;
+    const float* gg = G + (size_t)g * in * in;
+    const float* cc = C + (size_t)g * in * dt;
+    auto at = [](int r, int c) { return r * (r + 1) / 2 + c; };
+    float* zs = Lp + at(in, 0);            // [in][cols]
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nwarps = blockDim.x >> 5;
+    if (threadIdx.x == 0) bad = 0;
+    for (int r = warp; r < in; r += nwarps)
+        for (int c = lane; c <= r; c += 32) Lp[at(r, c)] = gg[(size_t)r * in + c] + (r == c ? lambda : 0.f);
+    __syncthreads();
+    // right-looking Cholesky: Lp = L with L L^T = X^T X + lambda I
+    for (int k = 0; k < in; ++k) {
+        if (threadIdx.x == 0) {
+            float d = Lp[at(k, k)];
+            if (!(d > 0.f)) { bad = 1; d = 1.f; }
+            Lp[at(k, k)] = sqrtf(d);
+        }
+        __syncthreads();
+        const float dk = Lp[at(k, k)];
+        for (int r = k + 1 + threadIdx.x; r < in; r += blockDim.x) {
+            const float v = Lp[at(r, k)] / dk;
+            Lp[at(r, k)] = v;
+            colk[r] = v;
+        }
+        __syncthreads();
+        for (int r = k + 1 + warp; r < in; r += nwarps) {
+            const float lr = colk[r];
+            for (int c = k + 1 + lane; c <= r; c += 32) Lp[at(r, c)] -= lr * colk[c];
+        }
+        __syncthreads();
+    }
+    T* w = (g & 1) ? wv : wk;
+    const size_t off = (size_t)(g >> 1) * in * dt;
+    for (int o0 = 0; o0 < dt; o0 += cols) {
+        const int nc = min(cols, dt - o0);
+        // one thread per output column: L u = c, then L^T w = u, four independent partial sums
+        for (int o = threadIdx.x; o < nc; o += blockDim.x) {
+            for (int r = 0; r < in; ++r) {
+                const float* lr = Lp + at(r, 0);
+                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+                int k = 0;
+                for (; k + 3 < r; k += 4) {
+                    s0 = fmaf(lr[k], zs[(k + 0) * cols + o], s0);
+                    s1 = fmaf(lr[k + 1], zs[(k + 1) * cols + o], s1);
+                    s2 = fmaf(lr[k + 2], zs[(k + 2) * cols + o], s2);
+                    s3 = fmaf(lr[k + 3], zs[(k + 3) * cols + o], s3);
+                }
+                for (; k < r; ++k) s0 = fmaf(lr[k], zs[k * cols + o], s0);
+                zs[r * cols + o] = (cc[(size_t)(o0 + o) * in + r] - ((s0 + s1) + (s2 + s3))) / lr[r];
+            }
+            for (int r = in - 1; r >= 0; --r) {
+                float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
+                int k = r + 1;
+                for (; k + 3 < in; k += 4) {
+                    s0 = fmaf(Lp[at(k, r)], zs[k * cols + o], s0);
+                    s1 = fmaf(Lp[at(k + 1, r)], zs[(k + 1) * cols + o], s1);
+                    s2 = fmaf(Lp[at(k + 2, r)], zs[(k + 2) * cols + o], s2);
+                    s3 = fmaf(Lp[at(k + 3, r)], zs[(k + 3) * cols + o], s3);
+                }
+                for (; k < in; ++k) s0 = fmaf(Lp[at(k, r)], zs[k * cols + o], s0);
+                zs[r * cols + o] = (zs[r * cols + o] - ((s0 + s1) + (s2 + s3))) / Lp[at(r, r)];
+            }
+        }
+        __syncthreads();
+        for (int i = threadIdx.x; i < in * nc; i += blockDim.x) {
+            const int r = i / nc, o = i - r * nc;
+            w[off + (size_t)r * dt + o0 + o] = from_f32<T>(bad ? 0.f : zs[r * cols + o]);
+        }
+        __syncthreads();
+    }
+    if (bad && threadIdx.x == 0) set_status(status, kFitNotPosDef);
+}
+
+// solution columns per block for the small solve, and its dynamic shared memory
+int small_solve_cols(int in, int dt)
+{
+    const int tri = in * (in + 1) / 2;
+    const int cols = (kSmallSolveSmem / 4 - tri) / in;
+    return cols < dt ? cols : dt;
+}
+size_t small_solve_smem(int in, int cols) { return ((size_t)in * (in + 1) / 2 + (size_t)in * cols) * sizeof(float); }
+
 }  // namespace
 }  // namespace kvx
 
@@ -385,7 +485,7 @@ extern "C" KVX_API kvx_status kvx_fit_solve(kvx_fitter* f, void* w_k, void* w_v,
     cudaStream_t s = (cudaStream_t)stream;
     // double scratch for the factorisation and the solutions: the row workspace is reused when it is
     // large enough, otherwise a temporary allocation (solve is not on the translation path)
-    const size_t need = (size_t)f->groups * in * (in + dt) * sizeof(double);
+    const size_t need = in <= kSmallSolve ? 0 : (size_t)f->groups * in * (in + dt) * sizeof(double);
     const size_t have = (size_t)f->groups * f->chunk * (in + dt) * fit_elt(f);
     double* scratch = nullptr;
     bool own = false;
@@ -400,7 +500,26 @@ extern "C" KVX_API kvx_status kvx_fit_solve(kvx_fitter* f, void* w_k, void* w_v,
     double* Z = scratch + (size_t)f->groups * in * in;
     const float* G = f->sums;
     const float* C = f->sums + (size_t)f->groups * in * in;
-    if (D.dtype == KVX_BF16)
+    if (in <= kSmallSolve) {
+        // fp32 factor and a block of solution columns in shared memory
+        const int cols = small_solve_cols(in, dt);
+        const int smem = (int)small_solve_smem(in, cols);
+        if (D.dtype == KVX_BF16) {
+            ce = cudaFuncSetAttribute(fit_solve_small_kernel<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+            if (ce == cudaSuccess)
+                fit_solve_small_kernel<__nv_bfloat16><<<f->groups, kSmallSolveThreads, smem, s>>>(
+                    G, C, (__nv_bfloat16*)w_k, (__nv_bfloat16*)w_v, in, dt, cols, (float)f->lambda, f->status);
+        } else {
+            ce = cudaFuncSetAttribute(fit_solve_small_kernel<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+            if (ce == cudaSuccess)
+                fit_solve_small_kernel<float><<<f->groups, kSmallSolveThreads, smem, s>>>(
+                    G, C, (float*)w_k, (float*)w_v, in, dt, cols, (float)f->lambda, f->status);
+        }
+        if (ce != cudaSuccess) {
+            if (own) cudaFree(scratch);
+            return fit_fail(KVX_ERR_CUDA, "fit_solve: %s", cudaGetErrorString(ce));
+        }
+    } else if (D.dtype == KVX_BF16)
         fit_solve_kernel<__nv_bfloat16><<<f->groups, kSolveThreads, 0, s>>>(G, C, A, Z, (__nv_bfloat16*)w_k,
                                                                             (__nv_bfloat16*)w_v, in, dt, f->lambda,
                                                                             f->status);
