@@ -413,8 +413,8 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
             tc_fence_after();
             // the staging row is shared by the two warps of this quadrant; the row's
-            // previous store (issued by the half-0 thread) must have read it
-            if (half == 0) bulk_wait_read0();
+            // previous store (issued by the thread of lane parity = half) must have read it
+            bulk_wait_read0();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2));
             if (!W.wait(bar(kBarPair + quad * 2), tcount & 1)) break;
@@ -466,7 +466,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2 + 1));
             if (!W.wait(bar(kBarPair + quad * 2 + 1), tcount & 1)) break;
-            if (half == 0 && valid && dst_off >= 0) {
+            if ((lane & 1) == half && valid && dst_off >= 0) {   // the quadrant's rows, split between its two warps
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      (P.paged ? (long long)x.h * P.dt : (long long)x.h * P.dh);
                 if (P.n_split == 1) {
