@@ -461,3 +461,26 @@ def test_two_translators_on_two_streams():
         np.testing.assert_array_equal(gk, rk)
         np.testing.assert_array_equal(gv, rv)
         assert g.status() == 0
+
+
+# ------------------------------------------------------------------ limits of the fast paths
+@pytest.mark.parametrize("batch", [300, 600])
+def test_large_batches(batch):
+    """More sequences than the identity kernel keeps on chip (256), and than the span kernel
+    caches in shared memory (512): both fall back to their general paths, same results."""
+    rng = np.random.default_rng(batch)
+    lens = [int(x) for x in rng.integers(1, 24, size=batch)]
+    for base in ("qwen7b_to_qwen1p5b_4k", "qwen1p5b_to_gemma2b_1k"):
+        spec = _shrink(SPECS[base], 2, 2)
+        c = make_case(spec, lens)
+        g, _, _ = _full_compare(c, kvx.KVX_PATH_AUTO)
+        assert g.tr.info().path == kvx.KVX_PATH_TCGEN05
+
+
+def test_more_target_layers_than_the_identity_kernel_takes():
+    """100 target layers (above the identity kernel's 96): the span kernel serves identity
+    alignment too."""
+    spec = synth.WorkloadSpec("deep", synth.ModelGeom(120, 2, 64, 1e4), synth.ModelGeom(100, 1, 64, 1e6), "bf16",
+                              [40], False, None, False)
+    c = make_case(spec, [40, 17])
+    _full_compare(c, kvx.KVX_PATH_AUTO)
