@@ -276,6 +276,15 @@ def main():
     src_len, seq_off = i32(wl.src_len), i32(wl.tgt_seq_off)
     span_lo, span_hi = i32(wl.span_lo), i32(wl.span_hi)
     page_table = i32(wl.page_table) if spec.paged else None
+    # cross-tokenizer workloads: every step first builds the token-span alignment on the device
+    # from the two tokenisations' byte offsets (kvx_build_alignment), then translates with it
+    align = None
+    if spec.cross_tokenizer:
+        align = dict(src_seq_off=i32(wl.src_seq_off), src_end=i32(wl.src_end), tgt_seq_off=seq_off,
+                     tgt_end=i32(wl.tgt_end), span_lo=torch.empty_like(span_lo), span_hi=torch.empty_like(span_hi))
+        span_lo, span_hi = align["span_lo"], align["span_hi"]
+        # the builder reads both byte-offset arrays and the sequence offsets, writes two span arrays
+        alg["bytes"] += 4 * (int(wl.src_end.size) + 3 * int(wl.tgt_end.size) + 2 * (wl.batch + 1))
     Lt, Ht, dt = spec.dst.num_layers, spec.dst.num_kv_heads, spec.dst.head_dim
     out_shape = (wl.num_pages, spec.page_size, Ht, dt) if spec.paged else (wl.batch, Ht, wl.t_max, dt)
 
@@ -294,8 +303,14 @@ def main():
         sets.append((src_k, src_v, dk, dv))
     stream = torch.cuda.current_stream()
 
+    def build_spans(stream_=None):
+        if align is not None:
+            kvx.build_alignment(align["src_seq_off"], align["src_end"], align["tgt_seq_off"], align["tgt_end"],
+                                align["span_lo"], align["span_hi"], stream=stream_)
+
     def step(i):
         src_k, src_v, dk, dv = sets[i % nsets]
+        build_spans()
         tr.translate(src_k, src_v, src_len, seq_off, wl.total_tgt, dk, dv, span_lo=span_lo, span_hi=span_hi,
                      page_table=page_table, page_size=spec.page_size, num_pages=wl.num_pages, stream=None)
 
@@ -333,7 +348,7 @@ def main():
     if dist:
         dist.barrier()
     elapsed_ms = t_start.elapsed_time(t_end)
-    launch_ms = [elapsed_ms / args.steps]   # one kernel per step, launched back to back
+    launch_ms = [elapsed_ms / args.steps]   # one step's launches, back to back
 
     # keep the GPU loaded long enough for the clock sampler to see it (>= 1 s)
     extra = 0
@@ -355,6 +370,11 @@ def main():
     e2e_steps = max(1, args.e2e_steps)
     host_out = [[torch.empty(out_shape, dtype=tdt).pin_memory() for _ in range(2 * Lt)] for _ in range(2)]
     h2d = sum(host_k[l].numel() * host_k[l].element_size() * 2 for l in mapped)
+    host_ends = None
+    if align is not None:   # the two tokenisations' byte offsets are inputs of every step too
+        host_ends = (torch.from_numpy(np.ascontiguousarray(wl.src_end, np.int32)).pin_memory(),
+                     torch.from_numpy(np.ascontiguousarray(wl.tgt_end, np.int32)).pin_memory())
+        h2d += 4 * (int(wl.src_end.size) + int(wl.tgt_end.size))
     d2h = sum(t.numel() * t.element_size() for t in sets[0][2]) * 2
     s_in, s_tr, s_out = torch.cuda.Stream(), torch.cuda.Stream(), torch.cuda.Stream()
     ev = lambda: torch.cuda.Event()
@@ -371,8 +391,12 @@ def main():
             for l in mapped:
                 src_k[l].copy_(host_k[l], non_blocking=True)
                 src_v[l].copy_(host_v[l], non_blocking=True)
+            if host_ends is not None:   # one device copy of the offsets: every step writes the same values
+                align["src_end"].copy_(host_ends[0], non_blocking=True)
+                align["tgt_end"].copy_(host_ends[1], non_blocking=True)
             in_done[k].record(s_in)
         s_tr.wait_event(in_done[k])
+        build_spans(s_tr)
         tr.translate(src_k, src_v, src_len, seq_off, wl.total_tgt, dk, dv, span_lo=span_lo, span_hi=span_hi,
                      page_table=page_table, page_size=spec.page_size, num_pages=wl.num_pages, stream=s_tr)
         tr_done[k].record(s_tr)
@@ -423,7 +447,7 @@ def main():
     traffic = None
     try:
         tr_info = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))
-        if tr_info.get("workload") == args.workload and tr_info.get("kernel_rev") == kernel_rev():
+        if tr_info.get("workload") == args.workload and tr_info.get("kernel_rev") == kernel_rev(tr_info.get("sources")):
             traffic = tr_info.get("dram_bytes_per_launch")
     except Exception:
         pass
@@ -448,6 +472,8 @@ def main():
                    "l2": f"inputs larger than L2: {nsets} rotating input/output sets of {set_bytes / 1e6:.1f} MB "
                          f"(L2 129 MB)",
                    "parallelism": f"replicas{world}" if world > 1 else "single",
+                   "step": ("kvx_build_alignment (byte offsets -> spans) + kvx_translate" if align is not None
+                            else "kvx_translate (same tokenizer: identity alignment)"),
                    "timing": "the K steps as one CUDA graph (programmatic dependent launch between steps); "
                              "CUDA events around it"},
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
@@ -458,9 +484,13 @@ def main():
         "clocks": clk,
         "e2e": {"value": e2e_value, "unit": "tokens/s",
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": e2e_ms / e2e_steps,
-                "how": "per step: H2D of the source caches from pinned memory, kvx_translate, D2H of the target "
-                       "caches; consecutive steps overlap on three streams over two buffer sets"},
-        "gpu_launches": args.steps * tr.launches_per_translate(),
+                "how": ("per step: H2D of the source caches " +
+                        ("and both tokenisations' byte offsets " if align is not None else "") +
+                        "from pinned memory, " +
+                        ("kvx_build_alignment, " if align is not None else "") +
+                        "kvx_translate, D2H of the target caches; consecutive steps overlap on three streams "
+                        "over two buffer sets")},
+        "gpu_launches": args.steps * (tr.launches_per_translate() + (1 if align is not None else 0)),
         "kernel_path": ({1: "simt", 2: "tcgen05"}.get(info.path, str(info.path)) +
                         ("+tma_identity" if info.path == 2 and span_lo is None else "")),
         "num_sms": info.num_sms,
@@ -589,14 +619,18 @@ def fit_bench(args, spec):
     f.close()
 
 
-def kernel_rev() -> str:
-    """Hash of the kernel sources, so a stored ncu traffic figure is only used for the kernel it measured."""
+def kernel_rev(sources=None) -> str:
+    """Hash of the sources a kernel is compiled from (its translation unit and the headers it
+    includes, paths relative to the repository root; all kernel sources when None), so a stored
+    ncu traffic figure is only used for the kernel it measured."""
     import hashlib
     h = hashlib.sha1()
-    csrc = os.path.join(ROOT, "paper_2608_30963_gb300", "csrc")
-    for f in sorted(os.listdir(csrc)):
-        if f.endswith((".cu", ".cuh", ".h")):
-            h.update(open(os.path.join(csrc, f), "rb").read())
+    if sources is None:
+        csrc = os.path.join("paper_2608_30963_gb300", "csrc")
+        sources = [os.path.join(csrc, f) for f in sorted(os.listdir(os.path.join(ROOT, csrc)))
+                   if f.endswith((".cu", ".cuh", ".h"))]
+    for f in sources:
+        h.update(open(os.path.join(ROOT, f), "rb").read())
     return h.hexdigest()[:12]
 
 

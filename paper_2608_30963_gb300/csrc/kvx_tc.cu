@@ -94,6 +94,7 @@ struct TcLaunch {
     unsigned hb_bytes; // one A head-block: 128 rows x d_s bf16
     unsigned cap_rows; // most source rows one window may stage
     int n_slots;       // window slots of slot_bytes each
+    int share;         // target heads that read the same source rows, walked by interleaved CTA sets (1 = off)
     int n_b;           // B slots: 1 = the group's image stays resident across its tiles;
                        // 2 = streamed, one piece (one source head's rows of W) per head-block
     unsigned b_bytes;  // one group's whole B image (in x n_tile bf16)
@@ -110,10 +111,15 @@ struct Unit {
 };
 // The CTA's units: an equal share of the K units, then of the V units (each share
 // group-major, so a group's weights stay resident), walked with counters only.
+// When `share` > 1 target heads read the same source rows (the `share` heads of a GQA
+// expansion group, or every head in the dense form), the CTAs form `share` interleaved
+// sets: set i walks head i of every group, and CTA k of each set takes the k-th share of
+// the same (layer, head group, tile) sequence.  The partners' reads of a window then come
+// at about the same time, so the second one hits L2 instead of going back to DRAM.
 struct Walker {
     int count, nK, it;
     int kv, j, h, nt, tile;
-    int u0, v0, m_tiles, n_split, Ht;
+    int u0, v0, m_tiles, n_split, Ht, E, hk, hv;
     Unit x;
     __device__ __forceinline__ void fill()
     {
@@ -126,20 +132,24 @@ struct Walker {
         const int hg = idx / m_tiles;
         tile = idx - hg * m_tiles;
         nt = hg % n_split;
-        const int jh = hg / n_split;
-        h = jh % Ht;
-        j = jh / Ht;
+        const int jq = hg / n_split;
+        const int HtE = Ht / E;
+        h = (jq % HtE) * E + (kv ? hv : hk);
+        j = jq / HtE;
         fill();
     }
     __device__ __forceinline__ void start(const TcLaunch& L, int Ht_)
     {
-        m_tiles = L.m_tiles; n_split = L.n_split; Ht = Ht_;
-        const long long UH = (long long)(L.groups / 2) * L.m_tiles;
-        const int G = gridDim.x, c = blockIdx.x, vr = G - 1 - c;
+        m_tiles = L.m_tiles; n_split = L.n_split; Ht = Ht_; E = L.share;
+        const long long UH = (long long)(L.groups / 2) * L.m_tiles / E;   // units of one head set
+        const int G = gridDim.x / E, c = blockIdx.x / E, vr = gridDim.x - 1 - (int)blockIdx.x;
+        hk = (int)blockIdx.x % E;
+        hv = vr % E;
+        const int cv = vr / E;
         u0 = (int)((long long)c * UH / G);
         const int u1 = (int)((long long)(c + 1) * UH / G);
-        v0 = (int)((long long)vr * UH / G);
-        const int v1 = (int)((long long)(vr + 1) * UH / G);
+        v0 = (int)((long long)cv * UH / G);
+        const int v1 = (int)((long long)(cv + 1) * UH / G);
         nK = u1 - u0;
         count = nK + (v1 - v0);
         it = 0;
@@ -155,7 +165,7 @@ struct Walker {
             tile = 0;
             if (++nt == n_split) {
                 nt = 0;
-                if (++h == Ht) { h = 0; ++j; }
+                if ((h += E) >= Ht) { h = kv ? hv : hk; ++j; }
             }
         }
         fill();
@@ -891,6 +901,9 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
         ++*launches;
         const long long UH = (long long)(L.groups / 2) * L.m_tiles;
         const int grid = (int)(UH < num_sms ? UH : num_sms);
+        // heads that share source rows: a GQA expansion group, or all heads of the dense form
+        const int E = P.dense ? P.Ht : (P.r == 1 ? P.e : 1);
+        L.share = E > 1 && P.Ht % E == 0 && grid % E == 0 ? E : 1;
         switch (P.ds) {
         case 256: e = launch_span_ds<256>(grid, stream, P, L); break;
         case 128: e = launch_span_ds<128>(grid, stream, P, L); break;
