@@ -37,18 +37,19 @@ def build(force: bool = False) -> str:
 
 class RopeSched(ctypes.Structure):
     _fields_ = [("base", ctypes.c_double), ("type", ctypes.c_int32), ("factor", ctypes.c_double),
-                ("low", ctypes.c_double), ("high", ctypes.c_double), ("orig_ctx", ctypes.c_int32)]
+                ("low", ctypes.c_double), ("high", ctypes.c_double), ("orig_ctx", ctypes.c_int32),
+                ("rot", ctypes.c_int32)]
 
 
 def rope_sched(g=None, base: Optional[float] = None) -> RopeSched:
     """The rotary schedule of a geometry object (attributes rope_base, rope_type, rope_factor,
-    rope_low_freq_factor, rope_high_freq_factor, rope_original_max_position; missing ones mean
-    the plain schedule), or the plain schedule of `base`."""
+    rope_low_freq_factor, rope_high_freq_factor, rope_original_max_position, rotary_dim; missing
+    ones mean the plain schedule over the whole head), or the plain schedule of `base`."""
     if g is None:
-        return RopeSched(float(base), 0, 1.0, 1.0, 1.0, 1)
+        return RopeSched(float(base), 0, 1.0, 1.0, 1.0, 1, 0)
     return RopeSched(float(g.rope_base), int(getattr(g, "rope_type", 0)), float(getattr(g, "rope_factor", 1.0)),
                      float(getattr(g, "rope_low_freq_factor", 1.0)), float(getattr(g, "rope_high_freq_factor", 4.0)),
-                     int(getattr(g, "rope_original_max_position", 8192)))
+                     int(getattr(g, "rope_original_max_position", 8192)), int(getattr(g, "rotary_dim", 0)))
 
 
 class Problem(ctypes.Structure):

@@ -121,6 +121,7 @@ typedef struct {
     int32_t type;
     double factor, low, high;
     int32_t orig_ctx;
+    int32_t rot;          /* channels that rotate (partial rotary: the first rot); 0 = all d */
 } kvxo_rope_sched;
 
 static double kvxo_theta(const kvxo_rope_sched* r, int i, int d)
@@ -139,15 +140,19 @@ static double kvxo_theta(const kvxo_rope_sched* r, int i, int d)
     return theta;
 }
 
-/* Half-split rotary map on one head vector of length d (d even):
- * x'[i] = x[i] cos a - x[i+d/2] sin a,  x'[i+d/2] = x[i+d/2] cos a + x[i] sin a,
- * a = sign * pos * theta_i.  sign = +1 applies the RoPE, -1 undoes it. */
+/* Half-split rotary map on one head vector of length d (d even).  With n rotated
+ * channels (n = r->rot, or d when 0; a partial rotary head rotates only its first
+ * n channels and passes the rest through) and h = n/2:
+ * x'[i] = x[i] cos a - x[i+h] sin a,  x'[i+h] = x[i+h] cos a + x[i] sin a  (i < h),
+ * a = sign * pos * theta_i, theta_i taken over the n rotated channels (base^(-2i/n)).
+ * sign = +1 applies the RoPE, -1 undoes it. */
 KVXO_API void kvxo_rope_sched_apply(double* x, int d, const kvxo_rope_sched* r, double pos, int sign)
 {
     if (r->base <= 0.0) return;
-    int h = d / 2;
+    int n = r->rot > 0 ? r->rot : d;
+    int h = n / 2;
     for (int i = 0; i < h; ++i) {
-        double a = (double)sign * pos * kvxo_theta(r, i, d);
+        double a = (double)sign * pos * kvxo_theta(r, i, n);
         double c = cos(a), sn = sin(a);
         double x0 = x[i], x1 = x[i + h];
         x[i]     = x0 * c - x1 * sn;
@@ -158,7 +163,7 @@ KVXO_API void kvxo_rope_sched_apply(double* x, int d, const kvxo_rope_sched* r, 
 /* The plain schedule (type 0) with the given base. */
 KVXO_API void kvxo_rope(double* x, int d, double base, double pos, int sign)
 {
-    kvxo_rope_sched r = {base, 0, 1.0, 1.0, 1.0, 1};
+    kvxo_rope_sched r = {base, 0, 1.0, 1.0, 1.0, 1, 0};
     kvxo_rope_sched_apply(x, d, &r, pos, sign);
 }
 

@@ -67,6 +67,7 @@ class ModelGeom:
     rope_low_freq_factor: float = 1.0
     rope_high_freq_factor: float = 4.0
     rope_original_max_position: int = 8192
+    rotary_dim: int = 0   # partial rotary: only the first rotary_dim channels rotate; 0 = all
 
 
 @dataclasses.dataclass

@@ -235,6 +235,65 @@ def test_scheduled_translation_undoes_and_reapplies_the_schedule():
         np.testing.assert_allclose(ok2[0, 0, t], oracle.rope(raw, 5e5, t, +1), atol=1e-6)
 
 
+# ------------------------------------------------------- partial rotary heads
+def test_partial_rotary_over_the_whole_head_is_the_plain_map():
+    rng = np.random.default_rng(31)
+    x = rng.standard_normal(128)
+    for kw in ({}, dict(rope_type=synth.ROPE_LINEAR, rope_factor=4.0)):
+        full = oracle.rope_g(x, synth.ModelGeom(1, 1, 128, 1e4, **kw), 321.0, +1)
+        same = oracle.rope_g(x, synth.ModelGeom(1, 1, 128, 1e4, rotary_dim=128, **kw), 321.0, +1)
+        np.testing.assert_array_equal(full, same)
+
+
+def test_partial_rotary_is_a_plain_head_of_the_rotated_width_and_passes_the_rest():
+    # A head of d channels rotating its first n: the first n channels are the plain map of an
+    # n-channel head (pairs (i, i + n/2), frequencies over n), the others are untouched.
+    rng = np.random.default_rng(32)
+    for d, n in ((128, 32), (128, 64), (128, 96), (256, 64), (64, 16)):
+        x = rng.standard_normal(d)
+        for kw in ({}, dict(rope_type=synth.ROPE_LINEAR, rope_factor=8.0)):
+            gp = synth.ModelGeom(1, 1, d, 1e4, rotary_dim=n, **kw)
+            gn = synth.ModelGeom(1, 1, n, 1e4, **kw)
+            for pos in (0.0, 5.0, 4095.0):
+                y = oracle.rope_g(x, gp, pos, +1)
+                np.testing.assert_array_equal(y[:n], oracle.rope_g(x[:n], gn, pos, +1))
+                np.testing.assert_array_equal(y[n:], x[n:])
+                np.testing.assert_allclose(oracle.rope_g(y, gp, pos, -1), x, atol=1e-12)
+
+
+def test_partial_rotary_pairs_and_frequency_closed_form():
+    # d = 96 with 24 rotated channels (a quarter of the head): channel 1 pairs with channel 13
+    # (1 + 24/2, not 1 + 96/2) and turns by theta_1 = base^(-2/24); at position base^(1/12)
+    # the angle is exactly 1 rad.
+    g = synth.ModelGeom(1, 1, 96, 1e4, rotary_dim=24)
+    x = np.zeros(96)
+    x[1] = 1.0
+    y = oracle.rope_g(x, g, 1e4 ** (1.0 / 12.0), +1)
+    want = np.zeros(96)
+    want[1], want[13] = np.cos(1.0), np.sin(1.0)
+    np.testing.assert_allclose(y, want, atol=1e-13)
+
+
+def test_partial_rotary_translation_round_trip_and_mixed_heads():
+    # Same partial-rotary geometry on both sides, W = I, identity alignment: the stored keys come
+    # back.  A fully rotating target instead gets the plain rotation of the un-rotated keys.
+    rng = np.random.default_rng(33)
+    g = synth.ModelGeom(1, 1, 128, 1e4, rotary_dim=64)
+    S = 29
+    k = oracle.rope_cache(rng.standard_normal((1, 1, S, 128)).astype(np.float32), g)
+    v = rng.standard_normal((1, 1, S, 128)).astype(np.float32)
+    W = np.eye(128, dtype=np.float32)[None, None]
+    ok, ov = oracle.OracleProblem(g, g, [0], [S], [0, S], S, S, [k], [v], W, W).translate()
+    np.testing.assert_allclose(ok[0, 0], k[0, 0], atol=1e-6)
+    np.testing.assert_array_equal(ov[0, 0], v[0, 0])
+    gf = synth.ModelGeom(1, 1, 128, 1e6)
+    ok2, _ = oracle.OracleProblem(g, gf, [0], [S], [0, S], S, S, [k], [v], W, W).translate()
+    for t in (0, 9, 28):
+        raw = oracle.rope_g(k[0, 0, t].astype(np.float64), g, t, -1)
+        np.testing.assert_array_equal(raw[64:], k[0, 0, t, 64:])          # the tail never rotated
+        np.testing.assert_allclose(ok2[0, 0, t], oracle.rope(raw, 1e6, t, +1), atol=1e-6)
+
+
 # ------------------------------------------------------------ translation
 def _geom(L, H, d, base):
     return synth.ModelGeom(L, H, d, base)
