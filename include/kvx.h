@@ -100,6 +100,11 @@ typedef struct {
     double  rope_low_freq_factor;       /* LLAMA3: > 0 */
     double  rope_high_freq_factor;      /* LLAMA3: > rope_low_freq_factor */
     int32_t rope_original_max_position; /* LLAMA3: context length of the unscaled model, > 0 */
+    int32_t rotary_dim;         /* partial rotary heads: only the first rotary_dim channels of K
+                                   rotate, as pairs (i, i + rotary_dim/2) with frequencies
+                                   base^(-2i/rotary_dim) under the schedule; the other channels
+                                   carry no position.  0 = head_dim (the whole head rotates);
+                                   else a multiple of 16 in [16, head_dim]. */
 } kvx_model_geom;
 
 /* Which source KV heads feed one target KV head.  Section 5 lists the granularities a

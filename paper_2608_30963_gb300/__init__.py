@@ -40,17 +40,18 @@ class kvx_model_geom(ctypes.Structure):
                 ("head_dim", ctypes.c_int32), ("rope_base", ctypes.c_double),
                 ("rope_type", ctypes.c_int32), ("rope_factor", ctypes.c_double),
                 ("rope_low_freq_factor", ctypes.c_double), ("rope_high_freq_factor", ctypes.c_double),
-                ("rope_original_max_position", ctypes.c_int32)]
+                ("rope_original_max_position", ctypes.c_int32), ("rotary_dim", ctypes.c_int32)]
 
 
 def model_geom(g) -> kvx_model_geom:
-    """kvx_model_geom from any object with the same attribute names (the RoPE schedule
-    attributes are optional and default to the plain schedule)."""
+    """kvx_model_geom from any object with the same attribute names (the RoPE schedule and
+    rotary_dim attributes are optional and default to the plain schedule over the whole head)."""
     return kvx_model_geom(g.num_layers, g.num_kv_heads, g.head_dim, g.rope_base,
                           int(getattr(g, "rope_type", 0)), float(getattr(g, "rope_factor", 1.0)),
                           float(getattr(g, "rope_low_freq_factor", 1.0)),
                           float(getattr(g, "rope_high_freq_factor", 4.0)),
-                          int(getattr(g, "rope_original_max_position", 8192)))
+                          int(getattr(g, "rope_original_max_position", 8192)),
+                          int(getattr(g, "rotary_dim", 0)))
 
 
 KVX_FORM_GROUPED, KVX_FORM_DENSE = 0, 1

@@ -19,17 +19,38 @@ constexpr int KVX_MAX_ALIGNED_BATCH = 256;   // sequences whose metadata it keep
 // exact up to the rounding of turns[i] (|error| <= p * 2^-53 turn), so the
 // range reduction costs one 64-bit multiply and no table of angles.
 struct RopeTable {
-    const unsigned long long* turns;   // device [d/2]
+    const unsigned long long* turns;   // device [d/2]; entries from rhalf on are 0
     int half;                          // d/2
     int enabled;                       // 0: no rotation
+    int rhalf;                         // rotating pairs (i, i + rhalf), i < rhalf: rotary_dim/2
+                                       // (= half unless the head is partial rotary)
 };
 
-// Rotation frequency f_i of channel pair (i, i + d/2) under the model's schedule
+// Channels of K that rotate (the first ones; all of them unless the head is partial rotary).
+__host__ __device__ inline int rope_rot_dim(const kvx_model_geom& g)
+{
+    return g.rotary_dim > 0 ? g.rotary_dim : g.head_dim;
+}
+
+// Kernels that pair element k of the first half of a head row with element k + d/2 walk
+// "pair slots" k < d/2.  A partial rotary head pairs channel i with i + rhalf (i < rhalf)
+// and leaves the channels from 2 rhalf on alone, so slot k covers the two channels
+//   (k, k + rhalf)       for k < rhalf  (a rotating pair), else
+//   (k + rhalf, k + d/2)                (two channels that do not rotate),
+// every channel exactly once; with rhalf = d/2 this is (k, k + d/2).  rhalf is a multiple
+// of 8, so a chunk of 8 (or 4) slots maps to two runs of consecutive channels.
+__host__ __device__ __forceinline__ void pair_channels(int k, int half, int rhalf, int& lo, int& hi)
+{
+    if (k < rhalf) { lo = k; hi = k + rhalf; }
+    else { lo = k + rhalf; hi = k + half; }
+}
+
+// Rotation frequency f_i of channel pair (i, i + n/2), n = rope_rot_dim, under the model's schedule
 // (kvx_rope_type in kvx.h), in double.  Host code turns it into fixed-point turns
 // once per translator; the allocation-free entry point does the same on the device.
 __host__ __device__ inline double rope_inv_freq(const kvx_model_geom& g, int i)
 {
-    const double f = pow(g.rope_base, -2.0 * (double)i / (double)g.head_dim);
+    const double f = pow(g.rope_base, -2.0 * (double)i / (double)rope_rot_dim(g));
     if (g.rope_type == KVX_ROPE_LINEAR) return f / g.rope_factor;
     if (g.rope_type != KVX_ROPE_LLAMA3) return f;
     const double wavelen = 6.283185307179586 / f;
@@ -43,6 +64,7 @@ __host__ __device__ inline double rope_inv_freq(const kvx_model_geom& g, int i)
 // Schedule parameters valid for the model's rope_type (host-side validation).
 inline bool rope_schedule_ok(const kvx_model_geom& g)
 {
+    if (g.rotary_dim != 0 && (g.rotary_dim < 16 || g.rotary_dim > g.head_dim || g.rotary_dim % 16)) return false;
     if (g.rope_base <= 0.0) return g.rope_type >= KVX_ROPE_DEFAULT && g.rope_type <= KVX_ROPE_LLAMA3;
     switch (g.rope_type) {
     case KVX_ROPE_DEFAULT: return true;

@@ -74,8 +74,9 @@ template <> struct Chunk<float> {
 };
 
 // One CTA per (32-token tile of the pass, target head, target layer * 2 + K|V).  A work item is
-// one chunk pair: VEC channels [c, c+VEC) of the first rotary half of one head row and their
-// partners [c+d/2, ...), read and written as 16-byte words, with one (cos, sin) per pair.
+// one chunk pair: VEC pair slots [c, c+VEC) of one head row, i.e. channels [c, c+VEC) and their
+// rotary partners [c+d/2, ...) (pair_channels for partial rotary heads), read and written as
+// 16-byte words, with one (cos, sin) per rotating pair.
 // X items: (token, head-block q, chunk pair); Y items: (token, chunk pair).
 template <typename T>
 __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_constant__ TranslateParams P, const FitRows R)
@@ -106,6 +107,8 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
         const int rem = it - tt * (heads * ncp_s);
         const int q = rem / ncp_s, cp = rem - q * ncp_s;
         const TokenInfo ti = tinfo[tt];
+        int c_lo, c_hi;
+        pair_channels(cp * VEC, hs, P.rs.rhalf, c_lo, c_hi);
         float a0[VEC], a1[VEC];
 #pragma unroll
         for (int e = 0; e < VEC; ++e) { a0[e] = 0.f; a1[e] = 0.f; }
@@ -113,13 +116,13 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
             int slot, gs;
             head_block(P, j, h, q, slot, gs);
             const T* base = (const T*)(kv ? P.src_v[slot] : P.src_k[slot]) + (long long)ti.b * P.sb +
-                            (long long)gs * P.sh + cp * VEC;
+                            (long long)gs * P.sh;
             for (int s = ti.lo; s < ti.hi; ++s) {
                 const T* row = base + (long long)s * P.ss;
                 float x0[VEC], x1[VEC];
-                Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row)), x0);
-                Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + hs)), x1);
-                if (rot_s) {
+                Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_lo)), x0);
+                Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_hi)), x1);
+                if (rot_s && cp * VEC < P.rs.rhalf) {
                     const int pos = src_pos_of(P, ti.b, s);
 #pragma unroll
                     for (int e = 0; e < VEC; ++e) {   // R(-theta)
@@ -136,20 +139,22 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
 #pragma unroll
             for (int e = 0; e < VEC; ++e) { a0[e] *= inv; a1[e] *= inv; }
         }
-        T* xr = X + (size_t)tt * P.in_dim + q * P.ds + cp * VEC;
-        *reinterpret_cast<uint4*>(xr) = Chunk<T>::pack(a0);
-        *reinterpret_cast<uint4*>(xr + hs) = Chunk<T>::pack(a1);
+        T* xr = X + (size_t)tt * P.in_dim + q * P.ds;
+        *reinterpret_cast<uint4*>(xr + c_lo) = Chunk<T>::pack(a0);
+        *reinterpret_cast<uint4*>(xr + c_hi) = Chunk<T>::pack(a1);
     }
     const int y_items = ntok * ncp_t;
     for (int it = threadIdx.x; it < y_items; it += blockDim.x) {
         const int tt = it / ncp_t, cp = it - tt * ncp_t;
         const TokenInfo ti = tinfo[tt];
+        int c_lo, c_hi;
+        pair_channels(cp * VEC, ht, P.rt.rhalf, c_lo, c_hi);
         float y0[VEC], y1[VEC];
         if (ti.dst_off >= 0 && ti.hi > ti.lo) {
-            const T* row = tgt + ti.dst_off + hoff + cp * VEC;
-            Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row)), y0);
-            Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + ht)), y1);
-            if (rot_t) {
+            const T* row = tgt + ti.dst_off + hoff;
+            Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_lo)), y0);
+            Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_hi)), y1);
+            if (rot_t && cp * VEC < P.rt.rhalf) {
 #pragma unroll
                 for (int e = 0; e < VEC; ++e) {   // R(-theta)
                     const float2 cs = rope_cs(P.rt, ti.pt, cp * VEC + e);
@@ -162,9 +167,9 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
 #pragma unroll
             for (int e = 0; e < VEC; ++e) { y0[e] = 0.f; y1[e] = 0.f; }
         }
-        T* yr = Y + (size_t)tt * P.dt + cp * VEC;
-        *reinterpret_cast<uint4*>(yr) = Chunk<T>::pack(y0);
-        *reinterpret_cast<uint4*>(yr + ht) = Chunk<T>::pack(y1);
+        T* yr = Y + (size_t)tt * P.dt;
+        *reinterpret_cast<uint4*>(yr + c_lo) = Chunk<T>::pack(y0);
+        *reinterpret_cast<uint4*>(yr + c_hi) = Chunk<T>::pack(y1);
     }
 }
 

@@ -153,8 +153,10 @@ kvx_status make_geometry(const kvx_translator_desc* desc, const char* who, Geome
     if (desc->path < KVX_PATH_AUTO || desc->path > KVX_PATH_TCGEN05)
         return bad(KVX_ERR_INVALID_ARG, "unknown path %d", desc->path);
     if (!rope_schedule_ok(s) || !rope_schedule_ok(d))
-        return bad(KVX_ERR_INVALID_ARG, "unknown rope_type or schedule parameters out of range "
-                                        "(source type %d, target type %d)", s.rope_type, d.rope_type);
+        return bad(KVX_ERR_INVALID_ARG, "unknown rope_type, schedule parameters out of range or rotary_dim "
+                                        "not 0 or a multiple of 16 in [16, head_dim] (source type %d rotary_dim "
+                                        "%d, target type %d rotary_dim %d)", s.rope_type, s.rotary_dim, d.rope_type,
+                   d.rotary_dim);
     const int max_pos = desc->max_position ? desc->max_position : (1 << 24);
     if (max_pos < 1 || max_pos > (1 << 30)) return bad(KVX_ERR_INVALID_ARG, "max_position must be in [1, 1<<30]");
     if (desc->form != KVX_FORM_GROUPED && desc->form != KVX_FORM_DENSE)
@@ -187,15 +189,15 @@ kvx_status make_geometry(const kvx_translator_desc* desc, const char* who, Geome
     if (g.in_dim > 1024) return bad(KVX_ERR_UNSUPPORTED, "translator input width %d > 1024", g.in_dim);
     // rotation frequencies as fixed-point turns (kvx_common.cuh)
     const int hs = s.head_dim / 2, hd = d.head_dim / 2;
-    auto fill = [&](const kvx_model_geom& m, unsigned long long* o) {
-        for (int i = 0; i < m.head_dim / 2; ++i)
+    auto fill = [&](const kvx_model_geom& m, unsigned long long* o) {   // pairs past rotary_dim/2: 0
+        for (int i = 0; i < rope_rot_dim(m) / 2; ++i)
             o[i] = m.rope_base <= 0.0 ? 0ull : (unsigned long long)ldexp(rope_inv_freq(m, i) / (2.0 * M_PI), 64);
     };
     memset(g.turns, 0, sizeof g.turns);
     fill(s, g.turns);
     fill(d, g.turns + hs);
-    // the two rotations coincide when head dims, enablement and every frequency agree
-    g.rope_same = hs == hd && (s.rope_base > 0.0) == (d.rope_base > 0.0) &&
+    // the two rotations coincide when head dims, rotating channels, enablement and every frequency agree
+    g.rope_same = hs == hd && rope_rot_dim(s) == rope_rot_dim(d) && (s.rope_base > 0.0) == (d.rope_base > 0.0) &&
                   memcmp(g.turns, g.turns + hs, (size_t)hs * sizeof(unsigned long long)) == 0;
     return KVX_OK;
 }
@@ -248,8 +250,8 @@ kvx_status make_params(const Geometry& g, const unsigned long long* dev_turns, u
     P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
     P.page_size = dst->page_size; P.num_pages = dst->num_pages;
     const int hs = D.src.head_dim / 2;
-    P.rs = RopeTable{dev_turns, hs, D.src.rope_base > 0.0};
-    P.rt = RopeTable{dev_turns + hs, D.dst.head_dim / 2, D.dst.rope_base > 0.0};
+    P.rs = RopeTable{dev_turns, hs, D.src.rope_base > 0.0, rope_rot_dim(D.src) / 2};
+    P.rt = RopeTable{dev_turns + hs, D.dst.head_dim / 2, D.dst.rope_base > 0.0, rope_rot_dim(D.dst) / 2};
     P.max_position = g.max_position;
     P.rope_same = g.rope_same;
     P.status = status;
@@ -342,7 +344,8 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
         if ((ce = cudaMemcpy(raw, w_k, one, kind)) != cudaSuccess ||
             (ce = cudaMemcpy((char*)raw + one, w_v, one, kind)) != cudaSuccess ||
             (ce = launch_tc_weight_relayout(raw, (char*)raw + one, t->w, d.num_layers, d.num_kv_heads,
-                                            t->in_dim, d.head_dim, t->tc.n_tile, 0)) != cudaSuccess ||
+                                            t->in_dim, d.head_dim, t->tc.n_tile, rope_rot_dim(d) / 2, 0)) !=
+                cudaSuccess ||
             (ce = cudaDeviceSynchronize()) != cudaSuccess) {
             st = fail(KVX_ERR_CUDA, "create: weight re-layout: %s", cudaGetErrorString(ce));
             goto err;
@@ -363,8 +366,8 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
             st = fail(KVX_ERR_CUDA, "create: table upload: %s", cudaGetErrorString(ce));
             goto err;
         }
-        t->rs = RopeTable{t->rope, hs, s.rope_base > 0.0};
-        t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0};
+        t->rs = RopeTable{t->rope, hs, s.rope_base > 0.0, rope_rot_dim(s) / 2};
+        t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0, rope_rot_dim(d) / 2};
     }
     if (cudaMalloc(&t->status, sizeof(unsigned)) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: status allocation"); goto err; }
     if (t->path == KVX_PATH_TCGEN05 && cudaMalloc(&t->plan, tc_plan_bytes(kvx_translator::kPlanTokens)) != cudaSuccess) {
@@ -446,7 +449,10 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
     }
     if (tgt->total_tokens == 0) return KVX_OK;
     cudaError_t ce;
-    if (tr->path == KVX_PATH_TCGEN05 && !tgt->span_lo &&
+    // partial rotary heads (rotary_dim < head_dim on either side) take the span kernel, which
+    // pairs channels at rotary_dim/2; the identity kernel pairs whole heads
+    const bool whole_head_rope = rope_rot_dim(D.src) == D.src.head_dim && rope_rot_dim(D.dst) == D.dst.head_dim;
+    if (tr->path == KVX_PATH_TCGEN05 && !tgt->span_lo && whole_head_rope &&
         aligned_supported(tr->in_dim, D.dst.head_dim, D.src.head_dim, Lt, src->batch, tr->kl)) {
         // identity alignment: tensor-TMA fed kernel
         if (tr->maps.empty()) tr->maps.resize((size_t)2 * KVX_MAX_ALIGNED_LAYERS * kvx_translator::kMapWays);

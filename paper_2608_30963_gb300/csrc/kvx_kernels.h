@@ -27,8 +27,9 @@ struct TcConfig {
 };
 TcConfig tc_config(int in_dim, int dt, int ds);
 size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht);
+// rhalf_t: rotating pairs of the target head (rotary_dim/2; d_t/2 unless partial rotary)
 cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
-                                      int dt, int n_tile, cudaStream_t stream);
+                                      int dt, int n_tile, int rhalf_t, cudaStream_t stream);
 size_t tc_plan_bytes(int tokens);
 // One span-plan launch and one translation launch per chunk of at most plan_tokens
 // target tokens; *launches receives the number of launches made.

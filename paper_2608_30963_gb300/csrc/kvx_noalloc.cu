@@ -44,12 +44,12 @@ kvx_status fail(kvx_status s, const char* fmt, ...)
 }
 
 // Fixed-point rotation turns round(2^64 f_i / 2 pi), f_i the model's scheduled frequency
-// of pair i, written on the device.
+// of pair i (0 for the pairs of a partial rotary head that do not rotate), written on the device.
 __global__ void static_turns_kernel(unsigned long long* out, const kvx_model_geom g)
 {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= g.head_dim / 2) return;
-    if (g.rope_base <= 0.0) { out[i] = 0ull; return; }
+    if (g.rope_base <= 0.0 || i >= rope_rot_dim(g) / 2) { out[i] = 0ull; return; }
     out[i] = (unsigned long long)ldexp(rope_inv_freq(g, i) / (2.0 * 3.14159265358979323846), 64);
 }
 
@@ -174,8 +174,8 @@ extern "C" KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* de
         P.db = dst->stride_b; P.dh = dst->stride_h; P.dts = dst->stride_t;
         P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
         P.page_size = dst->page_size; P.num_pages = dst->num_pages;
-        P.rs = RopeTable{turns, s.head_dim / 2, s.rope_base > 0.0};
-        P.rt = RopeTable{turns + 128, d.head_dim / 2, d.rope_base > 0.0};
+        P.rs = RopeTable{turns, s.head_dim / 2, s.rope_base > 0.0, rope_rot_dim(s) / 2};
+        P.rt = RopeTable{turns + 128, d.head_dim / 2, d.rope_base > 0.0, rope_rot_dim(d) / 2};
         P.max_position = max_pos;
         P.status = status;
         P.w = wts;

@@ -35,7 +35,7 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
 
     const bool rot_s = kv == 0 && P.rs.enabled;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int hs = P.ds >> 1;
+    const int hs = P.rs.rhalf;   // rotating pairs (c, c + hs), c < hs; channels from 2 hs on do not rotate
 
     // ---- phase 1: un-rotate + span mean
     for (int tt = warp; tt < kSimtTile; tt += kSimtThreads / 32) {
@@ -54,7 +54,7 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
             for (int s = ti.lo; s < ti.hi; ++s) {
                 const T* row = base + (long long)s * P.ss;
                 float x = to_f32<T>(row[c]);
-                if (rot_s) {
+                if (rot_s && c < 2 * hs) {
                     const int i = c < hs ? c : c - hs;
                     const float xp = to_f32<T>(row[c < hs ? c + hs : c - hs]);
                     const float2 cs = rope_cs(P.rs, src_pos_of(P, ti.b, s), i);
@@ -93,14 +93,14 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
     // ---- phase 3: target RoPE + store
     T* dst = (T*)(kv ? P.dst_v[j] : P.dst_k[j]);
     const bool rot_t = kv == 0 && P.rt.enabled;
-    const int ht = P.dt >> 1;
+    const int ht = P.rt.rhalf;   // rotating pairs (c, c + ht), c < ht
     const long long hoff = dst_head_off(P, h);
     for (int idx = threadIdx.x; idx < ntok * P.dt; idx += kSimtThreads) {
         const int tt = idx / P.dt, c = idx - tt * P.dt;
         const TokenInfo& ti = tinfo[tt];
         if (ti.dst_off < 0) continue;
         float y = Y[tt * P.dt + c];
-        if (rot_t) {
+        if (rot_t && c < 2 * ht) {
             const int i = c < ht ? c : c - ht;
             const float yp = Y[tt * P.dt + (c < ht ? c + ht : c - ht)];
             const float2 cs = rope_cs(P.rt, ti.pt, i);

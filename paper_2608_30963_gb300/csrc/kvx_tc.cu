@@ -514,7 +514,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 tmem_ld8(taddr + hw + pc, r1);
                 tmem_ld_wait();
                 uint4 out0, out1;
-                rotate8_to_bf16(r0, r1, cs, rot, out0, out1);
+                // pair slots from rhalf on (partial rotary heads) do not rotate
+                rotate8_to_bf16(r0, r1, cs, rot && x.nt * hw + pc < P.rt.rhalf, out0, out1);
                 if (rot) {
 #pragma unroll
                     for (int e = 0; e < 8; ++e) cs[e] = csn[e];
@@ -532,12 +533,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             if (half == 0 && valid && dst_off >= 0) {
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      dst_head_off(P, x.h);
-                if (L.n_split == 1) {
-                    bulk_s2g(dst, srow_u32, (uint32_t)P.dt * 2);
-                } else {
-                    bulk_s2g(dst + x.nt * hw, srow_u32, (uint32_t)hw * 2);
-                    bulk_s2g(dst + half_t + x.nt * hw, srow_u32 + hw * 2, (uint32_t)hw * 2);
-                }
+                store_row_slots(dst, srow_u32, x.nt * hw, hw, half_t, P.rt.rhalf);
                 bulk_commit();
             }
             ++tcount;
@@ -546,18 +542,23 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
     } else {
         // ------------------------------------------------------------ prologue (A head-blocks)
         // Lanes split into groups of LPT, one target token per group; a lane owns one
-        // chunk pair: channels [8cp, 8cp+8) and their rotary partners [DS/2+8cp, ...),
-        // so each source row is read as two 16-byte loads per lane (a group reads whole
-        // 128-byte row segments: no bank conflicts on the linear window rows).
+        // chunk pair: pair slots [8cp, 8cp+8), i.e. channels [8cp, 8cp+8) and their rotary
+        // partners [DS/2+8cp, ...) (pair_channels: a partial rotary head pairs at rhalf,
+        // and lanes past rhalf hold channels that do not rotate), so each source row is read
+        // as two 16-byte loads per lane (a group reads whole 128-byte row segments: no bank
+        // conflicts on the linear window rows) and A is written at the same channels.
         constexpr int LPT = DS / 16;
         constexpr int TPW = 32 / LPT;
         constexpr int HALF = DS / 2;
         const int tw = warp - kXfWarp0;
         const int cp = lane % LPT;
         const int u = lane / LPT;
-        const uint32_t c_lo = (uint32_t)cp * 16, c_hi = (uint32_t)(HALF / 8 + cp) * 16;
-        const uint32_t a_lo = (uint32_t)((8 * cp) >> 6) * (kTileM * 128), a_hi = (uint32_t)((HALF + 8 * cp) >> 6) * (kTileM * 128);
-        const int ch_lo = cp & 7, ch_hi = ((HALF + 8 * cp) >> 3) & 7;
+        int k_lo, k_hi;
+        pair_channels(8 * cp, HALF, P.rs.rhalf, k_lo, k_hi);
+        const bool lane_rot = 8 * cp < P.rs.rhalf;
+        const uint32_t c_lo = (uint32_t)k_lo * 2, c_hi = (uint32_t)k_hi * 2;
+        const uint32_t a_lo = (uint32_t)(k_lo >> 6) * (kTileM * 128), a_hi = (uint32_t)(k_hi >> 6) * (kTileM * 128);
+        const int ch_lo = (k_lo >> 3) & 7, ch_hi = (k_hi >> 3) & 7;
         unsigned long long turn[8];
 #pragma unroll
         for (int e = 0; e < 8; ++e) turn[e] = sTurnS[cp * 8 + e];
@@ -568,7 +569,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         Walker wk;
         for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
             const Unit& x = wk.x;
-            const bool rot = x.kv == 0 && P.rs.enabled;
+            const bool rot = x.kv == 0 && P.rs.enabled && lane_rot;
             for (int q = 0; q < L.r_heads && ok; ++q) {
                 int src_slot, gq;
                 head_block(P, x.j, x.h, q, src_slot, gq);
@@ -709,11 +710,13 @@ __global__ void __launch_bounds__(128) span_plan_kernel(const __grid_constant__ 
 }
 
 // Weight images: for group g = ((j*Ht + h)*2 + kv)*n_split + nt, the B operand
-// [n_tile rows = output columns][in] in K-major SW128 layout.  Output column of
-// image row n: n < n_tile/2 -> nt*hw + n, else d_t/2 + nt*hw + (n - hw), so an
-// image holds whole RoPE pairs.
+// [n_tile rows = output columns][in] in K-major SW128 layout.  Image row n holds pair
+// slot k = nt*hw + (n mod hw): its first channel for n < hw, its partner above
+// (pair_channels: (k, k + d_t/2), or the partial rotary pairing), so an image holds
+// whole RoPE pairs and the epilogue rotates columns n and n + hw together.
 __global__ void tc_weight_relayout_kernel(const __nv_bfloat16* __restrict__ wk, const __nv_bfloat16* __restrict__ wv,
-                                          uint8_t* __restrict__ img, int Lt, int Ht, int in_dim, int dt, int n_tile)
+                                          uint8_t* __restrict__ img, int Lt, int Ht, int in_dim, int dt, int n_tile,
+                                          int rhalf_t)
 {
     const int n_split = dt / n_tile, hw = n_tile / 2;
     const long long chunks_per_img = (long long)n_tile * in_dim / 8;
@@ -730,7 +733,9 @@ __global__ void tc_weight_relayout_kernel(const __nv_bfloat16* __restrict__ wk, 
     // chunk c enumerates (n, k/8) with k fastest
     const int n = c / (in_dim / 8);
     const int k8 = c - n * (in_dim / 8);
-    const int col = n < hw ? nt * hw + n : dt / 2 + nt * hw + (n - hw);
+    int c_lo, c_hi;
+    pair_channels(nt * hw + (n < hw ? n : n - hw), dt / 2, rhalf_t, c_lo, c_hi);
+    const int col = n < hw ? c_lo : c_hi;
     const __nv_bfloat16* w = (kv ? wv : wk) + ((size_t)j * Ht + h) * (size_t)in_dim * dt;
     uint32_t v[4];
     for (int e = 0; e < 4; ++e) {
@@ -833,12 +838,12 @@ size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht)
 }
 
 cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
-                                      int dt, int n_tile, cudaStream_t stream)
+                                      int dt, int n_tile, int rhalf_t, cudaStream_t stream)
 {
     const long long total = (long long)Lt * Ht * 2 * dt * in_dim / 8;
     const int threads = 256;
     tc_weight_relayout_kernel<<<(unsigned)((total + threads - 1) / threads), threads, 0, stream>>>(
-        (const __nv_bfloat16*)w_k, (const __nv_bfloat16*)w_v, (uint8_t*)image, Lt, Ht, in_dim, dt, n_tile);
+        (const __nv_bfloat16*)w_k, (const __nv_bfloat16*)w_v, (uint8_t*)image, Lt, Ht, in_dim, dt, n_tile, rhalf_t);
     return cudaGetLastError();
 }
 

@@ -102,6 +102,27 @@ __device__ __forceinline__ void bulk_s2g(void* dst, uint32_t src, uint32_t bytes
     asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
                  : "memory");
 }
+// Stores one output row of a tile from its staging row (bf16).  The tile holds pair slots
+// [a, a + hw) (pair_channels, kvx_common.cuh) of a head of 2 half channels; the staging
+// row has the slots' first channels, then their partners.  One bulk copy when the tile is
+// the whole row of a fully rotating head; else one per run of consecutive channels (at most
+// four).  Every run starts and ends on a multiple of 8 channels (16 bytes).
+__device__ __forceinline__ void store_row_slots(__nv_bfloat16* dst, uint32_t srow, int a, int hw, int half, int rhalf)
+{
+    if (hw == half && rhalf == half) {
+        bulk_s2g(dst, srow, (uint32_t)half * 4);
+        return;
+    }
+    const int n_rot = min(max(rhalf - a, 0), hw);   // slots of the tile that are rotating pairs
+    if (n_rot > 0) {
+        bulk_s2g(dst + a, srow, (uint32_t)n_rot * 2);
+        bulk_s2g(dst + a + rhalf, srow + (uint32_t)hw * 2, (uint32_t)n_rot * 2);
+    }
+    if (n_rot < hw) {
+        bulk_s2g(dst + a + n_rot + rhalf, srow + (uint32_t)n_rot * 2, (uint32_t)(hw - n_rot) * 2);
+        bulk_s2g(dst + a + n_rot + half, srow + (uint32_t)(hw + n_rot) * 2, (uint32_t)(hw - n_rot) * 2);
+    }
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }

@@ -112,6 +112,10 @@ CASES = {
     # name: (base spec, Ls, Lt, target lengths, extra spec fields)
     "qwen7b_qwen1p5b_identity": ("qwen7b_to_qwen1p5b_4k", 3, 2, [900, 600], {}),
     "gemma_expansion_spans": ("qwen1p5b_to_gemma2b_1k", 3, 2, [700, 500], {}),
+    # partial rotary heads on both sides (a half of the source head, a quarter of the target's)
+    "partial_rotary_identity": ("qwen7b_to_qwen1p5b_4k", 3, 2, [900, 600],
+                                dict(src=synth.ModelGeom(3, 4, 128, 1e6, rotary_dim=64),
+                                     dst=synth.ModelGeom(2, 2, 128, 1e6, rotary_dim=32))),
     # dense per-layer form over 2 source heads of 128 (in = 256), cross-tokenizer spans
     "dense_spans": ("llama70b_to_qwen7b_8k", 4, 2, [1100, 700], dict(form=synth.FORM_DENSE,
                                                                    src=synth.ModelGeom(4, 2, 128, 5e5),

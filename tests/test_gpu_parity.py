@@ -116,6 +116,38 @@ def test_rope_schedules(name, path):
     _full_compare(c, path)
 
 
+PARTIAL = {
+    # (base, Ls, Lt, target lengths, source rotary_dim, target geometry changes); identity
+    # alignment with a partial rotary head runs on the span kernel (the identity kernel
+    # rotates whole heads only)
+    # same partial head on both sides
+    "both64_identity": ("qwen7b_to_qwen1p5b_4k", 2, 2, [300, 5], 64, dict(rotary_dim=64)),
+    # a quarter of the source head rotates, the target head fully: source side only
+    "src32_identity": ("qwen7b_to_qwen1p5b_4k", 2, 2, [300], 32, {}),
+    # d_t = 256 in two output tiles, 96 rotating channels: row stores split in up to four runs
+    "dst96_identity_split": ("qwen7b_to_qwen1p5b_4k", 2, 2, [300, 41], 0,
+                             dict(head_dim=256, rope_base=1e4, rotary_dim=96)),
+    # cross-tokenizer spans: partial source (lanes past rhalf do not rotate), partial target
+    "src64_spans": ("llama70b_to_qwen7b_8k", 5, 3, [300, 41], 64, {}),
+    "dst128_spans_gemma": ("qwen1p5b_to_gemma2b_1k", 3, 2, [300], 0, dict(rotary_dim=128)),
+    # fp32 caches: the CUDA-core kernel
+    "both32_tiny_fp32": ("tiny_fp32", 4, 2, [256, 100], 32, dict(rotary_dim=32)),
+}
+
+
+@pytest.mark.parametrize("path", PATHS, ids=["simt", "auto"])
+@pytest.mark.parametrize("name", list(PARTIAL))
+def test_partial_rotary_heads(name, path):
+    base, Ls, Lt, lens, rot_s, dst_kw = PARTIAL[name]
+    spec = _shrink(SPECS[base], Ls, Lt)
+    spec = dataclasses.replace(spec, src=dataclasses.replace(spec.src, rotary_dim=rot_s),
+                               dst=dataclasses.replace(spec.dst, **dst_kw))
+    c = make_case(spec, lens, pad_value=float("nan"))
+    g, _, _ = _full_compare(c, path)
+    if path == kvx.KVX_PATH_AUTO and spec.dtype == "bf16":
+        assert g.tr.info().path == kvx.KVX_PATH_TCGEN05
+
+
 FORMS = {
     # one map per target layer over all 8 source heads: in = 1024, streamed weight pieces
     "dense_in1024_spans": ("llama70b_to_qwen7b_8k_dense", 5, 3, [300, 41], {}),

@@ -62,6 +62,11 @@ def _desc(src, dst, dtype=kvx.KVX_BF16, path=kvx.KVX_PATH_AUTO, layer_map=None):
     (synth.ModelGeom(2, 2, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6, rope_type=2, rope_factor=8.0,
                                                        rope_low_freq_factor=4.0, rope_high_freq_factor=1.0),
      kvx.KVX_ERR_INVALID_ARG),
+    # partial rotary: rotary_dim must be 0 or a multiple of 16 in [16, head_dim]
+    (synth.ModelGeom(2, 2, 128, 1e6, rotary_dim=24), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_INVALID_ARG),
+    (synth.ModelGeom(2, 2, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6, rotary_dim=256), kvx.KVX_ERR_INVALID_ARG),
+    (synth.ModelGeom(2, 2, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6, rotary_dim=-16), kvx.KVX_ERR_INVALID_ARG),
+    (synth.ModelGeom(2, 2, 64, 1e6, rotary_dim=8), synth.ModelGeom(2, 2, 128, 1e6), kvx.KVX_ERR_INVALID_ARG),
 ])
 def test_create_rejects_bad_geometry_without_touching_cuda(lib, src, dst, code):
     h = ctypes.c_void_p()
