@@ -19,11 +19,9 @@ constexpr int KVX_MAX_ALIGNED_BATCH = 256;   // sequences whose metadata it keep
 // exact up to the rounding of turns[i] (|error| <= p * 2^-53 turn), so the
 // range reduction costs one 64-bit multiply and no table of angles.
 struct RopeTable {
-    const unsigned long long* turns;   // device [d/2]; entries from rhalf on are 0
+    const unsigned long long* turns;   // device [d/2]; entries of pairs that do not rotate are 0
     int half;                          // d/2
     int enabled;                       // 0: no rotation
-    int rhalf;                         // rotating pairs (i, i + rhalf), i < rhalf: rotary_dim/2
-                                       // (= half unless the head is partial rotary)
 };
 
 // Channels of K that rotate (the first ones; all of them unless the head is partial rotary).
@@ -106,6 +104,8 @@ struct TranslateParams {
     int max_pages, page_size, num_pages;
     // rotation
     RopeTable rs, rt;
+    int rhalf_s, rhalf_t;   // rotating pairs (i, i + rhalf), i < rhalf, of the source / target head:
+                            // rotary_dim/2 (= d/2 unless the head is partial rotary)
     int rope_same;   // source and target rotations coincide (same head_dim, same frequencies)
     int max_position;
     unsigned* status;

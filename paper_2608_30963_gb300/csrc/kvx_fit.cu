@@ -108,7 +108,7 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
         const int q = rem / ncp_s, cp = rem - q * ncp_s;
         const TokenInfo ti = tinfo[tt];
         int c_lo, c_hi;
-        pair_channels(cp * VEC, hs, P.rs.rhalf, c_lo, c_hi);
+        pair_channels(cp * VEC, hs, P.rhalf_s, c_lo, c_hi);
         float a0[VEC], a1[VEC];
 #pragma unroll
         for (int e = 0; e < VEC; ++e) { a0[e] = 0.f; a1[e] = 0.f; }
@@ -122,7 +122,7 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
                 float x0[VEC], x1[VEC];
                 Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_lo)), x0);
                 Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_hi)), x1);
-                if (rot_s && cp * VEC < P.rs.rhalf) {
+                if (rot_s && cp * VEC < P.rhalf_s) {
                     const int pos = src_pos_of(P, ti.b, s);
 #pragma unroll
                     for (int e = 0; e < VEC; ++e) {   // R(-theta)
@@ -148,13 +148,13 @@ __global__ void __launch_bounds__(kFitThreads) fit_rows_kernel(const __grid_cons
         const int tt = it / ncp_t, cp = it - tt * ncp_t;
         const TokenInfo ti = tinfo[tt];
         int c_lo, c_hi;
-        pair_channels(cp * VEC, ht, P.rt.rhalf, c_lo, c_hi);
+        pair_channels(cp * VEC, ht, P.rhalf_t, c_lo, c_hi);
         float y0[VEC], y1[VEC];
         if (ti.dst_off >= 0 && ti.hi > ti.lo) {
             const T* row = tgt + ti.dst_off + hoff;
             Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_lo)), y0);
             Chunk<T>::unpack(__ldg(reinterpret_cast<const uint4*>(row + c_hi)), y1);
-            if (rot_t && cp * VEC < P.rt.rhalf) {
+            if (rot_t && cp * VEC < P.rhalf_t) {
 #pragma unroll
                 for (int e = 0; e < VEC; ++e) {   // R(-theta)
                     const float2 cs = rope_cs(P.rt, ti.pt, cp * VEC + e);

@@ -250,8 +250,10 @@ kvx_status make_params(const Geometry& g, const unsigned long long* dev_turns, u
     P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
     P.page_size = dst->page_size; P.num_pages = dst->num_pages;
     const int hs = D.src.head_dim / 2;
-    P.rs = RopeTable{dev_turns, hs, D.src.rope_base > 0.0, rope_rot_dim(D.src) / 2};
-    P.rt = RopeTable{dev_turns + hs, D.dst.head_dim / 2, D.dst.rope_base > 0.0, rope_rot_dim(D.dst) / 2};
+    P.rs = RopeTable{dev_turns, hs, D.src.rope_base > 0.0};
+    P.rt = RopeTable{dev_turns + hs, D.dst.head_dim / 2, D.dst.rope_base > 0.0};
+    P.rhalf_s = rope_rot_dim(D.src) / 2;
+    P.rhalf_t = rope_rot_dim(D.dst) / 2;
     P.max_position = g.max_position;
     P.rope_same = g.rope_same;
     P.status = status;
@@ -366,8 +368,8 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
             st = fail(KVX_ERR_CUDA, "create: table upload: %s", cudaGetErrorString(ce));
             goto err;
         }
-        t->rs = RopeTable{t->rope, hs, s.rope_base > 0.0, rope_rot_dim(s) / 2};
-        t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0, rope_rot_dim(d) / 2};
+        t->rs = RopeTable{t->rope, hs, s.rope_base > 0.0};
+        t->rt = RopeTable{t->rope + hs, hd, d.rope_base > 0.0};
     }
     if (cudaMalloc(&t->status, sizeof(unsigned)) != cudaSuccess) { st = fail(KVX_ERR_OOM, "create: status allocation"); goto err; }
     if (t->path == KVX_PATH_TCGEN05 && cudaMalloc(&t->plan, tc_plan_bytes(kvx_translator::kPlanTokens)) != cudaSuccess) {

@@ -174,8 +174,10 @@ extern "C" KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* de
         P.db = dst->stride_b; P.dh = dst->stride_h; P.dts = dst->stride_t;
         P.page_table = dst->page_table; P.max_pages = dst->max_pages_per_seq;
         P.page_size = dst->page_size; P.num_pages = dst->num_pages;
-        P.rs = RopeTable{turns, s.head_dim / 2, s.rope_base > 0.0, rope_rot_dim(s) / 2};
-        P.rt = RopeTable{turns + 128, d.head_dim / 2, d.rope_base > 0.0, rope_rot_dim(d) / 2};
+        P.rs = RopeTable{turns, s.head_dim / 2, s.rope_base > 0.0};
+        P.rt = RopeTable{turns + 128, d.head_dim / 2, d.rope_base > 0.0};
+        P.rhalf_s = rope_rot_dim(s) / 2;
+        P.rhalf_t = rope_rot_dim(d) / 2;
         P.max_position = max_pos;
         P.status = status;
         P.w = wts;

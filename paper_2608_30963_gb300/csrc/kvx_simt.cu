@@ -35,7 +35,7 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
 
     const bool rot_s = kv == 0 && P.rs.enabled;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int hs = P.rs.rhalf;   // rotating pairs (c, c + hs), c < hs; channels from 2 hs on do not rotate
+    const int hs = P.rhalf_s;   // rotating pairs (c, c + hs), c < hs; channels from 2 hs on do not rotate
 
     // ---- phase 1: un-rotate + span mean
     for (int tt = warp; tt < kSimtTile; tt += kSimtThreads / 32) {
@@ -93,7 +93,7 @@ __global__ void __launch_bounds__(kSimtThreads) translate_simt_kernel(const __gr
     // ---- phase 3: target RoPE + store
     T* dst = (T*)(kv ? P.dst_v[j] : P.dst_k[j]);
     const bool rot_t = kv == 0 && P.rt.enabled;
-    const int ht = P.rt.rhalf;   // rotating pairs (c, c + ht), c < ht
+    const int ht = P.rhalf_t;   // rotating pairs (c, c + ht), c < ht
     const long long hoff = dst_head_off(P, h);
     for (int idx = threadIdx.x; idx < ntok * P.dt; idx += kSimtThreads) {
         const int tt = idx / P.dt, c = idx - tt * P.dt;

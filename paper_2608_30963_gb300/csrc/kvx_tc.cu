@@ -515,7 +515,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 tmem_ld_wait();
                 uint4 out0, out1;
                 // pair slots from rhalf on (partial rotary heads) do not rotate
-                rotate8_to_bf16(r0, r1, cs, rot && x.nt * hw + pc < P.rt.rhalf, out0, out1);
+                rotate8_to_bf16(r0, r1, cs, rot && x.nt * hw + pc < P.rhalf_t, out0, out1);
                 if (rot) {
 #pragma unroll
                     for (int e = 0; e < 8; ++e) cs[e] = csn[e];
@@ -533,7 +533,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             if (half == 0 && valid && dst_off >= 0) {
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      dst_head_off(P, x.h);
-                store_row_slots(dst, srow_u32, x.nt * hw, hw, half_t, P.rt.rhalf);
+                store_row_slots(dst, srow_u32, x.nt * hw, hw, half_t, P.rhalf_t);
                 bulk_commit();
             }
             ++tcount;
@@ -554,8 +554,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         const int cp = lane % LPT;
         const int u = lane / LPT;
         int k_lo, k_hi;
-        pair_channels(8 * cp, HALF, P.rs.rhalf, k_lo, k_hi);
-        const bool lane_rot = 8 * cp < P.rs.rhalf;
+        pair_channels(8 * cp, HALF, P.rhalf_s, k_lo, k_hi);
+        const bool lane_rot = 8 * cp < P.rhalf_s;
         const uint32_t c_lo = (uint32_t)k_lo * 2, c_hi = (uint32_t)k_hi * 2;
         const uint32_t a_lo = (uint32_t)(k_lo >> 6) * (kTileM * 128), a_hi = (uint32_t)(k_hi >> 6) * (kTileM * 128);
         const int ch_lo = (k_lo >> 3) & 7, ch_hi = (k_hi >> 3) & 7;
