@@ -45,7 +45,7 @@ extern "C" {
 typedef enum {
     KVX_OK = 0,
     KVX_ERR_INVALID_ARG = 1,    /* a pointer, size or stride is invalid */
-    KVX_ERR_UNSUPPORTED = 2,    /* a geometry this build has no kernel for */
+    KVX_ERR_UNSUPPORTED = 2,    /* a geometry the library has no kernel for */
     KVX_ERR_CUDA = 3,           /* a CUDA runtime call failed */
     KVX_ERR_OOM = 4,            /* device allocation failed (create only) */
     KVX_ERR_DEVICE_STATUS = 5   /* kvx_get_device_status found a nonzero status */
