@@ -17,14 +17,18 @@ the max over ranks.
 from __future__ import annotations
 
 import argparse
+import hashlib
 import json
 import math
 import multiprocessing as mp
 import os
+import re
+import shutil
 import statistics
+import struct
 import subprocess
-import tempfile
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -215,7 +219,12 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--mode", default="translate", choices=["translate", "fit"],
                     help="translate: the hot path (default); fit: the closed-form translator fit's accumulation")
+    ap.add_argument("--rekey-traffic", metavar="REV",
+                    help="maintenance (no GPU): re-key profiles/traffic.json to the current sources if the "
+                         "identity kernel compiles to the same device code as at git revision REV")
     args = ap.parse_args()
+    if args.rekey_traffic:
+        return rekey_traffic(args.rekey_traffic)
     args.warmup = max(args.warmup, 3)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -632,6 +641,65 @@ def kernel_rev(sources=None) -> str:
     for f in sources:
         h.update(open(os.path.join(ROOT, f), "rb").read())
     return h.hexdigest()[:12]
+
+
+_TRAFFIC_REC = os.path.join(ROOT, "profiles", "traffic.json")
+
+
+def _cubin_sections(path):
+    b = open(path, "rb").read()
+    shoff = struct.unpack_from("<Q", b, 0x28)[0]
+    shentsize, shnum, shstrndx = struct.unpack_from("<HHH", b, 0x3A)
+    hdrs = [struct.unpack_from("<IIQQQQIIQQ", b, shoff + i * shentsize) for i in range(shnum)]
+    stro = hdrs[shstrndx][4]
+    out = {}
+    for h in hdrs:
+        end = b.index(b"\0", stro + h[0])
+        name = re.sub(r"_GLOBAL__N__[0-9a-f]+_", "_GLOBAL__N__", b[stro + h[0]:end].decode())
+        if name in (".shstrtab", ".strtab", ".symtab"):
+            continue
+        data = b[h[4]:h[4] + h[5]] if h[1] != 8 else b""
+        out[name] = (h[5], hashlib.sha256(data).hexdigest())
+    return out
+
+
+def _aligned_cubin(tree, out):
+    subprocess.check_call(["nvcc", "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17",
+                           "-I" + os.path.join(tree, "include"), "-cubin",
+                           os.path.join(tree, "paper_2608_30963_gb300", "csrc", "kvx_tc_aligned.cu"), "-o", out])
+    return _cubin_sections(out)
+
+
+def rekey_traffic(rev) -> int:
+    """Re-keys profiles/traffic.json to the current sources if the identity-alignment kernel
+    compiles to the same device code as at revision `rev`, the one whose DRAM traffic the record
+    holds: both revisions' kvx_tc_aligned.cu are compiled for sm_103a to cubins (no line info)
+    and every ELF section is compared by size and sha256 (the translation unit's anonymous-
+    namespace tag in section names normalised).  Only whole-section hashes are compared; no code
+    is decoded."""
+    tmp = tempfile.mkdtemp()
+    try:
+        old = os.path.join(tmp, "old")
+        subprocess.check_call(["git", "-C", ROOT, "worktree", "add", "-q", "--detach", old, rev])
+        try:
+            a = _aligned_cubin(old, os.path.join(tmp, "old.cubin"))
+        finally:
+            subprocess.call(["git", "-C", ROOT, "worktree", "remove", "--force", old])
+        b = _aligned_cubin(ROOT, os.path.join(tmp, "new.cubin"))
+    finally:
+        shutil.rmtree(tmp, ignore_errors=True)
+    diff = sorted(n for n in set(a) | set(b) if a.get(n) != b.get(n))
+    if diff:
+        print("device code differs in", len(diff), "sections, e.g.", diff[:3])
+        return 1
+    rec = json.load(open(_TRAFFIC_REC))
+    rec["kernel_rev"] = kernel_rev(rec["sources"])
+    rec["same_code_as"] = rev
+    with open(_TRAFFIC_REC, "w") as f:
+        json.dump(rec, f, indent=1)
+        f.write("\n")
+    print("identical device code; kernel_rev", rec["kernel_rev"])
+    return 0
 
 
 def reference_arm(args, spec, rank, world):
