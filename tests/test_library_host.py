@@ -126,3 +126,64 @@ def test_null_arguments_rejected(lib):
     assert lib.kvx_destroy(None) == kvx.KVX_OK
     assert lib.kvx_build_alignment(0, 0, 0, None, None, None, None, None, None, None, None) == \
         kvx.KVX_ERR_INVALID_ARG
+
+
+def _geom_desc(src, dst, **kw):
+    d = _desc(src, dst)
+    for k, v in kw.items():
+        setattr(d, k, v)
+    return d
+
+
+def test_fit_create_rejects_bad_arguments_without_touching_cuda(lib):
+    h = ctypes.c_void_p()
+    ok_src, ok_dst = synth.ModelGeom(2, 4, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6)
+    assert lib.kvx_fit_create(None, 0.1, 0, ctypes.byref(h)) == kvx.KVX_ERR_INVALID_ARG
+    for lam in (-1.0, float("nan")):
+        assert lib.kvx_fit_create(ctypes.byref(_desc(ok_src, ok_dst)), lam, 0, ctypes.byref(h)) == \
+            kvx.KVX_ERR_INVALID_ARG
+        assert "lambda" in kvx.kvx_last_error()
+    for chunk in (-1, (1 << 20) + 1):
+        assert lib.kvx_fit_create(ctypes.byref(_desc(ok_src, ok_dst)), 0.1, chunk, ctypes.byref(h)) == \
+            kvx.KVX_ERR_INVALID_ARG
+        assert "chunk_tokens" in kvx.kvx_last_error()
+    # the translator geometry is checked as for kvx_translator_create
+    bad = _desc(synth.ModelGeom(2, 4, 128, 1e6, rotary_dim=24), ok_dst)
+    assert lib.kvx_fit_create(ctypes.byref(bad), 0.1, 0, ctypes.byref(h)) == kvx.KVX_ERR_INVALID_ARG
+    # the fit takes translator inputs up to 512 wide: 8 grouped heads of 128 are 1024
+    wide = _desc(synth.ModelGeom(2, 16, 128, 1e6), ok_dst)
+    assert lib.kvx_fit_create(ctypes.byref(wide), 0.1, 0, ctypes.byref(h)) == kvx.KVX_ERR_UNSUPPORTED
+    assert h.value is None
+
+
+def test_fit_calls_reject_a_null_fitter(lib):
+    assert lib.kvx_fit_accumulate(None, None, None, None, None) == kvx.KVX_ERR_INVALID_ARG
+    assert lib.kvx_fit_solve(None, None, None, None, None) == kvx.KVX_ERR_INVALID_ARG
+    assert lib.kvx_fit_reset(None, None) == kvx.KVX_ERR_INVALID_ARG
+    assert lib.kvx_fit_tokens(None) == 0
+    assert lib.kvx_fit_destroy(None) == kvx.KVX_OK
+
+
+@pytest.mark.parametrize("src,dst,kw,code,words", [
+    (synth.ModelGeom(2, 2, 96, 1e6), synth.ModelGeom(2, 2, 128, 1e6), {}, kvx.KVX_ERR_UNSUPPORTED, "head dims"),
+    (synth.ModelGeom(2, 3, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), {}, kvx.KVX_ERR_UNSUPPORTED, "divides"),
+    (synth.ModelGeom(2, 4, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), dict(form=kvx.KVX_FORM_DENSE),
+     kvx.KVX_ERR_UNSUPPORTED, "per-KV-head"),
+    (synth.ModelGeom(2, 4, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), dict(layers_per_target=2),
+     kvx.KVX_ERR_UNSUPPORTED, "per-KV-head"),
+    (synth.ModelGeom(2, 4, 128, 1e6, rotary_dim=40), synth.ModelGeom(2, 2, 128, 1e6), {},
+     kvx.KVX_ERR_INVALID_ARG, "rope"),
+    (synth.ModelGeom(2, 4, 128, 1e6), synth.ModelGeom(2, 2, 128, 1e6), dict(dtype=7), kvx.KVX_ERR_INVALID_ARG,
+     "dtype"),
+])
+def test_static_entry_rejects_bad_descriptions_without_touching_cuda(lib, src, dst, kw, code, words):
+    d = _geom_desc(src, dst, **kw)
+    w = (ctypes.c_uint16 * 4)()
+    p = ctypes.cast(w, ctypes.c_void_p)
+    s, t, o = kvx.kvx_src_kv(), kvx.kvx_tgt_tokens(), kvx.kvx_dst_kv()
+    st = lib.kvx_translate_static(ctypes.byref(d), p, p, ctypes.byref(s), ctypes.byref(t), ctypes.byref(o), None,
+                                  None)
+    assert st == code
+    assert words in lib.kvx_static_last_error().decode()
+    assert lib.kvx_translate_static(None, p, p, ctypes.byref(s), ctypes.byref(t), ctypes.byref(o), None, None) == \
+        kvx.KVX_ERR_INVALID_ARG
