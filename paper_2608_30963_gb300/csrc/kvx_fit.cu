@@ -400,8 +400,9 @@ extern "C" KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, do
         return st;
     }
     if (f->geo.in_dim > 512) {
+        const int in_dim = f->geo.in_dim;
         delete f;
-        return fit_fail(KVX_ERR_UNSUPPORTED, "fit_create: translator input width %d > 512", f->geo.in_dim);
+        return fit_fail(KVX_ERR_UNSUPPORTED, "fit_create: translator input width %d > 512", in_dim);
     }
     const kvx_translator_desc& D = f->geo.desc;
     f->lambda = lambda;

@@ -311,9 +311,10 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
     t->tc = tc_config(t->in_dim, d.head_dim, s.head_dim);
     const bool tc_ok = desc->dtype == KVX_BF16 && t->tc.ok;
     if (desc->path == KVX_PATH_TCGEN05 && !tc_ok) {
+        const int in_dim = t->in_dim;
         delete t;
         return fail(KVX_ERR_UNSUPPORTED, "create: no tcgen05 kernel for this geometry/dtype (in=%d, d_t=%d)",
-                    t->in_dim, d.head_dim);
+                    in_dim, d.head_dim);
     }
     t->path = (desc->path == KVX_PATH_SIMT || !tc_ok) ? KVX_PATH_SIMT : KVX_PATH_TCGEN05;
     if (t->path == KVX_PATH_SIMT && simt_smem_bytes(t->in_dim, d.head_dim) > 200 * 1024) {
