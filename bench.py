@@ -17,15 +17,11 @@ the max over ranks.
 from __future__ import annotations
 
 import argparse
-import hashlib
 import json
 import math
 import multiprocessing as mp
 import os
-import re
-import shutil
 import statistics
-import struct
 import subprocess
 import sys
 import tempfile
@@ -39,6 +35,7 @@ sys.path.insert(0, ROOT)
 from paper_2608_30963_gb300 import synth  # noqa: E402  (numpy only)
 
 DEFAULT_WORKLOAD = "qwen7b_to_qwen1p5b_4k"
+NOMINAL_HBM_GBS = 8000.0   # nominal HBM3e bandwidth of a GB300 (vendor figure, about 8 TB/s)
 METRIC = "translated KV tokens/s and ms/handoff at 4K (7B→1.5B shapes); % of roofline"
 
 
@@ -219,12 +216,13 @@ def main():
     ap.add_argument("--e2e-steps", type=int, default=10)
     ap.add_argument("--mode", default="translate", choices=["translate", "fit"],
                     help="translate: the hot path (default); fit: the closed-form translator fit's accumulation")
-    ap.add_argument("--rekey-traffic", metavar="REV",
-                    help="maintenance (no GPU): re-key profiles/traffic.json to the current sources if the "
-                         "identity kernel compiles to the same device code as at git revision REV")
+    ap.add_argument("--record-traffic", metavar="CSV",
+                    help="maintenance (no GPU): write profiles/traffic.json from an ncu --csv capture of one "
+                         "identity-kernel launch of --workload")
+    ap.add_argument("--traffic-command", default="", help="the ncu command that produced --record-traffic's CSV")
     args = ap.parse_args()
-    if args.rekey_traffic:
-        return rekey_traffic(args.rekey_traffic)
+    if args.record_traffic:
+        return record_traffic(args.record_traffic, args.workload, args.traffic_command)
     args.warmup = max(args.warmup, 3)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -436,6 +434,39 @@ def main():
     if tr.device_status() != 0:
         raise RuntimeError("device status nonzero after the end-to-end steps")
 
+    # the host-link ceiling of the same copies with no translation: H2D alone, D2H alone, and
+    # both directions at once on two streams (what the overlapped end-to-end steps need per step)
+    def timed_copies(h2d_on, d2h_on, reps=3):
+        best = float("inf")
+        src_k, src_v, dk, dv = sets[0]
+        for _ in range(reps):
+            torch.cuda.synchronize()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(s_in)
+            s_out.wait_stream(s_in)
+            if h2d_on:
+                with torch.cuda.stream(s_in):
+                    for l in mapped:
+                        src_k[l].copy_(host_k[l], non_blocking=True)
+                        src_v[l].copy_(host_v[l], non_blocking=True)
+            if d2h_on:
+                with torch.cuda.stream(s_out):
+                    for j in range(Lt):
+                        host_out[0][j].copy_(dk[j], non_blocking=True)
+                        host_out[0][Lt + j].copy_(dv[j], non_blocking=True)
+            s_in.wait_stream(s_out)
+            b.record(s_in)
+            torch.cuda.synchronize()
+            best = min(best, a.elapsed_time(b))
+        return best
+
+    h2d_ms, d2h_ms, both_ms = timed_copies(True, False), timed_copies(False, True), timed_copies(True, True)
+    copy_ceiling = {"h2d_ms": h2d_ms, "d2h_ms": d2h_ms, "both_ms": both_ms,
+                    "h2d_gbs": h2d / (h2d_ms / 1e3) / 1e9, "d2h_gbs": d2h / (d2h_ms / 1e3) / 1e9,
+                    "tokens_per_s": wl.total_tgt / (both_ms / 1e3),
+                    "how": "the step's pinned copies alone (no translation), best of 3: H2D, D2H, and both "
+                           "directions at once on two streams; tokens_per_s = target tokens / both_ms"}
+
     if rank != 0:
         if dist:
             dist.destroy_process_group()
@@ -488,6 +519,8 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved / hbm_peak, "traffic": traffic,
                      "peak_source": f"{peak_src} hbm_gbs (copy)",
+                     # the same achieved bandwidth against the nominal HBM3e figure (about 8 TB/s)
+                     "nominal_peak": NOMINAL_HBM_GBS, "frac_nominal": achieved / NOMINAL_HBM_GBS,
                      "algorithmic_bytes_per_launch": alg["bytes"], "avg_launch_ms": avg_launch_ms,
                      "tensor_tflops": alg["flops"] / (avg_launch_ms / 1e3) / 1e12},
         "clocks": clk,
@@ -498,7 +531,9 @@ def main():
                         "from pinned memory, " +
                         ("kvx_build_alignment, " if align is not None else "") +
                         "kvx_translate, D2H of the target caches; consecutive steps overlap on three streams "
-                        "over two buffer sets")},
+                        "over two buffer sets"),
+                "copy_ceiling": copy_ceiling,
+                "frac_of_copy_ceiling": e2e_value / copy_ceiling["tokens_per_s"]},
         "gpu_launches": args.steps * (tr.launches_per_translate() + (1 if align is not None else 0)),
         "kernel_path": ({1: "simt", 2: "tcgen05"}.get(info.path, str(info.path)) +
                         ("+tma_identity" if info.path == 2 and span_lo is None else "")),
@@ -644,61 +679,49 @@ def kernel_rev(sources=None) -> str:
 
 
 _TRAFFIC_REC = os.path.join(ROOT, "profiles", "traffic.json")
+_TRAFFIC_SOURCES = ["paper_2608_30963_gb300/csrc/kvx_tc_aligned.cu", "paper_2608_30963_gb300/csrc/kvx_tc_common.cuh",
+                    "paper_2608_30963_gb300/csrc/kvx_common.cuh", "paper_2608_30963_gb300/csrc/kvx_kernels.h",
+                    "include/kvx.h"]
+_UNITS = {"byte": 1, "kbyte": 1e3, "mbyte": 1e6, "gbyte": 1e9, "nsecond": 1e-9, "usecond": 1e-6,
+          "msecond": 1e-3, "second": 1}
 
 
-def _cubin_sections(path):
-    b = open(path, "rb").read()
-    shoff = struct.unpack_from("<Q", b, 0x28)[0]
-    shentsize, shnum, shstrndx = struct.unpack_from("<HHH", b, 0x3A)
-    hdrs = [struct.unpack_from("<IIQQQQIIQQ", b, shoff + i * shentsize) for i in range(shnum)]
-    stro = hdrs[shstrndx][4]
-    out = {}
-    for h in hdrs:
-        end = b.index(b"\0", stro + h[0])
-        name = re.sub(r"_GLOBAL__N__[0-9a-f]+_", "_GLOBAL__N__", b[stro + h[0]:end].decode())
-        if name in (".shstrtab", ".strtab", ".symtab"):
+def record_traffic(csv_path: str, workload: str, command: str) -> int:
+    """Writes profiles/traffic.json from the CSV that `ncu --csv --metrics
+    gpu__time_duration.sum,dram__bytes_read.sum,dram__bytes_write.sum -k regex:aligned -c 1`
+    printed for one launch of the identity-alignment kernel, keyed to the hash of the kernel's
+    sources as they are now (a later change to them leaves the bench's traffic null)."""
+    import csv
+    rows = [r for r in csv.reader(l for l in open(csv_path) if l.startswith('"'))]
+    head, body = rows[0], rows[1:]
+    col = {n: i for i, n in enumerate(head)}
+    vals = {}
+    kernel = None
+    for r in body:
+        if "aligned" not in r[col["Kernel Name"]]:
             continue
-        data = b[h[4]:h[4] + h[5]] if h[1] != 8 else b""
-        out[name] = (h[5], hashlib.sha256(data).hexdigest())
-    return out
-
-
-def _aligned_cubin(tree, out):
-    subprocess.check_call(["nvcc", "-gencode", "arch=compute_103a,code=sm_103a", "-O3", "-std=c++17",
-                           "-I" + os.path.join(tree, "include"), "-cubin",
-                           os.path.join(tree, "paper_2608_30963_gb300", "csrc", "kvx_tc_aligned.cu"), "-o", out])
-    return _cubin_sections(out)
-
-
-def rekey_traffic(rev) -> int:
-    """Re-keys profiles/traffic.json to the current sources if the identity-alignment kernel
-    compiles to the same device code as at revision `rev`, the one whose DRAM traffic the record
-    holds: both revisions' kvx_tc_aligned.cu are compiled for sm_103a to cubins (no line info)
-    and every ELF section is compared by size and sha256 (the translation unit's anonymous-
-    namespace tag in section names normalised).  Only whole-section hashes are compared; no code
-    is decoded."""
-    tmp = tempfile.mkdtemp()
-    try:
-        old = os.path.join(tmp, "old")
-        subprocess.check_call(["git", "-C", ROOT, "worktree", "add", "-q", "--detach", old, rev])
-        try:
-            a = _aligned_cubin(old, os.path.join(tmp, "old.cubin"))
-        finally:
-            subprocess.call(["git", "-C", ROOT, "worktree", "remove", "--force", old])
-        b = _aligned_cubin(ROOT, os.path.join(tmp, "new.cubin"))
-    finally:
-        shutil.rmtree(tmp, ignore_errors=True)
-    diff = sorted(n for n in set(a) | set(b) if a.get(n) != b.get(n))
-    if diff:
-        print("device code differs in", len(diff), "sections, e.g.", diff[:3])
+        if kernel is None:
+            kernel = (r[col["ID"]], r[col["Kernel Name"]])
+        if r[col["ID"]] != kernel[0]:
+            continue
+        v = float(r[col["Metric Value"]].replace(",", ""))
+        vals[r[col["Metric Name"]]] = v * _UNITS.get(r[col["Metric Unit"]].lower(), 1)
+    need = ("dram__bytes_read.sum", "dram__bytes_write.sum")
+    if kernel is None or any(n not in vals for n in need):
+        print("no identity-kernel launch with DRAM counters in", csv_path)
         return 1
-    rec = json.load(open(_TRAFFIC_REC))
-    rec["kernel_rev"] = kernel_rev(rec["sources"])
-    rec["same_code_as"] = rev
+    rec = {"workload": workload, "kernel": kernel[1].split("(")[0],
+           "kernel_rev": kernel_rev(_TRAFFIC_SOURCES),
+           "dram_bytes_per_launch": int(round(vals[need[0]] + vals[need[1]])),
+           "dram_bytes_read": int(round(vals[need[0]])), "dram_bytes_write": int(round(vals[need[1]])),
+           "duration_s": vals.get("gpu__time_duration.sum"), "source": command,
+           "note": "dram__bytes_read.sum + dram__bytes_write.sum of one launch (writes still resident in L2 "
+                   "when the launch ends are not counted); kernel_rev hashes the listed sources",
+           "sources": _TRAFFIC_SOURCES}
     with open(_TRAFFIC_REC, "w") as f:
         json.dump(rec, f, indent=1)
         f.write("\n")
-    print("identical device code; kernel_rev", rec["kernel_rev"])
+    print(json.dumps(rec))
     return 0
 
 

@@ -222,7 +222,12 @@ typedef struct {
 /* Translate KV_A(C) into the target cache: KV^_B(C) = T_theta(KV_A(C)) (Sections 4 and 5).
  * Asynchronous on stream; allocates nothing; never synchronises.  The source, alignment and
  * position buffers must stay valid and unchanged until the work on stream completes.  Output
- * rows of distinct target tokens are written exactly once. */
+ * rows of distinct target tokens are written exactly once.
+ * Calls on one translator must be ordered: issue them on one stream, or serialise them on the
+ * host and order them on the device (events).  The translator owns per-call state that two
+ * overlapping calls would share: the span kernel's plan buffer on the device, the cache of
+ * source tensor descriptors and the launch count on the host.  Distinct translators may run
+ * concurrently on different streams and host threads. */
 KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
                                  const kvx_dst_kv* dst, void* stream);
 
@@ -341,12 +346,14 @@ KVX_API kvx_status kvx_fit_destroy(kvx_fitter* f);
  *     desc->dtype; they are copied into the scratch array on every call.  Both together must fit
  *     KVX_STATIC_SCRATCH_BYTES minus 2304 bytes, else KVX_ERR_UNSUPPORTED (nothing is launched).
  *   desc->path is ignored; desc->form must be KVX_FORM_GROUPED and desc->layers_per_target at
- *     most 1 (else KVX_ERR_UNSUPPORTED).
+ *     most 1, and the translator input width (r * src.head_dim, or src.head_dim when the target
+ *     has more KV heads) at most 512 (else KVX_ERR_UNSUPPORTED).  Paged targets are accepted.
  *   status_bits: host pointer or NULL.  If set, the call synchronises stream, writes the device
  *     status word there and returns KVX_ERR_DEVICE_STATUS when it is nonzero; if NULL, the call is
  *     asynchronous on stream like kvx_translate.
  * The first call on a device looks up the array's device address with that device current (a
- * one-time set-up); make that first call before any stream capture.  Every call shares the one
+ * one-time set-up, repeated when a call finds another driver context current than the one of
+ * the lookup, e.g. after cudaDeviceReset); make that first call before any stream capture.  Every call shares the one
  * array and clears the status word itself, so calls that overlap on the GPU (different streams,
  * or several host threads) race on the scratch and must be serialised by the caller.
  * Calls no cudaMalloc, cudaFree or other allocating routine.  Errors: kvx_static_last_error(). */

@@ -13,11 +13,11 @@ constexpr int KVX_MAX_ALIGNED_LAYERS = 96;   // target layers the identity-align
 constexpr int KVX_MAX_SRC_SLOTS = 256;       // (target layer, source-layer slot) pairs one launch addresses
 constexpr int KVX_MAX_ALIGNED_BATCH = 256;   // sequences whose metadata it keeps in shared memory
 
-// Rotation frequencies as fixed-point turns: turns[i] = round(2^64 * f_i / (2 pi)),
-// f_i = base^(-2i/d) (computed in double on the host).  For an integer position
-// p, p * turns[i] mod 2^64 is the fractional part of the angle p * f_i in turns,
-// exact up to the rounding of turns[i] (|error| <= p * 2^-53 turn), so the
-// range reduction costs one 64-bit multiply and no table of angles.
+// Rotation frequencies as fixed-point turns: turns[i] = 2^64 * f_i / (2 pi), evaluated in
+// double and converted to an integer by truncation, f_i = base^(-2i/d) (on the host).  For an
+// integer position p, p * turns[i] mod 2^64 is the fractional part of the angle p * f_i in
+// turns, exact up to the rounding of turns[i] (|error| <= p * 2^-52 turn), so the range
+// reduction costs one 64-bit multiply and no table of angles.
 struct RopeTable {
     const unsigned long long* turns;   // device [d/2]; entries of pairs that do not rotate are 0
     int half;                          // d/2

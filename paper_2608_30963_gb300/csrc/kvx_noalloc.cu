@@ -30,7 +30,28 @@ __device__ __align__(256) unsigned char g_static_scratch[KVX_STATIC_SCRATCH_BYTE
 
 constexpr int kMaxDevices = 64;
 std::mutex g_setup_mutex;
-unsigned char* g_scratch_addr[kMaxDevices];   // device address of g_static_scratch, per device
+// Device address of g_static_scratch per device, and the context it was looked up in: the
+// address belongs to that context, so a call under another context (a non-primary one, or the
+// primary context re-created after cudaDeviceReset) looks it up again.
+unsigned char* g_scratch_addr[kMaxDevices];
+void* g_scratch_ctx[kMaxDevices];
+
+// The calling thread's current driver context (NULL if it cannot be read).
+void* current_context()
+{
+    using GetCurrent = int (*)(void**);
+    static GetCurrent fn = [] {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess)
+            p = nullptr;
+        return (GetCurrent)p;
+    }();
+    void* ctx = nullptr;
+    if (!fn || fn(&ctx) != 0) return nullptr;
+    return ctx;
+}
 
 thread_local char g_msg[512];
 
@@ -43,8 +64,9 @@ kvx_status fail(kvx_status s, const char* fmt, ...)
     return s;
 }
 
-// Fixed-point rotation turns round(2^64 f_i / 2 pi), f_i the model's scheduled frequency
-// of pair i (0 for the pairs of a partial rotary head that do not rotate), written on the device.
+// Fixed-point rotation turns 2^64 f_i / 2 pi (in double, truncated to an integer, as on the
+// host), f_i the model's scheduled frequency of pair i (0 for the pairs of a partial rotary
+// head that do not rotate), written on the device.
 __global__ void static_turns_kernel(unsigned long long* out, const kvx_model_geom g)
 {
     const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -136,12 +158,14 @@ extern "C" KVX_API kvx_status kvx_translate_static(const kvx_translator_desc* de
     unsigned char* scratch = nullptr;
     {
         std::lock_guard<std::mutex> lock(g_setup_mutex);
-        if (!g_scratch_addr[dev]) {
+        void* ctx = current_context();
+        if (!g_scratch_addr[dev] || ctx != g_scratch_ctx[dev]) {
             void* ptr = nullptr;
             const cudaError_t ce = cudaGetSymbolAddress(&ptr, g_static_scratch);
             if (ce != cudaSuccess || !ptr)
                 return fail(KVX_ERR_CUDA, "translate_static: cudaGetSymbolAddress: %s", cudaGetErrorString(ce));
             g_scratch_addr[dev] = (unsigned char*)ptr;
+            g_scratch_ctx[dev] = current_context();   // the lookup made the runtime's context current
         }
         scratch = g_scratch_addr[dev];
     }
