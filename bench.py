@@ -220,9 +220,10 @@ def main():
                     help="maintenance (no GPU): write profiles/traffic.json from an ncu --csv capture of one "
                          "identity-kernel launch of --workload")
     ap.add_argument("--traffic-command", default="", help="the ncu command that produced --record-traffic's CSV")
+    ap.add_argument("--traffic-rev", default="", help="git revision whose sources the captured kernel was built from")
     args = ap.parse_args()
     if args.record_traffic:
-        return record_traffic(args.record_traffic, args.workload, args.traffic_command)
+        return record_traffic(args.record_traffic, args.workload, args.traffic_command, args.traffic_rev)
     args.warmup = max(args.warmup, 3)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -663,7 +664,7 @@ def fit_bench(args, spec):
     f.close()
 
 
-def kernel_rev(sources=None) -> str:
+def kernel_rev(sources=None, rev: str = "") -> str:
     """Hash of the sources a kernel is compiled from (its translation unit and the headers it
     includes, paths relative to the repository root; all kernel sources when None), so a stored
     ncu traffic figure is only used for the kernel it measured."""
@@ -674,7 +675,10 @@ def kernel_rev(sources=None) -> str:
         sources = [os.path.join(csrc, f) for f in sorted(os.listdir(os.path.join(ROOT, csrc)))
                    if f.endswith((".cu", ".cuh", ".h"))]
     for f in sources:
-        h.update(open(os.path.join(ROOT, f), "rb").read())
+        if rev:
+            h.update(subprocess.check_output(["git", "-C", ROOT, "show", f"{rev}:{f}"]))
+        else:
+            h.update(open(os.path.join(ROOT, f), "rb").read())
     return h.hexdigest()[:12]
 
 
@@ -683,14 +687,15 @@ _TRAFFIC_SOURCES = ["paper_2608_30963_gb300/csrc/kvx_tc_aligned.cu", "paper_2608
                     "paper_2608_30963_gb300/csrc/kvx_common.cuh", "paper_2608_30963_gb300/csrc/kvx_kernels.h",
                     "include/kvx.h"]
 _UNITS = {"byte": 1, "kbyte": 1e3, "mbyte": 1e6, "gbyte": 1e9, "nsecond": 1e-9, "usecond": 1e-6,
-          "msecond": 1e-3, "second": 1}
+          "msecond": 1e-3, "second": 1, "ns": 1e-9, "us": 1e-6, "ms": 1e-3, "s": 1}
 
 
-def record_traffic(csv_path: str, workload: str, command: str) -> int:
+def record_traffic(csv_path: str, workload: str, command: str, rev: str = "") -> int:
     """Writes profiles/traffic.json from the CSV that `ncu --csv --metrics
     gpu__time_duration.sum,dram__bytes_read.sum,dram__bytes_write.sum -k regex:aligned -c 1`
     printed for one launch of the identity-alignment kernel, keyed to the hash of the kernel's
-    sources as they are now (a later change to them leaves the bench's traffic null)."""
+    sources as they are now, or as git revision `rev` holds them when the capture ran on that
+    revision (a later change to them leaves the bench's traffic null)."""
     import csv
     rows = [r for r in csv.reader(l for l in open(csv_path) if l.startswith('"'))]
     head, body = rows[0], rows[1:]
@@ -710,8 +715,8 @@ def record_traffic(csv_path: str, workload: str, command: str) -> int:
     if kernel is None or any(n not in vals for n in need):
         print("no identity-kernel launch with DRAM counters in", csv_path)
         return 1
-    rec = {"workload": workload, "kernel": kernel[1].split("(")[0],
-           "kernel_rev": kernel_rev(_TRAFFIC_SOURCES),
+    rec = {"workload": workload, "kernel": kernel[1].split("(")[0].split("::")[-1],
+           "kernel_rev": kernel_rev(_TRAFFIC_SOURCES, rev),
            "dram_bytes_per_launch": int(round(vals[need[0]] + vals[need[1]])),
            "dram_bytes_read": int(round(vals[need[0]])), "dram_bytes_write": int(round(vals[need[1]])),
            "duration_s": vals.get("gpu__time_duration.sum"), "source": command,

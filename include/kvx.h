@@ -276,6 +276,16 @@ KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_translator_info* i
  * translation launch).  0 before the first call and after a call with no tokens. */
 KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
 
+/* Diagnostics of the token-span plan of the most recent kvx_translate on this translator, when
+ * that call ran the span kernel (its last chunk of up to 65536 target tokens).  The span kernel
+ * stages the source rows of each 32-token sub-tile as one window of consecutive rows (at most
+ * 48); a token whose span lies outside its sub-tile's window (a window cut at the cap, a span
+ * in another sequence, a non-monotone span) is gathered from global memory instead.
+ *   counts: host int64[4] = {sub-tiles, tokens staged in their window, tokens gathered from
+ *   global memory, sub-tiles with at least one such token}.
+ * Synchronises stream.  KVX_ERR_INVALID_ARG when the last call did not run the span kernel. */
+KVX_API kvx_status kvx_span_plan_stats(kvx_translator* tr, void* stream, int64_t* counts);
+
 /* ------------------------------------------------------------------------------------------
  * Closed-form fit of a linear translator (Section 5).  The paper gives the learning objective
  * L_KV = D(T_theta(KV_A(C)), KV_B(C)): the distance between the translated cache and the cache

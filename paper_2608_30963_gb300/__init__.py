@@ -92,7 +92,7 @@ class kvx_translator_info(ctypes.Structure):
 EXPORTS = ["kvx_translator_create", "kvx_translator_create_low_rank", "kvx_translate", "kvx_fit_create",
            "kvx_fit_accumulate", "kvx_fit_solve", "kvx_fit_reset", "kvx_fit_tokens", "kvx_fit_destroy", "kvx_build_alignment", "kvx_layer_map_nearest",
            "kvx_get_device_status", "kvx_get_info", "kvx_launches_per_translate", "kvx_last_error",
-           "kvx_destroy", "kvx_translate_static", "kvx_static_last_error"]
+           "kvx_destroy", "kvx_translate_static", "kvx_static_last_error", "kvx_span_plan_stats"]
 KVX_STATIC_SCRATCH_BYTES = 8 << 20
 
 _lib = None
@@ -148,6 +148,7 @@ def lib():
         L.kvx_fit_tokens.argtypes = [VP]
         L.kvx_fit_tokens.restype = ctypes.c_int64
         L.kvx_fit_destroy.argtypes = [VP]
+        L.kvx_span_plan_stats.argtypes = [VP, VP, ctypes.POINTER(ctypes.c_int64)]
         for name in EXPORTS:
             if name not in ("kvx_last_error", "kvx_launches_per_translate", "kvx_static_last_error",
                             "kvx_fit_tokens"):
@@ -226,6 +227,12 @@ def kvx_get_info(handle: int) -> kvx_translator_info:
 
 def kvx_launches_per_translate(handle: int) -> int:
     return lib().kvx_launches_per_translate(VP(handle))
+
+
+def kvx_span_plan_stats(handle: int, stream: int = 0) -> dict:
+    c = (ctypes.c_int64 * 4)()
+    _check(lib().kvx_span_plan_stats(VP(handle), VP(stream), c))
+    return {"subtiles": c[0], "staged_tokens": c[1], "global_tokens": c[2], "subtiles_with_global": c[3]}
 
 
 def kvx_destroy(handle: int):
@@ -368,6 +375,11 @@ class Translator:
         src, tgt, dst = _call_structs(src_k, src_v, src_seq_len, tgt_seq_off, total_tokens, dst_k, dst_v, span_lo,
                                       span_hi, src_pos, tgt_pos, page_table, page_size, num_pages)
         kvx_translate(self.handle, src, tgt, dst, _stream(stream))
+
+    def span_plan_stats(self, stream=None) -> dict:
+        """Token-span plan of the last translate (span kernel only): sub-tiles, tokens staged in
+        their sub-tile's window, tokens gathered from global memory."""
+        return kvx_span_plan_stats(self.handle, _stream(stream))
 
     def device_status(self, stream=None, clear: bool = True) -> int:
         return kvx_get_device_status(self.handle, _stream(stream), clear)

@@ -37,6 +37,7 @@ struct kvx_translator {
     static constexpr int kPlanTokens = 1 << 16;
     void* plan = nullptr;
     int last_launches = 0;       // kernel launches of the most recent kvx_translate
+    int last_span_tokens = 0;    // target tokens of the most recent call if it ran the span kernel, else 0
     // encoded source tensor maps of the identity-alignment kernel, a few per (target layer, K|V)
     struct MapEntry {
         const void* ptr = nullptr;
@@ -443,6 +444,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
     const kvx_translator_desc& D = tr->desc;
     const int Lt = D.dst.num_layers;
     tr->last_launches = 0;
+    tr->last_span_tokens = 0;
     TranslateParams P;
     char err[512];
     const kvx_status pst = make_params(tr->geo, tr->rope, tr->status, tr->w, src, tgt, dst, P, "translate", err);
@@ -472,6 +474,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
     } else if (tr->path == KVX_PATH_TCGEN05) {
         ce = launch_translate_tc(P, tr->tc, tr->num_sms, tr->plan, kvx_translator::kPlanTokens, (cudaStream_t)stream,
                                  &tr->last_launches);
+        tr->last_span_tokens = P.T_total;
     } else {
         ce = launch_translate_simt(P, D.dtype, (cudaStream_t)stream);
         tr->last_launches = 1;
@@ -525,6 +528,35 @@ extern "C" KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_transla
 }
 
 extern "C" KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr) { return tr ? tr->last_launches : 0; }
+
+extern "C" KVX_API kvx_status kvx_span_plan_stats(kvx_translator* tr, void* stream, int64_t* counts)
+{
+    if (!tr || !counts) return fail(KVX_ERR_INVALID_ARG, "span_plan_stats: NULL argument");
+    if (tr->last_span_tokens <= 0 || !tr->plan)
+        return fail(KVX_ERR_INVALID_ARG, "span_plan_stats: the last kvx_translate did not run the span kernel");
+    int nsub = 0, ent_off = 0;
+    tc_plan_layout(tr->last_span_tokens, kvx_translator::kPlanTokens, &nsub, &ent_off);
+    std::vector<int4> ent((size_t)nsub * 32);
+    CUDA_OR_FAIL(cudaStreamSynchronize((cudaStream_t)stream));
+    CUDA_OR_FAIL(cudaMemcpy(ent.data(), (const int4*)tr->plan + ent_off, ent.size() * sizeof(int4),
+                            cudaMemcpyDeviceToHost));
+    int64_t staged = 0, global = 0, subs_global = 0;
+    for (int sub = 0; sub < nsub; ++sub) {
+        bool any = false;
+        for (int i = 0; i < 32; ++i) {
+            const int4 e = ent[(size_t)sub * 32 + i];
+            if (((unsigned)e.x >> 16) >= 32u) continue;          // token past the end
+            if ((short)(e.x & 0xFFFF) < 0) { ++global; any = true; }
+            else ++staged;
+        }
+        subs_global += any;
+    }
+    counts[0] = nsub;
+    counts[1] = staged;
+    counts[2] = global;
+    counts[3] = subs_global;
+    return KVX_OK;
+}
 
 extern "C" KVX_API kvx_status kvx_destroy(kvx_translator* tr)
 {

@@ -31,6 +31,10 @@ size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht);
 cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
                                       int dt, int n_tile, int rhalf_t, cudaStream_t stream);
 size_t tc_plan_bytes(int tokens);
+// Where the plan of the last chunk of a span-kernel call lives in the plan buffer: its
+// sub-tile headers start at int4 0, its per-token entries (32 per sub-tile) at int4
+// *ent_off; *nsub sub-tiles.  T_total: target tokens of the call.
+void tc_plan_layout(int T_total, int plan_tokens, int* nsub, int* ent_off);
 // One span-plan launch and one translation launch per chunk of at most plan_tokens
 // target tokens; *launches receives the number of launches made.
 cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, void* plan,

@@ -879,6 +879,16 @@ size_t tc_plan_bytes(int tokens)
     return nsub * sizeof(int4) * (1 + kSub);
 }
 
+void tc_plan_layout(int T_total, int plan_tokens, int* nsub, int* ent_off)
+{
+    const int chunk = plan_tokens / kTileM * kTileM;
+    *ent_off = (chunk + kSub - 1) / kSub;
+    *nsub = 0;
+    if (chunk <= 0 || T_total <= 0) return;
+    const int last = (T_total - 1) / chunk * chunk;   // first token of the last chunk
+    *nsub = (T_total - last + kTileM - 1) / kTileM * kSubPerTile;
+}
+
 cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, int num_sms, void* plan,
                                 int plan_tokens, cudaStream_t stream, int* launches)
 {

@@ -7,6 +7,7 @@ cache a source model would hold.  Both sides then see bit-identical inputs.
 from __future__ import annotations
 
 import dataclasses
+import os
 from typing import Dict, List, Optional, Sequence
 
 import numpy as np
@@ -40,8 +41,10 @@ class Case:
 
 
 def make_case(spec: synth.WorkloadSpec, tgt_lens=None, layers: Optional[Sequence[int]] = None,
-              pad_value: float = 0.0, src_pos=None, tgt_pos=None) -> Case:
-    wl = synth.make_workload(spec, tgt_lens)
+              pad_value: float = 0.0, src_pos=None, tgt_pos=None, wl: Optional[synth.Workload] = None) -> Case:
+    """Inputs of one workload (wl: a prepared workload, e.g. with spans from two independent
+    tokenisations; default: the spec's own)."""
+    wl = synth.make_workload(spec, tgt_lens) if wl is None else wl
     lm = wl.layer_map if wl.layer_map is not None else oracle.layer_map_nearest(spec.src.num_layers,
                                                                                 spec.dst.num_layers)
     need = sorted(set(int(x) for x in np.asarray(lm).reshape(-1))) if layers is None else sorted(set(layers))
@@ -82,8 +85,21 @@ def oracle_problem(c: Case) -> oracle.OracleProblem:
                                 form=s.form, k_layers=s.layers_per_target, low_rank=c.low_rank)
 
 
-def compare(gpu: np.ndarray, ref: np.ndarray, dtype: str) -> dict:
-    """Element-by-element comparison; returns stats, raises AssertionError on failure."""
+# Every comparison of the session: rel-L2, the literal max-abs and the count of elements above
+# 3e-2, next to the test that made it (written out by conftest.py when KVX_PARITY_RECORD names
+# a file, and summarised at the end of the run).
+RECORD: List[dict] = []
+
+
+def record(stats: dict, label: str = "") -> None:
+    test = os.environ.get("PYTEST_CURRENT_TEST", "").split(" ")[0]
+    RECORD.append(dict(stats, test=test, label=label))
+    print(f"parity {test} {label}: rel_l2={stats['rel_l2']:.3e} max_abs={stats['max_abs']:.4e} "
+          f"n_above_3e-2={stats['n_above_3e-2']} of {stats['n']}")
+
+
+def compare(gpu: np.ndarray, ref: np.ndarray, dtype: str, label: str = "") -> dict:
+    """Element-by-element comparison; records and returns stats, raises AssertionError on failure."""
     gpu = np.asarray(gpu, np.float64)
     ref = np.asarray(ref, np.float64)
     assert gpu.shape == ref.shape, (gpu.shape, ref.shape)
@@ -93,6 +109,7 @@ def compare(gpu: np.ndarray, ref: np.ndarray, dtype: str) -> dict:
     rel = float(np.linalg.norm(gpu - ref) / nref) if nref > 0 else float(np.linalg.norm(gpu - ref))
     stats = {"rel_l2": rel, "max_abs": float(err.max(initial=0.0)), "n": int(err.size),
              "n_above_3e-2": int((err > ABS_TOL).sum())}
+    record(stats, label)
     assert rel <= REL_L2, stats
     if dtype == "bf16":
         bound = ABS_TOL + BF16_HALF_ULP_REL * np.abs(ref)
@@ -124,3 +141,36 @@ def sample_rows(c: Case, n: int, seed: int = 0) -> List[tuple]:
         tp = toks[i % len(toks)] if i < 2 * len(toks) else int(r.integers(T))
         rows.append((j, h, kv, tp))
     return rows
+
+
+def tokenization_workload(spec: synth.WorkloadSpec, n_bytes: Sequence[int], mean_src: float, mean_tgt: float,
+                          key: int) -> synth.Workload:
+    """A workload whose sequences are two independent tokenisations of byte strings of the given
+    lengths (synth.draw_tokenizations), aligned by the oracle's builder: a finer target maps
+    several target tokens to one source token, a coarser one gives long spans."""
+    src_ends, tgt_ends = [], []
+    for i, nb in enumerate(n_bytes):
+        se, te = synth.draw_tokenizations(int(nb), mean_src, mean_tgt, key * 10 + i)
+        src_ends.append(se)
+        tgt_ends.append(te)
+    so = np.concatenate([[0], np.cumsum([len(x) for x in src_ends])]).astype(np.int32)
+    to = np.concatenate([[0], np.cumsum([len(x) for x in tgt_ends])]).astype(np.int32)
+    se, te = np.concatenate(src_ends).astype(np.int32), np.concatenate(tgt_ends).astype(np.int32)
+    lo, hi, n = oracle.build_alignment(so, se, to, te)
+    assert n == 0
+    src_len, tgt_len = np.diff(so).astype(np.int32), np.diff(to).astype(np.int32)
+    return synth.Workload(spec, len(n_bytes), src_len, tgt_len, to, so, int(src_len.max()), int(tgt_len.max()),
+                          lo, hi, se, te, None if spec.layer_map is None else np.array(spec.layer_map, np.int32))
+
+
+def explicit_span_workload(spec: synth.WorkloadSpec, src_lens: Sequence[int], span_lo, span_hi) -> synth.Workload:
+    """A workload with caller-chosen spans (packed over the sequences, indices within each),
+    e.g. non-monotone or overlapping ones no tokenizer pair produces."""
+    span_lo, span_hi = [np.asarray(x, np.int32) for x in span_lo], [np.asarray(x, np.int32) for x in span_hi]
+    tgt_len = np.array([len(x) for x in span_lo], np.int32)
+    src_len = np.array(src_lens, np.int32)
+    to = np.concatenate([[0], np.cumsum(tgt_len)]).astype(np.int32)
+    so = np.concatenate([[0], np.cumsum(src_len)]).astype(np.int32)
+    return synth.Workload(spec, len(src_lens), src_len, tgt_len, to, so, int(src_len.max()), int(tgt_len.max()),
+                          np.concatenate(span_lo), np.concatenate(span_hi), None, None,
+                          None if spec.layer_map is None else np.array(spec.layer_map, np.int32))

@@ -1,5 +1,8 @@
 """The closed-form translator fit (kvx_fit_*) against the oracle's fit, through the C ABI.
 
+W is compared element by element against a bound derived from the two sides' arithmetic
+(_elementwise_bound), and also through rel-L2 and recovery of a planted translator.
+
 The oracle solves the normal equations in double from exact span means; the library rounds
 the input rows X and the target rows Y to the cache dtype and sums X^T X, X^T Y in fp32.
 Tolerance for bf16: the rounding of X and Y is about 2^-9 / sqrt(3) ~ 1.1e-3 relative (RMS),
@@ -54,6 +57,69 @@ def _targets_from(c, wk, wv):
     if s.dtype == "bf16":
         tk, tv = synth.bf16_round(tk), synth.bf16_round(tv)
     return tk, tv
+
+
+def _elementwise_bound(c, tk, tv, lam, wk_ref, wv_ref):
+    """Per-element bound on |W_gpu - W_oracle| from the arithmetic of the two sides.
+
+    The oracle solves (X^T X + lam I) W = X^T Y in double from exact input rows X.  The library
+    rounds X (and, for K, the un-rotated target rows Y) to the cache dtype, sums X^T X and X^T Y
+    over the T tokens in fp32 and factors in fp32.  To first order, with A = (X^T X + lam I)^-1,
+    P = A X^T and the residual R = Y - X W:
+        dW = A dX^T R - P dX W + P dY  (+ the effect of the fp32 sums and factorisation).
+    Rounding to nearest leaves independent errors |dX_tk| <= u |X_tk| of variance u^2 X_tk^2 / 3
+    (u = 2^-8 for bf16), so each element of dW has the standard deviation
+        sigma = sqrt(u^2/3 [A^2 (X^2)^T R^2]) + sqrt(u^2/3 [P^2 X^2 W^2]) (+) sqrt(u_y^2/3 [P^2 Y^2])
+    (squares elementwise, products matrix products; the first two share dX and are added, the
+    third in quadrature).  The fp32 sums of T terms add, with the probabilistic rounding-error
+    bound of Higham and Mary (confidence factor 6), at most gamma = 6 sqrt(T) 2^-24 relative to
+    the sums of |terms|, and the fp32 Cholesky a backward error of about 3 in 2^-24 |G|:
+        gamma |A| (|X|^T |Y| + |X|^T |X| |W|) + 3 in 2^-24 |A| |G| |W|.
+    The bound is 6 sigma plus those terms, per (layer, head, K|V) group."""
+    s = c.spec
+    p = oracle_problem(c)
+    wl = c.wl
+    T = wl.total_tgt
+    bf = s.dtype == "bf16"
+    u = 2.0 ** -8 if bf else 4 * 2.0 ** -24
+    gamma = 6 * np.sqrt(T) * 2.0 ** -24
+    din, dt = s.group_in, s.dst.head_dim
+    seq = np.searchsorted(wl.tgt_seq_off, np.arange(T), side="right") - 1
+    out = []
+    for kv, tgt, wref in ((0, tk, wk_ref), (1, tv, wv_ref)):
+        bk = np.zeros_like(wref)
+        for j in range(s.dst.num_layers):
+            for h in range(s.dst.num_kv_heads):
+                X = np.stack([p.input_row(j, h, kv, tp) for tp in range(T)])
+                Y = np.empty((T, dt))
+                for tp in range(T):
+                    b = int(seq[tp])
+                    t = tp - int(wl.tgt_seq_off[b])
+                    y = np.asarray(tgt[j][b, h, t], np.float64)
+                    Y[tp] = oracle.rope_g(y, s.dst, float(t), -1) if kv == 0 and s.dst.rope_base > 0 else y
+                W = wref[j, h]
+                G = X.T @ X + lam * np.eye(din)
+                A = np.linalg.inv(G)
+                P = A @ X.T
+                R = Y - X @ W
+                u_y = u if (kv == 0 or not bf) else 0.0
+                s1 = np.sqrt(u * u / 3 * ((A * A) @ ((X * X).T @ (R * R))))
+                s3 = np.sqrt(u * u / 3 * ((P * P) @ ((X * X) @ (W * W))))
+                s2 = np.sqrt(u_y * u_y / 3 * ((P * P) @ (Y * Y)))
+                sigma = np.sqrt((s1 + s3) ** 2 + s2 ** 2)
+                aX, aW, aA = np.abs(X), np.abs(W), np.abs(A)
+                bk[j, h] = (6 * sigma + gamma * (aA @ (aX.T @ np.abs(Y) + (aX.T @ aX) @ aW))
+                            + 3 * din * 2.0 ** -24 * (aA @ (np.abs(G) @ aW)))
+        out.append(bk)
+    return out
+
+
+def _assert_elementwise(gpu, ref, bound, label):
+    err = np.abs(np.asarray(gpu, np.float64) - ref)
+    bad = err > bound
+    worst = float((err / np.maximum(bound, 1e-300)).max())
+    print(f"fit {label}: max |dW| {err.max():.3e}, worst |dW| / bound {worst:.3f}, max bound {bound.max():.3e}")
+    assert not bad.any(), (label, int(bad.sum()), worst)
 
 
 def _fit_gpu(c, tk, tv, lam, chunk=0, split=None, paged=False):
@@ -142,8 +208,10 @@ def test_fit_recovers_planted_translator_and_matches_oracle(name):
     gk, gv, bits, _ = _fit_gpu(c, tk, tv, lam)
     assert bits == 0
     ok, ov = oracle_problem(c).fit(list(tk), list(tv), lam)
-    for gpu, ref, true in ((gk, ok, w_true[0]), (gv, ov, w_true[1])):
+    bk, bv = _elementwise_bound(c, tk, tv, lam, ok, ov)
+    for gpu, ref, true, bound, lab in ((gk, ok, w_true[0], bk, "K"), (gv, ov, w_true[1], bv, "V")):
         assert np.all(np.isfinite(gpu))
+        _assert_elementwise(gpu, ref, bound, f"{name} {lab}")
         assert _rel(gpu, ref) <= 1e-2, _rel(gpu, ref)
         assert _rel(gpu, true) <= 1e-2, _rel(gpu, true)
         assert _rel(ref, true) <= 5e-3, _rel(ref, true)
@@ -159,6 +227,9 @@ def test_fit_fp32_tiny_matches_oracle_tightly():
     gk, gv, bits, _ = _fit_gpu(c, tk, tv, lam)
     ok, ov = oracle_problem(c).fit(list(tk), list(tv), lam)
     assert bits == 0
+    bk, bv = _elementwise_bound(c, tk, tv, lam, ok, ov)
+    _assert_elementwise(gk, ok, bk, "tiny fp32 K")
+    _assert_elementwise(gv, ov, bv, "tiny fp32 V")
     assert _rel(gk, ok) <= 1e-4 and _rel(gv, ov) <= 1e-4
 
 

@@ -113,6 +113,55 @@ def test_rope_equals_complex_multiplication():
             np.testing.assert_allclose(y, np.concatenate([w.real, w.imag]), rtol=0, atol=1e-9)
 
 
+def _complex_rope(x, base, pos, d_rot=None, scale=1.0):
+    """Half-split RoPE by complex multiplication: pairs (i, i + n/2) of the first n channels as
+    z_i = x_i + 1j x_{i+n/2}, turned by (pos / scale) * base^(-2i/n); other channels unchanged."""
+    d = x.shape[-1]
+    n = d if d_rot is None else d_rot
+    h = n // 2
+    z = x[..., :h].astype(np.float64) + 1j * x[..., h:n].astype(np.float64)
+    ang = (np.asarray(pos, np.float64)[..., None] / scale) * np.power(float(base), -2.0 * np.arange(h) / n)
+    w = z * np.exp(1j * ang)
+    return np.concatenate([w.real, w.imag, x[..., n:].astype(np.float64)], axis=-1)
+
+
+def test_rope_cache_rotates_each_row_at_its_own_position():
+    """The input-synthesis rotation of whole caches: row (b, h, s) turns by the position of
+    token s of sequence b, 0..S-1 without a position array, pos[b, s] with one, backwards for
+    sign -1; and under a schedule it equals the single-row map at the same position."""
+    rng = np.random.default_rng(13)
+    B, H, S, d = 2, 3, 40, 64
+    x = rng.standard_normal((B, H, S, d)).astype(np.float32)
+    base = 1e4
+    pos = rng.permutation(np.arange(5, 5 + B * S)).reshape(B, S).astype(np.int32) * 37
+    # default positions: token index
+    y = oracle.rope_cache(x, base)
+    np.testing.assert_allclose(y, _complex_rope(x, base, np.arange(S)[None, None, :]), rtol=0, atol=2e-6)
+    # explicit positions, per sequence and token, shared by the heads
+    yp = oracle.rope_cache(x, base, pos)
+    np.testing.assert_allclose(yp, _complex_rope(x, base, pos[:, None, :]), rtol=0, atol=2e-6)
+    assert np.abs(yp - y).max() > 0.1        # the position array is used
+    # sign -1 turns backwards, so it undoes sign +1 at the same positions
+    ym = oracle.rope_cache(x, base, pos, -1)
+    np.testing.assert_allclose(ym, _complex_rope(x, base, -pos[:, None, :]), rtol=0, atol=2e-6)
+    # schedules and partial rotary heads: row by row the single-row map (itself pinned above)
+    geoms = [synth.ModelGeom(1, H, d, 1e4, rope_type=synth.ROPE_LINEAR, rope_factor=4.0),
+             synth.ModelGeom(1, H, d, 1e4, rotary_dim=32), synth.LLAMA70B_SCALED]
+    for g in geoms:
+        xg = x if g.head_dim == d else rng.standard_normal((B, H, S, g.head_dim)).astype(np.float32)
+        yg = oracle.rope_cache(xg, g, pos)
+        for b in range(B):
+            for hh in range(H):
+                for s_ in (0, 1, S // 2, S - 1):
+                    ref = oracle.rope_g(xg[b, hh, s_], g, float(pos[b, s_]), +1)
+                    np.testing.assert_allclose(yg[b, hh, s_], ref, rtol=0, atol=4e-6)
+    # the linear schedule is plain RoPE at pos / factor; the partial head rotates its first 32 channels
+    lin = oracle.rope_cache(x, geoms[0], pos)
+    np.testing.assert_allclose(lin, _complex_rope(x, 1e4, pos[:, None, :], scale=4.0), rtol=0, atol=2e-6)
+    part = oracle.rope_cache(x, geoms[1], pos)
+    np.testing.assert_allclose(part, _complex_rope(x, 1e4, pos[:, None, :], d_rot=32), rtol=0, atol=2e-6)
+
+
 def test_rope_inverse_norm_and_relative_position():
     rng = np.random.default_rng(12)
     for d, base in ((64, 1e4), (128, 1e6), (256, 1e4)):
