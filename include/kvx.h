@@ -231,6 +231,39 @@ typedef struct {
 KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
                                  const kvx_dst_kv* dst, void* stream);
 
+/* Writing the translation into the target model's GPU.  In the paper's handoff (Section 6.1,
+ * Table 4) the source model's GPU translates, a peer-to-peer copy moves the translated state to
+ * the target model's GPU, and the target cache is assembled there.  kvx_translate_to_device
+ * runs on the source GPU (the current device, which holds the source caches and the translator)
+ * and leaves the translated rows in a target cache on dst_device:
+ *   KVX_PEER_STORES  the translation kernels write every target row straight into dst (16-byte
+ *                    stores issued by the kernel's threads, over the peer mapping when dst_device
+ *                    is another GPU): copy and cache assembly fused into the translation; any
+ *                    layout (contiguous or paged).  Needs kvx_enable_peer(dst_device) first
+ *                    when dst_device is not the current device.
+ *   KVX_PEER_STAGED  translate into `staging` (a contiguous cache on the current device with the
+ *                    same layout as dst), then one cudaMemcpyPeerAsync per target tensor copies
+ *                    its whole [batch][heads][max_seq][head_dim] extent (padding rows included)
+ *                    to dst.  Contiguous targets only (KVX_ERR_UNSUPPORTED for paged ones).
+ * dst_device equal to the current device is allowed in both modes (the same kernels and copies
+ * on one GPU).  Every dst (and staging) tensor must be memory of dst_device (the current
+ * device), else KVX_ERR_INVALID_ARG.  Asynchronous on stream; allocates nothing; the ordering
+ * rule of kvx_translate applies. */
+typedef enum {
+    KVX_PEER_STORES = 0,
+    KVX_PEER_STAGED = 1
+} kvx_peer_mode;
+
+/* Enables access from the current device to peer_device's memory (cudaDeviceEnablePeerAccess;
+ * a one-time set-up per device pair, idempotent, to be called outside stream capture).
+ * KVX_ERR_UNSUPPORTED when the devices cannot reach each other.  peer_device equal to the
+ * current device is accepted and does nothing. */
+KVX_API kvx_status kvx_enable_peer(int32_t peer_device);
+
+KVX_API kvx_status kvx_translate_to_device(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
+                                           const kvx_dst_kv* dst, int32_t dst_device, int32_t mode,
+                                           const kvx_dst_kv* staging, void* stream);
+
 /* Token-span alignment from byte offsets (a target token is aligned to the source tokens whose
  * last byte lies in its byte range; a target token that receives none takes the source token
  * holding its own last byte).  Tokenizer differences are among the model differences the
@@ -298,17 +331,19 @@ KVX_API kvx_status kvx_span_plan_stats(kvx_translator* tr, void* stream, int64_t
  * un-rotated source rows, exactly as kvx_translate forms it, rounded to the cache dtype) and
  * row t of Y is the target model's own cache row of token t with the target RoPE undone (K;
  * the rotation is orthogonal, so the distance is unchanged) or as stored (V).
- * The fitter accumulates X^T X and X^T Y over any number of calibration calls (fp32, on the
- * tensor cores through cuBLAS batched GEMMs over the groups), then solves all systems at once
- * (Cholesky factorisation on the device: in fp32 shared memory for in <= 256, in double above).  Forms as for kvx_translator_create;
- * latent adapters are not fitted (fit W, then factor it if wanted). */
+ * The fitter accumulates X^T X and X^T Y over any number of calibration calls in fp32 sums (on the
+ * tensor cores for bf16 caches with in + out <= 512 and in a multiple of 128, X and Y built on
+ * chip; on the CUDA cores otherwise), then solves all systems at once (Cholesky factorisation on
+ * the device: in fp32 shared memory for in <= 256, where a system whose factor shows a condition
+ * number above 1e3 is factored again in double; in double above).  Forms as for
+ * kvx_translator_create; latent adapters are not fitted (fit W, then factor it if wanted). */
 typedef struct kvx_fitter kvx_fitter;
 
 /* desc: the translator to fit (its dtype is the cache dtype; desc->path is ignored).
  * lambda: ridge weight, >= 0 (0 needs at least `in` well-spread tokens per system).
  * chunk_tokens: target tokens one accumulation pass handles (calls longer than this run in
  *   several passes); 0 = 4096.  The fitter holds (L_t * H_t * 2) * chunk_tokens * (in + out)
- *   cache-dtype elements of row workspace plus the fp32 sums.
+ *   cache-dtype elements of row workspace (none on the tensor-core path) plus the fp32 sums.
  * Requires in <= 512.  Synchronous; on success *out owns device memory until kvx_fit_destroy. */
 KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, double lambda, int32_t chunk_tokens,
                                   kvx_fitter** out);
@@ -324,9 +359,10 @@ KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv* src, cons
 /* Solve every system from the sums so far and write W_K and W_V as DEVICE arrays
  * [dst.num_layers][dst.num_kv_heads][in][out] of the desc dtype (the layout
  * kvx_translator_create takes).  Synchronises stream.  status_bits (host, may be NULL) receives
- * the fitter's status word: KVX_DEV_* bits from the accumulation passes (rows left out) and
- * 0x20 when a system was not positive definite (lambda = 0 with too few tokens; its W is zero),
- * in which case the call returns KVX_ERR_DEVICE_STATUS.  Calls on one fitter must be ordered
+ * the fitter's status word: KVX_DEV_* bits from the accumulation passes (rows left out), 0x20
+ * when a system was not positive definite (lambda = 0 with too few tokens; its W is zero), in
+ * which case the call returns KVX_ERR_DEVICE_STATUS, and 0x40 (informational) when
+ * ill-conditioned systems were factored in double.  Calls on one fitter must be ordered
  * (one stream, or synchronised by the caller). */
 KVX_API kvx_status kvx_fit_solve(kvx_fitter* f, void* w_k, void* w_v, uint32_t* status_bits, void* stream);
 

@@ -92,7 +92,9 @@ class kvx_translator_info(ctypes.Structure):
 EXPORTS = ["kvx_translator_create", "kvx_translator_create_low_rank", "kvx_translate", "kvx_fit_create",
            "kvx_fit_accumulate", "kvx_fit_solve", "kvx_fit_reset", "kvx_fit_tokens", "kvx_fit_destroy", "kvx_build_alignment", "kvx_layer_map_nearest",
            "kvx_get_device_status", "kvx_get_info", "kvx_launches_per_translate", "kvx_last_error",
-           "kvx_destroy", "kvx_translate_static", "kvx_static_last_error", "kvx_span_plan_stats"]
+           "kvx_destroy", "kvx_translate_static", "kvx_static_last_error", "kvx_span_plan_stats",
+           "kvx_enable_peer", "kvx_translate_to_device"]
+KVX_PEER_STORES, KVX_PEER_STAGED = 0, 1
 KVX_STATIC_SCRATCH_BYTES = 8 << 20
 
 _lib = None
@@ -149,6 +151,10 @@ def lib():
         L.kvx_fit_tokens.restype = ctypes.c_int64
         L.kvx_fit_destroy.argtypes = [VP]
         L.kvx_span_plan_stats.argtypes = [VP, VP, ctypes.POINTER(ctypes.c_int64)]
+        L.kvx_enable_peer.argtypes = [ctypes.c_int32]
+        L.kvx_translate_to_device.argtypes = [VP, ctypes.POINTER(kvx_src_kv), ctypes.POINTER(kvx_tgt_tokens),
+                                              ctypes.POINTER(kvx_dst_kv), ctypes.c_int32, ctypes.c_int32,
+                                              ctypes.POINTER(kvx_dst_kv), VP]
         for name in EXPORTS:
             if name not in ("kvx_last_error", "kvx_launches_per_translate", "kvx_static_last_error",
                             "kvx_fit_tokens"):
@@ -227,6 +233,17 @@ def kvx_get_info(handle: int) -> kvx_translator_info:
 
 def kvx_launches_per_translate(handle: int) -> int:
     return lib().kvx_launches_per_translate(VP(handle))
+
+
+def kvx_enable_peer(peer_device: int):
+    _check(lib().kvx_enable_peer(peer_device))
+
+
+def kvx_translate_to_device(handle: int, src: kvx_src_kv, tgt: kvx_tgt_tokens, dst: kvx_dst_kv, dst_device: int,
+                            mode: int, staging: Optional[kvx_dst_kv] = None, stream: int = 0):
+    _check(lib().kvx_translate_to_device(VP(handle), ctypes.byref(src), ctypes.byref(tgt), ctypes.byref(dst),
+                                         dst_device, mode, None if staging is None else ctypes.byref(staging),
+                                         VP(stream)))
 
 
 def kvx_span_plan_stats(handle: int, stream: int = 0) -> dict:
@@ -375,6 +392,23 @@ class Translator:
         src, tgt, dst = _call_structs(src_k, src_v, src_seq_len, tgt_seq_off, total_tokens, dst_k, dst_v, span_lo,
                                       span_hi, src_pos, tgt_pos, page_table, page_size, num_pages)
         kvx_translate(self.handle, src, tgt, dst, _stream(stream))
+
+    def translate_to_device(self, src_k: Sequence, src_v: Sequence, src_seq_len, tgt_seq_off, total_tokens: int,
+                            dst_k: Sequence, dst_v: Sequence, dst_device: int, mode: int = KVX_PEER_STORES, *,
+                            staging_k: Optional[Sequence] = None, staging_v: Optional[Sequence] = None,
+                            span_lo=None, span_hi=None, src_pos=None, tgt_pos=None, page_table=None,
+                            page_size: int = 16, num_pages: int = 0, stream=None):
+        """As translate, with the target cache on device dst_device (kvx_translate_to_device):
+        mode KVX_PEER_STORES writes it from the kernels, KVX_PEER_STAGED translates into
+        staging_k / staging_v (current device, same layout) and copies them over."""
+        src, tgt, dst = _call_structs(src_k, src_v, src_seq_len, tgt_seq_off, total_tokens, dst_k, dst_v, span_lo,
+                                      span_hi, src_pos, tgt_pos, page_table, page_size, num_pages)
+        stg = None
+        if staging_k is not None:
+            _, _, stg = _call_structs(src_k, src_v, src_seq_len, tgt_seq_off, total_tokens, staging_k, staging_v,
+                                      span_lo, span_hi, src_pos, tgt_pos, page_table, page_size, num_pages)
+        self._keep = (dst, stg)
+        kvx_translate_to_device(self.handle, src, tgt, dst, dst_device, mode, stg, _stream(stream))
 
     def span_plan_stats(self, stream=None) -> dict:
         """Token-span plan of the last translate (span kernel only): sub-tiles, tokens staged in

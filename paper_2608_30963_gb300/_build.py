@@ -8,7 +8,6 @@ from __future__ import annotations
 
 import glob
 import os
-import shutil
 import subprocess
 import sys
 
@@ -66,11 +65,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     if failed:
         raise RuntimeError("nvcc failed:\n" + "\n".join(failed))
     tmp = LIB + f".tmp{os.getpid()}"
-    # cuBLAS: the fitter's Gram contractions (plain batched GEMMs), found through the toolkit's
-    # library directory next to nvcc
-    cuda_lib = os.path.join(os.path.dirname(os.path.dirname(os.path.realpath(shutil.which(nvcc) or nvcc))), "lib64")
-    subprocess.check_call([nvcc, *ARCH, "-shared", "-o", tmp, *objs, "-L" + cuda_lib, "-lcublas",
-                           "-Xlinker", "-rpath," + cuda_lib])
+    subprocess.check_call([nvcc, *ARCH, "-shared", "-o", tmp, *objs])
     os.replace(tmp, LIB)
     return LIB
 

@@ -108,6 +108,8 @@ struct TranslateParams {
                             // rotary_dim/2 (= d/2 unless the head is partial rotary)
     int rope_same;   // source and target rotations coincide (same head_dim, same frequencies)
     int max_position;
+    int plain_stores;   // write target rows with 16-byte stores from the threads instead of the bulk-copy
+                        // unit (destinations on another device, reached over the peer mapping)
     unsigned* status;
     // weights (layout depends on the kernel)
     const void* w;

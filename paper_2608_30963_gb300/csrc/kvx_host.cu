@@ -5,6 +5,7 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -437,8 +438,10 @@ extern "C" KVX_API kvx_status kvx_translator_create_low_rank(const kvx_translato
     return st;
 }
 
-extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
-                                            const kvx_dst_kv* dst, void* stream)
+// The translation launch(es) of kvx_translate; plain_stores: the kernels write the target rows
+// with thread stores (a destination on another device).
+static kvx_status translate_impl(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
+                                 const kvx_dst_kv* dst, void* stream, int plain_stores)
 {
     if (!tr || !src || !tgt || !dst) return fail(KVX_ERR_INVALID_ARG, "translate: NULL argument");
     const kvx_translator_desc& D = tr->desc;
@@ -453,6 +456,7 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
         return pst;
     }
     if (tgt->total_tokens == 0) return KVX_OK;
+    P.plain_stores = plain_stores;
     cudaError_t ce;
     // partial rotary heads (rotary_dim < head_dim on either side) take the span kernel, which
     // pairs channels at rotary_dim/2; the identity kernel pairs whole heads
@@ -480,6 +484,104 @@ extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv
         tr->last_launches = 1;
     }
     if (ce != cudaSuccess) return fail(KVX_ERR_CUDA, "translate: launch failed: %s", cudaGetErrorString(ce));
+    return KVX_OK;
+}
+
+extern "C" KVX_API kvx_status kvx_translate(kvx_translator* tr, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
+                                            const kvx_dst_kv* dst, void* stream)
+{
+    return translate_impl(tr, src, tgt, dst, stream, 0);
+}
+
+// ---------------------------------------------------------------------------------------------
+// Writing the translated cache into the target model's GPU (the handoff's peer copy).
+static std::mutex g_peer_mutex;
+static unsigned long long g_peer_enabled[64];   // [device] bit p: peer access to device p enabled by kvx_enable_peer
+
+extern "C" KVX_API kvx_status kvx_enable_peer(int32_t peer_device)
+{
+    int cur = 0, n = 0;
+    CUDA_OR_FAIL(cudaGetDevice(&cur));
+    CUDA_OR_FAIL(cudaGetDeviceCount(&n));
+    if (peer_device < 0 || peer_device >= n || peer_device >= 64 || cur >= 64)
+        return fail(KVX_ERR_INVALID_ARG, "enable_peer: no device %d", peer_device);
+    if (peer_device == cur) return KVX_OK;
+    std::lock_guard<std::mutex> lock(g_peer_mutex);
+    if (g_peer_enabled[cur] >> peer_device & 1ull) return KVX_OK;
+    int can = 0;
+    CUDA_OR_FAIL(cudaDeviceCanAccessPeer(&can, cur, peer_device));
+    if (!can) return fail(KVX_ERR_UNSUPPORTED, "enable_peer: device %d cannot access device %d", cur, peer_device);
+    cudaError_t e = cudaDeviceEnablePeerAccess(peer_device, 0);
+    if (e == cudaErrorPeerAccessAlreadyEnabled) {
+        cudaGetLastError();   // already enabled by the caller: not an error here
+        e = cudaSuccess;
+    }
+    if (e != cudaSuccess) return fail(KVX_ERR_CUDA, "enable_peer: %s", cudaGetErrorString(e));
+    g_peer_enabled[cur] |= 1ull << peer_device;
+    return KVX_OK;
+}
+
+// Device of a caller pointer (-1 if it is not device memory).
+static int pointer_device(const void* p)
+{
+    cudaPointerAttributes a{};
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        cudaGetLastError();
+        return -1;
+    }
+    return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged ? a.device : -1;
+}
+
+extern "C" KVX_API kvx_status kvx_translate_to_device(kvx_translator* tr, const kvx_src_kv* src,
+                                                      const kvx_tgt_tokens* tgt, const kvx_dst_kv* dst,
+                                                      int32_t dst_device, int32_t mode, const kvx_dst_kv* staging,
+                                                      void* stream)
+{
+    if (!tr || !src || !tgt || !dst) return fail(KVX_ERR_INVALID_ARG, "translate_to_device: NULL argument");
+    int cur = 0;
+    CUDA_OR_FAIL(cudaGetDevice(&cur));
+    const int Lt = tr->desc.dst.num_layers;
+    if (!dst->k || !dst->v) return fail(KVX_ERR_INVALID_ARG, "translate_to_device: NULL array");
+    for (int j = 0; j < Lt; ++j)
+        for (const void* p : {(const void*)dst->k[j], (const void*)dst->v[j]})
+            if (p && pointer_device(p) != dst_device)
+                return fail(KVX_ERR_INVALID_ARG, "translate_to_device: target layer %d is not memory of device %d",
+                            j, dst_device);
+    if (mode == KVX_PEER_STORES) {
+        if (dst_device != cur) {
+            std::lock_guard<std::mutex> lock(g_peer_mutex);
+            if (cur >= 64 || dst_device < 0 || dst_device >= 64 || !(g_peer_enabled[cur] >> dst_device & 1ull))
+                return fail(KVX_ERR_INVALID_ARG, "translate_to_device: call kvx_enable_peer(%d) on device %d first",
+                            dst_device, cur);
+        }
+        return translate_impl(tr, src, tgt, dst, stream, 1);
+    }
+    if (mode != KVX_PEER_STAGED) return fail(KVX_ERR_INVALID_ARG, "translate_to_device: unknown mode %d", mode);
+    if (!staging || !staging->k || !staging->v)
+        return fail(KVX_ERR_INVALID_ARG, "translate_to_device: the staged mode needs a staging cache");
+    if (dst->paged || staging->paged)
+        return fail(KVX_ERR_UNSUPPORTED, "translate_to_device: the staged mode copies whole contiguous caches; "
+                                         "write paged pools with KVX_PEER_STORES");
+    if (staging->stride_b != dst->stride_b || staging->stride_h != dst->stride_h ||
+        staging->stride_t != dst->stride_t || staging->max_seq != dst->max_seq)
+        return fail(KVX_ERR_INVALID_ARG, "translate_to_device: staging and target caches differ in layout");
+    for (int j = 0; j < Lt; ++j)
+        for (const void* p : {(const void*)staging->k[j], (const void*)staging->v[j]})
+            if (p && pointer_device(p) != cur)
+                return fail(KVX_ERR_INVALID_ARG, "translate_to_device: staging layer %d is not memory of device %d",
+                            j, cur);
+    const kvx_status st = translate_impl(tr, src, tgt, staging, stream, 0);
+    if (st != KVX_OK || tgt->total_tokens == 0) return st;
+    // every staged tensor, whole: [batch][heads][max_seq][head_dim] under the strides
+    const size_t elt = tr->desc.dtype == KVX_BF16 ? 2 : 4;
+    const int64_t extent = (int64_t)(src->batch - 1) * dst->stride_b + (int64_t)(tr->desc.dst.num_kv_heads - 1) * dst->stride_h +
+                           (int64_t)(dst->max_seq > 0 ? dst->max_seq - 1 : 0) * dst->stride_t + tr->desc.dst.head_dim;
+    for (int j = 0; j < Lt; ++j)
+        for (int kv = 0; kv < 2; ++kv) {
+            void* to = kv ? dst->v[j] : dst->k[j];
+            const void* from = kv ? staging->v[j] : staging->k[j];
+            CUDA_OR_FAIL(cudaMemcpyPeerAsync(to, dst_device, from, cur, (size_t)extent * elt, (cudaStream_t)stream));
+        }
     return KVX_OK;
 }
 

@@ -533,8 +533,12 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             if (half == 0 && valid && dst_off >= 0) {
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      dst_head_off(P, x.h);
-                store_row_slots(dst, srow_u32, x.nt * hw, hw, half_t, P.rhalf_t);
-                bulk_commit();
+                if (P.plain_stores) {
+                    store_row_slots_plain(dst, srow, x.nt * hw, hw, half_t, P.rhalf_t);
+                } else {
+                    store_row_slots(dst, srow_u32, x.nt * hw, hw, half_t, P.rhalf_t);
+                    bulk_commit();
+                }
             }
             ++tcount;
         }

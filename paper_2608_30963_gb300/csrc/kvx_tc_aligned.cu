@@ -79,6 +79,7 @@ struct AlignedParams {
     int max_pages, page_size, num_pages;
     RopeTable rs, rt;
     int max_position;
+    int plain_stores;   // target rows written with 16-byte thread stores (a peer device's cache)
     unsigned* status;
     const void* w;
     unsigned idesc, tmem_cols, b_bytes, stage_row_bytes;
@@ -469,13 +470,15 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             if ((lane & 1) == half && valid && dst_off >= 0) {   // the quadrant's rows, split between its two warps
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      (P.paged ? (long long)x.h * P.dt : (long long)x.h * P.dh);
-                if (P.n_split == 1) {
+                if (P.plain_stores) {
+                    store_row_slots_plain(dst, srow, x.nt * hw, hw, P.dt >> 1, P.dt >> 1);
+                } else if (P.n_split == 1) {
                     bulk_s2g(dst, srow_u32, (uint32_t)P.dt * 2);
                 } else {
                     bulk_s2g(dst + x.nt * hw, srow_u32, (uint32_t)hw * 2);
                     bulk_s2g(dst + (P.dt >> 1) + x.nt * hw, srow_u32 + hw * 2, (uint32_t)hw * 2);
                 }
-                bulk_commit();
+                if (!P.plain_stores) bulk_commit();
             }
             ++tcount;
         }
@@ -683,6 +686,7 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     P.paged = T.paged; P.dst_max_seq = T.dst_max_seq; P.db = T.db; P.dh = T.dh; P.dts = T.dts;
     P.page_table = T.page_table; P.max_pages = T.max_pages; P.page_size = T.page_size; P.num_pages = T.num_pages;
     P.rs = T.rs; P.rt = T.rt; P.max_position = T.max_position; P.status = T.status; P.w = T.w;
+    P.plain_stores = T.plain_stores;
     P.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(P.n_tile >> 3) << 17) | ((uint32_t)(kTileM >> 4) << 24);
     P.share_cs = T.rs.enabled && T.rt.enabled && T.ds == T.dt && !T.src_pos && !T.tgt_pos &&
                  T.rope_same && 2 * P.n_tile + 2 * T.dt <= 512;

@@ -123,6 +123,28 @@ __device__ __forceinline__ void store_row_slots(__nv_bfloat16* dst, uint32_t sro
         bulk_s2g(dst + a + n_rot + half, srow + (uint32_t)(hw + n_rot) * 2, (uint32_t)(hw - n_rot) * 2);
     }
 }
+// The same runs as store_row_slots, written by the calling thread with 16-byte stores (for
+// a target cache on another device, written through the peer mapping).
+__device__ __forceinline__ void store_row_slots_plain(__nv_bfloat16* dst, const uint8_t* srow, int a, int hw, int half,
+                                                      int rhalf)
+{
+    auto run = [](__nv_bfloat16* d, const uint8_t* s, int n) {
+        for (int i = 0; i < n; i += 8) *reinterpret_cast<uint4*>(d + i) = *reinterpret_cast<const uint4*>(s + 2 * i);
+    };
+    if (hw == half && rhalf == half) {
+        run(dst, srow, 2 * half);
+        return;
+    }
+    const int n_rot = min(max(rhalf - a, 0), hw);
+    if (n_rot > 0) {
+        run(dst + a, srow, n_rot);
+        run(dst + a + rhalf, srow + hw * 2, n_rot);
+    }
+    if (n_rot < hw) {
+        run(dst + a + n_rot + rhalf, srow + n_rot * 2, hw - n_rot);
+        run(dst + a + n_rot + half, srow + (hw + n_rot) * 2, hw - n_rot);
+    }
+}
 __device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait_read0() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
 __device__ __forceinline__ void bulk_wait0() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }

@@ -59,12 +59,12 @@ def _targets_from(c, wk, wv):
     return tk, tv
 
 
-def _elementwise_bound(c, tk, tv, lam, wk_ref, wv_ref):
+def _elementwise_bound(c, tk, tv, lam, wk_ref, wv_ref, chol_u=2.0 ** -24):
     """Per-element bound on |W_gpu - W_oracle| from the arithmetic of the two sides.
 
     The oracle solves (X^T X + lam I) W = X^T Y in double from exact input rows X.  The library
     rounds X (and, for K, the un-rotated target rows Y) to the cache dtype, sums X^T X and X^T Y
-    over the T tokens in fp32 and factors in fp32.  To first order, with A = (X^T X + lam I)^-1,
+    over the T tokens in fp32 and factors in fp32 (or double).  To first order, with A = (X^T X + lam I)^-1,
     P = A X^T and the residual R = Y - X W:
         dW = A dX^T R - P dX W + P dY  (+ the effect of the fp32 sums and factorisation).
     Rounding to nearest leaves independent errors |dX_tk| <= u |X_tk| of variance u^2 X_tk^2 / 3
@@ -73,8 +73,9 @@ def _elementwise_bound(c, tk, tv, lam, wk_ref, wv_ref):
     (squares elementwise, products matrix products; the first two share dX and are added, the
     third in quadrature).  The fp32 sums of T terms add, with the probabilistic rounding-error
     bound of Higham and Mary (confidence factor 6), at most gamma = 6 sqrt(T) 2^-24 relative to
-    the sums of |terms|, and the fp32 Cholesky a backward error of about 3 in 2^-24 |G|:
-        gamma |A| (|X|^T |Y| + |X|^T |X| |W|) + 3 in 2^-24 |A| |G| |W|.
+    the sums of |terms|, and the Cholesky factorisation a backward error of about 3 in u_c |G|
+    (u_c = 2^-24 for the fp32 factor, 2^-53 where the library factors in double):
+        gamma |A| (|X|^T |Y| + |X|^T |X| |W|) + 3 in u_c |A| |G| |W|.
     The bound is 6 sigma plus those terms, per (layer, head, K|V) group."""
     s = c.spec
     p = oracle_problem(c)
@@ -109,7 +110,7 @@ def _elementwise_bound(c, tk, tv, lam, wk_ref, wv_ref):
                 sigma = np.sqrt((s1 + s3) ** 2 + s2 ** 2)
                 aX, aW, aA = np.abs(X), np.abs(W), np.abs(A)
                 bk[j, h] = (6 * sigma + gamma * (aA @ (aX.T @ np.abs(Y) + (aX.T @ aX) @ aW))
-                            + 3 * din * 2.0 ** -24 * (aA @ (np.abs(G) @ aW)))
+                            + 3 * din * chol_u * (aA @ (np.abs(G) @ aW)))
         out.append(bk)
     return out
 
@@ -183,6 +184,10 @@ CASES = {
                                 dict(src=synth.ModelGeom(3, 4, 128, 1e6, rotary_dim=64),
                                      dst=synth.ModelGeom(2, 2, 128, 1e6, rotary_dim=32))),
     # dense per-layer form over 2 source heads of 128 (in = 256), cross-tokenizer spans
+    # 64-channel heads: in = 64 is not a multiple of the tensor-core row block (128), so the
+    # CUDA-core Gram path runs on bf16 caches
+    "small_heads_cuda_core": ("qwen7b_to_qwen1p5b_4k", 3, 2, [900, 300], dict(src=synth.ModelGeom(3, 2, 64, 1e6),
+                                                                             dst=synth.ModelGeom(2, 2, 64, 1e4))),
     "dense_spans": ("llama70b_to_qwen7b_8k", 4, 2, [1100, 700], dict(form=synth.FORM_DENSE,
                                                                    src=synth.ModelGeom(4, 2, 128, 5e5),
                                                                    dst=synth.ModelGeom(2, 2, 64, 1e6))),
@@ -231,6 +236,37 @@ def test_fit_fp32_tiny_matches_oracle_tightly():
     _assert_elementwise(gk, ok, bk, "tiny fp32 K")
     _assert_elementwise(gv, ov, bv, "tiny fp32 V")
     assert _rel(gk, ok) <= 1e-4 and _rel(gv, ov) <= 1e-4
+
+
+def test_fit_ill_conditioned_calibration_matches_oracle():
+    """A calibration set whose two source heads nearly coincide (head 1 = head 0 + 3e-3 noise):
+    X^T X + lambda I has a condition number above 1e6, where an fp32 Cholesky factor loses most
+    of its digits.  The fitter sees it in the factor's pivots and factors those systems again in
+    double (status bit 0x40); W then matches the oracle's fp64 solution within the bound of the
+    fp32 sums and a double factorisation.  fp32 caches, so the rows carry no bf16 rounding."""
+    spec = SPECS["tiny_fp32"]
+    c = make_case(spec, [456])
+    rng = np.random.default_rng(21)
+    for d in (c.src_k, c.src_v):
+        for l in d:
+            d[l][:, 1] = d[l][:, 0] + np.float32(3e-3) * rng.standard_normal(d[l][:, 0].shape).astype(np.float32)
+    w_true = [rng.standard_normal((2, 1, 128, 64)).astype(np.float32) / np.float32(np.sqrt(128)) for _ in range(2)]
+    tk, tv = _targets_from(c, *w_true)
+    tk = tk + np.float32(1e-3) * rng.standard_normal(tk.shape).astype(np.float32)   # not an exact fit
+    tv = tv + np.float32(1e-3) * rng.standard_normal(tv.shape).astype(np.float32)
+    lam = 1e-4
+    gk, gv, bits, _ = _fit_gpu(c, tk, tv, lam)
+    assert bits & 0x40, f"status 0x{bits:x}: no system was solved in double"
+    assert not bits & 0x20
+    ok, ov = oracle_problem(c).fit(list(tk), list(tv), lam)
+    p = oracle_problem(c)
+    X = np.stack([p.input_row(0, 0, 0, tp) for tp in range(c.wl.total_tgt)])
+    ev = np.linalg.eigvalsh(X.T @ X + lam * np.eye(X.shape[1]))
+    print(f"ill-conditioned fit: cond(X^T X + lambda I) = {ev[-1] / ev[0]:.3e}")
+    assert ev[-1] / ev[0] > 1e6
+    bk, bv = _elementwise_bound(c, tk, tv, lam, ok, ov, chol_u=2.0 ** -53)
+    _assert_elementwise(gk, ok, bk, "ill-conditioned K")
+    _assert_elementwise(gv, ov, bv, "ill-conditioned V")
 
 
 def test_fit_two_calls_chunked_and_paged_agree_with_one_call():
