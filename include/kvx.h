@@ -309,6 +309,16 @@ KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_translator_info* i
  * translation launch).  0 before the first call and after a call with no tokens. */
 KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr);
 
+/* Diagnostics of the kernels' bounded waits (the failure-detection path, tested without a GPU
+ * fault): the next kvx_translate on this translator bounds every on-chip wait by wait_us
+ * microseconds (1 .. 1e6) instead of about a second and, when that call runs the
+ * identity-alignment kernel, the kernel's first CTA issues no source copies from its unit-th
+ * work unit on, so the waits for them run out.  That call then records KVX_DEV_WAIT_TIMEOUT in
+ * the status word, drains the copies it started, frees its tensor memory and returns with its
+ * output incomplete; the context stays usable and later calls translate normally.  Applies to
+ * the next call only. */
+KVX_API kvx_status kvx_debug_stall_next_translate(kvx_translator* tr, int32_t unit, int32_t wait_us);
+
 /* Diagnostics of the token-span plan of the most recent kvx_translate on this translator, when
  * that call ran the span kernel (its last chunk of up to 65536 target tokens).  The span kernel
  * stages the source rows of each 32-token sub-tile as one window of consecutive rows (at most

@@ -93,7 +93,7 @@ EXPORTS = ["kvx_translator_create", "kvx_translator_create_low_rank", "kvx_trans
            "kvx_fit_accumulate", "kvx_fit_solve", "kvx_fit_reset", "kvx_fit_tokens", "kvx_fit_destroy", "kvx_build_alignment", "kvx_layer_map_nearest",
            "kvx_get_device_status", "kvx_get_info", "kvx_launches_per_translate", "kvx_last_error",
            "kvx_destroy", "kvx_translate_static", "kvx_static_last_error", "kvx_span_plan_stats",
-           "kvx_enable_peer", "kvx_translate_to_device"]
+           "kvx_enable_peer", "kvx_translate_to_device", "kvx_debug_stall_next_translate"]
 KVX_PEER_STORES, KVX_PEER_STAGED = 0, 1
 KVX_STATIC_SCRATCH_BYTES = 8 << 20
 
@@ -152,6 +152,7 @@ def lib():
         L.kvx_fit_destroy.argtypes = [VP]
         L.kvx_span_plan_stats.argtypes = [VP, VP, ctypes.POINTER(ctypes.c_int64)]
         L.kvx_enable_peer.argtypes = [ctypes.c_int32]
+        L.kvx_debug_stall_next_translate.argtypes = [VP, ctypes.c_int32, ctypes.c_int32]
         L.kvx_translate_to_device.argtypes = [VP, ctypes.POINTER(kvx_src_kv), ctypes.POINTER(kvx_tgt_tokens),
                                               ctypes.POINTER(kvx_dst_kv), ctypes.c_int32, ctypes.c_int32,
                                               ctypes.POINTER(kvx_dst_kv), VP]
@@ -409,6 +410,10 @@ class Translator:
                                       span_lo, span_hi, src_pos, tgt_pos, page_table, page_size, num_pages)
         self._keep = (dst, stg)
         kvx_translate_to_device(self.handle, src, tgt, dst, dst_device, mode, stg, _stream(stream))
+
+    def debug_stall_next_translate(self, unit: int, wait_us: int):
+        """Diagnostics: the next translate times out its on-chip waits (kvx_debug_stall_next_translate)."""
+        _check(lib().kvx_debug_stall_next_translate(VP(self.handle), unit, wait_us))
 
     def span_plan_stats(self, stream=None) -> dict:
         """Token-span plan of the last translate (span kernel only): sub-tiles, tokens staged in

@@ -110,6 +110,10 @@ struct TranslateParams {
     int max_position;
     int plain_stores;   // write target rows with 16-byte stores from the threads instead of the bulk-copy
                         // unit (destinations on another device, reached over the peer mapping)
+    // diagnostics of the bounded waits (kvx_debug_stall_next_translate): 0 = off
+    unsigned long long wait_ns;   // bound of each on-chip wait instead of ~1 s
+    int stall_unit1;              // identity kernel: CTA 0's producer issues no copies from its
+                                  // (stall_unit1 - 1)-th unit on, so the waits for them run out
     unsigned* status;
     // weights (layout depends on the kernel)
     const void* w;

@@ -431,6 +431,52 @@ __device__ __forceinline__ uint32_t gram_word(int r, int lw)
     return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((((lw >> 2) ^ (r & 7)) & 7) << 4) + (lw & 3) * 4);
 }
 
+// Bring the cache rows K-block w of unit `unit` reads into L2 ahead of its prologue: the
+// source rows of every head-block (one range from the first token's span start to the last
+// token's span end, within the first token's sequence) and the target rows (a range when the
+// target cache is contiguous).  Prefetches are hints: ranges are clipped to the caches.
+__device__ __forceinline__ void l2_prefetch(const void* p, uint32_t bytes)
+{
+    const char* c = (const char*)p;
+    for (uint32_t o = 0; o < bytes; o += 16384u) {   // pieces of at most 16 KB
+        const uint32_t n = bytes - o < 16384u ? bytes - o : 16384u;
+        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(c + o), "r"(n) : "memory");
+    }
+}
+__device__ void gram_prefetch(const TranslateParams& P, int unit, int kb, int mbs)
+{
+    const int g = unit / mbs, kv = g & 1, jh = g >> 1, h = jh % P.Ht, j = jh / P.Ht;
+    const int t0 = kb * kGramK, t1 = min(t0 + kGramK, P.T_total) - 1;
+    if (t1 < t0) return;
+    const int b = find_seq(P.seq_off, P.batch, t0);
+    const int off = __ldg(&P.seq_off[b]), end = __ldg(&P.seq_off[b + 1]);
+    int S = __ldg(&P.src_seq_len[b]);
+    S = S < 0 ? 0 : (S > P.src_max_seq ? P.src_max_seq : S);
+    const int tl = min(t1, end - 1);
+    int lo = t0 - off, hi = tl - off + 1;
+    if (P.span_lo) { lo = __ldg(&P.span_lo[t0]); hi = __ldg(&P.span_hi[tl]); }
+    lo = max(lo, 0);
+    hi = min(hi, S);
+    if (P.ss == P.ds && hi > lo) {
+        const int heads = P.in_dim / P.ds;
+        for (int q = 0; q < heads; ++q) {
+            int slot, gs;
+            head_block(P, j, h, q, slot, gs);
+            const __nv_bfloat16* base = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) +
+                                        (long long)b * P.sb + (long long)gs * P.sh + (long long)lo * P.ss;
+            l2_prefetch(base, (uint32_t)(hi - lo) * P.ds * 2);
+        }
+    }
+    if (!P.paged && P.dts == P.dt) {
+        const int ta = t0 - off, tb = min(tl - off + 1, P.dst_max_seq);
+        if (tb > ta) {
+            const __nv_bfloat16* rowp = (const __nv_bfloat16*)(kv ? P.dst_v[j] : P.dst_k[j]) + (long long)b * P.db +
+                                        (long long)h * P.dh + (long long)ta * P.dts;
+            l2_prefetch(rowp, (uint32_t)(tb - ta) * P.dt * 2);
+        }
+    }
+}
+
 template <int DS>
 __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __grid_constant__ TranslateParams P,
                                                                       const __grid_constant__ GramLaunch L)
@@ -547,9 +593,17 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
         const int nx = heads * CPH, items = nx + dt / 16;
         const int hs_t = dt >> 1;
         uint32_t it = 0;
+        if (xw == 0 && lane < 2 && w0 + lane < w1) {   // the first two K-blocks of the range
+            const int w = w0 + lane, unit = w / L.nkb;
+            gram_prefetch(P, unit, w - unit * L.nkb, L.mbs);
+        }
         for (int w = w0; w < w1; ++w, ++it) {
             const int unit = w / L.nkb, kb = w - unit * L.nkb;
             const int g = unit / L.mbs;
+            if (xw == 0 && lane == 0 && w + 2 < w1) {   // two K-blocks ahead
+                const int un = (w + 2) / L.nkb;
+                gram_prefetch(P, un, w + 2 - un * L.nkb, L.mbs);
+            }
             const int kv = g & 1, jh = g >> 1, h = jh % P.Ht, j = jh / P.Ht;
             const uint32_t s = it % (uint32_t)L.stages, ph = (it / (uint32_t)L.stages) & 1;
             if (!W.wait(bar(bEmpty + s), ph ^ 1)) break;

@@ -39,6 +39,8 @@ struct kvx_translator {
     void* plan = nullptr;
     int last_launches = 0;       // kernel launches of the most recent kvx_translate
     int last_span_tokens = 0;    // target tokens of the most recent call if it ran the span kernel, else 0
+    int dbg_stall_unit1 = 0;     // kvx_debug_stall_next_translate, for the next call only
+    unsigned long long dbg_wait_ns = 0;
     // encoded source tensor maps of the identity-alignment kernel, a few per (target layer, K|V)
     struct MapEntry {
         const void* ptr = nullptr;
@@ -455,6 +457,10 @@ static kvx_status translate_impl(kvx_translator* tr, const kvx_src_kv* src, cons
         g_last_error = err;
         return pst;
     }
+    P.wait_ns = tr->dbg_wait_ns;
+    P.stall_unit1 = tr->dbg_stall_unit1;
+    tr->dbg_wait_ns = 0;
+    tr->dbg_stall_unit1 = 0;
     if (tgt->total_tokens == 0) return KVX_OK;
     P.plain_stores = plain_stores;
     cudaError_t ce;
@@ -630,6 +636,15 @@ extern "C" KVX_API kvx_status kvx_get_info(const kvx_translator* tr, kvx_transla
 }
 
 extern "C" KVX_API int32_t kvx_launches_per_translate(const kvx_translator* tr) { return tr ? tr->last_launches : 0; }
+
+extern "C" KVX_API kvx_status kvx_debug_stall_next_translate(kvx_translator* tr, int32_t unit, int32_t wait_us)
+{
+    if (!tr || unit < 0 || wait_us < 1 || wait_us > 1000000)
+        return fail(KVX_ERR_INVALID_ARG, "debug_stall_next_translate: bad arguments");
+    tr->dbg_stall_unit1 = unit + 1;
+    tr->dbg_wait_ns = (unsigned long long)wait_us * 1000ull;
+    return KVX_OK;
+}
 
 extern "C" KVX_API kvx_status kvx_span_plan_stats(kvx_translator* tr, void* stream, int64_t* counts)
 {

@@ -68,7 +68,8 @@ constexpr int kBarDEmpty = kBarDFull + 2;       // +buf (2)
 constexpr int kBarSlotFull = kBarDEmpty + 2;    // +slot
 constexpr int kBarSlotEmpty = kBarSlotFull + kNumSlots;
 constexpr int kBarPair = kBarSlotEmpty + kNumSlots;   // +quad*2+{0,1}: the two epilogue warps of a quadrant meet
-constexpr int kNumBars = kBarPair + 8;
+constexpr int kBarMmaDone = kBarPair + 8;             // after an abort: the issued MMAs have completed
+constexpr int kNumBars = kBarMmaDone + 1;
 
 // Span plan of one 32-token sub-tile, written by span_plan_kernel once per
 // translation and read by every (layer, head, K|V) group of the tile:
@@ -295,6 +296,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             mbar_init(bar(kBarSlotEmpty + i), kNumXfWarps);
         }
         for (int i = 0; i < 8; ++i) mbar_init(bar(kBarPair + i), 2);
+        mbar_init(bar(kBarMmaDone), 1);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -320,7 +322,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
     tc_fence_after();
     const uint32_t tmem_base = *sTmemBase;
 
-    const Waiter W{sAbort, P.status};
+    const Waiter W{sAbort, P.status, P.wait_ns ? P.wait_ns : kWaitNs};
     const SeqView sv{L.seq_cached ? sSeqOff : P.seq_off, L.seq_cached ? sSrcLen : P.src_seq_len, P.batch};
 
     const int hw = L.n_tile >> 1;                 // pair half-width of an output split
@@ -472,6 +474,11 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 umma_commit(bar(kBarDFull + buf));
                 if (!b_stream && wk.last_of_group()) umma_commit(bar(kBarBEmpty));
                 ++tcount;
+            }
+            if (*sAbort) {   // MMAs whose results nobody waited for must finish before TMEM is freed
+                umma_commit(bar(kBarMmaDone));
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(bar(kBarMmaDone), 0) && globaltimer() - t0 < W.limit_ns) {}
             }
         }
         __syncwarp();

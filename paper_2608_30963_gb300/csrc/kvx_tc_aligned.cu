@@ -59,7 +59,9 @@ constexpr int kMaxKReady = kMaxSlots + 2;
 constexpr int kBarPair = kBarKReady + kMaxKReady;
 // +buf: the epilogue has read the (cos, sin) the prologue left in TMEM for a K tile
 constexpr int kBarCsFree = kBarPair + 8;
-constexpr int kNumBars = kBarCsFree + 2;
+// after an abort: every MMA the issuer started has completed (before TMEM is freed)
+constexpr int kBarMmaDone = kBarCsFree + 2;
+constexpr int kNumBars = kBarMmaDone + 1;
 
 struct AlignedParams {
     // geometry
@@ -80,6 +82,8 @@ struct AlignedParams {
     RopeTable rs, rt;
     int max_position;
     int plain_stores;   // target rows written with 16-byte thread stores (a peer device's cache)
+    unsigned long long wait_ns;   // bound of each wait (0: ~1 s)
+    int stall_unit1;              // diagnostics: CTA 0's producer stops before its (stall_unit1 - 1)-th unit with rows
     unsigned* status;
     const void* w;
     unsigned idesc, tmem_cols, b_bytes, stage_row_bytes;
@@ -232,6 +236,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         for (uint32_t i = 0; i < NKR; ++i) mbar_init(bar(kBarKReady + i), kNumXfWarps);
         for (int i = 0; i < 8; ++i) mbar_init(bar(kBarPair + i), 2);
         for (int i = 0; i < 2; ++i) mbar_init(bar(kBarCsFree + i), kNumEpiWarps);
+        mbar_init(bar(kBarMmaDone), 1);
         fence_mbar_init();
     }
     if (warp == kMmaWarp) {
@@ -259,7 +264,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     tc_fence_after();
     const uint32_t tmem_base = *sTmemBase;
 
-    const Waiter W{sAbort, P.status};
+    const Waiter W{sAbort, P.status, P.wait_ns ? P.wait_ns : kWaitNs};
     // Work split: each CTA takes an equal share of the K units and of the V units
     // (K units cost more: the source RoPE undo), K share first.  Within each share
     // units run group-major, so a group's weight tile stays resident.
@@ -283,10 +288,17 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             uint32_t b_loads = 0, slot_cnt = 0;
             SlotPos sp{0, 0};
             bool ok = true;
+            int nunit = 0;   // units with rows walked so far
             Walker wk;
             for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
                 const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
+                if (blockIdx.x == 0 && ++nunit == P.stall_unit1) {
+                    // diagnostics: a copy that never comes; the consumers' bounded waits run out
+                    const unsigned long long t0 = globaltimer();
+                    while (!*sAbort && globaltimer() - t0 < 4 * W.limit_ns) {}
+                    break;
+                }
                 // A K-blocks first: they do not depend on the weights, so at a group switch the
                 // ring refills while the previous group's last tiles drain
                 const CUtensorMap* map = &P.maps[x.j * 2 + x.kv];
@@ -319,9 +331,9 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 const unsigned long long t0 = globaltimer();
                 for (uint32_t c = slot_cnt > NS ? slot_cnt - NS : 0; c < slot_cnt; ++c)
                     while (!mbar_try_wait(bar(kBarFull + c % NS), (c / NS) & 1) &&
-                           globaltimer() - t0 < kWaitNs) {}
+                           globaltimer() - t0 < W.limit_ns) {}
                 if (b_loads)
-                    while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < kWaitNs) {}
+                    while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < W.limit_ns) {}
             }
         }
         __syncwarp();
@@ -372,6 +384,11 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                 const bool last = wk.last_of_group();
                 if (last) umma_commit(bar(kBarBEmpty));
                 ++tcount;
+            }
+            if (*sAbort) {   // MMAs whose results nobody waited for must finish before TMEM is freed
+                umma_commit(bar(kBarMmaDone));
+                const unsigned long long t0 = globaltimer();
+                while (!mbar_try_wait(bar(kBarMmaDone), 0) && globaltimer() - t0 < W.limit_ns) {}
             }
         }
         __syncwarp();
@@ -687,6 +704,8 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     P.page_table = T.page_table; P.max_pages = T.max_pages; P.page_size = T.page_size; P.num_pages = T.num_pages;
     P.rs = T.rs; P.rt = T.rt; P.max_position = T.max_position; P.status = T.status; P.w = T.w;
     P.plain_stores = T.plain_stores;
+    P.wait_ns = T.wait_ns;
+    P.stall_unit1 = T.stall_unit1;
     P.idesc = (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(P.n_tile >> 3) << 17) | ((uint32_t)(kTileM >> 4) << 24);
     P.share_cs = T.rs.enabled && T.rt.enabled && T.ds == T.dt && !T.src_pos && !T.tgt_pos &&
                  T.rope_same && 2 * P.n_tile + 2 * T.dt <= 512;

@@ -251,6 +251,7 @@ __device__ __forceinline__ uint32_t sw128_off(int row, int k, int rows)
 struct Waiter {
     volatile int* abort;
     unsigned* status;
+    unsigned long long limit_ns = kWaitNs;   // bound of each wait
     __device__ __forceinline__ bool wait(uint32_t bar, uint32_t parity) const
     {
         if (mbar_try_wait(bar, parity)) return true;
@@ -258,7 +259,7 @@ struct Waiter {
         while (true) {
             if (mbar_try_wait_sleep(bar, parity, 100000u)) return true;
             if (*abort) return false;
-            if (globaltimer() - t0 > kWaitNs) {
+            if (globaltimer() - t0 > limit_ns) {
                 *abort = 1;
                 set_status(status, KVX_DEV_WAIT_TIMEOUT);
                 return false;
