@@ -143,6 +143,11 @@ kvx_status make_params(const Geometry& g, const unsigned long long* dev_turns, u
 // Thread-local message returned by kvx_last_error().
 void set_last_error(const char* msg);
 
+// Target heads that read the same input rows: the e heads of a GQA expansion group, every head
+// in the dense per-layer form, else 1.
+__host__ __device__ inline int share_heads(int dense, int r, int e, int Ht) { return dense ? Ht : (r == 1 ? e : 1); }
+__host__ __device__ inline int share_heads(const TranslateParams& P) { return share_heads(P.dense, P.r, P.e, P.Ht); }
+
 // First source head feeding target head h: its GQA group (h*r), the source head it
 // repeats (h/e), or head 0 in the dense per-layer form.
 __device__ __forceinline__ int src_head0(const TranslateParams& P, int h)

@@ -312,7 +312,7 @@ extern "C" KVX_API kvx_status kvx_translator_create(const kvx_translator_desc* d
     }
 
     // kernel choice
-    t->tc = tc_config(t->in_dim, d.head_dim, s.head_dim);
+    t->tc = tc_config(t->in_dim, d.head_dim, s.head_dim, share_heads(t->dense, t->r, t->e, d.num_kv_heads));
     const bool tc_ok = desc->dtype == KVX_BF16 && t->tc.ok;
     if (desc->path == KVX_PATH_TCGEN05 && !tc_ok) {
         const int in_dim = t->in_dim;
@@ -468,7 +468,8 @@ static kvx_status translate_impl(kvx_translator* tr, const kvx_src_kv* src, cons
     // pairs channels at rotary_dim/2; the identity kernel pairs whole heads
     const bool whole_head_rope = rope_rot_dim(D.src) == D.src.head_dim && rope_rot_dim(D.dst) == D.dst.head_dim;
     if (tr->path == KVX_PATH_TCGEN05 && !tgt->span_lo && whole_head_rope &&
-        aligned_supported(tr->in_dim, D.dst.head_dim, D.src.head_dim, Lt, src->batch, tr->kl)) {
+        aligned_supported(tr->in_dim, D.dst.head_dim, D.src.head_dim, share_heads(tr->dense, tr->r, tr->e, D.dst.num_kv_heads),
+                          Lt, src->batch, tr->kl)) {
         // identity alignment: tensor-TMA fed kernel
         if (tr->maps.empty()) tr->maps.resize((size_t)2 * KVX_MAX_ALIGNED_LAYERS * kvx_translator::kMapWays);
         const void* maps[2 * KVX_MAX_ALIGNED_LAYERS];

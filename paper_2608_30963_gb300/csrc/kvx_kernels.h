@@ -25,7 +25,9 @@ struct TcConfig {
     int threads;
     int ok;            // geometry supported
 };
-TcConfig tc_config(int in_dim, int dt, int ds);
+// share: target heads that read the same input rows (share_heads); it decides how many heads
+// one unit of the span kernel covers and so the weight images' output split n_tile.
+TcConfig tc_config(int in_dim, int dt, int ds, int share);
 size_t tc_weight_image_bytes(int in_dim, int dt, int Lt, int Ht);
 // rhalf_t: rotating pairs of the target head (rotary_dim/2; d_t/2 unless partial rotary)
 cudaError_t launch_tc_weight_relayout(const void* w_k, const void* w_v, void* image, int Lt, int Ht, int in_dim,
@@ -41,7 +43,7 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
                                 int plan_tokens, cudaStream_t stream, int* launches);
 
 // identity-alignment tensor-core path (tensor-TMA fed)
-bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch, int kl);
+bool aligned_supported(int in_dim, int dt, int ds, int share, int Lt, int batch, int kl);
 size_t aligned_map_bytes();
 bool encode_source_map(void* map_out, const void* base, int ds, int S_max, int Hs, int batch, long long ss,
                        long long sh, long long sb);

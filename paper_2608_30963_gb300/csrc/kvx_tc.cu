@@ -5,25 +5,29 @@
 // (span gather, RoPE undo, span mean, RoPE apply, cache write) is streaming work
 // fused into the GEMM's prologue and epilogue.
 //
-// Persistent kernel, one CTA per SM, work unit = (group, 128-token tile) with
-// group = (target layer j, target head h, K|V, output split nt).  A CTA walks an
-// equal share of the K units and of the V units, group-major, so the group's
-// weight tile (B operand) stays in shared memory across its token tiles.  Warp
-// roles:
+// Persistent kernel, one CTA per SM.  Work unit = (target layer j, head set, K|V, output
+// split(s), 128-token tile), where the head set holds the target heads that read the same
+// input rows and fit one 512-column accumulator (the heads of a GQA expansion group, or every
+// head in the dense per-layer form; one head otherwise): the unit's A (span means of the
+// un-rotated source rows) is built once and multiplied by each (head, output split) "piece"
+// of W into the piece's own accumulator slot.  A CTA walks an equal share of the K units and
+// of the V units, group-major, so a one-piece unit's weight tile (B operand) stays in shared
+// memory across its token tiles.  Warp roles:
 //   warp 0      producer: resolves the spans of each 32-token sub-tile and, per
 //               source head, copies the sub-tile's window of consecutive source
-//               rows into a byte ring in shared memory with one cp.async.bulk
-//               (mbarrier transaction counts); loads B: a group's whole image,
-//               kept across its token tiles, when it fits 64 KB, else (wide
-//               inputs: the dense per-layer form, groups of source layers) one
-//               source head's piece of it per head-block through two slots.
-//   warp 1      MMA: allocates TMEM, issues tcgen05.mma (M=128, N=n_tile, K=16
-//               steps over in, one source head's block of A at a time) into a
-//               double-buffered fp32 accumulator.
+//               rows into a byte ring in shared memory with cp.async.bulk
+//               (mbarrier transaction counts); loads a one-piece unit's whole B
+//               image when it fits 64 KB, kept across the group's token tiles.
+//   warp 1      lane 0, MMA: allocates TMEM, issues tcgen05.mma (M=128, N=n_tile,
+//               K=16 steps over in, one source head's block of A at a time, one MMA
+//               per piece) into a ring of fp32 accumulator slots.
+//               lane 1, B-loader (streamed weights: several pieces per unit, or
+//               inputs too wide to keep resident): one source head's rows of one
+//               piece's W per (head-block, piece), through two slots.
 //   warps 2-9   epilogue: tcgen05.ld the accumulator (one thread per token row,
 //               two warps per TMEM lane quadrant), apply the target RoPE, round to
 //               bf16, stage the row and write it to the target cache (contiguous
-//               or paged) with cp.async.bulk.
+//               or paged) with cp.async.bulk, piece by piece.
 //   warps 10-17 prologue: groups of d_s/16 lanes per target token, 16-byte
 //               chunks per lane: undo the source RoPE of each span row, take the
 //               span mean, round to bf16 and store A, one source head's block at
@@ -55,6 +59,8 @@ constexpr int kMaxSeqCache = 512;         // sequences whose metadata is kept in
 constexpr int kMaxTcIn = 1024;            // widest translator input row (in) this kernel takes
 constexpr int kMaxA = 2;                  // A head-block slots
 constexpr int kMaxB = 2;                  // B slots (1: the group's whole image; 2: head-block pieces)
+constexpr int kMaxD = 8;                  // accumulator slots in TMEM (512 columns / n_tile)
+constexpr int kBLoaderLane = 1;           // lane of the MMA warp that streams B pieces
 constexpr unsigned kBResidentMax = 65536; // largest B image kept resident per group
 constexpr unsigned kBPieceMax = 32768;    // largest streamed B piece (one source head's rows)
 
@@ -63,9 +69,9 @@ constexpr int kBarBFull = 0;               // +B slot
 constexpr int kBarBEmpty = kBarBFull + kMaxB;
 constexpr int kBarAFull = kBarBEmpty + kMaxB;   // +A slot
 constexpr int kBarAEmpty = kBarAFull + kMaxA;
-constexpr int kBarDFull = kBarAEmpty + kMaxA;   // +buf (2)
-constexpr int kBarDEmpty = kBarDFull + 2;       // +buf (2)
-constexpr int kBarSlotFull = kBarDEmpty + 2;    // +slot
+constexpr int kBarDFull = kBarAEmpty + kMaxA;   // +accumulator slot
+constexpr int kBarDEmpty = kBarDFull + kMaxD;   // +accumulator slot
+constexpr int kBarSlotFull = kBarDEmpty + kMaxD;    // +slot
 constexpr int kBarSlotEmpty = kBarSlotFull + kNumSlots;
 constexpr int kBarPair = kBarSlotEmpty + kNumSlots;   // +quad*2+{0,1}: the two epilogue warps of a quadrant meet
 constexpr int kBarMmaDone = kBarPair + 8;             // after an abort: the issued MMAs have completed
@@ -95,9 +101,15 @@ struct TcLaunch {
     unsigned hb_bytes; // one A head-block: 128 rows x d_s bf16
     unsigned cap_rows; // most source rows one window may stage
     int n_slots;       // window slots of slot_bytes each
-    int share;         // target heads that read the same source rows, walked by interleaved CTA sets (1 = off)
+    int share;         // head units that read the same source rows, walked by interleaved CTA sets (1 = off)
+    int hpu, spu;      // target heads and output splits of one work unit: all of them share the unit's
+                       // A (its span-averaged input rows), each (head, split) is one piece with its own
+                       // accumulator slot
+    int np;            // pieces per unit: hpu * spu
+    int nd;            // accumulator slots (ring over the pieces, in order)
     int n_b;           // B slots: 1 = the group's image stays resident across its tiles;
-                       // 2 = streamed, one piece (one source head's rows of W) per head-block
+                       // 2 = streamed, one piece (one source head's rows of one piece's W) per
+                       // (head-block, piece), by the B-loader lane
     unsigned b_bytes;  // one group's whole B image (in x n_tile bf16)
     unsigned b_slot_bytes;   // one B slot: b_bytes (resident) or ds x n_tile bf16 (streamed)
     unsigned row_bytes, stage_row_bytes, slot_bytes;
@@ -108,41 +120,43 @@ struct TcLaunch {
 };
 
 struct Unit {
-    int j, h, kv, nt, tile, g;
+    int j, h, kv, nt, tile, g;   // first head and first split of the unit; g: B image of its first piece
 };
 // The CTA's units: an equal share of the K units, then of the V units (each share
-// group-major, so a group's weights stay resident), walked with counters only.
-// When `share` > 1 target heads read the same source rows (the `share` heads of a GQA
-// expansion group, or every head in the dense form), the CTAs form `share` interleaved
-// sets: set i walks head i of every group, and CTA k of each set takes the k-th share of
-// the same (layer, head group, tile) sequence.  The partners' reads of a window then come
-// at about the same time, so the second one hits L2 instead of going back to DRAM.
+// group-major, so a group's weights stay resident), walked with counters only.  A unit
+// covers hpu consecutive target heads and spu consecutive output splits.
+// When `share` > 1 head units read the same source rows (the heads of a GQA expansion group,
+// or every head in the dense form, beyond those a unit covers), the CTAs form `share`
+// interleaved sets: set i walks head unit i of every group, and CTA k of each set takes the
+// k-th share of the same (layer, head group, tile) sequence.  The partners' reads of a window
+// then come at about the same time, so the second one hits L2 instead of going back to DRAM.
 struct Walker {
     int count, nK, it;
     int kv, j, h, nt, tile;
-    int u0, v0, m_tiles, n_split, Ht, E, hk, hv;
+    int u0, v0, m_tiles, n_split, nsu, hpu, spu, Ht, E, hk, hv;
     Unit x;
     __device__ __forceinline__ void fill()
     {
-        x.j = j; x.h = h; x.kv = kv; x.nt = nt; x.tile = tile;
-        x.g = ((j * Ht + h) * 2 + kv) * n_split + nt;
+        x.j = j; x.h = h; x.kv = kv; x.nt = nt * spu; x.tile = tile;
+        x.g = ((j * Ht + h) * 2 + kv) * n_split + nt * spu;
     }
     __device__ __forceinline__ void seek(int idx, int kv_)
     {
         kv = kv_;
         const int hg = idx / m_tiles;
         tile = idx - hg * m_tiles;
-        nt = hg % n_split;
-        const int jq = hg / n_split;
-        const int HtE = Ht / E;
-        h = (jq % HtE) * E + (kv ? hv : hk);
+        nt = hg % nsu;
+        const int jq = hg / nsu;
+        const int HtE = Ht / (hpu * E);
+        h = (jq % HtE) * hpu * E + (kv ? hv : hk) * hpu;
         j = jq / HtE;
         fill();
     }
     __device__ __forceinline__ void start(const TcLaunch& L, int Ht_)
     {
-        m_tiles = L.m_tiles; n_split = L.n_split; Ht = Ht_; E = L.share;
-        const long long UH = (long long)(L.groups / 2) * L.m_tiles / E;   // units of one head set
+        m_tiles = L.m_tiles; n_split = L.n_split; Ht = Ht_; E = L.share; hpu = L.hpu; spu = L.spu;
+        nsu = n_split / spu;
+        const long long UH = (long long)(L.groups / 2) * L.m_tiles / ((long long)E * hpu * spu);   // units of one set
         const int G = gridDim.x / E, c = blockIdx.x / E, vr = gridDim.x - 1 - (int)blockIdx.x;
         hk = (int)blockIdx.x % E;
         hv = vr % E;
@@ -164,9 +178,9 @@ struct Walker {
         if (it == nK) { seek(v0, 1); return; }
         if (++tile == m_tiles) {
             tile = 0;
-            if (++nt == n_split) {
+            if (++nt == nsu) {
                 nt = 0;
-                if ((h += E) >= Ht) { h = kv ? hv : hk; ++j; }
+                if ((h += hpu * E) >= Ht) { h = (kv ? hv : hk) * hpu; ++j; }
             }
         }
         fill();
@@ -176,6 +190,13 @@ struct Walker {
         return it + 1 == count || it + 1 == nK || tile + 1 == m_tiles;
     }
 };
+
+// B image of piece p of unit x: head x.h + p / spu, split x.nt + p % spu.
+__device__ __forceinline__ int piece_group(const Unit& x, int p, int spu, int Ht, int n_split)
+{
+    const int hh = p / spu, s = p - hh * spu;
+    return ((x.j * Ht + x.h + hh) * 2 + x.kv) * n_split + x.nt + s;
+}
 
 // Sequence metadata view: shared-memory copies of seq_off / src_seq_len when the
 // batch is small enough, else the global arrays.
@@ -287,7 +308,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             mbar_init(bar(kBarAFull + i), kNumXfWarps);
             mbar_init(bar(kBarAEmpty + i), 1);
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < L.nd; ++i) {
             mbar_init(bar(kBarDFull + i), 1);
             mbar_init(bar(kBarDEmpty + i), kNumEpiWarps);
         }
@@ -341,17 +362,16 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         const bool rows_contig = P.ss == P.ds;
         const bool b_stream = L.n_b > 1;
         int cur_g = -1;
-        uint32_t b_loads = 0, issued = 0;   // B loads: slot b_loads % n_b, phase (b_loads / n_b) & 1
-        // one B load (the group's image or one head-block piece of it) into the next B slot
+        uint32_t b_loads = 0, issued = 0;   // resident B images loaded (one slot); window copies issued
+        // the group's whole B image into its slot (resident mode; streamed pieces come from the
+        // B-loader lane)
         auto load_b = [&](const uint8_t* from, uint32_t bytes) -> bool {
-            const uint32_t bs = b_loads % (uint32_t)L.n_b;
-            if (!W.wait(bar(kBarBEmpty + bs), ((b_loads / (uint32_t)L.n_b) & 1) ^ 1)) return false;
-            if (lane == 0) mbar_arrive_expect_tx(bar(kBarBFull + bs), bytes);
+            if (!W.wait(bar(kBarBEmpty), (b_loads & 1) ^ 1)) return false;
+            if (lane == 0) mbar_arrive_expect_tx(bar(kBarBFull), bytes);
             __syncwarp();
             const uint32_t piece = bytes / 4;
             if (lane < 4)
-                bulk_g2s(smem_u32(sB) + bs * L.b_slot_bytes + lane * piece, from + (size_t)lane * piece, piece,
-                         bar(kBarBFull + bs), pol_keep);
+                bulk_g2s(smem_u32(sB) + lane * piece, from + (size_t)lane * piece, piece, bar(kBarBFull), pol_keep);
             ++b_loads;
             return true;
         };
@@ -380,7 +400,6 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 int src_slot, gq;
                 head_block(P, x.j, x.h, q, src_slot, gq);
                 const __nv_bfloat16* src = (const __nv_bfloat16*)(x.kv ? P.src_v[src_slot] : P.src_k[src_slot]);
-                if (b_stream && !load_b(img + (size_t)q * L.b_slot_bytes, L.b_slot_bytes)) { ok = false; break; }
 #pragma unroll
                 for (int sq = 0; sq < kSubPerTile; ++sq) {
                     if (!ok) break;
@@ -419,18 +438,20 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             const unsigned long long t0 = globaltimer();
             const uint32_t ns = (uint32_t)L.n_slots;
             for (uint32_t c = issued > ns ? issued - ns : 0; c < issued; ++c)
-                while (!mbar_try_wait(bar(kBarSlotFull + c % ns), (c / ns) & 1) && globaltimer() - t0 < kWaitNs) {}
-            const uint32_t nb = (uint32_t)L.n_b;
-            for (uint32_t c = b_loads > nb ? b_loads - nb : 0; c < b_loads; ++c)
-                while (!mbar_try_wait(bar(kBarBFull + c % nb), (c / nb) & 1) && globaltimer() - t0 < kWaitNs) {}
+                while (!mbar_try_wait(bar(kBarSlotFull + c % ns), (c / ns) & 1) && globaltimer() - t0 < W.limit_ns) {}
+            if (b_loads)
+                while (!mbar_try_wait(bar(kBarBFull), (b_loads - 1) & 1) && globaltimer() - t0 < W.limit_ns) {}
         }
     } else if (warp == kMmaWarp) {
-        // ------------------------------------------------------------ MMA issuer
+        const bool b_stream = L.n_b > 1;
+        const uint32_t nb = (uint32_t)L.n_b, nd = (uint32_t)L.nd;
         if (lane == 0) {
+            // ------------------------------------------------------------ MMA issuer
+            // Per unit and head-block q: one MMA per piece (head, output split) into the piece's
+            // accumulator slot; the pieces' slots run as a ring of nd, in the order the epilogue
+            // drains them.
             int cur_g = -1;
-            uint32_t b_cnt = 0, tcount = 0, a_cnt = 0;   // B slot b_cnt % n_b, phase (b_cnt / n_b) & 1
-            const bool b_stream = L.n_b > 1;
-            const uint32_t nb = (uint32_t)L.n_b;
+            uint32_t b_cnt = 0, pcount = 0, a_cnt = 0;   // B slot b_cnt % n_b, phase (b_cnt / n_b) & 1
             bool ok = true;
             Walker wk;
             for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
@@ -440,61 +461,98 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     ++b_cnt;
                     cur_g = x.g;
                 }
-                const uint32_t buf = tcount & 1;
-                if (!W.wait(bar(kBarDEmpty + buf), ((tcount >> 1) & 1) ^ 1)) break;
-                const uint32_t d = tmem_base + buf * (uint32_t)L.n_tile;
+                for (int p = 0; p < L.np && ok; ++p) {
+                    const uint32_t c = pcount + (uint32_t)p;
+                    if (!W.wait(bar(kBarDEmpty + c % nd), ((c / nd) & 1) ^ 1)) ok = false;
+                }
+                if (!ok) break;
                 for (int q = 0; q < L.r_heads; ++q) {
                     const uint32_t sa = a_cnt % (uint32_t)L.n_a;
                     if (!W.wait(bar(kBarAFull + sa), (a_cnt / (uint32_t)L.n_a) & 1)) { ok = false; break; }
-                    // resident: the image's K-blocks of head-block q; streamed: the piece in its slot
-                    uint32_t b0 = smem_u32(sB), kb0 = (uint32_t)q * (DS / 64);
-                    const uint32_t bs = b_cnt % nb;
-                    if (b_stream) {
-                        if (!W.wait(bar(kBarBFull + bs), (b_cnt / nb) & 1)) { ok = false; break; }
-                        b0 += bs * L.b_slot_bytes;
-                        kb0 = 0;
-                    }
                     tc_fence_after();
                     const uint32_t a0 = smem_u32(sA) + sa * L.hb_bytes;
+                    for (int p = 0; p < L.np; ++p) {
+                        // resident: the image's K-blocks of head-block q; streamed: the piece in its slot
+                        uint32_t b0 = smem_u32(sB), kb0 = (uint32_t)q * (DS / 64);
+                        const uint32_t bs = b_cnt % nb;
+                        if (b_stream) {
+                            if (!W.wait(bar(kBarBFull + bs), (b_cnt / nb) & 1)) { ok = false; break; }
+                            tc_fence_after();
+                            b0 += bs * L.b_slot_bytes;
+                            kb0 = 0;
+                        }
+                        const uint32_t d = tmem_base + ((pcount + (uint32_t)p) % nd) * (uint32_t)L.n_tile;
 #pragma unroll
-                    for (int kk = 0; kk < DS / 16; ++kk) {
-                        const uint32_t kb = kk >> 2, ko = (kk & 3) * 32;
-                        const uint64_t ad = sw128_desc(a0 + kb * (kTileM * 128) + ko);
-                        const uint64_t bd = sw128_desc(b0 + (kb0 + kb) * (L.n_tile * 128) + ko);
-                        umma_bf16(d, ad, bd, L.idesc, (q > 0 || kk > 0) ? 1u : 0u);
+                        for (int kk = 0; kk < DS / 16; ++kk) {
+                            const uint32_t kb = kk >> 2, ko = (kk & 3) * 32;
+                            const uint64_t ad = sw128_desc(a0 + kb * (kTileM * 128) + ko);
+                            const uint64_t bd = sw128_desc(b0 + (kb0 + kb) * (L.n_tile * 128) + ko);
+                            umma_bf16(d, ad, bd, L.idesc, (q > 0 || kk > 0) ? 1u : 0u);
+                        }
+                        if (b_stream) {
+                            umma_commit(bar(kBarBEmpty + bs));
+                            ++b_cnt;
+                        }
                     }
+                    if (!ok) break;
                     umma_commit(bar(kBarAEmpty + sa));
                     ++a_cnt;
-                    if (b_stream) {
-                        umma_commit(bar(kBarBEmpty + bs));
-                        ++b_cnt;
-                    }
                 }
                 if (!ok) break;
-                umma_commit(bar(kBarDFull + buf));
+                for (int p = 0; p < L.np; ++p) umma_commit(bar(kBarDFull + (pcount + (uint32_t)p) % nd));
+                pcount += (uint32_t)L.np;
                 if (!b_stream && wk.last_of_group()) umma_commit(bar(kBarBEmpty));
-                ++tcount;
             }
             if (*sAbort) {   // MMAs whose results nobody waited for must finish before TMEM is freed
                 umma_commit(bar(kBarMmaDone));
                 const unsigned long long t0 = globaltimer();
                 while (!mbar_try_wait(bar(kBarMmaDone), 0) && globaltimer() - t0 < W.limit_ns) {}
             }
+        } else if (lane == kBLoaderLane && b_stream) {
+            // ------------------------------------------------------------ B-loader (streamed weights)
+            // Per unit, head-block q and piece p, in the MMA's order: the d_s rows of head-block q of
+            // the piece's B image (one source head's rows of W, n_tile output columns).
+            const uint64_t pol_keep = policy_evict_last();
+            uint32_t b_loads = 0;
+            bool ok = true;
+            Walker wk;
+            for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
+                const Unit& x = wk.x;
+                for (int q = 0; q < L.r_heads && ok; ++q)
+                    for (int p = 0; p < L.np; ++p) {
+                        const uint32_t bs = b_loads % nb;
+                        if (!W.wait(bar(kBarBEmpty + bs), ((b_loads / nb) & 1) ^ 1)) { ok = false; break; }
+                        const uint8_t* img = (const uint8_t*)P.w +
+                                             (size_t)piece_group(x, p, L.spu, P.Ht, L.n_split) * L.b_bytes +
+                                             (size_t)q * L.b_slot_bytes;
+                        mbar_arrive_expect_tx(bar(kBarBFull + bs), L.b_slot_bytes);
+                        bulk_g2s(smem_u32(sB) + bs * L.b_slot_bytes, img, L.b_slot_bytes, bar(kBarBFull + bs), pol_keep);
+                        ++b_loads;
+                    }
+            }
+            if (*sAbort) {   // let the copies in flight land before the CTA leaves
+                const unsigned long long t0 = globaltimer();
+                for (uint32_t c = b_loads > nb ? b_loads - nb : 0; c < b_loads; ++c)
+                    while (!mbar_try_wait(bar(kBarBFull + c % nb), (c / nb) & 1) && globaltimer() - t0 < W.limit_ns) {}
+            }
         }
         __syncwarp();
     } else if (warp < kEpiWarp0 + kNumEpiWarps) {
         // ------------------------------------------------------------ epilogue
+        // Per unit: the output rows are resolved once; then per piece (head, output split), in
+        // the MMA's order, the piece's accumulator slot is rotated, rounded, staged and stored.
         const int quad = warp & 3;
         const int half = (warp - kEpiWarp0) >> 2;          // which half of the rotary pairs
         const int m = quad * 32 + lane;
         const int pc_begin = half * (hw >> 1), pc_end = pc_begin + (hw >> 1);
         uint8_t* srow = sStage + (size_t)m * L.stage_row_bytes;
         const uint32_t srow_u32 = smem_u32(srow);
-        uint32_t tcount = 0;
+        const uint32_t nd = (uint32_t)L.nd;
+        uint32_t pcount = 0;
+        bool ok = true;
         Walker wk;
-        for (wk.start(L, P.Ht); wk.more(); wk.next()) {
+        for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
             const Unit& x = wk.x;
-            const uint32_t buf = tcount & 1;
             // resolve the output row while the tile is still being computed
             const int tp = L.t_begin + x.tile * kTileM + m;
             const bool valid = tp < L.t_end;
@@ -502,52 +560,56 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             int pt = 0;
             if (valid) resolve_dst(P, sv, tp, dst_off, pt);
             const bool rot = x.kv == 0 && P.rt.enabled;
-            float2 cs[8];
-            if (rot) rope_cs_vec<8>(sTurnT, pt, x.nt * hw + pc_begin, cs);
-            if (!W.wait(bar(kBarDFull + buf), (tcount >> 1) & 1)) break;
-            tc_fence_after();
-            // the staging row is shared by the two warps of this quadrant; the row's
-            // previous store (issued by the half-0 thread) must have read it
-            if (half == 0) bulk_wait_read0();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2));
-            if (!W.wait(bar(kBarPair + quad * 2), tcount & 1)) break;
-            const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)L.n_tile;
-            for (int pc = pc_begin; pc < pc_end; pc += 8) {
-                float2 csn[8];
-                if (rot && pc + 8 < pc_end) rope_cs_vec<8>(sTurnT, pt, x.nt * hw + pc + 8, csn);
-                uint32_t r0[8], r1[8];
-                tmem_ld8(taddr + pc, r0);
-                tmem_ld8(taddr + hw + pc, r1);
-                tmem_ld_wait();
-                uint4 out0, out1;
-                // pair slots from rhalf on (partial rotary heads) do not rotate
-                rotate8_to_bf16(r0, r1, cs, rot && x.nt * hw + pc < P.rhalf_t, out0, out1);
-                if (rot) {
+            for (int p = 0; p < L.np; ++p, ++pcount) {
+                const int hh = p / L.spu, nt = x.nt + (p - hh * L.spu);
+                const uint32_t buf = pcount % nd;
+                float2 cs[8];
+                if (rot) rope_cs_vec<8>(sTurnT, pt, nt * hw + pc_begin, cs);
+                if (!W.wait(bar(kBarDFull + buf), (pcount / nd) & 1)) { ok = false; break; }
+                tc_fence_after();
+                // the staging row is shared by the two warps of this quadrant; the row's
+                // previous store (issued by the thread of lane parity = half) must have read it
+                bulk_wait_read0();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2));
+                if (!W.wait(bar(kBarPair + quad * 2), pcount & 1)) { ok = false; break; }
+                const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16) + buf * (uint32_t)L.n_tile;
+                for (int pc = pc_begin; pc < pc_end; pc += 8) {
+                    float2 csn[8];
+                    if (rot && pc + 8 < pc_end) rope_cs_vec<8>(sTurnT, pt, nt * hw + pc + 8, csn);
+                    uint32_t r0[8], r1[8];
+                    tmem_ld8(taddr + pc, r0);
+                    tmem_ld8(taddr + hw + pc, r1);
+                    tmem_ld_wait();
+                    uint4 out0, out1;
+                    // pair slots from rhalf on (partial rotary heads) do not rotate
+                    rotate8_to_bf16(r0, r1, cs, rot && nt * hw + pc < P.rhalf_t, out0, out1);
+                    if (rot) {
 #pragma unroll
-                    for (int e = 0; e < 8; ++e) cs[e] = csn[e];
+                        for (int e = 0; e < 8; ++e) cs[e] = csn[e];
+                    }
+                    *reinterpret_cast<uint4*>(srow + pc * 2) = out0;
+                    *reinterpret_cast<uint4*>(srow + (hw + pc) * 2) = out1;
                 }
-                *reinterpret_cast<uint4*>(srow + pc * 2) = out0;
-                *reinterpret_cast<uint4*>(srow + (hw + pc) * 2) = out1;
-            }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kBarDEmpty + buf));
-            fence_proxy_async();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2 + 1));
-            if (!W.wait(bar(kBarPair + quad * 2 + 1), tcount & 1)) break;
-            if (half == 0 && valid && dst_off >= 0) {
-                __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
-                                     dst_head_off(P, x.h);
-                if (P.plain_stores) {
-                    store_row_slots_plain(dst, srow, x.nt * hw, hw, half_t, P.rhalf_t);
-                } else {
-                    store_row_slots(dst, srow_u32, x.nt * hw, hw, half_t, P.rhalf_t);
-                    bulk_commit();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(kBarDEmpty + buf));
+                fence_proxy_async();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2 + 1));
+                if (!W.wait(bar(kBarPair + quad * 2 + 1), pcount & 1)) { ok = false; break; }
+                // the quadrant's rows, split between its two warps by lane parity
+                if ((lane & 1) == half && valid && dst_off >= 0) {
+                    __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
+                                         dst_head_off(P, x.h + hh);
+                    if (P.plain_stores) {
+                        store_row_slots_plain(dst, srow, nt * hw, hw, half_t, P.rhalf_t);
+                    } else {
+                        store_row_slots(dst, srow_u32, nt * hw, hw, half_t, P.rhalf_t);
+                        bulk_commit();
+                    }
                 }
             }
-            ++tcount;
         }
         bulk_wait0();
     } else {
@@ -770,7 +832,9 @@ uint32_t make_idesc(int M, int N)
            | ((uint32_t)(M >> 4) << 24);   // A and B K-major, no negate, dense
 }
 
-bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
+// share: target heads that read the same input rows (the heads of a GQA expansion group, or
+// every head in the dense form; 1 otherwise).
+bool tc_layout(int in_dim, int dt, int ds, int share, TcLaunch& L)
 {
     if (in_dim % 64 || in_dim > kMaxTcIn || in_dim < 64) return false;
     if (dt != 64 && dt != 128 && dt != 256) return false;
@@ -778,16 +842,37 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
     if (in_dim % ds) return false;
     L.in_dim = in_dim;
     L.r_heads = in_dim / ds;
-    // B resident per group while one output split's image fits kBResidentMax; beyond that,
-    // streamed one head-block piece (ds x n_tile) at a time through two slots
-    L.n_tile = dt;
-    while ((unsigned)(in_dim * L.n_tile * 2) > kBResidentMax && L.n_tile > 64 && in_dim <= 256) L.n_tile >>= 1;
-    L.n_b = (unsigned)(in_dim * L.n_tile * 2) <= kBResidentMax ? 1 : kMaxB;
-    if (L.n_b > 1) {
+    // Heads per unit: as many of the heads sharing the input rows as the 512 accumulator columns
+    // hold (d_t each), so their A is built once; each (head, output split) is a piece, and the
+    // pieces' weights stream through two slots, one head-block (ds x n_tile) at a time.
+    int hpu = 1;
+    for (int c = share; c > 1; --c)
+        if (share % c == 0 && c * dt <= 512) { hpu = c; break; }
+    if (hpu > 1) {
+        L.n_b = kMaxB;
         L.n_tile = dt;
         while ((unsigned)(ds * L.n_tile * 2) > kBPieceMax && L.n_tile > 64) L.n_tile >>= 1;
+        L.n_split = dt / L.n_tile;
+        L.hpu = hpu;
+        L.spu = L.n_split;
+        L.nd = 512 / L.n_tile;
+    } else {
+        // one head per unit: B resident per group while one output split's image fits
+        // kBResidentMax; beyond that, streamed one head-block piece (ds x n_tile) at a time
+        L.n_tile = dt;
+        while ((unsigned)(in_dim * L.n_tile * 2) > kBResidentMax && L.n_tile > 64 && in_dim <= 256) L.n_tile >>= 1;
+        L.n_b = (unsigned)(in_dim * L.n_tile * 2) <= kBResidentMax ? 1 : kMaxB;
+        if (L.n_b > 1) {
+            L.n_tile = dt;
+            while ((unsigned)(ds * L.n_tile * 2) > kBPieceMax && L.n_tile > 64) L.n_tile >>= 1;
+        }
+        L.n_split = dt / L.n_tile;
+        L.hpu = 1;
+        L.spu = 1;
+        L.nd = 2;
     }
-    L.n_split = dt / L.n_tile;
+    L.np = L.hpu * L.spu;
+    if (L.nd > kMaxD || L.np > L.nd) return false;
     L.b_bytes = (unsigned)(in_dim * L.n_tile * 2);
     L.b_slot_bytes = L.n_b > 1 ? (unsigned)(ds * L.n_tile * 2) : L.b_bytes;
     L.hb_bytes = (unsigned)(kTileM * ds * 2);
@@ -824,18 +909,18 @@ bool tc_layout(int in_dim, int dt, int ds, TcLaunch& L)
     }
     L.idesc = make_idesc(kTileM, L.n_tile);
     unsigned cols = 32;
-    while (cols < 2u * (unsigned)L.n_tile) cols <<= 1;
+    while (cols < (unsigned)L.nd * (unsigned)L.n_tile) cols <<= 1;
     L.tmem_cols = cols;
     return cols <= 512;
 }
 
 }  // namespace
 
-TcConfig tc_config(int in_dim, int dt, int ds)
+TcConfig tc_config(int in_dim, int dt, int ds, int share)
 {
     TcLaunch L{};
     TcConfig c{0, 0, 0, kThreads, 0};
-    if (!tc_layout(in_dim, dt, ds, L)) return c;
+    if (!tc_layout(in_dim, dt, ds, share, L)) return c;
     c.n_tile = L.n_tile;
     c.n_split = L.n_split;
     c.smem_bytes = kSmemMax;
@@ -905,7 +990,7 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
 {
     *launches = 0;
     TcLaunch L{};
-    if (!tc_layout(P.in_dim, P.dt, P.ds, L)) return cudaErrorNotSupported;
+    if (!tc_layout(P.in_dim, P.dt, P.ds, share_heads(P), L)) return cudaErrorNotSupported;
     if (P.ds != 64 && P.ds != 128 && P.ds != 256) return cudaErrorNotSupported;
     L.groups = P.Lt * P.Ht * 2 * L.n_split;
     L.seq_cached = P.batch <= kMaxSeqCache;
@@ -925,11 +1010,12 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
         cudaError_t e = launch_pdl(span_plan_kernel, (nsub + 3) / 4, 128, 0, stream, P, t0, t1, (int)L.cap_rows, hdr, ent);
         if (e != cudaSuccess) return e;
         ++*launches;
-        const long long UH = (long long)(L.groups / 2) * L.m_tiles;
+        const long long UH = (long long)(L.groups / 2) * L.m_tiles / (L.hpu * L.spu);
         const int grid = (int)(UH < num_sms ? UH : num_sms);
-        // heads that share source rows: a GQA expansion group, or all heads of the dense form
-        const int E = P.dense ? P.Ht : (P.r == 1 ? P.e : 1);
-        L.share = E > 1 && P.Ht % E == 0 && grid % E == 0 ? E : 1;
+        // head units that share source rows beyond the heads one unit covers (a GQA expansion
+        // group, or all heads of the dense form): interleaved CTA sets
+        const int E = share_heads(P) / L.hpu;
+        L.share = E > 1 && P.Ht % (E * L.hpu) == 0 && grid % E == 0 ? E : 1;
         switch (P.ds) {
         case 256: e = launch_span_ds<256>(grid, stream, P, L); break;
         case 128: e = launch_span_ds<128>(grid, stream, P, L); break;

@@ -639,10 +639,10 @@ EncodeTiled encoder()
 
 }  // namespace
 
-bool aligned_supported(int in_dim, int dt, int ds, int Lt, int batch, int kl)
+bool aligned_supported(int in_dim, int dt, int ds, int share, int Lt, int batch, int kl)
 {
     // one source layer per target layer (one tensor map each) and a resident B image
-    TcConfig c = tc_config(in_dim, dt, ds);
+    TcConfig c = tc_config(in_dim, dt, ds, share);
     return c.ok && in_dim <= 256 && kl == 1 && Lt <= KVX_MAX_ALIGNED_LAYERS && batch <= KVX_MAX_ALIGNED_BATCH &&
            encoder() != nullptr;
 }
@@ -687,7 +687,7 @@ cudaError_t launch_pdl(K kernel, int grid, cudaStream_t stream, const AlignedPar
 cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps,
                                         const unsigned long long* host_turns, int num_sms, cudaStream_t stream)
 {
-    TcConfig cfg = tc_config(T.in_dim, T.dt, T.ds);
+    TcConfig cfg = tc_config(T.in_dim, T.dt, T.ds, share_heads(T));
     if (!cfg.ok || T.Lt > KVX_MAX_ALIGNED_LAYERS || T.batch > KVX_MAX_ALIGNED_BATCH) return cudaErrorNotSupported;
     static thread_local AlignedParams P;   // large (~27 KB): filled on the host, passed by value
     memset(&P, 0, offsetof(AlignedParams, maps));
