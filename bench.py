@@ -586,11 +586,13 @@ def fit_bench(args, spec):
     # pair of systems per process over up to 4096 tokens, scaled to all groups
     cores = os.cpu_count() or 1
     n_tok = min(4096, int(sum(spec.tgt_lens)))
-    with mp.get_context("spawn").Pool(cores) as pool:
-        secs = pool.map(_oracle_fit_worker, [(args.workload, n_tok)] * cores)
-    groups_per_proc = 1   # one target layer, one head: a K and a V system
     total_groups = spec.dst.num_layers * spec.dst.num_kv_heads
-    cpu_tok_s = n_tok * cores * groups_per_proc / max(secs) / total_groups
+    cpu_tok_s = None
+    if not args.no_cpu_baseline:
+        with mp.get_context("spawn").Pool(cores) as pool:
+            secs = pool.map(_oracle_fit_worker, [(args.workload, n_tok)] * cores)
+        groups_per_proc = 1   # one target layer, one head: a K and a V system
+        cpu_tok_s = n_tok * cores * groups_per_proc / max(secs) / total_groups
     import torch
     import paper_2608_30963_gb300 as kvx
     torch.cuda.set_device(0)
@@ -655,11 +657,12 @@ def fit_bench(args, spec):
                          "algorithmic_bytes": byts, "flops": flops, "roofline_ms": t_roof * 1e3,
                          "frac": t_roof * 1e3 / ms, "achieved_tflops": flops / (ms / 1e3) / 1e12,
                          "peaks": {"hbm_gbs": hbm, "bf16_tflops": tc}},
-            "solve_ms": solve_ms, "solve_status": bits,
-            "cpu_baseline": {"value": cpu_tok_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
-                             "sample": f"oracle fit (fp64 Gram sums and Cholesky) of target layer 0, head 0, K and V "
-                                       f"over {n_tok} tokens in each of {cores} spawned processes, scaled by "
-                                       f"{total_groups} (layer, head) pairs"}}
+            "solve_ms": solve_ms, "solve_status": bits}
+    if cpu_tok_s is not None:
+        line["cpu_baseline"] = {"value": cpu_tok_s, "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                                "sample": f"oracle fit (fp64 Gram sums and Cholesky) of target layer 0, head 0, K and "
+                                          f"V over {n_tok} tokens in each of {cores} spawned processes, scaled by "
+                                          f"{total_groups} (layer, head) pairs"}
     print(json.dumps(line), flush=True)
     f.close()
 

@@ -54,13 +54,13 @@ constexpr int kEpiWarp0 = 2;
 constexpr int kNumEpiWarps = 8;               // two per TMEM lane quadrant, splitting the rotary pairs
 constexpr int kXfWarp0 = kEpiWarp0 + kNumEpiWarps;
 constexpr int kNumXfWarps = 8;
-constexpr int kThreads = (kXfWarp0 + kNumXfWarps) * 32;
+constexpr int kBLoaderWarp = kXfWarp0 + kNumXfWarps;   // streams B pieces (streamed weights only)
+constexpr int kThreads = (kBLoaderWarp + 1) * 32;
 constexpr int kMaxSeqCache = 512;         // sequences whose metadata is kept in shared memory
 constexpr int kMaxTcIn = 1024;            // widest translator input row (in) this kernel takes
 constexpr int kMaxA = 2;                  // A head-block slots
 constexpr int kMaxB = 2;                  // B slots (1: the group's whole image; 2: head-block pieces)
 constexpr int kMaxD = 8;                  // accumulator slots in TMEM (512 columns / n_tile)
-constexpr int kBLoaderLane = 1;           // lane of the MMA warp that streams B pieces
 constexpr unsigned kBResidentMax = 65536; // largest B image kept resident per group
 constexpr unsigned kBPieceMax = 32768;    // largest streamed B piece (one source head's rows)
 
@@ -508,7 +508,12 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 const unsigned long long t0 = globaltimer();
                 while (!mbar_try_wait(bar(kBarMmaDone), 0) && globaltimer() - t0 < W.limit_ns) {}
             }
-        } else if (lane == kBLoaderLane && b_stream) {
+        }
+        __syncwarp();
+    } else if (warp == kBLoaderWarp) {
+        const bool b_stream = L.n_b > 1;
+        const uint32_t nb = (uint32_t)L.n_b;
+        if (lane == 0 && b_stream) {
             // ------------------------------------------------------------ B-loader (streamed weights)
             // Per unit, head-block q and piece p, in the MMA's order: the d_s rows of head-block q of
             // the piece's B image (one source head's rows of W, n_tile output columns).
@@ -537,7 +542,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             }
         }
         __syncwarp();
-    } else if (warp < kEpiWarp0 + kNumEpiWarps) {
+    } else if (warp >= kEpiWarp0 && warp < kEpiWarp0 + kNumEpiWarps) {
         // ------------------------------------------------------------ epilogue
         // Per unit: the output rows are resolved once; then per piece (head, output split), in
         // the MMA's order, the piece's accumulator slot is rotated, rounded, staged and stored.
@@ -568,7 +573,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 if (!W.wait(bar(kBarDFull + buf), (pcount / nd) & 1)) { ok = false; break; }
                 tc_fence_after();
                 // the staging row is shared by the two warps of this quadrant; the row's
-                // previous store (issued by the thread of lane parity = half) must have read it
+                // previous store must have read it
                 bulk_wait_read0();
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2));
@@ -598,8 +603,9 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 __syncwarp();
                 if (lane == 0) mbar_arrive(bar(kBarPair + quad * 2 + 1));
                 if (!W.wait(bar(kBarPair + quad * 2 + 1), pcount & 1)) { ok = false; break; }
-                // the quadrant's rows, split between its two warps by lane parity
-                if ((lane & 1) == half && valid && dst_off >= 0) {
+                // the quadrant's rows: stored by the half-0 warp when a unit has one piece, split
+                // between the two warps by lane parity when it has several
+                if ((L.np > 1 ? (lane & 1) == half : half == 0) && valid && dst_off >= 0) {
                     __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                          dst_head_off(P, x.h + hh);
                     if (P.plain_stores) {
@@ -612,7 +618,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             }
         }
         bulk_wait0();
-    } else {
+    } else if (warp >= kXfWarp0 && warp < kXfWarp0 + kNumXfWarps) {
         // ------------------------------------------------------------ prologue (A head-blocks)
         // Lanes split into groups of LPT, one target token per group; a lane owns one
         // chunk pair: pair slots [8cp, 8cp+8), i.e. channels [8cp, 8cp+8) and their rotary
@@ -845,9 +851,12 @@ bool tc_layout(int in_dim, int dt, int ds, int share, TcLaunch& L)
     // Heads per unit: as many of the heads sharing the input rows as the 512 accumulator columns
     // hold (d_t each), so their A is built once; each (head, output split) is a piece, and the
     // pieces' weights stream through two slots, one head-block (ds x n_tile) at a time.
+    // Only when one piece covers a whole output head (ds x dt weights within a streamed slot):
+    // splitting the heads' rows into narrower pieces multiplies the row stores.
     int hpu = 1;
-    for (int c = share; c > 1; --c)
-        if (share % c == 0 && c * dt <= 512) { hpu = c; break; }
+    if ((unsigned)(ds * dt * 2) <= kBPieceMax)
+        for (int c = share; c > 1; --c)
+            if (share % c == 0 && c * dt <= 512) { hpu = c; break; }
     if (hpu > 1) {
         L.n_b = kMaxB;
         L.n_tile = dt;
