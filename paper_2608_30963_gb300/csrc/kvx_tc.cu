@@ -975,7 +975,9 @@ static cudaError_t launch_span_ds(int grid, cudaStream_t stream, const Translate
 {
     const cudaError_t e = smem_opt_in<translate_tc_kernel<DS>>(kSmemMax);
     if (e != cudaSuccess) return e;
-    return launch_pdl(translate_tc_kernel<DS>, grid, kThreads, kSmemMax, stream, P, L);
+    // the B-loader warp (the last one) only when the weights stream
+    const int threads = L.n_b > 1 ? kThreads : kThreads - 32;
+    return launch_pdl(translate_tc_kernel<DS>, grid, threads, kSmemMax, stream, P, L);
 }
 
 size_t tc_plan_bytes(int tokens)

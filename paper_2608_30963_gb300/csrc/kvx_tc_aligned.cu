@@ -190,7 +190,10 @@ struct SlotPos {
     }
 };
 
-template <int HS>   // half head_dim of the source (32, 64 or 128)
+// HS: half head_dim of the source (32, 64 or 128).  NH: source heads in one A row when known at
+// compile time (the prologue's loop over them unrolls, so their shared-memory loads overlap), 0 =
+// from the parameters.
+template <int HS, int NH>
 __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const __grid_constant__ AlignedParams P)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -510,7 +513,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         const int xt = threadIdx.x - kXfWarp0 * 32;
         const int row = (warp & 3) * 32 + lane;
         const int part = (warp - kXfWarp0) >> 2;          // 0 or 1
-        const int heads = P.in_dim / (2 * HS);            // heads in one A row
+        const int heads = NH > 0 ? NH : P.in_dim / (2 * HS);   // heads in one A row
         constexpr int kChunks = HS / 8;                    // 16-byte chunks per half head
         constexpr int kMine = kChunks / 2;                 // chunks per thread
         const uint32_t cs_lane = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + P.cs_col;
@@ -562,7 +565,8 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                     for (int e2 = 0; e2 < 8; ++e2) { v[2 * e2] = __float_as_uint(cs[e2].x); v[2 * e2 + 1] = __float_as_uint(cs[e2].y); }
                     tmem_st16(cs_lane + csbuf * (uint32_t)(2 * HS) + 2 * i, v);
                 }
-                for (int q = 0; q < heads; ++q) {
+#pragma unroll
+                for (int q = 0; q < (NH > 0 ? NH : heads); ++q) {
                     // element i (and i+HS) of head q: K-block and column within it
                     const int k_lo = q * 2 * HS + i, k_hi = k_lo + HS;
                     uint32_t s_lo = sp.idx + (k_lo >> 6), s_hi = sp.idx + (k_hi >> 6);
@@ -684,6 +688,14 @@ cudaError_t launch_pdl(K kernel, int grid, cudaStream_t stream, const AlignedPar
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+template <int HS, int NH>
+static cudaError_t launch_aligned(int grid, cudaStream_t stream, const AlignedParams& P)
+{
+    const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<HS, NH>>(kSmemMax);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(translate_tc_aligned_kernel<HS, NH>, grid, stream, P);
+}
+
 cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps,
                                         const unsigned long long* host_turns, int num_sms, cudaStream_t stream)
 {
@@ -745,30 +757,13 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     }
     const long long UH = (long long)(P.groups / 2) * P.m_tiles_max;
     const int grid = (int)(UH < num_sms ? UH : num_sms);
+    // the 7B -> 1.5B geometry (two 128-channel source heads per A row) has its own instantiation
+    const int heads = T.in_dim / T.ds;
     switch (T.ds) {
-    case 64:
-        {
-            const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<32>>(kSmemMax);
-            if (e != cudaSuccess) return e;
-        }
-        return launch_pdl(translate_tc_aligned_kernel<32>, grid, stream, P);
-        break;
-    case 128:
-        {
-            const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<64>>(kSmemMax);
-            if (e != cudaSuccess) return e;
-        }
-        return launch_pdl(translate_tc_aligned_kernel<64>, grid, stream, P);
-        break;
-    case 256:
-        {
-            const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<128>>(kSmemMax);
-            if (e != cudaSuccess) return e;
-        }
-        return launch_pdl(translate_tc_aligned_kernel<128>, grid, stream, P);
-        break;
-    default:
-        return cudaErrorNotSupported;
+    case 64: return launch_aligned<32, 0>(grid, stream, P);
+    case 128: return heads == 2 ? launch_aligned<64, 2>(grid, stream, P) : launch_aligned<64, 0>(grid, stream, P);
+    case 256: return launch_aligned<128, 0>(grid, stream, P);
+    default: return cudaErrorNotSupported;
     }
     return cudaGetLastError();
 }
