@@ -390,39 +390,70 @@ __global__ void __launch_bounds__(256) fit_gram_simt_kernel(const T* __restrict_
 
 // ------------------------------------------------------------------ Gram sums on the tensor cores (bf16)
 // Work: per group g = (j*Ht + h)*2 + kv, row block mb (128 input channels) and 64-token K-block
-// kb of the call:  D[i, n] += sum_t Z^T[mb*128 + i, t] * Z^T[n, t],  Z = [X | Y] (in + dt columns).
-// The prologue warps build the block Z^T[in + dt rows][64 tokens] straight into shared memory in
-// the UMMA K-major 128-byte-swizzled layout (the tokens are the contraction dimension, so they
-// are the contiguous K of both operands; a 4-byte word holds two consecutive tokens of one
-// channel), from the source and target caches exactly as fit_rows_kernel forms X and Y.  The MMA
-// thread issues M = 128 (the block's rows of Z^T as A), N = in + dt (all rows of Z^T as B, in
-// pieces of <= 256), K = 16 tokens per instruction into one fp32 TMEM accumulator that lives for
-// the CTA's whole range of a (g, mb) unit; the epilogue warps then add it into the fp32 sums
-// (vector atomics for X^T X rows, coalesced atomics for X^T Y columns).  Each CTA takes a
-// contiguous range of the (unit, K-block) space, units ordered (g, mb) with mb fastest, so the
-// two row blocks of a group read the same cache rows at about the same time (L2 hits).
+// kb of the call:  D[i, n] += sum_t Z^T[mb*128 + i, t] * Z^T[n, t],  Z = [X | Y].  Only the
+// lower triangle of X^T X is formed (the solves read it): row block mb takes the X columns
+// [0, (mb+1)*128) and the dt columns of Y, so its accumulator holds (mb+1)*128 + dt columns.
+//   loader warp  resolves the block's 64 tokens into a table in shared memory and copies the
+//                source rows of the block's span window (per source head-block) and the 64 target
+//                rows into padded shared-memory rows with bulk copies (a ring of raw slots).
+//   8 prologue warps  build the transposed block Z^T[rows][64 tokens] in the UMMA K-major
+//                128-byte-swizzled layout (tokens are the contraction dimension): one lane per
+//                token, one 16-channel chunk pair per pass, (cos, sin) once per token and pair
+//                for every source head of the input row; tokens 2w and 2w+1 (adjacent lanes)
+//                exchange values by shuffle and write one 4-byte word each.  X rows as the
+//                translation forms them (span mean of un-rotated source rows), Y rows with the
+//                target RoPE undone for K, both rounded to bf16.  Tokens whose span leaves the
+//                window read their rows from global memory.
+//   MMA thread   M = 128 (the block's rows of Z^T as A), N over the needed rows of Z^T as B (in
+//                pieces of <= 256), K = 16 tokens per instruction, into one fp32 TMEM
+//                accumulator that lives for the CTA's range of a unit.
+//   4 epilogue warps  add the accumulator into the fp32 sums (vector atomics for X^T X rows,
+//                coalesced atomics for X^T Y columns).
+// Units are (g, chunk of K-blocks, mb) with mb fastest, so the two row blocks of a chunk read
+// the same cache rows back to back (the second read hits L2); each CTA takes a contiguous range
+// of the (unit, K-block) space.
 constexpr int kGramK = 64;
 constexpr int kGramMmaWarp = 0;
 constexpr int kGramEpiWarp0 = 1;
 constexpr int kGramNumEpi = 4;
 constexpr int kGramXfWarp0 = kGramEpiWarp0 + kGramNumEpi;
 constexpr int kGramNumXf = 8;
-constexpr int kGramThreads = (kGramXfWarp0 + kGramNumXf) * 32;
+constexpr int kGramLoadWarp = kGramXfWarp0 + kGramNumXf;
+constexpr int kGramThreads = (kGramLoadWarp + 1) * 32;
 constexpr int kGramMaxStages = 4;
+constexpr int kGramMaxRaw = 2;
 constexpr int kGramMaxRows = 512;   // in + dt: one 128 x 512 fp32 accumulator fills TMEM
+constexpr int kGramMaxHeads = 4;    // source head-blocks in one input row
+
+struct GramTok {
+    int b, lo, hi, pt;       // sequence, clamped source span, target position
+    long long dst_off;       // target row offset (head 0), -1: none
+    int ok;                  // contributes (a valid row with a span)
+    int pad;
+};
 
 struct GramLaunch {
-    int nrows;             // in + dt
+    int nrows;             // in + dt (rows of a full Z^T block)
     int mbs;               // row blocks of 128 input channels: in / 128
-    int units;             // groups * mbs
     int nkb;               // K-blocks of 64 tokens in the call
-    int stages;            // K-block ring depth
+    int kc;                // K-blocks per unit (a chunk); nkb % kc == 0
+    int nch;               // chunks: nkb / kc
+    int units;             // groups * nch * mbs
+    int stages;            // Z^T block ring depth
     unsigned stage_bytes;  // nrows * 128
-    int n0;                // first N piece: columns [0, n0); second: [n0, nrows)
-    unsigned idesc0, idesc1;
+    int raw_slots;         // raw staging ring depth
+    int rcap;              // source rows one window holds
+    unsigned src_row, tgt_row;   // padded row pitches of the staged source / target rows (bytes)
+    unsigned raw_bytes;    // one raw slot: token table, header, source window, target rows
+    unsigned off_raw, off_bar;
     float* G;              // [groups][in][in]
     float* C;              // [groups][dt][in]
 };
+
+__host__ __device__ inline uint32_t gram_idesc_dev(int N)
+{
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+}
 
 // Byte offset of the 4-byte word holding tokens (2 lw, 2 lw + 1) of row r in a K-major SW128
 // block of 64 tokens (rows 128 bytes apart within an 8-row atom of 1024 bytes).
@@ -431,49 +462,30 @@ __device__ __forceinline__ uint32_t gram_word(int r, int lw)
     return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((((lw >> 2) ^ (r & 7)) & 7) << 4) + (lw & 3) * 4);
 }
 
-// Bring the cache rows K-block w of unit `unit` reads into L2 ahead of its prologue: the
-// source rows of every head-block (one range from the first token's span start to the last
-// token's span end, within the first token's sequence) and the target rows (a range when the
-// target cache is contiguous).  Prefetches are hints: ranges are clipped to the caches.
-__device__ __forceinline__ void l2_prefetch(const void* p, uint32_t bytes)
+// Unit u of the (g, chunk, mb) space and K-block index within the unit.
+struct GramUnit {
+    int g, mb, kb;   // kb: K-block of the call
+};
+__device__ __forceinline__ GramUnit gram_unit(const GramLaunch& L, int w)
 {
-    const char* c = (const char*)p;
-    for (uint32_t o = 0; o < bytes; o += 16384u) {   // pieces of at most 16 KB
-        const uint32_t n = bytes - o < 16384u ? bytes - o : 16384u;
-        asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(c + o), "r"(n) : "memory");
-    }
+    const int u = w / L.kc, kbi = w - u * L.kc;
+    const int mb = u % L.mbs, gc = u / L.mbs;
+    const int ch = gc % L.nch, g = gc / L.nch;
+    return GramUnit{g, mb, ch * L.kc + kbi};
 }
-__device__ void gram_prefetch(const TranslateParams& P, int unit, int kb, int mbs)
+
+// Writes this lane's token (even or odd of a pair) into 8 rows of the block, exchanging with the
+// neighbouring lane so that each lane writes one word per row: the even lane rows r_lo + e, the odd
+// lane rows r_hi + e.
+__device__ __forceinline__ void gram_put(uint8_t* st, int r_lo, int r_hi, int lw, bool odd, const float (&lo)[8],
+                                         const float (&hi)[8])
 {
-    const int g = unit / mbs, kv = g & 1, jh = g >> 1, h = jh % P.Ht, j = jh / P.Ht;
-    const int t0 = kb * kGramK, t1 = min(t0 + kGramK, P.T_total) - 1;
-    if (t1 < t0) return;
-    const int b = find_seq(P.seq_off, P.batch, t0);
-    const int off = __ldg(&P.seq_off[b]), end = __ldg(&P.seq_off[b + 1]);
-    int S = __ldg(&P.src_seq_len[b]);
-    S = S < 0 ? 0 : (S > P.src_max_seq ? P.src_max_seq : S);
-    const int tl = min(t1, end - 1);
-    int lo = t0 - off, hi = tl - off + 1;
-    if (P.span_lo) { lo = __ldg(&P.span_lo[t0]); hi = __ldg(&P.span_hi[tl]); }
-    lo = max(lo, 0);
-    hi = min(hi, S);
-    if (P.ss == P.ds && hi > lo) {
-        const int heads = P.in_dim / P.ds;
-        for (int q = 0; q < heads; ++q) {
-            int slot, gs;
-            head_block(P, j, h, q, slot, gs);
-            const __nv_bfloat16* base = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) +
-                                        (long long)b * P.sb + (long long)gs * P.sh + (long long)lo * P.ss;
-            l2_prefetch(base, (uint32_t)(hi - lo) * P.ds * 2);
-        }
-    }
-    if (!P.paged && P.dts == P.dt) {
-        const int ta = t0 - off, tb = min(tl - off + 1, P.dst_max_seq);
-        if (tb > ta) {
-            const __nv_bfloat16* rowp = (const __nv_bfloat16*)(kv ? P.dst_v[j] : P.dst_k[j]) + (long long)b * P.db +
-                                        (long long)h * P.dh + (long long)ta * P.dts;
-            l2_prefetch(rowp, (uint32_t)(tb - ta) * P.dt * 2);
-        }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float send = odd ? lo[e] : hi[e];
+        const float got = __shfl_xor_sync(0xffffffffu, send, 1);
+        if (!odd) *reinterpret_cast<uint32_t*>(st + gram_word(r_lo + e, lw)) = pack_bf16(lo[e], got);
+        else *reinterpret_cast<uint32_t*>(st + gram_word(r_hi + e, lw)) = pack_bf16(got, hi[e]);
     }
 }
 
@@ -483,25 +495,35 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
 {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-    uint64_t* sBar = reinterpret_cast<uint64_t*>(smem + (size_t)L.stages * L.stage_bytes);
-    // barriers: full[s] (prologue warps), empty[s] (MMA commit), dfull (MMA commit), dempty (epilogue
-    // warps), done (the MMA thread's last commit)
-    const int bFull = 0, bEmpty = kGramMaxStages, bDFull = 2 * kGramMaxStages, bDEmpty = bDFull + 1, bDone = bDFull + 2;
+    uint8_t* sRaw = smem + L.off_raw;
+    uint64_t* sBar = reinterpret_cast<uint64_t*>(smem + L.off_bar);
+    // barriers: zfull[s] (prologue warps), zempty[s] (MMA commit), rfull[r] (loader + copies),
+    // rempty[r] (prologue warps), dfull (MMA commit), dempty (epilogue warps), done (MMA)
+    constexpr int bZFull = 0, bZEmpty = kGramMaxStages, bRFull = 2 * kGramMaxStages, bREmpty = bRFull + kGramMaxRaw;
+    constexpr int bDFull = bREmpty + kGramMaxRaw, bDEmpty = bDFull + 1, bDone = bDFull + 2;
     volatile int* sAbort = reinterpret_cast<volatile int*>(sBar + bDone + 1);
     uint32_t* sTmem = reinterpret_cast<uint32_t*>(sBar + bDone + 2);
+    unsigned long long* sTurn = reinterpret_cast<unsigned long long*>(sBar + bDone + 4);   // source | target
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     auto bar = [&](int i) { return smem_u32(&sBar[i]); };
     if (threadIdx.x == 0) {
         *sAbort = 0;
         for (int i = 0; i < L.stages; ++i) {
-            mbar_init(bar(bFull + i), kGramNumXf);
-            mbar_init(bar(bEmpty + i), 1);
+            mbar_init(bar(bZFull + i), kGramNumXf);
+            mbar_init(bar(bZEmpty + i), 1);
+        }
+        for (int i = 0; i < L.raw_slots; ++i) {
+            mbar_init(bar(bRFull + i), 1);
+            mbar_init(bar(bREmpty + i), kGramNumXf);
         }
         mbar_init(bar(bDFull), 1);
         mbar_init(bar(bDEmpty), kGramNumEpi);
         mbar_init(bar(bDone), 1);
         fence_mbar_init();
     }
+    for (int i = threadIdx.x; i < (P.ds >> 1); i += blockDim.x) sTurn[i] = P.rs.enabled ? __ldg(&P.rs.turns[i]) : 0ull;
+    for (int i = threadIdx.x; i < (P.dt >> 1); i += blockDim.x)
+        sTurn[(P.ds >> 1) + i] = P.rt.enabled ? __ldg(&P.rt.turns[i]) : 0ull;
     if (warp == kGramMmaWarp) {
         tmem_alloc(smem_u32(sTmem), 512);
         tmem_relinquish();
@@ -511,34 +533,48 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
     tc_fence_after();
     const uint32_t tmem_base = *sTmem;
     const Waiter W{sAbort, P.status};
-    const long long total = (long long)L.units * L.nkb;
+    const long long total = (long long)L.units * L.kc;
     const int w0 = (int)((long long)blockIdx.x * total / gridDim.x);
     const int w1 = (int)((long long)(blockIdx.x + 1) * total / gridDim.x);
     const int in = P.in_dim, dt = P.dt;
+    const int heads = in / DS;
+    auto tok_tab = [&](int r) { return reinterpret_cast<GramTok*>(sRaw + (size_t)r * L.raw_bytes); };
+    auto win_hdr = [&](int r) { return reinterpret_cast<int*>(sRaw + (size_t)r * L.raw_bytes + kGramK * sizeof(GramTok)); };
+    auto src_rows = [&](int r, int q) {
+        return sRaw + (size_t)r * L.raw_bytes + kGramK * sizeof(GramTok) + 16 + (size_t)q * L.rcap * L.src_row;
+    };
+    auto tgt_rows = [&](int r) {
+        return sRaw + (size_t)r * L.raw_bytes + kGramK * sizeof(GramTok) + 16 + (size_t)heads * L.rcap * L.src_row;
+    };
 
     if (warp == kGramMmaWarp) {
         if (lane == 0) {
             uint32_t it = 0, ucount = 0;
             bool issued = false;
             for (int w = w0; w < w1; ++w, ++it) {
-                const int unit = w / L.nkb, kb = w - unit * L.nkb;
-                const bool first = w == w0 || kb == 0, last = w == w1 - 1 || kb == L.nkb - 1;
+                const GramUnit x = gram_unit(L, w);
+                const int kbi = w % L.kc;
+                const bool first = w == w0 || kbi == 0, last = w == w1 - 1 || kbi == L.kc - 1;
                 const uint32_t s = it % (uint32_t)L.stages, ph = (it / (uint32_t)L.stages) & 1;
                 if (first && !W.wait(bar(bDEmpty), (ucount & 1) ^ 1)) break;
-                if (!W.wait(bar(bFull + s), ph)) break;
+                if (!W.wait(bar(bZFull + s), ph)) break;
                 tc_fence_after();
                 const uint32_t st = smem_u32(smem) + s * L.stage_bytes;
-                const uint32_t a0 = st + (uint32_t)(unit % L.mbs) * (128 / 8) * 1024;
+                const uint32_t a0 = st + (uint32_t)x.mb * (128 / 8) * 1024;
+                const int nx = (x.mb + 1) * 128;   // X columns of the lower triangle
 #pragma unroll
                 for (int k = 0; k < kGramK / 16; ++k) {
                     const uint32_t acc = (first && k == 0) ? 0u : 1u;
                     const uint64_t ad = sw128_desc(a0 + k * 32);
-                    umma_bf16(tmem_base, ad, sw128_desc(st + k * 32), L.idesc0, acc);
-                    if (L.n0 < L.nrows)
-                        umma_bf16(tmem_base + (uint32_t)L.n0, ad, sw128_desc(st + (uint32_t)(L.n0 / 8) * 1024 + k * 32),
-                                  L.idesc1, acc);
+                    for (int c0 = 0; c0 < nx; c0 += 256) {   // X columns in pieces of <= 256
+                        const int n = nx - c0 < 256 ? nx - c0 : 256;
+                        umma_bf16(tmem_base + (uint32_t)c0, ad, sw128_desc(st + (uint32_t)(c0 / 8) * 1024 + k * 32),
+                                  gram_idesc_dev(n), acc);
+                    }
+                    umma_bf16(tmem_base + (uint32_t)nx, ad, sw128_desc(st + (uint32_t)(in / 8) * 1024 + k * 32),
+                              gram_idesc_dev(dt), acc);
                 }
-                umma_commit(bar(bEmpty + s));
+                umma_commit(bar(bZEmpty + s));
                 issued = true;
                 if (last) {
                     umma_commit(bar(bDFull));
@@ -557,19 +593,21 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
         // ------------------------------------------------------------ epilogue: accumulator -> sums
         const int quad = warp & 3;
         uint32_t ucount = 0;
-        const int u_first = w0 / L.nkb, u_last = w1 > w0 ? (w1 - 1) / L.nkb : u_first - 1;
+        const int u_first = w0 / L.kc, u_last = w1 > w0 ? (w1 - 1) / L.kc : u_first - 1;
         for (int u = u_first; u <= u_last; ++u, ++ucount) {
             if (!W.wait(bar(bDFull), ucount & 1)) break;
             tc_fence_after();
-            const int g = u / L.mbs, row = (u % L.mbs) * 128 + quad * 32 + lane;
-            float* grow = L.G + ((size_t)g * in + row) * in;
-            float* cg = L.C + (size_t)g * dt * in + row;
+            const GramUnit x = gram_unit(L, u * L.kc);
+            const int nx = (x.mb + 1) * 128;
+            const int row = x.mb * 128 + quad * 32 + lane;
+            float* grow = L.G + ((size_t)x.g * in + row) * in;
+            float* cg = L.C + (size_t)x.g * dt * in + row;
             const uint32_t taddr = tmem_base + ((uint32_t)(quad * 32) << 16);
-            for (int c0 = 0; c0 < L.nrows; c0 += 32) {
+            for (int c0 = 0; c0 < nx + dt; c0 += 32) {
                 uint32_t r[32];
                 tmem_ld32(taddr + c0, r);
                 tmem_ld_wait();
-                if (c0 < in) {
+                if (c0 < nx) {
 #pragma unroll
                     for (int q = 0; q < 8; ++q)
                         atomicAdd(reinterpret_cast<float4*>(grow + c0 + 4 * q),
@@ -577,141 +615,211 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                                               __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3])));
                 } else {
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) atomicAdd(cg + (size_t)(c0 - in + e) * in, __uint_as_float(r[e]));
+                    for (int e = 0; e < 32; ++e) atomicAdd(cg + (size_t)(c0 - nx + e) * in, __uint_as_float(r[e]));
                 }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(bar(bDEmpty));
         }
+    } else if (warp == kGramLoadWarp) {
+        // ------------------------------------------------------------ loader: tokens and raw rows
+        const uint64_t pol = policy_evict_last();   // the partner row block reads them again
+        uint32_t it = 0, issued = 0;
+        bool ok = true;
+        for (int w = w0; w < w1 && ok; ++w, ++it) {
+            const GramUnit x = gram_unit(L, w);
+            const int kv = x.g & 1, jh = x.g >> 1, h = jh % P.Ht, j = jh / P.Ht;
+            const uint32_t r = it % (uint32_t)L.raw_slots, ph = (it / (uint32_t)L.raw_slots) & 1;
+            if (!W.wait(bar(bREmpty + r), ph ^ 1)) break;
+            GramTok* tt = tok_tab((int)r);
+            GramTok tk[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int i = lane + 32 * u, tp = x.kb * kGramK + i;
+                tk[u] = GramTok{0, 0, 0, 0, -1, 0, 0};
+                if (tp < P.T_total) {
+                    const TokenInfo ti = resolve_token(P, tp);
+                    tk[u] = GramTok{ti.b, ti.lo, ti.hi, ti.pt, ti.dst_off, ti.dst_off >= 0 && ti.hi > ti.lo, 0};
+                }
+                tt[i] = tk[u];
+            }
+            // the window: from the first token's span start, within its sequence, up to rcap rows
+            const int b0 = __shfl_sync(0xffffffffu, tk[0].b, 0), c0 = __shfl_sync(0xffffffffu, tk[0].lo, 0);
+            const int ok0 = __shfl_sync(0xffffffffu, tk[0].ok, 0);
+            int hm = INT_MIN;
+#pragma unroll
+            for (int u = 0; u < 2; ++u)
+                if (tk[u].ok && tk[u].b == b0) hm = max(hm, tk[u].hi);
+            hm = __reduce_max_sync(0xffffffffu, hm);
+            const int R = ok0 && hm > c0 ? min(hm - c0, L.rcap) : 0;
+            const int n_tgt = __popc(__ballot_sync(0xffffffffu, tk[0].ok)) + __popc(__ballot_sync(0xffffffffu, tk[1].ok));
+            if (lane == 0) {
+                int* hd = win_hdr((int)r);
+                hd[0] = b0;
+                hd[1] = c0;
+                hd[2] = R;
+            }
+            __syncwarp();
+            const uint32_t bytes = (uint32_t)R * (uint32_t)DS * 2u * (uint32_t)heads + (uint32_t)n_tgt * (uint32_t)dt * 2u;
+            if (lane == 0) mbar_arrive_expect_tx(bar(bRFull + r), bytes);
+            __syncwarp();
+            for (int q = 0; q < heads; ++q) {
+                int slot, gs;
+                head_block(P, j, h, q, slot, gs);
+                const __nv_bfloat16* base = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) +
+                                            (long long)b0 * P.sb + (long long)gs * P.sh;
+                uint8_t* dstq = src_rows((int)r, q);
+                for (int rr = lane; rr < R; rr += 32)
+                    bulk_g2s(smem_u32(dstq + (size_t)rr * L.src_row), base + (long long)(c0 + rr) * P.ss, DS * 2,
+                             bar(bRFull + r), pol);
+            }
+            const __nv_bfloat16* tgt = (const __nv_bfloat16*)(kv ? P.dst_v[j] : P.dst_k[j]);
+            const long long hoff = dst_head_off(P, h);
+#pragma unroll
+            for (int u = 0; u < 2; ++u)
+                if (tk[u].ok)
+                    bulk_g2s(smem_u32(tgt_rows((int)r) + (size_t)(lane + 32 * u) * L.tgt_row), tgt + tk[u].dst_off + hoff,
+                             (uint32_t)dt * 2u, bar(bRFull + r), pol);
+            ++issued;
+        }
+        if (*sAbort) {   // let the copies in flight land before the CTA leaves
+            const unsigned long long t0 = globaltimer();
+            const uint32_t ns = (uint32_t)L.raw_slots;
+            for (uint32_t c = issued > ns ? issued - ns : 0; c < issued; ++c)
+                while (!mbar_try_wait(bar(bRFull + c % ns), (c / ns) & 1) && globaltimer() - t0 < kWaitNs) {}
+        }
     } else {
         // ------------------------------------------------------------ prologue: Z^T blocks in shared memory
         constexpr int HS = DS / 2;
         constexpr int CPH = DS / 16;                 // chunk pairs (16 channels) per source head
         const int xw = warp - kGramXfWarp0;
-        const int heads = in / DS;
-        const int nx = heads * CPH, items = nx + dt / 16;
-        const int hs_t = dt >> 1;
+        const int cpt = dt / 16;                     // chunk pairs of a target row
+        const unsigned long long* sTurnS = sTurn;
+        const unsigned long long* sTurnT = sTurn + (P.ds >> 1);
+        const bool odd = lane & 1;
         uint32_t it = 0;
-        if (xw == 0 && lane < 2 && w0 + lane < w1) {   // the first two K-blocks of the range
-            const int w = w0 + lane, unit = w / L.nkb;
-            gram_prefetch(P, unit, w - unit * L.nkb, L.mbs);
-        }
         for (int w = w0; w < w1; ++w, ++it) {
-            const int unit = w / L.nkb, kb = w - unit * L.nkb;
-            const int g = unit / L.mbs;
-            if (xw == 0 && lane == 0 && w + 2 < w1) {   // two K-blocks ahead
-                const int un = (w + 2) / L.nkb;
-                gram_prefetch(P, un, w + 2 - un * L.nkb, L.mbs);
-            }
-            const int kv = g & 1, jh = g >> 1, h = jh % P.Ht, j = jh / P.Ht;
+            const GramUnit x = gram_unit(L, w);
+            const int kv = x.g & 1, jh = x.g >> 1, h = jh % P.Ht, j = jh / P.Ht;
+            // X head-blocks this row block needs: the rows [0, (mb+1)*128) of the lower triangle
+            const int nh = min(heads, ((x.mb + 1) * 128 + DS - 1) / DS);
             const uint32_t s = it % (uint32_t)L.stages, ph = (it / (uint32_t)L.stages) & 1;
-            if (!W.wait(bar(bEmpty + s), ph ^ 1)) break;
+            const uint32_t r = it % (uint32_t)L.raw_slots, rph = (it / (uint32_t)L.raw_slots) & 1;
+            if (!W.wait(bar(bZEmpty + s), ph ^ 1)) break;
+            if (!W.wait(bar(bRFull + r), rph)) break;
             uint8_t* st = smem + (size_t)s * L.stage_bytes;
-            // this lane's two tokens of the block
-            TokenInfo ti[2];
-            bool ok[2];
-#pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const int tp = kb * kGramK + 2 * lane + u;
-                ok[u] = tp < P.T_total;
-                if (ok[u]) {
-                    ti[u] = resolve_token(P, tp);
-                    ok[u] = ti[u].dst_off >= 0 && ti[u].hi > ti[u].lo;
-                }
-            }
+            const GramTok* tt = tok_tab((int)r);
+            const int* hd = win_hdr((int)r);
+            const int b0 = hd[0], c0 = hd[1], R = hd[2];
             const bool rot_s = kv == 0 && P.rs.enabled, rot_t = kv == 0 && P.rt.enabled;
-            const __nv_bfloat16* tgt = (const __nv_bfloat16*)(kv ? P.dst_v[j] : P.dst_k[j]);
-            const long long hoff = dst_head_off(P, h);
-            for (int item = xw; item < items; item += kGramNumXf) {
-                float a0[2][8], a1[2][8];
-                int r_lo, r_hi;
-                if (item < nx) {
-                    // X: head-block q, chunk pair cp: span mean of the un-rotated source rows
-                    const int q = item / CPH, cp = item - q * CPH;
+            const int pieces = (CPH + cpt) * 2;
+            for (int pc = xw; pc < pieces; pc += kGramNumXf) {
+                const int half = pc & 1, item = pc >> 1;
+                const int i = half * 32 + lane;               // this lane's token
+                const int lw = i >> 1;
+                const GramTok tk = tt[i];
+                if (item < CPH) {
+                    // X: chunk pair `item` of every needed source head, span mean of un-rotated rows
+                    const int cp = item;
                     int c_lo, c_hi;
                     pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
-                    r_lo = q * DS + c_lo;
-                    r_hi = q * DS + c_hi;
-                    int slot, gs;
-                    head_block(P, j, h, q, slot, gs);
                     const bool rot = rot_s && cp * 8 < P.rhalf_s;
+                    float a0[kGramMaxHeads][8], a1[kGramMaxHeads][8];
 #pragma unroll
-                    for (int u = 0; u < 2; ++u) {
+                    for (int q = 0; q < kGramMaxHeads; ++q)
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) { a0[u][e] = 0.f; a1[u][e] = 0.f; }
-                        if (!ok[u]) continue;
-                        const __nv_bfloat16* base = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) +
-                                                    (long long)ti[u].b * P.sb + (long long)gs * P.sh;
-                        for (int sidx = ti[u].lo; sidx < ti[u].hi; ++sidx) {
-                            const __nv_bfloat16* rowp = base + (long long)sidx * P.ss;
-                            const uint4 w0v = __ldg(reinterpret_cast<const uint4*>(rowp + c_lo));
-                            const uint4 w1v = __ldg(reinterpret_cast<const uint4*>(rowp + c_hi));
-                            const uint32_t v0[4] = {w0v.x, w0v.y, w0v.z, w0v.w}, v1[4] = {w1v.x, w1v.y, w1v.z, w1v.w};
+                        for (int e = 0; e < 8; ++e) { a0[q][e] = 0.f; a1[q][e] = 0.f; }
+                    if (tk.ok) {
+                        const bool inwin = tk.b == b0 && tk.lo >= c0 && tk.hi <= c0 + R;
+                        for (int sidx = tk.lo; sidx < tk.hi; ++sidx) {
+                            float2 cs[8];
                             if (rot) {
-                                const int pos = src_pos_of(P, ti[u].b, sidx);
+                                const int pos = src_pos_of(P, tk.b, sidx);
 #pragma unroll
-                                for (int e = 0; e < 8; ++e) {   // R(-theta)
-                                    const float x0 = (e & 1) ? bf_hi(v0[e >> 1]) : bf_lo(v0[e >> 1]);
-                                    const float x1 = (e & 1) ? bf_hi(v1[e >> 1]) : bf_lo(v1[e >> 1]);
-                                    const float2 cs = rope_cs(P.rs, pos, cp * 8 + e);
-                                    a0[u][e] += fmaf(x0, cs.x, x1 * cs.y);
-                                    a1[u][e] += fmaf(x1, cs.x, -x0 * cs.y);
+                                for (int e = 0; e < 8; ++e) cs[e] = turn_cs(sTurnS[cp * 8 + e], pos);
+                            }
+#pragma unroll
+                            for (int q = 0; q < kGramMaxHeads; ++q) {
+                                if (q >= nh) break;
+                                uint4 w0v, w1v;
+                                if (inwin) {
+                                    const uint8_t* rp = src_rows((int)r, q) + (size_t)(sidx - c0) * L.src_row;
+                                    w0v = *reinterpret_cast<const uint4*>(rp + c_lo * 2);
+                                    w1v = *reinterpret_cast<const uint4*>(rp + c_hi * 2);
+                                } else {
+                                    int slot, gs;
+                                    head_block(P, j, h, q, slot, gs);
+                                    const __nv_bfloat16* rp = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) +
+                                                              (long long)tk.b * P.sb + (long long)gs * P.sh +
+                                                              (long long)sidx * P.ss;
+                                    w0v = __ldg(reinterpret_cast<const uint4*>(rp + c_lo));
+                                    w1v = __ldg(reinterpret_cast<const uint4*>(rp + c_hi));
                                 }
-                            } else {
+                                const uint32_t v0[4] = {w0v.x, w0v.y, w0v.z, w0v.w}, v1[4] = {w1v.x, w1v.y, w1v.z, w1v.w};
 #pragma unroll
                                 for (int e = 0; e < 8; ++e) {
-                                    a0[u][e] += (e & 1) ? bf_hi(v0[e >> 1]) : bf_lo(v0[e >> 1]);
-                                    a1[u][e] += (e & 1) ? bf_hi(v1[e >> 1]) : bf_lo(v1[e >> 1]);
+                                    const float x0 = (e & 1) ? bf_hi(v0[e >> 1]) : bf_lo(v0[e >> 1]);
+                                    const float x1 = (e & 1) ? bf_hi(v1[e >> 1]) : bf_lo(v1[e >> 1]);
+                                    if (rot) {   // R(-theta)
+                                        a0[q][e] += fmaf(x0, cs[e].x, x1 * cs[e].y);
+                                        a1[q][e] += fmaf(x1, cs[e].x, -x0 * cs[e].y);
+                                    } else {
+                                        a0[q][e] += x0;
+                                        a1[q][e] += x1;
+                                    }
                                 }
                             }
                         }
-                        const float inv = 1.f / (float)(ti[u].hi - ti[u].lo);
+                        const float inv = 1.f / (float)(tk.hi - tk.lo);
 #pragma unroll
-                        for (int e = 0; e < 8; ++e) { a0[u][e] *= inv; a1[u][e] *= inv; }
+                        for (int q = 0; q < kGramMaxHeads; ++q)
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) { a0[q][e] *= inv; a1[q][e] *= inv; }
+                    }
+#pragma unroll
+                    for (int q = 0; q < kGramMaxHeads; ++q) {
+                        if (q >= nh) break;
+                        gram_put(st, q * DS + c_lo, q * DS + c_hi, lw, odd, a0[q], a1[q]);
                     }
                 } else {
-                    // Y: chunk pair cp of the target row, target RoPE undone for K
-                    const int cp = item - nx;
+                    // Y: chunk pair of the target row, target RoPE undone for K
+                    const int cp = item - CPH;
                     int c_lo, c_hi;
-                    pair_channels(cp * 8, hs_t, P.rhalf_t, c_lo, c_hi);
-                    r_lo = in + c_lo;
-                    r_hi = in + c_hi;
+                    pair_channels(cp * 8, dt >> 1, P.rhalf_t, c_lo, c_hi);
                     const bool rot = rot_t && cp * 8 < P.rhalf_t;
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-#pragma unroll
-                        for (int e = 0; e < 8; ++e) { a0[u][e] = 0.f; a1[u][e] = 0.f; }
-                        if (!ok[u]) continue;
-                        const __nv_bfloat16* rowp = tgt + ti[u].dst_off + hoff;
-                        const uint4 w0v = __ldg(reinterpret_cast<const uint4*>(rowp + c_lo));
-                        const uint4 w1v = __ldg(reinterpret_cast<const uint4*>(rowp + c_hi));
+                    float y0[8], y1[8];
+                    if (tk.ok) {
+                        const uint8_t* rp = tgt_rows((int)r) + (size_t)i * L.tgt_row;
+                        const uint4 w0v = *reinterpret_cast<const uint4*>(rp + c_lo * 2);
+                        const uint4 w1v = *reinterpret_cast<const uint4*>(rp + c_hi * 2);
                         const uint32_t v0[4] = {w0v.x, w0v.y, w0v.z, w0v.w}, v1[4] = {w1v.x, w1v.y, w1v.z, w1v.w};
 #pragma unroll
                         for (int e = 0; e < 8; ++e) {
-                            const float y0 = (e & 1) ? bf_hi(v0[e >> 1]) : bf_lo(v0[e >> 1]);
-                            const float y1 = (e & 1) ? bf_hi(v1[e >> 1]) : bf_lo(v1[e >> 1]);
+                            const float u0 = (e & 1) ? bf_hi(v0[e >> 1]) : bf_lo(v0[e >> 1]);
+                            const float u1 = (e & 1) ? bf_hi(v1[e >> 1]) : bf_lo(v1[e >> 1]);
                             if (rot) {   // R(-theta)
-                                const float2 cs = rope_cs(P.rt, ti[u].pt, cp * 8 + e);
-                                a0[u][e] = fmaf(y0, cs.x, y1 * cs.y);
-                                a1[u][e] = fmaf(y1, cs.x, -y0 * cs.y);
+                                const float2 cs = turn_cs(sTurnT[cp * 8 + e], tk.pt);
+                                y0[e] = fmaf(u0, cs.x, u1 * cs.y);
+                                y1[e] = fmaf(u1, cs.x, -u0 * cs.y);
                             } else {
-                                a0[u][e] = y0;
-                                a1[u][e] = y1;
+                                y0[e] = u0;
+                                y1[e] = u1;
                             }
                         }
-                    }
-                }
-                // rows r_lo + e and r_hi + e, tokens (2 lane, 2 lane + 1) of the block: one word each
+                    } else {
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    *reinterpret_cast<uint32_t*>(st + gram_word(r_lo + e, lane)) = pack_bf16(a0[0][e], a0[1][e]);
-                    *reinterpret_cast<uint32_t*>(st + gram_word(r_hi + e, lane)) = pack_bf16(a1[0][e], a1[1][e]);
+                        for (int e = 0; e < 8; ++e) { y0[e] = 0.f; y1[e] = 0.f; }
+                    }
+                    gram_put(st, in + c_lo, in + c_hi, lw, odd, y0, y1);
                 }
             }
             fence_proxy_async();
             __syncwarp();
-            if (lane == 0) mbar_arrive(bar(bFull + s));
+            if (lane == 0) {
+                mbar_arrive(bar(bZFull + s));
+                mbar_arrive(bar(bREmpty + r));
+            }
         }
     }
     tc_fence_before();
@@ -722,10 +830,6 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
     }
 }
 
-uint32_t gram_idesc(int N)
-{
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
-}
 
 // solution columns per block for the small solve, and its dynamic shared memory
 int small_solve_cols(int in, int dt)
@@ -816,7 +920,7 @@ extern "C" KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, do
     // tensor-core Gram sums for bf16 caches whose input rows split into 128-channel blocks and
     // whose [X | Y] rows fit one TMEM accumulator; the CUDA-core path otherwise
     f->tc = D.dtype == KVX_BF16 && in % 128 == 0 && in + dt <= (size_t)kGramMaxRows && in % ds == 0 &&
-            (ds == 64 || ds == 128 || ds == 256);
+            (ds == 64 || ds == 128 || ds == 256) && in / ds <= kGramMaxHeads;
     f->rows_bytes = f->tc ? 0 : (size_t)f->groups * f->chunk * (in + dt) * fit_elt(f);
     const size_t rope_bytes = (size_t)(D.src.head_dim / 2 + D.dst.head_dim / 2) * sizeof(unsigned long long);
     cudaError_t ce;
@@ -872,24 +976,43 @@ extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv
     float* G = f->sums;
     float* C = f->sums + (size_t)f->groups * in * in;
     if (f->tc) {
+        const int ds = D.src.head_dim;
         GramLaunch L{};
         L.nrows = in + dt;
         L.mbs = in / 128;
-        L.units = f->groups * L.mbs;
         L.nkb = (tgt->total_tokens + kGramK - 1) / kGramK;
+        // units of 8..16 K-blocks when the call divides into them (the two row blocks of a unit
+        // then reread a few hundred KB from L2), else one unit per group and row block
+        L.kc = L.nkb;
+        for (int c = L.nkb < 16 ? L.nkb : 16; c >= 8; --c)
+            if (L.nkb % c == 0) { L.kc = c; break; }
+        L.nch = L.nkb / L.kc;
+        L.units = f->groups * L.nch * L.mbs;
         L.stage_bytes = (unsigned)L.nrows * 128;
-        L.stages = (int)((kSmemMax - 1024 - 256) / L.stage_bytes);
-        if (L.stages > kGramMaxStages) L.stages = kGramMaxStages;
-        L.n0 = L.nrows < 256 ? L.nrows : 256;
-        L.idesc0 = gram_idesc(L.n0);
-        L.idesc1 = L.nrows > L.n0 ? gram_idesc(L.nrows - L.n0) : 0u;
+        L.src_row = (unsigned)ds * 2 + 16;   // padded: lanes reading consecutive rows hit distinct banks
+        L.tgt_row = (unsigned)dt * 2 + 16;
+        const unsigned tail = 32 * 8 + (unsigned)(ds / 2 + dt / 2) * 8;   // barriers, flags, turns
+        bool fits = false;
+        for (int raw = 2; raw >= 1 && !fits; --raw)
+            for (int rcap = 128; rcap >= 64 && !fits; rcap -= 16) {
+                const unsigned rb = (unsigned)(kGramK * sizeof(GramTok) + 16 + (size_t)(in / ds) * rcap * L.src_row +
+                                               (size_t)kGramK * L.tgt_row + 15) / 16 * 16;
+                L.stages = 2;
+                L.raw_slots = raw;
+                L.rcap = rcap;
+                L.raw_bytes = rb;
+                L.off_raw = (unsigned)L.stages * L.stage_bytes;
+                L.off_bar = L.off_raw + (unsigned)raw * rb;
+                fits = 1024 + L.off_bar + tail <= (unsigned)kSmemMax;
+            }
+        if (!fits) return fit_fail(KVX_ERR_UNSUPPORTED, "fit_accumulate: Gram blocks do not fit shared memory");
         L.G = G;
         L.C = C;
-        const long long work = (long long)L.units * L.nkb;
+        const long long work = (long long)L.units * L.kc;
         const int grid = (int)(work < f->num_sms ? work : f->num_sms);
-        const size_t smem = 1024 + (size_t)L.stages * L.stage_bytes + 256;
+        const size_t smem = 1024 + (size_t)L.off_bar + tail;
         cudaError_t ce;
-        switch (D.src.head_dim) {
+        switch (ds) {
         case 64: ce = launch_gram_tc<64>(P, L, grid, smem, s); break;
         case 128: ce = launch_gram_tc<128>(P, L, grid, smem, s); break;
         default: ce = launch_gram_tc<256>(P, L, grid, smem, s); break;

@@ -277,10 +277,15 @@ __device__ __forceinline__ void rope_cs_vec(const unsigned long long* turns, int
 // DS: source head dim.  A is built one head-block (128 tokens x DS channels of one
 // source head) at a time into a ring of n_a head-block slots, so the MMA of one
 // head-block overlaps the build of the next.
-template <int DS>
+// MULTI: units carry several pieces (shared A); false compiles the one-piece path with a ring of
+// two accumulator slots and no piece loops.
+template <int DS, bool MULTI>
 __global__ void __launch_bounds__(kThreads, 1)
 translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_constant__ TcLaunch L)
 {
+    const int NP = MULTI ? L.np : 1;                       // pieces per unit
+    const uint32_t ND = MULTI ? (uint32_t)L.nd : 2u;       // accumulator slots
+    const int SPU = MULTI ? L.spu : 1;
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte aligned base, derived from smem_raw by pointer arithmetic so that the
     // compiler keeps every access below in the shared address space
@@ -308,7 +313,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             mbar_init(bar(kBarAFull + i), kNumXfWarps);
             mbar_init(bar(kBarAEmpty + i), 1);
         }
-        for (int i = 0; i < L.nd; ++i) {
+        for (uint32_t i = 0; i < ND; ++i) {
             mbar_init(bar(kBarDFull + i), 1);
             mbar_init(bar(kBarDEmpty + i), kNumEpiWarps);
         }
@@ -444,7 +449,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         }
     } else if (warp == kMmaWarp) {
         const bool b_stream = L.n_b > 1;
-        const uint32_t nb = (uint32_t)L.n_b, nd = (uint32_t)L.nd;
+        const uint32_t nb = (uint32_t)L.n_b, nd = ND;
         if (lane == 0) {
             // ------------------------------------------------------------ MMA issuer
             // Per unit and head-block q: one MMA per piece (head, output split) into the piece's
@@ -461,7 +466,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     ++b_cnt;
                     cur_g = x.g;
                 }
-                for (int p = 0; p < L.np && ok; ++p) {
+                for (int p = 0; p < NP && ok; ++p) {
                     const uint32_t c = pcount + (uint32_t)p;
                     if (!W.wait(bar(kBarDEmpty + c % nd), ((c / nd) & 1) ^ 1)) ok = false;
                 }
@@ -471,7 +476,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     if (!W.wait(bar(kBarAFull + sa), (a_cnt / (uint32_t)L.n_a) & 1)) { ok = false; break; }
                     tc_fence_after();
                     const uint32_t a0 = smem_u32(sA) + sa * L.hb_bytes;
-                    for (int p = 0; p < L.np; ++p) {
+                    for (int p = 0; p < NP; ++p) {
                         // resident: the image's K-blocks of head-block q; streamed: the piece in its slot
                         uint32_t b0 = smem_u32(sB), kb0 = (uint32_t)q * (DS / 64);
                         const uint32_t bs = b_cnt % nb;
@@ -499,8 +504,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                     ++a_cnt;
                 }
                 if (!ok) break;
-                for (int p = 0; p < L.np; ++p) umma_commit(bar(kBarDFull + (pcount + (uint32_t)p) % nd));
-                pcount += (uint32_t)L.np;
+                for (int p = 0; p < NP; ++p) umma_commit(bar(kBarDFull + (pcount + (uint32_t)p) % nd));
+                pcount += (uint32_t)NP;
                 if (!b_stream && wk.last_of_group()) umma_commit(bar(kBarBEmpty));
             }
             if (*sAbort) {   // MMAs whose results nobody waited for must finish before TMEM is freed
@@ -524,11 +529,11 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             for (wk.start(L, P.Ht); wk.more() && ok; wk.next()) {
                 const Unit& x = wk.x;
                 for (int q = 0; q < L.r_heads && ok; ++q)
-                    for (int p = 0; p < L.np; ++p) {
+                    for (int p = 0; p < NP; ++p) {
                         const uint32_t bs = b_loads % nb;
                         if (!W.wait(bar(kBarBEmpty + bs), ((b_loads / nb) & 1) ^ 1)) { ok = false; break; }
                         const uint8_t* img = (const uint8_t*)P.w +
-                                             (size_t)piece_group(x, p, L.spu, P.Ht, L.n_split) * L.b_bytes +
+                                             (size_t)piece_group(x, p, SPU, P.Ht, L.n_split) * L.b_bytes +
                                              (size_t)q * L.b_slot_bytes;
                         mbar_arrive_expect_tx(bar(kBarBFull + bs), L.b_slot_bytes);
                         bulk_g2s(smem_u32(sB) + bs * L.b_slot_bytes, img, L.b_slot_bytes, bar(kBarBFull + bs), pol_keep);
@@ -552,7 +557,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
         const int pc_begin = half * (hw >> 1), pc_end = pc_begin + (hw >> 1);
         uint8_t* srow = sStage + (size_t)m * L.stage_row_bytes;
         const uint32_t srow_u32 = smem_u32(srow);
-        const uint32_t nd = (uint32_t)L.nd;
+        const uint32_t nd = ND;
         uint32_t pcount = 0;
         bool ok = true;
         Walker wk;
@@ -565,8 +570,8 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
             int pt = 0;
             if (valid) resolve_dst(P, sv, tp, dst_off, pt);
             const bool rot = x.kv == 0 && P.rt.enabled;
-            for (int p = 0; p < L.np; ++p, ++pcount) {
-                const int hh = p / L.spu, nt = x.nt + (p - hh * L.spu);
+            for (int p = 0; p < NP; ++p, ++pcount) {
+                const int hh = p / SPU, nt = x.nt + (p - hh * SPU);
                 const uint32_t buf = pcount % nd;
                 float2 cs[8];
                 if (rot) rope_cs_vec<8>(sTurnT, pt, nt * hw + pc_begin, cs);
@@ -605,7 +610,7 @@ translate_tc_kernel(const __grid_constant__ TranslateParams P, const __grid_cons
                 if (!W.wait(bar(kBarPair + quad * 2 + 1), pcount & 1)) { ok = false; break; }
                 // the quadrant's rows: stored by the half-0 warp when a unit has one piece, split
                 // between the two warps by lane parity when it has several
-                if ((L.np > 1 ? (lane & 1) == half : half == 0) && valid && dst_off >= 0) {
+                if ((NP > 1 ? (lane & 1) == half : half == 0) && valid && dst_off >= 0) {
                     __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                          dst_head_off(P, x.h + hh);
                     if (P.plain_stores) {
@@ -970,14 +975,19 @@ static cudaError_t launch_pdl(K kernel, int grid, int threads, size_t smem, cuda
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-template <int DS>
+template <int DS, bool MULTI>
 static cudaError_t launch_span_ds(int grid, cudaStream_t stream, const TranslateParams& P, const TcLaunch& L)
 {
-    const cudaError_t e = smem_opt_in<translate_tc_kernel<DS>>(kSmemMax);
+    const cudaError_t e = smem_opt_in<translate_tc_kernel<DS, MULTI>>(kSmemMax);
     if (e != cudaSuccess) return e;
     // the B-loader warp (the last one) only when the weights stream
     const int threads = L.n_b > 1 ? kThreads : kThreads - 32;
-    return launch_pdl(translate_tc_kernel<DS>, grid, threads, kSmemMax, stream, P, L);
+    return launch_pdl(translate_tc_kernel<DS, MULTI>, grid, threads, kSmemMax, stream, P, L);
+}
+template <int DS>
+static cudaError_t launch_span(int grid, cudaStream_t stream, const TranslateParams& P, const TcLaunch& L)
+{
+    return L.np > 1 ? launch_span_ds<DS, true>(grid, stream, P, L) : launch_span_ds<DS, false>(grid, stream, P, L);
 }
 
 size_t tc_plan_bytes(int tokens)
@@ -1028,9 +1038,9 @@ cudaError_t launch_translate_tc(const TranslateParams& P, const TcConfig& cfg, i
         const int E = share_heads(P) / L.hpu;
         L.share = E > 1 && P.Ht % (E * L.hpu) == 0 && grid % E == 0 ? E : 1;
         switch (P.ds) {
-        case 256: e = launch_span_ds<256>(grid, stream, P, L); break;
-        case 128: e = launch_span_ds<128>(grid, stream, P, L); break;
-        default: e = launch_span_ds<64>(grid, stream, P, L); break;
+        case 256: e = launch_span<256>(grid, stream, P, L); break;
+        case 128: e = launch_span<128>(grid, stream, P, L); break;
+        default: e = launch_span<64>(grid, stream, P, L); break;
         }
         if (e != cudaSuccess) return e;
         ++*launches;

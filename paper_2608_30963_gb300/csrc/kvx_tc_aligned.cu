@@ -190,10 +190,9 @@ struct SlotPos {
     }
 };
 
-// HS: half head_dim of the source (32, 64 or 128).  NH: source heads in one A row when known at
-// compile time (the prologue's loop over them unrolls, so their shared-memory loads overlap), 0 =
-// from the parameters.
-template <int HS, int NH>
+// HS: half head_dim of the source (32, 64 or 128).  DIAG: the diagnostics of the bounded waits
+// (a wait bound other than ~1 s, a stalled producer) are compiled in.
+template <int HS, bool DIAG>
 __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const __grid_constant__ AlignedParams P)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -267,7 +266,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     tc_fence_after();
     const uint32_t tmem_base = *sTmemBase;
 
-    const Waiter W{sAbort, P.status, P.wait_ns ? P.wait_ns : kWaitNs};
+    const Waiter W{sAbort, P.status, DIAG && P.wait_ns ? P.wait_ns : kWaitNs};
     // Work split: each CTA takes an equal share of the K units and of the V units
     // (K units cost more: the source RoPE undo), K share first.  Within each share
     // units run group-major, so a group's weight tile stays resident.
@@ -296,7 +295,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
                 const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
-                if (blockIdx.x == 0 && ++nunit == P.stall_unit1) {
+                if (DIAG && blockIdx.x == 0 && ++nunit == P.stall_unit1) {
                     // diagnostics: a copy that never comes; the consumers' bounded waits run out
                     const unsigned long long t0 = globaltimer();
                     while (!*sAbort && globaltimer() - t0 < 4 * W.limit_ns) {}
@@ -513,7 +512,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         const int xt = threadIdx.x - kXfWarp0 * 32;
         const int row = (warp & 3) * 32 + lane;
         const int part = (warp - kXfWarp0) >> 2;          // 0 or 1
-        const int heads = NH > 0 ? NH : P.in_dim / (2 * HS);   // heads in one A row
+        const int heads = P.in_dim / (2 * HS);            // heads in one A row
         constexpr int kChunks = HS / 8;                    // 16-byte chunks per half head
         constexpr int kMine = kChunks / 2;                 // chunks per thread
         const uint32_t cs_lane = tmem_base + ((uint32_t)((warp & 3) * 32) << 16) + P.cs_col;
@@ -565,8 +564,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                     for (int e2 = 0; e2 < 8; ++e2) { v[2 * e2] = __float_as_uint(cs[e2].x); v[2 * e2 + 1] = __float_as_uint(cs[e2].y); }
                     tmem_st16(cs_lane + csbuf * (uint32_t)(2 * HS) + 2 * i, v);
                 }
-#pragma unroll
-                for (int q = 0; q < (NH > 0 ? NH : heads); ++q) {
+                for (int q = 0; q < heads; ++q) {
                     // element i (and i+HS) of head q: K-block and column within it
                     const int k_lo = q * 2 * HS + i, k_hi = k_lo + HS;
                     uint32_t s_lo = sp.idx + (k_lo >> 6), s_hi = sp.idx + (k_hi >> 6);
@@ -688,12 +686,12 @@ cudaError_t launch_pdl(K kernel, int grid, cudaStream_t stream, const AlignedPar
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-template <int HS, int NH>
+template <int HS, bool DIAG>
 static cudaError_t launch_aligned(int grid, cudaStream_t stream, const AlignedParams& P)
 {
-    const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<HS, NH>>(kSmemMax);
+    const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<HS, DIAG>>(kSmemMax);
     if (e != cudaSuccess) return e;
-    return launch_pdl(translate_tc_aligned_kernel<HS, NH>, grid, stream, P);
+    return launch_pdl(translate_tc_aligned_kernel<HS, DIAG>, grid, stream, P);
 }
 
 cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps,
@@ -757,12 +755,12 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     }
     const long long UH = (long long)(P.groups / 2) * P.m_tiles_max;
     const int grid = (int)(UH < num_sms ? UH : num_sms);
-    // the 7B -> 1.5B geometry (two 128-channel source heads per A row) has its own instantiation
-    const int heads = T.in_dim / T.ds;
+    // the diagnostics' instantiation only when they are asked for
+    const bool diag = P.wait_ns != 0 || P.stall_unit1 != 0;
     switch (T.ds) {
-    case 64: return launch_aligned<32, 0>(grid, stream, P);
-    case 128: return heads == 2 ? launch_aligned<64, 2>(grid, stream, P) : launch_aligned<64, 0>(grid, stream, P);
-    case 256: return launch_aligned<128, 0>(grid, stream, P);
+    case 64: return diag ? launch_aligned<32, true>(grid, stream, P) : launch_aligned<32, false>(grid, stream, P);
+    case 128: return diag ? launch_aligned<64, true>(grid, stream, P) : launch_aligned<64, false>(grid, stream, P);
+    case 256: return diag ? launch_aligned<128, true>(grid, stream, P) : launch_aligned<128, false>(grid, stream, P);
     default: return cudaErrorNotSupported;
     }
     return cudaGetLastError();
