@@ -950,7 +950,8 @@ extern "C" KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, do
 template <int DS>
 static cudaError_t launch_gram_tc(const TranslateParams& P, const GramLaunch& L, int grid, size_t smem, cudaStream_t s)
 {
-    const cudaError_t e = smem_opt_in<fit_gram_tc_kernel<DS>>((int)smem);
+    // the opt-in is set once per device, so at the largest size any launch asks for
+    const cudaError_t e = smem_opt_in<fit_gram_tc_kernel<DS>>(kSmemMax);
     if (e != cudaSuccess) return e;
     fit_gram_tc_kernel<DS><<<grid, kGramThreads, smem, s>>>(P, L);
     return cudaGetLastError();
