@@ -446,20 +446,36 @@ struct GramLaunch {
     unsigned src_row, tgt_row;   // padded row pitches of the staged source / target rows (bytes)
     unsigned raw_bytes;    // one raw slot: token table, header, source window, target rows
     unsigned off_raw, off_bar;
+    unsigned lbo, sbo;     // MN-major operand strides: between 64-channel blocks, between 8-token groups
     float* G;              // [groups][in][in]
     float* C;              // [groups][dt][in]
 };
 
+// Instruction descriptor: bf16 A and B, fp32 D, M = 128, N; both operands MN-major (bits 15, 16):
+// the block holds token rows with the channels contiguous, and the contraction runs over tokens.
 __host__ __device__ inline uint32_t gram_idesc_dev(int N)
 {
-    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(128 >> 4) << 24);
+    return (1u << 4) | (1u << 7) | (1u << 10) | (1u << 15) | (1u << 16) | ((uint32_t)(N >> 3) << 17) |
+           ((uint32_t)(128 >> 4) << 24);
+}
+// Shared-memory descriptor of an MN-major operand in 128-byte-swizzled atoms of 64 channels x 8
+// tokens: lbo between consecutive 64-channel blocks, sbo between consecutive 8-token groups.
+__device__ __forceinline__ uint64_t sw128_mn_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo)
+{
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
 }
 
-// Byte offset of the 4-byte word holding tokens (2 lw, 2 lw + 1) of row r in a K-major SW128
-// block of 64 tokens (rows 128 bytes apart within an 8-row atom of 1024 bytes).
-__device__ __forceinline__ uint32_t gram_word(int r, int lw)
+// Byte offset of the 16-byte chunk of channels [c, c + 8) (c a multiple of 8) of token i in a block:
+// 64-channel column blocks of 64 tokens x 128 bytes, 128-byte-swizzled in atoms of 8 tokens.
+__device__ __forceinline__ uint32_t gram_chunk(int i, int c)
 {
-    return (uint32_t)((r >> 3) * 1024 + (r & 7) * 128 + ((((lw >> 2) ^ (r & 7)) & 7) << 4) + (lw & 3) * 4);
+    return (uint32_t)((c >> 6) * (kGramK * 128) + (i >> 3) * 1024 + (i & 7) * 128 + ((((c >> 3) & 7) ^ (i & 7)) << 4));
 }
 
 // Unit u of the (g, chunk, mb) space and K-block index within the unit.
@@ -474,19 +490,13 @@ __device__ __forceinline__ GramUnit gram_unit(const GramLaunch& L, int w)
     return GramUnit{g, mb, ch * L.kc + kbi};
 }
 
-// Writes this lane's token (even or odd of a pair) into 8 rows of the block, exchanging with the
-// neighbouring lane so that each lane writes one word per row: the even lane rows r_lo + e, the odd
-// lane rows r_hi + e.
-__device__ __forceinline__ void gram_put(uint8_t* st, int r_lo, int r_hi, int lw, bool odd, const float (&lo)[8],
-                                         const float (&hi)[8])
+// Channels [c_lo, +8) and [c_hi, +8) of token i, rounded to bf16, into the block.
+__device__ __forceinline__ void gram_put(uint8_t* st, int i, int c_lo, int c_hi, const float (&lo)[8], const float (&hi)[8])
 {
-#pragma unroll
-    for (int e = 0; e < 8; ++e) {
-        const float send = odd ? lo[e] : hi[e];
-        const float got = __shfl_xor_sync(0xffffffffu, send, 1);
-        if (!odd) *reinterpret_cast<uint32_t*>(st + gram_word(r_lo + e, lw)) = pack_bf16(lo[e], got);
-        else *reinterpret_cast<uint32_t*>(st + gram_word(r_hi + e, lw)) = pack_bf16(got, hi[e]);
-    }
+    *reinterpret_cast<uint4*>(st + gram_chunk(i, c_lo)) =
+        make_uint4(pack_bf16(lo[0], lo[1]), pack_bf16(lo[2], lo[3]), pack_bf16(lo[4], lo[5]), pack_bf16(lo[6], lo[7]));
+    *reinterpret_cast<uint4*>(st + gram_chunk(i, c_hi)) =
+        make_uint4(pack_bf16(hi[0], hi[1]), pack_bf16(hi[2], hi[3]), pack_bf16(hi[4], hi[5]), pack_bf16(hi[6], hi[7]));
 }
 
 template <int DS>
@@ -560,18 +570,21 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                 if (!W.wait(bar(bZFull + s), ph)) break;
                 tc_fence_after();
                 const uint32_t st = smem_u32(smem) + s * L.stage_bytes;
-                const uint32_t a0 = st + (uint32_t)x.mb * (128 / 8) * 1024;
+                const uint32_t colblk = kGramK * 128;            // one 64-channel column block
+                const uint32_t a0 = st + (uint32_t)(x.mb * 2) * colblk;
                 const int nx = (x.mb + 1) * 128;   // X columns of the lower triangle
 #pragma unroll
-                for (int k = 0; k < kGramK / 16; ++k) {
+                for (int k = 0; k < kGramK / 16; ++k) {   // 16 tokens = two 8-token atom rows
                     const uint32_t acc = (first && k == 0) ? 0u : 1u;
-                    const uint64_t ad = sw128_desc(a0 + k * 32);
+                    const uint64_t ad = sw128_mn_desc(a0 + k * 2048, L.lbo, L.sbo);
                     for (int c0 = 0; c0 < nx; c0 += 256) {   // X columns in pieces of <= 256
                         const int n = nx - c0 < 256 ? nx - c0 : 256;
-                        umma_bf16(tmem_base + (uint32_t)c0, ad, sw128_desc(st + (uint32_t)(c0 / 8) * 1024 + k * 32),
+                        umma_bf16(tmem_base + (uint32_t)c0, ad,
+                                  sw128_mn_desc(st + (uint32_t)(c0 / 64) * colblk + k * 2048, L.lbo, L.sbo),
                                   gram_idesc_dev(n), acc);
                     }
-                    umma_bf16(tmem_base + (uint32_t)nx, ad, sw128_desc(st + (uint32_t)(in / 8) * 1024 + k * 32),
+                    umma_bf16(tmem_base + (uint32_t)nx, ad,
+                              sw128_mn_desc(st + (uint32_t)(in / 64) * colblk + k * 2048, L.lbo, L.sbo),
                               gram_idesc_dev(dt), acc);
                 }
                 umma_commit(bar(bZEmpty + s));
@@ -697,7 +710,6 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
         const int cpt = dt / 16;                     // chunk pairs of a target row
         const unsigned long long* sTurnS = sTurn;
         const unsigned long long* sTurnT = sTurn + (P.ds >> 1);
-        const bool odd = lane & 1;
         uint32_t it = 0;
         for (int w = w0; w < w1; ++w, ++it) {
             const GramUnit x = gram_unit(L, w);
@@ -717,7 +729,6 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
             for (int pc = xw; pc < pieces; pc += kGramNumXf) {
                 const int half = pc & 1, item = pc >> 1;
                 const int i = half * 32 + lane;               // this lane's token
-                const int lw = i >> 1;
                 const GramTok tk = tt[i];
                 if (item < CPH) {
                     // X: chunk pair `item` of every needed source head, span mean of un-rotated rows
@@ -780,7 +791,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
 #pragma unroll
                     for (int q = 0; q < kGramMaxHeads; ++q) {
                         if (q >= nh) break;
-                        gram_put(st, q * DS + c_lo, q * DS + c_hi, lw, odd, a0[q], a1[q]);
+                        gram_put(st, i, q * DS + c_lo, q * DS + c_hi, a0[q], a1[q]);
                     }
                 } else {
                     // Y: chunk pair of the target row, target RoPE undone for K
@@ -811,7 +822,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
 #pragma unroll
                         for (int e = 0; e < 8; ++e) { y0[e] = 0.f; y1[e] = 0.f; }
                     }
-                    gram_put(st, in + c_lo, in + c_hi, lw, odd, y0, y1);
+                    gram_put(st, i, in + c_lo, in + c_hi, y0, y1);
                 }
             }
             fence_proxy_async();
@@ -1007,6 +1018,8 @@ extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv
                 fits = 1024 + L.off_bar + tail <= (unsigned)kSmemMax;
             }
         if (!fits) return fit_fail(KVX_ERR_UNSUPPORTED, "fit_accumulate: Gram blocks do not fit shared memory");
+        L.lbo = kGramK * 128;   // next 64-channel column block
+        L.sbo = 1024;           // next 8-token atom row
         L.G = G;
         L.C = C;
         const long long work = (long long)L.units * L.kc;
