@@ -417,13 +417,13 @@ constexpr int kGramMmaWarp = 0;
 constexpr int kGramEpiWarp0 = 1;
 constexpr int kGramNumEpi = 4;
 constexpr int kGramXfWarp0 = kGramEpiWarp0 + kGramNumEpi;
-constexpr int kGramNumXf = 8;
+constexpr int kGramNumXf = 12;
 constexpr int kGramLoadWarp = kGramXfWarp0 + kGramNumXf;
 constexpr int kGramThreads = (kGramLoadWarp + 1) * 32;
 constexpr int kGramMaxStages = 4;
 constexpr int kGramMaxRaw = 2;
 constexpr int kGramMaxRows = 512;   // in + dt: one 128 x 512 fp32 accumulator fills TMEM
-constexpr int kGramMaxHeads = 4;    // source head-blocks in one input row
+constexpr int kGramMaxHeads = 6;    // source head-blocks in one input row
 
 struct GramTok {
     int b, lo, hi, pt;       // sequence, clamped source span, target position
@@ -499,7 +499,8 @@ __device__ __forceinline__ void gram_put(uint8_t* st, int i, int c_lo, int c_hi,
         make_uint4(pack_bf16(hi[0], hi[1]), pack_bf16(hi[2], hi[3]), pack_bf16(hi[4], hi[5]), pack_bf16(hi[6], hi[7]));
 }
 
-template <int DS>
+// DS: source head dim; NHD: source head-blocks in one input row (in / DS).
+template <int DS, int NHD>
 __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __grid_constant__ TranslateParams P,
                                                                       const __grid_constant__ GramLaunch L)
 {
@@ -546,8 +547,8 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
     const long long total = (long long)L.units * L.kc;
     const int w0 = (int)((long long)blockIdx.x * total / gridDim.x);
     const int w1 = (int)((long long)(blockIdx.x + 1) * total / gridDim.x);
-    const int in = P.in_dim, dt = P.dt;
-    const int heads = in / DS;
+    const int in = NHD * DS, dt = P.dt;
+    constexpr int heads = NHD;
     auto tok_tab = [&](int r) { return reinterpret_cast<GramTok*>(sRaw + (size_t)r * L.raw_bytes); };
     auto win_hdr = [&](int r) { return reinterpret_cast<int*>(sRaw + (size_t)r * L.raw_bytes + kGramK * sizeof(GramTok)); };
     auto src_rows = [&](int r, int q) {
@@ -736,9 +737,9 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                     int c_lo, c_hi;
                     pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
                     const bool rot = rot_s && cp * 8 < P.rhalf_s;
-                    float a0[kGramMaxHeads][8], a1[kGramMaxHeads][8];
+                    float a0[NHD][8], a1[NHD][8];
 #pragma unroll
-                    for (int q = 0; q < kGramMaxHeads; ++q)
+                    for (int q = 0; q < NHD; ++q)
 #pragma unroll
                         for (int e = 0; e < 8; ++e) { a0[q][e] = 0.f; a1[q][e] = 0.f; }
                     if (tk.ok) {
@@ -751,7 +752,7 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                                 for (int e = 0; e < 8; ++e) cs[e] = turn_cs(sTurnS[cp * 8 + e], pos);
                             }
 #pragma unroll
-                            for (int q = 0; q < kGramMaxHeads; ++q) {
+                            for (int q = 0; q < NHD; ++q) {
                                 if (q >= nh) break;
                                 uint4 w0v, w1v;
                                 if (inwin) {
@@ -784,12 +785,12 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                         }
                         const float inv = 1.f / (float)(tk.hi - tk.lo);
 #pragma unroll
-                        for (int q = 0; q < kGramMaxHeads; ++q)
+                        for (int q = 0; q < NHD; ++q)
 #pragma unroll
                             for (int e = 0; e < 8; ++e) { a0[q][e] *= inv; a1[q][e] *= inv; }
                     }
 #pragma unroll
-                    for (int q = 0; q < kGramMaxHeads; ++q) {
+                    for (int q = 0; q < NHD; ++q) {
                         if (q >= nh) break;
                         gram_put(st, i, q * DS + c_lo, q * DS + c_hi, a0[q], a1[q]);
                     }
@@ -958,13 +959,13 @@ extern "C" KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, do
     return KVX_OK;
 }
 
-template <int DS>
+template <int DS, int NHD>
 static cudaError_t launch_gram_tc(const TranslateParams& P, const GramLaunch& L, int grid, size_t smem, cudaStream_t s)
 {
     // the opt-in is set once per device, so at the largest size any launch asks for
-    const cudaError_t e = smem_opt_in<fit_gram_tc_kernel<DS>>(kSmemMax);
+    const cudaError_t e = smem_opt_in<fit_gram_tc_kernel<DS, NHD>>(kSmemMax);
     if (e != cudaSuccess) return e;
-    fit_gram_tc_kernel<DS><<<grid, kGramThreads, smem, s>>>(P, L);
+    fit_gram_tc_kernel<DS, NHD><<<grid, kGramThreads, smem, s>>>(P, L);
     return cudaGetLastError();
 }
 
@@ -993,11 +994,7 @@ extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv
         L.nrows = in + dt;
         L.mbs = in / 128;
         L.nkb = (tgt->total_tokens + kGramK - 1) / kGramK;
-        // units of 8..16 K-blocks when the call divides into them (the two row blocks of a unit
-        // then reread a few hundred KB from L2), else one unit per group and row block
-        L.kc = L.nkb;
-        for (int c = L.nkb < 16 ? L.nkb : 16; c >= 8; --c)
-            if (L.nkb % c == 0) { L.kc = c; break; }
+        L.kc = L.nkb;   // one unit per (group, row block): one accumulator flush each
         L.nch = L.nkb / L.kc;
         L.units = f->groups * L.nch * L.mbs;
         L.stage_bytes = (unsigned)L.nrows * 128;
@@ -1026,10 +1023,16 @@ extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv
         const int grid = (int)(work < f->num_sms ? work : f->num_sms);
         const size_t smem = 1024 + (size_t)L.off_bar + tail;
         cudaError_t ce;
-        switch (ds) {
-        case 64: ce = launch_gram_tc<64>(P, L, grid, smem, s); break;
-        case 128: ce = launch_gram_tc<128>(P, L, grid, smem, s); break;
-        default: ce = launch_gram_tc<256>(P, L, grid, smem, s); break;
+        // in = NHD * ds with in a multiple of 128 and in + dt <= 512
+        switch (ds * 8 + in / ds) {
+        case 64 * 8 + 2: ce = launch_gram_tc<64, 2>(P, L, grid, smem, s); break;
+        case 64 * 8 + 4: ce = launch_gram_tc<64, 4>(P, L, grid, smem, s); break;
+        case 64 * 8 + 6: ce = launch_gram_tc<64, 6>(P, L, grid, smem, s); break;
+        case 128 * 8 + 1: ce = launch_gram_tc<128, 1>(P, L, grid, smem, s); break;
+        case 128 * 8 + 2: ce = launch_gram_tc<128, 2>(P, L, grid, smem, s); break;
+        case 128 * 8 + 3: ce = launch_gram_tc<128, 3>(P, L, grid, smem, s); break;
+        case 256 * 8 + 1: ce = launch_gram_tc<256, 1>(P, L, grid, smem, s); break;
+        default: return fit_fail(KVX_ERR_UNSUPPORTED, "fit_accumulate: no Gram kernel for in %d, d_s %d", in, ds);
         }
         if (ce != cudaSuccess) return fit_fail(KVX_ERR_CUDA, "fit_accumulate: %s", cudaGetErrorString(ce));
         f->tokens += tgt->total_tokens;
