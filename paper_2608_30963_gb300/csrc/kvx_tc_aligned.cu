@@ -190,9 +190,10 @@ struct SlotPos {
     }
 };
 
-// HS: half head_dim of the source (32, 64 or 128).  DIAG: the diagnostics of the bounded waits
-// (a wait bound other than ~1 s, a stalled producer) are compiled in.
-template <int HS, bool DIAG>
+// HS: half head_dim of the source (32, 64 or 128).  VAR: 0 = the normal kernel; 1 = with the
+// diagnostics of the bounded waits (a wait bound other than ~1 s, a stalled producer); 2 = target
+// rows written with thread stores (a target cache on another device).
+template <int HS, int VAR>
 __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const __grid_constant__ AlignedParams P)
 {
     extern __shared__ __align__(1024) uint8_t smem_raw[];
@@ -266,6 +267,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     tc_fence_after();
     const uint32_t tmem_base = *sTmemBase;
 
+    constexpr bool DIAG = VAR == 1, PLAIN = VAR == 2;
     const Waiter W{sAbort, P.status, DIAG && P.wait_ns ? P.wait_ns : kWaitNs};
     // Work split: each CTA takes an equal share of the K units and of the V units
     // (K units cost more: the source RoPE undo), K share first.  Within each share
@@ -489,7 +491,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             if ((lane & 1) == half && valid && dst_off >= 0) {   // the quadrant's rows, split between its two warps
                 __nv_bfloat16* dst = (__nv_bfloat16*)(x.kv ? P.dst_v[x.j] : P.dst_k[x.j]) + dst_off +
                                      (P.paged ? (long long)x.h * P.dt : (long long)x.h * P.dh);
-                if (P.plain_stores) {
+                if (PLAIN) {
                     store_row_slots_plain(dst, srow, x.nt * hw, hw, P.dt >> 1, P.dt >> 1);
                 } else if (P.n_split == 1) {
                     bulk_s2g(dst, srow_u32, (uint32_t)P.dt * 2);
@@ -497,7 +499,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
                     bulk_s2g(dst + x.nt * hw, srow_u32, (uint32_t)hw * 2);
                     bulk_s2g(dst + (P.dt >> 1) + x.nt * hw, srow_u32 + hw * 2, (uint32_t)hw * 2);
                 }
-                if (!P.plain_stores) bulk_commit();
+                if (!PLAIN) bulk_commit();
             }
             ++tcount;
         }
@@ -686,12 +688,12 @@ cudaError_t launch_pdl(K kernel, int grid, cudaStream_t stream, const AlignedPar
     return e != cudaSuccess ? e : cudaGetLastError();
 }
 
-template <int HS, bool DIAG>
+template <int HS, int VAR>
 static cudaError_t launch_aligned(int grid, cudaStream_t stream, const AlignedParams& P)
 {
-    const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<HS, DIAG>>(kSmemMax);
+    const cudaError_t e = smem_opt_in<translate_tc_aligned_kernel<HS, VAR>>(kSmemMax);
     if (e != cudaSuccess) return e;
-    return launch_pdl(translate_tc_aligned_kernel<HS, DIAG>, grid, stream, P);
+    return launch_pdl(translate_tc_aligned_kernel<HS, VAR>, grid, stream, P);
 }
 
 cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* const* maps,
@@ -755,12 +757,18 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     }
     const long long UH = (long long)(P.groups / 2) * P.m_tiles_max;
     const int grid = (int)(UH < num_sms ? UH : num_sms);
-    // the diagnostics' instantiation only when they are asked for
-    const bool diag = P.wait_ns != 0 || P.stall_unit1 != 0;
-    switch (T.ds) {
-    case 64: return diag ? launch_aligned<32, true>(grid, stream, P) : launch_aligned<32, false>(grid, stream, P);
-    case 128: return diag ? launch_aligned<64, true>(grid, stream, P) : launch_aligned<64, false>(grid, stream, P);
-    case 256: return diag ? launch_aligned<128, true>(grid, stream, P) : launch_aligned<128, false>(grid, stream, P);
+    // the diagnostics' and the thread-store instantiations only when they are asked for
+    const int var = P.plain_stores ? 2 : (P.wait_ns != 0 || P.stall_unit1 != 0 ? 1 : 0);
+    switch (T.ds * 4 + var) {
+    case 64 * 4 + 0: return launch_aligned<32, 0>(grid, stream, P);
+    case 64 * 4 + 1: return launch_aligned<32, 1>(grid, stream, P);
+    case 64 * 4 + 2: return launch_aligned<32, 2>(grid, stream, P);
+    case 128 * 4 + 0: return launch_aligned<64, 0>(grid, stream, P);
+    case 128 * 4 + 1: return launch_aligned<64, 1>(grid, stream, P);
+    case 128 * 4 + 2: return launch_aligned<64, 2>(grid, stream, P);
+    case 256 * 4 + 0: return launch_aligned<128, 0>(grid, stream, P);
+    case 256 * 4 + 1: return launch_aligned<128, 1>(grid, stream, P);
+    case 256 * 4 + 2: return launch_aligned<128, 2>(grid, stream, P);
     default: return cudaErrorNotSupported;
     }
     return cudaGetLastError();
