@@ -678,23 +678,40 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
             const uint32_t bytes = (uint32_t)R * (uint32_t)DS * 2u * (uint32_t)heads + (uint32_t)n_tgt * (uint32_t)dt * 2u;
             if (lane == 0) mbar_arrive_expect_tx(bar(bRFull + r), bytes);
             __syncwarp();
+            // source window: one copy per head-block when the rows are contiguous, else one per row
             for (int q = 0; q < heads; ++q) {
                 int slot, gs;
                 head_block(P, j, h, q, slot, gs);
                 const __nv_bfloat16* base = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) +
                                             (long long)b0 * P.sb + (long long)gs * P.sh;
                 uint8_t* dstq = src_rows((int)r, q);
-                for (int rr = lane; rr < R; rr += 32)
-                    bulk_g2s(smem_u32(dstq + (size_t)rr * L.src_row), base + (long long)(c0 + rr) * P.ss, DS * 2,
-                             bar(bRFull + r), pol);
+                if (P.ss == DS) {
+                    if (lane == 0 && R > 0)
+                        bulk_g2s(smem_u32(dstq), base + (long long)c0 * P.ss, (uint32_t)R * DS * 2, bar(bRFull + r), pol);
+                } else {
+                    for (int rr = lane; rr < R; rr += 32)
+                        bulk_g2s(smem_u32(dstq + (size_t)rr * L.src_row), base + (long long)(c0 + rr) * P.ss, DS * 2,
+                                 bar(bRFull + r), pol);
+                }
             }
+            // target rows: one copy when the 64 rows are consecutive in a contiguous cache, else one per token
             const __nv_bfloat16* tgt = (const __nv_bfloat16*)(kv ? P.dst_v[j] : P.dst_k[j]);
             const long long hoff = dst_head_off(P, h);
+            const long long off0 = __shfl_sync(0xffffffffu, tk[0].dst_off, 0);
+            const bool run = __all_sync(0xffffffffu, tk[0].ok && tk[1].ok && tk[0].b == b0 && tk[1].b == b0 &&
+                                                         tk[0].dst_off == off0 + (long long)lane * P.dts &&
+                                                         tk[1].dst_off == off0 + (long long)(lane + 32) * P.dts) &&
+                             !P.paged && P.dts == dt;
+            if (run) {
+                if (lane == 0)
+                    bulk_g2s(smem_u32(tgt_rows((int)r)), tgt + off0 + hoff, (uint32_t)kGramK * dt * 2u, bar(bRFull + r), pol);
+            } else {
 #pragma unroll
-            for (int u = 0; u < 2; ++u)
-                if (tk[u].ok)
-                    bulk_g2s(smem_u32(tgt_rows((int)r) + (size_t)(lane + 32 * u) * L.tgt_row), tgt + tk[u].dst_off + hoff,
-                             (uint32_t)dt * 2u, bar(bRFull + r), pol);
+                for (int u = 0; u < 2; ++u)
+                    if (tk[u].ok)
+                        bulk_g2s(smem_u32(tgt_rows((int)r) + (size_t)(lane + 32 * u) * L.tgt_row),
+                                 tgt + tk[u].dst_off + hoff, (uint32_t)dt * 2u, bar(bRFull + r), pol);
+            }
             ++issued;
         }
         if (*sAbort) {   // let the copies in flight land before the CTA leaves
@@ -704,11 +721,16 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                 while (!mbar_try_wait(bar(bRFull + c % ns), (c / ns) & 1) && globaltimer() - t0 < kWaitNs) {}
         }
     } else {
-        // ------------------------------------------------------------ prologue: Z^T blocks in shared memory
+        // ------------------------------------------------------------ prologue: token-row blocks in shared memory
+        // A pass covers a few tokens of the block with the lanes across 16-channel chunk pairs
+        // (LX lanes per token for the source head, LY for the target row), so a warp reads whole
+        // 128-byte segments of the staged rows and writes whole swizzled rows of the block.
         constexpr int HS = DS / 2;
         constexpr int CPH = DS / 16;                 // chunk pairs (16 channels) per source head
+        constexpr int LX = CPH < 32 ? CPH : 32;      // lanes per token, X
         const int xw = warp - kGramXfWarp0;
         const int cpt = dt / 16;                     // chunk pairs of a target row
+        const int LY = cpt < 32 ? cpt : 32;          // lanes per token, Y
         const unsigned long long* sTurnS = sTurn;
         const unsigned long long* sTurnT = sTurn + (P.ds >> 1);
         uint32_t it = 0;
@@ -726,14 +748,12 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
             const int* hd = win_hdr((int)r);
             const int b0 = hd[0], c0 = hd[1], R = hd[2];
             const bool rot_s = kv == 0 && P.rs.enabled, rot_t = kv == 0 && P.rt.enabled;
-            const int pieces = (CPH + cpt) * 2;
-            for (int pc = xw; pc < pieces; pc += kGramNumXf) {
-                const int half = pc & 1, item = pc >> 1;
-                const int i = half * 32 + lane;               // this lane's token
-                const GramTok tk = tt[i];
-                if (item < CPH) {
-                    // X: chunk pair `item` of every needed source head, span mean of un-rotated rows
-                    const int cp = item;
+            const int xpass = kGramK * LX / 32, ypass = kGramK * LY / 32;
+            for (int pc = xw; pc < xpass + ypass; pc += kGramNumXf) {
+                if (pc < xpass) {
+                    // X: chunk pair cp of every needed source head, span mean of un-rotated rows
+                    const int i = pc * (32 / LX) + lane / LX, cp = lane % LX;
+                    const GramTok tk = tt[i];
                     int c_lo, c_hi;
                     pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
                     const bool rot = rot_s && cp * 8 < P.rhalf_s;
@@ -795,8 +815,10 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                         gram_put(st, i, q * DS + c_lo, q * DS + c_hi, a0[q], a1[q]);
                     }
                 } else {
-                    // Y: chunk pair of the target row, target RoPE undone for K
-                    const int cp = item - CPH;
+                    // Y: chunk pair cp of the target row, target RoPE undone for K
+                    const int yp = pc - xpass;
+                    const int i = yp * (32 / LY) + lane / LY, cp = lane % LY;
+                    const GramTok tk = tt[i];
                     int c_lo, c_hi;
                     pair_channels(cp * 8, dt >> 1, P.rhalf_t, c_lo, c_hi);
                     const bool rot = rot_t && cp * 8 < P.rhalf_t;
@@ -998,8 +1020,8 @@ extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv
         L.nch = L.nkb / L.kc;
         L.units = f->groups * L.nch * L.mbs;
         L.stage_bytes = (unsigned)L.nrows * 128;
-        L.src_row = (unsigned)ds * 2 + 16;   // padded: lanes reading consecutive rows hit distinct banks
-        L.tgt_row = (unsigned)dt * 2 + 16;
+        L.src_row = (unsigned)ds * 2;   // rows as in the caches: whole windows move in one copy
+        L.tgt_row = (unsigned)dt * 2;
         const unsigned tail = 32 * 8 + (unsigned)(ds / 2 + dt / 2) * 8;   // barriers, flags, turns
         bool fits = false;
         for (int raw = 2; raw >= 1 && !fits; --raw)
