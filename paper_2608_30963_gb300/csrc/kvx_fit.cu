@@ -421,7 +421,10 @@ constexpr int kGramNumXf = 12;
 constexpr int kGramLoadWarp = kGramXfWarp0 + kGramNumXf;
 constexpr int kGramThreads = (kGramLoadWarp + 1) * 32;
 constexpr int kGramMaxStages = 4;
-constexpr int kGramMaxRaw = 2;
+constexpr int kGramMaxRaw = 8;
+// Direct blocks (every span one source row): the prologue warps work in teams, one 64-token block each.
+constexpr int kGramTeams = 4;
+constexpr int kGramTeamWarps = kGramNumXf / kGramTeams;
 constexpr int kGramMaxRows = 512;   // in + dt: one 128 x 512 fp32 accumulator fills TMEM
 constexpr int kGramMaxHeads = 6;    // source head-blocks in one input row
 
@@ -429,7 +432,7 @@ struct GramTok {
     int b, lo, hi, pt;       // sequence, clamped source span, target position
     long long dst_off;       // target row offset (head 0), -1: none
     int ok;                  // contributes (a valid row with a span)
-    int pad;
+    int ps;                  // direct blocks: source position of the span's row
 };
 
 struct GramLaunch {
@@ -499,8 +502,29 @@ __device__ __forceinline__ void gram_put(uint8_t* st, int i, int c_lo, int c_hi,
         make_uint4(pack_bf16(hi[0], hi[1]), pack_bf16(hi[2], hi[3]), pack_bf16(hi[4], hi[5]), pack_bf16(hi[6], hi[7]));
 }
 
-// DS: source head dim; NHD: source head-blocks in one input row (in / DS).
-template <int DS, int NHD>
+// Rotates the 8 channel pairs of the chunks at lo and hi of a block in place by R(-theta).
+__device__ __forceinline__ void gram_unrotate(uint8_t* lo, uint8_t* hi, const float2 (&cs)[8])
+{
+    const uint4 a = *reinterpret_cast<const uint4*>(lo), b = *reinterpret_cast<const uint4*>(hi);
+    const uint32_t va[4] = {a.x, a.y, a.z, a.w}, vb[4] = {b.x, b.y, b.z, b.w};
+    float y0[8], y1[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        const float u0 = (e & 1) ? bf_hi(va[e >> 1]) : bf_lo(va[e >> 1]);
+        const float u1 = (e & 1) ? bf_hi(vb[e >> 1]) : bf_lo(vb[e >> 1]);
+        y0[e] = fmaf(u0, cs[e].x, u1 * cs[e].y);
+        y1[e] = fmaf(u1, cs[e].x, -u0 * cs[e].y);
+    }
+    *reinterpret_cast<uint4*>(lo) =
+        make_uint4(pack_bf16(y0[0], y0[1]), pack_bf16(y0[2], y0[3]), pack_bf16(y0[4], y0[5]), pack_bf16(y0[6], y0[7]));
+    *reinterpret_cast<uint4*>(hi) =
+        make_uint4(pack_bf16(y1[0], y1[1]), pack_bf16(y1[2], y1[3]), pack_bf16(y1[4], y1[5]), pack_bf16(y1[6], y1[7]));
+}
+
+// DS: source head dim; NHD: source head-blocks in one input row (in / DS).  DIRECT: identity
+// alignment (every span one source row): the loader writes token tables only, and the prologue
+// teams gather the rows with 16-byte asynchronous copies straight into the block.
+template <int DS, int NHD, bool DIRECT>
 __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __grid_constant__ TranslateParams P,
                                                                       const __grid_constant__ GramLaunch L)
 {
@@ -520,12 +544,12 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
     if (threadIdx.x == 0) {
         *sAbort = 0;
         for (int i = 0; i < L.stages; ++i) {
-            mbar_init(bar(bZFull + i), kGramNumXf);
+            mbar_init(bar(bZFull + i), DIRECT ? kGramTeamWarps : kGramNumXf);
             mbar_init(bar(bZEmpty + i), 1);
         }
         for (int i = 0; i < L.raw_slots; ++i) {
             mbar_init(bar(bRFull + i), 1);
-            mbar_init(bar(bREmpty + i), kGramNumXf);
+            mbar_init(bar(bREmpty + i), DIRECT ? kGramTeamWarps : kGramNumXf);
         }
         mbar_init(bar(bDFull), 1);
         mbar_init(bar(bDEmpty), kGramNumEpi);
@@ -654,9 +678,16 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                 tk[u] = GramTok{0, 0, 0, 0, -1, 0, 0};
                 if (tp < P.T_total) {
                     const TokenInfo ti = resolve_token(P, tp);
-                    tk[u] = GramTok{ti.b, ti.lo, ti.hi, ti.pt, ti.dst_off, ti.dst_off >= 0 && ti.hi > ti.lo, 0};
+                    const bool ok = ti.dst_off >= 0 && ti.hi > ti.lo;
+                    const int ps = DIRECT && ok && kv == 0 && P.rs.enabled ? src_pos_of(P, ti.b, ti.lo) : 0;
+                    tk[u] = GramTok{ti.b, ti.lo, ti.hi, ti.pt, ti.dst_off, ok, ps};
                 }
                 tt[i] = tk[u];
+            }
+            if (DIRECT) {   // the prologue gathers the rows itself
+                __syncwarp();
+                if (lane == 0) mbar_arrive(bar(bRFull + r));
+                continue;
             }
             // the window: from the first token's span start, within its sequence, up to rcap rows
             const int b0 = __shfl_sync(0xffffffffu, tk[0].b, 0), c0 = __shfl_sync(0xffffffffu, tk[0].lo, 0);
@@ -719,6 +750,114 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
             const uint32_t ns = (uint32_t)L.raw_slots;
             for (uint32_t c = issued > ns ? issued - ns : 0; c < issued; ++c)
                 while (!mbar_try_wait(bar(bRFull + c % ns), (c / ns) & 1) && globaltimer() - t0 < kWaitNs) {}
+        }
+    } else if (DIRECT) {
+        // ------------------------------------------------------------ prologue, direct blocks
+        // Team `team` of kGramTeamWarps warps takes every kGramTeams-th block.  A thread owns items
+        // (token i, chunk pair cp): it copies the pair's two 16-byte chunks of every needed source
+        // head and of the target row into their swizzled places, waits for its own copies, and for
+        // K un-rotates them in place, with one (cos, sin) per pair for the source heads and, when the
+        // two rotations and positions coincide, for the target row as well.
+        constexpr int HS = DS / 2;
+        constexpr int CPH = DS / 16;
+        const int xw = warp - kGramXfWarp0, team = xw / kGramTeamWarps, tw = xw - team * kGramTeamWarps;
+        const int cpt = dt / 16, CPM = CPH > cpt ? CPH : cpt;
+        const unsigned long long* sTurnS = sTurn;
+        const unsigned long long* sTurnT = sTurn + (P.ds >> 1);
+        uint32_t it = (uint32_t)team;
+        for (int w = w0 + team; w < w1; w += kGramTeams, it += kGramTeams) {
+            const GramUnit x = gram_unit(L, w);
+            const int kv = x.g & 1, jh = x.g >> 1, h = jh % P.Ht, j = jh / P.Ht;
+            const int nh = min(heads, ((x.mb + 1) * 128 + DS - 1) / DS);
+            const uint32_t s = it % (uint32_t)L.stages, ph = (it / (uint32_t)L.stages) & 1;
+            const uint32_t r = it % (uint32_t)L.raw_slots, rph = (it / (uint32_t)L.raw_slots) & 1;
+            if (!W.wait(bar(bZEmpty + s), ph ^ 1)) break;
+            if (!W.wait(bar(bRFull + r), rph)) break;
+            uint8_t* st = smem + (size_t)s * L.stage_bytes;
+            const uint32_t st32 = smem_u32(st);
+            const GramTok* tt = tok_tab((int)r);
+            const __nv_bfloat16* hb[NHD];
+#pragma unroll
+            for (int q = 0; q < NHD; ++q) {
+                int slot, gs;
+                head_block(P, j, h, q, slot, gs);
+                hb[q] = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) + (long long)gs * P.sh;
+            }
+            const __nv_bfloat16* tgt = (const __nv_bfloat16*)(kv ? P.dst_v[j] : P.dst_k[j]) + dst_head_off(P, h);
+            const int nitems = kGramK * CPM;
+            const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
+            for (int item = tw * 32 + lane; item < nitems; item += kGramTeamWarps * 32) {
+                const int i = item / CPM, cp = item - i * CPM;
+                const GramTok tk = tt[i];
+                if (cp < CPH) {
+                    int c_lo, c_hi;
+                    pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
+#pragma unroll
+                    for (int q = 0; q < NHD; ++q) {
+                        if (q >= nh) break;
+                        const uint32_t d_lo = gram_chunk(i, q * DS + c_lo), d_hi = gram_chunk(i, q * DS + c_hi);
+                        if (tk.ok) {
+                            const __nv_bfloat16* src = hb[q] + (long long)tk.b * P.sb + (long long)tk.lo * P.ss;
+                            cp_async16(st32 + d_lo, src + c_lo);
+                            cp_async16(st32 + d_hi, src + c_hi);
+                        } else {
+                            *reinterpret_cast<uint4*>(st + d_lo) = zero;
+                            *reinterpret_cast<uint4*>(st + d_hi) = zero;
+                        }
+                    }
+                }
+                if (cp < cpt) {
+                    int c_lo, c_hi;
+                    pair_channels(cp * 8, dt >> 1, P.rhalf_t, c_lo, c_hi);
+                    const uint32_t d_lo = gram_chunk(i, in + c_lo), d_hi = gram_chunk(i, in + c_hi);
+                    if (tk.ok) {
+                        const __nv_bfloat16* src = tgt + tk.dst_off;
+                        cp_async16(st32 + d_lo, src + c_lo);
+                        cp_async16(st32 + d_hi, src + c_hi);
+                    } else {
+                        *reinterpret_cast<uint4*>(st + d_lo) = zero;
+                        *reinterpret_cast<uint4*>(st + d_hi) = zero;
+                    }
+                }
+            }
+            cp_async_wait_all();
+            const bool rot_s = kv == 0 && P.rs.enabled, rot_t = kv == 0 && P.rt.enabled;
+            if (rot_s || rot_t) {
+                for (int item = tw * 32 + lane; item < nitems; item += kGramTeamWarps * 32) {
+                    const int i = item / CPM, cp = item - i * CPM;
+                    const GramTok tk = tt[i];
+                    if (!tk.ok) continue;
+                    float2 cs[8];
+                    bool have = false;
+                    if (rot_s && cp < CPH && cp * 8 < P.rhalf_s) {
+                        int c_lo, c_hi;
+                        pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) cs[e] = turn_cs(sTurnS[cp * 8 + e], tk.ps);
+                        have = true;
+#pragma unroll
+                        for (int q = 0; q < NHD; ++q) {
+                            if (q >= nh) break;
+                            gram_unrotate(st + gram_chunk(i, q * DS + c_lo), st + gram_chunk(i, q * DS + c_hi), cs);
+                        }
+                    }
+                    if (rot_t && cp < cpt && cp * 8 < P.rhalf_t) {
+                        int c_lo, c_hi;
+                        pair_channels(cp * 8, dt >> 1, P.rhalf_t, c_lo, c_hi);
+                        if (!(have && P.rope_same && tk.ps == tk.pt)) {
+#pragma unroll
+                            for (int e = 0; e < 8; ++e) cs[e] = turn_cs(sTurnT[cp * 8 + e], tk.pt);
+                        }
+                        gram_unrotate(st + gram_chunk(i, in + c_lo), st + gram_chunk(i, in + c_hi), cs);
+                    }
+                }
+            }
+            fence_proxy_async();
+            __syncwarp();
+            if (lane == 0) {
+                mbar_arrive(bar(bZFull + s));
+                mbar_arrive(bar(bREmpty + r));
+            }
         }
     } else {
         // ------------------------------------------------------------ prologue: token-row blocks in shared memory
@@ -981,14 +1120,22 @@ extern "C" KVX_API kvx_status kvx_fit_create(const kvx_translator_desc* desc, do
     return KVX_OK;
 }
 
-template <int DS, int NHD>
-static cudaError_t launch_gram_tc(const TranslateParams& P, const GramLaunch& L, int grid, size_t smem, cudaStream_t s)
+template <int DS, int NHD, bool DIRECT>
+static cudaError_t launch_gram_tc_v(const TranslateParams& P, const GramLaunch& L, int grid, size_t smem, cudaStream_t s)
 {
     // the opt-in is set once per device, so at the largest size any launch asks for
-    const cudaError_t e = smem_opt_in<fit_gram_tc_kernel<DS, NHD>>(kSmemMax);
+    const cudaError_t e = smem_opt_in<fit_gram_tc_kernel<DS, NHD, DIRECT>>(kSmemMax);
     if (e != cudaSuccess) return e;
-    fit_gram_tc_kernel<DS, NHD><<<grid, kGramThreads, smem, s>>>(P, L);
+    fit_gram_tc_kernel<DS, NHD, DIRECT><<<grid, kGramThreads, smem, s>>>(P, L);
     return cudaGetLastError();
+}
+
+template <int DS, int NHD>
+static cudaError_t launch_gram_tc(const TranslateParams& P, const GramLaunch& L, bool direct, int grid, size_t smem,
+                                  cudaStream_t s)
+{
+    return direct ? launch_gram_tc_v<DS, NHD, true>(P, L, grid, smem, s)
+                  : launch_gram_tc_v<DS, NHD, false>(P, L, grid, smem, s);
 }
 
 extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv* src, const kvx_tgt_tokens* tgt,
@@ -1023,7 +1170,21 @@ extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv
         L.src_row = (unsigned)ds * 2;   // rows as in the caches: whole windows move in one copy
         L.tgt_row = (unsigned)dt * 2;
         const unsigned tail = 32 * 8 + (unsigned)(ds / 2 + dt / 2) * 8;   // barriers, flags, turns
+        // identity alignment: every span is one source row (or none), gathered by the prologue
+        const bool direct = P.span_lo == nullptr;
         bool fits = false;
+        if (direct) {   // token tables only in the raw slots; as many block stages as fit
+            const unsigned rb = (unsigned)(kGramK * sizeof(GramTok) + 16 + 15) / 16 * 16;
+            for (int st = kGramMaxStages; st >= 2 && !fits; --st) {
+                L.stages = st;
+                L.raw_slots = kGramMaxRaw;
+                L.rcap = 0;
+                L.raw_bytes = rb;
+                L.off_raw = (unsigned)L.stages * L.stage_bytes;
+                L.off_bar = L.off_raw + (unsigned)kGramMaxRaw * rb;
+                fits = 1024 + L.off_bar + tail <= (unsigned)kSmemMax;
+            }
+        }
         for (int raw = 2; raw >= 1 && !fits; --raw)
             for (int rcap = 128; rcap >= 64 && !fits; rcap -= 16) {
                 const unsigned rb = (unsigned)(kGramK * sizeof(GramTok) + 16 + (size_t)(in / ds) * rcap * L.src_row +
@@ -1047,13 +1208,13 @@ extern "C" KVX_API kvx_status kvx_fit_accumulate(kvx_fitter* f, const kvx_src_kv
         cudaError_t ce;
         // in = NHD * ds with in a multiple of 128 and in + dt <= 512
         switch (ds * 8 + in / ds) {
-        case 64 * 8 + 2: ce = launch_gram_tc<64, 2>(P, L, grid, smem, s); break;
-        case 64 * 8 + 4: ce = launch_gram_tc<64, 4>(P, L, grid, smem, s); break;
-        case 64 * 8 + 6: ce = launch_gram_tc<64, 6>(P, L, grid, smem, s); break;
-        case 128 * 8 + 1: ce = launch_gram_tc<128, 1>(P, L, grid, smem, s); break;
-        case 128 * 8 + 2: ce = launch_gram_tc<128, 2>(P, L, grid, smem, s); break;
-        case 128 * 8 + 3: ce = launch_gram_tc<128, 3>(P, L, grid, smem, s); break;
-        case 256 * 8 + 1: ce = launch_gram_tc<256, 1>(P, L, grid, smem, s); break;
+        case 64 * 8 + 2: ce = launch_gram_tc<64, 2>(P, L, direct, grid, smem, s); break;
+        case 64 * 8 + 4: ce = launch_gram_tc<64, 4>(P, L, direct, grid, smem, s); break;
+        case 64 * 8 + 6: ce = launch_gram_tc<64, 6>(P, L, direct, grid, smem, s); break;
+        case 128 * 8 + 1: ce = launch_gram_tc<128, 1>(P, L, direct, grid, smem, s); break;
+        case 128 * 8 + 2: ce = launch_gram_tc<128, 2>(P, L, direct, grid, smem, s); break;
+        case 128 * 8 + 3: ce = launch_gram_tc<128, 3>(P, L, direct, grid, smem, s); break;
+        case 256 * 8 + 1: ce = launch_gram_tc<256, 1>(P, L, direct, grid, smem, s); break;
         default: return fit_fail(KVX_ERR_UNSUPPORTED, "fit_accumulate: no Gram kernel for in %d, d_s %d", in, ds);
         }
         if (ce != cudaSuccess) return fit_fail(KVX_ERR_CUDA, "fit_accumulate: %s", cudaGetErrorString(ce));

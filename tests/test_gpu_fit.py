@@ -97,7 +97,8 @@ def _elementwise_bound(c, tk, tv, lam, wk_ref, wv_ref, chol_u=2.0 ** -24):
                     b = int(seq[tp])
                     t = tp - int(wl.tgt_seq_off[b])
                     y = np.asarray(tgt[j][b, h, t], np.float64)
-                    Y[tp] = oracle.rope_g(y, s.dst, float(t), -1) if kv == 0 and s.dst.rope_base > 0 else y
+                    pt = float(t if c.tgt_pos is None else c.tgt_pos[tp])
+                    Y[tp] = oracle.rope_g(y, s.dst, pt, -1) if kv == 0 and s.dst.rope_base > 0 else y
                 W = wref[j, h]
                 G = X.T @ X + lam * np.eye(din)
                 A = np.linalg.inv(G)
@@ -132,7 +133,7 @@ def _fit_gpu(c, tk, tv, lam, chunk=0, split=None, paged=False):
     f = kvx.Fitter(s.src, s.dst, lam, layer_map=c.layer_map.tolist(), dtype=g.tr.desc.dtype, form=s.form,
                    layers_per_target=s.layers_per_target, chunk_tokens=chunk)
     wl = c.wl
-    kw = dict(span_lo=g.span_lo, span_hi=g.span_hi)
+    kw = dict(span_lo=g.span_lo, span_hi=g.span_hi, src_pos=g.src_pos, tgt_pos=g.tgt_pos)
     if paged:
         P = s.page_size
         pages = [(int(t) + P - 1) // P for t in wl.tgt_len]
@@ -220,6 +221,36 @@ def test_fit_recovers_planted_translator_and_matches_oracle(name):
         assert _rel(gpu, ref) <= 1e-2, _rel(gpu, ref)
         assert _rel(gpu, true) <= 1e-2, _rel(gpu, true)
         assert _rel(ref, true) <= 5e-3, _rel(ref, true)
+
+
+def test_fit_with_explicit_positions_matches_oracle():
+    """Identity alignment with position arrays on both sides: source rows at s + 3b, target rows
+    at t + 3b for even t and t + 3b + 7 for odd t, so half the tokens share their source
+    rotation with the target's and half do not.  Both rotations are the same schedule here
+    (7B -> 1.5B shapes), the case where one (cos, sin) may serve both sides of a token."""
+    spec = _shrink(SPECS["qwen7b_to_qwen1p5b_4k"], 3, 2)
+    lens = [700, 500]
+    wl = synth.make_workload(spec, lens)
+    src_pos = np.stack([np.arange(wl.s_max) + 3 * b for b in range(wl.batch)]).astype(np.int32)
+    tgt_pos = np.empty(wl.total_tgt, np.int32)
+    for b in range(wl.batch):
+        a, e = int(wl.tgt_seq_off[b]), int(wl.tgt_seq_off[b + 1])
+        t = np.arange(e - a)
+        tgt_pos[a:e] = t + 3 * b + 7 * (t & 1)
+    c = make_case(spec, lens, src_pos=src_pos, tgt_pos=tgt_pos, wl=wl)
+    rng = np.random.default_rng(23)
+    din, dt = spec.group_in, spec.dst.head_dim
+    w_true = [synth.bf16_round(rng.standard_normal((2, spec.dst.num_kv_heads, din, dt)).astype(np.float32)
+                               / np.float32(np.sqrt(din))) for _ in range(2)]
+    tk, tv = _targets_from(c, *w_true)
+    lam = 1e-3
+    gk, gv, bits, _ = _fit_gpu(c, tk, tv, lam)
+    assert bits == 0
+    ok, ov = oracle_problem(c).fit(list(tk), list(tv), lam)
+    bk, bv = _elementwise_bound(c, tk, tv, lam, ok, ov)
+    for gpu, ref, true, bound, lab in ((gk, ok, w_true[0], bk, "K"), (gv, ov, w_true[1], bv, "V")):
+        _assert_elementwise(gpu, ref, bound, f"positions {lab}")
+        assert _rel(gpu, true) <= 1e-2, _rel(gpu, true)
 
 
 def test_fit_fp32_tiny_matches_oracle_tightly():
