@@ -120,7 +120,7 @@ struct AUnit {
 // Iterates a CTA's units in order with counters only (no divisions per unit):
 // its share of K units, then its share of V units; each share group-major.
 struct Walker {
-    int count, nK, it;
+    int count, n1, it;   // n1: units of the first share (the V share)
     int kv, j, h, nt, k, b;
     int u0, v0, m_tiles, n_split, Ht, batch;
     const int* tile_off;
@@ -153,17 +153,17 @@ struct Walker {
     __device__ __forceinline__ void start(int u0_, int u1_, int v0_, int v1_, const AlignedParams& P,
                                           const int* tile_off_, const int* seq_off_)
     {
-        u0 = u0_; v0 = v0_; nK = u1_ - u0_; count = nK + (v1_ - v0_); it = 0;
+        u0 = u0_; v0 = v0_; n1 = v1_ - v0_; count = n1 + (u1_ - u0_); it = 0;
         m_tiles = P.m_tiles_max; n_split = P.n_split; Ht = P.Ht; batch = P.batch;
         tile_off = tile_off_; seq_off = seq_off_;
-        if (nK > 0) seek(u0, 0);
-        else if (count > 0) seek(v0, 1);
+        if (n1 > 0) seek(v0, 1);
+        else if (count > 0) seek(u0, 0);
     }
     __device__ __forceinline__ bool more() const { return it < count; }
     __device__ __forceinline__ void next()
     {
         if (++it >= count) return;
-        if (it == nK) { seek(v0, 1); return; }
+        if (it == n1) { seek(u0, 0); return; }
         if (++k == m_tiles) {
             k = 0;
             b = 0;
@@ -177,7 +177,7 @@ struct Walker {
     // no later unit of this CTA uses the current group's weights
     __device__ __forceinline__ bool last_of_group() const
     {
-        return it + 1 == count || it + 1 == nK || k + 1 >= tile_off[batch];
+        return it + 1 == count || it + 1 == n1 || k + 1 >= tile_off[batch];
     }
 };
 
@@ -270,7 +270,8 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     constexpr bool DIAG = VAR == 1, PLAIN = VAR == 2;
     const Waiter W{sAbort, P.status, DIAG && P.wait_ns ? P.wait_ns : kWaitNs};
     // Work split: each CTA takes an equal share of the K units and of the V units
-    // (K units cost more: the source RoPE undo), K share first.  Within each share
+    // (K units cost more: the source RoPE undo), V share first: V tiles need no
+    // un-rotation, so a launch's first MMA does not wait for one.  Within each share
     // units run group-major, so a group's weight tile stays resident.
     const int hgroups = P.groups / 2;                          // (j, h, nt) per K|V
     const long long UH = (long long)hgroups * P.m_tiles_max;
