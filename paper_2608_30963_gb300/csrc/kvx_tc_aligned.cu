@@ -120,7 +120,8 @@ struct AUnit {
 // Iterates a CTA's units in order with counters only (no divisions per unit):
 // its share of K units, then its share of V units; each share group-major.
 struct Walker {
-    int count, n1, it;   // n1: units of the first share (the V share)
+    int count, n1, it;   // n1: units of the first share
+    int kv1;             // K|V of the first share
     int kv, j, h, nt, k, b;
     int u0, v0, m_tiles, n_split, Ht, batch;
     const int* tile_off;
@@ -149,21 +150,27 @@ struct Walker {
         b = 0;
         fill();
     }
-    // K units [u0, u1) and V units [v0, v1) of the per-K|V unit index space
+    // K units [u0, u1) and V units [v0, v1) of the per-K|V unit index space; the V share first
+    // when v_first, else the K share first
     __device__ __forceinline__ void start(int u0_, int u1_, int v0_, int v1_, const AlignedParams& P,
-                                          const int* tile_off_, const int* seq_off_)
+                                          const int* tile_off_, const int* seq_off_, bool v_first)
     {
-        u0 = u0_; v0 = v0_; n1 = v1_ - v0_; count = n1 + (u1_ - u0_); it = 0;
+        kv1 = v_first ? 1 : 0;
+        u0 = v_first ? v0_ : u0_;   // first share
+        v0 = v_first ? u0_ : v0_;   // second share
+        n1 = v_first ? v1_ - v0_ : u1_ - u0_;
+        count = (u1_ - u0_) + (v1_ - v0_);
+        it = 0;
         m_tiles = P.m_tiles_max; n_split = P.n_split; Ht = P.Ht; batch = P.batch;
         tile_off = tile_off_; seq_off = seq_off_;
-        if (n1 > 0) seek(v0, 1);
-        else if (count > 0) seek(u0, 0);
+        if (n1 > 0) seek(u0, kv1);
+        else if (count > 0) seek(v0, kv1 ^ 1);
     }
     __device__ __forceinline__ bool more() const { return it < count; }
     __device__ __forceinline__ void next()
     {
         if (++it >= count) return;
-        if (it == n1) { seek(u0, 0); return; }
+        if (it == n1) { seek(v0, kv1 ^ 1); return; }
         if (++k == m_tiles) {
             k = 0;
             b = 0;
@@ -270,9 +277,11 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     constexpr bool DIAG = VAR == 1, PLAIN = VAR == 2;
     const Waiter W{sAbort, P.status, DIAG && P.wait_ns ? P.wait_ns : kWaitNs};
     // Work split: each CTA takes an equal share of the K units and of the V units
-    // (K units cost more: the source RoPE undo), V share first: V tiles need no
-    // un-rotation, so a launch's first MMA does not wait for one.  Within each share
+    // (K units cost more: the source RoPE undo).  Even CTAs walk their V share first and
+    // odd CTAs their K share first, so that at any time about half the SMs run K tiles
+    // (bound by the un-rotation) and half V tiles (bound by HBM).  Within each share
     // units run group-major, so a group's weight tile stays resident.
+    const bool v_first = (blockIdx.x & 1) == 0;
     const int hgroups = P.groups / 2;                          // (j, h, nt) per K|V
     const long long UH = (long long)hgroups * P.m_tiles_max;
     const int u0 = (int)((long long)blockIdx.x * UH / gridDim.x);
@@ -295,7 +304,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             bool ok = true;
             int nunit = 0;   // units with rows walked so far
             Walker wk;
-            for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+            for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff, v_first); wk.more(); wk.next()) {
                 const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
                 if (DIAG && blockIdx.x == 0 && ++nunit == P.stall_unit1) {
@@ -351,7 +360,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
             uint32_t kr_idx = 0, kr_phase = 0;
             bool ok = true;
             Walker wk;
-            for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+            for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff, v_first); wk.more(); wk.next()) {
                 const AUnit& x = wk.x;
                 if (x.rows <= 0) continue;
                 if (x.g != cur_g) {
@@ -407,7 +416,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         const uint32_t srow_u32 = (uint32_t)__cvta_generic_to_shared(srow);
         uint32_t tcount = 0, kc = 0;   // kc: K tiles seen (selects the shared (cos, sin) buffer)
         Walker wk;
-        for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+        for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff, v_first); wk.more(); wk.next()) {
             const AUnit& x = wk.x;
             if (x.rows <= 0) continue;
             const uint32_t buf = tcount & 1;
@@ -523,7 +532,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
         uint32_t kr_idx = 0, kc = 0;
         bool ok = true;
         Walker wk;
-        for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff); wk.more(); wk.next()) {
+        for (wk.start(u0, u1, v0, v1, P, sTileOff, sSeqOff, v_first); wk.more(); wk.next()) {
             const AUnit& x = wk.x;
             if (x.rows <= 0) continue;
             const bool rot = x.kv == 0 && P.rs.enabled;
