@@ -8,16 +8,17 @@
 //           translation forms them), rounded to the cache dtype;
 //   Y rows: the target model's own cache rows, target RoPE undone for K.
 // Accumulation (kvx_fit_accumulate), bf16 caches with in + d_t <= 512:
-//   fit_gram_tc_kernel builds the transposed rows [X | Y]^T of 64 tokens at a time in shared
-//   memory and adds X^T X and X^T Y on the tensor cores (tokens are the contraction dimension),
-//   accumulating in TMEM; X and Y never go to global memory.
+//   fit_gram_tc_kernel builds the rows [X | Y] of 64 tokens at a time in shared memory and adds
+//   X^T X and X^T Y on the tensor cores (tokens are the contraction dimension), accumulating in
+//   TMEM; X and Y never go to global memory.
 // Otherwise (fp32 caches, wider inputs):
 //   fit_rows_kernel builds X and Y for one pass of up to chunk tokens, then fit_gram_simt_kernel
 //   adds their products into the sums on the CUDA cores.
 // Solve (kvx_fit_solve): one CTA per group factors X^T X + lambda I = L L^T and runs the two
 //   triangular solves per output column: fit_solve_small_kernel in fp32 shared memory for
-//   in <= 256 (with one step of iterative refinement against the fp32 sums), fit_solve_kernel in
-//   double global memory above.
+//   in <= 256, handing the systems whose factor shows a condition number above 10^3 to
+//   fit_solve_kernel, which solves in double in global memory (and solves every system above
+//   in = 256).
 #include <math.h>
 #include <stdarg.h>
 #include <stdio.h>
@@ -393,25 +394,31 @@ __global__ void __launch_bounds__(256) fit_gram_simt_kernel(const T* __restrict_
 // kb of the call:  D[i, n] += sum_t Z^T[mb*128 + i, t] * Z^T[n, t],  Z = [X | Y].  Only the
 // lower triangle of X^T X is formed (the solves read it): row block mb takes the X columns
 // [0, (mb+1)*128) and the dt columns of Y, so its accumulator holds (mb+1)*128 + dt columns.
-//   loader warp  resolves the block's 64 tokens into a table in shared memory and copies the
-//                source rows of the block's span window (per source head-block) and the 64 target
-//                rows into padded shared-memory rows with bulk copies (a ring of raw slots).
-//   8 prologue warps  build the transposed block Z^T[rows][64 tokens] in the UMMA K-major
-//                128-byte-swizzled layout (tokens are the contraction dimension): one lane per
-//                token, one 16-channel chunk pair per pass, (cos, sin) once per token and pair
-//                for every source head of the input row; tokens 2w and 2w+1 (adjacent lanes)
-//                exchange values by shuffle and write one 4-byte word each.  X rows as the
-//                translation forms them (span mean of un-rotated source rows), Y rows with the
-//                target RoPE undone for K, both rounded to bf16.  Tokens whose span leaves the
-//                window read their rows from global memory.
-//   MMA thread   M = 128 (the block's rows of Z^T as A), N over the needed rows of Z^T as B (in
+//   loader warp  resolves the block's 64 tokens into a table in shared memory.  For a call with
+//                spans it also copies the block's source window (one bulk copy per source head
+//                when the rows are contiguous) and its 64 target rows (one bulk copy when they are
+//                consecutive) into a ring of raw slots.
+//   12 prologue warps  build the block [X | Y] of 64 token rows, channels contiguous, in
+//                128-byte-swizzled atoms of 64 channels x 8 tokens: the layout tcgen05 reads as
+//                an MN-major operand, so both A and B are this block and nothing is transposed.
+//                X rows as the translation forms them (span mean of un-rotated source rows), Y
+//                rows with the target RoPE undone for K, both rounded to bf16.
+//                With spans: all 12 warps on one block, lanes across a row's 16-channel chunk
+//                pairs (8 lanes per 128-channel head), each lane taking the span mean of its
+//                chunk pair; tokens whose span leaves the window read their rows from global
+//                memory.
+//                Identity alignment ("direct" blocks): 4 teams of 3 warps, one block per team.
+//                A thread gathers its (token, chunk pair) items straight into their swizzled
+//                places with 16-byte cp.async, waits for its own copies and un-rotates K in
+//                place, one (cos, sin) per pair for every source head and, when the rotations
+//                and the token's positions coincide, for its target row too.
+//   MMA thread   M = 128 (the row block's channels as A), N over the needed columns (B, in
 //                pieces of <= 256), K = 16 tokens per instruction, into one fp32 TMEM
 //                accumulator that lives for the CTA's range of a unit.
 //   4 epilogue warps  add the accumulator into the fp32 sums (vector atomics for X^T X rows,
 //                coalesced atomics for X^T Y columns).
-// Units are (g, chunk of K-blocks, mb) with mb fastest, so the two row blocks of a chunk read
-// the same cache rows back to back (the second read hits L2); each CTA takes a contiguous range
-// of the (unit, K-block) space.
+// Units are (g, chunk of K-blocks, mb) with mb fastest; each CTA takes an equal contiguous
+// range of the (unit, K-block) space, so a range may start or end inside a unit.
 constexpr int kGramK = 64;
 constexpr int kGramMmaWarp = 0;
 constexpr int kGramEpiWarp0 = 1;
