@@ -18,6 +18,7 @@
 //                    two warps per TMEM lane quadrant, each taking half of the RoPE pairs
 //   warps 10-17      prologue: in-place source-RoPE undo of K tiles
 // Every wait is bounded (~1 s, then KVX_DEV_WAIT_TIMEOUT and a drained exit).
+#include <algorithm>
 #include <cuda.h>
 #include <stddef.h>
 #include <string.h>
@@ -98,7 +99,12 @@ struct AlignedParams {
     void* dst_k[KVX_MAX_ALIGNED_LAYERS];
     void* dst_v[KVX_MAX_ALIGNED_LAYERS];
     CUtensorMap maps[2 * KVX_MAX_ALIGNED_LAYERS];   // [j*2 + kv]: source K/V of target layer j
+    // V share of each CTA (an index of the same equal split as the K shares), chosen on the host
+    // so that CTAs with a costly K share get a cheap V share; unused above kMaxVmap CTAs
+    int use_vmap;
+    unsigned short vmap[256];
 };
+constexpr int kMaxVmap = 256;
 
 __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
                                             uint32_t bar, uint64_t pol)
@@ -287,7 +293,7 @@ __global__ void __launch_bounds__(kThreads, 1) translate_tc_aligned_kernel(const
     const int u0 = (int)((long long)blockIdx.x * UH / gridDim.x);
     const int u1 = (int)((long long)(blockIdx.x + 1) * UH / gridDim.x);
     // the V share mirrors the CTA order, so a CTA with one K unit more gets one V unit fewer
-    const int vr = gridDim.x - 1 - blockIdx.x;
+    const int vr = P.use_vmap ? (int)P.vmap[blockIdx.x] : (int)gridDim.x - 1 - (int)blockIdx.x;
     const int v0 = (int)((long long)vr * UH / gridDim.x);
     const int v1 = (int)((long long)(vr + 1) * UH / gridDim.x);
     const int blk_per_head = (2 * HS) / kBlockK;       // K-blocks of one source head
@@ -767,6 +773,26 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     }
     const long long UH = (long long)(P.groups / 2) * P.m_tiles_max;
     const int grid = (int)(UH < num_sms ? UH : num_sms);
+    // V shares: share r is units [r*UH/grid, (r+1)*UH/grid) of the per-K|V unit space, CTA c's K
+    // share is share c.  A share costs its units (a K unit about 1.41 V units: the un-rotation)
+    // plus about 0.57 V units per extra weight image it needs (a group switch); the costliest K
+    // shares get the cheapest V shares.
+    P.use_vmap = grid <= kMaxVmap;
+    if (P.use_vmap) {
+        struct Share { double k, v; int idx; };
+        Share sh[kMaxVmap];
+        for (int r = 0; r < grid; ++r) {
+            const long long a = (long long)r * UH / grid, b = (long long)(r + 1) * UH / grid;
+            const int groups = b > a ? (int)((b - 1) / P.m_tiles_max - a / P.m_tiles_max) + 1 : 0;
+            const double sw = 0.57 * (groups > 1 ? groups - 1 : 0);
+            sh[r] = Share{1.41 * (double)(b - a) + sw, (double)(b - a) + sw, r};
+        }
+        int byk[kMaxVmap], byv[kMaxVmap];
+        for (int r = 0; r < grid; ++r) byk[r] = byv[r] = r;
+        std::sort(byk, byk + grid, [&](int x, int y) { return sh[x].k > sh[y].k || (sh[x].k == sh[y].k && x < y); });
+        std::sort(byv, byv + grid, [&](int x, int y) { return sh[x].v < sh[y].v || (sh[x].v == sh[y].v && x > y); });
+        for (int i = 0; i < grid; ++i) P.vmap[byk[i]] = (unsigned short)byv[i];
+    }
     // the diagnostics' and the thread-store instantiations only when they are asked for
     const int var = P.plain_stores ? 2 : (P.wait_ns != 0 || P.stall_unit1 != 0 ? 1 : 0);
     switch (T.ds * 4 + var) {
