@@ -791,36 +791,46 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                 hb[q] = (const __nv_bfloat16*)(kv ? P.src_v[slot] : P.src_k[slot]) + (long long)gs * P.sh;
             }
             const __nv_bfloat16* tgt = (const __nv_bfloat16*)(kv ? P.dst_v[j] : P.dst_k[j]) + dst_head_off(P, h);
-            const int nitems = kGramK * CPM;
+            // This thread's chunk pair cp for every token i0, i0 + istep, ... of the block: the
+            // destination columns (64-channel block and 16-byte chunk within the swizzled row)
+            // depend only on cp, a token adds its row offset and the swizzle phase i & 7.
             const uint4 zero = make_uint4(0u, 0u, 0u, 0u);
-            for (int item = tw * 32 + lane; item < nitems; item += kGramTeamWarps * 32) {
-                const int i = item / CPM, cp = item - i * CPM;
+            // (threads past the last whole stride stay idle: no token is copied or rotated twice)
+            const int ttid = tw * 32 + lane, cp = ttid % CPM, istep = kGramTeamWarps * 32 / CPM;
+            const int i0 = ttid < istep * CPM ? ttid / CPM : kGramK;
+            const bool has_x = cp < CPH, has_y = cp < cpt;
+            int c_lo = 0, c_hi = 0, y_lo = 0, y_hi = 0;
+            if (has_x) pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
+            if (has_y) pair_channels(cp * 8, dt >> 1, P.rhalf_t, y_lo, y_hi);
+            auto col = [](int c) { return (uint32_t)((c >> 6) * (kGramK * 128)); };
+            auto chk = [](int c) { return (uint32_t)((c >> 3) & 7); };
+            for (int i = i0; i < kGramK; i += istep) {
                 const GramTok tk = tt[i];
-                if (cp < CPH) {
-                    int c_lo, c_hi;
-                    pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
+                const uint32_t row = (uint32_t)((i >> 3) * 1024 + (i & 7) * 128), x7 = (uint32_t)(i & 7);
+                if (has_x) {
+                    const long long so = (long long)tk.b * P.sb + (long long)tk.lo * P.ss;
 #pragma unroll
                     for (int q = 0; q < NHD; ++q) {
                         if (q >= nh) break;
-                        const uint32_t d_lo = gram_chunk(i, q * DS + c_lo), d_hi = gram_chunk(i, q * DS + c_hi);
+                        const int cl = q * DS + c_lo, ch = q * DS + c_hi;
+                        const uint32_t d_lo = col(cl) + row + ((chk(cl) ^ x7) << 4);
+                        const uint32_t d_hi = col(ch) + row + ((chk(ch) ^ x7) << 4);
                         if (tk.ok) {
-                            const __nv_bfloat16* src = hb[q] + (long long)tk.b * P.sb + (long long)tk.lo * P.ss;
-                            cp_async16(st32 + d_lo, src + c_lo);
-                            cp_async16(st32 + d_hi, src + c_hi);
+                            cp_async16(st32 + d_lo, hb[q] + so + c_lo);
+                            cp_async16(st32 + d_hi, hb[q] + so + c_hi);
                         } else {
                             *reinterpret_cast<uint4*>(st + d_lo) = zero;
                             *reinterpret_cast<uint4*>(st + d_hi) = zero;
                         }
                     }
                 }
-                if (cp < cpt) {
-                    int c_lo, c_hi;
-                    pair_channels(cp * 8, dt >> 1, P.rhalf_t, c_lo, c_hi);
-                    const uint32_t d_lo = gram_chunk(i, in + c_lo), d_hi = gram_chunk(i, in + c_hi);
+                if (has_y) {
+                    const uint32_t d_lo = col(in + y_lo) + row + ((chk(in + y_lo) ^ x7) << 4);
+                    const uint32_t d_hi = col(in + y_hi) + row + ((chk(in + y_hi) ^ x7) << 4);
                     if (tk.ok) {
                         const __nv_bfloat16* src = tgt + tk.dst_off;
-                        cp_async16(st32 + d_lo, src + c_lo);
-                        cp_async16(st32 + d_hi, src + c_hi);
+                        cp_async16(st32 + d_lo, src + y_lo);
+                        cp_async16(st32 + d_hi, src + y_hi);
                     } else {
                         *reinterpret_cast<uint4*>(st + d_lo) = zero;
                         *reinterpret_cast<uint4*>(st + d_hi) = zero;
@@ -828,34 +838,32 @@ __global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __gr
                 }
             }
             cp_async_wait_all();
-            const bool rot_s = kv == 0 && P.rs.enabled, rot_t = kv == 0 && P.rt.enabled;
+            const bool rot_s = kv == 0 && P.rs.enabled && has_x && cp * 8 < P.rhalf_s;
+            const bool rot_t = kv == 0 && P.rt.enabled && has_y && cp * 8 < P.rhalf_t;
             if (rot_s || rot_t) {
-                for (int item = tw * 32 + lane; item < nitems; item += kGramTeamWarps * 32) {
-                    const int i = item / CPM, cp = item - i * CPM;
+                for (int i = i0; i < kGramK; i += istep) {
                     const GramTok tk = tt[i];
                     if (!tk.ok) continue;
+                    const uint32_t row = (uint32_t)((i >> 3) * 1024 + (i & 7) * 128), x7 = (uint32_t)(i & 7);
                     float2 cs[8];
-                    bool have = false;
-                    if (rot_s && cp < CPH && cp * 8 < P.rhalf_s) {
-                        int c_lo, c_hi;
-                        pair_channels(cp * 8, HS, P.rhalf_s, c_lo, c_hi);
+                    if (rot_s) {
 #pragma unroll
                         for (int e = 0; e < 8; ++e) cs[e] = turn_cs(sTurnS[cp * 8 + e], tk.ps);
-                        have = true;
 #pragma unroll
                         for (int q = 0; q < NHD; ++q) {
                             if (q >= nh) break;
-                            gram_unrotate(st + gram_chunk(i, q * DS + c_lo), st + gram_chunk(i, q * DS + c_hi), cs);
+                            const int cl = q * DS + c_lo, ch = q * DS + c_hi;
+                            gram_unrotate(st + col(cl) + row + ((chk(cl) ^ x7) << 4),
+                                          st + col(ch) + row + ((chk(ch) ^ x7) << 4), cs);
                         }
                     }
-                    if (rot_t && cp < cpt && cp * 8 < P.rhalf_t) {
-                        int c_lo, c_hi;
-                        pair_channels(cp * 8, dt >> 1, P.rhalf_t, c_lo, c_hi);
-                        if (!(have && P.rope_same && tk.ps == tk.pt)) {
+                    if (rot_t) {
+                        if (!(rot_s && P.rope_same && tk.ps == tk.pt)) {
 #pragma unroll
                             for (int e = 0; e < 8; ++e) cs[e] = turn_cs(sTurnT[cp * 8 + e], tk.pt);
                         }
-                        gram_unrotate(st + gram_chunk(i, in + c_lo), st + gram_chunk(i, in + c_hi), cs);
+                        gram_unrotate(st + col(in + y_lo) + row + ((chk(in + y_lo) ^ x7) << 4),
+                                      st + col(in + y_hi) + row + ((chk(in + y_hi) ^ x7) << 4), cs);
                     }
                 }
             }
