@@ -424,14 +424,15 @@ constexpr int kGramMmaWarp = 0;
 constexpr int kGramEpiWarp0 = 1;
 constexpr int kGramNumEpi = 4;
 constexpr int kGramXfWarp0 = kGramEpiWarp0 + kGramNumEpi;
-constexpr int kGramNumXf = 12;
-constexpr int kGramLoadWarp = kGramXfWarp0 + kGramNumXf;
-constexpr int kGramThreads = (kGramLoadWarp + 1) * 32;
+// prologue warps: 12 for staged blocks, 16 (4 teams of 4) for direct blocks, whose prologue needs
+// fewer registers (the CTA's 22 warps leave 88 a thread)
+__host__ __device__ constexpr int gram_num_xf(bool direct) { return direct ? 16 : 12; }
+__host__ __device__ constexpr int gram_load_warp(bool direct) { return kGramXfWarp0 + gram_num_xf(direct); }
+__host__ __device__ constexpr int gram_threads(bool direct) { return (gram_load_warp(direct) + 1) * 32; }
 constexpr int kGramMaxStages = 4;
 constexpr int kGramMaxRaw = 8;
 // Direct blocks (every span one source row): the prologue warps work in teams, one 64-token block each.
 constexpr int kGramTeams = 4;
-constexpr int kGramTeamWarps = kGramNumXf / kGramTeams;
 constexpr int kGramMaxRows = 512;   // in + dt: one 128 x 512 fp32 accumulator fills TMEM
 constexpr int kGramMaxHeads = 6;    // source head-blocks in one input row
 
@@ -532,9 +533,12 @@ __device__ __forceinline__ void gram_unrotate(uint8_t* lo, uint8_t* hi, const fl
 // alignment (every span one source row): the loader writes token tables only, and the prologue
 // teams gather the rows with 16-byte asynchronous copies straight into the block.
 template <int DS, int NHD, bool DIRECT>
-__global__ void __launch_bounds__(kGramThreads, 1) fit_gram_tc_kernel(const __grid_constant__ TranslateParams P,
+__global__ void __launch_bounds__(gram_threads(DIRECT), 1) fit_gram_tc_kernel(const __grid_constant__ TranslateParams P,
                                                                       const __grid_constant__ GramLaunch L)
 {
+    constexpr int kGramNumXf = gram_num_xf(DIRECT);
+    constexpr int kGramLoadWarp = gram_load_warp(DIRECT);
+    constexpr int kGramTeamWarps = kGramNumXf / kGramTeams;
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
     uint8_t* sRaw = smem + L.off_raw;
@@ -1141,7 +1145,7 @@ static cudaError_t launch_gram_tc_v(const TranslateParams& P, const GramLaunch& 
     // the opt-in is set once per device, so at the largest size any launch asks for
     const cudaError_t e = smem_opt_in<fit_gram_tc_kernel<DS, NHD, DIRECT>>(kSmemMax);
     if (e != cudaSuccess) return e;
-    fit_gram_tc_kernel<DS, NHD, DIRECT><<<grid, kGramThreads, smem, s>>>(P, L);
+    fit_gram_tc_kernel<DS, NHD, DIRECT><<<grid, gram_threads(DIRECT), smem, s>>>(P, L);
     return cudaGetLastError();
 }
 
