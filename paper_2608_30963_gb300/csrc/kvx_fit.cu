@@ -889,6 +889,7 @@ __global__ void __launch_bounds__(gram_threads(DIRECT), 1) fit_gram_tc_kernel(co
         const int xw = warp - kGramXfWarp0;
         const int cpt = dt / 16;                     // chunk pairs of a target row
         const int LY = cpt < 32 ? cpt : 32;          // lanes per token, Y
+        const int y_tpp = 32 / LY, y_tok = lane / LY, y_cp = lane % LY;   // per Y pass: tokens, this lane's token and pair
         const unsigned long long* sTurnS = sTurn;
         const unsigned long long* sTurnT = sTurn + (P.ds >> 1);
         uint32_t it = 0;
@@ -975,7 +976,7 @@ __global__ void __launch_bounds__(gram_threads(DIRECT), 1) fit_gram_tc_kernel(co
                 } else {
                     // Y: chunk pair cp of the target row, target RoPE undone for K
                     const int yp = pc - xpass;
-                    const int i = yp * (32 / LY) + lane / LY, cp = lane % LY;
+                    const int i = yp * y_tpp + y_tok, cp = y_cp;
                     const GramTok tk = tt[i];
                     int c_lo, c_hi;
                     pair_channels(cp * 8, dt >> 1, P.rhalf_t, c_lo, c_hi);
