@@ -688,7 +688,7 @@ def kernel_rev(sources=None, rev: str = "") -> str:
 _TRAFFIC_REC = os.path.join(ROOT, "profiles", "traffic.json")
 _TRAFFIC_SOURCES = ["paper_2608_30963_gb300/csrc/kvx_tc_aligned.cu", "paper_2608_30963_gb300/csrc/kvx_tc_common.cuh",
                     "paper_2608_30963_gb300/csrc/kvx_common.cuh", "paper_2608_30963_gb300/csrc/kvx_kernels.h",
-                    "include/kvx.h"]
+                    "paper_2608_30963_gb300/csrc/kvx_schedule.h", "include/kvx.h"]
 _UNITS = {"byte": 1, "kbyte": 1e3, "mbyte": 1e6, "gbyte": 1e9, "nsecond": 1e-9, "usecond": 1e-6,
           "msecond": 1e-3, "second": 1, "ns": 1e-9, "us": 1e-6, "ms": 1e-3, "s": 1}
 

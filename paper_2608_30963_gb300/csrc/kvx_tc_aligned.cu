@@ -18,13 +18,13 @@
 //                    two warps per TMEM lane quadrant, each taking half of the RoPE pairs
 //   warps 10-17      prologue: in-place source-RoPE undo of K tiles
 // Every wait is bounded (~1 s, then KVX_DEV_WAIT_TIMEOUT and a drained exit).
-#include <algorithm>
 #include <cuda.h>
 #include <stddef.h>
 #include <string.h>
 
 #include "kvx_common.cuh"
 #include "kvx_kernels.h"
+#include "kvx_schedule.h"
 #include "kvx_tc_common.cuh"
 
 namespace kvx {
@@ -773,26 +773,9 @@ cudaError_t launch_translate_tc_aligned(const TranslateParams& T, const void* co
     }
     const long long UH = (long long)(P.groups / 2) * P.m_tiles_max;
     const int grid = (int)(UH < num_sms ? UH : num_sms);
-    // V shares: share r is units [r*UH/grid, (r+1)*UH/grid) of the per-K|V unit space, CTA c's K
-    // share is share c.  A share costs its units (a K unit about 1.41 V units: the un-rotation)
-    // plus about 0.57 V units per extra weight image it needs (a group switch); the costliest K
-    // shares get the cheapest V shares.
+    // V shares paired with the K shares by cost (kvx_schedule.h)
     P.use_vmap = grid <= kMaxVmap;
-    if (P.use_vmap) {
-        struct Share { double k, v; int idx; };
-        Share sh[kMaxVmap];
-        for (int r = 0; r < grid; ++r) {
-            const long long a = (long long)r * UH / grid, b = (long long)(r + 1) * UH / grid;
-            const int groups = b > a ? (int)((b - 1) / P.m_tiles_max - a / P.m_tiles_max) + 1 : 0;
-            const double sw = 0.57 * (groups > 1 ? groups - 1 : 0);
-            sh[r] = Share{1.41 * (double)(b - a) + sw, (double)(b - a) + sw, r};
-        }
-        int byk[kMaxVmap], byv[kMaxVmap];
-        for (int r = 0; r < grid; ++r) byk[r] = byv[r] = r;
-        std::sort(byk, byk + grid, [&](int x, int y) { return sh[x].k > sh[y].k || (sh[x].k == sh[y].k && x < y); });
-        std::sort(byv, byv + grid, [&](int x, int y) { return sh[x].v < sh[y].v || (sh[x].v == sh[y].v && x > y); });
-        for (int i = 0; i < grid; ++i) P.vmap[byk[i]] = (unsigned short)byv[i];
-    }
+    if (P.use_vmap) pair_v_shares(grid, UH, P.m_tiles_max, P.vmap);
     // the diagnostics' and the thread-store instantiations only when they are asked for
     const int var = P.plain_stores ? 2 : (P.wait_ns != 0 || P.stall_unit1 != 0 ? 1 : 0);
     switch (T.ds * 4 + var) {

@@ -3,11 +3,14 @@
 //   pairs <d> <rhalf> then d/2 lines "<slot> <lo> <hi>"       -- pair_channels
 //   freq <d> <rotary_dim> <type> <factor> <low> <high> <orig> <base> then d/2 lines "<i> <f_i>"
 //   ok <1|0>                                                  -- rope_schedule_ok
-// for the cases read from standard input (one per line, same fields).
+//   vshares <grid> then grid lines "<cta> <v share>"           -- pair_v_shares
+// for the cases read from standard input (one per line, same fields; vshares reads
+// <grid> <units per K|V> <units per group>).
 #include <cstdio>
 #include <cstring>
 
 #include "../paper_2608_30963_gb300/csrc/kvx_common.cuh"
+#include "../paper_2608_30963_gb300/csrc/kvx_schedule.h"
 
 int main()
 {
@@ -36,6 +39,14 @@ int main()
             }
             std::printf("freq %d\n", kvx::rope_rot_dim(g) / 2);
             for (int i = 0; i < kvx::rope_rot_dim(g) / 2; ++i) std::printf("%d %.17g\n", i, kvx::rope_inv_freq(g, i));
+        } else if (!std::strcmp(kind, "vshares")) {
+            int grid;
+            long long uh, mt;
+            if (std::scanf("%d %lld %lld", &grid, &uh, &mt) != 3 || grid < 1 || grid > 4096) return 2;
+            unsigned short v[4096];
+            kvx::pair_v_shares(grid, uh, mt, v);
+            std::printf("vshares %d\n", grid);
+            for (int c = 0; c < grid; ++c) std::printf("%d %d\n", c, (int)v[c]);
         } else {
             return 2;
         }

@@ -7,7 +7,10 @@ helpers compute:
   rotating slots pair (i, i + n/2), and chunks of 8 slots map to runs of 8 channels;
 - rope_inv_freq: the per-pair frequency under each schedule and rotary width equals the angle
   the oracle turns a unit vector by at position 1;
-- rope_schedule_ok: the rotary-width rule (0, or a multiple of 16 in [16, head_dim]).
+- rope_schedule_ok: the rotary-width rule (0, or a multiple of 16 in [16, head_dim]);
+- pair_v_shares (`kvx_schedule.h`): the identity-alignment kernel's V shares form a permutation
+  of the CTAs, and under the split's own cost model the costliest CTA costs no more than with
+  each CTA taking the mirrored V share.
 """
 import os
 import shutil
@@ -87,3 +90,23 @@ def test_library_frequencies_equal_the_oracle_angles(probe, d, n, base, si):
                                     (128, 8, 0), (128, 144, 0), (128, -16, 0), (64, 64, 1), (256, 256, 1)])
 def test_rotary_width_rule(probe, d, n, ok):
     assert probe([f"ok {d} {n} 0 1 1 4 8192 10000"]) == [f"ok {ok}"]
+
+
+def _share_cost(r, grid, uh, mt, per_unit):
+    a, b = r * uh // grid, (r + 1) * uh // grid
+    groups = (b - 1) // mt - a // mt + 1 if b > a else 0
+    return per_unit * (b - a) + 0.57 * max(groups - 1, 0)
+
+
+@pytest.mark.parametrize("grid,uh,mt", [(152, 56 * 32, 32), (152, 56 * 67, 67), (152, 56 * 259, 259), (148, 1000, 9),
+                                        (20, 13, 13), (1, 5, 5), (152, 152, 32)])
+def test_v_shares_are_a_permutation_that_lowers_the_costliest_cta(probe, grid, uh, mt):
+    out = probe([f"vshares {grid} {uh} {mt}"])
+    assert out[0] == f"vshares {grid}"
+    v = [int(line.split()[1]) for line in out[1:1 + grid]]
+    assert sorted(v) == list(range(grid))
+    k = [_share_cost(c, grid, uh, mt, 1.41) for c in range(grid)]
+    vc = [_share_cost(r, grid, uh, mt, 1.0) for r in range(grid)]
+    paired = max(k[c] + vc[v[c]] for c in range(grid))
+    mirrored = max(k[c] + vc[grid - 1 - c] for c in range(grid))
+    assert paired <= mirrored + 1e-9
