@@ -485,13 +485,7 @@ def main():
     peak_src = "measured" if hbm_peak else "fallback"
     hbm_peak = hbm_peak or 6800.0
     achieved = alg["bytes"] / (avg_launch_ms / 1e3) / 1e9
-    traffic = None
-    try:
-        tr_info = json.load(open(os.path.join(ROOT, "profiles", "traffic.json")))
-        if tr_info.get("workload") == args.workload and tr_info.get("kernel_rev") == kernel_rev(tr_info.get("sources")):
-            traffic = tr_info.get("dram_bytes_per_launch")
-    except Exception:
-        pass
+    traffic = traffic_for(args.workload)
     line = {
         "metric": METRIC,
         "value": value,
@@ -691,6 +685,18 @@ _TRAFFIC_SOURCES = ["paper_2608_30963_gb300/csrc/kvx_tc_aligned.cu", "paper_2608
                     "paper_2608_30963_gb300/csrc/kvx_schedule.h", "include/kvx.h"]
 _UNITS = {"byte": 1, "kbyte": 1e3, "mbyte": 1e6, "gbyte": 1e9, "nsecond": 1e-9, "usecond": 1e-6,
           "msecond": 1e-3, "second": 1, "ns": 1e-9, "us": 1e-6, "ms": 1e-3, "s": 1}
+
+
+def traffic_for(workload: str, rec_path: str = "") -> "int | None":
+    """DRAM bytes of one identity-kernel launch from the traffic record, or None when the record
+    is for another workload or the kernel's sources have changed since the capture."""
+    try:
+        rec = json.load(open(rec_path or _TRAFFIC_REC))
+    except Exception:
+        return None
+    if rec.get("workload") != workload or rec.get("kernel_rev") != kernel_rev(rec.get("sources")):
+        return None
+    return rec.get("dram_bytes_per_launch")
 
 
 def record_traffic(csv_path: str, workload: str, command: str, rev: str = "") -> int:
