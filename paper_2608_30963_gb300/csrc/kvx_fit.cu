@@ -764,11 +764,12 @@ __global__ void __launch_bounds__(gram_threads(DIRECT), 1) fit_gram_tc_kernel(co
         }
     } else if (DIRECT) {
         // ------------------------------------------------------------ prologue, direct blocks
-        // Team `team` of kGramTeamWarps warps takes every kGramTeams-th block.  A thread owns items
-        // (token i, chunk pair cp): it copies the pair's two 16-byte chunks of every needed source
-        // head and of the target row into their swizzled places, waits for its own copies, and for
-        // K un-rotates them in place, with one (cos, sin) per pair for the source heads and, when the
-        // two rotations and positions coincide, for the target row as well.
+        // Team `team` of kGramTeamWarps warps takes every kGramTeams-th block.  A thread keeps one
+        // chunk pair cp and steps over the block's tokens: per token it copies the pair's two
+        // 16-byte chunks of every needed source head and of the target row into their swizzled
+        // places, waits for its own copies, and for K un-rotates them in place, with one (cos, sin)
+        // per pair for the source heads and, when the two rotations and positions coincide, for
+        // the target row as well.
         constexpr int HS = DS / 2;
         constexpr int CPH = DS / 16;
         const int xw = warp - kGramXfWarp0, team = xw / kGramTeamWarps, tw = xw - team * kGramTeamWarps;
